@@ -1,0 +1,295 @@
+"""Plain fp64 CPU oracle of one BOM step and of the BOM-AdamW update.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path may import, call or
+execute this module: only ``tests/``, ``__graft_entry__.smoke()`` and the
+CPU-baseline / reference legs of ``bench.py`` use it.  It shares no code with
+the CUDA path (no kernels, headers, helpers, tables or constants); the two
+meet only in the seeded input generator, which holds none of the method's
+arithmetic.
+
+Everything is numpy float64.  Inputs arrive as the exact values the GPU sees
+(fp32 values, or bf16 values already expanded), promoted to float64, so only
+the compute precision differs between the two sides.
+
+What it computes (paper: "Backpropagated Output Momentum", Algorithm 1 in the
+per-dataset-results appendix, with the equations of Section 3):
+
+  1. supervised set I_t = rows whose label is not ``ignore_index``,
+     N_t = |I_t| > 0 (Algorithm 1, first step; LM construction appendix);
+  2. r_i = softmax(z_i) - onehot(y_i),  s_t = N_t^-1 sum_{i in I_t} r_i
+     (Algorithm 1; Section 3.2, "Formal update");
+  3. q_t = beta1 q_{t-1} + (1 - beta1) s_t,  qhat_t = q_t / (1 - beta1^t)
+     (Section 3.2, the EMA equation);
+  4. L_mix = (1 - lambda) L_CE + lambda N_t^-1 sum_i <z_i, qhat_t>
+     (Eq. mix-objective); its gradient u = (1 - lambda) g + lambda Jbar^T qhat
+     (Eq. mix-gradient).  The oracle back-propagates the logit cotangent of
+     L_mix by hand:  dL_mix/dz_i = N_t^-1 [(1 - lambda) r_i + lambda qhat_t]
+     for i in I_t and 0 otherwise.  g (cotangent r_i / N_t) and
+     h = Jbar^T qhat (cotangent qhat / N_t) are also returned separately;
+  5. v = beta2 v + (1 - beta2) u^2,  vhat = v / (1 - beta2^t)
+     (Section 3.4, the second-moment equation);
+  6. theta <- (1 - eta omega) theta - eta u / (sqrt(vhat) + eps)
+     (Section 3.4 update equation; Algorithm 1, last step).  No first-moment
+     bias correction is applied to u (Section 3.5, "The substitution").
+
+Backbone layers supported (shapes of the paper's settings; see the workload
+module): Linear, Linear+GELU (exact erf form) and the SwiGLU MLP sublayer
+x <- x + W_d (SiLU(W_g x) * W_u x).  The head is Linear d -> d_out, with an
+optional bias.
+
+Every function here is pinned by ``tests/test_oracle_pins.py`` against facts
+the paper or mathematics fix (finite-difference Jacobians and the exact batch
+decomposition, an independent autograd implementation, the EMA closed form of
+Lemma 2, the beta1 = 0 and lambda = 0 reductions, AdamW with beta1 = 0, the
+output-bias closed form and the zero-sum invariant).
+"""
+from __future__ import annotations
+
+import math
+from typing import Dict, List, Sequence, Tuple
+
+import numpy as np
+from scipy.special import erf as _erf
+
+F64 = np.float64
+
+
+class OracleError(Exception):
+    pass
+
+
+class LabelError(OracleError):
+    """A label outside [0, d_out) that is not the ignore index."""
+
+
+class EmptyError(OracleError):
+    """N_t = 0: Algorithm 1 requires at least one supervised output."""
+
+
+# --------------------------------------------------------------------------
+# Activations (exact GELU; SiLU = x * sigmoid(x))
+# --------------------------------------------------------------------------
+def gelu(x):
+    return 0.5 * x * (1.0 + _erf(x / math.sqrt(2.0)))
+
+
+def gelu_prime(x):
+    # d/dx [x Phi(x)] = Phi(x) + x phi(x)
+    Phi = 0.5 * (1.0 + _erf(x / math.sqrt(2.0)))
+    phi = np.exp(-0.5 * x * x) / math.sqrt(2.0 * math.pi)
+    return Phi + x * phi
+
+
+def sigmoid(x):
+    return 1.0 / (1.0 + np.exp(-x))
+
+
+def silu(x):
+    return x * sigmoid(x)
+
+
+def silu_prime(x):
+    sg = sigmoid(x)
+    return sg * (1.0 + x * (1.0 - sg))
+
+
+# --------------------------------------------------------------------------
+# Model: layers are (kind, d_in, d_out, has_bias) with kind in
+# {"linear", "linear_gelu", "swiglu"}; parameters are listed per layer
+# (W [d_out, d_in], b [d_out]) or (W_gate [ffn, d], W_up [ffn, d],
+# W_down [d, ffn]) followed by the head (W [d_out, d], optional b).
+# --------------------------------------------------------------------------
+def _split_params(layers, head_bias, params):
+    it = iter(params)
+    per_layer = []
+    for kind, d_in, d_out, has_bias in layers:
+        if kind == "swiglu":
+            per_layer.append((next(it), next(it), next(it)))
+        else:
+            w = next(it)
+            b = next(it) if has_bias else None
+            per_layer.append((w, b))
+    hw = next(it)
+    hb = next(it) if head_bias else None
+    rest = list(it)
+    if rest:
+        raise OracleError("too many parameter tensors")
+    return per_layer, (hw, hb)
+
+
+def forward(layers, head_bias, params, X):
+    """Logits Z = f(theta; X) and the saved activations of every layer."""
+    per_layer, (hw, hb) = _split_params(layers, head_bias, params)
+    x = np.asarray(X, dtype=F64)
+    tape = []
+    for (kind, d_in, d_out, has_bias), p in zip(layers, per_layer):
+        if kind == "swiglu":
+            wg, wu, wd = p
+            G = x @ wg.T
+            U = x @ wu.T
+            A = silu(G) * U
+            y = x + A @ wd.T
+            tape.append(("swiglu", x, G, U, A))
+            x = y
+        else:
+            w, b = p
+            pre = x @ w.T
+            if b is not None:
+                pre = pre + b
+            tape.append((kind, x, pre))
+            x = gelu(pre) if kind == "linear_gelu" else pre
+    Z = x @ hw.T
+    if hb is not None:
+        Z = Z + hb
+    return Z, (tape, x)
+
+
+def backward(layers, head_bias, params, saved, dZ):
+    """Vector-Jacobian product of the logit cotangent dZ through the network.
+
+    Returns (grads per parameter tensor in interface order, cotangent of the
+    head input)."""
+    per_layer, (hw, hb) = _split_params(layers, head_bias, params)
+    tape, h_last = saved
+    dZ = np.asarray(dZ, dtype=F64)
+    g_hw = dZ.T @ h_last
+    g_hb = dZ.sum(axis=0) if hb is not None else None
+    dx = dZ @ hw
+    dx_head = dx
+    grads_rev: List[np.ndarray] = []
+    if hb is not None:
+        grads_rev.append(g_hb)
+    grads_rev.append(g_hw)
+    for li in range(len(layers) - 1, -1, -1):
+        kind = layers[li][0]
+        rec = tape[li]
+        if kind == "swiglu":
+            wg, wu, wd = per_layer[li]
+            _, x, G, U, A = rec
+            dy = dx
+            g_wd = dy.T @ A
+            dA = dy @ wd
+            dG = dA * U * silu_prime(G)
+            dU = dA * silu(G)
+            g_wg = dG.T @ x
+            g_wu = dU.T @ x
+            dx = dy + dG @ wg + dU @ wu
+            grads_rev.extend([g_wd, g_wu, g_wg])
+        else:
+            w, b = per_layer[li]
+            _, x, pre = rec
+            dpre = dx * gelu_prime(pre) if kind == "linear_gelu" else dx
+            g_w = dpre.T @ x
+            if b is not None:
+                grads_rev.append(dpre.sum(axis=0))
+            grads_rev.append(g_w)
+            dx = dpre @ w
+    return grads_rev[::-1], dx_head
+
+
+# --------------------------------------------------------------------------
+# Task-space quantities (Algorithm 1, residual / EMA / objective steps)
+# --------------------------------------------------------------------------
+def supervised_set(labels, d_out, ignore_index=-100):
+    """Boolean mask of I_t and N_t; raises on bad labels or N_t = 0."""
+    y = np.asarray(labels, dtype=np.int64)
+    valid = y != ignore_index
+    bad = valid & ((y < 0) | (y >= d_out))
+    if bad.any():
+        raise LabelError(f"{int(bad.sum())} labels outside [0, {d_out})")
+    n_t = int(valid.sum())
+    if n_t == 0:
+        raise EmptyError("no supervised outputs in the batch (N_t = 0)")
+    return valid, n_t
+
+
+def log_sum_exp_rows(Z):
+    m = Z.max(axis=1, keepdims=True)
+    return (m + np.log(np.exp(Z - m).sum(axis=1, keepdims=True)))[:, 0]
+
+
+def softmax_rows(Z):
+    m = Z.max(axis=1, keepdims=True)
+    e = np.exp(Z - m)
+    return e / e.sum(axis=1, keepdims=True)
+
+
+def residuals(Z, labels, valid):
+    """r_i = softmax(z_i) - onehot(y_i) on supervised rows, 0 elsewhere."""
+    R = softmax_rows(np.asarray(Z, dtype=F64))
+    rows = np.nonzero(valid)[0]
+    R[rows, np.asarray(labels)[rows]] -= 1.0
+    R[~valid] = 0.0
+    return R
+
+
+def batch_mean_residual(R, n_t):
+    """s_t = N_t^-1 sum_{i in I_t} r_i (ignored rows of R are zero)."""
+    return R.sum(axis=0) / n_t
+
+
+def ema_update(q_prev, s, t, beta1):
+    """q_t = beta1 q_{t-1} + (1 - beta1) s_t and qhat_t = q_t / (1 - beta1^t)."""
+    q = beta1 * np.asarray(q_prev, dtype=F64) + (1.0 - beta1) * np.asarray(s, dtype=F64)
+    qhat = q / (1.0 - beta1 ** t)
+    return q, qhat
+
+
+def cross_entropy(Z, labels, valid, n_t):
+    lse = log_sum_exp_rows(Z)
+    rows = np.nonzero(valid)[0]
+    zy = Z[rows, np.asarray(labels)[rows]]
+    return float((lse[rows] - zy).sum() / n_t), lse
+
+
+def bom_step(layers, head_bias, params, X, labels, q_prev, t, lam=0.5, beta1=0.9,
+             ignore_index=-100) -> Dict[str, object]:
+    """One BOM step up to the update numerator (Algorithm 1, first five steps).
+
+    Returns a dict with the logits ``Z``, row log-sum-exp ``lse``, ``ce``,
+    ``n_t``, ``valid``, ``s``, ``q``, ``qhat`` and per-tensor lists ``g``, ``h``,
+    ``u``, plus the head-input cotangents ``dx_g``, ``dx_h``, ``dx_u``."""
+    if t < 1:
+        raise OracleError("t is 1-based")
+    params = [np.asarray(p, dtype=F64) for p in params]
+    Z, saved = forward(layers, head_bias, params, X)
+    d_out = Z.shape[1]
+    valid, n_t = supervised_set(labels, d_out, ignore_index)
+    R = residuals(Z, labels, valid)
+    s = batch_mean_residual(R, n_t)
+    q, qhat = ema_update(q_prev, s, t, beta1)
+    ce, lse = cross_entropy(Z, labels, valid, n_t)
+    # Logit cotangents of the three objectives.
+    d_g = R / n_t                                   # CE part: g
+    d_h = valid[:, None] * qhat[None, :] / n_t      # surrogate part: Jbar^T qhat
+    d_u = (1.0 - lam) * d_g + lam * d_h             # L_mix (Eq. mix-objective)
+    g, dx_g = backward(layers, head_bias, params, saved, d_g)
+    h, dx_h = backward(layers, head_bias, params, saved, d_h)
+    u, dx_u = backward(layers, head_bias, params, saved, d_u)
+    return dict(Z=Z, lse=lse, ce=ce, n_t=n_t, valid=valid, R=R, s=s, q=q, qhat=qhat,
+                g=g, h=h, u=u, dx_g=dx_g, dx_h=dx_h, dx_u=dx_u)
+
+
+# --------------------------------------------------------------------------
+# BOM-AdamW update (Section 3.4; Algorithm 1, last two steps)
+# --------------------------------------------------------------------------
+def bom_update(theta, u, v, lr, wd, t, beta2=0.999, eps=1e-8):
+    """Returns (theta_new, v_new) in float64."""
+    if t < 1:
+        raise OracleError("t is 1-based")
+    theta = np.asarray(theta, dtype=F64)
+    u = np.asarray(u, dtype=F64)
+    v_new = beta2 * np.asarray(v, dtype=F64) + (1.0 - beta2) * u * u
+    vhat = v_new / (1.0 - beta2 ** t)
+    theta_new = (1.0 - lr * wd) * theta - lr * u / (np.sqrt(vhat) + eps)
+    return theta_new, v_new
+
+
+def mix_numerator(g, h, lam):
+    """u = (1 - lambda) g + lambda h (Eq. mix-gradient)."""
+    return (1.0 - lam) * np.asarray(g, dtype=F64) + lam * np.asarray(h, dtype=F64)
+
+
+def bom_update_gh(theta, g, h, v, lr, wd, lam, t, beta2=0.999, eps=1e-8):
+    """Update from the separate supervised gradient g and reprojection h."""
+    return bom_update(theta, mix_numerator(g, h, lam), v, lr, wd, t, beta2, eps)

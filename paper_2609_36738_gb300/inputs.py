@@ -1,0 +1,242 @@
+"""Seeded synthetic workloads for the BOM task-space momentum pass.
+
+This module only *generates data*: model shapes, parameter initialisations,
+batches of inputs and labels, and the flat buffers of the update sweep.  It
+holds none of the method's arithmetic (no softmax, no residual, no EMA, no
+gradient, no update rule), so that the fp64 oracle under ``oracle/`` and the
+CUDA path can both be fed from it without sharing any computation.
+
+Every tensor comes from ``numpy.random.default_rng([seed, tag])`` (PCG64), so
+the same seed yields the same bytes on x86 and on Arm.  bf16 tensors are
+returned as their raw ``uint16`` bit patterns (round-to-nearest-even from the
+float32 draw); the float value each side computes with is exactly the value
+those bits encode.
+
+Workloads (shapes follow the paper's settings; the data are synthetic because
+the paper's corpora and datasets are not available here):
+
+* ``tiny_mlp_f32``     64 -> 128 (GELU) -> 10 classes, batch 32, fp32
+  (the STL10-like classification setting of Table cost-model, B*C = 320).
+* ``vision_head_bf16`` 768 -> 3072 -> 768 (GELU after each) -> 1000 classes,
+  batch 256, bf16 (ImageNet-like output space, B = 256, C = 1000).
+* ``lm_head_bf16``     hidden states 8192 x 768, head 50257 x 768, Zipf(1.1)
+  next-token labels (the vocabulary-space construction of the LM appendix).
+* ``lm_mlp_bf16``      two SwiGLU MLP sublayers (d = 2048, ffn = 8192) under a
+  32000-token head, 16384 tokens, Zipf(1.1) labels.
+* update sweep         flat fp32 theta / fp32 h / fp32 v and bf16 g buffers.
+
+Small variants with the same structure and ragged sizes serve the parity
+tests.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import List, Optional, Sequence, Tuple
+
+import numpy as np
+
+IGNORE_INDEX = -100
+
+# Layer kinds of the backbone, in the order the C interface numbers them.
+LINEAR = "linear"
+LINEAR_GELU = "linear_gelu"
+SWIGLU = "swiglu"
+
+
+# --------------------------------------------------------------------------
+# bf16 storage helpers (bit-level data marshalling only)
+# --------------------------------------------------------------------------
+def bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round float32 values to bf16 (nearest, ties to even); return uint16 bits."""
+    f = np.ascontiguousarray(x, dtype=np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    nan = np.isnan(f)
+    rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    out = rounded.astype(np.uint16)
+    out[nan] = 0x7FC0
+    return out
+
+
+def bf16_to_f32(bits: np.ndarray) -> np.ndarray:
+    """Expand uint16 bf16 bit patterns to the float32 values they encode."""
+    b = np.ascontiguousarray(bits, dtype=np.uint16)
+    return (b.astype(np.uint32) << 16).view(np.float32)
+
+
+def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
+    return bf16_to_f32(bits).astype(np.float64)
+
+
+# --------------------------------------------------------------------------
+# Model / workload description
+# --------------------------------------------------------------------------
+@dataclasses.dataclass(frozen=True)
+class Layer:
+    kind: str          # LINEAR, LINEAR_GELU or SWIGLU
+    d_in: int          # input width (d_model for SWIGLU)
+    d_out: int         # output width (ffn width for SWIGLU; output stays d_model)
+    has_bias: bool = False
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    n_rows: int                  # supervised rows per batch (examples / tokens)
+    d_in: int                    # width of the input X
+    layers: Tuple[Layer, ...]    # backbone, applied in order
+    vocab: int                   # d_out of the head (classes / vocabulary)
+    head_bias: bool
+    dtype: str                   # "f32" or "bf16"
+    labels: str                  # "uniform" or "zipf"
+    steps: int = 1
+    head_init: str = "kaiming"   # "kaiming" or "normal002"
+    ignore_frac: float = 0.0     # fraction of rows whose label is IGNORE_INDEX
+
+    @property
+    def d_model(self) -> int:
+        w = self.d_in
+        for l in self.layers:
+            w = l.d_in if l.kind == SWIGLU else l.d_out
+        return w
+
+    def param_shapes(self) -> List[Tuple[str, Tuple[int, ...], bool]]:
+        """(name, shape, is_matrix) of every trainable tensor, in interface order."""
+        out = []
+        w = self.d_in
+        for li, l in enumerate(self.layers):
+            if l.kind == SWIGLU:
+                assert l.d_in == w
+                out.append((f"l{li}.w_gate", (l.d_out, l.d_in), True))
+                out.append((f"l{li}.w_up", (l.d_out, l.d_in), True))
+                out.append((f"l{li}.w_down", (l.d_in, l.d_out), True))
+            else:
+                assert l.d_in == w
+                out.append((f"l{li}.weight", (l.d_out, l.d_in), True))
+                if l.has_bias:
+                    out.append((f"l{li}.bias", (l.d_out,), False))
+                w = l.d_out
+        out.append(("head.weight", (self.vocab, w), True))
+        if self.head_bias:
+            out.append(("head.bias", (self.vocab,), False))
+        return out
+
+    def n_params(self) -> int:
+        return int(sum(int(np.prod(s)) for _, s, _ in self.param_shapes()))
+
+
+def _rng(seed: int, *tag: int) -> np.random.Generator:
+    return np.random.default_rng([int(seed) & 0xFFFFFFFF, *[int(t) for t in tag]])
+
+
+def _store(x32: np.ndarray, dtype: str) -> np.ndarray:
+    return bf16_bits(x32) if dtype == "bf16" else np.ascontiguousarray(x32, dtype=np.float32)
+
+
+def init_params(wl: Workload, seed: int = 0) -> List[np.ndarray]:
+    """Initial parameters in storage form (float32, or bf16 bits as uint16).
+
+    Matrices: Kaiming-uniform U(-sqrt(6/fan_in), +sqrt(6/fan_in)); the LM head
+    uses N(0, 0.02) when ``head_init == "normal002"``.  Biases start at zero.
+    """
+    out = []
+    for k, (name, shape, is_mat) in enumerate(wl.param_shapes()):
+        g = _rng(seed, 1000 + k)
+        if not is_mat:
+            x = np.zeros(shape, dtype=np.float32)
+        elif name == "head.weight" and wl.head_init == "normal002":
+            x = (g.standard_normal(shape, dtype=np.float32) * np.float32(0.02))
+        else:
+            bound = np.float32(np.sqrt(6.0 / shape[1]))
+            x = g.uniform(-1.0, 1.0, size=shape).astype(np.float32) * bound
+        out.append(_store(x, wl.dtype))
+    return out
+
+
+def zipf_labels(g: np.random.Generator, n: int, vocab: int, a: float = 1.1) -> np.ndarray:
+    """Zipf(a) over ranks 1..vocab (truncated), rank k -> token id k-1 (inverse CDF)."""
+    ranks = np.arange(1, vocab + 1, dtype=np.float64)
+    w = ranks ** (-a)
+    cdf = np.cumsum(w)
+    cdf /= cdf[-1]
+    u = g.random(n)
+    idx = np.searchsorted(cdf, u, side="right")
+    return np.minimum(idx, vocab - 1).astype(np.int32)
+
+
+def make_batch(wl: Workload, seed: int = 0, step: int = 1) -> Tuple[np.ndarray, np.ndarray]:
+    """(X, labels) for optimizer step ``step`` (1-based).  X is N(0,1)."""
+    g = _rng(seed, 2000 + step)
+    x = g.standard_normal((wl.n_rows, wl.d_in), dtype=np.float32)
+    if wl.labels == "zipf":
+        y = zipf_labels(g, wl.n_rows, wl.vocab)
+    else:
+        y = g.integers(0, wl.vocab, size=wl.n_rows, dtype=np.int64).astype(np.int32)
+    if wl.ignore_frac > 0:
+        drop = g.random(wl.n_rows) < wl.ignore_frac
+        y[drop] = IGNORE_INDEX
+    return _store(x, wl.dtype), y
+
+
+def weight_decay_mask(wl: Workload, omega: float) -> List[float]:
+    """Decoupled weight-decay coefficient per tensor: omega for matrices, 0 for biases."""
+    return [omega if is_mat else 0.0 for _, _, is_mat in wl.param_shapes()]
+
+
+# --------------------------------------------------------------------------
+# Named workloads
+# --------------------------------------------------------------------------
+TINY_MLP_F32 = Workload("tiny_mlp_f32", 32, 64, (Layer(LINEAR_GELU, 64, 128, True),),
+                        10, True, "f32", "uniform", steps=5)
+VISION_HEAD_BF16 = Workload("vision_head_bf16", 256, 768,
+                            (Layer(LINEAR_GELU, 768, 3072, True), Layer(LINEAR_GELU, 3072, 768, True)),
+                            1000, True, "bf16", "uniform", steps=20)
+LM_HEAD_BF16 = Workload("lm_head_bf16", 8192, 768, (), 50257, False, "bf16", "zipf",
+                        head_init="normal002")
+LM_MLP_BF16 = Workload("lm_mlp_bf16", 16384, 2048,
+                       (Layer(SWIGLU, 2048, 8192), Layer(SWIGLU, 2048, 8192)),
+                       32000, False, "bf16", "zipf", head_init="normal002")
+UPDATE_SIZES = (10_000_000, 125_000_000, 1_000_000_000)
+
+# Small variants: same structure, ragged sizes (not multiples of the tiles).
+LM_HEAD_SMALL = Workload("lm_head_small", 300, 136, (), 1003, False, "bf16", "zipf",
+                         head_init="normal002", ignore_frac=0.1)
+LM_MLP_SMALL = Workload("lm_mlp_small", 260, 128,
+                        (Layer(SWIGLU, 128, 320), Layer(SWIGLU, 128, 320)),
+                        777, False, "bf16", "zipf", head_init="normal002", ignore_frac=0.05)
+VISION_SMALL = Workload("vision_small", 70, 96,
+                        (Layer(LINEAR_GELU, 96, 200, True), Layer(LINEAR_GELU, 200, 88, True)),
+                        130, True, "bf16", "uniform", steps=3)
+TINY_RAGGED_F32 = Workload("tiny_ragged_f32", 37, 29, (Layer(LINEAR_GELU, 29, 45, True),
+                                                       Layer(LINEAR, 45, 33, True)),
+                           7, True, "f32", "uniform", steps=3, ignore_frac=0.1)
+
+WORKLOADS = {w.name: w for w in (TINY_MLP_F32, VISION_HEAD_BF16, LM_HEAD_BF16, LM_MLP_BF16,
+                                  LM_HEAD_SMALL, LM_MLP_SMALL, VISION_SMALL, TINY_RAGGED_F32)}
+
+
+# --------------------------------------------------------------------------
+# Update sweep buffers
+# --------------------------------------------------------------------------
+def update_sweep_host(n: int, seed: int = 0):
+    """theta, g (bf16 bits), h, v for the flat update sweep: N(0, 1e-3) values,
+    v = (N(0, 1e-3))^2 >= 0."""
+    g = _rng(seed, 3000)
+    theta = g.standard_normal(n, dtype=np.float32) * np.float32(1e-3)
+    grad = bf16_bits(g.standard_normal(n, dtype=np.float32) * np.float32(1e-3))
+    h = g.standard_normal(n, dtype=np.float32) * np.float32(1e-3)
+    z = g.standard_normal(n, dtype=np.float32) * np.float32(1e-3)
+    v = z * z
+    return theta, grad, h, v
+
+
+def update_sweep_device(n: int, seed: int, device):
+    """Same distribution as :func:`update_sweep_host`, drawn on the device with a
+    seeded ``torch.Generator`` (used where the host would take too long)."""
+    import torch
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed) * 7919 + 3000)
+    theta = torch.randn(n, generator=gen, device=device, dtype=torch.float32).mul_(1e-3)
+    grad = torch.randn(n, generator=gen, device=device, dtype=torch.float32).mul_(1e-3).to(torch.bfloat16)
+    h = torch.randn(n, generator=gen, device=device, dtype=torch.float32).mul_(1e-3)
+    v = torch.randn(n, generator=gen, device=device, dtype=torch.float32).mul_(1e-3).square_()
+    return theta, grad, h, v
