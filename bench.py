@@ -1,0 +1,454 @@
+#!/usr/bin/env python
+"""Benchmark of the BOM (Backpropagated Output Momentum) hot path on GB300.
+
+One timed step = one pass of the whole path over one batch: backbone forward
+(two SwiGLU MLP sublayers), logits + cross-entropy statistics, residuals, s_t,
+the q_t EMA, the head and backbone backward with the reprojection folded in,
+and the BOM-AdamW update of every parameter.  The workload is the largest
+single-GPU configuration: 16384 tokens, d = 2048, ffn = 8192, vocabulary 32000,
+166,199,296 parameters (fp32 master weights, bf16 compute copies).
+
+Prints ONE JSON line (rank 0).  Besides the headline tokens/s it carries the
+roofline of the dominant kernel (device time measured with CUDA events around
+its launches inside the timed steps), the end-to-end number through host
+buffers, the clocks sampled during the timed region, and the oracle timed on
+the host cores on a bounded sample (cpu_baseline).  Two sub-measurements of the
+same metric family ride along: the head-only LM output block (8192 x 768 x
+50257) in tokens/s and the update alone over 1e9 elements in GB/s.
+
+--impl reference times the fp64 CPU oracle on the host cores instead (the
+only reference implementation this method has here).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2609_36738_gb300 import inputs as I  # noqa: E402
+
+METRIC = "BOM step tokens/s (fused head+reprojection) and update GB/s vs GB300 roofline"
+LR, WD, LAM, B1, B2, EPS = 1e-3, 0.1, 0.5, 0.9, 0.999, 1e-8
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def _args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default="lm_mlp_bf16")
+    p.add_argument("--no-extra", action="store_true", help="skip the head-only and update sub-measurements")
+    p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
+    return p.parse_args()
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        d = json.load(open(path))
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def _workload_desc(wl):
+    if wl.name == "lm_mlp_bf16":
+        return ("LM output block + 2 SwiGLU MLP sublayers: 16384 tokens, d=2048, ffn=8192, vocab 32000, "
+                "full BOM backward and BOM-AdamW update over 166,199,296 params")
+    return wl.name
+
+
+# --------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.hw_slowdown",
+              "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
+              "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = os.path.join("/tmp", f"bom_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={','.join(self.FIELDS)}", "--format=csv,noheader,nounits",
+                 "-i", str(self.gpu_id), "-lms", "200"], stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        os.remove(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------- CPU oracle legs
+_ORACLE_INPUTS = {}
+
+
+def oracle_sample(wl, seed=0, n_rows=None, budget_s=15.0):
+    """Times the fp64 oracle on a bounded sample of the workload: one BOM step on
+    the first n_rows rows of the batch through the full-size network, plus the
+    update over the same fraction of the parameters.  Returns (tokens/s, desc)."""
+    import oracle as O
+    key = (wl.name, seed)
+    if key not in _ORACLE_INPUTS:
+        params = I.init_params(wl, seed)
+        p64 = [I.bf16_to_f64(p) if wl.dtype == "bf16" else p.astype(np.float64) for p in params]
+        x, y = I.make_batch(wl, seed, 1)
+        xs = I.bf16_to_f64(x) if wl.dtype == "bf16" else x.astype(np.float64)
+        _ORACLE_INPUTS.clear()
+        _ORACLE_INPUTS[key] = (p64, xs, y)
+    p64, xs, y = _ORACLE_INPUTS[key]
+    layers = [(l.kind, l.d_in, l.d_out, l.has_bias) for l in wl.layers]
+    n = n_rows or 16
+    while True:
+        t0 = time.perf_counter()
+        out = O.bom_step(layers, wl.head_bias, p64, xs[:n], y[:n], np.zeros(wl.vocab), 1)
+        frac = n / wl.n_rows
+        for k, p in enumerate(p64):
+            m = max(1, int(p.size * frac))
+            O.bom_update(p.ravel()[:m], out["u"][k].ravel()[:m], np.zeros(m), LR, WD, 1, B2, EPS)
+        dt = time.perf_counter() - t0
+        if n_rows is not None or dt > budget_s / 4 or n * 2 > wl.n_rows:
+            break
+        n *= 2
+    desc = (f"{n} of {wl.n_rows} rows through the full-size network (forward, task-space pass, the "
+            f"oracle's three reverse passes for g, h and u) + the update over {n}/{wl.n_rows} of the "
+            f"{wl.n_params()} parameters; fp64 numpy")
+    return n / dt, desc, n
+
+
+def run_reference(a):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    wl = I.WORKLOADS[a.workload]
+    cores = os.cpu_count()
+    _, desc, n = oracle_sample(wl, budget_s=8.0)
+    for _ in range(a.warmup):
+        oracle_sample(wl, n_rows=n)
+    vals = []
+    t_all = time.perf_counter()
+    for _ in range(a.steps):
+        v, _, _ = oracle_sample(wl, n_rows=n)
+        vals.append(v)
+    total = time.perf_counter() - t_all
+    value = a.steps * n / total
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": a.steps, "warmup": a.warmup, "ms_per_step": 1e3 * total / a.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": _workload_desc(wl), "sample_rows_per_step": n},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": desc},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------- GPU leg
+def main():
+    a = _args()
+    if a.impl == "reference":
+        return run_reference(a)
+    import torch
+
+    from paper_2609_36738_gb300 import bom as B
+    from paper_2609_36738_gb300 import build as builder
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if rank == 0:
+        builder.build()
+    if dist is not None:
+        dist.barrier()
+    B.lib()
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+    peaks, peak_src = _peaks()
+
+    # ---------------------------------------------------------------- workload state
+    wl = I.WORKLOADS[a.workload]
+    params_np = I.init_params(wl, seed=rank)
+    shapes = [s for _, s, _ in wl.param_shapes()]
+    sizes = [int(np.prod(s)) for s in shapes]
+    offs = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int64)
+    # pad every tensor to 8 elements so each view is 16-byte aligned
+    offs_al = np.concatenate([[0], np.cumsum([(s + 7) // 8 * 8 for s in sizes])]).astype(np.int64)
+    P = int(offs_al[-1])
+    bf16 = wl.dtype == "bf16"
+    master = torch.zeros(P, dtype=torch.float32, device=dev)
+    shadow = torch.zeros(P, dtype=torch.bfloat16 if bf16 else torch.float32, device=dev)
+    gradf = torch.zeros(P, dtype=shadow.dtype, device=dev)
+    vstate = torch.zeros(P, dtype=torch.float32, device=dev)
+    for k, p in enumerate(params_np):
+        o = int(offs_al[k])
+        vals = I.bf16_to_f32(p) if bf16 else p
+        master[o:o + sizes[k]] = torch.from_numpy(vals.ravel()).to(dev)
+    shadow.copy_(master.to(shadow.dtype))
+    pviews = [shadow[int(offs_al[k]):int(offs_al[k]) + sizes[k]].view(shapes[k]) for k in range(len(shapes))]
+    gviews = [gradf[int(offs_al[k]):int(offs_al[k]) + sizes[k]].view(shapes[k]) for k in range(len(shapes))]
+    x_np, y_np = I.make_batch(wl, seed=rank, step=1)
+    x_host = torch.from_numpy(x_np.view(np.int16) if bf16 else x_np).pin_memory()
+    y_host = torch.from_numpy(y_np).pin_memory()
+    x_dev = (x_host.to(dev).view(torch.bfloat16) if bf16 else x_host.to(dev))
+    y_dev = y_host.to(dev)
+    q = torch.zeros(wl.vocab, dtype=torch.float32, device=dev)
+    model = B.BomModel(B.config_for(wl, LAM, B1))
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)   # 256 MiB > L2
+    gt = B.BOM_BF16 if bf16 else B.BOM_F32
+    N = wl.n_rows
+
+    def step(t, xx=x_dev, yy=y_dev):
+        model.step(xx, yy, N, pviews, q, t, gviews, None, stream)
+        B.bom_update(master, gradf, gt, None, vstate, shadow if bf16 else None, P, LR, WD, LAM, B2, EPS, t, stream)
+
+    t = 0
+    for _ in range(a.warmup):
+        t += 1
+        step(t)
+    model.stats(stream)   # sync + raises if the device latched an error
+
+    # ---------------------------------------------------------------- timed region
+    props = torch.cuda.get_device_properties(dev)
+    if all(hasattr(props, f) for f in ("pci_domain_id", "pci_bus_id", "pci_device_id")):
+        gpu_id = f"{props.pci_domain_id:08X}:{props.pci_bus_id:02X}:{props.pci_device_id:02X}.0"
+    else:
+        gpu_id = local
+    clocks = ClockSampler(gpu_id)
+    B.bom_trace(model.h, True)
+    per_kernel = {}
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(a.steps)]
+    launches0 = B.bom_launch_count()
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    for i in range(a.steps):
+        flush.zero_()
+        t += 1
+        ev[i][0].record(stream)
+        step(t)
+        ev[i][1].record(stream)
+        for name, fl, by, ms in B.bom_trace_read(model.h, stream):
+            d = per_kernel.setdefault(name, [0.0, 0.0, 0.0, 0])
+            d[0] += fl
+            d[1] += by
+            d[2] += ms
+            d[3] += 1
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    launches = B.bom_launch_count() - launches0
+    B.bom_trace(model.h, False)
+    st = model.stats(stream)
+    step_ms = [e0.elapsed_time(e1) for e0, e1 in ev]
+    tot_ms = sum(step_ms)
+    if dist is not None:
+        tt = torch.tensor([tot_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        tot_ms = float(tt.item())
+    value = world * N * a.steps / (tot_ms / 1e3)
+
+    # ---------------------------------------------------------------- dominant kernel roofline
+    dom = max(per_kernel.items(), key=lambda kv: kv[1][2])
+    total_dev = sum(v[2] for v in per_kernel.values())
+    name, (fl, by, ms, cnt) = dom
+    if fl > 0:
+        achieved = fl / (ms / 1e3) / 1e12
+        roof = {"bound": "tensor", "kernel": name, "achieved": achieved, "peak": peaks["bf16_tflops_sustained"],
+                "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops_sustained"],
+                "peak_source": f"{peak_src} (sustained bf16; kernel timed inside a long step)",
+                "flops_per_launch": fl / cnt, "launches": cnt, "avg_launch_ms": ms / cnt,
+                "share_of_device_time": ms / total_dev}
+    else:
+        achieved = by / (ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "kernel": name, "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"], "peak_source": peak_src, "bytes_per_launch": by / cnt,
+                "launches": cnt, "avg_launch_ms": ms / cnt, "share_of_device_time": ms / total_dev}
+    # GEMM engine as a whole (all tcgen05 launches of the step)
+    gem = [v for k, v in per_kernel.items() if k.startswith("gemm_tc")]
+    if gem:
+        gfl = sum(v[0] for v in gem)
+        gms = sum(v[2] for v in gem)
+        roof["all_gemm_tflops"] = gfl / (gms / 1e3) / 1e12
+        roof["all_gemm_frac"] = roof["all_gemm_tflops"] / peaks["bf16_tflops_sustained"]
+        roof["all_gemm_share_of_device_time"] = gms / total_dev
+    roof["traffic"] = _ncu_traffic(name)
+
+    kernels = {k: {"ms_per_step": v[2] / a.steps, "launches_per_step": v[3] / a.steps,
+                   "tflops": (v[0] / (v[2] / 1e3) / 1e12) if v[0] else None,
+                   "gbs": v[1] / (v[2] / 1e3) / 1e9} for k, v in sorted(per_kernel.items(), key=lambda kv: -kv[1][2])}
+
+    # ---------------------------------------------------------------- end to end through host buffers
+    e2e_steps = max(3, a.steps // 2)
+    h2d = x_host.numel() * x_host.element_size() + y_host.numel() * y_host.element_size()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(e2e_steps):
+        t += 1
+        xx = x_host.to(dev, non_blocking=True)
+        yy = y_host.to(dev, non_blocking=True)
+        step(t, xx.view(torch.bfloat16) if bf16 else xx, yy)
+        model.stats(stream)        # device -> host read of the step's loss / status (syncs)
+    e2e_s = time.perf_counter() - t0
+    e2e = {"value": world * N * e2e_steps / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+           "d2h_bytes_per_step": B.STATS_D2H_BYTES}
+
+    # ---------------------------------------------------------------- sub-measurements
+    extra = {}
+    if not a.no_extra and rank == 0:
+        extra["lm_head_bf16"] = _head_only(B, torch, dev, stream, a, peaks)
+        extra["update_1e9"] = _update_only(B, torch, dev, stream, a, peaks)
+
+    cpu = None
+    if rank == 0 and world == 1 and not a.no_cpu:
+        v, desc, _ = oracle_sample(wl)
+        cpu = {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle", "sample": desc}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": a.steps,
+                "warmup": a.warmup, "ms_per_step": tot_ms / a.steps, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16" if bf16 else "f32",
+                "data": "synthetic: seeded N(0,1) inputs, Kaiming-uniform MLP weights, N(0,0.02) head, "
+                        "Zipf(1.1) labels",
+                "config": {"workload": _workload_desc(wl), "global_batch": world * N, "tokens_per_gpu": N,
+                           "parallelism": f"replicas x{world} (no data-path collective)",
+                           "l2": "flushed between timed steps (256 MiB write outside the step events)",
+                           "lr": LR, "weight_decay": WD, "lambda": LAM, "beta1": B1, "beta2": B2},
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
+                "clocks": clk, "loss": st["loss"], "kernels": kernels, "sub": extra}
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def _ncu_traffic(kernel_name):
+    """DRAM bytes per launch of `kernel_name` from the committed ncu summary,
+    valid only while the kernel source is unchanged since the capture."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(path):
+        return None
+    try:
+        import hashlib
+        d = json.load(open(path))
+        rec = d.get(kernel_name)
+        if not rec:
+            return None
+        src = open(os.path.join(ROOT, rec["source"]), "rb").read()
+        if hashlib.sha256(src).hexdigest() != rec["sha256"]:
+            return None
+        return rec["dram_bytes_per_launch"]
+    except Exception:
+        return None
+
+
+def _head_only(B, torch, dev, stream, a, peaks):
+    """LM output block alone: 8192 tokens x d 768, vocab 50257 (forward logits,
+    CE statistics, residuals, s/q, head dW and dH with the reprojection)."""
+    wl = I.LM_HEAD_BF16
+    params = [torch.from_numpy(p.view(np.int16)).to(dev).view(torch.bfloat16) for p in I.init_params(wl, 0)]
+    x_np, y_np = I.make_batch(wl, 0, 1)
+    x = torch.from_numpy(x_np.view(np.int16)).to(dev).view(torch.bfloat16)
+    y = torch.from_numpy(y_np).to(dev)
+    grads = [torch.empty_like(p) for p in params]
+    dx = torch.empty_like(x)
+    q = torch.zeros(wl.vocab, dtype=torch.float32, device=dev)
+    m = B.BomModel(B.config_for(wl))
+    B.bom_set_input_grad(m.h, dx)
+    for t in range(1, a.warmup + 1):
+        m.step(x, y, wl.n_rows, params, q, t, grads, None, stream)
+    m.stats(stream)
+    B.bom_trace(m.h, True)
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)
+    tot = 0.0
+    gem_fl = gem_ms = 0.0
+    for i in range(a.steps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        m.step(x, y, wl.n_rows, params, q, a.warmup + 1 + i, grads, None, stream)
+        e1.record(stream)
+        for name, fl, by, ms in B.bom_trace_read(m.h, stream):
+            if name.startswith("gemm_tc"):
+                gem_fl += fl
+                gem_ms += ms
+        tot += e0.elapsed_time(e1)
+    m.stats(stream)
+    m.close()
+    flops = 3 * 2.0 * wl.n_rows * wl.d_in * wl.vocab
+    return {"workload": "LM output block: H 8192x768, head 50257x768 (tied-head shape), Zipf(1.1) labels; "
+                        "logits + CE, residuals, s_t, q_t, head dW and dH with the reprojection",
+            "value": wl.n_rows * a.steps / (tot / 1e3), "unit": "tokens/s", "ms_per_step": tot / a.steps,
+            "step_tflops": flops / (tot / a.steps / 1e3) / 1e12,
+            "step_frac_of_bf16_peak": flops / (tot / a.steps / 1e3) / 1e12 / peaks["bf16_tflops"],
+            "gemm_tflops": gem_fl / (gem_ms / 1e3) / 1e12 if gem_ms else None}
+
+
+def _update_only(B, torch, dev, stream, a, peaks):
+    """BOM-AdamW update alone over 1e9 elements (fp32 theta/h/v, bf16 g)."""
+    n = I.UPDATE_SIZES[-1]
+    theta, g, h, v = I.update_sweep_device(n, 0, dev)
+    for t in range(1, 4):
+        B.bom_update(theta, g, B.BOM_BF16, h, v, None, n, LR, 0.01, LAM, B2, EPS, t, stream)
+    torch.cuda.synchronize()
+    ms = []
+    for i in range(max(5, a.steps // 2)):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        B.bom_update(theta, g, B.BOM_BF16, h, v, None, n, LR, 0.01, LAM, B2, EPS, 4 + i, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    med = statistics.median(ms)
+    gbs = 22.0 * n / (med / 1e3) / 1e9
+    del theta, g, h, v
+    torch.cuda.empty_cache()
+    return {"workload": "update sweep, 1e9 elements: read theta f32, g bf16, h f32, v f32; write theta, v "
+                        "(22 B/element)", "value": gbs, "unit": "GB/s", "ms": med,
+            "frac_of_hbm": gbs / peaks["hbm_gbs"], "peak_source": "measured copy bandwidth"}
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,215 @@
+/*
+ * bom.h - C ABI of the GB300-native BOM (Backpropagated Output Momentum)
+ *         task-space momentum pass.
+ *
+ * One optimizer step of BOM (paper, Algorithm 1) splits into two calls:
+ *
+ *   bom_step    forward through the backbone and the linear head, the
+ *               residuals r_i = softmax(z_i) - onehot(y_i), their batch mean
+ *               s_t over the supervised set I_t, the task-space EMA
+ *               q_t = beta1 q_{t-1} + (1-beta1) s_t with qhat_t = q_t/(1-beta1^t),
+ *               and ONE backward pass of the logit cotangent
+ *               N_t^-1 [(1-lambda) r_i + lambda qhat_t], which yields the
+ *               update numerator u = (1-lambda) g + lambda Jbar^T qhat for
+ *               every tensor (Section 3.2, Eq. mix-objective and Eq. mix-gradient;
+ *               LM construction appendix for I_t and N_t).
+ *   bom_update  v = beta2 v + (1-beta2) u^2, vhat = v/(1-beta2^t),
+ *               theta <- (1 - lr*wd) theta - lr u/(sqrt(vhat)+eps)
+ *               (Section 3.4; Algorithm 1, last two steps).  No first-moment
+ *               state exists and no first-moment bias correction is applied.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every tensor argument is a caller-owned DEVICE pointer (cudaMalloc or a
+ *   PyTorch CUDA tensor), row-major and dense, unless stated otherwise.  The
+ *   library never frees or keeps caller pointers beyond the call.
+ * - bf16 values are passed as raw 16-bit patterns (uint16_t / void*).
+ * - `stream` is a cudaStream_t passed as void*; NULL means the legacy default
+ *   stream.  All work is enqueued asynchronously on it; no entry point except
+ *   bom_get_stats synchronises.
+ * - Host-checkable problems (null pointers, bad sizes, t < 1, unaligned
+ *   pointers) return an error immediately and enqueue nothing.  Problems only
+ *   the device can see (a bad label, N_t = 0, a bounded wait that ran out) are
+ *   latched in a device status word of the handle; every later kernel of the
+ *   step skips its work, q is left unmodified, and bom_get_stats returns the
+ *   latched code.  The word is cleared at the start of each bom_step.
+ * - Alignment: every bf16 tensor used by the tensor-core path needs a 16-byte
+ *   aligned base and a row length that is a multiple of 8 elements (TMA rule);
+ *   otherwise BOM_ENOTSUP.
+ */
+#ifndef BOM_H
+#define BOM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    BOM_OK = 0,
+    BOM_EINVAL = 1,    /* bad argument (host-detected, nothing enqueued)             */
+    BOM_ENOMEM = 2,    /* workspace allocation failed                                 */
+    BOM_ECUDA = 3,     /* a CUDA runtime / driver call failed                         */
+    BOM_ELABEL = 4,    /* device: a label outside [0, d_out) that is not ignore_index */
+    BOM_EEMPTY = 5,    /* device: N_t = 0 (Algorithm 1 requires N_t > 0)              */
+    BOM_ETIMEOUT = 6,  /* device: a bounded wait inside a kernel ran out              */
+    BOM_ENOTSUP = 7    /* shape or alignment this build does not handle               */
+} bom_status;
+
+typedef enum { BOM_F32 = 0, BOM_BF16 = 1 } bom_dtype;
+
+typedef enum {
+    BOM_LAYER_LINEAR = 0,       /* y = x W^T (+ b)                                         */
+    BOM_LAYER_LINEAR_GELU = 1,  /* y = GELU(x W^T (+ b)), exact erf GELU                  */
+    BOM_LAYER_SWIGLU = 2        /* y = x + W_d (SiLU(x W_g^T) * (x W_u^T)); d_out = ffn    */
+} bom_layer_kind;
+
+typedef enum {
+    BOM_OUT_U = 0,        /* one backward pass: grads[] receive u                        */
+    BOM_OUT_G_AND_H = 1   /* diagnostic: grads[] receive g (cotangent r_i/N_t) and      */
+                          /* h_out[] receive h = Jbar^T qhat (cotangent qhat/N_t)       */
+} bom_out_mode;
+
+typedef struct {
+    int32_t kind;      /* bom_layer_kind                                                */
+    int32_t has_bias;  /* LINEAR / LINEAR_GELU: 1 adds a bias of length d_out           */
+    int64_t d_in;      /* input width                                                   */
+    int64_t d_out;     /* output width (SWIGLU: the ffn width; output stays d_in)       */
+} bom_layer;
+
+typedef struct {
+    int64_t max_rows;         /* largest n_rows bom_step accepts (sizes the workspace)   */
+    int64_t d_in;             /* width of the input X                                   */
+    int64_t d_out;            /* classes / vocabulary size (head output width)          */
+    int32_t n_layers;         /* backbone layers before the head (0 = head only)        */
+    const bom_layer* layers;  /* host array of n_layers entries, copied by bom_init     */
+    int32_t head_bias;        /* 1: the head has a bias of length d_out                 */
+    int32_t compute;          /* bom_dtype of X, parameters and grads                   */
+    float lambda;             /* mixture weight (paper default 0.5)                     */
+    float beta1;              /* task-space EMA decay (paper default 0.9)               */
+    int32_t ignore_index;     /* label value excluded from I_t (usually -100)           */
+    int32_t out_mode;         /* bom_out_mode                                           */
+} bom_config;
+
+typedef struct {
+    float loss;          /* mean cross-entropy over I_t                               */
+    int32_t n_t;         /* |I_t|                                                     */
+    int32_t status;      /* bom_status latched on the device during the last step    */
+    float s_norm;        /* ||s_t||_2                                                */
+} bom_stats;
+
+typedef struct bom_handle bom_handle;
+
+/* Parameter tensors, in this order (the grads[] and h_out[] arrays follow the
+ * same order and shapes):
+ *   for each backbone layer:
+ *     LINEAR / LINEAR_GELU : W [d_out, d_in], then b [d_out] if has_bias
+ *     SWIGLU               : W_g [ffn, d], W_u [ffn, d], W_d [d, ffn]
+ *   head                   : W [d_out, d_model], then b [d_out] if head_bias
+ * bom_param_count returns the number of tensors (-1 for a malformed cfg);
+ * bom_param_shape the shape of tensor `index`: rows x cols for matrices, and
+ * rows = length, cols = 0 for bias vectors. */
+int32_t bom_param_count(const bom_config* cfg);
+bom_status bom_param_shape(const bom_config* cfg, int32_t index, int64_t* rows, int64_t* cols);
+
+/* Creates a handle: validates cfg, copies it, and allocates the device
+ * workspace (activations, logits/residuals, row statistics, column partial
+ * sums, scalars) for max_rows rows on the current device.  The handle owns
+ * only that workspace.  Returns BOM_EINVAL on a bad config, BOM_ENOMEM when
+ * the workspace does not fit. */
+bom_status bom_init(bom_handle** out, const bom_config* cfg);
+
+/* Bytes of device workspace bom_init would allocate for cfg. */
+int64_t bom_workspace_bytes(const bom_config* cfg);
+
+/* One BOM step (Algorithm 1 up to the update numerator).
+ *   x       [n_rows, d_in] compute dtype.
+ *   labels  [n_rows] int32; ignore_index rows are not supervised.
+ *   params  bom_param_count device pointers (compute dtype), read only.
+ *   q       [d_out] fp32, in/out: q_{t-1} on entry, q_t on exit (unchanged if
+ *           the device latches an error).
+ *   t       1-based step index (t >= 1) used by the bias correction.
+ *   grads   bom_param_count output pointers (compute dtype): u, or g in
+ *           BOM_OUT_G_AND_H mode.
+ *   h_out   BOM_OUT_G_AND_H only: bom_param_count fp32 outputs receiving h;
+ *           must be NULL in BOM_OUT_U mode.
+ * Requires 1 <= n_rows <= max_rows.  Not re-entrant on one handle: two steps
+ * on the same handle must be ordered on one stream. */
+bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                    void* const* params, float* q, int64_t t,
+                    void* const* grads, void* const* h_out, void* stream);
+
+/* Registers a device buffer dx [max_rows, d_in] (compute dtype) that every
+ * following bom_step fills with the cotangent of the input X (the u, or in
+ * BOM_OUT_G_AND_H mode the g, cotangent): for a head-only configuration
+ * this is dH = N_t^-1 [(1-lambda) R W + lambda 1_{I_t} (W^T qhat)^T], the
+ * input-side half of the head backward.  NULL disables it (the default). */
+bom_status bom_set_input_grad(bom_handle* h, void* dx);
+
+/* Device-side outputs of the last step that are useful for checks:
+ *   qhat [d_out] fp32, s [d_out] fp32, lse [n_rows] fp32 (row log-sum-exp).
+ * Pointers stay valid until bom_destroy; contents until the next bom_step. */
+bom_status bom_step_outputs(bom_handle* h, const float** qhat, const float** s, const float** lse);
+
+/* Synchronises `stream` and copies the statistics of the last step.  Returns
+ * the latched device status (BOM_OK when the step succeeded). */
+bom_status bom_get_stats(bom_handle* h, bom_stats* out, void* stream);
+
+/* BOM-AdamW update over a flat range of n elements (Section 3.4).
+ *   theta       [n] fp32 master parameters, updated in place.
+ *   g           [n] in g_dtype (BOM_F32 or BOM_BF16): u itself when hvec is
+ *               NULL, otherwise the supervised gradient g and the kernel forms
+ *               u = (1-lambda) g + lambda hvec (Eq. mix-gradient).
+ *   hvec        [n] fp32 reprojection h, or NULL.
+ *   v           [n] fp32 second moment, updated in place (v_0 = 0).
+ *   theta_bf16  [n] optional bf16 copy of the updated theta (NULL: none).
+ *   lr, wd      eta_t and the decoupled weight-decay coefficient omega.
+ *   t           1-based step index.
+ * All pointers 16-byte aligned.  n = 0 is a no-op. */
+bom_status bom_update(float* theta, const void* g, int32_t g_dtype, const float* hvec, float* v,
+                      uint16_t* theta_bf16, int64_t n, float lr, float wd, float lambda,
+                      float beta2, float eps, int64_t t, void* stream);
+
+/* Auxiliary: D = alpha * op(A) op(B)^T on the bf16 tensor-core GEMM engine the
+ * step uses (tcgen05 MMA, TMEM accumulators, TMA loads), fp32 accumulation,
+ * fp32 output D [M, N] with row pitch ldd.  A is M x K: a_mn_major = 0 means
+ * element (m,k) is at A[m*lda + k], 1 means at A[k*lda + m]; B likewise for
+ * N x K.  Exposed so the engine can be tested on its own. */
+bom_status bom_gemm_bf16(const uint16_t* A, int64_t lda, int32_t a_mn_major,
+                         const uint16_t* B, int64_t ldb, int32_t b_mn_major,
+                         float* D, int64_t ldd, int64_t M, int64_t N, int64_t K,
+                         float alpha, void* stream);
+
+/* Tracing (the measurement support of the step; the paper times whole steps
+ * with CUDA events, Appendix measurement-protocol).  While enabled on a
+ * handle, bom_step records a CUDA event pair on `stream` around every kernel
+ * it launches, with the algorithmic FLOPs and HBM bytes of that launch.
+ * bom_trace(h, 1) enables and clears the record, bom_trace(h, 0) disables. */
+typedef struct {
+    const char* name;   /* kernel class, e.g. "gemm_tc.logits" (static string)   */
+    double flops;       /* algorithmic floating-point operations of the launch   */
+    double bytes;       /* algorithmic HBM bytes of the launch                   */
+    float ms;           /* device time between the event pair                    */
+} bom_trace_entry;
+bom_status bom_trace(bom_handle* h, int32_t enable);
+
+/* Synchronises `stream`, then copies up to `max` entries of the launches of
+ * the most recent bom_step into `out`; returns how many the step recorded
+ * (or -1 on error). */
+int32_t bom_trace_read(bom_handle* h, bom_trace_entry* out, int32_t max, void* stream);
+
+/* Number of kernels this library has launched in the process so far. */
+int64_t bom_launch_count(void);
+
+/* Frees the workspace and the handle.  NULL is a no-op. */
+void bom_destroy(bom_handle* h);
+
+/* Static string naming a status code. */
+const char* bom_status_string(bom_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BOM_H */

@@ -148,7 +148,7 @@ def backward(layers, head_bias, params, saved, dZ):
     """Vector-Jacobian product of the logit cotangent dZ through the network.
 
     Returns (grads per parameter tensor in interface order, cotangent of the
-    head input)."""
+    head input, cotangent of the network input X)."""
     per_layer, (hw, hb) = _split_params(layers, head_bias, params)
     tape, h_last = saved
     dZ = np.asarray(dZ, dtype=F64)
@@ -184,7 +184,7 @@ def backward(layers, head_bias, params, saved, dZ):
                 grads_rev.append(dpre.sum(axis=0))
             grads_rev.append(g_w)
             dx = dpre @ w
-    return grads_rev[::-1], dx_head
+    return grads_rev[::-1], dx_head, dx
 
 
 # --------------------------------------------------------------------------
@@ -248,7 +248,8 @@ def bom_step(layers, head_bias, params, X, labels, q_prev, t, lam=0.5, beta1=0.9
 
     Returns a dict with the logits ``Z``, row log-sum-exp ``lse``, ``ce``,
     ``n_t``, ``valid``, ``s``, ``q``, ``qhat`` and per-tensor lists ``g``, ``h``,
-    ``u``, plus the head-input cotangents ``dx_g``, ``dx_h``, ``dx_u``."""
+    ``u``, plus the head-input cotangents ``dx_g``, ``dx_h``, ``dx_u`` and the
+    input cotangents ``dX_g``, ``dX_h``, ``dX_u``."""
     if t < 1:
         raise OracleError("t is 1-based")
     params = [np.asarray(p, dtype=F64) for p in params]
@@ -263,11 +264,11 @@ def bom_step(layers, head_bias, params, X, labels, q_prev, t, lam=0.5, beta1=0.9
     d_g = R / n_t                                   # CE part: g
     d_h = valid[:, None] * qhat[None, :] / n_t      # surrogate part: Jbar^T qhat
     d_u = (1.0 - lam) * d_g + lam * d_h             # L_mix (Eq. mix-objective)
-    g, dx_g = backward(layers, head_bias, params, saved, d_g)
-    h, dx_h = backward(layers, head_bias, params, saved, d_h)
-    u, dx_u = backward(layers, head_bias, params, saved, d_u)
+    g, dx_g, dX_g = backward(layers, head_bias, params, saved, d_g)
+    h, dx_h, dX_h = backward(layers, head_bias, params, saved, d_h)
+    u, dx_u, dX_u = backward(layers, head_bias, params, saved, d_u)
     return dict(Z=Z, lse=lse, ce=ce, n_t=n_t, valid=valid, R=R, s=s, q=q, qhat=qhat,
-                g=g, h=h, u=u, dx_g=dx_g, dx_h=dx_h, dx_u=dx_u)
+                g=g, h=h, u=u, dx_g=dx_g, dx_h=dx_h, dx_u=dx_u, dX_g=dX_g, dX_h=dX_h, dX_u=dX_u)
 
 
 # --------------------------------------------------------------------------

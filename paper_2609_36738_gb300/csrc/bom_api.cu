@@ -1,0 +1,702 @@
+// C ABI of the BOM task-space momentum pass: handle and workspace, argument
+// checks, and the orchestration of one step (Algorithm 1) as a sequence of
+// stream-ordered kernels.  Nothing here synchronises except bom_get_stats.
+//
+// Step, for a batch of n rows (paper: Algorithm 1; Section 3.2):
+//   forward   backbone GEMMs with fused bias/GELU/SwiGLU/residual epilogues,
+//             logits GEMM Z = H W^T (+b) whose epilogue stores Z and per-tile
+//             (max, sum exp) row statistics;
+//   task      label scan (N_t), row log-sum-exp, residual pass Z -> R with
+//             column partial sums, s_t, q_t = beta1 q + (1-beta1) s_t,
+//             qhat_t = q_t / (1-beta1^t), c = colsum_{I_t}(H), w = W^T qhat;
+//   backward  head dW = a R^T H + b qhat (x) c      (rank-1 epilogue),
+//             head dH = a R W + b 1_{I_t} w^T       (broadcast-row epilogue),
+//             then the backbone VJPs, with (a, b) = N_t^-1 (1-lambda, lambda)
+//             for u, N_t^-1 (1, 0) for g and N_t^-1 (0, 1) for h.
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <atomic>
+#include <vector>
+
+#include "gemm.h"
+#include "kernels.h"
+
+using namespace bom;
+
+namespace {
+
+struct LayerWs {
+    int kind = 0;
+    int64_t d_in = 0, d_out = 0;
+    bool bias = false;
+    int64_t width_out = 0;   // width of the layer output
+    void* pre = nullptr;     // LINEAR_GELU pre-activation [n, d_out]
+    void* out = nullptr;     // layer output [n, width_out]
+    void* G = nullptr;       // SWIGLU gate pre-activation [n, ffn]
+    void* U = nullptr;       // SWIGLU up projection [n, ffn]
+    void* A = nullptr;       // SWIGLU SiLU(G) * U [n, ffn]
+};
+
+int64_t round_up(int64_t a, int64_t b) { return (a + b - 1) / b * b; }
+
+}  // namespace
+
+struct bom_handle {
+    bom_config cfg{};
+    std::vector<bom_layer> layers;
+    std::vector<LayerWs> lw;
+    bool bf16 = false;
+    int64_t esz = 4;
+    int64_t d_model = 0;
+    int64_t max_width = 0;
+    int64_t max_ffn = 0;
+    char* ws = nullptr;
+    size_t ws_bytes = 0;
+    DevScalars* sc = nullptr;
+    void* Z = nullptr;
+    int64_t ldz = 0;
+    float* stats = nullptr;
+    int64_t ntiles = 1;
+    float* lse = nullptr;
+    float* ce = nullptr;
+    float* colpart = nullptr;
+    float* s = nullptr;
+    float* qhat = nullptr;
+    float* cvec = nullptr;
+    float* wvec = nullptr;
+    float* part = nullptr;
+    void* dx[2] = {nullptr, nullptr};
+    void* dG = nullptr;
+    void* dU = nullptr;
+    void* dx_in = nullptr;   // caller buffer for the cotangent of X (bom_set_input_grad)
+    int64_t last_n = 0;
+    // tracing: one event pair per launch of the current step
+    struct TraceRec {
+        const char* name = nullptr;
+        double flops = 0, bytes = 0;
+        cudaEvent_t a = nullptr, b = nullptr;
+    };
+    std::vector<TraceRec> trace;
+    int trace_n = 0;
+    bool tracing = false;
+};
+
+namespace bom {
+static std::atomic<long long> g_launches{0};
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+}  // namespace bom
+
+namespace {
+
+bom_status check_config(const bom_config* cfg, std::vector<LayerWs>* lw_out, int64_t* d_model, int64_t* max_width,
+                        int64_t* max_ffn) {
+    if (!cfg) return BOM_EINVAL;
+    if (cfg->max_rows < 1 || cfg->d_in < 1 || cfg->d_out < 1 || cfg->n_layers < 0) return BOM_EINVAL;
+    if (cfg->n_layers > 0 && !cfg->layers) return BOM_EINVAL;
+    if (cfg->compute != BOM_F32 && cfg->compute != BOM_BF16) return BOM_EINVAL;
+    if (cfg->out_mode != BOM_OUT_U && cfg->out_mode != BOM_OUT_G_AND_H) return BOM_EINVAL;
+    if (!(cfg->lambda >= 0.0f && cfg->lambda <= 1.0f)) return BOM_EINVAL;
+    if (!(cfg->beta1 >= 0.0f && cfg->beta1 < 1.0f)) return BOM_EINVAL;
+    if (cfg->max_rows > (1ll << 30) || cfg->d_out > (1ll << 30)) return BOM_ENOTSUP;
+    const bool bf16 = cfg->compute == BOM_BF16;
+    std::vector<LayerWs> lw;
+    int64_t w = cfg->d_in, mw = cfg->d_in, mf = 0;
+    for (int i = 0; i < cfg->n_layers; ++i) {
+        const bom_layer& L = cfg->layers[i];
+        LayerWs x;
+        x.kind = L.kind;
+        x.d_in = L.d_in;
+        x.d_out = L.d_out;
+        x.bias = L.has_bias != 0;
+        if (L.d_in != w || L.d_out < 1) return BOM_EINVAL;
+        if (L.kind == BOM_LAYER_SWIGLU) {
+            if (L.has_bias) return BOM_EINVAL;
+            if (!bf16) return BOM_ENOTSUP;
+            x.width_out = L.d_in;
+            mf = mf > L.d_out ? mf : L.d_out;
+        } else if (L.kind == BOM_LAYER_LINEAR || L.kind == BOM_LAYER_LINEAR_GELU) {
+            x.width_out = L.d_out;
+        } else {
+            return BOM_EINVAL;
+        }
+        w = x.width_out;
+        mw = mw > w ? mw : w;
+        mw = mw > L.d_out ? mw : L.d_out;
+        lw.push_back(x);
+    }
+    if (bf16) {
+        // TMA needs 16-byte row pitches: every width must be a multiple of 8.
+        if (cfg->d_in % 8) return BOM_ENOTSUP;
+        for (auto& x : lw)
+            if (x.d_out % 8 || x.d_in % 8) return BOM_ENOTSUP;
+    }
+    *d_model = w;
+    *max_width = mw;
+    *max_ffn = mf;
+    if (lw_out) *lw_out = lw;
+    return BOM_OK;
+}
+
+struct Carver {
+    size_t off = 0;
+    char* base = nullptr;
+    void* take(size_t bytes) {
+        off = (off + 255) & ~size_t(255);
+        void* p = base ? base + off : nullptr;
+        off += bytes;
+        return p;
+    }
+};
+
+// Lays out (base == nullptr: only measures) the workspace of a handle.
+size_t carve(bom_handle* h, char* base) {
+    Carver c;
+    c.base = base;
+    const int64_t n = h->cfg.max_rows, V = h->cfg.d_out, e = h->esz;
+    h->sc = static_cast<DevScalars*>(c.take(sizeof(DevScalars)));
+    for (auto& L : h->lw) {
+        if (L.kind == BOM_LAYER_SWIGLU) {
+            L.G = c.take(n * L.d_out * e);
+            L.U = c.take(n * L.d_out * e);
+            L.A = c.take(n * L.d_out * e);
+        } else if (L.kind == BOM_LAYER_LINEAR_GELU) {
+            L.pre = c.take(n * L.d_out * e);
+        }
+        L.out = c.take(n * L.width_out * e);
+    }
+    h->ldz = round_up(V, 8);
+    h->Z = c.take(n * h->ldz * e);
+    h->ntiles = h->bf16 ? tc_logit_tiles(V) : 1;
+    h->stats = static_cast<float*>(c.take(n * h->ntiles * 8));
+    h->lse = static_cast<float*>(c.take(n * 4));
+    h->ce = static_cast<float*>(c.take(n * 4));
+    h->colpart = static_cast<float*>(c.take(row_blocks(n) * V * 4));
+    h->s = static_cast<float*>(c.take(V * 4));
+    h->qhat = static_cast<float*>(c.take(V * 4));
+    h->cvec = static_cast<float*>(c.take(h->d_model * 4));
+    h->wvec = static_cast<float*>(c.take(h->d_model * 4));
+    const int64_t rb = row_blocks(n) > row_blocks(V) ? row_blocks(n) : row_blocks(V);
+    h->part = static_cast<float*>(c.take(rb * h->max_width * 4));
+    h->dx[0] = c.take(n * h->max_width * e);
+    h->dx[1] = c.take(n * h->max_width * e);
+    if (h->max_ffn > 0) {
+        h->dG = c.take(n * h->max_ffn * e);
+        h->dU = c.take(n * h->max_ffn * e);
+    }
+    return c.off + 256;
+}
+
+Operand kmaj(const void* p, int64_t ld) { return Operand{p, ld, false}; }
+Operand mnmaj(const void* p, int64_t ld) { return Operand{p, ld, true}; }
+
+// Runs `launch` between an event pair when the handle traces.
+template <class F>
+int traced(bom_handle* h, cudaStream_t s, const char* name, double flops, double bytes, F&& launch) {
+    if (!h->tracing) return launch();
+    if (h->trace_n == static_cast<int>(h->trace.size())) {
+        bom_handle::TraceRec r;
+        if (cudaEventCreate(&r.a) != cudaSuccess || cudaEventCreate(&r.b) != cudaSuccess) return BOM_ECUDA;
+        h->trace.push_back(r);
+    }
+    bom_handle::TraceRec& r = h->trace[h->trace_n++];
+    r.name = name;
+    r.flops = flops;
+    r.bytes = bytes;
+    cudaEventRecord(r.a, s);
+    const int rc = launch();
+    cudaEventRecord(r.b, s);
+    return rc;
+}
+
+const char* gemm_name(const GemmDesc& g, bool bf16) {
+    if (!bf16) return "gemm_simt";
+    switch (g.epi_kind) {
+        case EPI_LOGITS: return "gemm_tc.logits";
+        case EPI_SWIGLU_FWD: return "gemm_tc.swiglu_fwd";
+        case EPI_SWIGLU_BWD: return "gemm_tc.swiglu_bwd";
+        default: break;
+    }
+    const bool a = g.A[0].mn_major, b = g.B[0].mn_major;
+    return a ? (b ? "gemm_tc.linear.mm" : "gemm_tc.linear.mk") : (b ? "gemm_tc.linear.km" : "gemm_tc.linear.kk");
+}
+
+int run_gemm(bom_handle* h, GemmDesc& g, cudaStream_t s) {
+    g.epi.sc = h->sc;
+    g.epi.in_f32 = h->bf16 ? 0 : 1;
+    double k = 0;
+    for (int i = 0; i < g.nseg; ++i) k += static_cast<double>(g.K[i]);
+    const double n_mma = g.dual_b ? 2.0 * g.N : static_cast<double>(g.N);
+    const double flops = 2.0 * static_cast<double>(g.M) * n_mma * k;
+    const double bytes = h->esz * (static_cast<double>(g.M) * k + n_mma * k) +
+                         (g.epi.out_f32 ? 4.0 : h->esz) * static_cast<double>(g.M) * g.N;
+    return traced(h, s, gemm_name(g, h->bf16), flops, bytes,
+                  [&] { return h->bf16 ? launch_gemm_tc(g, s) : launch_gemm_simt(g, s); });
+}
+
+#define BOM_TRACED(name, flops, bytes, stmt) \
+    traced(h, s, name, (flops), (bytes), [&] { stmt; return static_cast<int>(BOM_OK); })
+
+GemmDesc gemm1(int64_t M, int64_t N, int64_t K, Operand A, Operand B) {
+    GemmDesc g;
+    g.M = M;
+    g.N = N;
+    g.K[0] = K;
+    g.A[0] = A;
+    g.B[0] = B;
+    g.nseg = 1;
+    g.epi.alpha_const = 1.0f;
+    g.epi.beta_const = 1.0f;
+    return g;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" {
+
+int32_t bom_param_count(const bom_config* cfg) {
+    if (!cfg || cfg->n_layers < 0 || (cfg->n_layers > 0 && !cfg->layers)) return -1;
+    int32_t k = 0;
+    for (int i = 0; i < cfg->n_layers; ++i)
+        k += cfg->layers[i].kind == BOM_LAYER_SWIGLU ? 3 : (cfg->layers[i].has_bias ? 2 : 1);
+    return k + (cfg->head_bias ? 2 : 1);
+}
+
+bom_status bom_param_shape(const bom_config* cfg, int32_t index, int64_t* rows, int64_t* cols) {
+    if (!cfg || !rows || !cols || index < 0) return BOM_EINVAL;
+    int32_t k = 0;
+    int64_t w = cfg->d_in;
+    for (int i = 0; i < cfg->n_layers; ++i) {
+        const bom_layer& L = cfg->layers[i];
+        if (L.kind == BOM_LAYER_SWIGLU) {
+            const int64_t r[3] = {L.d_out, L.d_out, L.d_in}, c[3] = {L.d_in, L.d_in, L.d_out};
+            for (int j = 0; j < 3; ++j, ++k)
+                if (k == index) { *rows = r[j]; *cols = c[j]; return BOM_OK; }
+        } else {
+            if (k++ == index) { *rows = L.d_out; *cols = L.d_in; return BOM_OK; }
+            if (L.has_bias && k++ == index) { *rows = L.d_out; *cols = 0; return BOM_OK; }
+            w = L.d_out;
+        }
+    }
+    if (k++ == index) { *rows = cfg->d_out; *cols = w; return BOM_OK; }
+    if (cfg->head_bias && k++ == index) { *rows = cfg->d_out; *cols = 0; return BOM_OK; }
+    return BOM_EINVAL;
+}
+
+int64_t bom_workspace_bytes(const bom_config* cfg) {
+    bom_handle h;
+    int64_t dm, mw, mf;
+    if (check_config(cfg, &h.lw, &dm, &mw, &mf) != BOM_OK) return -1;
+    h.cfg = *cfg;
+    h.bf16 = cfg->compute == BOM_BF16;
+    h.esz = h.bf16 ? 2 : 4;
+    h.d_model = dm;
+    h.max_width = mw;
+    h.max_ffn = mf;
+    return static_cast<int64_t>(carve(&h, nullptr));
+}
+
+bom_status bom_init(bom_handle** out, const bom_config* cfg) {
+    if (!out) return BOM_EINVAL;
+    *out = nullptr;
+    bom_handle* h = new (std::nothrow) bom_handle();
+    if (!h) return BOM_ENOMEM;
+    int64_t dm, mw, mf;
+    bom_status st = check_config(cfg, &h->lw, &dm, &mw, &mf);
+    if (st != BOM_OK) {
+        delete h;
+        return st;
+    }
+    h->cfg = *cfg;
+    h->layers.assign(cfg->layers, cfg->layers + cfg->n_layers);
+    h->cfg.layers = h->layers.data();
+    h->bf16 = cfg->compute == BOM_BF16;
+    h->esz = h->bf16 ? 2 : 4;
+    h->d_model = dm;
+    h->max_width = mw;
+    h->max_ffn = mf;
+    const size_t bytes = carve(h, nullptr);
+    void* p = nullptr;
+    if (cudaMalloc(&p, bytes) != cudaSuccess) {
+        cudaGetLastError();
+        delete h;
+        return BOM_ENOMEM;
+    }
+    h->ws = static_cast<char*>(p);
+    h->ws_bytes = bytes;
+    carve(h, h->ws + ((256 - (reinterpret_cast<uintptr_t>(h->ws) & 255)) & 255));
+    // Zero everything once: the padding columns of Z and the scalar block start defined.
+    if (cudaMemset(h->ws, 0, bytes) != cudaSuccess) {
+        cudaFree(p);
+        delete h;
+        return BOM_ECUDA;
+    }
+    *out = h;
+    return BOM_OK;
+}
+
+void bom_destroy(bom_handle* h) {
+    if (!h) return;
+    if (h->ws) cudaFree(h->ws);
+    for (auto& r : h->trace) {
+        cudaEventDestroy(r.a);
+        cudaEventDestroy(r.b);
+    }
+    delete h;
+}
+
+bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t n, void* const* params, float* q,
+                    int64_t t, void* const* grads, void* const* h_out, void* stream) {
+    if (!h || !x || !labels || !params || !q || !grads) return BOM_EINVAL;
+    if (n < 1 || n > h->cfg.max_rows || t < 1) return BOM_EINVAL;
+    const bool gh = h->cfg.out_mode == BOM_OUT_G_AND_H;
+    if (gh != (h_out != nullptr)) return BOM_EINVAL;
+    const int np = bom_param_count(&h->cfg);
+    for (int i = 0; i < np; ++i) {
+        if (!params[i] || !grads[i] || (gh && !h_out[i])) return BOM_EINVAL;
+        if (!aligned16(params[i]) || !aligned16(grads[i]) || (gh && !aligned16(h_out[i]))) return BOM_ENOTSUP;
+    }
+    if (!aligned16(x) || !aligned16(q)) return BOM_ENOTSUP;
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const bom_config& cfg = h->cfg;
+    const int64_t V = cfg.d_out, dm = h->d_model;
+    const int cf32 = h->bf16 ? 0 : 1;
+    h->last_n = n;
+    h->trace_n = 0;
+    int rc = BOM_OK;
+#define BOM_TRY(expr)                                     \
+    do {                                                  \
+        rc = (expr);                                      \
+        if (rc != BOM_OK) return static_cast<bom_status>(rc); \
+    } while (0)
+
+    if (cudaMemsetAsync(&h->sc->status, 0, sizeof(int32_t), s) != cudaSuccess) return BOM_ECUDA;
+    BOM_TRACED("labels_scan", 0, 4.0 * n, launch_labels_scan(labels, n, V, cfg.ignore_index, cfg.lambda, h->sc, s));
+
+    // ---------------------------------------------------------------- forward
+    const void* xin = x;
+    int pi = 0;
+    std::vector<int> pidx(h->lw.size());
+    for (size_t l = 0; l < h->lw.size(); ++l) {
+        LayerWs& L = h->lw[l];
+        pidx[l] = pi;
+        if (L.kind == BOM_LAYER_SWIGLU) {
+            const void* Wg = params[pi];
+            const void* Wu = params[pi + 1];
+            const void* Wd = params[pi + 2];
+            pi += 3;
+            const int64_t d = L.d_in, f = L.d_out;
+            GemmDesc g = gemm1(n, f, d, kmaj(xin, d), kmaj(Wg, d));
+            g.B[1] = kmaj(Wu, d);
+            g.dual_b = true;
+            g.epi_kind = EPI_SWIGLU_FWD;
+            g.epi.out = L.A;
+            g.epi.ld_out = f;
+            g.epi.out2 = L.G;
+            g.epi.ld_out2 = f;
+            g.epi.out3 = L.U;
+            g.epi.ld_out3 = f;
+            BOM_TRY(run_gemm(h, g, s));
+            GemmDesc g2 = gemm1(n, d, f, kmaj(L.A, f), kmaj(Wd, f));
+            g2.epi.resid = xin;
+            g2.epi.ld_resid = d;
+            g2.epi.out = L.out;
+            g2.epi.ld_out = d;
+            BOM_TRY(run_gemm(h, g2, s));
+        } else {
+            const void* W = params[pi++];
+            const void* b = L.bias ? params[pi++] : nullptr;
+            GemmDesc g = gemm1(n, L.d_out, L.d_in, kmaj(xin, L.d_in), kmaj(W, L.d_in));
+            g.epi.bias = b;
+            g.epi.out = L.out;
+            g.epi.ld_out = L.d_out;
+            g.epi.out_f32 = cf32;
+            if (L.kind == BOM_LAYER_LINEAR_GELU) {
+                g.epi.act = ACT_GELU;
+                g.epi.out2 = L.pre;
+                g.epi.ld_out2 = L.d_out;
+                g.epi.out2_f32 = cf32;
+            }
+            BOM_TRY(run_gemm(h, g, s));
+        }
+        xin = L.out;
+    }
+    const int head_w = pi;
+    const void* Wh = params[pi++];
+    const int head_b = cfg.head_bias ? pi++ : -1;
+    const void* bh = head_b >= 0 ? params[head_b] : nullptr;
+    {
+        GemmDesc g = gemm1(n, V, dm, kmaj(xin, dm), kmaj(Wh, dm));
+        g.epi_kind = EPI_LOGITS;
+        g.epi.bias = bh;
+        g.epi.out = h->Z;
+        g.epi.ld_out = h->ldz;
+        g.epi.out_f32 = cf32;
+        g.epi.stats = h->stats;
+        g.epi.ld_stats = h->ntiles;
+        BOM_TRY(run_gemm(h, g, s));
+    }
+    if (!h->bf16)
+        BOM_TRACED("row_stats_f32", 0, 4.0 * n * V,
+                   launch_row_stats_f32(static_cast<const float*>(h->Z), h->ldz, n, V, h->stats, h->sc, s));
+
+    // ---------------------------------------------------------------- task space
+    BOM_TRACED("row_lse", 0, 8.0 * n * h->ntiles + 12.0 * n,
+               launch_row_lse(h->Z, cf32, h->ldz, n, V, h->stats, h->ntiles, labels, cfg.ignore_index, h->lse,
+                              h->ce, h->sc, s));
+    // residual pass: reads and rewrites Z once, writes the column partial sums
+    BOM_TRACED("residual", 0, 2.0 * h->esz * n * h->ldz + 4.0 * row_blocks(n) * V + 8.0 * n,
+               launch_residual(h->Z, cf32, h->ldz, n, V, h->lse, labels, cfg.ignore_index, h->colpart, h->sc, s));
+    const float inv_bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(cfg.beta1), static_cast<double>(t))));
+    BOM_TRACED("finish_sq", 0, 4.0 * row_blocks(n) * V + 20.0 * V,
+               launch_finish_sq(h->colpart, row_blocks(n), V, cfg.beta1, inv_bc1, q, h->s, h->qhat, h->sc, s));
+    BOM_TRACED("scalars", 0, 4.0 * (n + V), launch_scalars(h->ce, n, h->s, V, h->sc, s));
+    // c = colsum_{I_t}(H) and w = W^T qhat (the rank-1 / broadcast factors of the reprojection)
+    BOM_TRACED("colsum", 2.0 * n * dm, h->esz * n * dm,
+               launch_colsum(xin, cf32, dm, n, dm, labels, cfg.ignore_index, nullptr, 1.0f, h->part, h->cvec, 1,
+                             h->sc, s));
+    BOM_TRACED("colsum", 2.0 * V * dm, h->esz * V * dm,
+               launch_colsum(Wh, cf32, dm, V, dm, nullptr, 0, h->qhat, 1.0f, h->part, h->wvec, 1, h->sc, s));
+
+    // ---------------------------------------------------------------- backward
+    const int passes[2] = {gh ? 1 : 0, 2};
+    const int npass = gh ? 2 : 1;
+    for (int pp = 0; pp < npass; ++pp) {
+        const int pass = passes[pp];
+        void* const* outp = pass == 2 ? h_out : grads;
+        const int of32 = pass == 2 ? 1 : cf32;
+        const float* cr = &h->sc->coef_r[pass];
+        const float* cq = &h->sc->coef_q[pass];
+        const int64_t kfull = pass == 2 ? 0 : 1;  // the h pass has no residual term
+        {   // head weight: a R^T H + b qhat (x) c
+            GemmDesc g = gemm1(V, dm, kfull * n, mnmaj(h->Z, h->ldz), mnmaj(xin, dm));
+            g.epi.alpha_const = 1.0f;
+            g.epi.alpha_dev = cr;
+            g.epi.beta_dev = cq;
+            g.epi.r1u = h->qhat;
+            g.epi.r1v = h->cvec;
+            g.epi.out = outp[head_w];
+            g.epi.ld_out = dm;
+            g.epi.out_f32 = of32;
+            BOM_TRY(run_gemm(h, g, s));
+        }
+        if (head_b >= 0) {
+            const float a = pass == 0 ? 1.0f - cfg.lambda : (pass == 1 ? 1.0f : 0.0f);
+            const float b = pass == 0 ? cfg.lambda : (pass == 1 ? 0.0f : 1.0f);
+            BOM_TRACED("axpby", 3.0 * V, 12.0 * V, launch_axpby(h->s, h->qhat, a, b, V, outp[head_b], of32, h->sc, s));
+        }
+        // the cotangent of X goes out with the u (or g) pass when requested
+        const bool want_dx = h->dx_in != nullptr && pass != 2;
+        if (h->lw.empty() && !want_dx) continue;
+        int cur = 0;
+        {   // head input: a R W + b 1_{I_t} w^T  (times GELU' of the last layer)
+            GemmDesc g = gemm1(n, dm, kfull * V, kmaj(h->Z, h->ldz), mnmaj(Wh, dm));
+            g.epi.alpha_dev = cr;
+            g.epi.beta_dev = cq;
+            g.epi.bw = h->wvec;
+            g.epi.mask_labels = labels;
+            g.epi.ignore_index = cfg.ignore_index;
+            if (!h->lw.empty() && h->lw.back().kind == BOM_LAYER_LINEAR_GELU) {
+                g.epi.act = ACT_DGELU;
+                g.epi.aux = h->lw.back().pre;
+                g.epi.ld_aux = h->lw.back().d_out;
+            }
+            g.epi.out = h->lw.empty() ? h->dx_in : h->dx[cur];
+            g.epi.ld_out = dm;
+            g.epi.out_f32 = cf32;
+            BOM_TRY(run_gemm(h, g, s));
+        }
+        for (int l = static_cast<int>(h->lw.size()) - 1; l >= 0; --l) {
+            const LayerWs& L = h->lw[l];
+            const void* xl = l == 0 ? x : h->lw[l - 1].out;
+            const void* dcur = h->dx[cur];
+            const int p0 = pidx[l];
+            const LayerWs* prev = l > 0 ? &h->lw[l - 1] : nullptr;
+            if (L.kind == BOM_LAYER_SWIGLU) {
+                const int64_t d = L.d_in, f = L.d_out;
+                const void* Wg = params[p0];
+                const void* Wu = params[p0 + 1];
+                const void* Wd = params[p0 + 2];
+                {   // dW_d = dy^T A
+                    GemmDesc g = gemm1(d, f, n, mnmaj(dcur, d), mnmaj(L.A, f));
+                    g.epi.out = outp[p0 + 2];
+                    g.epi.ld_out = f;
+                    g.epi.out_f32 = of32;
+                    BOM_TRY(run_gemm(h, g, s));
+                }
+                {   // dA = dy W_d, then dG = dA u SiLU'(g), dU = dA SiLU(g)
+                    GemmDesc g = gemm1(n, f, d, kmaj(dcur, d), mnmaj(Wd, f));
+                    g.epi_kind = EPI_SWIGLU_BWD;
+                    g.epi.aux = L.G;
+                    g.epi.ld_aux = f;
+                    g.epi.aux2 = L.U;
+                    g.epi.ld_aux2 = f;
+                    g.epi.out = h->dG;
+                    g.epi.ld_out = f;
+                    g.epi.out2 = h->dU;
+                    g.epi.ld_out2 = f;
+                    BOM_TRY(run_gemm(h, g, s));
+                }
+                {   // dW_g = dG^T x, dW_u = dU^T x
+                    GemmDesc g = gemm1(f, d, n, mnmaj(h->dG, f), mnmaj(xl, d));
+                    g.epi.out = outp[p0];
+                    g.epi.ld_out = d;
+                    g.epi.out_f32 = of32;
+                    BOM_TRY(run_gemm(h, g, s));
+                    GemmDesc g2 = gemm1(f, d, n, mnmaj(h->dU, f), mnmaj(xl, d));
+                    g2.epi.out = outp[p0 + 1];
+                    g2.epi.ld_out = d;
+                    g2.epi.out_f32 = of32;
+                    BOM_TRY(run_gemm(h, g2, s));
+                }
+                if (prev || want_dx) {   // dx = dy + dG W_g + dU W_u
+                    GemmDesc g = gemm1(n, d, f, kmaj(h->dG, f), mnmaj(Wg, d));
+                    g.nseg = 2;
+                    g.A[1] = kmaj(h->dU, f);
+                    g.B[1] = mnmaj(Wu, d);
+                    g.K[1] = f;
+                    g.epi.resid = dcur;
+                    g.epi.ld_resid = d;
+                    if (prev && prev->kind == BOM_LAYER_LINEAR_GELU) {
+                        g.epi.act = ACT_DGELU;
+                        g.epi.aux = prev->pre;
+                        g.epi.ld_aux = prev->d_out;
+                    }
+                    g.epi.out = prev ? h->dx[cur ^ 1] : h->dx_in;
+                    g.epi.ld_out = d;
+                    g.epi.out_f32 = cf32;
+                    BOM_TRY(run_gemm(h, g, s));
+                    cur ^= 1;
+                }
+            } else {
+                const void* W = params[p0];
+                {   // dW = dPre^T x
+                    GemmDesc g = gemm1(L.d_out, L.d_in, n, mnmaj(dcur, L.d_out), mnmaj(xl, L.d_in));
+                    g.epi.out = outp[p0];
+                    g.epi.ld_out = L.d_in;
+                    g.epi.out_f32 = of32;
+                    BOM_TRY(run_gemm(h, g, s));
+                }
+                if (L.bias)
+                    BOM_TRACED("colsum", 2.0 * n * L.d_out, h->esz * n * L.d_out,
+                               launch_colsum(dcur, cf32, L.d_out, n, L.d_out, nullptr, 0, nullptr, 1.0f, h->part,
+                                             outp[p0 + 1], of32, h->sc, s));
+                if (prev || want_dx) {   // dx = dPre W (times GELU' of the previous layer)
+                    GemmDesc g = gemm1(n, L.d_in, L.d_out, kmaj(dcur, L.d_out), mnmaj(W, L.d_in));
+                    if (prev && prev->kind == BOM_LAYER_LINEAR_GELU) {
+                        g.epi.act = ACT_DGELU;
+                        g.epi.aux = prev->pre;
+                        g.epi.ld_aux = prev->d_out;
+                    }
+                    g.epi.out = prev ? h->dx[cur ^ 1] : h->dx_in;
+                    g.epi.ld_out = L.d_in;
+                    g.epi.out_f32 = cf32;
+                    BOM_TRY(run_gemm(h, g, s));
+                    cur ^= 1;
+                }
+            }
+        }
+    }
+#undef BOM_TRY
+    return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+bom_status bom_set_input_grad(bom_handle* h, void* dx) {
+    if (!h) return BOM_EINVAL;
+    if (dx && !aligned16(dx)) return BOM_ENOTSUP;
+    h->dx_in = dx;
+    return BOM_OK;
+}
+
+bom_status bom_step_outputs(bom_handle* h, const float** qhat, const float** s, const float** lse) {
+    if (!h) return BOM_EINVAL;
+    if (qhat) *qhat = h->qhat;
+    if (s) *s = h->s;
+    if (lse) *lse = h->lse;
+    return BOM_OK;
+}
+
+bom_status bom_get_stats(bom_handle* h, bom_stats* out, void* stream) {
+    if (!h || !out) return BOM_EINVAL;
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return BOM_ECUDA;
+    DevScalars sc;
+    if (cudaMemcpy(&sc, h->sc, sizeof(sc), cudaMemcpyDeviceToHost) != cudaSuccess) return BOM_ECUDA;
+    out->loss = sc.loss;
+    out->n_t = sc.n_t;
+    out->status = sc.status;
+    out->s_norm = sc.s_norm;
+    return static_cast<bom_status>(sc.status);
+}
+
+bom_status bom_update(float* theta, const void* g, int32_t g_dtype, const float* hvec, float* v, uint16_t* theta_bf16,
+                      int64_t n, float lr, float wd, float lambda, float beta2, float eps, int64_t t, void* stream) {
+    if (n < 0 || t < 1) return BOM_EINVAL;
+    if (n == 0) return BOM_OK;
+    if (!theta || !g || !v) return BOM_EINVAL;
+    if (g_dtype != BOM_F32 && g_dtype != BOM_BF16) return BOM_EINVAL;
+    if (!(beta2 >= 0.0f && beta2 < 1.0f) || !(eps >= 0.0f)) return BOM_EINVAL;
+    if (!aligned16(theta) || !aligned16(g) || !aligned16(v) || (hvec && !aligned16(hvec)) ||
+        (theta_bf16 && !aligned16(theta_bf16)))
+        return BOM_ENOTSUP;
+    const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
+    return static_cast<bom_status>(launch_update(theta, g, g_dtype == BOM_BF16, hvec, v, theta_bf16, n, lr, wd,
+                                                 lambda, beta2, eps, inv_bc2, static_cast<cudaStream_t>(stream)));
+}
+
+bom_status bom_gemm_bf16(const uint16_t* A, int64_t lda, int32_t a_mn_major, const uint16_t* B, int64_t ldb,
+                         int32_t b_mn_major, float* D, int64_t ldd, int64_t M, int64_t N, int64_t K, float alpha,
+                         void* stream) {
+    if (!A || !B || !D || M < 1 || N < 1 || K < 0) return BOM_EINVAL;
+    if ((ldd % 4) != 0 || !aligned16(D) || ldd < N) return BOM_ENOTSUP;
+    GemmDesc g = gemm1(M, N, K, Operand{A, lda, a_mn_major != 0}, Operand{B, ldb, b_mn_major != 0});
+    g.epi.alpha_const = alpha;
+    g.epi.out = D;
+    g.epi.ld_out = ldd;
+    g.epi.out_f32 = 1;
+    g.epi.sc = nullptr;
+    return static_cast<bom_status>(launch_gemm_tc(g, static_cast<cudaStream_t>(stream)));
+}
+
+bom_status bom_trace(bom_handle* h, int32_t enable) {
+    if (!h) return BOM_EINVAL;
+    h->tracing = enable != 0;
+    h->trace_n = 0;
+    return BOM_OK;
+}
+
+int32_t bom_trace_read(bom_handle* h, bom_trace_entry* out, int32_t max, void* stream) {
+    if (!h || (max > 0 && !out)) return -1;
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return -1;
+    for (int i = 0; i < h->trace_n && i < max; ++i) {
+        const auto& r = h->trace[i];
+        float ms = 0.0f;
+        if (cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess) return -1;
+        out[i].name = r.name;
+        out[i].flops = r.flops;
+        out[i].bytes = r.bytes;
+        out[i].ms = ms;
+    }
+    return h->trace_n;
+}
+
+int64_t bom_launch_count(void) { return static_cast<int64_t>(bom::g_launches.load()); }
+
+const char* bom_status_string(bom_status s) {
+    switch (s) {
+        case BOM_OK: return "BOM_OK";
+        case BOM_EINVAL: return "BOM_EINVAL: invalid argument";
+        case BOM_ENOMEM: return "BOM_ENOMEM: device workspace allocation failed";
+        case BOM_ECUDA: return "BOM_ECUDA: CUDA call failed";
+        case BOM_ELABEL: return "BOM_ELABEL: label outside [0, d_out) that is not ignore_index";
+        case BOM_EEMPTY: return "BOM_EEMPTY: no supervised outputs (N_t = 0)";
+        case BOM_ETIMEOUT: return "BOM_ETIMEOUT: a bounded device wait ran out";
+        case BOM_ENOTSUP: return "BOM_ENOTSUP: shape or alignment not supported";
+    }
+    return "unknown bom_status";
+}
+
+}  // extern "C"

@@ -1,0 +1,252 @@
+// Shared device-side definitions of the BOM CUDA path: the device scalar
+// block of a step, the GEMM epilogue parameter block, element load/store
+// helpers and the activation functions of the backbone.
+#pragma once
+#include <cstdint>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "bom.h"
+
+namespace bom {
+
+// Host-side count of kernel launches made by the library (bom_launch_count).
+void count_launch();
+
+// Per-step scalars that live on the device so that no host round trip is
+// needed between the label scan and the kernels that scale by 1/N_t.
+struct DevScalars {
+    int32_t status;        // latched bom_status (first error wins), 0 = OK
+    int32_t n_t;           // |I_t|
+    float inv_nt;          // 1 / N_t
+    float coef_r[3];       // coefficient of r_i in the logit cotangent: [U pass, G pass, H pass]
+    float coef_q[3];       // coefficient of qhat in the logit cotangent
+    float loss;            // mean CE over I_t
+    float s_norm;          // ||s_t||
+};
+
+__device__ __forceinline__ void latch_status(DevScalars* sc, int code) {
+    atomicCAS(&sc->status, 0, code);
+}
+
+enum EpiKind : int { EPI_LINEAR = 0, EPI_LOGITS = 1, EPI_SWIGLU_FWD = 2, EPI_SWIGLU_BWD = 3 };
+enum ActKind : int { ACT_NONE = 0, ACT_GELU = 1, ACT_DGELU = 2 };
+
+// What a GEMM does with its fp32 accumulator acc[m][n] (m: output row, n: column):
+//   EPI_LINEAR     v = alpha*acc + bias[n] + beta*r1u[m]*r1v[n] + beta*mask(m)*bw[n] + resid[m][n]
+//                  then ACT_GELU (out2 <- v, out <- GELU(v)), ACT_DGELU (out <- v*GELU'(aux[m][n]))
+//                  or ACT_NONE (out <- v).
+//   EPI_LOGITS     out <- z = acc + bias[n] rounded to the compute dtype; per (row, column tile)
+//                  the pair (max_n z, sum_n exp(z - max)) goes to stats.
+//   EPI_SWIGLU_FWD the accumulator tile holds [g | u] halves: out2 <- g, out3 <- u, out <- SiLU(g)*u.
+//   EPI_SWIGLU_BWD acc = dA: out <- dA*u*SiLU'(g) (= dG), out2 <- dA*SiLU(g) (= dU), g = aux, u = aux2.
+struct EpiParams {
+    float alpha_const;
+    const float* alpha_dev;      // optional device factor of alpha
+    float beta_const;
+    const float* beta_dev;       // optional device factor of beta
+    const void* bias;            // [N] compute dtype, or null
+    const float* r1u;            // [M] rank-1 row factor, or null
+    const float* r1v;            // [N] rank-1 column factor
+    const float* bw;             // [N] broadcast-row vector, or null
+    const int32_t* mask_labels;  // labels: mask(m) = labels[m] != ignore_index (null: mask = 1)
+    int32_t ignore_index;
+    const void* resid;           // [M, ld_resid] compute dtype, or null
+    int64_t ld_resid;
+    int32_t act;                 // ActKind
+    int32_t in_f32;              // compute dtype of bias / resid / aux: 1 = fp32, 0 = bf16
+    const void* aux;             // DGELU: pre-activation; SWIGLU_BWD: g
+    int64_t ld_aux;
+    const void* aux2;            // SWIGLU_BWD: u
+    int64_t ld_aux2;
+    void* out;
+    int64_t ld_out;
+    int32_t out_f32;             // dtype of out: 1 = fp32, 0 = bf16
+    int32_t out2_f32;            // dtype of out2 / out3
+    void* out2;
+    int64_t ld_out2;
+    void* out3;
+    int64_t ld_out3;
+    float* stats;                // EPI_LOGITS: [M, ld_stats] float2 pairs
+    int64_t ld_stats;            // pairs per row (number of column tiles)
+    const DevScalars* sc;        // kernels return early when sc->status != 0
+};
+
+// ------------------------------------------------------------ activations
+__device__ __forceinline__ float gelu_f(float x) {
+    return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
+}
+__device__ __forceinline__ float gelu_grad_f(float x) {
+    const float Phi = 0.5f * (1.0f + erff(x * 0.70710678118654752f));
+    const float phi = 0.39894228040143268f * expf(-0.5f * x * x);
+    return Phi + x * phi;
+}
+__device__ __forceinline__ float sigmoid_f(float x) { return 1.0f / (1.0f + expf(-x)); }
+__device__ __forceinline__ float silu_f(float x) { return x * sigmoid_f(x); }
+__device__ __forceinline__ float silu_grad_f(float x) {
+    const float sg = sigmoid_f(x);
+    return sg * (1.0f + x * (1.0f - sg));
+}
+
+// ------------------------------------------------------------ element access
+__device__ __forceinline__ float ld_elem(const void* base, int64_t idx, int is_f32) {
+    if (is_f32) return static_cast<const float*>(base)[idx];
+    return __bfloat162float(static_cast<const __nv_bfloat16*>(base)[idx]);
+}
+__device__ __forceinline__ void st_elem(void* base, int64_t idx, int is_f32, float v) {
+    if (is_f32)
+        static_cast<float*>(base)[idx] = v;
+    else
+        static_cast<__nv_bfloat16*>(base)[idx] = __float2bfloat16_rn(v);
+}
+__device__ __forceinline__ float round_bf16(float v) { return __bfloat162float(__float2bfloat16_rn(v)); }
+
+// 32 consecutive elements of one row, [n, n+32) clipped to n < N.
+__device__ __forceinline__ void load_row32(const void* base, int64_t row_off, int n, int N, int is_f32,
+                                           float (&v)[32]) {
+    if (n + 32 <= N) {
+        if (is_f32) {
+            const float4* p = reinterpret_cast<const float4*>(static_cast<const float*>(base) + row_off + n);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                float4 f = p[i];
+                v[4 * i] = f.x; v[4 * i + 1] = f.y; v[4 * i + 2] = f.z; v[4 * i + 3] = f.w;
+            }
+        } else {
+            const uint4* p = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(base) + row_off + n);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                uint4 w = p[i];
+                const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    v[8 * i + 2 * j] = __uint_as_float(ws[j] << 16);
+                    v[8 * i + 2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
+                }
+            }
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = (n + i < N) ? ld_elem(base, row_off + n + i, is_f32) : 0.0f;
+    }
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__device__ __forceinline__ void store_row32(void* base, int64_t row_off, int n, int N, int is_f32,
+                                            const float (&v)[32]) {
+    if (n + 32 <= N) {
+        if (is_f32) {
+            float4* p = reinterpret_cast<float4*>(static_cast<float*>(base) + row_off + n);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) p[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        } else {
+            uint4* p = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(base) + row_off + n);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                p[i] = make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                                  pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+            if (n + i < N) st_elem(base, row_off + n + i, is_f32, v[i]);
+    }
+}
+
+__device__ __forceinline__ void load_vec32(const float* p, int n, int N, float (&v)[32]) {
+    if (n + 32 <= N) {
+        const float4* q = reinterpret_cast<const float4*>(p + n);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            float4 f = __ldg(q + i);
+            v[4 * i] = f.x; v[4 * i + 1] = f.y; v[4 * i + 2] = f.z; v[4 * i + 3] = f.w;
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = (n + i < N) ? p[n + i] : 0.0f;
+    }
+}
+
+// Row-constant part of the EPI_LINEAR epilogue.
+struct EpiRow {
+    float alpha, beta_r1, beta_bw;
+    bool valid;
+};
+
+__device__ __forceinline__ EpiRow epi_row(const EpiParams& e, int m, int M) {
+    EpiRow r;
+    const float a = e.alpha_const * (e.alpha_dev ? *e.alpha_dev : 1.0f);
+    const float b = e.beta_const * (e.beta_dev ? *e.beta_dev : 1.0f);
+    r.valid = m < M;
+    r.alpha = a;
+    r.beta_r1 = (e.r1u && r.valid) ? b * e.r1u[m] : 0.0f;
+    float mask = 1.0f;
+    if (e.mask_labels && r.valid) mask = (e.mask_labels[m] != e.ignore_index) ? 1.0f : 0.0f;
+    r.beta_bw = e.bw ? b * mask : 0.0f;
+    return r;
+}
+
+// Applies EPI_LINEAR to 32 accumulator values of row m, columns [n, n+32).
+__device__ __forceinline__ void epi_linear32(const EpiParams& e, const EpiRow& r, int m, int n, int N,
+                                             float (&v)[32]) {
+    float t[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] *= r.alpha;
+    if (e.bias) {
+        load_row32(e.bias, 0, n, N, e.in_f32, t);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] += t[i];
+    }
+    if (e.r1u) {
+        load_vec32(e.r1v, n, N, t);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] += r.beta_r1 * t[i];
+    }
+    if (e.bw) {
+        load_vec32(e.bw, n, N, t);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] += r.beta_bw * t[i];
+    }
+    if (e.resid) {
+        load_row32(e.resid, static_cast<int64_t>(m) * e.ld_resid, n, N, e.in_f32, t);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] += t[i];
+    }
+    if (e.act == ACT_GELU) {
+        store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, N, e.out2_f32, v);
+        if (!e.out2_f32) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = round_bf16(v[i]);
+        }
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = gelu_f(v[i]);
+    } else if (e.act == ACT_DGELU) {
+        load_row32(e.aux, static_cast<int64_t>(m) * e.ld_aux, n, N, e.in_f32, t);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(t[i]);
+    }
+    store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, N, e.out_f32, v);
+}
+
+// Scalar form of EPI_LINEAR (SIMT GEMM).
+__device__ __forceinline__ float epi_linear1(const EpiParams& e, const EpiRow& r, int m, int n, float acc) {
+    float v = r.alpha * acc;
+    if (e.bias) v += ld_elem(e.bias, n, e.in_f32);
+    if (e.r1u) v += r.beta_r1 * e.r1v[n];
+    if (e.bw) v += r.beta_bw * e.bw[n];
+    if (e.resid) v += ld_elem(e.resid, static_cast<int64_t>(m) * e.ld_resid + n, e.in_f32);
+    if (e.act == ACT_GELU) {
+        st_elem(e.out2, static_cast<int64_t>(m) * e.ld_out2 + n, e.out2_f32, v);
+        if (!e.out2_f32) v = round_bf16(v);
+        v = gelu_f(v);
+    } else if (e.act == ACT_DGELU) {
+        v *= gelu_grad_f(ld_elem(e.aux, static_cast<int64_t>(m) * e.ld_aux + n, e.in_f32));
+    }
+    return v;
+}
+
+}  // namespace bom

@@ -1,0 +1,107 @@
+// SIMT fp32 GEMM (no TF32) for the fp32 configuration, where the parity bar is
+// a relative L2 error of 1e-5 that TF32 tensor cores cannot meet.  64 x 64
+// output tile per 256-thread block, 4 x 4 outputs per thread, K in steps of 16
+// through shared memory; operands in either K-major or MN-major layout.
+#include "gemm.h"
+
+namespace bom {
+namespace simt {
+
+constexpr int TM = 64, TN = 64, TK = 16;
+
+struct Params {
+    const float* A[2];
+    const float* B[2];
+    int64_t a_sm[2], a_sk[2];  // element (m, k) of A at A[m*a_sm + k*a_sk]
+    int64_t b_sn[2], b_sk[2];
+    int64_t K[2];
+    int nseg;
+    int M, N;
+    int epi_kind;
+    EpiParams epi;
+};
+
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const Params p) {
+    if (p.epi.sc != nullptr && p.epi.sc->status != 0) return;
+    __shared__ float As[TK][TM + 1];
+    __shared__ float Bs[TK][TN + 1];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const int m0 = blockIdx.y * TM, n0 = blockIdx.x * TN;
+    float acc[4][4] = {};
+    for (int s = 0; s < p.nseg; ++s) {
+        const float* A = p.A[s];
+        const float* B = p.B[s];
+        for (int64_t k0 = 0; k0 < p.K[s]; k0 += TK) {
+            for (int i = threadIdx.x; i < TK * TM; i += 256) {
+                const int kk = i / TM, mm = i % TM;
+                const int m = m0 + mm;
+                const int64_t k = k0 + kk;
+                As[kk][mm] = (m < p.M && k < p.K[s]) ? A[m * p.a_sm[s] + k * p.a_sk[s]] : 0.0f;
+                const int n = n0 + mm;
+                Bs[kk][mm] = (n < p.N && k < p.K[s]) ? B[n * p.b_sn[s] + k * p.b_sk[s]] : 0.0f;
+            }
+            __syncthreads();
+#pragma unroll
+            for (int kk = 0; kk < TK; ++kk) {
+                float a[4], b[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) a[i] = As[kk][ty + 16 * i];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx + 16 * j];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+            }
+            __syncthreads();
+        }
+    }
+    const EpiParams& e = p.epi;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int m = m0 + ty + 16 * i;
+        if (m >= p.M) continue;
+        const EpiRow r = epi_row(e, m, p.M);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int n = n0 + tx + 16 * j;
+            if (n >= p.N) continue;
+            float v;
+            if (p.epi_kind == EPI_LOGITS) {
+                v = acc[i][j] + (e.bias ? ld_elem(e.bias, n, e.in_f32) : 0.0f);
+            } else {
+                v = epi_linear1(e, r, m, n, acc[i][j]);
+            }
+            st_elem(e.out, static_cast<int64_t>(m) * e.ld_out + n, e.out_f32, v);
+        }
+    }
+}
+
+}  // namespace simt
+
+int launch_gemm_simt(const GemmDesc& g, cudaStream_t stream) {
+    if (g.M <= 0 || g.N <= 0) return BOM_OK;
+    if (g.dual_b || (g.epi_kind != EPI_LINEAR && g.epi_kind != EPI_LOGITS)) return BOM_ENOTSUP;
+    if (g.M > INT32_MAX / 2 || g.N > INT32_MAX / 2) return BOM_ENOTSUP;
+    simt::Params p{};
+    p.nseg = g.nseg;
+    for (int s = 0; s < g.nseg; ++s) {
+        p.A[s] = static_cast<const float*>(g.A[s].ptr);
+        p.B[s] = static_cast<const float*>(g.B[s].ptr);
+        p.a_sm[s] = g.A[s].mn_major ? 1 : g.A[s].ld;
+        p.a_sk[s] = g.A[s].mn_major ? g.A[s].ld : 1;
+        p.b_sn[s] = g.B[s].mn_major ? 1 : g.B[s].ld;
+        p.b_sk[s] = g.B[s].mn_major ? g.B[s].ld : 1;
+        p.K[s] = g.K[s];
+    }
+    p.M = static_cast<int>(g.M);
+    p.N = static_cast<int>(g.N);
+    p.epi_kind = g.epi_kind;
+    p.epi = g.epi;
+    dim3 grid(static_cast<unsigned>((g.N + simt::TN - 1) / simt::TN), static_cast<unsigned>((g.M + simt::TM - 1) / simt::TM));
+    if (grid.y > 65535) return BOM_ENOTSUP;
+    simt::gemm_simt_kernel<<<grid, 256, 0, stream>>>(p); count_launch();
+    return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+}  // namespace bom

@@ -1,0 +1,60 @@
+// Launchers of the non-GEMM kernels of the BOM step and of the update.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+namespace bom {
+
+// Row-block height of the residual pass and of the column reductions.  The
+// column partial sums of one block are summed in a fixed order afterwards, so
+// every reduction of the step is deterministic (no float atomics).
+constexpr int kRowBlock = 128;
+
+inline int64_t row_blocks(int64_t n) { return (n + kRowBlock - 1) / kRowBlock; }
+
+// Counts N_t, checks every label, latches BOM_ELABEL / BOM_EEMPTY and writes
+// the cotangent coefficients of the three passes into sc.
+void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda,
+                        DevScalars* sc, cudaStream_t s);
+
+// fp32 path: per-row (max, sum exp) of Z [n, ldz] over V columns (one tile).
+void launch_row_stats_f32(const float* Z, int64_t ldz, int64_t n, int64_t V, float* stats, const DevScalars* sc,
+                          cudaStream_t s);
+
+// Merges per-tile (max, sum exp) pairs into lse[i]; ce[i] = lse_i - z_{i,y_i}
+// for supervised rows, 0 otherwise.
+void launch_row_lse(const void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* stats, int64_t ntiles,
+                    const int32_t* labels, int32_t ignore, float* lse, float* ce, const DevScalars* sc,
+                    cudaStream_t s);
+
+// Z -> R in place: r_ij = exp(z_ij - lse_i) - [j = y_i] on supervised rows, 0 on
+// the others and in the padding columns [V, ldz); colpart[b, j] receives the
+// fp32 column sums of r over row block b.
+void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* lse, const int32_t* labels,
+                     int32_t ignore, float* colpart, const DevScalars* sc, cudaStream_t s);
+
+// s_j = N_t^-1 sum_b colpart[b, j]; q_j <- beta1 q_j + (1-beta1) s_j;
+// qhat_j = q_j * inv_bc1.  q is only written when the status word is clear.
+void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float inv_bc1, float* q,
+                      float* s_out, float* qhat, DevScalars* sc, cudaStream_t s);
+
+// loss = N_t^-1 sum_i ce_i and ||s||.
+void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, DevScalars* sc, cudaStream_t s);
+
+// out[j] = scale * sum_i w_i X[i, j]  (w_i = 1, the row mask from labels, or wvec[i]).
+// `part` must hold row_blocks(n) * d floats.
+void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, const int32_t* labels,
+                   int32_t ignore, const float* wvec, float scale, float* part, void* out, int out_f32,
+                   const DevScalars* sc, cudaStream_t s);
+
+// out[j] = a * s[j] + b * qhat[j] (head bias numerator).
+void launch_axpby(const float* s_vec, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
+                  const DevScalars* sc, cudaStream_t s);
+
+// BOM-AdamW update (see bom_update in bom.h).
+int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,
+                  float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, cudaStream_t s);
+
+}  // namespace bom

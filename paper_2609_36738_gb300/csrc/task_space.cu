@@ -1,0 +1,344 @@
+// Task-space part of the BOM step (Algorithm 1, residual / EMA steps):
+// label scan and N_t, row log-sum-exp from the logits epilogue's per-tile
+// statistics, the residual pass r = softmax(z) - onehot(y) with deterministic
+// column partial sums, s_t and the q_t EMA with bias correction, and the
+// column reductions colsum_{I_t}(H), W^T qhat and bias gradients.
+#include "kernels.h"
+
+namespace bom {
+
+namespace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ int warp_sum_i(int v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Deterministic block sum of a float (fixed tree for a fixed block size).
+template <int NT>
+__device__ float block_sum(float v, float* red) {
+    v = warp_sum(v);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    if (l == 0) red[w] = v;
+    __syncthreads();
+    float r = 0.0f;
+    if (w == 0) {
+        r = (l < NT / 32) ? red[l] : 0.0f;
+        r = warp_sum(r);
+    }
+    __syncthreads();
+    return r;  // valid in thread 0
+}
+
+__global__ void labels_scan_kernel(const int32_t* __restrict__ labels, int64_t n, int64_t V, int32_t ignore,
+                                   float lambda, DevScalars* sc) {
+    __shared__ int s_cnt[32], s_bad[32];
+    int cnt = 0, bad = 0;
+    for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+        const int32_t y = labels[i];
+        if (y == ignore) continue;
+        if (y < 0 || y >= V)
+            ++bad;
+        else
+            ++cnt;
+    }
+    cnt = warp_sum_i(cnt);
+    bad = warp_sum_i(bad);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    if (l == 0) {
+        s_cnt[w] = cnt;
+        s_bad[w] = bad;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int c = 0, b = 0;
+        for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
+            c += s_cnt[k];
+            b += s_bad[k];
+        }
+        sc->n_t = c;
+        if (b > 0)
+            latch_status(sc, BOM_ELABEL);
+        else if (c == 0)
+            latch_status(sc, BOM_EEMPTY);
+        const float inv = c > 0 ? 1.0f / static_cast<float>(c) : 0.0f;
+        sc->inv_nt = inv;
+        sc->coef_r[0] = (1.0f - lambda) * inv;  // u pass: N_t^-1 (1-lambda) r_i
+        sc->coef_q[0] = lambda * inv;           //         N_t^-1 lambda qhat
+        sc->coef_r[1] = inv;                    // g pass: N_t^-1 r_i
+        sc->coef_q[1] = 0.0f;
+        sc->coef_r[2] = 0.0f;                   // h pass: N_t^-1 qhat
+        sc->coef_q[2] = inv;
+        sc->loss = 0.0f;
+        sc->s_norm = 0.0f;
+    }
+}
+
+// One warp per row.
+__global__ void row_stats_f32_kernel(const float* __restrict__ Z, int64_t ldz, int64_t n, int64_t V,
+                                     float2* __restrict__ stats, const DevScalars* sc) {
+    if (sc->status != 0) return;
+    const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int l = threadIdx.x & 31;
+    if (row >= n) return;
+    const float* z = Z + row * ldz;
+    float m = -INFINITY;
+    for (int64_t j = l; j < V; j += 32) m = fmaxf(m, z[j]);
+    m = warp_max(m);
+    float s = 0.0f;
+    for (int64_t j = l; j < V; j += 32) s += expf(z[j] - m);
+    s = warp_sum(s);
+    if (l == 0) stats[row] = make_float2(m, s);
+}
+
+__global__ void row_lse_kernel(const void* __restrict__ Z, int z_f32, int64_t ldz, int64_t n, int64_t V,
+                               const float2* __restrict__ stats, int64_t ntiles, const int32_t* __restrict__ labels,
+                               int32_t ignore, float* __restrict__ lse, float* __restrict__ ce, const DevScalars* sc) {
+    if (sc->status != 0) return;
+    const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int l = threadIdx.x & 31;
+    if (row >= n) return;
+    const float2* st = stats + row * ntiles;
+    float m = -INFINITY;
+    for (int64_t t = l; t < ntiles; t += 32) m = fmaxf(m, st[t].x);
+    m = warp_max(m);
+    float s = 0.0f;
+    for (int64_t t = l; t < ntiles; t += 32) {
+        const float2 p = st[t];
+        if (p.x != -INFINITY) s += p.y * expf(p.x - m);
+    }
+    s = warp_sum(s);
+    if (l == 0) {
+        const float L = m + logf(s);
+        lse[row] = L;
+        const int32_t y = labels[row];
+        float c = 0.0f;
+        if (y != ignore && y >= 0 && y < V) c = L - ld_elem(Z, row * ldz + y, z_f32);
+        ce[row] = c;
+    }
+}
+
+// Block: 256 threads x VEC consecutive columns; grid.y: row blocks.
+template <typename T, int VEC>
+__global__ void __launch_bounds__(256) residual_kernel(T* __restrict__ Z, int64_t ldz, int64_t n, int64_t V,
+                                                       const float* __restrict__ lse,
+                                                       const int32_t* __restrict__ labels, int32_t ignore,
+                                                       float* __restrict__ colpart, const DevScalars* sc) {
+    if (sc->status != 0) return;
+    const int64_t col0 = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) * VEC;
+    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kRowBlock;
+    const int64_t r1 = min(r0 + kRowBlock, n);
+    float csum[VEC];
+#pragma unroll
+    for (int k = 0; k < VEC; ++k) csum[k] = 0.0f;
+    if (col0 < ldz) {
+        constexpr int UNROLL = 4;
+        for (int64_t rb = r0; rb < r1; rb += UNROLL) {
+            float zv[UNROLL][VEC];
+#pragma unroll
+            for (int u = 0; u < UNROLL; ++u) {
+                const int64_t r = rb + u;
+                if (r < r1) {
+                    const T* src = Z + r * ldz + col0;
+                    if constexpr (sizeof(T) == 2) {
+                        const uint4 w = *reinterpret_cast<const uint4*>(src);
+                        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            zv[u][2 * j] = __uint_as_float(ws[j] << 16);
+                            zv[u][2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
+                        }
+                    } else {
+                        const float4 f = *reinterpret_cast<const float4*>(src);
+                        zv[u][0] = f.x; zv[u][1] = f.y; zv[u][2] = f.z; zv[u][3] = f.w;
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < UNROLL; ++u) {
+                const int64_t r = rb + u;
+                if (r >= r1) break;
+                const int32_t y = labels[r];
+                const bool valid = (y != ignore);
+                const float L = lse[r];
+                float rv[VEC];
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) {
+                    const int64_t c = col0 + k;
+                    float p = (valid && c < V) ? expf(zv[u][k] - L) : 0.0f;
+                    if (valid && c == y) p -= 1.0f;
+                    rv[k] = p;
+                    csum[k] += p;
+                }
+                T* dst = Z + r * ldz + col0;
+                if constexpr (sizeof(T) == 2) {
+                    *reinterpret_cast<uint4*>(dst) = make_uint4(pack_bf16x2(rv[0], rv[1]), pack_bf16x2(rv[2], rv[3]),
+                                                                pack_bf16x2(rv[4], rv[5]), pack_bf16x2(rv[6], rv[7]));
+                } else {
+                    *reinterpret_cast<float4*>(dst) = make_float4(rv[0], rv[1], rv[2], rv[3]);
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < VEC; ++k)
+            if (col0 + k < V) colpart[static_cast<int64_t>(blockIdx.y) * V + col0 + k] = csum[k];
+    }
+}
+
+__global__ void finish_sq_kernel(const float* __restrict__ colpart, int64_t nblocks, int64_t V, float beta1,
+                                 float inv_bc1, float* __restrict__ q, float* __restrict__ s_out,
+                                 float* __restrict__ qhat, const DevScalars* sc) {
+    if (sc->status != 0) return;
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (j >= V) return;
+    float acc = 0.0f;
+    for (int64_t b = 0; b < nblocks; ++b) acc += colpart[b * V + j];
+    const float s = acc * sc->inv_nt;
+    const float qn = beta1 * q[j] + (1.0f - beta1) * s;
+    q[j] = qn;
+    s_out[j] = s;
+    qhat[j] = qn * inv_bc1;
+}
+
+__global__ void __launch_bounds__(1024) scalars_kernel(const float* __restrict__ ce, int64_t n,
+                                                       const float* __restrict__ s_vec, int64_t V, DevScalars* sc) {
+    __shared__ float red[32];
+    if (sc->status != 0) return;
+    float a = 0.0f;
+    for (int64_t i = threadIdx.x; i < n; i += 1024) a += ce[i];
+    a = block_sum<1024>(a, red);
+    float b = 0.0f;
+    for (int64_t j = threadIdx.x; j < V; j += 1024) b += s_vec[j] * s_vec[j];
+    b = block_sum<1024>(b, red);
+    if (threadIdx.x == 0) {
+        sc->loss = a * sc->inv_nt;
+        sc->s_norm = sqrtf(b);
+    }
+}
+
+// part[b, j] = sum_{i in row block b} w_i X[i, j]; 256 threads x 4 columns.
+__global__ void __launch_bounds__(256) colsum_part_kernel(const void* __restrict__ X, int x_f32, int64_t ldx,
+                                                          int64_t n, int64_t d, const int32_t* __restrict__ labels,
+                                                          int32_t ignore, const float* __restrict__ wvec,
+                                                          float* __restrict__ part, const DevScalars* sc) {
+    if (sc->status != 0) return;
+    const int64_t c0 = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) * 4;
+    if (c0 >= d) return;
+    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kRowBlock;
+    const int64_t r1 = min(r0 + kRowBlock, n);
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    const bool vec = (c0 + 4 <= d) && ((ldx & 3) == 0);
+    for (int64_t r = r0; r < r1; ++r) {
+        float w = 1.0f;
+        if (labels) w = (labels[r] != ignore) ? 1.0f : 0.0f;
+        if (wvec) w = wvec[r];
+        if (w == 0.0f) continue;
+        float x[4];
+        if (vec) {
+            if (x_f32) {
+                const float4 f = *reinterpret_cast<const float4*>(static_cast<const float*>(X) + r * ldx + c0);
+                x[0] = f.x; x[1] = f.y; x[2] = f.z; x[3] = f.w;
+            } else {
+                const uint2 u = *reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(X) + r * ldx + c0);
+                x[0] = __uint_as_float(u.x << 16); x[1] = __uint_as_float(u.x & 0xFFFF0000u);
+                x[2] = __uint_as_float(u.y << 16); x[3] = __uint_as_float(u.y & 0xFFFF0000u);
+            }
+        } else {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) x[k] = (c0 + k < d) ? ld_elem(X, r * ldx + c0 + k, x_f32) : 0.0f;
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) acc[k] = fmaf(w, x[k], acc[k]);
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        if (c0 + k < d) part[static_cast<int64_t>(blockIdx.y) * d + c0 + k] = acc[k];
+}
+
+__global__ void colsum_finish_kernel(const float* __restrict__ part, int64_t nblocks, int64_t d, float scale,
+                                     void* __restrict__ out, int out_f32, const DevScalars* sc) {
+    if (sc->status != 0) return;
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (j >= d) return;
+    float a = 0.0f;
+    for (int64_t b = 0; b < nblocks; ++b) a += part[b * d + j];
+    st_elem(out, j, out_f32, a * scale);
+}
+
+__global__ void axpby_kernel(const float* __restrict__ s, const float* __restrict__ qh, float a, float b, int64_t V,
+                             void* __restrict__ out, int out_f32, const DevScalars* sc) {
+    if (sc->status != 0) return;
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (j >= V) return;
+    st_elem(out, j, out_f32, a * s[j] + b * qh[j]);
+}
+
+inline unsigned cdiv(int64_t a, int64_t b) { return static_cast<unsigned>((a + b - 1) / b); }
+
+}  // namespace
+
+void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda, DevScalars* sc,
+                        cudaStream_t s) {
+    labels_scan_kernel<<<1, 1024, 0, s>>>(labels, n, V, ignore, lambda, sc); count_launch();
+}
+
+void launch_row_stats_f32(const float* Z, int64_t ldz, int64_t n, int64_t V, float* stats, const DevScalars* sc,
+                          cudaStream_t s) {
+    row_stats_f32_kernel<<<cdiv(n * 32, 256), 256, 0, s>>>(Z, ldz, n, V, reinterpret_cast<float2*>(stats), sc); count_launch();
+}
+
+void launch_row_lse(const void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* stats, int64_t ntiles,
+                    const int32_t* labels, int32_t ignore, float* lse, float* ce, const DevScalars* sc,
+                    cudaStream_t s) {
+    row_lse_kernel<<<cdiv(n * 32, 256), 256, 0, s>>>(Z, z_f32, ldz, n, V, reinterpret_cast<const float2*>(stats),
+                                                      ntiles, labels, ignore, lse, ce, sc); count_launch();
+}
+
+void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* lse, const int32_t* labels,
+                     int32_t ignore, float* colpart, const DevScalars* sc, cudaStream_t s) {
+    if (z_f32) {
+        dim3 grid(cdiv(ldz, 256 * 4), static_cast<unsigned>(row_blocks(n)));
+        residual_kernel<float, 4><<<grid, 256, 0, s>>>(static_cast<float*>(Z), ldz, n, V, lse, labels, ignore,
+                                                       colpart, sc); count_launch();
+    } else {
+        dim3 grid(cdiv(ldz, 256 * 8), static_cast<unsigned>(row_blocks(n)));
+        residual_kernel<__nv_bfloat16, 8><<<grid, 256, 0, s>>>(static_cast<__nv_bfloat16*>(Z), ldz, n, V, lse,
+                                                               labels, ignore, colpart, sc); count_launch();
+    }
+}
+
+void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float inv_bc1, float* q,
+                      float* s_out, float* qhat, DevScalars* sc, cudaStream_t s) {
+    finish_sq_kernel<<<cdiv(V, 256), 256, 0, s>>>(colpart, nblocks, V, beta1, inv_bc1, q, s_out, qhat, sc); count_launch();
+}
+
+void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, DevScalars* sc, cudaStream_t s) {
+    scalars_kernel<<<1, 1024, 0, s>>>(ce, n, s_vec, V, sc); count_launch();
+}
+
+void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, const int32_t* labels,
+                   int32_t ignore, const float* wvec, float scale, float* part, void* out, int out_f32,
+                   const DevScalars* sc, cudaStream_t s) {
+    const int64_t nb = row_blocks(n);
+    dim3 grid(cdiv(d, 1024), static_cast<unsigned>(nb));
+    colsum_part_kernel<<<grid, 256, 0, s>>>(X, x_f32, ldx, n, d, labels, ignore, wvec, part, sc); count_launch();
+    colsum_finish_kernel<<<cdiv(d, 256), 256, 0, s>>>(part, nb, d, scale, out, out_f32, sc); count_launch();
+}
+
+void launch_axpby(const float* s_vec, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
+                  const DevScalars* sc, cudaStream_t s) {
+    axpby_kernel<<<cdiv(V, 256), 256, 0, s>>>(s_vec, qhat, a, b, V, out, out_f32, sc); count_launch();
+}
+
+}  // namespace bom

@@ -1,0 +1,121 @@
+// BOM-AdamW update (Section 3.4; Algorithm 1, last two steps), one HBM pass:
+//   u     = g                      (numerator supplied directly), or
+//   u     = (1-lambda) g + lambda h  (Eq. mix-gradient, from separate g and h)
+//   v    <- beta2 v + (1-beta2) u^2
+//   theta <- (1 - lr wd) theta - lr u / (sqrt(v / (1-beta2^t)) + eps)
+// There is no first-moment buffer and no first-moment bias correction.
+// Each thread moves 4 elements per access with 128-bit (fp32) / 64-bit (bf16)
+// streaming loads and stores; the grid is a multiple of the SM count and
+// strides over the range.
+#include "kernels.h"
+
+namespace bom {
+namespace {
+
+struct UpdCoef {
+    float lr, decay, lam, beta2, one_m_beta2, eps, inv_bc2;
+};
+
+__device__ __forceinline__ float upd1(float& th, float& vv, float u, const UpdCoef& c) {
+    vv = fmaf(c.beta2, vv, c.one_m_beta2 * u * u);
+    const float den = sqrtf(vv * c.inv_bc2) + c.eps;
+    th = c.decay * th - c.lr * (u / den);
+    return th;
+}
+
+template <bool G_BF16, bool HAS_H, bool SHADOW>
+__global__ void __launch_bounds__(256) update_kernel(float* __restrict__ theta, const void* __restrict__ g,
+                                                     const float* __restrict__ h, float* __restrict__ v,
+                                                     uint16_t* __restrict__ shadow, int64_t n, UpdCoef c) {
+    const int64_t n4 = n >> 2;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
+        float4 th = __ldcs(reinterpret_cast<const float4*>(theta) + i);
+        float4 vv = __ldcs(reinterpret_cast<const float4*>(v) + i);
+        float u[4];
+        if constexpr (G_BF16) {
+            const uint2 w = __ldcs(reinterpret_cast<const uint2*>(g) + i);
+            u[0] = __uint_as_float(w.x << 16);
+            u[1] = __uint_as_float(w.x & 0xFFFF0000u);
+            u[2] = __uint_as_float(w.y << 16);
+            u[3] = __uint_as_float(w.y & 0xFFFF0000u);
+        } else {
+            const float4 f = __ldcs(reinterpret_cast<const float4*>(g) + i);
+            u[0] = f.x; u[1] = f.y; u[2] = f.z; u[3] = f.w;
+        }
+        if constexpr (HAS_H) {
+            const float4 hh = __ldcs(reinterpret_cast<const float4*>(h) + i);
+            const float om = 1.0f - c.lam;
+            u[0] = om * u[0] + c.lam * hh.x;
+            u[1] = om * u[1] + c.lam * hh.y;
+            u[2] = om * u[2] + c.lam * hh.z;
+            u[3] = om * u[3] + c.lam * hh.w;
+        }
+        upd1(th.x, vv.x, u[0], c);
+        upd1(th.y, vv.y, u[1], c);
+        upd1(th.z, vv.z, u[2], c);
+        upd1(th.w, vv.w, u[3], c);
+        __stcs(reinterpret_cast<float4*>(theta) + i, th);
+        __stcs(reinterpret_cast<float4*>(v) + i, vv);
+        if constexpr (SHADOW) {
+            uint2 sh;
+            sh.x = pack_bf16x2(th.x, th.y);
+            sh.y = pack_bf16x2(th.z, th.w);
+            __stcs(reinterpret_cast<uint2*>(shadow) + i, sh);
+        }
+    }
+    // tail (n not a multiple of 4)
+    const int64_t t = (n4 << 2) + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (t < n && t < (n4 << 2) + 4) {
+        float u = G_BF16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(g)[t]) : static_cast<const float*>(g)[t];
+        if (HAS_H) u = (1.0f - c.lam) * u + c.lam * h[t];
+        float th = theta[t], vv = v[t];
+        upd1(th, vv, u, c);
+        theta[t] = th;
+        v[t] = vv;
+        if (SHADOW) reinterpret_cast<__nv_bfloat16*>(shadow)[t] = __float2bfloat16_rn(th);
+    }
+}
+
+template <bool G_BF16, bool HAS_H>
+void dispatch_shadow(float* theta, const void* g, const float* h, float* v, uint16_t* shadow, int64_t n,
+                     const UpdCoef& c, int grid, cudaStream_t s) {
+    if (shadow) {
+        update_kernel<G_BF16, HAS_H, true><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c);
+    } else {
+        update_kernel<G_BF16, HAS_H, false><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c);
+    }
+    count_launch();
+}
+
+}  // namespace
+
+int device_sm_count();
+
+int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,
+                  float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, cudaStream_t s) {
+    if (n <= 0) return BOM_OK;
+    UpdCoef c;
+    c.lr = lr;
+    c.decay = 1.0f - lr * wd;
+    c.lam = lambda;
+    c.beta2 = beta2;
+    c.one_m_beta2 = 1.0f - beta2;
+    c.eps = eps;
+    c.inv_bc2 = inv_bc2;
+    const int64_t n4 = (n >> 2) > 0 ? (n >> 2) : 1;
+    int64_t grid = static_cast<int64_t>(device_sm_count()) * 8;
+    const int64_t need = (n4 + 255) / 256;
+    if (grid > need) grid = need;
+    if (grid < 1) grid = 1;
+    if (g_bf16) {
+        if (h) dispatch_shadow<true, true>(theta, g, h, v, shadow, n, c, (int)grid, s);
+        else dispatch_shadow<true, false>(theta, g, h, v, shadow, n, c, (int)grid, s);
+    } else {
+        if (h) dispatch_shadow<false, true>(theta, g, h, v, shadow, n, c, (int)grid, s);
+        else dispatch_shadow<false, false>(theta, g, h, v, shadow, n, c, (int)grid, s);
+    }
+    return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+}  // namespace bom

@@ -1,0 +1,71 @@
+"""Helpers of the GPU parity tests: upload seeded inputs, run the C-ABI step and
+update through the Python binding, and run the fp64 oracle on the same inputs."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle as O
+from paper_2609_36738_gb300 import bom as B
+from paper_2609_36738_gb300 import inputs as I
+from tests import _indep as X
+
+DEV = "cuda"
+TOL = {"f32": 1e-5, "bf16": 2e-2}
+
+
+def ensure_built():
+    from paper_2609_36738_gb300 import build
+    build.build()
+    B.lib()
+
+
+def to_dev(arr: np.ndarray) -> torch.Tensor:
+    if arr.dtype == np.uint16:
+        return torch.from_numpy(np.ascontiguousarray(arr).view(np.int16)).to(DEV).view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(arr)).to(DEV)
+
+
+def np64(t: torch.Tensor) -> np.ndarray:
+    return t.detach().float().cpu().double().numpy()
+
+
+def host_f32(ptr: int, count: int) -> np.ndarray:
+    return np.frombuffer(B.copy_to_host(ptr, 4 * count), dtype=np.float32).astype(np.float64)
+
+
+rel_l2 = X.rel_l2
+
+
+class GpuBom:
+    """A handle plus device copies of a workload's parameters."""
+
+    def __init__(self, wl: I.Workload, params_np, out_mode=B.BOM_OUT_U, lam=0.5, beta1=0.9, max_rows=None):
+        self.wl = wl
+        self.out_mode = out_mode
+        self.model = B.BomModel(B.config_for(wl, lam, beta1, out_mode, max_rows))
+        self.params = [to_dev(p) for p in params_np]
+        self.q = torch.zeros(wl.vocab, dtype=torch.float32, device=DEV)
+
+    def step(self, x_np, y_np, t, check=True):
+        x = to_dev(x_np)
+        y = torch.from_numpy(np.ascontiguousarray(y_np, dtype=np.int32)).to(DEV)
+        grads = [torch.empty_like(p) for p in self.params]
+        hs = None
+        if self.out_mode == B.BOM_OUT_G_AND_H:
+            hs = [torch.empty(p.shape, dtype=torch.float32, device=DEV) for p in self.params]
+        self.model.step(x, y, x.shape[0], self.params, self.q, t, grads, hs)
+        st = self.model.stats(check=check)
+        qp, sp, lp = self.model.outputs()
+        V = self.wl.vocab
+        out = dict(stats=st, grads=grads, h=hs, q=np64(self.q))
+        if st["code"] == B.BOM_OK:
+            out["qhat"] = host_f32(qp, V)
+            out["s"] = host_f32(sp, V)
+            out["lse"] = host_f32(lp, x.shape[0])
+        return out
+
+
+def oracle_step(wl, params64, x_np, y_np, q_prev, t, lam=0.5, beta1=0.9):
+    return O.bom_step(X.oracle_layers(wl), wl.head_bias, params64, X.x_f64(wl, x_np), y_np, q_prev, t,
+                      lam=lam, beta1=beta1)

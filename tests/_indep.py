@@ -50,7 +50,7 @@ def torch_forward(wl: I.Workload, params, X):
 def autograd_mix(wl, params_np, X_np, labels, qhat, lam, ignore_index=-100):
     """Gradient of L_mix = (1-lam) CE + lam/N_t sum_i <z_i, qhat> via autograd."""
     ps = [torch.tensor(p, requires_grad=True) for p in params_np]
-    X = torch.tensor(X_np)
+    X = torch.tensor(X_np, requires_grad=True)
     Z = torch_forward(wl, ps, X)
     y = torch.tensor(np.asarray(labels, dtype=np.int64))
     valid = y != ignore_index
@@ -58,8 +58,9 @@ def autograd_mix(wl, params_np, X_np, labels, qhat, lam, ignore_index=-100):
     ce = F.cross_entropy(Z, y, ignore_index=ignore_index, reduction="sum") / n_t
     sur = (Z[valid] @ torch.tensor(qhat)).sum() / n_t
     loss = (1 - lam) * ce + lam * sur
-    grads = torch.autograd.grad(loss, ps)
-    return [g.numpy() for g in grads], float(ce)
+    grads = torch.autograd.grad(loss, ps + [X])
+    autograd_mix.last_dX = grads[-1].numpy()
+    return [g.numpy() for g in grads[:-1]], float(ce.detach())
 
 
 def fd_jacobians(wl, params_np, X_np, eps=1e-6):

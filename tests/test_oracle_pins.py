@@ -130,6 +130,7 @@ def test_u_matches_autograd_of_mix_objective(name):
         assert a.shape == b.shape
         assert X.rel_l2(a, b) < 1e-12
     assert math.isclose(out["ce"], ce, rel_tol=1e-13)
+    assert X.rel_l2(out["dX_u"], X.autograd_mix.last_dX) < 1e-12      # input cotangent
     g_grads, _ = X.autograd_mix(wl, params, x, y, out["qhat"], 0.0)
     for a, b in zip(out["g"], g_grads):
         assert X.rel_l2(a, b) < 1e-12
