@@ -51,6 +51,8 @@ def _args():
     p.add_argument("--workload", default="lm_mlp_bf16")
     p.add_argument("--no-extra", action="store_true", help="skip the head-only and update sub-measurements")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
+    p.add_argument("--tokens", type=int, default=0,
+                   help="smaller batch of the same workload (profiling captures); 0 = the workload's own")
     return p.parse_args()
 
 
@@ -209,6 +211,9 @@ def main():
 
     # ---------------------------------------------------------------- workload state
     wl = I.WORKLOADS[a.workload]
+    if a.tokens:
+        import dataclasses
+        wl = dataclasses.replace(wl, n_rows=a.tokens)
     params_np = I.init_params(wl, seed=rank)
     shapes = [s for _, s, _ in wl.param_shapes()]
     sizes = [int(np.prod(s)) for s in shapes]
@@ -404,6 +409,7 @@ def _head_only(B, torch, dev, stream, a, peaks):
     flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)
     tot = 0.0
     gem_fl = gem_ms = 0.0
+    per = {}
     for i in range(a.steps):
         flush.zero_()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -411,6 +417,7 @@ def _head_only(B, torch, dev, stream, a, peaks):
         m.step(x, y, wl.n_rows, params, q, a.warmup + 1 + i, grads, None, stream)
         e1.record(stream)
         for name, fl, by, ms in B.bom_trace_read(m.h, stream):
+            per[name] = per.get(name, 0.0) + ms / a.steps
             if name.startswith("gemm_tc"):
                 gem_fl += fl
                 gem_ms += ms
@@ -423,7 +430,8 @@ def _head_only(B, torch, dev, stream, a, peaks):
             "value": wl.n_rows * a.steps / (tot / 1e3), "unit": "tokens/s", "ms_per_step": tot / a.steps,
             "step_tflops": flops / (tot / a.steps / 1e3) / 1e12,
             "step_frac_of_bf16_peak": flops / (tot / a.steps / 1e3) / 1e12 / peaks["bf16_tflops"],
-            "gemm_tflops": gem_fl / (gem_ms / 1e3) / 1e12 if gem_ms else None}
+            "gemm_tflops": gem_fl / (gem_ms / 1e3) / 1e12 if gem_ms else None,
+            "kernels_ms_per_step": {k: round(v, 4) for k, v in sorted(per.items(), key=lambda kv: -kv[1])}}
 
 
 def _update_only(B, torch, dev, stream, a, peaks):
