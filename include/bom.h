@@ -202,6 +202,30 @@ int32_t bom_trace_read(bom_handle* h, bom_trace_entry* out, int32_t max, void* s
 /* Number of kernels this library has launched in the process so far. */
 int64_t bom_launch_count(void);
 
+/* Allocation-free weighted column sum (the paper has no counterpart; this is
+ * a convenience of this library).
+ *   out[j] = sum_i w_i * x[i, j]   for j < n_cols, with w_i = weights[i], or 1
+ *   when weights is NULL; fp32 accumulation, fp32 out [n_cols].
+ * This is the reduction bom_step uses to form colsum_{I_t}(H) and W^T qhat,
+ * for callers that may not allocate device memory: code running while its
+ * stream is being captured into a CUDA graph in global capture mode, where
+ * cudaMalloc is an error, and runtimes that manage every device byte through
+ * their own pool.  It calls no cudaMalloc/cudaFree and no allocating library
+ * routine.  Its scratch is one fixed device array of 4 MiB (2^20 floats) in
+ * the library; every GPU that loads the library keeps it until exit.
+ *   x        [n_rows, ldx] in dtype (BOM_F32 or BOM_BF16), 16-byte aligned.
+ *   weights  [n_rows] fp32 device vector, or NULL.
+ *   out      [n_cols] fp32 device vector.
+ * Limits: ceil(n_rows / 128) * n_cols <= 2^20 and n_rows <= 128 * 65535;
+ * larger sizes return BOM_ENOTSUP without touching the device.
+ * The first call on each device looks up the array's device address with
+ * cudaGetSymbolAddress; make that first call before any stream capture.
+ * All calls share the array: calls that overlap on the GPU (on different
+ * streams without ordering) race and produce wrong sums.  Each call writes
+ * every scratch element it later reads, so nothing needs to start at zero. */
+bom_status bom_colsum_noalloc(const void* x, int32_t dtype, int64_t ldx, int64_t n_rows, int64_t n_cols,
+                              const float* weights, float* out, void* stream);
+
 /* Frees the workspace and the handle.  NULL is a no-op. */
 void bom_destroy(bom_handle* h);
 

@@ -28,7 +28,7 @@ BOM_OUT_U, BOM_OUT_G_AND_H = 0, 1
 # Every symbol include/bom.h declares.
 EXPORTED = ("bom_param_count", "bom_param_shape", "bom_init", "bom_workspace_bytes", "bom_step",
             "bom_set_input_grad", "bom_step_outputs", "bom_get_stats", "bom_update", "bom_gemm_bf16", "bom_trace", "bom_trace_read",
-            "bom_launch_count", "bom_destroy", "bom_status_string")
+            "bom_launch_count", "bom_colsum_noalloc", "bom_destroy", "bom_status_string")
 
 # Bytes bom_get_stats copies from the device (the scalar block of a step).
 STATS_D2H_BYTES = 44
@@ -97,6 +97,8 @@ def lib() -> C.CDLL:
     L.bom_trace_read.restype = i32
     L.bom_launch_count.argtypes = []
     L.bom_launch_count.restype = i64
+    L.bom_colsum_noalloc.argtypes = [vp, i32, i64, i64, i64, vp, vp, vp]
+    L.bom_colsum_noalloc.restype = i32
     L.bom_destroy.argtypes = [vp]
     L.bom_destroy.restype = None
     L.bom_status_string.argtypes = [i32]
@@ -236,6 +238,13 @@ def bom_trace_read(h, stream=None, max_entries: int = 256):
 
 def bom_launch_count() -> int:
     return int(lib().bom_launch_count())
+
+
+def bom_colsum_noalloc(x, dtype: int, ldx: int, n_rows: int, n_cols: int, weights, out, stream=None) -> None:
+    """out[j] = sum_i w_i x[i, j] without any device allocation (fixed 4 MiB
+    scratch inside the library; see include/bom.h for the limits)."""
+    _check(lib().bom_colsum_noalloc(_ptr(x), int(dtype), int(ldx), int(n_rows), int(n_cols), _ptr(weights),
+                                    _ptr(out), _stream(stream)), "bom_colsum_noalloc")
 
 
 class BomModel:
