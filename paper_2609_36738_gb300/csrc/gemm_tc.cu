@@ -59,6 +59,49 @@ __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, 
     nt = r / gsz;
 }
 
+// 256 bf16 values of one row, columns [n0, n0 + 256) clipped at N (zeros past
+// N), as 16 packed 16-byte words.  Issued before the accumulator wait so that
+// the latency of these epilogue operands hides under the mainloop.
+__device__ __forceinline__ void load_row256_bf16(const void* base, int64_t row_off, int n0, int N,
+                                                 uint4 (&pk)[16]) {
+    const uint16_t* p = static_cast<const uint16_t*>(base) + row_off + n0;
+    if (n0 + 256 <= N) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) pk[i] = __ldg(reinterpret_cast<const uint4*>(p) + i);
+    } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            uint32_t w[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int c = 8 * i + 2 * j;
+                const uint32_t lo = (n0 + c < N) ? p[c] : 0u;
+                const uint32_t hi = (n0 + c + 1 < N) ? p[c + 1] : 0u;
+                w[j] = lo | (hi << 16);
+            }
+            pk[i] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+    }
+}
+
+// Chunk c (32 values) of a packed 256-value row; c is a constant once the
+// chunk loops are fully unrolled, so pk stays in registers.
+__device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[16], int c, float (&v)[32]) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint4 w = pk[4 * c + i];
+        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            v[8 * i + 2 * j] = __uint_as_float(ws[j] << 16);
+            v[8 * i + 2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
+        }
+    }
+}
+
+__device__ __forceinline__ float fast_exp(float x) { return exp2f(x * 1.4426950408889634f); }
+__device__ __forceinline__ float fast_sigmoid(float x) { return __frcp_rn(1.0f + fast_exp(-x)); }
+
 __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
     uint32_t r[32];
     __syncwarp();
@@ -223,17 +266,32 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int m0 = mt * BM;
             const int n0 = nt * p.bn_out;
             const int acc = it & 1;
+            const int m = m0 + row;
+            const bool valid = m < p.M;
+            // Per-row epilogue operands do not depend on the accumulator: load
+            // the whole 256-column row segment now, before the mainloop wait.
+            uint4 xa[16], xb[16];
+            const bool has_a = (EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.resid != nullptr);
+            const bool has_b = (EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.act == ACT_DGELU);
+            if (valid && has_a)
+                load_row256_bf16(EPI == EPI_SWIGLU_BWD ? e.aux : e.resid,
+                                 static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid), n0, p.N,
+                                 xa);
+            if (valid && has_b)
+                load_row256_bf16(EPI == EPI_SWIGLU_BWD ? e.aux2 : e.aux,
+                                 static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux), n0, p.N,
+                                 xb);
             if (kb_total > 0) {
                 if (!mbar_wait_bounded(&tfull[acc], (it >> 1) & 1, abort_flag)) break;
                 tc_fence_after();
             }
-            const int m = m0 + row;
-            const bool valid = m < p.M;
             const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
             float v[32];
 
             if constexpr (EPI == EPI_LINEAR) {
                 const EpiRow r = epi_row(e, m, p.M);
+                float t[32];
+#pragma unroll
                 for (int c = 0; c < BN / 32; ++c) {
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
@@ -243,17 +301,51 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] = 0.0f;
                     }
-                    if (valid) epi_linear32(e, r, m, n, p.N, v);
+                    if (valid) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] *= r.alpha;
+                        if (e.bias) {
+                            load_row32(e.bias, 0, n, p.N, 0, t);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] += t[i];
+                        }
+                        if (e.r1u) {
+                            load_vec32(e.r1v, n, p.N, t);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] += r.beta_r1 * t[i];
+                        }
+                        if (e.bw) {
+                            load_vec32(e.bw, n, p.N, t);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] += r.beta_bw * t[i];
+                        }
+                        if (e.resid) {
+                            unpack32_dyn(xa, c, t);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] += t[i];
+                        }
+                        if (e.act == ACT_GELU) {
+                            store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, p.N, e.out2_f32, v);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] = gelu_f(e.out2_f32 ? v[i] : round_bf16(v[i]));
+                        } else if (e.act == ACT_DGELU) {
+                            unpack32_dyn(xb, c, t);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(t[i]);
+                        }
+                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
+                    }
                 }
             } else if constexpr (EPI == EPI_LOGITS) {
                 float mx = -INFINITY, sm = 0.0f;
                 float t[32];
+#pragma unroll
                 for (int c = 0; c < BN / 32; ++c) {
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
                     if (e.bias) {
-                        load_row32(e.bias, 0, n, p.N, e.in_f32, t);
+                        load_row32(e.bias, 0, n, p.N, 0, t);
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] += t[i];
                     }
@@ -267,10 +359,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     for (int i = 0; i < 32; ++i)
                         if (n + i < p.N) cm = fmaxf(cm, v[i]);
                     const float nm = fmaxf(mx, cm);
-                    float s = (mx == -INFINITY) ? 0.0f : sm * expf(mx - nm);
+                    float s = (mx == -INFINITY) ? 0.0f : sm * fast_exp(mx - nm);
 #pragma unroll
                     for (int i = 0; i < 32; ++i)
-                        if (n + i < p.N) s += expf(v[i] - nm);
+                        if (n + i < p.N) s += fast_exp(v[i] - nm);
                     mx = nm;
                     sm = s;
                 }
@@ -280,6 +372,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 }
             } else if constexpr (EPI == EPI_SWIGLU_FWD) {
                 float u[32];
+#pragma unroll
                 for (int c = 0; c < 4; ++c) {
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
@@ -289,23 +382,27 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, p.N, e.out2_f32, v);
                         store_row32(e.out3, static_cast<int64_t>(m) * e.ld_out3, n, p.N, e.out2_f32, u);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = silu_f(round_bf16(v[i])) * round_bf16(u[i]);
+                        for (int i = 0; i < 32; ++i) {
+                            const float g = round_bf16(v[i]);
+                            v[i] = g * fast_sigmoid(g) * round_bf16(u[i]);
+                        }
                         store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
                     }
                 }
             } else if constexpr (EPI == EPI_SWIGLU_BWD) {
                 float g[32], u[32];
+#pragma unroll
                 for (int c = 0; c < BN / 32; ++c) {
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
                     if (valid) {
-                        load_row32(e.aux, static_cast<int64_t>(m) * e.ld_aux, n, p.N, e.in_f32, g);
-                        load_row32(e.aux2, static_cast<int64_t>(m) * e.ld_aux2, n, p.N, e.in_f32, u);
+                        unpack32_dyn(xa, c, g);
+                        unpack32_dyn(xb, c, u);
                         float du[32];
 #pragma unroll
                         for (int i = 0; i < 32; ++i) {
-                            const float sg = sigmoid_f(g[i]);
+                            const float sg = fast_sigmoid(g[i]);
                             du[i] = v[i] * g[i] * sg;
                             v[i] = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
                         }
@@ -399,6 +496,7 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     using namespace tc;
     if (g.M <= 0 || g.N <= 0) return BOM_OK;
     if (g.M > INT32_MAX / 2 || g.N > INT32_MAX / 2) return BOM_ENOTSUP;
+    if (g.epi.in_f32) return BOM_ENOTSUP;   // epilogue operands are bf16 on this engine
     Params p;
     memset(&p, 0, sizeof(p));
     const bool a_mn = g.A[0].mn_major, b_mn = g.B[0].mn_major;

@@ -143,7 +143,7 @@ __global__ void __launch_bounds__(256) residual_kernel(T* __restrict__ Z, int64_
 #pragma unroll
     for (int k = 0; k < VEC; ++k) csum[k] = 0.0f;
     if (col0 < ldz) {
-        constexpr int UNROLL = 4;
+        constexpr int UNROLL = 8;
         for (int64_t rb = r0; rb < r1; rb += UNROLL) {
             float zv[UNROLL][VEC];
 #pragma unroll
@@ -172,11 +172,16 @@ __global__ void __launch_bounds__(256) residual_kernel(T* __restrict__ Z, int64_
                 const int32_t y = labels[r];
                 const bool valid = (y != ignore);
                 const float L = lse[r];
+                // bf16 logits: exp2 of a pre-scaled argument (the result is
+                // stored in bf16); fp32 logits keep the accurate expf.
+                const float Ls = L * 1.4426950408889634f;
                 float rv[VEC];
 #pragma unroll
                 for (int k = 0; k < VEC; ++k) {
                     const int64_t c = col0 + k;
-                    float p = (valid && c < V) ? expf(zv[u][k] - L) : 0.0f;
+                    float p = 0.0f;
+                    if (valid && c < V)
+                        p = (sizeof(T) == 2) ? exp2f(fmaf(zv[u][k], 1.4426950408889634f, -Ls)) : expf(zv[u][k] - L);
                     if (valid && c == y) p -= 1.0f;
                     rv[k] = p;
                     csum[k] += p;
@@ -227,43 +232,77 @@ __global__ void __launch_bounds__(1024) scalars_kernel(const float* __restrict__
     }
 }
 
-// part[b, j] = sum_{i in row block b} w_i X[i, j]; 256 threads x 4 columns.
-__global__ void __launch_bounds__(256) colsum_part_kernel(const void* __restrict__ X, int x_f32, int64_t ldx,
-                                                          int64_t n, int64_t d, const int32_t* __restrict__ labels,
-                                                          int32_t ignore, const float* __restrict__ wvec,
-                                                          float* __restrict__ part, const DevScalars* sc) {
+// part[b, j] = sum_{i in row block b} w_i X[i, j].  A block covers 32 x VEC
+// columns of one row block: every warp reads 16-byte words of the same
+// columns, the 8 warps take interleaved rows, and the 8 warp sums are added
+// in a fixed order in shared memory (deterministic).
+template <typename T>
+__global__ void __launch_bounds__(256) colsum_part_kernel(const T* __restrict__ X, int64_t ldx, int64_t n, int64_t d,
+                                                          const int32_t* __restrict__ labels, int32_t ignore,
+                                                          const float* __restrict__ wvec, float* __restrict__ part,
+                                                          const DevScalars* sc) {
+    constexpr int VEC = 16 / sizeof(T);
+    __shared__ float red[8][32 * VEC];
     if (sc->status != 0) return;
-    const int64_t c0 = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) * 4;
-    if (c0 >= d) return;
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    const int64_t c0 = static_cast<int64_t>(blockIdx.x) * (32 * VEC) + l * VEC;
     const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kRowBlock;
     const int64_t r1 = min(r0 + kRowBlock, n);
-    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-    const bool vec = (c0 + 4 <= d) && ((ldx & 3) == 0);
-    for (int64_t r = r0; r < r1; ++r) {
-        float w = 1.0f;
-        if (labels) w = (labels[r] != ignore) ? 1.0f : 0.0f;
-        if (wvec) w = wvec[r];
-        if (w == 0.0f) continue;
-        float x[4];
-        if (vec) {
-            if (x_f32) {
-                const float4 f = *reinterpret_cast<const float4*>(static_cast<const float*>(X) + r * ldx + c0);
-                x[0] = f.x; x[1] = f.y; x[2] = f.z; x[3] = f.w;
-            } else {
-                const uint2 u = *reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(X) + r * ldx + c0);
-                x[0] = __uint_as_float(u.x << 16); x[1] = __uint_as_float(u.x & 0xFFFF0000u);
-                x[2] = __uint_as_float(u.y << 16); x[3] = __uint_as_float(u.y & 0xFFFF0000u);
-            }
-        } else {
+    float acc[VEC];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) x[k] = (c0 + k < d) ? ld_elem(X, r * ldx + c0 + k, x_f32) : 0.0f;
+    for (int k = 0; k < VEC; ++k) acc[k] = 0.0f;
+    const bool vec = (c0 + VEC <= d) && ((ldx % VEC) == 0);
+    constexpr int UNROLL = 4;
+    for (int64_t rb = r0 + w; rb < r1; rb += 8 * UNROLL) {
+        float x[UNROLL][VEC];
+        float wt[UNROLL];
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int64_t r = rb + 8 * u;
+            wt[u] = 0.0f;
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) x[u][k] = 0.0f;
+            if (r >= r1 || c0 >= d) continue;
+            float wr = 1.0f;
+            if (labels) wr = (labels[r] != ignore) ? 1.0f : 0.0f;
+            if (wvec) wr = wvec[r];
+            wt[u] = wr;
+            const T* src = X + r * ldx + c0;
+            if (vec) {
+                const uint4 q = *reinterpret_cast<const uint4*>(src);
+                if constexpr (sizeof(T) == 2) {
+                    const uint32_t ws[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        x[u][2 * j] = __uint_as_float(ws[j] << 16);
+                        x[u][2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
+                    }
+                } else {
+                    x[u][0] = __uint_as_float(q.x); x[u][1] = __uint_as_float(q.y);
+                    x[u][2] = __uint_as_float(q.z); x[u][3] = __uint_as_float(q.w);
+                }
+            } else {
+#pragma unroll
+                for (int k = 0; k < VEC; ++k)
+                    if (c0 + k < d) x[u][k] = ld_elem(src, k, sizeof(T) == 4);
+            }
         }
 #pragma unroll
-        for (int k = 0; k < 4; ++k) acc[k] = fmaf(w, x[k], acc[k]);
+        for (int u = 0; u < UNROLL; ++u)
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) acc[k] = fmaf(wt[u], x[u][k], acc[k]);
     }
 #pragma unroll
-    for (int k = 0; k < 4; ++k)
-        if (c0 + k < d) part[static_cast<int64_t>(blockIdx.y) * d + c0 + k] = acc[k];
+    for (int k = 0; k < VEC; ++k) red[w][l * VEC + k] = acc[k];
+    __syncthreads();
+    for (int j = threadIdx.x; j < 32 * VEC; j += 256) {
+        const int64_t c = static_cast<int64_t>(blockIdx.x) * (32 * VEC) + j;
+        if (c >= d) continue;
+        float a = 0.0f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) a += red[k][j];
+        part[static_cast<int64_t>(blockIdx.y) * d + c] = a;
+    }
 }
 
 __global__ void colsum_finish_kernel(const float* __restrict__ part, int64_t nblocks, int64_t d, float scale,
@@ -331,8 +370,16 @@ void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, 
                    int32_t ignore, const float* wvec, float scale, float* part, void* out, int out_f32,
                    const DevScalars* sc, cudaStream_t s) {
     const int64_t nb = row_blocks(n);
-    dim3 grid(cdiv(d, 1024), static_cast<unsigned>(nb));
-    colsum_part_kernel<<<grid, 256, 0, s>>>(X, x_f32, ldx, n, d, labels, ignore, wvec, part, sc); count_launch();
+    if (x_f32) {
+        dim3 grid(cdiv(d, 128), static_cast<unsigned>(nb));
+        colsum_part_kernel<float><<<grid, 256, 0, s>>>(static_cast<const float*>(X), ldx, n, d, labels, ignore, wvec,
+                                                       part, sc);
+    } else {
+        dim3 grid(cdiv(d, 256), static_cast<unsigned>(nb));
+        colsum_part_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(X), ldx, n, d,
+                                                               labels, ignore, wvec, part, sc);
+    }
+    count_launch();
     colsum_finish_kernel<<<cdiv(d, 256), 256, 0, s>>>(part, nb, d, scale, out, out_f32, sc); count_launch();
 }
 
