@@ -59,37 +59,38 @@ __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, 
     nt = r / gsz;
 }
 
-// 256 bf16 values of one row, columns [n0, n0 + 256) clipped at N (zeros past
-// N), as 16 packed 16-byte words.  Issued before the accumulator wait so that
-// the latency of these epilogue operands hides under the mainloop.
-__device__ __forceinline__ void load_row256_bf16(const void* base, int64_t row_off, int n0, int N,
-                                                 uint4 (&pk)[16]) {
-    const uint16_t* p = static_cast<const uint16_t*>(base) + row_off + n0;
-    if (n0 + 256 <= N) {
+// Epilogue operands (bf16, one row, 32 columns per chunk) are prefetched into
+// a 4-slot register ring: chunks 0-3 are loaded before the accumulator wait,
+// so their latency hides under the mainloop, and the slot a chunk frees is
+// refilled with the chunk four ahead.  Slot s holds words pk[4s .. 4s+3].
+__device__ __forceinline__ void load_chunk_bf16(const void* base, int64_t row_off, int n, int N, uint4 (&pk)[16],
+                                                int slot) {
+    const uint16_t* p = static_cast<const uint16_t*>(base) + row_off + n;
+    if (n + 32 <= N) {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) pk[i] = __ldg(reinterpret_cast<const uint4*>(p) + i);
+        for (int i = 0; i < 4; ++i) pk[4 * slot + i] = __ldg(reinterpret_cast<const uint4*>(p) + i);
     } else {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
+        for (int i = 0; i < 4; ++i) {
             uint32_t w[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const int c = 8 * i + 2 * j;
-                const uint32_t lo = (n0 + c < N) ? p[c] : 0u;
-                const uint32_t hi = (n0 + c + 1 < N) ? p[c + 1] : 0u;
+                const uint32_t lo = (n + c < N) ? p[c] : 0u;
+                const uint32_t hi = (n + c + 1 < N) ? p[c + 1] : 0u;
                 w[j] = lo | (hi << 16);
             }
-            pk[i] = make_uint4(w[0], w[1], w[2], w[3]);
+            pk[4 * slot + i] = make_uint4(w[0], w[1], w[2], w[3]);
         }
     }
 }
 
-// Chunk c (32 values) of a packed 256-value row; c is a constant once the
-// chunk loops are fully unrolled, so pk stays in registers.
-__device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[16], int c, float (&v)[32]) {
+// The 32 values of ring slot `slot`; the slot index is a constant once the
+// chunk loops are fully unrolled, so the ring stays in registers.
+__device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[16], int slot, float (&v)[32]) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const uint4 w = pk[4 * c + i];
+        const uint4 w = pk[4 * slot + i];
         const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
@@ -268,19 +269,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int acc = it & 1;
             const int m = m0 + row;
             const bool valid = m < p.M;
-            // Per-row epilogue operands do not depend on the accumulator: load
-            // the whole 256-column row segment now, before the mainloop wait.
+            // Per-row epilogue operands do not depend on the accumulator: the
+            // first four chunks are loaded now, before the mainloop wait.
             uint4 xa[16], xb[16];
-            const bool has_a = (EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.resid != nullptr);
-            const bool has_b = (EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.act == ACT_DGELU);
-            if (valid && has_a)
-                load_row256_bf16(EPI == EPI_SWIGLU_BWD ? e.aux : e.resid,
-                                 static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid), n0, p.N,
-                                 xa);
-            if (valid && has_b)
-                load_row256_bf16(EPI == EPI_SWIGLU_BWD ? e.aux2 : e.aux,
-                                 static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux), n0, p.N,
-                                 xb);
+            const bool has_a = valid && ((EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.resid != nullptr));
+            const bool has_b = valid && ((EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.act == ACT_DGELU));
+            const void* pa = EPI == EPI_SWIGLU_BWD ? e.aux : e.resid;
+            const void* pb = EPI == EPI_SWIGLU_BWD ? e.aux2 : e.aux;
+            const int64_t ra = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid);
+            const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c, p.N, xa, c);
+                if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c, p.N, xb, c);
+            }
             if (kb_total > 0) {
                 if (!mbar_wait_bounded(&tfull[acc], (it >> 1) & 1, abort_flag)) break;
                 tc_fence_after();
@@ -319,8 +321,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] += r.beta_bw * t[i];
                         }
-                        if (e.resid) {
-                            unpack32_dyn(xa, c, t);
+                        if (has_a) {
+                            unpack32_dyn(xa, c & 3, t);
+                            if (c + 4 < BN / 32) load_chunk_bf16(pa, ra, n + 128, p.N, xa, c & 3);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] += t[i];
                         }
@@ -328,8 +331,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                             store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, p.N, e.out2_f32, v);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] = gelu_f(e.out2_f32 ? v[i] : round_bf16(v[i]));
-                        } else if (e.act == ACT_DGELU) {
-                            unpack32_dyn(xb, c, t);
+                        } else if (has_b) {
+                            unpack32_dyn(xb, c & 3, t);
+                            if (c + 4 < BN / 32) load_chunk_bf16(pb, rb, n + 128, p.N, xb, c & 3);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(t[i]);
                         }
@@ -397,8 +401,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
                     if (valid) {
-                        unpack32_dyn(xa, c, g);
-                        unpack32_dyn(xb, c, u);
+                        unpack32_dyn(xa, c & 3, g);
+                        unpack32_dyn(xb, c & 3, u);
+                        if (c + 4 < BN / 32) {
+                            load_chunk_bf16(pa, ra, n + 128, p.N, xa, c & 3);
+                            load_chunk_bf16(pb, rb, n + 128, p.N, xb, c & 3);
+                        }
                         float du[32];
 #pragma unroll
                         for (int i = 0; i < 32; ++i) {
