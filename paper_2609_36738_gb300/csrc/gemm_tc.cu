@@ -36,6 +36,10 @@ constexpr int NUM_THREADS = 192;
 constexpr int TMEM_COLS = 512;
 constexpr int SMEM_BYTES = STAGES * (A_STAGE_BYTES + B_STAGE_BYTES) + 1024 + 256;
 constexpr int GROUP_M = 8;
+// Depth (in 32-column chunks) of the epilogue-operand prefetch ring; 0 loads
+// each chunk's operands just before it is used.
+constexpr int kPf = 2;
+constexpr int kRing = kPf > 0 ? kPf : 1;
 
 struct Params {
     CUtensorMap mapA[2];
@@ -63,7 +67,8 @@ __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, 
 // a 4-slot register ring: chunks 0-3 are loaded before the accumulator wait,
 // so their latency hides under the mainloop, and the slot a chunk frees is
 // refilled with the chunk four ahead.  Slot s holds words pk[4s .. 4s+3].
-__device__ __forceinline__ void load_chunk_bf16(const void* base, int64_t row_off, int n, int N, uint4 (&pk)[16],
+template <int NW>
+__device__ __forceinline__ void load_chunk_bf16(const void* base, int64_t row_off, int n, int N, uint4 (&pk)[NW],
                                                 int slot) {
     const uint16_t* p = static_cast<const uint16_t*>(base) + row_off + n;
     if (n + 32 <= N) {
@@ -87,7 +92,8 @@ __device__ __forceinline__ void load_chunk_bf16(const void* base, int64_t row_of
 
 // The 32 values of ring slot `slot`; the slot index is a constant once the
 // chunk loops are fully unrolled, so the ring stays in registers.
-__device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[16], int slot, float (&v)[32]) {
+template <int NW>
+__device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[NW], int slot, float (&v)[32]) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const uint4 w = pk[4 * slot + i];
@@ -271,7 +277,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const bool valid = m < p.M;
             // Per-row epilogue operands do not depend on the accumulator: the
             // first four chunks are loaded now, before the mainloop wait.
-            uint4 xa[16], xb[16];
+            uint4 xa[4 * kRing], xb[4 * kRing];
             const bool has_a = valid && ((EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.resid != nullptr));
             const bool has_b = valid && ((EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.act == ACT_DGELU));
             const void* pa = EPI == EPI_SWIGLU_BWD ? e.aux : e.resid;
@@ -279,7 +285,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t ra = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid);
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int c = 0; c < kPf; ++c) {
                 if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c, p.N, xa, c);
                 if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c, p.N, xb, c);
             }
@@ -322,8 +328,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                             for (int i = 0; i < 32; ++i) v[i] += r.beta_bw * t[i];
                         }
                         if (has_a) {
-                            unpack32_dyn(xa, c & 3, t);
-                            if (c + 4 < BN / 32) load_chunk_bf16(pa, ra, n + 128, p.N, xa, c & 3);
+                            if (kPf == 0) load_chunk_bf16(pa, ra, n, p.N, xa, 0);
+                            unpack32_dyn(xa, kPf ? c % kPf : 0, t);
+                            if (kPf && c + kPf < BN / 32) load_chunk_bf16(pa, ra, n + 32 * kPf, p.N, xa, c % kPf);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] += t[i];
                         }
@@ -332,8 +339,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] = gelu_f(e.out2_f32 ? v[i] : round_bf16(v[i]));
                         } else if (has_b) {
-                            unpack32_dyn(xb, c & 3, t);
-                            if (c + 4 < BN / 32) load_chunk_bf16(pb, rb, n + 128, p.N, xb, c & 3);
+                            if (kPf == 0) load_chunk_bf16(pb, rb, n, p.N, xb, 0);
+                            unpack32_dyn(xb, kPf ? c % kPf : 0, t);
+                            if (kPf && c + kPf < BN / 32) load_chunk_bf16(pb, rb, n + 32 * kPf, p.N, xb, c % kPf);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(t[i]);
                         }
@@ -401,11 +409,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
                     if (valid) {
-                        unpack32_dyn(xa, c & 3, g);
-                        unpack32_dyn(xb, c & 3, u);
-                        if (c + 4 < BN / 32) {
-                            load_chunk_bf16(pa, ra, n + 128, p.N, xa, c & 3);
-                            load_chunk_bf16(pb, rb, n + 128, p.N, xb, c & 3);
+                        if (kPf == 0) {
+                            load_chunk_bf16(pa, ra, n, p.N, xa, 0);
+                            load_chunk_bf16(pb, rb, n, p.N, xb, 0);
+                        }
+                        unpack32_dyn(xa, kPf ? c % kPf : 0, g);
+                        unpack32_dyn(xb, kPf ? c % kPf : 0, u);
+                        if (kPf && c + kPf < BN / 32) {
+                            load_chunk_bf16(pa, ra, n + 32 * kPf, p.N, xa, c % kPf);
+                            load_chunk_bf16(pb, rb, n + 32 * kPf, p.N, xb, c % kPf);
                         }
                         float du[32];
 #pragma unroll
