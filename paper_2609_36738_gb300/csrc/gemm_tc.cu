@@ -8,10 +8,11 @@
 //   warp 1     allocates 512 TMEM columns (two 128 x 256 fp32 accumulators)
 //              and one thread issues the UMMAs (M = 128, N = 256, K = 16),
 //              releasing each smem stage with tcgen05.commit;
-//   warps 2-5  epilogue: tcgen05.ld of the accumulator (one TMEM lane = one
-//              output row per thread), the fused epilogue of the step, and
-//              global stores.  With two accumulators the epilogue of tile i
-//              overlaps the mainloop of tile i+1.
+//   warps 2-9  epilogue: tcgen05.ld of the accumulator (one TMEM lane = one
+//              output row per thread; two warps per lane quarter, one per
+//              column half), the fused epilogue of the step, and global
+//              stores.  With two accumulators the epilogue of tile i overlaps
+//              the mainloop of tile i+1.
 // Every mbarrier wait is bounded; a wait that runs out latches BOM_ETIMEOUT,
 // all roles unwind, in-flight TMA loads and UMMAs are drained, TMEM is freed.
 #include <cstdio>
@@ -32,14 +33,10 @@ constexpr int BK = 64;  // one 128-byte swizzle atom of bf16 along K
 constexpr int STAGES = 4;
 constexpr int A_STAGE_BYTES = BM * BK * 2;  // 16 KB
 constexpr int B_STAGE_BYTES = BN * BK * 2;  // 32 KB
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_THREADS = 320;  // producer warp, UMMA warp, 8 epilogue warps
 constexpr int TMEM_COLS = 512;
 constexpr int SMEM_BYTES = STAGES * (A_STAGE_BYTES + B_STAGE_BYTES) + 1024 + 256;
 constexpr int GROUP_M = 8;
-// Depth (in 32-column chunks) of the epilogue-operand prefetch ring; 0 loads
-// each chunk's operands just before it is used.
-constexpr int kPf = 2;
-constexpr int kRing = kPf > 0 ? kPf : 1;
 
 struct Params {
     CUtensorMap mapA[2];
@@ -63,10 +60,8 @@ __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, 
     nt = r / gsz;
 }
 
-// Epilogue operands (bf16, one row, 32 columns per chunk) are prefetched into
-// a 4-slot register ring: chunks 0-3 are loaded before the accumulator wait,
-// so their latency hides under the mainloop, and the slot a chunk frees is
-// refilled with the chunk four ahead.  Slot s holds words pk[4s .. 4s+3].
+// One 32-column chunk of a bf16 epilogue operand row (zeros past N) into
+// words pk[4*slot .. 4*slot+3].
 template <int NW>
 __device__ __forceinline__ void load_chunk_bf16(const void* base, int64_t row_off, int n, int N, uint4 (&pk)[NW],
                                                 int slot) {
@@ -90,8 +85,7 @@ __device__ __forceinline__ void load_chunk_bf16(const void* base, int64_t row_of
     }
 }
 
-// The 32 values of ring slot `slot`; the slot index is a constant once the
-// chunk loops are fully unrolled, so the ring stays in registers.
+// The 32 values held in words pk[4*slot .. 4*slot+3].
 template <int NW>
 __device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[NW], int slot, float (&v)[32]) {
 #pragma unroll
@@ -144,7 +138,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
-            mbar_init(&tempty[a], 128);
+            mbar_init(&tempty[a], 256);
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -263,9 +257,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         }
     } else if (!skip && warp >= 2) {
         // ------------------------------------------------------------ epilogue
-        const int q = warp & 3;  // TMEM lane quarter this warp may access
+        // Eight warps: warp w reads TMEM lane quarter (w & 3) (its 32 output
+        // rows) and column half h of the tile, so every TMEM quarter has two
+        // warps and the epilogue's global-memory latency is overlapped twice.
+        const int q = warp & 3;
+        const int h = (warp - 2) >> 2;
         const int row = q * 32 + lane;
         const EpiParams& e = p.epi;
+        constexpr int CPW = BN / 64;  // 32-column chunks per warp
         int it = 0;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
             int mt, nt;
@@ -275,20 +274,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int acc = it & 1;
             const int m = m0 + row;
             const bool valid = m < p.M;
+            const int c0 = h * CPW;
             // Per-row epilogue operands do not depend on the accumulator: the
-            // first four chunks are loaded now, before the mainloop wait.
-            uint4 xa[4 * kRing], xb[4 * kRing];
+            // warp's first chunk is loaded before the mainloop wait, and each
+            // later chunk while the previous one is being processed.
+            uint4 xa[4], xb[4];
             const bool has_a = valid && ((EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.resid != nullptr));
             const bool has_b = valid && ((EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.act == ACT_DGELU));
             const void* pa = EPI == EPI_SWIGLU_BWD ? e.aux : e.resid;
             const void* pb = EPI == EPI_SWIGLU_BWD ? e.aux2 : e.aux;
             const int64_t ra = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid);
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
-#pragma unroll
-            for (int c = 0; c < kPf; ++c) {
-                if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c, p.N, xa, c);
-                if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c, p.N, xb, c);
-            }
+            if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
+            if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
             if (kb_total > 0) {
                 if (!mbar_wait_bounded(&tfull[acc], (it >> 1) & 1, abort_flag)) break;
                 tc_fence_after();
@@ -299,8 +297,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             if constexpr (EPI == EPI_LINEAR) {
                 const EpiRow r = epi_row(e, m, p.M);
                 float t[32];
-#pragma unroll
-                for (int c = 0; c < BN / 32; ++c) {
+#pragma unroll 1
+                for (int j = 0; j < CPW; ++j) {
+                    const int c = c0 + j;
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
                     if (kb_total > 0) {
@@ -328,9 +327,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                             for (int i = 0; i < 32; ++i) v[i] += r.beta_bw * t[i];
                         }
                         if (has_a) {
-                            if (kPf == 0) load_chunk_bf16(pa, ra, n, p.N, xa, 0);
-                            unpack32_dyn(xa, kPf ? c % kPf : 0, t);
-                            if (kPf && c + kPf < BN / 32) load_chunk_bf16(pa, ra, n + 32 * kPf, p.N, xa, c % kPf);
+                            unpack32_dyn(xa, 0, t);
+                            if (j + 1 < CPW) load_chunk_bf16(pa, ra, n + 32, p.N, xa, 0);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] += t[i];
                         }
@@ -339,9 +337,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] = gelu_f(e.out2_f32 ? v[i] : round_bf16(v[i]));
                         } else if (has_b) {
-                            if (kPf == 0) load_chunk_bf16(pb, rb, n, p.N, xb, 0);
-                            unpack32_dyn(xb, kPf ? c % kPf : 0, t);
-                            if (kPf && c + kPf < BN / 32) load_chunk_bf16(pb, rb, n + 32 * kPf, p.N, xb, c % kPf);
+                            unpack32_dyn(xb, 0, t);
+                            if (j + 1 < CPW) load_chunk_bf16(pb, rb, n + 32, p.N, xb, 0);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(t[i]);
                         }
@@ -349,10 +346,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     }
                 }
             } else if constexpr (EPI == EPI_LOGITS) {
+                // per (row, column half) softmax statistics: stats pair nt*2 + h
                 float mx = -INFINITY, sm = 0.0f;
                 float t[32];
-#pragma unroll
-                for (int c = 0; c < BN / 32; ++c) {
+#pragma unroll 1
+                for (int j = 0; j < CPW; ++j) {
+                    const int c = c0 + j;
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
@@ -379,13 +378,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     sm = s;
                 }
                 if (valid) {
-                    float2* st = reinterpret_cast<float2*>(e.stats) + static_cast<int64_t>(m) * e.ld_stats + nt;
+                    float2* st = reinterpret_cast<float2*>(e.stats) + static_cast<int64_t>(m) * e.ld_stats + 2 * nt + h;
                     *st = make_float2(mx, sm);
                 }
             } else if constexpr (EPI == EPI_SWIGLU_FWD) {
+                // gate columns [0, 128) and up columns [128, 256) of the accumulator
                 float u[32];
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
+#pragma unroll 1
+                for (int j = 0; j < 2; ++j) {
+                    const int c = 2 * h + j;
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
@@ -403,21 +404,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 }
             } else if constexpr (EPI == EPI_SWIGLU_BWD) {
                 float g[32], u[32];
-#pragma unroll
-                for (int c = 0; c < BN / 32; ++c) {
+#pragma unroll 1
+                for (int j = 0; j < CPW; ++j) {
+                    const int c = c0 + j;
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
                     if (valid) {
-                        if (kPf == 0) {
-                            load_chunk_bf16(pa, ra, n, p.N, xa, 0);
-                            load_chunk_bf16(pb, rb, n, p.N, xb, 0);
-                        }
-                        unpack32_dyn(xa, kPf ? c % kPf : 0, g);
-                        unpack32_dyn(xb, kPf ? c % kPf : 0, u);
-                        if (kPf && c + kPf < BN / 32) {
-                            load_chunk_bf16(pa, ra, n + 32 * kPf, p.N, xa, c % kPf);
-                            load_chunk_bf16(pb, rb, n + 32 * kPf, p.N, xb, c % kPf);
+                        unpack32_dyn(xa, 0, g);
+                        unpack32_dyn(xb, 0, u);
+                        if (j + 1 < CPW) {
+                            load_chunk_bf16(pa, ra, n + 32, p.N, xa, 0);
+                            load_chunk_bf16(pb, rb, n + 32, p.N, xb, 0);
                         }
                         float du[32];
 #pragma unroll
@@ -510,7 +508,7 @@ int device_sm_count() {
     return n;
 }
 
-int64_t tc_logit_tiles(int64_t N) { return (N + tc::BN - 1) / tc::BN; }
+int64_t tc_logit_tiles(int64_t N) { return 2 * ((N + tc::BN - 1) / tc::BN); }  // one pair per column half
 
 int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     using namespace tc;
