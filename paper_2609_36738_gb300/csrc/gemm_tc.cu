@@ -30,12 +30,8 @@ namespace tc {
 constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = 64;  // one 128-byte swizzle atom of bf16 along K
-constexpr int STAGES = 4;
-constexpr int A_STAGE_BYTES = BM * BK * 2;  // 16 KB
-constexpr int B_STAGE_BYTES = BN * BK * 2;  // 32 KB
 constexpr int NUM_THREADS = 320;  // producer warp, UMMA warp, 8 epilogue warps
 constexpr int TMEM_COLS = 512;
-constexpr int SMEM_BYTES = STAGES * (A_STAGE_BYTES + B_STAGE_BYTES) + 1024 + 256;
 constexpr int GROUP_M = 8;
 
 struct Params {
@@ -112,13 +108,30 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-template <bool A_MN, bool B_MN, int EPI>
+// Shared-memory pipeline of one CTA.  CG = 1: the CTA computes 128 x 256
+// tiles alone.  CG = 2: a CTA pair (cluster of 2) computes 256 x 256 tiles
+// with tcgen05 cta_group::2 UMMAs issued by the even CTA; each CTA stages its
+// own 128 rows of A and its half (128 rows) of B, so a stage is 32 KB and six
+// stages fit.
+template <int CG>
+struct Cfg {
+    static constexpr int B_ROWS = CG == 2 ? 128 : 256;
+    static constexpr int STAGES = CG == 2 ? 6 : 4;
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = B_ROWS * BK * 2;
+    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + 1024 + 256;
+    static constexpr int TILE_M = BM * CG;
+};
+
+template <int CG, bool A_MN, bool B_MN, int EPI>
 __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_constant__ Params p) {
+    using C = Cfg<CG>;
+    constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sA = smem;
-    uint8_t* sB = smem + STAGES * A_STAGE_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + STAGES * B_STAGE_BYTES);
+    uint8_t* sB = smem + STAGES * C::A_BYTES;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + STAGES * C::B_BYTES);
     uint64_t* full = bars;
     uint64_t* empty = bars + STAGES;
     uint64_t* tfull = bars + 2 * STAGES;
@@ -130,6 +143,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    const uint32_t rank = CG == 2 ? cluster_ctarank() : 0u;
+    const bool leader = rank == 0;
+    const int unit = CG == 2 ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+    const int nunits = CG == 2 ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -138,7 +155,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
-            mbar_init(&tempty[a], 256);
+            // CG = 2: one elected arrival per CTA of the pair on the even CTA's barrier
+            mbar_init(&tempty[a], CG == 2 ? 2 : 256);
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -150,11 +168,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         prefetch_tensormap(&p.mapB[0]);
     }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, TMEM_COLS);
-        tmem_relinquish();
+        if constexpr (CG == 2) {
+            tmem_alloc_pair(tmem_slot, TMEM_COLS);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(tmem_slot, TMEM_COLS);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
     __syncthreads();
+    if constexpr (CG == 2) cluster_sync();   // barriers of both CTAs initialised before any remote use
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     const bool skip = *skip_flag != 0;
@@ -169,36 +193,46 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_phase = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
+            for (int tile = unit; ok && tile < num_tiles; tile += nunits) {
                 int mt, nt;
                 tile_coords(tile, p.tiles_m, p.tiles_n, mt, nt);
-                const int m0 = mt * BM;
+                const int m_own = mt * C::TILE_M + static_cast<int>(rank) * BM;
                 const int n0 = nt * p.bn_out;
+                const int n_own = n0 + (CG == 2 && !p.dual_b ? static_cast<int>(rank) * C::B_ROWS : 0);
                 for (int seg = 0; ok && seg < p.nseg; ++seg) {
                     for (int kb = 0; kb < p.kb[seg]; ++kb) {
                         if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag)) {
                             ok = false;
                             break;
                         }
-                        mbar_arrive_expect_tx(&full[stage], A_STAGE_BYTES + B_STAGE_BYTES);
+                        if (leader) mbar_arrive_expect_tx(&full[stage], CG * (C::A_BYTES + C::B_BYTES));
                         const int k0 = kb * BK;
-                        uint8_t* a = sA + stage * A_STAGE_BYTES;
-                        uint8_t* b = sB + stage * B_STAGE_BYTES;
+                        uint8_t* a = sA + stage * C::A_BYTES;
+                        uint8_t* b = sB + stage * C::B_BYTES;
+                        auto load = [&](void* dst, const CUtensorMap* map, int x, int y) {
+                            if constexpr (CG == 2)
+                                tma_load_2d_pair(dst, map, mapa_shared(smem_u32(&full[stage]), 0), x, y);
+                            else
+                                tma_load_2d(dst, map, &full[stage], x, y);
+                        };
                         if (!A_MN) {
-                            tma_load_2d(a, &p.mapA[seg], &full[stage], k0, m0);
+                            load(a, &p.mapA[seg], k0, m_own);
                         } else {
-                            tma_load_2d(a, &p.mapA[seg], &full[stage], m0, k0);
-                            tma_load_2d(a + 8192, &p.mapA[seg], &full[stage], m0 + 64, k0);
+                            load(a, &p.mapA[seg], m_own, k0);
+                            load(a + 8192, &p.mapA[seg], m_own + 64, k0);
                         }
                         if (p.dual_b) {
-                            tma_load_2d(b, &p.mapB[0], &full[stage], k0, n0);
-                            tma_load_2d(b + 16384, &p.mapB[1], &full[stage], k0, n0);
+                            if constexpr (CG == 2) {
+                                load(b, &p.mapB[rank], k0, n0);   // even CTA: gate rows, odd CTA: up rows
+                            } else {
+                                load(b, &p.mapB[0], k0, n0);
+                                load(b + 16384, &p.mapB[1], k0, n0);
+                            }
                         } else if (!B_MN) {
-                            tma_load_2d(b, &p.mapB[seg], &full[stage], k0, n0);
+                            load(b, &p.mapB[seg], k0, n_own);
                         } else {
 #pragma unroll
-                            for (int j = 0; j < 4; ++j)
-                                tma_load_2d(b + j * 8192, &p.mapB[seg], &full[stage], n0 + 64 * j, k0);
+                            for (int j = 0; j < C::B_ROWS / 64; ++j) load(b + j * 8192, &p.mapB[seg], n_own + 64 * j, k0);
                         }
                         issued_mask |= 1u << stage;
                         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -209,19 +243,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     }
                 }
             }
-            // Every issued load must land before the CTA may exit.
-            for (int s = 0; s < STAGES; ++s)
-                if (issued_mask & (1u << s)) mbar_wait_bounded(&full[s], (issued_phase >> s) & 1u, nullptr);
+            // Every issued load must land before the CTA may exit (the even CTA's
+            // full barriers also count the odd CTA's loads).
+            if (leader)
+                for (int s = 0; s < STAGES; ++s)
+                    if (issued_mask & (1u << s)) mbar_wait_bounded(&full[s], (issued_phase >> s) & 1u, nullptr);
         }
     } else if (!skip && warp == 1) {
-        // ------------------------------------------------------------ UMMA issuer
-        if (lane == 0 && kb_total > 0) {
-            constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, A_MN, B_MN);
+        // ------------------------------------------------------------ UMMA issuer (even CTA)
+        if (lane == 0 && kb_total > 0 && leader) {
+            constexpr uint32_t idesc = idesc_bf16_f32(C::TILE_M, BN, A_MN, B_MN);
+            constexpr uint32_t b_lbo = 8192;   // MN-major: next 64-column chunk
             int stage = 0;
             uint32_t phase = 0;
             bool ok = true;
             int it = 0;
-            for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x, ++it) {
+            for (int tile = unit; ok && tile < num_tiles; tile += nunits, ++it) {
                 const int acc = it & 1;
                 const uint32_t aph = (it >> 1) & 1;
                 if (!mbar_wait_bounded(&tempty[acc], aph ^ 1u, abort_flag)) break;
@@ -233,26 +270,40 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a0 = smem_u32(sA + stage * A_STAGE_BYTES);
-                    const uint32_t b0 = smem_u32(sB + stage * B_STAGE_BYTES);
+                    const uint32_t a0 = smem_u32(sA + stage * C::A_BYTES);
+                    const uint32_t b0 = smem_u32(sB + stage * C::B_BYTES);
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk) {
                         const uint64_t ad = A_MN ? smem_desc_sw128(a0 + kk * 2048, 8192, 1024)
                                                  : smem_desc_sw128(a0 + kk * 32, 16, 1024);
-                        const uint64_t bd = B_MN ? smem_desc_sw128(b0 + kk * 2048, 8192, 1024)
+                        const uint64_t bd = B_MN ? smem_desc_sw128(b0 + kk * 2048, b_lbo, 1024)
                                                  : smem_desc_sw128(b0 + kk * 32, 16, 1024);
-                        umma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+                        if constexpr (CG == 2)
+                            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+                        else
+                            umma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
                     }
-                    umma_commit(&empty[stage]);
+                    if constexpr (CG == 2)
+                        umma_commit_pair(&empty[stage], 0x3);
+                    else
+                        umma_commit(&empty[stage]);
                     if (++stage == STAGES) {
                         stage = 0;
                         phase ^= 1u;
                     }
                 }
-                if (ok) umma_commit(&tfull[acc]);
+                if (ok) {
+                    if constexpr (CG == 2)
+                        umma_commit_pair(&tfull[acc], 0x3);
+                    else
+                        umma_commit(&tfull[acc]);
+                }
             }
             // All issued UMMAs must finish before TMEM is released.
-            umma_commit(drain);
+            if constexpr (CG == 2)
+                umma_commit_pair(drain, 0x1);
+            else
+                umma_commit(drain);
             mbar_wait_bounded(drain, 0, nullptr);
         }
     } else if (!skip && warp >= 2) {
@@ -266,10 +317,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         const EpiParams& e = p.epi;
         constexpr int CPW = BN / 64;  // 32-column chunks per warp
         int it = 0;
-        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
+        for (int tile = unit; tile < num_tiles; tile += nunits, ++it) {
             int mt, nt;
             tile_coords(tile, p.tiles_m, p.tiles_n, mt, nt);
-            const int m0 = mt * BM;
+            const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
             const int n0 = nt * p.bn_out;
             const int acc = it & 1;
             const int m = m0 + row;
@@ -430,15 +481,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 }
             }
             tc_fence_before();
-            mbar_arrive(&tempty[acc]);
+            if constexpr (CG == 2) {
+                // one arrival per CTA on the even CTA's barrier once all 8 epilogue warps are done
+                named_bar_sync(1, 256);
+                if (warp == 2 && lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[acc]), 0));
+            } else {
+                mbar_arrive(&tempty[acc]);
+            }
         }
     }
 
     __syncthreads();
+    if constexpr (CG == 2) cluster_sync();   // no remote arrival, load or UMMA is still in flight
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(tmem_base, TMEM_COLS);
+        if constexpr (CG == 2)
+            tmem_dealloc_pair(tmem_base, TMEM_COLS);
+        else
+            tmem_dealloc(tmem_base, TMEM_COLS);
     }
     if (threadIdx.x == 0 && *abort_flag && p.epi.sc != nullptr)
         latch_status(const_cast<DevScalars*>(p.epi.sc), BOM_ETIMEOUT);
@@ -482,17 +543,80 @@ static bool map_operand(CUtensorMap* map, const Operand& o, int64_t rows, int64_
     return make_map(map, o.ptr, K, rows, o.ld, 64, rows_box);
 }
 
-template <bool A_MN, bool B_MN, int EPI>
-static int launch_inst(const Params& p, int grid, cudaStream_t stream) {
-    static bool attr_set = false;
-    auto k = gemm_kernel<A_MN, B_MN, EPI>;
-    if (!attr_set) {
-        if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES) != cudaSuccess)
+template <int CG, bool A_MN, bool B_MN, int EPI>
+static int launch_inst(const Params& p, cudaStream_t stream) {
+    using C = Cfg<CG>;
+    auto k = gemm_kernel<CG, A_MN, B_MN, EPI>;
+    // Resident tile walkers: CTAs (CG = 1) or CTA pairs (CG = 2) that fit at once.
+    static int max_units = 0;
+    if (max_units == 0) {
+        if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) != cudaSuccess)
             return BOM_ECUDA;
-        attr_set = true;
+        if constexpr (CG == 2) {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(static_cast<unsigned>(device_sm_count() & ~1));
+            cfg.blockDim = dim3(NUM_THREADS);
+            cfg.dynamicSmemBytes = C::SMEM;
+            cudaLaunchAttribute at;
+            at.id = cudaLaunchAttributeClusterDimension;
+            at.val.clusterDim.x = 2;
+            at.val.clusterDim.y = 1;
+            at.val.clusterDim.z = 1;
+            cfg.attrs = &at;
+            cfg.numAttrs = 1;
+            int n = 0;
+            if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess || n < 1) {
+                cudaGetLastError();
+                n = device_sm_count() / 2;
+            }
+            max_units = n;
+        } else {
+            max_units = device_sm_count();
+        }
     }
-    k<<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(p); count_launch();
+    const int tiles = p.tiles_m * p.tiles_n;
+    const int units = tiles < max_units ? tiles : max_units;
+    if constexpr (CG == 2) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(static_cast<unsigned>(2 * units));
+        cfg.blockDim = dim3(NUM_THREADS);
+        cfg.dynamicSmemBytes = C::SMEM;
+        cfg.stream = stream;
+        cudaLaunchAttribute at;
+        at.id = cudaLaunchAttributeClusterDimension;
+        at.val.clusterDim.x = 2;
+        at.val.clusterDim.y = 1;
+        at.val.clusterDim.z = 1;
+        cfg.attrs = &at;
+        cfg.numAttrs = 1;
+        if (cudaLaunchKernelEx(&cfg, k, p) != cudaSuccess) return BOM_ECUDA;
+    } else {
+        k<<<units, NUM_THREADS, C::SMEM, stream>>>(p);
+    }
+    count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+template <int CG>
+static int dispatch(const Params& p, int epi_kind, bool a_mn, bool b_mn, bool dual_b, cudaStream_t stream) {
+    switch (epi_kind) {
+        case EPI_LINEAR:
+            if (!a_mn && !b_mn) return launch_inst<CG, false, false, EPI_LINEAR>(p, stream);
+            if (!a_mn && b_mn) return launch_inst<CG, false, true, EPI_LINEAR>(p, stream);
+            if (a_mn && b_mn) return launch_inst<CG, true, true, EPI_LINEAR>(p, stream);
+            return launch_inst<CG, true, false, EPI_LINEAR>(p, stream);
+        case EPI_LOGITS:
+            if (a_mn || b_mn) return BOM_ENOTSUP;
+            return launch_inst<CG, false, false, EPI_LOGITS>(p, stream);
+        case EPI_SWIGLU_FWD:
+            if (a_mn || b_mn || !dual_b) return BOM_ENOTSUP;
+            return launch_inst<CG, false, false, EPI_SWIGLU_FWD>(p, stream);
+        case EPI_SWIGLU_BWD:
+            if (a_mn || !b_mn) return BOM_ENOTSUP;
+            return launch_inst<CG, false, true, EPI_SWIGLU_BWD>(p, stream);
+        default:
+            return BOM_EINVAL;
+    }
 }
 
 }  // namespace tc
@@ -515,9 +639,12 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     if (g.M <= 0 || g.N <= 0) return BOM_OK;
     if (g.M > INT32_MAX / 2 || g.N > INT32_MAX / 2) return BOM_ENOTSUP;
     if (g.epi.in_f32) return BOM_ENOTSUP;   // epilogue operands are bf16 on this engine
+    // CTA pairs (256-row tiles) whenever there is more than one 128-row tile.
+    const int cg = g.M > BM ? 2 : 1;
     Params p;
     memset(&p, 0, sizeof(p));
     const bool a_mn = g.A[0].mn_major, b_mn = g.B[0].mn_major;
+    const uint32_t b_rows = (cg == 2 || g.dual_b) ? 128 : 256;   // B rows one CTA loads per stage
     for (int s = 0; s < g.nseg; ++s) {
         if (g.A[s].mn_major != a_mn || g.B[s].mn_major != b_mn) return BOM_ENOTSUP;
         p.kb[s] = static_cast<int>((g.K[s] + BK - 1) / BK);
@@ -527,7 +654,7 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
             if (b_mn || g.nseg != 1) return BOM_ENOTSUP;
             if (!map_operand(&p.mapB[0], g.B[0], g.N, g.K[0], 128)) return BOM_ENOTSUP;
             if (!map_operand(&p.mapB[1], g.B[1], g.N, g.K[0], 128)) return BOM_ENOTSUP;
-        } else if (!map_operand(&p.mapB[s], g.B[s], g.N, g.K[s], BN)) {
+        } else if (!map_operand(&p.mapB[s], g.B[s], g.N, g.K[s], b_rows)) {
             return BOM_ENOTSUP;
         }
     }
@@ -536,30 +663,11 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     p.nseg = g.nseg;
     p.dual_b = g.dual_b ? 1 : 0;
     p.bn_out = g.dual_b ? 128 : BN;
-    p.tiles_m = static_cast<int>((g.M + BM - 1) / BM);
+    p.tiles_m = static_cast<int>((g.M + BM * cg - 1) / (BM * cg));
     p.tiles_n = static_cast<int>((g.N + p.bn_out - 1) / p.bn_out);
     p.epi = g.epi;
-    const int tiles = p.tiles_m * p.tiles_n;
-    const int grid = tiles < device_sm_count() ? tiles : device_sm_count();
-
-    switch (g.epi_kind) {
-        case EPI_LINEAR:
-            if (!a_mn && !b_mn) return launch_inst<false, false, EPI_LINEAR>(p, grid, stream);
-            if (!a_mn && b_mn) return launch_inst<false, true, EPI_LINEAR>(p, grid, stream);
-            if (a_mn && b_mn) return launch_inst<true, true, EPI_LINEAR>(p, grid, stream);
-            return launch_inst<true, false, EPI_LINEAR>(p, grid, stream);
-        case EPI_LOGITS:
-            if (a_mn || b_mn) return BOM_ENOTSUP;
-            return launch_inst<false, false, EPI_LOGITS>(p, grid, stream);
-        case EPI_SWIGLU_FWD:
-            if (a_mn || !g.dual_b) return BOM_ENOTSUP;
-            return launch_inst<false, false, EPI_SWIGLU_FWD>(p, grid, stream);
-        case EPI_SWIGLU_BWD:
-            if (a_mn || !b_mn) return BOM_ENOTSUP;
-            return launch_inst<false, true, EPI_SWIGLU_BWD>(p, grid, stream);
-        default:
-            return BOM_EINVAL;
-    }
+    return cg == 2 ? dispatch<2>(p, g.epi_kind, a_mn, b_mn, g.dual_b, stream)
+                   : dispatch<1>(p, g.epi_kind, a_mn, b_mn, g.dual_b, stream);
 }
 
 }  // namespace bom
