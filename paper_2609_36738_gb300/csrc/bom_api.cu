@@ -71,6 +71,8 @@ struct bom_handle {
     void* dG = nullptr;
     void* dU = nullptr;
     void* dx_in = nullptr;   // caller buffer for the cotangent of X (bom_set_input_grad)
+    float* splitk = nullptr; // fp32 partial tiles of split-K GEMMs
+    int64_t splitk_elems = 0;
     int64_t last_n = 0;
     // tracing: one event pair per launch of the current step
     struct TraceRec {
@@ -172,7 +174,7 @@ size_t carve(bom_handle* h, char* base) {
     h->stats = static_cast<float*>(c.take(n * h->ntiles * 8));
     h->lse = static_cast<float*>(c.take(n * 4));
     h->ce = static_cast<float*>(c.take(n * 4));
-    h->colpart = static_cast<float*>(c.take(row_blocks(n) * V * 4));
+    h->colpart = static_cast<float*>(c.take(resid_blocks(n) * V * 4));
     h->s = static_cast<float*>(c.take(V * 4));
     h->qhat = static_cast<float*>(c.take(V * 4));
     h->cvec = static_cast<float*>(c.take(h->d_model * 4));
@@ -184,6 +186,13 @@ size_t carve(bom_handle* h, char* base) {
     if (h->max_ffn > 0) {
         h->dG = c.take(n * h->max_ffn * e);
         h->dU = c.take(n * h->max_ffn * e);
+    }
+    if (h->bf16) {
+        const int64_t rows = n > V ? n : V;
+        const int64_t cols = h->max_width > h->max_ffn ? h->max_width : h->max_ffn;
+        const int64_t cap = int64_t(32) << 20;   // 128 MB of fp32 partials at most
+        h->splitk_elems = 8 * rows * cols < cap ? 8 * rows * cols : cap;
+        h->splitk = static_cast<float*>(c.take(h->splitk_elems * 4));
     }
     return c.off + 256;
 }
@@ -225,6 +234,10 @@ const char* gemm_name(const GemmDesc& g, bool bf16) {
 int run_gemm(bom_handle* h, GemmDesc& g, cudaStream_t s) {
     g.epi.sc = h->sc;
     g.epi.in_f32 = h->bf16 ? 0 : 1;
+    if (h->bf16 && g.epi_kind == EPI_LINEAR) {
+        g.splitk_ws = h->splitk;
+        g.splitk_ws_elems = h->splitk_elems;
+    }
     double k = 0;
     for (int i = 0; i < g.nseg; ++i) k += static_cast<double>(g.K[i]);
     const double n_mma = g.dual_b ? 2.0 * g.N : static_cast<double>(g.N);
@@ -449,11 +462,11 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                launch_row_lse(h->Z, cf32, h->ldz, n, V, h->stats, h->ntiles, labels, cfg.ignore_index, h->lse,
                               h->ce, h->sc, s));
     // residual pass: reads and rewrites Z once, writes the column partial sums
-    BOM_TRACED("residual", 0, 2.0 * h->esz * n * h->ldz + 4.0 * row_blocks(n) * V + 8.0 * n,
+    BOM_TRACED("residual", 0, 2.0 * h->esz * n * h->ldz + 4.0 * resid_blocks(n) * V + 8.0 * n,
                launch_residual(h->Z, cf32, h->ldz, n, V, h->lse, labels, cfg.ignore_index, h->colpart, h->sc, s));
     const float inv_bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(cfg.beta1), static_cast<double>(t))));
-    BOM_TRACED("finish_sq", 0, 4.0 * row_blocks(n) * V + 20.0 * V,
-               launch_finish_sq(h->colpart, row_blocks(n), V, cfg.beta1, inv_bc1, q, h->s, h->qhat, h->sc, s));
+    BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 20.0 * V,
+               launch_finish_sq(h->colpart, resid_blocks(n), V, cfg.beta1, inv_bc1, q, h->s, h->qhat, h->sc, s));
     BOM_TRACED("scalars", 0, 4.0 * (n + V), launch_scalars(h->ce, n, h->s, V, h->sc, s));
     // c = colsum_{I_t}(H) and w = W^T qhat (the rank-1 / broadcast factors of the reprojection)
     BOM_TRACED("colsum", 2.0 * n * dm, h->esz * n * dm,

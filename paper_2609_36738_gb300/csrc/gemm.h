@@ -30,6 +30,11 @@ struct GemmDesc {
     bool dual_b = false;
     int epi_kind = EPI_LINEAR;
     EpiParams epi = {};
+    // Optional fp32 scratch for split-K (EPI_LINEAR only): when the output has
+    // too few tiles to fill the GPU, the K range is split, fp32 partial tiles go
+    // here and a fixed-order reduction applies the epilogue.
+    float* splitk_ws = nullptr;
+    int64_t splitk_ws_elems = 0;
 };
 
 // Returns BOM_OK or an error status (BOM_ENOTSUP for unsupported layouts,

@@ -15,6 +15,7 @@
 //              the mainloop of tile i+1.
 // Every mbarrier wait is bounded; a wait that runs out latches BOM_ETIMEOUT,
 // all roles unwind, in-flight TMA loads and UMMAs are drained, TMEM is freed.
+#include <cmath>
 #include <cstdio>
 #include <mutex>
 
@@ -43,6 +44,9 @@ struct Params {
     int tiles_m, tiles_n;
     int dual_b;
     int bn_out;
+    int ksplit;            // K ranges per output tile (1: no split)
+    int kb_split;          // k-blocks per K range
+    int64_t split_bytes;   // byte distance between the fp32 partial slices of e.out
     EpiParams epi;
 };
 
@@ -184,6 +188,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
     const bool skip = *skip_flag != 0;
 
     const int num_tiles = p.tiles_m * p.tiles_n;
+    const int num_work = num_tiles * p.ksplit;   // (tile, K-split) work units
     const int kb_total = p.kb[0] + (p.nseg > 1 ? p.kb[1] : 0);
 
     if (!skip && warp == 0) {
@@ -193,14 +198,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_phase = 0;
             bool ok = true;
-            for (int tile = unit; ok && tile < num_tiles; tile += nunits) {
+            for (int w = unit; ok && w < num_work; w += nunits) {
+                const int tile = w / p.ksplit;
+                const int sp = w - tile * p.ksplit;
                 int mt, nt;
                 tile_coords(tile, p.tiles_m, p.tiles_n, mt, nt);
                 const int m_own = mt * C::TILE_M + static_cast<int>(rank) * BM;
                 const int n0 = nt * p.bn_out;
                 const int n_own = n0 + (CG == 2 && !p.dual_b ? static_cast<int>(rank) * C::B_ROWS : 0);
-                for (int seg = 0; ok && seg < p.nseg; ++seg) {
-                    for (int kb = 0; kb < p.kb[seg]; ++kb) {
+                const int g0 = sp * p.kb_split;
+                const int g1 = min(g0 + p.kb_split, kb_total);
+                {
+                    for (int gk = g0; gk < g1; ++gk) {
+                        const int seg = gk < p.kb[0] ? 0 : 1;
+                        const int kb = seg == 0 ? gk : gk - p.kb[0];
                         if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag)) {
                             ok = false;
                             break;
@@ -258,13 +269,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             uint32_t phase = 0;
             bool ok = true;
             int it = 0;
-            for (int tile = unit; ok && tile < num_tiles; tile += nunits, ++it) {
+            for (int w = unit; ok && w < num_work; w += nunits, ++it) {
                 const int acc = it & 1;
                 const uint32_t aph = (it >> 1) & 1;
+                const int sp = w % p.ksplit;
+                const int nk = min(p.kb_split, kb_total - sp * p.kb_split);
                 if (!mbar_wait_bounded(&tempty[acc], aph ^ 1u, abort_flag)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-                for (int kb = 0; kb < kb_total; ++kb) {
+                for (int kb = 0; kb < nk; ++kb) {
                     if (!mbar_wait_bounded(&full[stage], phase, abort_flag)) {
                         ok = false;
                         break;
@@ -317,7 +330,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         const EpiParams& e = p.epi;
         constexpr int CPW = BN / 64;  // 32-column chunks per warp
         int it = 0;
-        for (int tile = unit; tile < num_tiles; tile += nunits, ++it) {
+        for (int w = unit; w < num_work; w += nunits, ++it) {
+            const int tile = w / p.ksplit;
+            // split-K: each K range stores its raw fp32 tile into its own slice
+            void* const out_base = static_cast<char*>(e.out) + static_cast<int64_t>(w - tile * p.ksplit) * p.split_bytes;
             int mt, nt;
             tile_coords(tile, p.tiles_m, p.tiles_n, mt, nt);
             const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
@@ -393,7 +409,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(t[i]);
                         }
-                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
+                        store_row32(out_base, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
                     }
                 }
             } else if constexpr (EPI == EPI_LOGITS) {
@@ -574,8 +590,8 @@ static int launch_inst(const Params& p, cudaStream_t stream) {
             max_units = device_sm_count();
         }
     }
-    const int tiles = p.tiles_m * p.tiles_n;
-    const int units = tiles < max_units ? tiles : max_units;
+    const int work = p.tiles_m * p.tiles_n * p.ksplit;
+    const int units = work < max_units ? work : max_units;
     if constexpr (CG == 2) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(static_cast<unsigned>(2 * units));
@@ -595,6 +611,48 @@ static int launch_inst(const Params& p, cudaStream_t stream) {
     }
     count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+// Split-K reduction: sums the fp32 partial slices in a fixed order and applies
+// the GEMM's linear epilogue.
+__global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restrict__ ws, int S, int M, int N,
+                                                            const EpiParams e) {
+    if (e.sc != nullptr && e.sc->status != 0) return;
+    const int64_t total = static_cast<int64_t>(M) * N;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total; i += stride) {
+        float acc = 0.0f;
+        for (int s = 0; s < S; ++s) acc += ws[s * total + i];
+        const int m = static_cast<int>(i / N), n = static_cast<int>(i - static_cast<int64_t>(m) * N);
+        const EpiRow r = epi_row(e, m, M);
+        st_elem(e.out, static_cast<int64_t>(m) * e.ld_out + n, e.out_f32, epi_linear1(e, r, m, n, acc));
+    }
+}
+
+// Number of K ranges for a GEMM with `tiles` output tiles on `units` resident
+// tile walkers.  Split only when the waves would leave the GPU under 90% busy;
+// among 2..8 ranges (>= 16 k-blocks each, partials fitting the scratch) take
+// the best busy fraction less 1 point per range, if it beats no split by more
+// than 8 points.
+static int choose_split(int tiles, int units, int kb_total, int64_t mn, int64_t ws_elems) {
+    auto eff = [&](int s) {
+        const double w = static_cast<double>(tiles) * s;
+        const double waves = std::ceil(w / units);
+        return w / (waves * units);
+    };
+    const double e1 = eff(1);
+    if (e1 >= 0.9) return 1;
+    int best = 1;
+    double best_score = e1 - 0.01;
+    for (int s = 2; s <= 8; ++s) {
+        if (kb_total / s < 16 || static_cast<int64_t>(s) * mn > ws_elems) break;
+        const double e = eff(s);
+        if (e >= e1 + 0.08 && e - 0.01 * s > best_score) {
+            best = s;
+            best_score = e - 0.01 * s;
+        }
+    }
+    return best;
 }
 
 template <int CG>
@@ -666,8 +724,36 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     p.tiles_m = static_cast<int>((g.M + BM * cg - 1) / (BM * cg));
     p.tiles_n = static_cast<int>((g.N + p.bn_out - 1) / p.bn_out);
     p.epi = g.epi;
-    return cg == 2 ? dispatch<2>(p, g.epi_kind, a_mn, b_mn, g.dual_b, stream)
-                   : dispatch<1>(p, g.epi_kind, a_mn, b_mn, g.dual_b, stream);
+    const int kb_total = p.kb[0] + (p.nseg > 1 ? p.kb[1] : 0);
+    const int tiles = p.tiles_m * p.tiles_n;
+    const int units = cg == 2 ? device_sm_count() / 2 : device_sm_count();
+    int S = 1;
+    if (g.epi_kind == EPI_LINEAR && g.splitk_ws != nullptr)
+        S = choose_split(tiles, units, kb_total, static_cast<int64_t>(g.M) * g.N, g.splitk_ws_elems);
+    p.ksplit = S;
+    p.kb_split = S > 1 ? (kb_total + S - 1) / S : kb_total;
+    if (S > 1) {
+        // raw fp32 partial tiles into the scratch; the real epilogue runs in the reduction
+        p.ksplit = (kb_total + p.kb_split - 1) / p.kb_split;
+        EpiParams raw = {};
+        raw.alpha_const = 1.0f;
+        raw.beta_const = 0.0f;
+        raw.out = g.splitk_ws;
+        raw.ld_out = g.N;
+        raw.out_f32 = 1;
+        raw.sc = g.epi.sc;
+        p.epi = raw;
+        p.split_bytes = static_cast<int64_t>(g.M) * g.N * 4;
+    }
+    const int rc = cg == 2 ? dispatch<2>(p, g.epi_kind, a_mn, b_mn, g.dual_b, stream)
+                           : dispatch<1>(p, g.epi_kind, a_mn, b_mn, g.dual_b, stream);
+    if (rc != BOM_OK || S == 1) return rc;
+    const int64_t total = static_cast<int64_t>(g.M) * g.N;
+    int64_t blocks = (total + 255) / 256;
+    if (blocks > 8 * device_sm_count()) blocks = 8 * device_sm_count();
+    splitk_reduce_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(g.splitk_ws, p.ksplit, p.M, p.N, g.epi);
+    count_launch();
+    return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }
 
 }  // namespace bom

@@ -14,6 +14,10 @@ constexpr int kRowBlock = 128;
 
 inline int64_t row_blocks(int64_t n) { return (n + kRowBlock - 1) / kRowBlock; }
 
+// Row-block height of the residual pass (its column partial sums feed s_t).
+constexpr int kResidRows = 32;
+inline int64_t resid_blocks(int64_t n) { return (n + kResidRows - 1) / kResidRows; }
+
 // Counts N_t, checks every label, latches BOM_ELABEL / BOM_EEMPTY and writes
 // the cotangent coefficients of the three passes into sc.
 void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda,

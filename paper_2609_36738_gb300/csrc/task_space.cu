@@ -25,6 +25,34 @@ __device__ __forceinline__ int warp_sum_i(int v) {
     return v;
 }
 
+// Sum over the nblocks rows of part[nblocks, ncols] for 32 consecutive columns
+// per 256-thread block: warp w adds rows w, w+8, ..., then warp 0 adds the 8
+// warp sums in order.  Fixed order for fixed sizes (deterministic); the result
+// is valid in warp 0 (lane l holds column `col` of lane l).
+__device__ __forceinline__ float fixed_order_column_sum(const float* __restrict__ part, int64_t nblocks,
+                                                        int64_t ncols, int64_t col, float (*red)[33]) {
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    float a0 = 0.0f, a1 = 0.0f, a2 = 0.0f, a3 = 0.0f;
+    if (col < ncols) {
+        int64_t b = w;
+        for (; b + 24 < nblocks; b += 32) {
+            a0 += part[b * ncols + col];
+            a1 += part[(b + 8) * ncols + col];
+            a2 += part[(b + 16) * ncols + col];
+            a3 += part[(b + 24) * ncols + col];
+        }
+        for (; b < nblocks; b += 8) a0 += part[b * ncols + col];
+    }
+    red[w][l] = (a0 + a1) + (a2 + a3);
+    __syncthreads();
+    float r = 0.0f;
+    if (w == 0) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) r += red[k][l];
+    }
+    return r;
+}
+
 // Deterministic block sum of a float (fixed tree for a fixed block size).
 template <int NT>
 __device__ float block_sum(float v, float* red) {
@@ -137,8 +165,8 @@ __global__ void __launch_bounds__(256) residual_kernel(T* __restrict__ Z, int64_
                                                        float* __restrict__ colpart, const DevScalars* sc) {
     if (sc->status != 0) return;
     const int64_t col0 = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) * VEC;
-    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kRowBlock;
-    const int64_t r1 = min(r0 + kRowBlock, n);
+    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kResidRows;
+    const int64_t r1 = min(r0 + kResidRows, n);
     float csum[VEC];
 #pragma unroll
     for (int k = 0; k < VEC; ++k) csum[k] = 0.0f;
@@ -201,14 +229,15 @@ __global__ void __launch_bounds__(256) residual_kernel(T* __restrict__ Z, int64_
     }
 }
 
-__global__ void finish_sq_kernel(const float* __restrict__ colpart, int64_t nblocks, int64_t V, float beta1,
-                                 float inv_bc1, float* __restrict__ q, float* __restrict__ s_out,
-                                 float* __restrict__ qhat, const DevScalars* sc) {
+__global__ void __launch_bounds__(256) finish_sq_kernel(const float* __restrict__ colpart, int64_t nblocks, int64_t V,
+                                                        float beta1, float inv_bc1, float* __restrict__ q,
+                                                        float* __restrict__ s_out, float* __restrict__ qhat,
+                                                        const DevScalars* sc) {
+    __shared__ float red[8][33];
     if (sc->status != 0) return;
-    const int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-    if (j >= V) return;
-    float acc = 0.0f;
-    for (int64_t b = 0; b < nblocks; ++b) acc += colpart[b * V + j];
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + (threadIdx.x & 31);
+    const float acc = fixed_order_column_sum(colpart, nblocks, V, j, red);
+    if (threadIdx.x >= 32 || j >= V) return;
     const float s = acc * sc->inv_nt;
     const float qn = beta1 * q[j] + (1.0f - beta1) * s;
     q[j] = qn;
@@ -305,14 +334,14 @@ __global__ void __launch_bounds__(256) colsum_part_kernel(const T* __restrict__ 
     }
 }
 
-__global__ void colsum_finish_kernel(const float* __restrict__ part, int64_t nblocks, int64_t d, float scale,
-                                     void* __restrict__ out, int out_f32, const DevScalars* sc) {
+__global__ void __launch_bounds__(256) colsum_finish_kernel(const float* __restrict__ part, int64_t nblocks,
+                                                            int64_t d, float scale, void* __restrict__ out,
+                                                            int out_f32, const DevScalars* sc) {
+    __shared__ float red[8][33];
     if (sc->status != 0) return;
-    const int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-    if (j >= d) return;
-    float a = 0.0f;
-    for (int64_t b = 0; b < nblocks; ++b) a += part[b * d + j];
-    st_elem(out, j, out_f32, a * scale);
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + (threadIdx.x & 31);
+    const float a = fixed_order_column_sum(part, nblocks, d, j, red);
+    if (threadIdx.x < 32 && j < d) st_elem(out, j, out_f32, a * scale);
 }
 
 __global__ void axpby_kernel(const float* __restrict__ s, const float* __restrict__ qh, float a, float b, int64_t V,
@@ -347,11 +376,11 @@ void launch_row_lse(const void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V,
 void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* lse, const int32_t* labels,
                      int32_t ignore, float* colpart, const DevScalars* sc, cudaStream_t s) {
     if (z_f32) {
-        dim3 grid(cdiv(ldz, 256 * 4), static_cast<unsigned>(row_blocks(n)));
+        dim3 grid(cdiv(ldz, 256 * 4), static_cast<unsigned>(resid_blocks(n)));
         residual_kernel<float, 4><<<grid, 256, 0, s>>>(static_cast<float*>(Z), ldz, n, V, lse, labels, ignore,
                                                        colpart, sc); count_launch();
     } else {
-        dim3 grid(cdiv(ldz, 256 * 8), static_cast<unsigned>(row_blocks(n)));
+        dim3 grid(cdiv(ldz, 256 * 8), static_cast<unsigned>(resid_blocks(n)));
         residual_kernel<__nv_bfloat16, 8><<<grid, 256, 0, s>>>(static_cast<__nv_bfloat16*>(Z), ldz, n, V, lse,
                                                                labels, ignore, colpart, sc); count_launch();
     }
@@ -359,7 +388,7 @@ void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, cons
 
 void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float inv_bc1, float* q,
                       float* s_out, float* qhat, DevScalars* sc, cudaStream_t s) {
-    finish_sq_kernel<<<cdiv(V, 256), 256, 0, s>>>(colpart, nblocks, V, beta1, inv_bc1, q, s_out, qhat, sc); count_launch();
+    finish_sq_kernel<<<cdiv(V, 32), 256, 0, s>>>(colpart, nblocks, V, beta1, inv_bc1, q, s_out, qhat, sc); count_launch();
 }
 
 void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, DevScalars* sc, cudaStream_t s) {
@@ -380,7 +409,7 @@ void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, 
                                                                labels, ignore, wvec, part, sc);
     }
     count_launch();
-    colsum_finish_kernel<<<cdiv(d, 256), 256, 0, s>>>(part, nb, d, scale, out, out_f32, sc); count_launch();
+    colsum_finish_kernel<<<cdiv(d, 32), 256, 0, s>>>(part, nb, d, scale, out, out_f32, sc); count_launch();
 }
 
 void launch_axpby(const float* s_vec, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,

@@ -210,8 +210,13 @@ TINY_RAGGED_F32 = Workload("tiny_ragged_f32", 37, 29, (Layer(LINEAR_GELU, 29, 45
                                                        Layer(LINEAR, 45, 33, True)),
                            7, True, "f32", "uniform", steps=3, ignore_frac=0.1)
 
+# Few output tiles and a long contraction in the head's input-side backward
+# (256 rows x 128 columns, K = 8192): exercises the split-K path of the GEMMs.
+LM_HEAD_WIDE = Workload("lm_head_wide", 256, 128, (), 8192, False, "bf16", "zipf",
+                        head_init="normal002", ignore_frac=0.05)
+
 WORKLOADS = {w.name: w for w in (TINY_MLP_F32, VISION_HEAD_BF16, LM_HEAD_BF16, LM_MLP_BF16,
-                                  LM_HEAD_SMALL, LM_MLP_SMALL, VISION_SMALL, TINY_RAGGED_F32)}
+                                  LM_HEAD_SMALL, LM_MLP_SMALL, VISION_SMALL, TINY_RAGGED_F32, LM_HEAD_WIDE)}
 
 
 # --------------------------------------------------------------------------

@@ -143,7 +143,7 @@ def test_deterministic_reruns():
         assert torch.equal(ga, gb)
 
 
-@pytest.mark.parametrize("name", ["lm_head_small", "lm_mlp_small", "tiny_ragged_f32"])
+@pytest.mark.parametrize("name", ["lm_head_small", "lm_mlp_small", "tiny_ragged_f32", "lm_head_wide"])
 def test_input_cotangent(name):
     """bom_set_input_grad: the cotangent of X (for the head-only block this is
     dH, the input-side half of the head backward)."""
