@@ -304,6 +304,7 @@ def main():
         roof = {"bound": "tensor", "kernel": name, "achieved": achieved, "peak": peaks["bf16_tflops_sustained"],
                 "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops_sustained"],
                 "peak_source": f"{peak_src} (sustained bf16; kernel timed inside a long step)",
+                "frac_of_burst_peak": achieved / peaks["bf16_tflops"],
                 "flops_per_launch": fl / cnt, "launches": cnt, "avg_launch_ms": ms / cnt,
                 "share_of_device_time": ms / total_dev}
     else:
