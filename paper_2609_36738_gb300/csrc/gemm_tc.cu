@@ -630,7 +630,8 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restr
 }
 
 // Number of K ranges for a GEMM with `tiles` output tiles on `units` resident
-// tile walkers.  Split only when the waves would leave the GPU under 90% busy;
+// tile walkers.  Split only when the waves would leave the GPU under 75% busy
+// (the fp32 partials cost more than milder quantisation does);
 // among 2..8 ranges (>= 16 k-blocks each, partials fitting the scratch) take
 // the best busy fraction less 1 point per range, if it beats no split by more
 // than 8 points.
@@ -641,7 +642,7 @@ static int choose_split(int tiles, int units, int kb_total, int64_t mn, int64_t 
         return w / (waves * units);
     };
     const double e1 = eff(1);
-    if (e1 >= 0.9) return 1;
+    if (e1 >= 0.75) return 1;
     int best = 1;
     double best_score = e1 - 0.01;
     for (int s = 2; s <= 8; ++s) {

@@ -157,12 +157,15 @@ __global__ void row_lse_kernel(const void* __restrict__ Z, int z_f32, int64_t ld
     }
 }
 
-// Block: 256 threads x VEC consecutive columns; grid.y: row blocks.
+// Block: 256 threads x VEC consecutive columns (one 16-byte word each) of
+// kResidRows rows.  The words of UNROLL rows are loaded before any is used and
+// stay packed until then, so a thread keeps 128 bytes in flight with few
+// registers and three blocks fit on an SM.
 template <typename T, int VEC>
-__global__ void __launch_bounds__(256) residual_kernel(T* __restrict__ Z, int64_t ldz, int64_t n, int64_t V,
-                                                       const float* __restrict__ lse,
-                                                       const int32_t* __restrict__ labels, int32_t ignore,
-                                                       float* __restrict__ colpart, const DevScalars* sc) {
+__global__ void __launch_bounds__(256, 3) residual_kernel(T* __restrict__ Z, int64_t ldz, int64_t n, int64_t V,
+                                                          const float* __restrict__ lse,
+                                                          const int32_t* __restrict__ labels, int32_t ignore,
+                                                          float* __restrict__ colpart, const DevScalars* sc) {
     if (sc->status != 0) return;
     const int64_t col0 = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) * VEC;
     const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kResidRows;
@@ -173,26 +176,10 @@ __global__ void __launch_bounds__(256) residual_kernel(T* __restrict__ Z, int64_
     if (col0 < ldz) {
         constexpr int UNROLL = 8;
         for (int64_t rb = r0; rb < r1; rb += UNROLL) {
-            float zv[UNROLL][VEC];
+            uint4 raw[UNROLL];
 #pragma unroll
-            for (int u = 0; u < UNROLL; ++u) {
-                const int64_t r = rb + u;
-                if (r < r1) {
-                    const T* src = Z + r * ldz + col0;
-                    if constexpr (sizeof(T) == 2) {
-                        const uint4 w = *reinterpret_cast<const uint4*>(src);
-                        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            zv[u][2 * j] = __uint_as_float(ws[j] << 16);
-                            zv[u][2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
-                        }
-                    } else {
-                        const float4 f = *reinterpret_cast<const float4*>(src);
-                        zv[u][0] = f.x; zv[u][1] = f.y; zv[u][2] = f.z; zv[u][3] = f.w;
-                    }
-                }
-            }
+            for (int u = 0; u < UNROLL; ++u)
+                if (rb + u < r1) raw[u] = *reinterpret_cast<const uint4*>(Z + (rb + u) * ldz + col0);
 #pragma unroll
             for (int u = 0; u < UNROLL; ++u) {
                 const int64_t r = rb + u;
@@ -203,13 +190,25 @@ __global__ void __launch_bounds__(256) residual_kernel(T* __restrict__ Z, int64_
                 // bf16 logits: exp2 of a pre-scaled argument (the result is
                 // stored in bf16); fp32 logits keep the accurate expf.
                 const float Ls = L * 1.4426950408889634f;
+                const uint32_t ws[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
+                float z[VEC];
+                if constexpr (sizeof(T) == 2) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        z[2 * j] = __uint_as_float(ws[j] << 16);
+                        z[2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) z[j] = __uint_as_float(ws[j]);
+                }
                 float rv[VEC];
 #pragma unroll
                 for (int k = 0; k < VEC; ++k) {
                     const int64_t c = col0 + k;
                     float p = 0.0f;
                     if (valid && c < V)
-                        p = (sizeof(T) == 2) ? exp2f(fmaf(zv[u][k], 1.4426950408889634f, -Ls)) : expf(zv[u][k] - L);
+                        p = (sizeof(T) == 2) ? exp2f(fmaf(z[k], 1.4426950408889634f, -Ls)) : expf(z[k] - L);
                     if (valid && c == y) p -= 1.0f;
                     rv[k] = p;
                     csum[k] += p;
@@ -266,10 +265,10 @@ __global__ void __launch_bounds__(1024) scalars_kernel(const float* __restrict__
 // columns, the 8 warps take interleaved rows, and the 8 warp sums are added
 // in a fixed order in shared memory (deterministic).
 template <typename T>
-__global__ void __launch_bounds__(256) colsum_part_kernel(const T* __restrict__ X, int64_t ldx, int64_t n, int64_t d,
-                                                          const int32_t* __restrict__ labels, int32_t ignore,
-                                                          const float* __restrict__ wvec, float* __restrict__ part,
-                                                          const DevScalars* sc) {
+__global__ void __launch_bounds__(256, 2) colsum_part_kernel(const T* __restrict__ X, int64_t ldx, int64_t n,
+                                                             int64_t d, const int32_t* __restrict__ labels,
+                                                             int32_t ignore, const float* __restrict__ wvec,
+                                                             float* __restrict__ part, const DevScalars* sc) {
     constexpr int VEC = 16 / sizeof(T);
     __shared__ float red[8][32 * VEC];
     if (sc->status != 0) return;
@@ -281,16 +280,15 @@ __global__ void __launch_bounds__(256) colsum_part_kernel(const T* __restrict__ 
 #pragma unroll
     for (int k = 0; k < VEC; ++k) acc[k] = 0.0f;
     const bool vec = (c0 + VEC <= d) && ((ldx % VEC) == 0);
-    constexpr int UNROLL = 4;
+    constexpr int UNROLL = 8;
     for (int64_t rb = r0 + w; rb < r1; rb += 8 * UNROLL) {
-        float x[UNROLL][VEC];
+        uint4 raw[UNROLL];
         float wt[UNROLL];
 #pragma unroll
         for (int u = 0; u < UNROLL; ++u) {
             const int64_t r = rb + 8 * u;
             wt[u] = 0.0f;
-#pragma unroll
-            for (int k = 0; k < VEC; ++k) x[u][k] = 0.0f;
+            raw[u] = make_uint4(0u, 0u, 0u, 0u);
             if (r >= r1 || c0 >= d) continue;
             float wr = 1.0f;
             if (labels) wr = (labels[r] != ignore) ? 1.0f : 0.0f;
@@ -298,28 +296,33 @@ __global__ void __launch_bounds__(256) colsum_part_kernel(const T* __restrict__ 
             wt[u] = wr;
             const T* src = X + r * ldx + c0;
             if (vec) {
-                const uint4 q = *reinterpret_cast<const uint4*>(src);
-                if constexpr (sizeof(T) == 2) {
-                    const uint32_t ws[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        x[u][2 * j] = __uint_as_float(ws[j] << 16);
-                        x[u][2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
-                    }
-                } else {
-                    x[u][0] = __uint_as_float(q.x); x[u][1] = __uint_as_float(q.y);
-                    x[u][2] = __uint_as_float(q.z); x[u][3] = __uint_as_float(q.w);
-                }
+                raw[u] = *reinterpret_cast<const uint4*>(src);
             } else {
+                uint32_t q[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
-                for (int k = 0; k < VEC; ++k)
-                    if (c0 + k < d) x[u][k] = ld_elem(src, k, sizeof(T) == 4);
+                for (int k = 0; k < VEC; ++k) {
+                    if (c0 + k >= d) continue;
+                    if constexpr (sizeof(T) == 2)
+                        q[k >> 1] |= static_cast<uint32_t>(reinterpret_cast<const uint16_t*>(src)[k]) << (16 * (k & 1));
+                    else
+                        q[k] = reinterpret_cast<const uint32_t*>(src)[k];
+                }
+                raw[u] = make_uint4(q[0], q[1], q[2], q[3]);
             }
         }
 #pragma unroll
-        for (int u = 0; u < UNROLL; ++u)
+        for (int u = 0; u < UNROLL; ++u) {
+            const uint32_t ws[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
 #pragma unroll
-            for (int k = 0; k < VEC; ++k) acc[k] = fmaf(wt[u], x[u][k], acc[k]);
+            for (int k = 0; k < VEC; ++k) {
+                float x;
+                if constexpr (sizeof(T) == 2)
+                    x = __uint_as_float((k & 1) ? (ws[k >> 1] & 0xFFFF0000u) : (ws[k >> 1] << 16));
+                else
+                    x = __uint_as_float(ws[k]);
+                acc[k] = fmaf(wt[u], x, acc[k]);
+            }
+        }
     }
 #pragma unroll
     for (int k = 0; k < VEC; ++k) red[w][l * VEC + k] = acc[k];
