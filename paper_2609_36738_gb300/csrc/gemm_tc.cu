@@ -100,6 +100,88 @@ __device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[NW], int slot, fl
     }
 }
 
+// ---------------------------------------------------------------- staged epilogue I/O
+// A warp owns 32 consecutive output rows (one per lane).  Reading or writing
+// "its row" directly makes every warp instruction touch 32 different rows;
+// instead a 32 x 32 bf16 block goes through a per-warp shared-memory buffer:
+// global accesses are coalesced (lane l covers row l/4 + 8i, 16-byte segment
+// l%4) and each lane then reads / writes its own row in shared memory.  The
+// 80-byte row pitch (64 data + 16 pad) keeps both access patterns at the
+// minimum number of shared-memory wavefronts.
+constexpr int kStgPitch = 80;
+constexpr int kStgBytes = 32 * kStgPitch;
+
+// Issues the coalesced loads of block (rows row0.., columns n..n+31) into w.
+__device__ __forceinline__ void stg_gather_issue(const void* base, int64_t ld, int row0, int M, int n, int N,
+                                                 uint4 (&w)[4]) {
+    const int lane = threadIdx.x & 31;
+    const int c = n + 8 * (lane & 3);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int r = row0 + (lane >> 2) + 8 * i;
+        const uint16_t* p = static_cast<const uint16_t*>(base) + static_cast<int64_t>(r) * ld + c;
+        if (r < M && c + 8 <= N) {
+            w[i] = __ldg(reinterpret_cast<const uint4*>(p));
+        } else {
+            uint32_t q[4] = {0u, 0u, 0u, 0u};
+            if (r < M)
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    if (c + k < N) q[k >> 1] |= static_cast<uint32_t>(p[k]) << (16 * (k & 1));
+            w[i] = make_uint4(q[0], q[1], q[2], q[3]);
+        }
+    }
+}
+// Puts the loaded block through the staging buffer; lane l receives row l.
+__device__ __forceinline__ void stg_gather_finish(uint8_t* stg, const uint4 (&w)[4], float (&v)[32]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        *reinterpret_cast<uint4*>(stg + ((lane >> 2) + 8 * i) * kStgPitch + (lane & 3) * 16) = w[i];
+    __syncwarp();
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint4 x = *reinterpret_cast<const uint4*>(stg + lane * kStgPitch + k * 16);
+        const uint32_t ws[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            v[8 * k + 2 * j] = __uint_as_float(ws[j] << 16);
+            v[8 * k + 2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
+        }
+    }
+    __syncwarp();
+}
+// Lane l contributes row l of a 32 x 32 block; the warp stores it coalesced as bf16.
+__device__ __forceinline__ void stg_scatter(void* base, int64_t ld, int row0, int M, int n, int N, uint8_t* stg,
+                                            const float (&v)[32]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        *reinterpret_cast<uint4*>(stg + lane * kStgPitch + k * 16) =
+            make_uint4(pack_bf16x2(v[8 * k], v[8 * k + 1]), pack_bf16x2(v[8 * k + 2], v[8 * k + 3]),
+                       pack_bf16x2(v[8 * k + 4], v[8 * k + 5]), pack_bf16x2(v[8 * k + 6], v[8 * k + 7]));
+    __syncwarp();
+    const int c = n + 8 * (lane & 3);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int rl = (lane >> 2) + 8 * i;
+        const int r = row0 + rl;
+        const uint4 x = *reinterpret_cast<const uint4*>(stg + rl * kStgPitch + (lane & 3) * 16);
+        uint16_t* p = static_cast<uint16_t*>(base) + static_cast<int64_t>(r) * ld + c;
+        if (r < M) {
+            if (c + 8 <= N) {
+                *reinterpret_cast<uint4*>(p) = x;
+            } else {
+                const uint32_t ws[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    if (c + k < N) p[k] = static_cast<uint16_t>(ws[k >> 1] >> (16 * (k & 1)));
+            }
+        }
+    }
+    __syncwarp();
+}
+
 __device__ __forceinline__ float fast_exp(float x) { return exp2f(x * 1.4426950408889634f); }
 __device__ __forceinline__ float fast_sigmoid(float x) { return __frcp_rn(1.0f + fast_exp(-x)); }
 
@@ -112,30 +194,34 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Shared-memory pipeline of one CTA.  CG = 1: the CTA computes 128 x 256
-// tiles alone.  CG = 2: a CTA pair (cluster of 2) computes 256 x 256 tiles
-// with tcgen05 cta_group::2 UMMAs issued by the even CTA; each CTA stages its
-// own 128 rows of A and its half (128 rows) of B, so a stage is 32 KB and six
-// stages fit.
-template <int CG>
+// Shared-memory layout of one CTA.  CG = 1: the CTA computes 128 x 256 tiles
+// alone.  CG = 2: a CTA pair (cluster of 2) computes 256 x 256 tiles with
+// tcgen05 cta_group::2 UMMAs issued by the even CTA; each CTA stages its own
+// 128 rows of A and its half (128 rows) of B, so a stage is 32 KB.  Epilogues
+// that move several bf16 streams (logits, SwiGLU) take NBUF staging blocks per
+// epilogue warp and give up pipeline stages for them.
+template <int CG, int EPI>
 struct Cfg {
+    static constexpr int NBUF = EPI == EPI_SWIGLU_BWD ? 4 : EPI == EPI_SWIGLU_FWD ? 3 : EPI == EPI_LOGITS ? 1 : 0;
     static constexpr int B_ROWS = CG == 2 ? 128 : 256;
-    static constexpr int STAGES = CG == 2 ? 6 : 4;
+    static constexpr int STAGES = NBUF > 0 ? (CG == 2 ? 4 : 3) : (CG == 2 ? 6 : 4);
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
-    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + 1024 + 256;
+    static constexpr int STG_BYTES = 8 * NBUF * kStgBytes;
+    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 1024 + 256;
     static constexpr int TILE_M = BM * CG;
 };
 
 template <int CG, bool A_MN, bool B_MN, int EPI>
 __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_constant__ Params p) {
-    using C = Cfg<CG>;
+    using C = Cfg<CG, EPI>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sA = smem;
     uint8_t* sB = smem + STAGES * C::A_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + STAGES * C::B_BYTES);
+    uint8_t* stg_all = sB + STAGES * C::B_BYTES;   // epilogue staging blocks
+    uint64_t* bars = reinterpret_cast<uint64_t*>(stg_all + C::STG_BYTES);
     uint64_t* full = bars;
     uint64_t* empty = bars + STAGES;
     uint64_t* tfull = bars + 2 * STAGES;
@@ -352,8 +438,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const void* pb = EPI == EPI_SWIGLU_BWD ? e.aux2 : e.aux;
             const int64_t ra = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid);
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
-            if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
-            if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
+            const int row0 = m0 + q * 32;   // first of the warp's 32 rows
+            uint8_t* stg = stg_all + (warp - 2) * C::NBUF * kStgBytes;
+            if constexpr (EPI == EPI_SWIGLU_BWD) {
+                stg_gather_issue(e.aux, e.ld_aux, row0, p.M, n0 + 32 * c0, p.N, xa);
+                stg_gather_issue(e.aux2, e.ld_aux2, row0, p.M, n0 + 32 * c0, p.N, xb);
+            } else {
+                if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
+                if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
+            }
             if (kb_total > 0) {
                 if (!mbar_wait_bounded(&tfull[acc], (it >> 1) & 1, abort_flag)) break;
                 tc_fence_after();
@@ -427,11 +520,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] += t[i];
                     }
-                    if (!e.out_f32) {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = round_bf16(v[i]);
-                    }
-                    if (valid) store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
+                    for (int i = 0; i < 32; ++i) v[i] = round_bf16(v[i]);
+                    stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg, v);
                     float cm = -INFINITY;
 #pragma unroll
                     for (int i = 0; i < 32; ++i)
@@ -458,16 +549,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
                     tmem_load32(tbase + 128 + c * 32, u);
-                    if (valid) {
-                        store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, p.N, e.out2_f32, v);
-                        store_row32(e.out3, static_cast<int64_t>(m) * e.ld_out3, n, p.N, e.out2_f32, u);
+                    stg_scatter(e.out2, e.ld_out2, row0, p.M, n, p.N, stg + kStgBytes, v);
+                    stg_scatter(e.out3, e.ld_out3, row0, p.M, n, p.N, stg + 2 * kStgBytes, u);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const float g = round_bf16(v[i]);
-                            v[i] = g * fast_sigmoid(g) * round_bf16(u[i]);
-                        }
-                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
+                    for (int i = 0; i < 32; ++i) {
+                        const float g = round_bf16(v[i]);
+                        v[i] = g * fast_sigmoid(g) * round_bf16(u[i]);
                     }
+                    stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg, v);
                 }
             } else if constexpr (EPI == EPI_SWIGLU_BWD) {
                 float g[32], u[32];
@@ -477,23 +566,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
-                    if (valid) {
-                        unpack32_dyn(xa, 0, g);
-                        unpack32_dyn(xb, 0, u);
-                        if (j + 1 < CPW) {
-                            load_chunk_bf16(pa, ra, n + 32, p.N, xa, 0);
-                            load_chunk_bf16(pb, rb, n + 32, p.N, xb, 0);
-                        }
-                        float du[32];
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const float sg = fast_sigmoid(g[i]);
-                            du[i] = v[i] * g[i] * sg;
-                            v[i] = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
-                        }
-                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
-                        store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, p.N, e.out2_f32, du);
+                    stg_gather_finish(stg, xa, g);
+                    stg_gather_finish(stg + kStgBytes, xb, u);
+                    if (j + 1 < CPW) {
+                        stg_gather_issue(e.aux, e.ld_aux, row0, p.M, n + 32, p.N, xa);
+                        stg_gather_issue(e.aux2, e.ld_aux2, row0, p.M, n + 32, p.N, xb);
                     }
+                    float du[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const float sg = fast_sigmoid(g[i]);
+                        du[i] = v[i] * g[i] * sg;
+                        v[i] = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
+                    }
+                    stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg + 2 * kStgBytes, v);
+                    stg_scatter(e.out2, e.ld_out2, row0, p.M, n, p.N, stg + 3 * kStgBytes, du);
                 }
             }
             tc_fence_before();
@@ -561,7 +648,7 @@ static bool map_operand(CUtensorMap* map, const Operand& o, int64_t rows, int64_
 
 template <int CG, bool A_MN, bool B_MN, int EPI>
 static int launch_inst(const Params& p, cudaStream_t stream) {
-    using C = Cfg<CG>;
+    using C = Cfg<CG, EPI>;
     auto k = gemm_kernel<CG, A_MN, B_MN, EPI>;
     // Resident tile walkers: CTAs (CG = 1) or CTA pairs (CG = 2) that fit at once.
     static int max_units = 0;
