@@ -294,3 +294,28 @@ def mix_numerator(g, h, lam):
 def bom_update_gh(theta, g, h, v, lr, wd, lam, t, beta2=0.999, eps=1e-8):
     """Update from the separate supervised gradient g and reprojection h."""
     return bom_update(theta, mix_numerator(g, h, lam), v, lr, wd, t, beta2, eps)
+
+
+# --------------------------------------------------------------------------
+# Sampled head gradients (full-size checks where the full reverse pass is too
+# slow in fp64).  Same formulas as `backward` for the head, restricted to a
+# subset of output rows: with the L_mix logit cotangent
+#   dZ = N_t^-1 [(1 - lambda) R + lambda 1_{I_t} qhat^T],
+# the head weight gradient is dZ^T H and the head-input cotangent is dZ W.
+# --------------------------------------------------------------------------
+def mix_cotangent_rows(R, valid, qhat, n_t, lam, rows):
+    """Rows `rows` of dZ (Eq. mix-objective, differentiated in the logits)."""
+    rows = np.asarray(rows)
+    return ((1.0 - lam) * R[rows] + lam * valid[rows, None] * np.asarray(qhat)[None, :]) / n_t
+
+
+def head_weight_grad_rows(R, H, valid, qhat, n_t, lam, vocab_rows):
+    """Rows `vocab_rows` of the head weight gradient dZ^T H."""
+    vocab_rows = np.asarray(vocab_rows)
+    dZ_cols = ((1.0 - lam) * R[:, vocab_rows] + lam * valid[:, None] * np.asarray(qhat)[None, vocab_rows]) / n_t
+    return dZ_cols.T @ np.asarray(H, dtype=F64)
+
+
+def head_input_grad_rows(R, W, valid, qhat, n_t, lam, token_rows):
+    """Rows `token_rows` of the head-input cotangent dZ W."""
+    return mix_cotangent_rows(R, valid, qhat, n_t, lam, token_rows) @ np.asarray(W, dtype=F64)
