@@ -37,6 +37,11 @@ def host_f32(ptr: int, count: int) -> np.ndarray:
 rel_l2 = X.rel_l2
 
 
+def bf16_round(a: np.ndarray) -> np.ndarray:
+    """float64 values rounded to the nearest bf16 (through float32), as float64."""
+    return I.bf16_to_f64(I.bf16_bits(np.asarray(a, dtype=np.float32)))
+
+
 class GpuBom:
     """A handle plus device copies of a workload's parameters."""
 

@@ -139,7 +139,9 @@ def test_vision_head_twenty_steps_full_size():
     for t in range(1, wl.steps + 1):
         xb, y = I.make_batch(wl, seed=11, step=t)
         gout = gpu.step(xb, y, t)
-        oref = G.oracle_step(wl, p64, xb, y, q, t)
+        # both sides compute with bf16 copies of their own master weights
+        # (fp32 on the GPU, fp64 here): the bf16-autocast protocol of the paper
+        oref = G.oracle_step(wl, [G.bf16_round(p) for p in p64], xb, y, q, t)
         q = oref["q"]
         assert gout["stats"]["n_t"] == oref["n_t"]
         assert G.rel_l2(gout["q"], oref["q"]) < TOL

@@ -82,7 +82,9 @@ def test_multi_step_trajectory(name, steps):
     for t in range(1, steps + 1):
         x, y = I.make_batch(wl, seed=5, step=t)
         gout = gpu.step(x, y, t)
-        oref = G.oracle_step(wl, p64, x, y, q, t)
+        # bf16 workloads compute with bf16 copies of the master weights on both sides
+        pin = [G.bf16_round(p) for p in p64] if wl.dtype == "bf16" else p64
+        oref = G.oracle_step(wl, pin, x, y, q, t)
         q = oref["q"]
         _compare_step(wl, gout, oref, tol, False)
         for k in range(len(params)):
