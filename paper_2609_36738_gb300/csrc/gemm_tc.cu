@@ -200,9 +200,13 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
 // 128 rows of A and its half (128 rows) of B, so a stage is 32 KB.  Epilogues
 // that move several bf16 streams (logits, SwiGLU) take NBUF staging blocks per
 // epilogue warp and give up pipeline stages for them.
+// Logits epilogue with its output staged through shared memory (chosen when
+// the contraction is short and the epilogue, not the mainloop, sets the pace).
+constexpr int EPI_LOGITS_STG = 16;
+
 template <int CG, int EPI>
 struct Cfg {
-    static constexpr int NBUF = EPI == EPI_SWIGLU_BWD ? 4 : EPI == EPI_SWIGLU_FWD ? 3 : EPI == EPI_LOGITS ? 1 : 0;
+    static constexpr int NBUF = EPI == EPI_SWIGLU_FWD ? 3 : EPI == EPI_LOGITS_STG ? 1 : 0;
     static constexpr int B_ROWS = CG == 2 ? 128 : 256;
     static constexpr int STAGES = NBUF > 0 ? (CG == 2 ? 4 : 3) : (CG == 2 ? 6 : 4);
     static constexpr int A_BYTES = BM * BK * 2;
@@ -440,13 +444,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
             uint8_t* stg = stg_all + (warp - 2) * C::NBUF * kStgBytes;
-            if constexpr (EPI == EPI_SWIGLU_BWD) {
-                stg_gather_issue(e.aux, e.ld_aux, row0, p.M, n0 + 32 * c0, p.N, xa);
-                stg_gather_issue(e.aux2, e.ld_aux2, row0, p.M, n0 + 32 * c0, p.N, xb);
-            } else {
-                if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
-                if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
-            }
+            if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
+            if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
             if (kb_total > 0) {
                 if (!mbar_wait_bounded(&tfull[acc], (it >> 1) & 1, abort_flag)) break;
                 tc_fence_after();
@@ -505,7 +504,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         store_row32(out_base, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
                     }
                 }
-            } else if constexpr (EPI == EPI_LOGITS) {
+            } else if constexpr (EPI == EPI_LOGITS || EPI == EPI_LOGITS_STG) {
                 // per (row, column half) softmax statistics: stats pair nt*2 + h
                 float mx = -INFINITY, sm = 0.0f;
                 float t[32];
@@ -522,7 +521,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     }
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = round_bf16(v[i]);
-                    stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg, v);
+                    if constexpr (EPI == EPI_LOGITS_STG)
+                        stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg, v);
+                    else if (valid)
+                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, 0, v);
                     float cm = -INFINITY;
 #pragma unroll
                     for (int i = 0; i < 32; ++i)
@@ -566,21 +568,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
                     tmem_load32(tbase + c * 32, v);
-                    stg_gather_finish(stg, xa, g);
-                    stg_gather_finish(stg + kStgBytes, xb, u);
-                    if (j + 1 < CPW) {
-                        stg_gather_issue(e.aux, e.ld_aux, row0, p.M, n + 32, p.N, xa);
-                        stg_gather_issue(e.aux2, e.ld_aux2, row0, p.M, n + 32, p.N, xb);
-                    }
-                    float du[32];
+                    if (valid) {
+                        unpack32_dyn(xa, 0, g);
+                        unpack32_dyn(xb, 0, u);
+                        if (j + 1 < CPW) {
+                            load_chunk_bf16(pa, ra, n + 32, p.N, xa, 0);
+                            load_chunk_bf16(pb, rb, n + 32, p.N, xb, 0);
+                        }
+                        float du[32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const float sg = fast_sigmoid(g[i]);
-                        du[i] = v[i] * g[i] * sg;
-                        v[i] = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
+                        for (int i = 0; i < 32; ++i) {
+                            const float sg = fast_sigmoid(g[i]);
+                            du[i] = v[i] * g[i] * sg;
+                            v[i] = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
+                        }
+                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
+                        store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, p.N, e.out2_f32, du);
                     }
-                    stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg + 2 * kStgBytes, v);
-                    stg_scatter(e.out2, e.ld_out2, row0, p.M, n, p.N, stg + 3 * kStgBytes, du);
                 }
             }
             tc_fence_before();
@@ -753,6 +757,8 @@ static int dispatch(const Params& p, int epi_kind, bool a_mn, bool b_mn, bool du
             return launch_inst<CG, true, false, EPI_LINEAR>(p, stream);
         case EPI_LOGITS:
             if (a_mn || b_mn) return BOM_ENOTSUP;
+            // short contractions: the epilogue dominates, so stage its stores
+            if (p.kb[0] <= 16) return launch_inst<CG, false, false, EPI_LOGITS_STG>(p, stream);
             return launch_inst<CG, false, false, EPI_LOGITS>(p, stream);
         case EPI_SWIGLU_FWD:
             if (a_mn || b_mn || !dual_b) return BOM_ENOTSUP;
