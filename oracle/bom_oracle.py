@@ -30,7 +30,11 @@ per-dataset-results appendix, with the equations of Section 3):
      (Section 3.4, the second-moment equation);
   6. theta <- (1 - eta omega) theta - eta u / (sqrt(vhat) + eps)
      (Section 3.4 update equation; Algorithm 1, last step).  No first-moment
-     bias correction is applied to u (Section 3.5, "The substitution").
+     bias correction is applied to u (Section 3.5, "The substitution");
+  7. drift telemetry and the own-step control (Section 3.3, Eq.
+     drift-telemetry; stale-control and drift-measurement appendices): the
+     own-step projection Jbar_t^T s_t, its EMA M_t with Mhat_t, the cosine and
+     relative size of Mhat_t - h_t, and the within-batch cancellation ratio.
 
 Backbone layers supported (shapes of the paper's settings; see the workload
 module): Linear, Linear+GELU (exact erf form) and the SwiGLU MLP sublayer
@@ -41,7 +45,10 @@ Every function here is pinned by ``tests/test_oracle_pins.py`` against facts
 the paper or mathematics fix (finite-difference Jacobians and the exact batch
 decomposition, an independent autograd implementation, the EMA closed form of
 Lemma 2, the beta1 = 0 and lambda = 0 reductions, AdamW with beta1 = 0, the
-output-bias closed form and the zero-sum invariant).
+output-bias closed form and the zero-sum invariant); the telemetry functions
+by ``tests/test_oracle_telemetry_pins.py`` (finite-difference Jbar^T s, no drift
+at t = 1 and for a linear model on a fixed batch, Mhat = qhat on the head bias,
+closed forms and a brute-force loop for the statistics).
 """
 from __future__ import annotations
 
@@ -319,3 +326,57 @@ def head_weight_grad_rows(R, H, valid, qhat, n_t, lam, vocab_rows):
 def head_input_grad_rows(R, W, valid, qhat, n_t, lam, token_rows):
     """Rows `token_rows` of the head-input cotangent dZ W."""
     return mix_cotangent_rows(R, valid, qhat, n_t, lam, token_rows) @ np.asarray(W, dtype=F64)
+
+
+# --------------------------------------------------------------------------
+# Drift telemetry and the own-step control (Section 3.3, Eq. jacobian-drift
+# and Eq. drift-telemetry; stale-control and drift-measurement appendices).
+#
+# The own-step control keeps BOM's task-space signal s_t but projects it
+# through the model and examples of its own step, accumulating the
+# parameter-shaped  M_t = beta1 M_{t-1} + (1 - beta1) Jbar_t^T s_t  and using
+# u = (1 - lambda) g_t + lambda Mhat_t,  Mhat_t = M_t / (1 - beta1^t).
+# On one trajectory, Mhat_t - h_t (h_t = Jbar_t^T qhat_t) is the
+# bias-corrected historical-projection drift; the telemetry reports its cosine
+# and relative size, and the within-batch cancellation ratio
+# ||s_t|| / (N_t^-1 sum_{i in I_t} ||r_i||).
+# --------------------------------------------------------------------------
+def own_step_projection(layers, head_bias, params, X, labels, ignore_index=-100):
+    """Jbar_t^T s_t per tensor: the reverse pass of the logit cotangent
+    1_{I_t} s_t^T / N_t.  Returns (per-tensor list, s_t, N_t)."""
+    params = [np.asarray(p, dtype=F64) for p in params]
+    Z, saved = forward(layers, head_bias, params, X)
+    valid, n_t = supervised_set(labels, Z.shape[1], ignore_index)
+    s = batch_mean_residual(residuals(Z, labels, valid), n_t)
+    o, _, _ = backward(layers, head_bias, params, saved, valid[:, None] * s[None, :] / n_t)
+    return o, s, n_t
+
+
+def own_step_moment(M_prev, o, t, beta1):
+    """M_t = beta1 M_{t-1} + (1 - beta1) o_t and Mhat_t = M_t / (1 - beta1^t)
+    (stale-control appendix; the bias correction as for q)."""
+    if t < 1:
+        raise OracleError("t is 1-based")
+    M = beta1 * np.asarray(M_prev, dtype=F64) + (1.0 - beta1) * np.asarray(o, dtype=F64)
+    return M, M / (1.0 - beta1 ** t)
+
+
+def drift_statistics(mhat_list, h_list):
+    """cos(Mhat, h) and ||Mhat - h|| / ||Mhat|| over the concatenation of the
+    given tensors (Eq. drift-telemetry), with the four sums they come from."""
+    a = np.concatenate([np.ravel(np.asarray(x, dtype=F64)) for x in mhat_list])
+    b = np.concatenate([np.ravel(np.asarray(x, dtype=F64)) for x in h_list])
+    dot, mm, hh = float(a @ b), float(a @ a), float(b @ b)
+    dd = float((a - b) @ (a - b))
+    return dict(dot=dot, mm=mm, hh=hh, dd=dd, cos=dot / math.sqrt(mm * hh), rel=math.sqrt(dd / mm))
+
+
+def cancellation_ratio(R, valid, n_t):
+    """||s_t|| / (N_t^-1 sum_{i in I_t} ||r_i||) (drift-measurement appendix:
+    the share of the mean per-example residual norm that survives batch
+    averaging).  Returns (ratio, ||s_t||, mean residual norm)."""
+    rows = np.nonzero(valid)[0]
+    s = R[rows].sum(axis=0) / n_t
+    mean_norm = float(np.sqrt((R[rows] ** 2).sum(axis=1)).sum() / n_t)
+    s_norm = float(np.sqrt(s @ s))
+    return s_norm / mean_norm, s_norm, mean_norm
