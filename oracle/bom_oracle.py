@@ -34,7 +34,9 @@ per-dataset-results appendix, with the equations of Section 3):
   7. drift telemetry and the own-step control (Section 3.3, Eq.
      drift-telemetry; stale-control and drift-measurement appendices): the
      own-step projection Jbar_t^T s_t, its EMA M_t with Mhat_t, the cosine and
-     relative size of Mhat_t - h_t, and the within-batch cancellation ratio.
+     relative size of Mhat_t - h_t, and the within-batch cancellation ratio;
+  8. BOM-Adam-mini (Section 3.5, composition with Adam-mini): the update with
+     one second-moment scalar shared by each block of a tensor.
 
 Backbone layers supported (shapes of the paper's settings; see the workload
 module): Linear, Linear+GELU (exact erf form) and the SwiGLU MLP sublayer
@@ -380,3 +382,37 @@ def cancellation_ratio(R, valid, n_t):
     mean_norm = float(np.sqrt((R[rows] ** 2).sum(axis=1)).sum() / n_t)
     s_norm = float(np.sqrt(s @ s))
     return s_norm / mean_norm, s_norm, mean_norm
+
+
+# --------------------------------------------------------------------------
+# BOM-Adam-mini (Section 3.5 "The substitution", composition with Adam-mini;
+# optimizer-implementation appendix): Adam-mini keeps one second-moment scalar
+# per block of a tensor (per attention head, per output neuron, the whole
+# tensor, or per element) and scales every element of the block by it.  The
+# BOM composition feeds it u instead of a first moment:
+#   v_b = beta2 v_b + (1 - beta2) mean_{i in b} u_i^2,   vhat_b = v_b / (1 - beta2^t)
+#   theta_i <- (1 - eta omega) theta_i - eta u_i / (sqrt(vhat_b) + eps).
+# Blocks here are consecutive runs of `block` elements of the flat tensor (a
+# row-major [d_out, d_in] matrix with block = d_in shares v per output neuron;
+# block = n is the whole tensor, block = 1 is elementwise BOM-AdamW); the last
+# block may be shorter.
+# --------------------------------------------------------------------------
+def bom_update_blockshared(theta, u, v_blocks, block, lr, wd, t, beta2=0.999, eps=1e-8):
+    """Returns (theta_new, v_blocks_new) in float64."""
+    if t < 1:
+        raise OracleError("t is 1-based")
+    if block < 1:
+        raise OracleError("block >= 1")
+    theta = np.asarray(theta, dtype=F64).ravel()
+    u = np.asarray(u, dtype=F64).ravel()
+    n = theta.size
+    nb = -(-n // block)
+    v_blocks = np.asarray(v_blocks, dtype=F64).ravel()
+    if v_blocks.size != nb:
+        raise OracleError("one second-moment entry per block")
+    mean_sq = np.array([np.mean(u[b * block:(b + 1) * block] ** 2) for b in range(nb)])
+    v_new = beta2 * v_blocks + (1.0 - beta2) * mean_sq
+    vhat = v_new / (1.0 - beta2 ** t)
+    denom = np.repeat(np.sqrt(vhat) + eps, block)[:n]
+    theta_new = (1.0 - lr * wd) * theta - lr * u / denom
+    return theta_new, v_new
