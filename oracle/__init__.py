@@ -10,5 +10,5 @@ from .bom_oracle import (  # noqa: F401
     batch_mean_residual, ema_update, cross_entropy, bom_step, bom_update,
     mix_numerator, bom_update_gh, mix_cotangent_rows, head_weight_grad_rows, head_input_grad_rows,
     own_step_projection, own_step_moment, drift_statistics, cancellation_ratio,
-    bom_update_blockshared,
+    bom_update_blockshared, clip_factor, bom_update_clipped,
 )

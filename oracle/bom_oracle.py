@@ -36,7 +36,9 @@ per-dataset-results appendix, with the equations of Section 3):
      own-step projection Jbar_t^T s_t, its EMA M_t with Mhat_t, the cosine and
      relative size of Mhat_t - h_t, and the within-batch cancellation ratio;
   8. BOM-Adam-mini (Section 3.5, composition with Adam-mini): the update with
-     one second-moment scalar shared by each block of a tensor.
+     one second-moment scalar shared by each block of a tensor;
+  9. global-norm clipping of u before the update (pretraining-parameters and
+     convergence appendices).
 
 Backbone layers supported (shapes of the paper's settings; see the workload
 module): Linear, Linear+GELU (exact erf form) and the SwiGLU MLP sublayer
@@ -416,3 +418,28 @@ def bom_update_blockshared(theta, u, v_blocks, block, lr, wd, t, beta2=0.999, ep
     denom = np.repeat(np.sqrt(vhat) + eps, block)[:n]
     theta_new = (1.0 - lr * wd) * theta - lr * u / denom
     return theta_new, v_new
+
+
+# --------------------------------------------------------------------------
+# Global-norm clipping of the numerator (pretraining-parameters appendix: the
+# language-modeling runs clip at 1.0; convergence appendix: the clipped
+# numerator is what the adaptive update receives).  The norm runs over every
+# trainable tensor together; the factor follows the common PyTorch rule
+#   c = min(1, max_norm / (||u||_2 + 1e-6)),  u <- c u  before v and theta.
+# --------------------------------------------------------------------------
+def clip_factor(u_list, max_norm):
+    """Scale applied to every tensor of u so that the global L2 norm is at most max_norm."""
+    sq = sum(float(np.sum(np.asarray(u, dtype=F64) ** 2)) for u in u_list)
+    return min(1.0, max_norm / (math.sqrt(sq) + 1e-6))
+
+
+def bom_update_clipped(theta_list, u_list, v_list, lr, wd_list, t, max_norm, beta2=0.999, eps=1e-8):
+    """BOM-AdamW update of several tensors with their numerator clipped to a
+    global norm of max_norm.  Returns (theta_list, v_list, factor)."""
+    c = clip_factor(u_list, max_norm)
+    out_t, out_v = [], []
+    for th, u, v, wd in zip(theta_list, u_list, v_list, wd_list):
+        a, b = bom_update(th, c * np.asarray(u, dtype=F64), v, lr, wd, t, beta2, eps)
+        out_t.append(a)
+        out_v.append(b)
+    return out_t, out_v, c
