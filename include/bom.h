@@ -97,6 +97,10 @@ typedef struct {
     int32_t n_t;         /* |I_t|                                                     */
     int32_t status;      /* bom_status latched on the device during the last step    */
     float s_norm;        /* ||s_t||_2                                                */
+    float r_norm_mean;   /* N_t^-1 sum_{i in I_t} ||r_i||_2; only on steps with an
+                            own-step output registered, else 0                      */
+    float cancel;        /* within-batch cancellation ratio s_norm / r_norm_mean
+                            (drift-measurement appendix), 0 when not measured        */
 } bom_stats;
 
 typedef struct bom_handle bom_handle;
@@ -147,6 +151,35 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
  * input-side half of the head backward.  NULL disables it (the default). */
 bom_status bom_set_input_grad(bom_handle* h, void* dx);
 
+/* Drift telemetry and the own-step control (Section 3.3, Eq. drift-telemetry;
+ * stale-control and drift-measurement appendices).
+ * Registers bom_param_count fp32 device buffers (shapes as the parameters)
+ * that every following bom_step fills with the own-step projection
+ * o_t = Jbar_t^T s_t: one extra backward of the logit cotangent
+ * N_t^-1 1_{I_t} s_t^T through the current model and batch.  Such steps also
+ * measure the per-row residual norms for bom_stats.r_norm_mean / cancel.
+ * NULL disables it (the default).  Returns BOM_ENOTSUP for a buffer that is
+ * not 16-byte aligned. */
+bom_status bom_set_own_step_output(bom_handle* h, void* const* o);
+
+/* Own-step moment over a flat range of n fp32 elements:
+ *   M <- beta1 M + (1 - beta1) o,   mhat = M / (1 - beta1^t)
+ * (M_0 = 0; the own-step control then updates with u = (1-lambda) g +
+ * lambda mhat, i.e. bom_update with hvec = mhat).  When sums is non-NULL,
+ * hvec ([n] fp32: h_t = Jbar_t^T qhat_t of the same step) must be given and
+ *   sums[0..3] += ( <mhat,h>, <mhat,mhat>, <h,h>, <mhat-h,mhat-h> )
+ * in fp64 and a fixed summation order, from which cos(Mhat_t, h_t) and
+ * ||Mhat_t - h_t|| / ||Mhat_t|| follow; calling it per tensor range with one
+ * sums buffer per group (e.g. head, encoder) gives the paper's split.
+ * M, o, hvec, mhat: device fp32 [n]; sums: device fp64 [4] or NULL.
+ * Uses a per-handle partials buffer: calls on one handle must be ordered on
+ * one stream.  Asynchronous; t >= 1 and 0 <= beta1 < 1 or BOM_EINVAL. */
+bom_status bom_own_step_moment(bom_handle* h, float* M, const float* o, const float* hvec, float* mhat,
+                               int64_t n, float beta1, int64_t t, double* sums, void* stream);
+
+/* Bytes bom_get_stats copies from the device per call. */
+int64_t bom_stats_transfer_bytes(void);
+
 /* Device-side outputs of the last step that are useful for checks:
  *   qhat [d_out] fp32, s [d_out] fp32, lse [n_rows] fp32 (row log-sum-exp).
  * Pointers stay valid until bom_destroy; contents until the next bom_step. */
@@ -170,6 +203,21 @@ bom_status bom_get_stats(bom_handle* h, bom_stats* out, void* stream);
 bom_status bom_update(float* theta, const void* g, int32_t g_dtype, const float* hvec, float* v,
                       uint16_t* theta_bf16, int64_t n, float lr, float wd, float lambda,
                       float beta2, float eps, int64_t t, void* stream);
+
+/* BOM-Adam-mini update (Section 3.5, composition with Adam-mini; the
+ * optimizer-implementation appendix): as bom_update, but one second-moment
+ * scalar is shared by each block of `block` consecutive elements,
+ *   v_b  <- beta2 v_b + (1-beta2) mean_{i in b} u_i^2,
+ *   theta <- (1 - lr wd) theta - lr u / (sqrt(v_b / (1-beta2^t)) + eps).
+ * A row-major [d_out, d_in] weight with block = d_in shares v per output
+ * neuron, block = n shares it over the whole tensor, block = 1 is bom_update;
+ * the last block may be shorter.
+ *   v_blocks    [ceil(n / block)] fp32, updated in place (v_0 = 0).
+ * Other arguments as bom_update.  block >= 1; sums of u^2 are formed per
+ * block in a fixed order (deterministic). */
+bom_status bom_update_blockshared(float* theta, const void* g, int32_t g_dtype, const float* hvec, float* v_blocks,
+                                  uint16_t* theta_bf16, int64_t n, int64_t block, float lr, float wd, float lambda,
+                                  float beta2, float eps, int64_t t, void* stream);
 
 /* Auxiliary: D = alpha * op(A) op(B)^T on the bf16 tensor-core GEMM engine the
  * step uses (tcgen05 MMA, TMEM accumulators, TMA loads), fp32 accumulation,

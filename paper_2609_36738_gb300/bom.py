@@ -28,10 +28,8 @@ BOM_OUT_U, BOM_OUT_G_AND_H = 0, 1
 # Every symbol include/bom.h declares.
 EXPORTED = ("bom_param_count", "bom_param_shape", "bom_init", "bom_workspace_bytes", "bom_step",
             "bom_set_input_grad", "bom_step_outputs", "bom_get_stats", "bom_update", "bom_gemm_bf16", "bom_trace", "bom_trace_read",
-            "bom_launch_count", "bom_colsum_noalloc", "bom_destroy", "bom_status_string")
-
-# Bytes bom_get_stats copies from the device (the scalar block of a step).
-STATS_D2H_BYTES = 44
+            "bom_launch_count", "bom_colsum_noalloc", "bom_set_own_step_output", "bom_own_step_moment",
+            "bom_stats_transfer_bytes", "bom_update_blockshared", "bom_destroy", "bom_status_string")
 
 
 class bom_trace_entry(C.Structure):
@@ -50,7 +48,8 @@ class bom_config(C.Structure):
 
 
 class bom_stats(C.Structure):
-    _fields_ = [("loss", C.c_float), ("n_t", C.c_int32), ("status", C.c_int32), ("s_norm", C.c_float)]
+    _fields_ = [("loss", C.c_float), ("n_t", C.c_int32), ("status", C.c_int32), ("s_norm", C.c_float),
+                ("r_norm_mean", C.c_float), ("cancel", C.c_float)]
 
 
 class BomError(RuntimeError):
@@ -99,6 +98,14 @@ def lib() -> C.CDLL:
     L.bom_launch_count.restype = i64
     L.bom_colsum_noalloc.argtypes = [vp, i32, i64, i64, i64, vp, vp, vp]
     L.bom_colsum_noalloc.restype = i32
+    L.bom_set_own_step_output.argtypes = [vp, C.POINTER(vp)]
+    L.bom_set_own_step_output.restype = i32
+    L.bom_own_step_moment.argtypes = [vp, vp, vp, vp, vp, i64, f32, i64, vp, vp]
+    L.bom_own_step_moment.restype = i32
+    L.bom_stats_transfer_bytes.argtypes = []
+    L.bom_stats_transfer_bytes.restype = i64
+    L.bom_update_blockshared.argtypes = [vp, vp, i32, vp, vp, vp, i64, i64, f32, f32, f32, f32, f32, i64, vp]
+    L.bom_update_blockshared.restype = i32
     L.bom_destroy.argtypes = [vp]
     L.bom_destroy.restype = None
     L.bom_status_string.argtypes = [i32]
@@ -207,7 +214,8 @@ def bom_get_stats(h, stream=None, check: bool = True) -> dict:
     code = lib().bom_get_stats(h, C.byref(st), _stream(stream))
     if check:
         _check(code, "bom_get_stats")
-    return dict(loss=st.loss, n_t=st.n_t, status=st.status, s_norm=st.s_norm, code=code)
+    return dict(loss=st.loss, n_t=st.n_t, status=st.status, s_norm=st.s_norm, r_norm_mean=st.r_norm_mean,
+                cancel=st.cancel, code=code)
 
 
 def bom_update(theta, g, g_dtype: int, hvec, v, theta_bf16, n: int, lr: float, wd: float, lam: float,
@@ -215,6 +223,13 @@ def bom_update(theta, g, g_dtype: int, hvec, v, theta_bf16, n: int, lr: float, w
     _check(lib().bom_update(_ptr(theta), _ptr(g), int(g_dtype), _ptr(hvec), _ptr(v), _ptr(theta_bf16), int(n),
                             float(lr), float(wd), float(lam), float(beta2), float(eps), int(t), _stream(stream)),
            "bom_update")
+
+
+def bom_update_blockshared(theta, g, g_dtype: int, hvec, v_blocks, theta_bf16, n: int, block: int, lr: float,
+                           wd: float, lam: float, beta2: float, eps: float, t: int, stream=None) -> None:
+    _check(lib().bom_update_blockshared(_ptr(theta), _ptr(g), int(g_dtype), _ptr(hvec), _ptr(v_blocks),
+                                        _ptr(theta_bf16), int(n), int(block), float(lr), float(wd), float(lam),
+                                        float(beta2), float(eps), int(t), _stream(stream)), "bom_update_blockshared")
 
 
 def bom_gemm_bf16(A, lda: int, a_mn_major: bool, B, ldb: int, b_mn_major: bool, D, ldd: int, M: int, N: int,
@@ -245,6 +260,25 @@ def bom_colsum_noalloc(x, dtype: int, ldx: int, n_rows: int, n_cols: int, weight
     scratch inside the library; see include/bom.h for the limits)."""
     _check(lib().bom_colsum_noalloc(_ptr(x), int(dtype), int(ldx), int(n_rows), int(n_cols), _ptr(weights),
                                     _ptr(out), _stream(stream)), "bom_colsum_noalloc")
+
+
+def bom_set_own_step_output(h, o) -> None:
+    """Registers per-tensor fp32 outputs of the own-step projection Jbar^T s_t
+    (``None`` disables it)."""
+    if o is None:
+        _check(lib().bom_set_own_step_output(h, None), "bom_set_own_step_output")
+        return
+    O = (C.c_void_p * len(o))(*[_ptr(p) for p in o])
+    _check(lib().bom_set_own_step_output(h, O), "bom_set_own_step_output")
+
+
+def bom_own_step_moment(h, M, o, hvec, mhat, n: int, beta1: float, t: int, sums=None, stream=None) -> None:
+    _check(lib().bom_own_step_moment(h, _ptr(M), _ptr(o), _ptr(hvec), _ptr(mhat), int(n), float(beta1), int(t),
+                                     _ptr(sums), _stream(stream)), "bom_own_step_moment")
+
+
+def bom_stats_transfer_bytes() -> int:
+    return int(lib().bom_stats_transfer_bytes())
 
 
 class BomModel:

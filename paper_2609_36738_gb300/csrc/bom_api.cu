@@ -12,7 +12,8 @@
 //   backward  head dW = a R^T H + b qhat (x) c      (rank-1 epilogue),
 //             head dH = a R W + b 1_{I_t} w^T       (broadcast-row epilogue),
 //             then the backbone VJPs, with (a, b) = N_t^-1 (1-lambda, lambda)
-//             for u, N_t^-1 (1, 0) for g and N_t^-1 (0, 1) for h.
+//             for u, N_t^-1 (1, 0) for g and N_t^-1 (0, 1) for h; the
+//             own-step pass (telemetry) broadcasts s_t in place of qhat.
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -66,6 +67,10 @@ struct bom_handle {
     float* qhat = nullptr;
     float* cvec = nullptr;
     float* wvec = nullptr;
+    float* wsvec = nullptr;  // W^T s_t (own-step pass)
+    float* rnorm = nullptr;  // ||r_i|| per row (own-step telemetry)
+    double* tel_part = nullptr;  // per-block partials of bom_own_step_moment
+    std::vector<void*> own_out;  // own-step projection outputs (bom_set_own_step_output)
     float* part = nullptr;
     void* dx[2] = {nullptr, nullptr};
     void* dG = nullptr;
@@ -179,6 +184,9 @@ size_t carve(bom_handle* h, char* base) {
     h->qhat = static_cast<float*>(c.take(V * 4));
     h->cvec = static_cast<float*>(c.take(h->d_model * 4));
     h->wvec = static_cast<float*>(c.take(h->d_model * 4));
+    h->wsvec = static_cast<float*>(c.take(h->d_model * 4));
+    h->rnorm = static_cast<float*>(c.take(n * 4));
+    h->tel_part = static_cast<double*>(c.take(4 * kOwnStepMaxBlocks * sizeof(double)));
     const int64_t rb = row_blocks(n) > row_blocks(V) ? row_blocks(n) : row_blocks(V);
     h->part = static_cast<float*>(c.take(rb * h->max_width * 4));
     h->dx[0] = c.take(n * h->max_width * e);
@@ -467,30 +475,42 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
     const float inv_bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(cfg.beta1), static_cast<double>(t))));
     BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 20.0 * V,
                launch_finish_sq(h->colpart, resid_blocks(n), V, cfg.beta1, inv_bc1, q, h->s, h->qhat, h->sc, s));
-    BOM_TRACED("scalars", 0, 4.0 * (n + V), launch_scalars(h->ce, n, h->s, V, h->sc, s));
+    const bool own = !h->own_out.empty();
+    if (own)   // per-row residual norms for the cancellation ratio
+        BOM_TRACED("row_norm", 2.0 * n * V, h->esz * n * h->ldz + 4.0 * n,
+                   launch_row_norm(h->Z, cf32, h->ldz, n, V, h->rnorm, h->sc, s));
+    BOM_TRACED("scalars", 0, 4.0 * (n + V), launch_scalars(h->ce, n, h->s, V, own ? h->rnorm : nullptr, h->sc, s));
     // c = colsum_{I_t}(H) and w = W^T qhat (the rank-1 / broadcast factors of the reprojection)
     BOM_TRACED("colsum", 2.0 * n * dm, h->esz * n * dm,
                launch_colsum(xin, cf32, dm, n, dm, labels, cfg.ignore_index, nullptr, 1.0f, h->part, h->cvec, 1,
                              h->sc, s));
     BOM_TRACED("colsum", 2.0 * V * dm, h->esz * V * dm,
                launch_colsum(Wh, cf32, dm, V, dm, nullptr, 0, h->qhat, 1.0f, h->part, h->wvec, 1, h->sc, s));
+    if (own)
+        BOM_TRACED("colsum", 2.0 * V * dm, h->esz * V * dm,
+                   launch_colsum(Wh, cf32, dm, V, dm, nullptr, 0, h->s, 1.0f, h->part, h->wsvec, 1, h->sc, s));
 
     // ---------------------------------------------------------------- backward
-    const int passes[2] = {gh ? 1 : 0, 2};
-    const int npass = gh ? 2 : 1;
+    // passes: 0 = u, 1 = g, 2 = h = Jbar^T qhat, 3 = own-step projection Jbar^T s_t
+    int passes[3], npass = 0;
+    passes[npass++] = gh ? 1 : 0;
+    if (gh) passes[npass++] = 2;
+    if (own) passes[npass++] = 3;
     for (int pp = 0; pp < npass; ++pp) {
         const int pass = passes[pp];
-        void* const* outp = pass == 2 ? h_out : grads;
-        const int of32 = pass == 2 ? 1 : cf32;
+        void* const* outp = pass == 3 ? h->own_out.data() : (pass == 2 ? h_out : grads);
+        const int of32 = pass >= 2 ? 1 : cf32;
         const float* cr = &h->sc->coef_r[pass];
         const float* cq = &h->sc->coef_q[pass];
-        const int64_t kfull = pass == 2 ? 0 : 1;  // the h pass has no residual term
+        const int64_t kfull = pass >= 2 ? 0 : 1;  // the h and own-step passes have no residual term
+        const float* tvec = pass == 3 ? h->s : h->qhat;      // broadcast task-space vector
+        const float* wtvec = pass == 3 ? h->wsvec : h->wvec; // W^T of it
         {   // head weight: a R^T H + b qhat (x) c
             GemmDesc g = gemm1(V, dm, kfull * n, mnmaj(h->Z, h->ldz), mnmaj(xin, dm));
             g.epi.alpha_const = 1.0f;
             g.epi.alpha_dev = cr;
             g.epi.beta_dev = cq;
-            g.epi.r1u = h->qhat;
+            g.epi.r1u = tvec;
             g.epi.r1v = h->cvec;
             g.epi.out = outp[head_w];
             g.epi.ld_out = dm;
@@ -498,19 +518,19 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
             BOM_TRY(run_gemm(h, g, s));
         }
         if (head_b >= 0) {
-            const float a = pass == 0 ? 1.0f - cfg.lambda : (pass == 1 ? 1.0f : 0.0f);
-            const float b = pass == 0 ? cfg.lambda : (pass == 1 ? 0.0f : 1.0f);
+            const float a = pass == 0 ? 1.0f - cfg.lambda : (pass == 1 || pass == 3 ? 1.0f : 0.0f);
+            const float b = pass == 0 ? cfg.lambda : (pass == 2 ? 1.0f : 0.0f);
             BOM_TRACED("axpby", 3.0 * V, 12.0 * V, launch_axpby(h->s, h->qhat, a, b, V, outp[head_b], of32, h->sc, s));
         }
         // the cotangent of X goes out with the u (or g) pass when requested
-        const bool want_dx = h->dx_in != nullptr && pass != 2;
+        const bool want_dx = h->dx_in != nullptr && pass < 2;
         if (h->lw.empty() && !want_dx) continue;
         int cur = 0;
         {   // head input: a R W + b 1_{I_t} w^T  (times GELU' of the last layer)
             GemmDesc g = gemm1(n, dm, kfull * V, kmaj(h->Z, h->ldz), mnmaj(Wh, dm));
             g.epi.alpha_dev = cr;
             g.epi.beta_dev = cq;
-            g.epi.bw = h->wvec;
+            g.epi.bw = wtvec;
             g.epi.mask_labels = labels;
             g.epi.ignore_index = cfg.ignore_index;
             if (!h->lw.empty() && h->lw.back().kind == BOM_LAYER_LINEAR_GELU) {
@@ -625,6 +645,36 @@ bom_status bom_set_input_grad(bom_handle* h, void* dx) {
     return BOM_OK;
 }
 
+bom_status bom_set_own_step_output(bom_handle* h, void* const* o) {
+    if (!h) return BOM_EINVAL;
+    if (!o) {
+        h->own_out.clear();
+        return BOM_OK;
+    }
+    const int np = bom_param_count(&h->cfg);
+    std::vector<void*> v(o, o + np);
+    for (void* p : v) {
+        if (!p) return BOM_EINVAL;
+        if (!aligned16(p)) return BOM_ENOTSUP;
+    }
+    h->own_out = v;
+    return BOM_OK;
+}
+
+bom_status bom_own_step_moment(bom_handle* h, float* M, const float* o, const float* hvec, float* mhat, int64_t n,
+                               float beta1, int64_t t, double* sums, void* stream) {
+    if (!h || n < 0 || t < 1 || !(beta1 >= 0.0f && beta1 < 1.0f)) return BOM_EINVAL;
+    if (n == 0) return BOM_OK;
+    if (!M || !o || !mhat || (sums && !hvec)) return BOM_EINVAL;
+    const float inv_bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta1), static_cast<double>(t))));
+    const int nb = own_step_blocks(n, device_sm_count());
+    launch_own_step_moment(M, o, hvec, mhat, n, beta1, inv_bc1, h->tel_part, nb, sums,
+                           static_cast<cudaStream_t>(stream));
+    return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+int64_t bom_stats_transfer_bytes(void) { return static_cast<int64_t>(sizeof(DevScalars)); }
+
 bom_status bom_step_outputs(bom_handle* h, const float** qhat, const float** s, const float** lse) {
     if (!h) return BOM_EINVAL;
     if (qhat) *qhat = h->qhat;
@@ -642,6 +692,8 @@ bom_status bom_get_stats(bom_handle* h, bom_stats* out, void* stream) {
     out->n_t = sc.n_t;
     out->status = sc.status;
     out->s_norm = sc.s_norm;
+    out->r_norm_mean = sc.r_norm_mean;
+    out->cancel = sc.r_norm_mean > 0.0f ? sc.s_norm / sc.r_norm_mean : 0.0f;
     return static_cast<bom_status>(sc.status);
 }
 
@@ -658,6 +710,22 @@ bom_status bom_update(float* theta, const void* g, int32_t g_dtype, const float*
     const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
     return static_cast<bom_status>(launch_update(theta, g, g_dtype == BOM_BF16, hvec, v, theta_bf16, n, lr, wd,
                                                  lambda, beta2, eps, inv_bc2, static_cast<cudaStream_t>(stream)));
+}
+
+bom_status bom_update_blockshared(float* theta, const void* g, int32_t g_dtype, const float* hvec, float* v_blocks,
+                                  uint16_t* theta_bf16, int64_t n, int64_t block, float lr, float wd, float lambda,
+                                  float beta2, float eps, int64_t t, void* stream) {
+    if (n < 0 || t < 1 || block < 1) return BOM_EINVAL;
+    if (n == 0) return BOM_OK;
+    if (!theta || !g || !v_blocks) return BOM_EINVAL;
+    if (g_dtype != BOM_F32 && g_dtype != BOM_BF16) return BOM_EINVAL;
+    if (!(beta2 >= 0.0f && beta2 < 1.0f) || !(eps >= 0.0f)) return BOM_EINVAL;
+    if (!aligned16(theta) || !aligned16(g) || (hvec && !aligned16(hvec)) || (theta_bf16 && !aligned16(theta_bf16)))
+        return BOM_ENOTSUP;
+    const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
+    return static_cast<bom_status>(launch_update_blockshared(theta, g, g_dtype == BOM_BF16, hvec, v_blocks, theta_bf16,
+                                                             n, block, lr, wd, lambda, beta2, eps, inv_bc2,
+                                                             static_cast<cudaStream_t>(stream)));
 }
 
 bom_status bom_gemm_bf16(const uint16_t* A, int64_t lda, int32_t a_mn_major, const uint16_t* B, int64_t ldb,

@@ -19,10 +19,11 @@ struct DevScalars {
     int32_t status;        // latched bom_status (first error wins), 0 = OK
     int32_t n_t;           // |I_t|
     float inv_nt;          // 1 / N_t
-    float coef_r[3];       // coefficient of r_i in the logit cotangent: [U pass, G pass, H pass]
-    float coef_q[3];       // coefficient of qhat in the logit cotangent
+    float coef_r[4];       // coefficient of r_i in the logit cotangent: [U, G, H, own-step pass]
+    float coef_q[4];       // coefficient of the broadcast task-space vector (qhat; s_t in the own-step pass)
     float loss;            // mean CE over I_t
     float s_norm;          // ||s_t||
+    float r_norm_mean;     // N_t^-1 sum_{i in I_t} ||r_i|| (own-step telemetry steps only, else 0)
 };
 
 __device__ __forceinline__ void latch_status(DevScalars* sc, int code) {
@@ -100,6 +101,51 @@ __device__ __forceinline__ void st_elem(void* base, int64_t idx, int is_f32, flo
         static_cast<__nv_bfloat16*>(base)[idx] = __float2bfloat16_rn(v);
 }
 __device__ __forceinline__ float round_bf16(float v) { return __bfloat162float(__float2bfloat16_rn(v)); }
+
+// ---------------------------------------------------------------- packed arithmetic
+// Instruction-lean forms for the epilogues and streaming passes that are
+// issue-bound: one instruction covers two values (sm_100 family).
+constexpr float kLog2e = 1.4426950408889634f;
+
+// Hardware base-2 exponential (PTX ex2.approx.ftz.f32: relative error about
+// 2^-22; -inf gives +0).
+__device__ __forceinline__ float ex2_fast(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+// Two fp32 values rounded to nearest bf16, `lo` in the low half.
+__device__ __forceinline__ uint32_t cvt_bf16x2(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+__device__ __forceinline__ uint32_t max_bf16x2(uint32_t a, uint32_t b) {
+    uint32_t r;
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
+}
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+// a * b + c and a + b on fp32 pairs (fma.rn.f32x2 / add.rn.f32x2).
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+        "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
 
 // 32 consecutive elements of one row, [n, n+32) clipped to n < N.
 __device__ __forceinline__ void load_row32(const void* base, int64_t row_off, int n, int N, int is_f32,

@@ -1,12 +1,15 @@
 // tcgen05 GEMM engine for sm_103a: bf16 operands, fp32 accumulation in TMEM.
 //
-// One persistent CTA per SM walks the output tiles (128 x 256, or 128 x 128
-// output columns when the B tile is split between gate and up weights).
-// Warp roles:
+// Persistent kernel.  When M > 128, CTA pairs (clusters of two, one pair per
+// two SMs) compute 256 x 256 output tiles with cta_group::2 UMMAs; otherwise
+// single CTAs compute 128 x 256 tiles (128 x 128 output columns when the B
+// tile is split between gate and up weights).  Warp roles:
 //   warp 0     one thread issues TMA tile loads (128-byte swizzle) into a
-//              4-stage shared-memory ring guarded by mbarriers;
-//   warp 1     allocates 512 TMEM columns (two 128 x 256 fp32 accumulators)
-//              and one thread issues the UMMAs (M = 128, N = 256, K = 16),
+//              shared-memory ring guarded by mbarriers: 32 KB stages (A rows
+//              and this CTA's half of B), as many as fit beside the epilogue
+//              staging blocks, up to six;
+//   warp 1     allocates 512 TMEM columns (two 256-column fp32 accumulators)
+//              and, in the even CTA, one thread issues the UMMAs (K = 16),
 //              releasing each smem stage with tcgen05.commit;
 //   warps 2-9  epilogue: tcgen05.ld of the accumulator (one TMEM lane = one
 //              output row per thread; two warps per lane quarter, one per
@@ -38,6 +41,7 @@ constexpr int GROUP_M = 8;
 struct Params {
     CUtensorMap mapA[2];
     CUtensorMap mapB[2];
+    CUtensorMap mapOut;    // staged logits output: 32 x 32 boxes, 64-byte swizzle
     int M, N;
     int kb[2];
     int nseg;
@@ -101,72 +105,28 @@ __device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[NW], int slot, fl
 }
 
 // ---------------------------------------------------------------- staged epilogue I/O
-// A warp owns 32 consecutive output rows (one per lane).  Reading or writing
-// "its row" directly makes every warp instruction touch 32 different rows;
-// instead a 32 x 32 bf16 block goes through a per-warp shared-memory buffer:
-// global accesses are coalesced (lane l covers row l/4 + 8i, 16-byte segment
-// l%4) and each lane then reads / writes its own row in shared memory.  The
-// 80-byte row pitch (64 data + 16 pad) keeps both access patterns at the
-// minimum number of shared-memory wavefronts.
+// A warp owns 32 consecutive output rows (one per lane).  Writing "its row"
+// directly makes every warp instruction touch 32 different rows; instead a
+// 32 x 32 bf16 block goes through a per-warp shared-memory buffer: lane l
+// writes row l there, then the warp stores 8 rows per instruction, lane l
+// covering row (l % 8) + 8i and 16-byte segment l / 8, so each row's 64 bytes
+// leave in one coalesced access.  With the 80-byte row pitch (64 data + 16
+// pad) both the row-per-lane writes and the segment reads hit eight distinct
+// 4-bank groups per quarter-warp phase: no bank conflicts.
 constexpr int kStgPitch = 80;
 constexpr int kStgBytes = 32 * kStgPitch;
 
-// Issues the coalesced loads of block (rows row0.., columns n..n+31) into w.
-__device__ __forceinline__ void stg_gather_issue(const void* base, int64_t ld, int row0, int M, int n, int N,
-                                                 uint4 (&w)[4]) {
+// Stores the staged block (rows row0.., columns n..n+31) to global memory.
+__device__ __forceinline__ void stg_flush(void* base, int64_t ld, int row0, int M, int n, int N, const uint8_t* stg) {
     const int lane = threadIdx.x & 31;
-    const int c = n + 8 * (lane & 3);
+    const int seg = lane >> 3;
+    const int c = n + 8 * seg;
+    __syncwarp();
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const int r = row0 + (lane >> 2) + 8 * i;
-        const uint16_t* p = static_cast<const uint16_t*>(base) + static_cast<int64_t>(r) * ld + c;
-        if (r < M && c + 8 <= N) {
-            w[i] = __ldg(reinterpret_cast<const uint4*>(p));
-        } else {
-            uint32_t q[4] = {0u, 0u, 0u, 0u};
-            if (r < M)
-#pragma unroll
-                for (int k = 0; k < 8; ++k)
-                    if (c + k < N) q[k >> 1] |= static_cast<uint32_t>(p[k]) << (16 * (k & 1));
-            w[i] = make_uint4(q[0], q[1], q[2], q[3]);
-        }
-    }
-}
-// Puts the loaded block through the staging buffer; lane l receives row l.
-__device__ __forceinline__ void stg_gather_finish(uint8_t* stg, const uint4 (&w)[4], float (&v)[32]) {
-    const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-        *reinterpret_cast<uint4*>(stg + ((lane >> 2) + 8 * i) * kStgPitch + (lane & 3) * 16) = w[i];
-    __syncwarp();
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const uint4 x = *reinterpret_cast<const uint4*>(stg + lane * kStgPitch + k * 16);
-        const uint32_t ws[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            v[8 * k + 2 * j] = __uint_as_float(ws[j] << 16);
-            v[8 * k + 2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
-        }
-    }
-    __syncwarp();
-}
-// Lane l contributes row l of a 32 x 32 block; the warp stores it coalesced as bf16.
-__device__ __forceinline__ void stg_scatter(void* base, int64_t ld, int row0, int M, int n, int N, uint8_t* stg,
-                                            const float (&v)[32]) {
-    const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-        *reinterpret_cast<uint4*>(stg + lane * kStgPitch + k * 16) =
-            make_uint4(pack_bf16x2(v[8 * k], v[8 * k + 1]), pack_bf16x2(v[8 * k + 2], v[8 * k + 3]),
-                       pack_bf16x2(v[8 * k + 4], v[8 * k + 5]), pack_bf16x2(v[8 * k + 6], v[8 * k + 7]));
-    __syncwarp();
-    const int c = n + 8 * (lane & 3);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int rl = (lane >> 2) + 8 * i;
+        const int rl = (lane & 7) + 8 * i;
         const int r = row0 + rl;
-        const uint4 x = *reinterpret_cast<const uint4*>(stg + rl * kStgPitch + (lane & 3) * 16);
+        const uint4 x = *reinterpret_cast<const uint4*>(stg + rl * kStgPitch + seg * 16);
         uint16_t* p = static_cast<uint16_t*>(base) + static_cast<int64_t>(r) * ld + c;
         if (r < M) {
             if (c + 8 <= N) {
@@ -180,6 +140,50 @@ __device__ __forceinline__ void stg_scatter(void* base, int64_t ld, int row0, in
         }
     }
     __syncwarp();
+}
+// Lane l contributes row l of a 32 x 32 block as 16 packed bf16 pairs.
+__device__ __forceinline__ void stg_scatter_bf16(void* base, int64_t ld, int row0, int M, int n, int N, uint8_t* stg,
+                                                 const uint32_t (&b)[16]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        *reinterpret_cast<uint4*>(stg + lane * kStgPitch + k * 16) =
+            make_uint4(b[4 * k], b[4 * k + 1], b[4 * k + 2], b[4 * k + 3]);
+    stg_flush(base, ld, row0, M, n, N, stg);
+}
+// Lane l contributes row l of a 32 x 32 block as fp32 values, stored as bf16.
+__device__ __forceinline__ void stg_scatter(void* base, int64_t ld, int row0, int M, int n, int N, uint8_t* stg,
+                                            const float (&v)[32]) {
+    uint32_t b[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) b[i] = cvt_bf16x2(v[2 * i], v[2 * i + 1]);
+    stg_scatter_bf16(base, ld, row0, M, n, N, stg, b);
+}
+
+// Logits output through TMA: lane l writes row l of a 32 x 32 bf16 block into
+// `buf` in the 64-byte swizzled layout of mapOut (16-byte chunk k of row r at
+// r * 64 + 16 * (k ^ ((r >> 1) & 3)): no bank conflicts), then lane 0 stores
+// the block with one bulk copy, which clips rows >= M and columns >= N, under
+// the given L2 policy.  Two
+// buffers per warp alternate; before one is rewritten, lane 0 waits until the
+// store issued from it has finished reading it.
+constexpr int kTmaStgBytes = 32 * 64;
+__device__ __forceinline__ void tma_store_block(const CUtensorMap* map, uint8_t* buf, int x, int y,
+                                                const uint32_t (&b)[16], uint64_t policy) {
+    const int lane = threadIdx.x & 31;
+    if (lane == 0) bulk_wait_group_read<1>();
+    __syncwarp();
+    const int sw = (lane >> 1) & 3;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        *reinterpret_cast<uint4*>(buf + lane * 64 + 16 * (k ^ sw)) =
+            make_uint4(b[4 * k], b[4 * k + 1], b[4 * k + 2], b[4 * k + 3]);
+    fence_proxy_async_shared();
+    __syncwarp();
+    if (lane == 0) {
+        tma_store_2d_hint(map, buf, x, y, policy);
+        bulk_commit_group();
+    }
 }
 
 __device__ __forceinline__ float fast_exp(float x) { return exp2f(x * 1.4426950408889634f); }
@@ -206,13 +210,18 @@ constexpr int EPI_LOGITS_STG = 16;
 
 template <int CG, int EPI>
 struct Cfg {
-    static constexpr int NBUF = EPI == EPI_SWIGLU_FWD ? 3 : EPI == EPI_LOGITS_STG ? 1 : 0;
+    static constexpr int NBUF = EPI == EPI_SWIGLU_FWD ? 3 : 0;
     static constexpr int B_ROWS = CG == 2 ? 128 : 256;
-    static constexpr int STAGES = NBUF > 0 ? (CG == 2 ? 4 : 3) : (CG == 2 ? 6 : 4);
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
-    static constexpr int STG_BYTES = 8 * NBUF * kStgBytes;
+    static constexpr int STG_BYTES = EPI == EPI_LOGITS_STG ? 8 * 2 * kTmaStgBytes : 8 * NBUF * kStgBytes;
+    // as many stages as fit in the 227 KB a CTA may use beside the staging
+    // blocks, the 1 KB alignment slack and the barrier block, at most six (a
+    // seventh 32 KB stage measured slower on the linear epilogues)
+    static constexpr int STAGES_FIT = (227 * 1024 - STG_BYTES - 1024 - 256) / (A_BYTES + B_BYTES);
+    static constexpr int STAGES = STAGES_FIT < 6 ? STAGES_FIT : 6;
     static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 1024 + 256;
+    static_assert(STAGES >= 2, "pipeline needs two stages");
     static constexpr int TILE_M = BM * CG;
 };
 
@@ -420,6 +429,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         const EpiParams& e = p.epi;
         constexpr int CPW = BN / 64;  // 32-column chunks per warp
         int it = 0;
+        int sblk = 0;   // TMA-stored logits blocks issued by this warp
+        // the logits stream (read back once, by the residual pass) must not
+        // evict the operand tiles that later output tiles reuse from L2
+        const uint64_t zpol = make_policy_evict_first();
         for (int w = unit; w < num_work; w += nunits, ++it) {
             const int tile = w / p.ksplit;
             // split-K: each K range stores its raw fp32 tile into its own slice
@@ -443,7 +456,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t ra = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid);
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
-            uint8_t* stg = stg_all + (warp - 2) * C::NBUF * kStgBytes;
+            uint8_t* stg = EPI == EPI_LOGITS_STG ? stg_all + (warp - 2) * 2 * kTmaStgBytes
+                                                 : stg_all + (warp - 2) * C::NBUF * kStgBytes;
             if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
             if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
             if (kb_total > 0) {
@@ -505,7 +519,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     }
                 }
             } else if constexpr (EPI == EPI_LOGITS || EPI == EPI_LOGITS_STG) {
-                // per (row, column half) softmax statistics: stats pair nt*2 + h
+                // per (row, column half) softmax statistics: stats pair nt*2 + h.
+                // The statistics are taken over the bf16-rounded logits that
+                // are stored, so the residual pass sees a consistent row.
                 float mx = -INFINITY, sm = 0.0f;
                 float t[32];
 #pragma unroll 1
@@ -519,11 +535,54 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] += t[i];
                     }
+                    if (n + 32 <= p.N) {
+                        // full chunk: packed rounding, packed max, paired exponentials
+                        uint32_t b[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) b[i] = cvt_bf16x2(v[2 * i], v[2 * i + 1]);
+                        if constexpr (EPI == EPI_LOGITS_STG) {
+                            tma_store_block(&p.mapOut, stg + (sblk & 1) * kTmaStgBytes, n, row0, b, zpol);
+                            ++sblk;
+                        } else if (valid) {
+                            uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(e.out) +
+                                                                  static_cast<int64_t>(m) * e.ld_out + n);
+#pragma unroll
+                            for (int i = 0; i < 4; ++i)
+                                dst[i] = make_uint4(b[4 * i], b[4 * i + 1], b[4 * i + 2], b[4 * i + 3]);
+                        }
+                        uint32_t mb[8];
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) mb[i] = max_bf16x2(b[2 * i], b[2 * i + 1]);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) mb[i] = max_bf16x2(mb[i], mb[i + 4]);
+                        mb[0] = max_bf16x2(max_bf16x2(mb[0], mb[2]), max_bf16x2(mb[1], mb[3]));
+                        const float nm = fmaxf(mx, fmaxf(bf16_lo(mb[0]), bf16_hi(mb[0])));
+                        const float2 l2 = make_float2(kLog2e, kLog2e);
+                        const float2 off = make_float2(-nm * kLog2e, -nm * kLog2e);
+                        float2 a0 = make_float2(0.0f, 0.0f), a1 = a0;
+#pragma unroll
+                        for (int i = 0; i < 16; i += 2) {
+                            const float2 x0 = fma2(make_float2(bf16_lo(b[i]), bf16_hi(b[i])), l2, off);
+                            const float2 x1 = fma2(make_float2(bf16_lo(b[i + 1]), bf16_hi(b[i + 1])), l2, off);
+                            a0 = add2(a0, make_float2(ex2_fast(x0.x), ex2_fast(x0.y)));
+                            a1 = add2(a1, make_float2(ex2_fast(x1.x), ex2_fast(x1.y)));
+                        }
+                        a0 = add2(a0, a1);
+                        const float scale = (mx == -INFINITY) ? 0.0f : ex2_fast((mx - nm) * kLog2e);
+                        sm = sm * scale + (a0.x + a0.y);
+                        mx = nm;
+                        continue;
+                    }
+                    // ragged last chunk
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = round_bf16(v[i]);
-                    if constexpr (EPI == EPI_LOGITS_STG)
-                        stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg, v);
-                    else if (valid)
+                    if constexpr (EPI == EPI_LOGITS_STG) {
+                        uint32_t b[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) b[i] = cvt_bf16x2(v[2 * i], v[2 * i + 1]);
+                        tma_store_block(&p.mapOut, stg + (sblk & 1) * kTmaStgBytes, n, row0, b, zpol);
+                        ++sblk;
+                    } else if (valid)
                         store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, 0, v);
                     float cm = -INFINITY;
 #pragma unroll
@@ -596,6 +655,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 mbar_arrive(&tempty[acc]);
             }
         }
+        // the logits blocks this warp stored must be complete before the CTA exits
+        if (EPI == EPI_LOGITS_STG && lane == 0) bulk_wait_group<0>();
     }
 
     __syncthreads();
@@ -630,7 +691,8 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // 2-D bf16 tensor map: `inner` contiguous elements per row, `outer` rows of
 // pitch `ld` elements; box of box_inner x box_outer with 128-byte swizzle.
 static bool make_map(CUtensorMap* map, const void* ptr, int64_t inner, int64_t outer, int64_t ld,
-                     uint32_t box_inner, uint32_t box_outer) {
+                     uint32_t box_inner, uint32_t box_outer,
+                     CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
     auto fn = encode_fn();
     if (!fn) return false;
     if ((reinterpret_cast<uintptr_t>(ptr) & 15u) != 0) return false;
@@ -640,7 +702,7 @@ static bool make_map(CUtensorMap* map, const void* ptr, int64_t inner, int64_t o
     cuuint32_t box[2] = {box_inner, box_outer};
     cuuint32_t estr[2] = {1, 1};
     CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
@@ -810,6 +872,9 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
             return BOM_ENOTSUP;
         }
     }
+    if (g.epi_kind == EPI_LOGITS && !g.epi.out_f32 &&
+        !make_map(&p.mapOut, g.epi.out, g.N, g.M, g.epi.ld_out, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
+        return BOM_ENOTSUP;
     p.M = static_cast<int>(g.M);
     p.N = static_cast<int>(g.N);
     p.nseg = g.nseg;

@@ -19,7 +19,7 @@ constexpr int kResidRows = 32;
 inline int64_t resid_blocks(int64_t n) { return (n + kResidRows - 1) / kResidRows; }
 
 // Counts N_t, checks every label, latches BOM_ELABEL / BOM_EEMPTY and writes
-// the cotangent coefficients of the three passes into sc.
+// the cotangent coefficients of the four backward passes into sc.
 void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda,
                         DevScalars* sc, cudaStream_t s);
 
@@ -44,8 +44,23 @@ void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, cons
 void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float inv_bc1, float* q,
                       float* s_out, float* qhat, DevScalars* sc, cudaStream_t s);
 
-// loss = N_t^-1 sum_i ce_i and ||s||.
-void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, DevScalars* sc, cudaStream_t s);
+// loss = N_t^-1 sum_i ce_i, ||s|| and, when rnorm is given, r_norm_mean = N_t^-1 sum_i rnorm_i.
+void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, const float* rnorm, DevScalars* sc,
+                    cudaStream_t s);
+
+// rnorm[i] = ||R[i, 0:V]||_2 (one warp per row).
+void launch_row_norm(const void* R, int r_f32, int64_t ldr, int64_t n, int64_t V, float* rnorm, const DevScalars* sc,
+                     cudaStream_t s);
+
+// Grid of the own-step moment pass for n elements on a device with `sms` SMs;
+// the pass needs 4 * own_step_blocks(n) doubles of partials.
+constexpr int kOwnStepMaxBlocks = 1024;
+int own_step_blocks(int64_t n, int sms);
+
+// M <- beta1 M + (1-beta1) o; mhat = M * inv_bc1; when sums is given (and hv),
+// sums[0..3] += (<mhat,hv>, <mhat,mhat>, <hv,hv>, <mhat-hv,mhat-hv>) in a fixed order.
+void launch_own_step_moment(float* M, const float* o, const float* hv, float* mhat, int64_t n, float beta1,
+                            float inv_bc1, double* part, int nblocks, double* sums, cudaStream_t s);
 
 // out[j] = scale * sum_i w_i X[i, j]  (w_i = 1, the row mask from labels, or wvec[i]).
 // `part` must hold row_blocks(n) * d floats.
@@ -56,6 +71,11 @@ void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, 
 // out[j] = a * s[j] + b * qhat[j] (head bias numerator).
 void launch_axpby(const float* s_vec, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
                   const DevScalars* sc, cudaStream_t s);
+
+// BOM-Adam-mini update with one second moment per block (see bom_update_blockshared in bom.h).
+int launch_update_blockshared(float* theta, const void* g, int g_bf16, const float* h, float* vb, uint16_t* shadow,
+                              int64_t n, int64_t block, float lr, float wd, float lambda, float beta2, float eps,
+                              float inv_bc2, cudaStream_t s);
 
 // BOM-AdamW update (see bom_update in bom.h).
 int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,

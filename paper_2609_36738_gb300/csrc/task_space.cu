@@ -3,6 +3,8 @@
 // statistics, the residual pass r = softmax(z) - onehot(y) with deterministic
 // column partial sums, s_t and the q_t EMA with bias correction, and the
 // column reductions colsum_{I_t}(H), W^T qhat and bias gradients.
+#include <algorithm>
+
 #include "kernels.h"
 
 namespace bom {
@@ -32,18 +34,19 @@ __device__ __forceinline__ int warp_sum_i(int v) {
 __device__ __forceinline__ float fixed_order_column_sum(const float* __restrict__ part, int64_t nblocks,
                                                         int64_t ncols, int64_t col, float (*red)[33]) {
     const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
-    float a0 = 0.0f, a1 = 0.0f, a2 = 0.0f, a3 = 0.0f;
+    // eight independent loads in flight per thread: the pass is latency-bound
+    float a[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) a[k] = 0.0f;
     if (col < ncols) {
         int64_t b = w;
-        for (; b + 24 < nblocks; b += 32) {
-            a0 += part[b * ncols + col];
-            a1 += part[(b + 8) * ncols + col];
-            a2 += part[(b + 16) * ncols + col];
-            a3 += part[(b + 24) * ncols + col];
+        for (; b + 56 < nblocks; b += 64) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) a[k] += part[(b + 8 * k) * ncols + col];
         }
-        for (; b < nblocks; b += 8) a0 += part[b * ncols + col];
+        for (; b < nblocks; b += 8) a[0] += part[b * ncols + col];
     }
-    red[w][l] = (a0 + a1) + (a2 + a3);
+    red[w][l] = ((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]));
     __syncthreads();
     float r = 0.0f;
     if (w == 0) {
@@ -108,8 +111,11 @@ __global__ void labels_scan_kernel(const int32_t* __restrict__ labels, int64_t n
         sc->coef_q[1] = 0.0f;
         sc->coef_r[2] = 0.0f;                   // h pass: N_t^-1 qhat
         sc->coef_q[2] = inv;
+        sc->coef_r[3] = 0.0f;                   // own-step pass: N_t^-1 s_t
+        sc->coef_q[3] = inv;
         sc->loss = 0.0f;
         sc->s_norm = 0.0f;
+        sc->r_norm_mean = 0.0f;
     }
 }
 
@@ -160,7 +166,10 @@ __global__ void row_lse_kernel(const void* __restrict__ Z, int z_f32, int64_t ld
 // Block: 256 threads x VEC consecutive columns (one 16-byte word each) of
 // kResidRows rows.  The words of UNROLL rows are loaded before any is used and
 // stay packed until then, so a thread keeps 128 bytes in flight with few
-// registers and three blocks fit on an SM.
+// registers and three blocks fit on an SM.  The pass is issue-bound as much as
+// HBM-bound, so the bf16 form works on value pairs (paired fma / add, one
+// exponential per value), decides row validity once per row and subtracts the
+// one-hot only in the thread whose columns hold the label.
 template <typename T, int VEC>
 __global__ void __launch_bounds__(256, 3) residual_kernel(T* __restrict__ Z, int64_t ldz, int64_t n, int64_t V,
                                                           const float* __restrict__ lse,
@@ -170,11 +179,70 @@ __global__ void __launch_bounds__(256, 3) residual_kernel(T* __restrict__ Z, int
     const int64_t col0 = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) * VEC;
     const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kResidRows;
     const int64_t r1 = min(r0 + kResidRows, n);
-    float csum[VEC];
+    if (col0 >= ldz) return;
+    constexpr int UNROLL = 8;
+    if constexpr (sizeof(T) == 2) {
+        static_assert(VEC == 8, "bf16 rows are handled as 16-byte words");
+        const bool full = col0 + VEC <= V;
+        float2 cs[4];
 #pragma unroll
-    for (int k = 0; k < VEC; ++k) csum[k] = 0.0f;
-    if (col0 < ldz) {
-        constexpr int UNROLL = 8;
+        for (int k = 0; k < 4; ++k) cs[k] = make_float2(0.0f, 0.0f);
+        const float2 l2 = make_float2(kLog2e, kLog2e);
+        for (int64_t rb = r0; rb < r1; rb += UNROLL) {
+            uint4 raw[UNROLL];
+#pragma unroll
+            for (int u = 0; u < UNROLL; ++u)
+                if (rb + u < r1) raw[u] = *reinterpret_cast<const uint4*>(Z + (rb + u) * ldz + col0);
+#pragma unroll
+            for (int u = 0; u < UNROLL; ++u) {
+                const int64_t r = rb + u;
+                if (r >= r1) break;
+                uint4* dst = reinterpret_cast<uint4*>(Z + r * ldz + col0);
+                const int32_t y = labels[r];
+                if (y == ignore) {   // ignored rows contribute nothing
+                    *dst = make_uint4(0u, 0u, 0u, 0u);
+                    continue;
+                }
+                const float Ls = lse[r] * kLog2e;
+                const float2 off = make_float2(-Ls, -Ls);
+                const uint32_t ws[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
+                float2 pr[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float2 x = fma2(make_float2(bf16_lo(ws[j]), bf16_hi(ws[j])), l2, off);
+                    pr[j] = make_float2(ex2_fast(x.x), ex2_fast(x.y));
+                }
+                if (!full) {   // the last word of the row reaches into the padding
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        if (col0 + 2 * j >= V) pr[j].x = 0.0f;
+                        if (col0 + 2 * j + 1 >= V) pr[j].y = 0.0f;
+                    }
+                }
+                const int64_t yy = static_cast<int64_t>(y) - col0;
+                if (yy >= 0 && yy < VEC) {   // this word holds the label column
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        if (yy == 2 * j) pr[j].x -= 1.0f;
+                        if (yy == 2 * j + 1) pr[j].y -= 1.0f;
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < 4; ++j) cs[j] = add2(cs[j], pr[j]);
+                *dst = make_uint4(cvt_bf16x2(pr[0].x, pr[0].y), cvt_bf16x2(pr[1].x, pr[1].y),
+                                  cvt_bf16x2(pr[2].x, pr[2].y), cvt_bf16x2(pr[3].x, pr[3].y));
+            }
+        }
+        float* out = colpart + static_cast<int64_t>(blockIdx.y) * V + col0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (col0 + 2 * j < V) out[2 * j] = cs[j].x;
+            if (col0 + 2 * j + 1 < V) out[2 * j + 1] = cs[j].y;
+        }
+    } else {
+        float csum[VEC];
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) csum[k] = 0.0f;
         for (int64_t rb = r0; rb < r1; rb += UNROLL) {
             uint4 raw[UNROLL];
 #pragma unroll
@@ -187,39 +255,18 @@ __global__ void __launch_bounds__(256, 3) residual_kernel(T* __restrict__ Z, int
                 const int32_t y = labels[r];
                 const bool valid = (y != ignore);
                 const float L = lse[r];
-                // bf16 logits: exp2 of a pre-scaled argument (the result is
-                // stored in bf16); fp32 logits keep the accurate expf.
-                const float Ls = L * 1.4426950408889634f;
                 const uint32_t ws[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
-                float z[VEC];
-                if constexpr (sizeof(T) == 2) {
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        z[2 * j] = __uint_as_float(ws[j] << 16);
-                        z[2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
-                    }
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) z[j] = __uint_as_float(ws[j]);
-                }
                 float rv[VEC];
 #pragma unroll
                 for (int k = 0; k < VEC; ++k) {
                     const int64_t c = col0 + k;
                     float p = 0.0f;
-                    if (valid && c < V)
-                        p = (sizeof(T) == 2) ? exp2f(fmaf(z[k], 1.4426950408889634f, -Ls)) : expf(z[k] - L);
+                    if (valid && c < V) p = expf(__uint_as_float(ws[k]) - L);
                     if (valid && c == y) p -= 1.0f;
                     rv[k] = p;
                     csum[k] += p;
                 }
-                T* dst = Z + r * ldz + col0;
-                if constexpr (sizeof(T) == 2) {
-                    *reinterpret_cast<uint4*>(dst) = make_uint4(pack_bf16x2(rv[0], rv[1]), pack_bf16x2(rv[2], rv[3]),
-                                                                pack_bf16x2(rv[4], rv[5]), pack_bf16x2(rv[6], rv[7]));
-                } else {
-                    *reinterpret_cast<float4*>(dst) = make_float4(rv[0], rv[1], rv[2], rv[3]);
-                }
+                *reinterpret_cast<float4*>(Z + r * ldz + col0) = make_float4(rv[0], rv[1], rv[2], rv[3]);
             }
         }
 #pragma unroll
@@ -245,7 +292,8 @@ __global__ void __launch_bounds__(256) finish_sq_kernel(const float* __restrict_
 }
 
 __global__ void __launch_bounds__(1024) scalars_kernel(const float* __restrict__ ce, int64_t n,
-                                                       const float* __restrict__ s_vec, int64_t V, DevScalars* sc) {
+                                                       const float* __restrict__ s_vec, int64_t V,
+                                                       const float* __restrict__ rnorm, DevScalars* sc) {
     __shared__ float red[32];
     if (sc->status != 0) return;
     float a = 0.0f;
@@ -254,10 +302,79 @@ __global__ void __launch_bounds__(1024) scalars_kernel(const float* __restrict__
     float b = 0.0f;
     for (int64_t j = threadIdx.x; j < V; j += 1024) b += s_vec[j] * s_vec[j];
     b = block_sum<1024>(b, red);
+    float c = 0.0f;
+    if (rnorm) {
+        for (int64_t i = threadIdx.x; i < n; i += 1024) c += rnorm[i];
+        c = block_sum<1024>(c, red);
+    }
     if (threadIdx.x == 0) {
         sc->loss = a * sc->inv_nt;
         sc->s_norm = sqrtf(b);
+        sc->r_norm_mean = c * sc->inv_nt;
     }
+}
+
+// ||r_i|| of every row of R (0 on ignored rows, whose residual is zero): one
+// warp per row, lane-strided fp32 sums reduced by a fixed shuffle tree.
+template <typename T>
+__global__ void __launch_bounds__(256) row_norm_kernel(const T* __restrict__ R, int64_t ldr, int64_t n, int64_t V,
+                                                       float* __restrict__ rnorm, const DevScalars* sc) {
+    if (sc->status != 0) return;
+    const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int l = threadIdx.x & 31;
+    if (row >= n) return;
+    const T* r = R + row * ldr;
+    float a = 0.0f;
+    for (int64_t j = l; j < V; j += 32) {
+        const float x = ld_elem(r, j, sizeof(T) == 4);
+        a = fmaf(x, x, a);
+    }
+    a = warp_sum(a);
+    if (l == 0) rnorm[row] = sqrtf(a);
+}
+
+// Own-step moment and drift sums over a flat range (see bom_own_step_moment):
+// per-thread fp32 sums, then per-block fp64 partials in a fixed slot each.
+__global__ void __launch_bounds__(256) own_step_moment_kernel(float* __restrict__ M, const float* __restrict__ o,
+                                                              const float* __restrict__ hv, float* __restrict__ mhat,
+                                                              int64_t n, float beta1, float inv_bc1,
+                                                              double* __restrict__ part) {
+    float s_dot = 0.0f, s_mm = 0.0f, s_hh = 0.0f, s_dd = 0.0f;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += stride) {
+        const float m = fmaf(beta1, M[i], (1.0f - beta1) * o[i]);
+        M[i] = m;
+        const float mh = m * inv_bc1;
+        mhat[i] = mh;
+        if (hv) {
+            const float h = hv[i];
+            const float d = mh - h;
+            s_dot = fmaf(mh, h, s_dot);
+            s_mm = fmaf(mh, mh, s_mm);
+            s_hh = fmaf(h, h, s_hh);
+            s_dd = fmaf(d, d, s_dd);
+        }
+    }
+    if (!part) return;
+    __shared__ double red[4][8];
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    const float v4[4] = {warp_sum(s_dot), warp_sum(s_mm), warp_sum(s_hh), warp_sum(s_dd)};
+    if (l == 0)
+        for (int k = 0; k < 4; ++k) red[k][w] = static_cast<double>(v4[k]);
+    __syncthreads();
+    if (threadIdx.x < 4) {
+        double acc = 0.0;
+        for (int k = 0; k < 8; ++k) acc += red[threadIdx.x][k];
+        part[4 * static_cast<int64_t>(blockIdx.x) + threadIdx.x] = acc;
+    }
+}
+
+// sums[k] += sum_b part[4b + k], in block order.
+__global__ void drift_finish_kernel(const double* __restrict__ part, int nblocks, double* __restrict__ sums) {
+    if (threadIdx.x >= 4) return;
+    double acc = 0.0;
+    for (int b = 0; b < nblocks; ++b) acc += part[4 * b + threadIdx.x];
+    sums[threadIdx.x] += acc;
 }
 
 // part[b, j] = sum_{i in row block b} w_i X[i, j].  A block covers 32 x VEC
@@ -394,8 +511,37 @@ void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float be
     finish_sq_kernel<<<cdiv(V, 32), 256, 0, s>>>(colpart, nblocks, V, beta1, inv_bc1, q, s_out, qhat, sc); count_launch();
 }
 
-void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, DevScalars* sc, cudaStream_t s) {
-    scalars_kernel<<<1, 1024, 0, s>>>(ce, n, s_vec, V, sc); count_launch();
+void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, const float* rnorm, DevScalars* sc,
+                    cudaStream_t s) {
+    scalars_kernel<<<1, 1024, 0, s>>>(ce, n, s_vec, V, rnorm, sc); count_launch();
+}
+
+void launch_row_norm(const void* R, int r_f32, int64_t ldr, int64_t n, int64_t V, float* rnorm, const DevScalars* sc,
+                     cudaStream_t s) {
+    const unsigned grid = static_cast<unsigned>(cdiv(n * 32, 256));
+    if (r_f32)
+        row_norm_kernel<float><<<grid, 256, 0, s>>>(static_cast<const float*>(R), ldr, n, V, rnorm, sc);
+    else
+        row_norm_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(R), ldr, n, V, rnorm,
+                                                             sc);
+    count_launch();
+}
+
+int own_step_blocks(int64_t n, int sms) {
+    int64_t b = cdiv(n, 256 * 16);
+    const int64_t cap = std::min<int64_t>(4 * static_cast<int64_t>(sms > 0 ? sms : 1), kOwnStepMaxBlocks);
+    b = b < cap ? b : cap;
+    return static_cast<int>(b < 1 ? 1 : b);
+}
+
+void launch_own_step_moment(float* M, const float* o, const float* hv, float* mhat, int64_t n, float beta1,
+                            float inv_bc1, double* part, int nblocks, double* sums, cudaStream_t s) {
+    own_step_moment_kernel<<<nblocks, 256, 0, s>>>(M, o, hv, mhat, n, beta1, inv_bc1, sums ? part : nullptr);
+    count_launch();
+    if (sums) {
+        drift_finish_kernel<<<1, 32, 0, s>>>(part, nblocks, sums);
+        count_launch();
+    }
 }
 
 void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, const int32_t* labels,

@@ -7,6 +7,14 @@
 // Each thread moves 4 elements per access with 128-bit (fp32) / 64-bit (bf16)
 // streaming loads and stores; the grid is a multiple of the SM count and
 // strides over the range.
+//
+// BOM-Adam-mini (Section 3.5, composition with Adam-mini) shares one second
+// moment per block of `block` consecutive elements:
+//   v_b  <- beta2 v_b + (1-beta2) mean_{i in b} u_i^2
+//   theta <- (1 - lr wd) theta - lr u / (sqrt(v_b / (1-beta2^t)) + eps)
+// One CTA per block (grid-stride over blocks): a first sweep forms sum u^2 in
+// a fixed order, thread 0 advances v_b, a second sweep applies the update; the
+// second sweep's reads of g and h hit L2.
 #include "kernels.h"
 
 namespace bom {
@@ -77,6 +85,114 @@ __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ theta, 
     }
 }
 
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// u of VEC consecutive elements starting at i.
+template <bool G_BF16, bool HAS_H, int VEC>
+__device__ __forceinline__ void load_u(const void* g, const float* h, int64_t i, float lam, float (&u)[VEC]) {
+    if constexpr (VEC == 4) {
+        if constexpr (G_BF16) {
+            const uint2 w = *(reinterpret_cast<const uint2*>(static_cast<const uint16_t*>(g) + i));
+            u[0] = __uint_as_float(w.x << 16);
+            u[1] = __uint_as_float(w.x & 0xFFFF0000u);
+            u[2] = __uint_as_float(w.y << 16);
+            u[3] = __uint_as_float(w.y & 0xFFFF0000u);
+        } else {
+            const float4 f = *(reinterpret_cast<const float4*>(static_cast<const float*>(g) + i));
+            u[0] = f.x; u[1] = f.y; u[2] = f.z; u[3] = f.w;
+        }
+        if constexpr (HAS_H) {
+            const float4 hh = *(reinterpret_cast<const float4*>(h + i));
+            const float hv[4] = {hh.x, hh.y, hh.z, hh.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) u[k] = (1.0f - lam) * u[k] + lam * hv[k];
+        }
+    } else {
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) {
+            float x = G_BF16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(g)[i + k])
+                             : static_cast<const float*>(g)[i + k];
+            if (HAS_H) x = (1.0f - lam) * x + lam * h[i + k];
+            u[k] = x;
+        }
+    }
+}
+
+template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
+__global__ void __launch_bounds__(256) update_blockshared_kernel(float* __restrict__ theta, const void* __restrict__ g,
+                                                                 const float* __restrict__ h, float* __restrict__ vb,
+                                                                 uint16_t* __restrict__ shadow, int64_t n,
+                                                                 int64_t block, UpdCoef c) {
+    __shared__ float red[8];
+    __shared__ float s_den;
+    const int64_t nb = (n + block - 1) / block;
+    for (int64_t b = blockIdx.x; b < nb; b += gridDim.x) {
+        const int64_t e0 = b * block;
+        const int64_t e1 = e0 + block < n ? e0 + block : n;
+        float acc = 0.0f;
+        for (int64_t i = e0 + static_cast<int64_t>(threadIdx.x) * VEC; i < e1; i += 256 * VEC) {
+            float u[VEC];
+            load_u<G_BF16, HAS_H, VEC>(g, h, i, c.lam, u);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) acc = fmaf(u[k], u[k], acc);
+        }
+        acc = warp_sum_f(acc);
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float tot = 0.0f;
+#pragma unroll
+            for (int w = 0; w < 8; ++w) tot += red[w];
+            const float vv = fmaf(c.beta2, vb[b], c.one_m_beta2 * (tot / static_cast<float>(e1 - e0)));
+            vb[b] = vv;
+            s_den = sqrtf(vv * c.inv_bc2) + c.eps;
+        }
+        __syncthreads();
+        const float den = s_den;
+        for (int64_t i = e0 + static_cast<int64_t>(threadIdx.x) * VEC; i < e1; i += 256 * VEC) {
+            float u[VEC];
+            load_u<G_BF16, HAS_H, VEC>(g, h, i, c.lam, u);
+            if constexpr (VEC == 4) {
+                float4 th = __ldcs(reinterpret_cast<const float4*>(theta + i));
+                th.x = c.decay * th.x - c.lr * (u[0] / den);
+                th.y = c.decay * th.y - c.lr * (u[1] / den);
+                th.z = c.decay * th.z - c.lr * (u[2] / den);
+                th.w = c.decay * th.w - c.lr * (u[3] / den);
+                __stcs(reinterpret_cast<float4*>(theta + i), th);
+                if constexpr (SHADOW) {
+                    uint2 sh;
+                    sh.x = pack_bf16x2(th.x, th.y);
+                    sh.y = pack_bf16x2(th.z, th.w);
+                    __stcs(reinterpret_cast<uint2*>(shadow + i), sh);
+                }
+            } else {
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) {
+                    const float th = c.decay * theta[i + k] - c.lr * (u[k] / den);
+                    theta[i + k] = th;
+                    if (SHADOW) reinterpret_cast<__nv_bfloat16*>(shadow)[i + k] = __float2bfloat16_rn(th);
+                }
+            }
+        }
+        __syncthreads();   // red and s_den are reused by the next block
+    }
+}
+
+template <bool G_BF16, bool HAS_H, int VEC>
+void dispatch_blockshared(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
+                          int64_t block, const UpdCoef& c, int grid, cudaStream_t s) {
+    if (shadow)
+        update_blockshared_kernel<G_BF16, HAS_H, true, VEC><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n, block, c);
+    else
+        update_blockshared_kernel<G_BF16, HAS_H, false, VEC><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n, block,
+                                                                                  c);
+    count_launch();
+}
+
 template <bool G_BF16, bool HAS_H>
 void dispatch_shadow(float* theta, const void* g, const float* h, float* v, uint16_t* shadow, int64_t n,
                      const UpdCoef& c, int grid, cudaStream_t s) {
@@ -114,6 +230,43 @@ int launch_update(float* theta, const void* g, int g_bf16, const float* h, float
     } else {
         if (h) dispatch_shadow<false, true>(theta, g, h, v, shadow, n, c, (int)grid, s);
         else dispatch_shadow<false, false>(theta, g, h, v, shadow, n, c, (int)grid, s);
+    }
+    return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+int launch_update_blockshared(float* theta, const void* g, int g_bf16, const float* h, float* vb, uint16_t* shadow,
+                              int64_t n, int64_t block, float lr, float wd, float lambda, float beta2, float eps,
+                              float inv_bc2, cudaStream_t s) {
+    if (n <= 0) return BOM_OK;
+    UpdCoef c;
+    c.lr = lr;
+    c.decay = 1.0f - lr * wd;
+    c.lam = lambda;
+    c.beta2 = beta2;
+    c.one_m_beta2 = 1.0f - beta2;
+    c.eps = eps;
+    c.inv_bc2 = inv_bc2;
+    const int64_t nb = (n + block - 1) / block;
+    int64_t grid = static_cast<int64_t>(device_sm_count()) * 8;
+    if (grid > nb) grid = nb;
+    const bool vec = (block % 4 == 0) && (n % 4 == 0);
+    const int gi = static_cast<int>(grid);
+    if (vec) {
+        if (g_bf16) {
+            if (h) dispatch_blockshared<true, true, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            else dispatch_blockshared<true, false, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
+        } else {
+            if (h) dispatch_blockshared<false, true, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            else dispatch_blockshared<false, false, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
+        }
+    } else {
+        if (g_bf16) {
+            if (h) dispatch_blockshared<true, true, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            else dispatch_blockshared<true, false, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
+        } else {
+            if (h) dispatch_blockshared<false, true, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            else dispatch_blockshared<false, false, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
+        }
     }
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }

@@ -124,7 +124,10 @@ def test_lm_block_with_swiglu_mlps_full_size():
 
 def test_vision_head_twenty_steps_full_size():
     """768 -> 3072 -> 768 -> 1000 classes, batch 256, bf16: 20 BOM steps, each
-    followed by the update of every tensor, against the oracle's trajectory."""
+    followed by the update of every tensor.  Every step is checked on the same
+    inputs the GPU step read (its bf16 parameters and q_{t-1}); the oracle also
+    runs its own fp64 trajectory, and the final master weights of the two
+    trajectories must agree."""
     wl = I.VISION_HEAD_BF16
     lr, b2, eps = 1e-3, 0.999, 1e-8
     F = lambda v: float(np.float32(v))
@@ -136,20 +139,28 @@ def test_vision_head_twenty_steps_full_size():
     vs = [torch.zeros(p.shape, dtype=torch.float32, device=G.DEV) for p in params]
     vo = [np.zeros(p.shape) for p in p64]
     q = np.zeros(wl.vocab)
+    worst = 0.0
     for t in range(1, wl.steps + 1):
         xb, y = I.make_batch(wl, seed=11, step=t)
+        p_in = [G.np64(p) for p in gpu.params]
+        q_in = G.np64(gpu.q)
         gout = gpu.step(xb, y, t)
-        # both sides compute with bf16 copies of their own master weights
-        # (fp32 on the GPU, fp64 here): the bf16-autocast protocol of the paper
-        oref = G.oracle_step(wl, [G.bf16_round(p) for p in p64], xb, y, q, t)
-        q = oref["q"]
-        assert gout["stats"]["n_t"] == oref["n_t"]
-        assert G.rel_l2(gout["q"], oref["q"]) < TOL
+        same = G.oracle_step(wl, p_in, xb, y, q_in, t)
+        assert gout["stats"]["n_t"] == same["n_t"]
+        assert G.rel_l2(gout["q"], same["q"]) < TOL
         for k in range(len(params)):
-            assert G.rel_l2(G.np64(gout["grads"][k]), oref["u"][k]) < TOL, (t, k)
+            err = G.rel_l2(G.np64(gout["grads"][k]), same["u"][k])
+            worst = max(worst, err)
+            assert err < TOL, (t, k, err)
             B.bom_update(master[k], gout["grads"][k], B.BOM_BF16, None, vs[k], gpu.params[k], master[k].numel(),
                          lr, wds[k], 0.5, b2, eps, t)
+        # the oracle's own trajectory computes with bf16 copies of its fp64
+        # master weights, as the GPU does with its fp32 ones (bf16 autocast)
+        oref = G.oracle_step(wl, [G.bf16_round(p) for p in p64], xb, y, q, t)
+        q = oref["q"]
+        for k in range(len(params)):
             p64[k], vo[k] = O.bom_update(p64[k], oref["u"][k], vo[k], F(lr), F(wds[k]), t, F(b2), F(eps))
         torch.cuda.synchronize()
+    print(f"vision head, 20 steps: worst per-step relative L2 of u {worst:.3e}")
     for k in range(len(params)):
         assert G.rel_l2(G.np64(master[k]), p64[k]) < TOL

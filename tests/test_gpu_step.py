@@ -66,7 +66,9 @@ def test_single_step_parity(name, mode):
 @pytest.mark.parametrize("name,steps", [("tiny_mlp_f32", 5), ("vision_small", 3), ("lm_mlp_small", 3)])
 def test_multi_step_trajectory(name, steps):
     """Several BOM steps, each followed by the update of every tensor (fp32
-    master parameters on the device, bf16 copies for the bf16 path)."""
+    master parameters on the device, bf16 copies for the bf16 path).  Each
+    step is checked on the inputs the GPU read, and the master weights against
+    the oracle's own trajectory."""
     wl = I.WORKLOADS[name]
     lr, b2, eps, lam = 1e-3, 0.999, 1e-8, 0.5
     wds = I.weight_decay_mask(wl, 0.01)
@@ -81,12 +83,16 @@ def test_multi_step_trajectory(name, steps):
     tol = G.TOL[wl.dtype]
     for t in range(1, steps + 1):
         x, y = I.make_batch(wl, seed=5, step=t)
+        p_in = [G.np64(p) for p in gpu.params]
+        q_in = G.np64(gpu.q)
         gout = gpu.step(x, y, t)
-        # bf16 workloads compute with bf16 copies of the master weights on both sides
+        # the step on the inputs the GPU read: its parameters and q_{t-1}
+        _compare_step(wl, gout, G.oracle_step(wl, p_in, x, y, q_in, t), tol, False)
+        # the oracle's own trajectory; bf16 workloads compute with bf16 copies
+        # of the master weights on both sides
         pin = [G.bf16_round(p) for p in p64] if wl.dtype == "bf16" else p64
         oref = G.oracle_step(wl, pin, x, y, q, t)
         q = oref["q"]
-        _compare_step(wl, gout, oref, tol, False)
         for k in range(len(params)):
             n = master[k].numel()
             gt = B.BOM_BF16 if wl.dtype == "bf16" else B.BOM_F32
