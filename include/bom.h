@@ -62,7 +62,9 @@ typedef enum { BOM_F32 = 0, BOM_BF16 = 1 } bom_dtype;
 typedef enum {
     BOM_LAYER_LINEAR = 0,       /* y = x W^T (+ b)                                         */
     BOM_LAYER_LINEAR_GELU = 1,  /* y = GELU(x W^T (+ b)), exact erf GELU                  */
-    BOM_LAYER_SWIGLU = 2        /* y = x + W_d (SiLU(x W_g^T) * (x W_u^T)); d_out = ffn    */
+    BOM_LAYER_SWIGLU = 2,       /* y = x + W_d (SiLU(x W_g^T) * (x W_u^T)); d_out = ffn    */
+    BOM_LAYER_RMSNORM = 3       /* y = x / sqrt(mean_j x_j^2 + 1e-6) * gamma; d_out = d_in,
+                                   no bias (the norm tensors of the language-model setting) */
 } bom_layer_kind;
 
 typedef enum {
@@ -110,6 +112,7 @@ typedef struct bom_handle bom_handle;
  *   for each backbone layer:
  *     LINEAR / LINEAR_GELU : W [d_out, d_in], then b [d_out] if has_bias
  *     SWIGLU               : W_g [ffn, d], W_u [ffn, d], W_d [d, ffn]
+ *     RMSNORM              : gamma [d]
  *   head                   : W [d_out, d_model], then b [d_out] if head_bias
  * bom_param_count returns the number of tensors (-1 for a malformed cfg);
  * bom_param_shape the shape of tensor `index`: rows x cols for matrices, and
@@ -215,6 +218,23 @@ bom_status bom_update(float* theta, const void* g, int32_t g_dtype, const float*
  *   v_blocks    [ceil(n / block)] fp32, updated in place (v_0 = 0).
  * Other arguments as bom_update.  block >= 1; sums of u^2 are formed per
  * block in a fixed order (deterministic). */
+/* Global-norm clipping of the numerator (pretraining-parameters appendix:
+ * language-modeling runs clip at 1.0; convergence appendix: the clipped
+ * numerator is what the adaptive update receives).  Two calls:
+ *   bom_sqnorm          *sq += sum u_i^2 over a flat range (u = g, or
+ *                       (1-lambda) g + lambda hvec when hvec is given), in fp64
+ *                       and a fixed order; call it for every range of the
+ *                       clipping group into one zeroed device double;
+ *   bom_update_clipped  bom_update with u scaled first by
+ *                       c = min(1, max_norm / (sqrt(*sq) + 1e-6)).
+ * bom_sqnorm uses the handle's partials buffer: calls on one handle must be
+ * ordered on one stream.  max_norm > 0; other arguments as bom_update. */
+bom_status bom_sqnorm(bom_handle* h, const void* g, int32_t g_dtype, const float* hvec, float lambda, int64_t n,
+                      double* sq, void* stream);
+bom_status bom_update_clipped(float* theta, const void* g, int32_t g_dtype, const float* hvec, float* v,
+                              uint16_t* theta_bf16, int64_t n, float lr, float wd, float lambda, float beta2,
+                              float eps, int64_t t, const double* sq, float max_norm, void* stream);
+
 bom_status bom_update_blockshared(float* theta, const void* g, int32_t g_dtype, const float* hvec, float* v_blocks,
                                   uint16_t* theta_bf16, int64_t n, int64_t block, float lr, float wd, float lambda,
                                   float beta2, float eps, int64_t t, void* stream);

@@ -41,9 +41,10 @@ per-dataset-results appendix, with the equations of Section 3):
      convergence appendices).
 
 Backbone layers supported (shapes of the paper's settings; see the workload
-module): Linear, Linear+GELU (exact erf form) and the SwiGLU MLP sublayer
-x <- x + W_d (SiLU(W_g x) * W_u x).  The head is Linear d -> d_out, with an
-optional bias.
+module): Linear, Linear+GELU (exact erf form), the SwiGLU MLP sublayer
+x <- x + W_d (SiLU(W_g x) * W_u x) and RMSNorm x / sqrt(mean x^2 + 1e-6) * gamma
+(the norm tensors of the language-model setting).  The head is Linear
+d -> d_out, with an optional bias.
 
 Every function here is pinned by ``tests/test_oracle_pins.py`` against facts
 the paper or mathematics fix (finite-difference Jacobians and the exact batch
@@ -104,11 +105,17 @@ def silu_prime(x):
     return sg * (1.0 + x * (1.0 - sg))
 
 
+# RMSNorm (the norm tensors of the paper's Qwen3 language models, weight decay
+# 0): y = x / sqrt(mean_j x_j^2 + eps) * gamma with the Qwen3 epsilon.
+RMS_EPS = 1e-6
+
+
 # --------------------------------------------------------------------------
 # Model: layers are (kind, d_in, d_out, has_bias) with kind in
-# {"linear", "linear_gelu", "swiglu"}; parameters are listed per layer
-# (W [d_out, d_in], b [d_out]) or (W_gate [ffn, d], W_up [ffn, d],
-# W_down [d, ffn]) followed by the head (W [d_out, d], optional b).
+# {"linear", "linear_gelu", "swiglu", "rmsnorm"}; parameters are listed per
+# layer (W [d_out, d_in], b [d_out]), (W_gate [ffn, d], W_up [ffn, d],
+# W_down [d, ffn]) or (gamma [d]), followed by the head (W [d_out, d],
+# optional b).
 # --------------------------------------------------------------------------
 def _split_params(layers, head_bias, params):
     it = iter(params)
@@ -116,6 +123,8 @@ def _split_params(layers, head_bias, params):
     for kind, d_in, d_out, has_bias in layers:
         if kind == "swiglu":
             per_layer.append((next(it), next(it), next(it)))
+        elif kind == "rmsnorm":
+            per_layer.append((next(it),))
         else:
             w = next(it)
             b = next(it) if has_bias else None
@@ -142,6 +151,12 @@ def forward(layers, head_bias, params, X):
             y = x + A @ wd.T
             tape.append(("swiglu", x, G, U, A))
             x = y
+        elif kind == "rmsnorm":
+            (gamma,) = p
+            r = 1.0 / np.sqrt(np.mean(x * x, axis=1, keepdims=True) + RMS_EPS)
+            xhat = x * r
+            tape.append(("rmsnorm", x, r, xhat))
+            x = xhat * gamma
         else:
             w, b = p
             pre = x @ w.T
@@ -186,6 +201,13 @@ def backward(layers, head_bias, params, saved, dZ):
             g_wu = dU.T @ x
             dx = dy + dG @ wg + dU @ wu
             grads_rev.extend([g_wd, g_wu, g_wg])
+        elif kind == "rmsnorm":
+            (gamma,) = per_layer[li]
+            _, x, r, xhat = rec
+            grads_rev.append((dx * xhat).sum(axis=0))
+            dxhat = dx * gamma
+            # d/dx of x r(x): r (dxhat - xhat mean_j(dxhat_j xhat_j))
+            dx = r * (dxhat - xhat * np.mean(dxhat * xhat, axis=1, keepdims=True))
         else:
             w, b = per_layer[li]
             _, x, pre = rec

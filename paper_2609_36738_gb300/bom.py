@@ -22,14 +22,15 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libbom.so")
 
 BOM_OK, BOM_EINVAL, BOM_ENOMEM, BOM_ECUDA, BOM_ELABEL, BOM_EEMPTY, BOM_ETIMEOUT, BOM_ENOTSUP = range(8)
 BOM_F32, BOM_BF16 = 0, 1
-BOM_LAYER_LINEAR, BOM_LAYER_LINEAR_GELU, BOM_LAYER_SWIGLU = 0, 1, 2
+BOM_LAYER_LINEAR, BOM_LAYER_LINEAR_GELU, BOM_LAYER_SWIGLU, BOM_LAYER_RMSNORM = 0, 1, 2, 3
 BOM_OUT_U, BOM_OUT_G_AND_H = 0, 1
 
 # Every symbol include/bom.h declares.
 EXPORTED = ("bom_param_count", "bom_param_shape", "bom_init", "bom_workspace_bytes", "bom_step",
             "bom_set_input_grad", "bom_step_outputs", "bom_get_stats", "bom_update", "bom_gemm_bf16", "bom_trace", "bom_trace_read",
             "bom_launch_count", "bom_colsum_noalloc", "bom_set_own_step_output", "bom_own_step_moment",
-            "bom_stats_transfer_bytes", "bom_update_blockshared", "bom_destroy", "bom_status_string")
+            "bom_stats_transfer_bytes", "bom_update_blockshared", "bom_sqnorm", "bom_update_clipped",
+            "bom_destroy", "bom_status_string")
 
 
 class bom_trace_entry(C.Structure):
@@ -106,6 +107,10 @@ def lib() -> C.CDLL:
     L.bom_stats_transfer_bytes.restype = i64
     L.bom_update_blockshared.argtypes = [vp, vp, i32, vp, vp, vp, i64, i64, f32, f32, f32, f32, f32, i64, vp]
     L.bom_update_blockshared.restype = i32
+    L.bom_sqnorm.argtypes = [vp, vp, i32, vp, f32, i64, vp, vp]
+    L.bom_sqnorm.restype = i32
+    L.bom_update_clipped.argtypes = [vp, vp, i32, vp, vp, vp, i64, f32, f32, f32, f32, f32, i64, vp, f32, vp]
+    L.bom_update_clipped.restype = i32
     L.bom_destroy.argtypes = [vp]
     L.bom_destroy.restype = None
     L.bom_status_string.argtypes = [i32]
@@ -154,7 +159,7 @@ def make_config(max_rows: int, d_in: int, d_out: int, layers: Sequence, head_bia
 
 
 _KIND = {_inputs.LINEAR: BOM_LAYER_LINEAR, _inputs.LINEAR_GELU: BOM_LAYER_LINEAR_GELU,
-         _inputs.SWIGLU: BOM_LAYER_SWIGLU}
+         _inputs.SWIGLU: BOM_LAYER_SWIGLU, _inputs.RMSNORM: BOM_LAYER_RMSNORM}
 
 
 def config_for(wl: "_inputs.Workload", lam: float = 0.5, beta1: float = 0.9, out_mode: int = BOM_OUT_U,
@@ -230,6 +235,18 @@ def bom_update_blockshared(theta, g, g_dtype: int, hvec, v_blocks, theta_bf16, n
     _check(lib().bom_update_blockshared(_ptr(theta), _ptr(g), int(g_dtype), _ptr(hvec), _ptr(v_blocks),
                                         _ptr(theta_bf16), int(n), int(block), float(lr), float(wd), float(lam),
                                         float(beta2), float(eps), int(t), _stream(stream)), "bom_update_blockshared")
+
+
+def bom_sqnorm(h, g, g_dtype: int, hvec, lam: float, n: int, sq, stream=None) -> None:
+    _check(lib().bom_sqnorm(h, _ptr(g), int(g_dtype), _ptr(hvec), float(lam), int(n), _ptr(sq), _stream(stream)),
+           "bom_sqnorm")
+
+
+def bom_update_clipped(theta, g, g_dtype: int, hvec, v, theta_bf16, n: int, lr: float, wd: float, lam: float,
+                       beta2: float, eps: float, t: int, sq, max_norm: float, stream=None) -> None:
+    _check(lib().bom_update_clipped(_ptr(theta), _ptr(g), int(g_dtype), _ptr(hvec), _ptr(v), _ptr(theta_bf16), int(n),
+                                    float(lr), float(wd), float(lam), float(beta2), float(eps), int(t), _ptr(sq),
+                                    float(max_norm), _stream(stream)), "bom_update_clipped")
 
 
 def bom_gemm_bf16(A, lda: int, a_mn_major: bool, B, ldb: int, b_mn_major: bool, D, ldd: int, M: int, N: int,

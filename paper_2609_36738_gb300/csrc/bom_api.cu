@@ -38,6 +38,7 @@ struct LayerWs {
     void* G = nullptr;       // SWIGLU gate pre-activation [n, ffn]
     void* U = nullptr;       // SWIGLU up projection [n, ffn]
     void* A = nullptr;       // SWIGLU SiLU(G) * U [n, ffn]
+    float* rstd = nullptr;   // RMSNORM 1 / sqrt(mean x^2 + eps) per row [n]
 };
 
 int64_t round_up(int64_t a, int64_t b) { return (a + b - 1) / b * b; }
@@ -125,6 +126,9 @@ bom_status check_config(const bom_config* cfg, std::vector<LayerWs>* lw_out, int
             mf = mf > L.d_out ? mf : L.d_out;
         } else if (L.kind == BOM_LAYER_LINEAR || L.kind == BOM_LAYER_LINEAR_GELU) {
             x.width_out = L.d_out;
+        } else if (L.kind == BOM_LAYER_RMSNORM) {
+            if (L.has_bias || L.d_out != L.d_in) return BOM_EINVAL;
+            x.width_out = L.d_in;
         } else {
             return BOM_EINVAL;
         }
@@ -170,10 +174,15 @@ size_t carve(bom_handle* h, char* base) {
             L.A = c.take(n * L.d_out * e);
         } else if (L.kind == BOM_LAYER_LINEAR_GELU) {
             L.pre = c.take(n * L.d_out * e);
+        } else if (L.kind == BOM_LAYER_RMSNORM) {
+            L.rstd = static_cast<float*>(c.take(n * 4));
         }
         L.out = c.take(n * L.width_out * e);
     }
-    h->ldz = round_up(V, 8);
+    // logits rows start on 128-byte boundaries: each 64-byte row segment an
+    // epilogue warp stores then covers whole 32-byte sectors (no partial-sector
+    // merges in L2) and the residual pass reads aligned lines
+    h->ldz = round_up(V, h->bf16 ? 64 : 32);
     h->Z = c.take(n * h->ldz * e);
     h->ntiles = h->bf16 ? tc_logit_tiles(V) : 1;
     h->stats = static_cast<float*>(c.take(n * h->ntiles * 8));
@@ -281,8 +290,10 @@ extern "C" {
 int32_t bom_param_count(const bom_config* cfg) {
     if (!cfg || cfg->n_layers < 0 || (cfg->n_layers > 0 && !cfg->layers)) return -1;
     int32_t k = 0;
-    for (int i = 0; i < cfg->n_layers; ++i)
-        k += cfg->layers[i].kind == BOM_LAYER_SWIGLU ? 3 : (cfg->layers[i].has_bias ? 2 : 1);
+    for (int i = 0; i < cfg->n_layers; ++i) {
+        const bom_layer& L = cfg->layers[i];
+        k += L.kind == BOM_LAYER_SWIGLU ? 3 : (L.kind == BOM_LAYER_RMSNORM ? 1 : (L.has_bias ? 2 : 1));
+    }
     return k + (cfg->head_bias ? 2 : 1);
 }
 
@@ -296,6 +307,8 @@ bom_status bom_param_shape(const bom_config* cfg, int32_t index, int64_t* rows, 
             const int64_t r[3] = {L.d_out, L.d_out, L.d_in}, c[3] = {L.d_in, L.d_in, L.d_out};
             for (int j = 0; j < 3; ++j, ++k)
                 if (k == index) { *rows = r[j]; *cols = c[j]; return BOM_OK; }
+        } else if (L.kind == BOM_LAYER_RMSNORM) {
+            if (k++ == index) { *rows = L.d_in; *cols = 0; return BOM_OK; }
         } else {
             if (k++ == index) { *rows = L.d_out; *cols = L.d_in; return BOM_OK; }
             if (L.has_bias && k++ == index) { *rows = L.d_out; *cols = 0; return BOM_OK; }
@@ -428,6 +441,10 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
             g2.epi.out = L.out;
             g2.epi.ld_out = d;
             BOM_TRY(run_gemm(h, g2, s));
+        } else if (L.kind == BOM_LAYER_RMSNORM) {
+            const void* gamma = params[pi++];
+            BOM_TRACED("rmsnorm_fwd", 4.0 * n * L.d_in, 2.0 * h->esz * n * L.d_in + 4.0 * n,
+                       launch_rmsnorm_fwd(xin, gamma, L.out, L.rstd, n, L.d_in, cf32, h->sc, s));
         } else {
             const void* W = params[pi++];
             const void* b = L.bias ? params[pi++] : nullptr;
@@ -605,6 +622,20 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                     BOM_TRY(run_gemm(h, g, s));
                     cur ^= 1;
                 }
+            } else if (L.kind == BOM_LAYER_RMSNORM) {
+                const int64_t d = L.d_in;
+                const void* gamma = params[p0];
+                // dgamma_j = sum_i rstd_i dy_ij x_ij
+                BOM_TRACED("colsum", 3.0 * n * d, 2.0 * h->esz * n * d,
+                           launch_colsum2(dcur, xl, cf32, d, n, d, nullptr, 0, L.rstd, 1.0f, h->part, outp[p0], of32,
+                                          h->sc, s));
+                if (prev || want_dx) {
+                    const void* pre = (prev && prev->kind == BOM_LAYER_LINEAR_GELU) ? prev->pre : nullptr;
+                    void* dxo = prev ? h->dx[cur ^ 1] : h->dx_in;
+                    BOM_TRACED("rmsnorm_bwd", 8.0 * n * d, 3.0 * h->esz * n * d + 4.0 * n,
+                               launch_rmsnorm_bwd(dcur, xl, gamma, L.rstd, pre, dxo, n, d, cf32, h->sc, s));
+                    cur ^= 1;
+                }
             } else {
                 const void* W = params[p0];
                 {   // dW = dPre^T x
@@ -709,7 +740,35 @@ bom_status bom_update(float* theta, const void* g, int32_t g_dtype, const float*
         return BOM_ENOTSUP;
     const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
     return static_cast<bom_status>(launch_update(theta, g, g_dtype == BOM_BF16, hvec, v, theta_bf16, n, lr, wd,
-                                                 lambda, beta2, eps, inv_bc2, static_cast<cudaStream_t>(stream)));
+                                                 lambda, beta2, eps, inv_bc2, nullptr, 0.0f,
+                                                 static_cast<cudaStream_t>(stream)));
+}
+
+bom_status bom_sqnorm(bom_handle* h, const void* g, int32_t g_dtype, const float* hvec, float lambda, int64_t n,
+                      double* sq, void* stream) {
+    if (!h || n < 0 || !sq) return BOM_EINVAL;
+    if (n == 0) return BOM_OK;
+    if (!g || (g_dtype != BOM_F32 && g_dtype != BOM_BF16)) return BOM_EINVAL;
+    if (!aligned16(g) || (hvec && !aligned16(hvec))) return BOM_ENOTSUP;
+    return static_cast<bom_status>(launch_sqnorm(g, g_dtype == BOM_BF16, hvec, lambda, n, h->tel_part, sq,
+                                                 static_cast<cudaStream_t>(stream)));
+}
+
+bom_status bom_update_clipped(float* theta, const void* g, int32_t g_dtype, const float* hvec, float* v,
+                              uint16_t* theta_bf16, int64_t n, float lr, float wd, float lambda, float beta2,
+                              float eps, int64_t t, const double* sq, float max_norm, void* stream) {
+    if (n < 0 || t < 1 || !sq || !(max_norm > 0.0f)) return BOM_EINVAL;
+    if (n == 0) return BOM_OK;
+    if (!theta || !g || !v) return BOM_EINVAL;
+    if (g_dtype != BOM_F32 && g_dtype != BOM_BF16) return BOM_EINVAL;
+    if (!(beta2 >= 0.0f && beta2 < 1.0f) || !(eps >= 0.0f)) return BOM_EINVAL;
+    if (!aligned16(theta) || !aligned16(g) || !aligned16(v) || (hvec && !aligned16(hvec)) ||
+        (theta_bf16 && !aligned16(theta_bf16)))
+        return BOM_ENOTSUP;
+    const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
+    return static_cast<bom_status>(launch_update(theta, g, g_dtype == BOM_BF16, hvec, v, theta_bf16, n, lr, wd,
+                                                 lambda, beta2, eps, inv_bc2, sq, max_norm,
+                                                 static_cast<cudaStream_t>(stream)));
 }
 
 bom_status bom_update_blockshared(float* theta, const void* g, int32_t g_dtype, const float* hvec, float* v_blocks,

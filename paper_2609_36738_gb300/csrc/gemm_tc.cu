@@ -41,7 +41,6 @@ constexpr int GROUP_M = 8;
 struct Params {
     CUtensorMap mapA[2];
     CUtensorMap mapB[2];
-    CUtensorMap mapOut;    // staged logits output: 32 x 32 boxes, 64-byte swizzle
     int M, N;
     int kb[2];
     int nseg;
@@ -160,32 +159,6 @@ __device__ __forceinline__ void stg_scatter(void* base, int64_t ld, int row0, in
     stg_scatter_bf16(base, ld, row0, M, n, N, stg, b);
 }
 
-// Logits output through TMA: lane l writes row l of a 32 x 32 bf16 block into
-// `buf` in the 64-byte swizzled layout of mapOut (16-byte chunk k of row r at
-// r * 64 + 16 * (k ^ ((r >> 1) & 3)): no bank conflicts), then lane 0 stores
-// the block with one bulk copy, which clips rows >= M and columns >= N, under
-// the given L2 policy.  Two
-// buffers per warp alternate; before one is rewritten, lane 0 waits until the
-// store issued from it has finished reading it.
-constexpr int kTmaStgBytes = 32 * 64;
-__device__ __forceinline__ void tma_store_block(const CUtensorMap* map, uint8_t* buf, int x, int y,
-                                                const uint32_t (&b)[16], uint64_t policy) {
-    const int lane = threadIdx.x & 31;
-    if (lane == 0) bulk_wait_group_read<1>();
-    __syncwarp();
-    const int sw = (lane >> 1) & 3;
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-        *reinterpret_cast<uint4*>(buf + lane * 64 + 16 * (k ^ sw)) =
-            make_uint4(b[4 * k], b[4 * k + 1], b[4 * k + 2], b[4 * k + 3]);
-    fence_proxy_async_shared();
-    __syncwarp();
-    if (lane == 0) {
-        tma_store_2d_hint(map, buf, x, y, policy);
-        bulk_commit_group();
-    }
-}
-
 __device__ __forceinline__ float fast_exp(float x) { return exp2f(x * 1.4426950408889634f); }
 __device__ __forceinline__ float fast_sigmoid(float x) { return __frcp_rn(1.0f + fast_exp(-x)); }
 
@@ -210,11 +183,11 @@ constexpr int EPI_LOGITS_STG = 16;
 
 template <int CG, int EPI>
 struct Cfg {
-    static constexpr int NBUF = EPI == EPI_SWIGLU_FWD ? 3 : 0;
+    static constexpr int NBUF = EPI == EPI_SWIGLU_FWD ? 3 : EPI == EPI_LOGITS_STG ? 1 : 0;
     static constexpr int B_ROWS = CG == 2 ? 128 : 256;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
-    static constexpr int STG_BYTES = EPI == EPI_LOGITS_STG ? 8 * 2 * kTmaStgBytes : 8 * NBUF * kStgBytes;
+    static constexpr int STG_BYTES = 8 * NBUF * kStgBytes;
     // as many stages as fit in the 227 KB a CTA may use beside the staging
     // blocks, the 1 KB alignment slack and the barrier block, at most six (a
     // seventh 32 KB stage measured slower on the linear epilogues)
@@ -429,10 +402,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         const EpiParams& e = p.epi;
         constexpr int CPW = BN / 64;  // 32-column chunks per warp
         int it = 0;
-        int sblk = 0;   // TMA-stored logits blocks issued by this warp
-        // the logits stream (read back once, by the residual pass) must not
-        // evict the operand tiles that later output tiles reuse from L2
-        const uint64_t zpol = make_policy_evict_first();
         for (int w = unit; w < num_work; w += nunits, ++it) {
             const int tile = w / p.ksplit;
             // split-K: each K range stores its raw fp32 tile into its own slice
@@ -456,8 +425,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t ra = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid);
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
-            uint8_t* stg = EPI == EPI_LOGITS_STG ? stg_all + (warp - 2) * 2 * kTmaStgBytes
-                                                 : stg_all + (warp - 2) * C::NBUF * kStgBytes;
+            uint8_t* stg = stg_all + (warp - 2) * C::NBUF * kStgBytes;
             if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
             if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
             if (kb_total > 0) {
@@ -540,10 +508,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         uint32_t b[16];
 #pragma unroll
                         for (int i = 0; i < 16; ++i) b[i] = cvt_bf16x2(v[2 * i], v[2 * i + 1]);
-                        if constexpr (EPI == EPI_LOGITS_STG) {
-                            tma_store_block(&p.mapOut, stg + (sblk & 1) * kTmaStgBytes, n, row0, b, zpol);
-                            ++sblk;
-                        } else if (valid) {
+                        if constexpr (EPI == EPI_LOGITS_STG)
+                            stg_scatter_bf16(e.out, e.ld_out, row0, p.M, n, p.N, stg, b);
+                        else if (valid) {
                             uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(e.out) +
                                                                   static_cast<int64_t>(m) * e.ld_out + n);
 #pragma unroll
@@ -576,13 +543,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     // ragged last chunk
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = round_bf16(v[i]);
-                    if constexpr (EPI == EPI_LOGITS_STG) {
-                        uint32_t b[16];
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) b[i] = cvt_bf16x2(v[2 * i], v[2 * i + 1]);
-                        tma_store_block(&p.mapOut, stg + (sblk & 1) * kTmaStgBytes, n, row0, b, zpol);
-                        ++sblk;
-                    } else if (valid)
+                    if constexpr (EPI == EPI_LOGITS_STG)
+                        stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg, v);
+                    else if (valid)
                         store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, 0, v);
                     float cm = -INFINITY;
 #pragma unroll
@@ -655,8 +618,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 mbar_arrive(&tempty[acc]);
             }
         }
-        // the logits blocks this warp stored must be complete before the CTA exits
-        if (EPI == EPI_LOGITS_STG && lane == 0) bulk_wait_group<0>();
     }
 
     __syncthreads();
@@ -691,8 +652,7 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // 2-D bf16 tensor map: `inner` contiguous elements per row, `outer` rows of
 // pitch `ld` elements; box of box_inner x box_outer with 128-byte swizzle.
 static bool make_map(CUtensorMap* map, const void* ptr, int64_t inner, int64_t outer, int64_t ld,
-                     uint32_t box_inner, uint32_t box_outer,
-                     CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
+                     uint32_t box_inner, uint32_t box_outer) {
     auto fn = encode_fn();
     if (!fn) return false;
     if ((reinterpret_cast<uintptr_t>(ptr) & 15u) != 0) return false;
@@ -702,7 +662,7 @@ static bool make_map(CUtensorMap* map, const void* ptr, int64_t inner, int64_t o
     cuuint32_t box[2] = {box_inner, box_outer};
     cuuint32_t estr[2] = {1, 1};
     CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
@@ -872,9 +832,6 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
             return BOM_ENOTSUP;
         }
     }
-    if (g.epi_kind == EPI_LOGITS && !g.epi.out_f32 &&
-        !make_map(&p.mapOut, g.epi.out, g.N, g.M, g.epi.ld_out, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
-        return BOM_ENOTSUP;
     p.M = static_cast<int>(g.M);
     p.N = static_cast<int>(g.N);
     p.nseg = g.nseg;

@@ -68,6 +68,19 @@ void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, 
                    int32_t ignore, const float* wvec, float scale, float* part, void* out, int out_f32,
                    const DevScalars* sc, cudaStream_t s);
 
+// As launch_colsum with an elementwise second factor: out[j] = scale * sum_i w_i X[i, j] Y[i, j]
+// (Y has X's layout; Y = NULL is launch_colsum).
+void launch_colsum2(const void* X, const void* Y, int x_f32, int64_t ldx, int64_t n, int64_t d,
+                    const int32_t* labels, int32_t ignore, const float* wvec, float scale, float* part, void* out,
+                    int out_f32, const DevScalars* sc, cudaStream_t s);
+
+// RMSNorm (norm.cu): rstd[i] = 1 / sqrt(mean_j x_ij^2 + 1e-6), y = x rstd gamma.
+void launch_rmsnorm_fwd(const void* x, const void* gamma, void* y, float* rstd, int64_t n, int64_t d, int f32,
+                        const DevScalars* sc, cudaStream_t s);
+// dx = rstd (dy gamma - xhat mean_j(dy gamma xhat)), times GELU'(pre) when pre is given.
+void launch_rmsnorm_bwd(const void* dy, const void* x, const void* gamma, const float* rstd, const void* pre,
+                        void* dx, int64_t n, int64_t d, int f32, const DevScalars* sc, cudaStream_t s);
+
 // out[j] = a * s[j] + b * qhat[j] (head bias numerator).
 void launch_axpby(const float* s_vec, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
                   const DevScalars* sc, cudaStream_t s);
@@ -77,8 +90,15 @@ int launch_update_blockshared(float* theta, const void* g, int g_bf16, const flo
                               int64_t n, int64_t block, float lr, float wd, float lambda, float beta2, float eps,
                               float inv_bc2, cudaStream_t s);
 
-// BOM-AdamW update (see bom_update in bom.h).
+// BOM-AdamW update (see bom_update in bom.h).  With clip_sq, u is first scaled
+// by min(1, max_norm / (sqrt(*clip_sq) + 1e-6)) (bom_update_clipped).
 int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,
-                  float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, cudaStream_t s);
+                  float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, const double* clip_sq,
+                  float max_norm, cudaStream_t s);
+
+// *sq += sum u^2 over n elements (u = g, or (1-lambda) g + lambda h), in a fixed
+// order; `part` holds kOwnStepMaxBlocks doubles.
+int launch_sqnorm(const void* g, int g_bf16, const float* h, float lambda, int64_t n, double* part, double* sq,
+                  cudaStream_t s);
 
 }  // namespace bom

@@ -377,12 +377,14 @@ __global__ void drift_finish_kernel(const double* __restrict__ part, int nblocks
     sums[threadIdx.x] += acc;
 }
 
-// part[b, j] = sum_{i in row block b} w_i X[i, j].  A block covers 32 x VEC
-// columns of one row block: every warp reads 16-byte words of the same
-// columns, the 8 warps take interleaved rows, and the 8 warp sums are added
-// in a fixed order in shared memory (deterministic).
-template <typename T>
-__global__ void __launch_bounds__(256, 2) colsum_part_kernel(const T* __restrict__ X, int64_t ldx, int64_t n,
+// part[b, j] = sum_{i in row block b} w_i X[i, j] (times Y[i, j] when Y is
+// given, same layout as X).  A block covers 32 x VEC columns of one row
+// block: every warp reads 16-byte words of the same columns, the 8 warps take
+// interleaved rows, and the 8 warp sums are added in a fixed order in shared
+// memory (deterministic).
+template <typename T, bool HAS_Y>
+__global__ void __launch_bounds__(256, 2) colsum_part_kernel(const T* __restrict__ X, const T* __restrict__ Y,
+                                                             int64_t ldx, int64_t n,
                                                              int64_t d, const int32_t* __restrict__ labels,
                                                              int32_t ignore, const float* __restrict__ wvec,
                                                              float* __restrict__ part, const DevScalars* sc) {
@@ -398,45 +400,49 @@ __global__ void __launch_bounds__(256, 2) colsum_part_kernel(const T* __restrict
     for (int k = 0; k < VEC; ++k) acc[k] = 0.0f;
     const bool vec = (c0 + VEC <= d) && ((ldx % VEC) == 0);
     constexpr int UNROLL = 8;
+    auto load_word = [&](const T* src) {
+        if (vec) return *reinterpret_cast<const uint4*>(src);
+        uint32_t q[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) {
+            if (c0 + k >= d) continue;
+            if constexpr (sizeof(T) == 2)
+                q[k >> 1] |= static_cast<uint32_t>(reinterpret_cast<const uint16_t*>(src)[k]) << (16 * (k & 1));
+            else
+                q[k] = reinterpret_cast<const uint32_t*>(src)[k];
+        }
+        return make_uint4(q[0], q[1], q[2], q[3]);
+    };
+    auto elem = [](const uint4& w, int k) {
+        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+        if constexpr (sizeof(T) == 2)
+            return __uint_as_float((k & 1) ? (ws[k >> 1] & 0xFFFF0000u) : (ws[k >> 1] << 16));
+        else
+            return __uint_as_float(ws[k]);
+    };
     for (int64_t rb = r0 + w; rb < r1; rb += 8 * UNROLL) {
-        uint4 raw[UNROLL];
+        uint4 raw[UNROLL], raw2[HAS_Y ? UNROLL : 1];
         float wt[UNROLL];
 #pragma unroll
         for (int u = 0; u < UNROLL; ++u) {
             const int64_t r = rb + 8 * u;
             wt[u] = 0.0f;
             raw[u] = make_uint4(0u, 0u, 0u, 0u);
+            if constexpr (HAS_Y) raw2[u] = make_uint4(0u, 0u, 0u, 0u);
             if (r >= r1 || c0 >= d) continue;
             float wr = 1.0f;
             if (labels) wr = (labels[r] != ignore) ? 1.0f : 0.0f;
             if (wvec) wr = wvec[r];
             wt[u] = wr;
-            const T* src = X + r * ldx + c0;
-            if (vec) {
-                raw[u] = *reinterpret_cast<const uint4*>(src);
-            } else {
-                uint32_t q[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-                for (int k = 0; k < VEC; ++k) {
-                    if (c0 + k >= d) continue;
-                    if constexpr (sizeof(T) == 2)
-                        q[k >> 1] |= static_cast<uint32_t>(reinterpret_cast<const uint16_t*>(src)[k]) << (16 * (k & 1));
-                    else
-                        q[k] = reinterpret_cast<const uint32_t*>(src)[k];
-                }
-                raw[u] = make_uint4(q[0], q[1], q[2], q[3]);
-            }
+            raw[u] = load_word(X + r * ldx + c0);
+            if constexpr (HAS_Y) raw2[u] = load_word(Y + r * ldx + c0);
         }
 #pragma unroll
         for (int u = 0; u < UNROLL; ++u) {
-            const uint32_t ws[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
 #pragma unroll
             for (int k = 0; k < VEC; ++k) {
-                float x;
-                if constexpr (sizeof(T) == 2)
-                    x = __uint_as_float((k & 1) ? (ws[k >> 1] & 0xFFFF0000u) : (ws[k >> 1] << 16));
-                else
-                    x = __uint_as_float(ws[k]);
+                float x = elem(raw[u], k);
+                if constexpr (HAS_Y) x *= elem(raw2[u], k);
                 acc[k] = fmaf(wt[u], x, acc[k]);
             }
         }
@@ -547,15 +553,29 @@ void launch_own_step_moment(float* M, const float* o, const float* hv, float* mh
 void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, const int32_t* labels,
                    int32_t ignore, const float* wvec, float scale, float* part, void* out, int out_f32,
                    const DevScalars* sc, cudaStream_t s) {
+    launch_colsum2(X, nullptr, x_f32, ldx, n, d, labels, ignore, wvec, scale, part, out, out_f32, sc, s);
+}
+
+void launch_colsum2(const void* X, const void* Y, int x_f32, int64_t ldx, int64_t n, int64_t d,
+                    const int32_t* labels, int32_t ignore, const float* wvec, float scale, float* part, void* out,
+                    int out_f32, const DevScalars* sc, cudaStream_t s) {
     const int64_t nb = row_blocks(n);
     if (x_f32) {
         dim3 grid(cdiv(d, 128), static_cast<unsigned>(nb));
-        colsum_part_kernel<float><<<grid, 256, 0, s>>>(static_cast<const float*>(X), ldx, n, d, labels, ignore, wvec,
-                                                       part, sc);
+        auto x = static_cast<const float*>(X);
+        auto y = static_cast<const float*>(Y);
+        if (Y) colsum_part_kernel<float, true><<<grid, 256, 0, s>>>(x, y, ldx, n, d, labels, ignore, wvec, part, sc);
+        else colsum_part_kernel<float, false><<<grid, 256, 0, s>>>(x, y, ldx, n, d, labels, ignore, wvec, part, sc);
     } else {
         dim3 grid(cdiv(d, 256), static_cast<unsigned>(nb));
-        colsum_part_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(X), ldx, n, d,
-                                                               labels, ignore, wvec, part, sc);
+        auto x = static_cast<const __nv_bfloat16*>(X);
+        auto y = static_cast<const __nv_bfloat16*>(Y);
+        if (Y)
+            colsum_part_kernel<__nv_bfloat16, true><<<grid, 256, 0, s>>>(x, y, ldx, n, d, labels, ignore, wvec,
+                                                                         part, sc);
+        else
+            colsum_part_kernel<__nv_bfloat16, false><<<grid, 256, 0, s>>>(x, y, ldx, n, d, labels, ignore, wvec,
+                                                                          part, sc);
     }
     count_launch();
     colsum_finish_kernel<<<cdiv(d, 32), 256, 0, s>>>(part, nb, d, scale, out, out_f32, sc); count_launch();

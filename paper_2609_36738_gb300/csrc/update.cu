@@ -31,10 +31,17 @@ __device__ __forceinline__ float upd1(float& th, float& vv, float u, const UpdCo
     return th;
 }
 
-template <bool G_BF16, bool HAS_H, bool SHADOW>
+// Factor of global-norm clipping: min(1, max_norm / (||u|| + 1e-6)).
+__device__ __forceinline__ float clip_scale(const double* sq, float max_norm) {
+    return static_cast<float>(fmin(1.0, static_cast<double>(max_norm) / (sqrt(*sq) + 1e-6)));
+}
+
+template <bool G_BF16, bool HAS_H, bool SHADOW, bool CLIP>
 __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ theta, const void* __restrict__ g,
                                                      const float* __restrict__ h, float* __restrict__ v,
-                                                     uint16_t* __restrict__ shadow, int64_t n, UpdCoef c) {
+                                                     uint16_t* __restrict__ shadow, int64_t n, UpdCoef c,
+                                                     const double* __restrict__ clip_sq, float max_norm) {
+    const float cs = CLIP ? clip_scale(clip_sq, max_norm) : 1.0f;
     const int64_t n4 = n >> 2;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
@@ -59,6 +66,10 @@ __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ theta, 
             u[2] = om * u[2] + c.lam * hh.z;
             u[3] = om * u[3] + c.lam * hh.w;
         }
+        if constexpr (CLIP) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) u[k] *= cs;
+        }
         upd1(th.x, vv.x, u[0], c);
         upd1(th.y, vv.y, u[1], c);
         upd1(th.z, vv.z, u[2], c);
@@ -77,6 +88,7 @@ __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ theta, 
     if (t < n && t < (n4 << 2) + 4) {
         float u = G_BF16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(g)[t]) : static_cast<const float*>(g)[t];
         if (HAS_H) u = (1.0f - c.lam) * u + c.lam * h[t];
+        if (CLIP) u *= cs;
         float th = theta[t], vv = v[t];
         upd1(th, vv, u, c);
         theta[t] = th;
@@ -195,13 +207,60 @@ void dispatch_blockshared(float* theta, const void* g, const float* h, float* vb
 
 template <bool G_BF16, bool HAS_H>
 void dispatch_shadow(float* theta, const void* g, const float* h, float* v, uint16_t* shadow, int64_t n,
-                     const UpdCoef& c, int grid, cudaStream_t s) {
-    if (shadow) {
-        update_kernel<G_BF16, HAS_H, true><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c);
+                     const UpdCoef& c, int grid, const double* clip_sq, float max_norm, cudaStream_t s) {
+    if (clip_sq) {
+        if (shadow)
+            update_kernel<G_BF16, HAS_H, true, true><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, clip_sq,
+                                                                          max_norm);
+        else
+            update_kernel<G_BF16, HAS_H, false, true><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, clip_sq,
+                                                                           max_norm);
     } else {
-        update_kernel<G_BF16, HAS_H, false><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c);
+        if (shadow)
+            update_kernel<G_BF16, HAS_H, true, false><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, nullptr,
+                                                                           0.0f);
+        else
+            update_kernel<G_BF16, HAS_H, false, false><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, nullptr,
+                                                                            0.0f);
     }
     count_launch();
+}
+
+// sum u^2 over a flat range: per-thread fp32 sums, per-block fp64 partials in
+// fixed slots, then one block adds them in order to *sq.
+template <bool G_BF16, bool HAS_H>
+__global__ void __launch_bounds__(256) sqnorm_part_kernel(const void* __restrict__ g, const float* __restrict__ h,
+                                                          float lam, int64_t n, double* __restrict__ part) {
+    float acc = 0.0f;
+    const int64_t n4 = n >> 2;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
+        float u[4];
+        load_u<G_BF16, HAS_H, 4>(g, h, 4 * i, lam, u);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) acc = fmaf(u[k], u[k], acc);
+    }
+    if (blockIdx.x == 0 && threadIdx.x < (n & 3)) {
+        float u[1];
+        load_u<G_BF16, HAS_H, 1>(g, h, (n4 << 2) + threadIdx.x, lam, u);
+        acc = fmaf(u[0], u[0], acc);
+    }
+    __shared__ float red[8];
+    acc = warp_sum_f(acc);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < 8; ++w) t += static_cast<double>(red[w]);
+        part[blockIdx.x] = t;
+    }
+}
+
+__global__ void sqnorm_finish_kernel(const double* __restrict__ part, int nblocks, double* __restrict__ sq) {
+    if (threadIdx.x != 0) return;
+    double t = 0.0;
+    for (int b = 0; b < nblocks; ++b) t += part[b];
+    *sq += t;
 }
 
 }  // namespace
@@ -209,7 +268,8 @@ void dispatch_shadow(float* theta, const void* g, const float* h, float* v, uint
 int device_sm_count();
 
 int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,
-                  float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, cudaStream_t s) {
+                  float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, const double* clip_sq,
+                  float max_norm, cudaStream_t s) {
     if (n <= 0) return BOM_OK;
     UpdCoef c;
     c.lr = lr;
@@ -225,12 +285,37 @@ int launch_update(float* theta, const void* g, int g_bf16, const float* h, float
     if (grid > need) grid = need;
     if (grid < 1) grid = 1;
     if (g_bf16) {
-        if (h) dispatch_shadow<true, true>(theta, g, h, v, shadow, n, c, (int)grid, s);
-        else dispatch_shadow<true, false>(theta, g, h, v, shadow, n, c, (int)grid, s);
+        if (h) dispatch_shadow<true, true>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, s);
+        else dispatch_shadow<true, false>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, s);
     } else {
-        if (h) dispatch_shadow<false, true>(theta, g, h, v, shadow, n, c, (int)grid, s);
-        else dispatch_shadow<false, false>(theta, g, h, v, shadow, n, c, (int)grid, s);
+        if (h) dispatch_shadow<false, true>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, s);
+        else dispatch_shadow<false, false>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, s);
     }
+    return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+int sqnorm_blocks(int64_t n) {
+    int64_t b = static_cast<int64_t>(device_sm_count()) * 4;
+    const int64_t need = ((n >> 2) + 255) / 256;
+    if (b > need) b = need;
+    if (b > kOwnStepMaxBlocks) b = kOwnStepMaxBlocks;
+    return static_cast<int>(b < 1 ? 1 : b);
+}
+
+int launch_sqnorm(const void* g, int g_bf16, const float* h, float lambda, int64_t n, double* part, double* sq,
+                  cudaStream_t s) {
+    if (n <= 0) return BOM_OK;
+    const int nb = sqnorm_blocks(n);
+    if (g_bf16) {
+        if (h) sqnorm_part_kernel<true, true><<<nb, 256, 0, s>>>(g, h, lambda, n, part);
+        else sqnorm_part_kernel<true, false><<<nb, 256, 0, s>>>(g, h, lambda, n, part);
+    } else {
+        if (h) sqnorm_part_kernel<false, true><<<nb, 256, 0, s>>>(g, h, lambda, n, part);
+        else sqnorm_part_kernel<false, false><<<nb, 256, 0, s>>>(g, h, lambda, n, part);
+    }
+    count_launch();
+    sqnorm_finish_kernel<<<1, 32, 0, s>>>(part, nb, sq);
+    count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }
 

@@ -41,6 +41,7 @@ IGNORE_INDEX = -100
 LINEAR = "linear"
 LINEAR_GELU = "linear_gelu"
 SWIGLU = "swiglu"
+RMSNORM = "rmsnorm"
 
 
 # --------------------------------------------------------------------------
@@ -72,7 +73,7 @@ def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
 # --------------------------------------------------------------------------
 @dataclasses.dataclass(frozen=True)
 class Layer:
-    kind: str          # LINEAR, LINEAR_GELU or SWIGLU
+    kind: str          # LINEAR, LINEAR_GELU, SWIGLU or RMSNORM (d_out = d_in)
     d_in: int          # input width (d_model for SWIGLU)
     d_out: int         # output width (ffn width for SWIGLU; output stays d_model)
     has_bias: bool = False
@@ -109,6 +110,9 @@ class Workload:
                 out.append((f"l{li}.w_gate", (l.d_out, l.d_in), True))
                 out.append((f"l{li}.w_up", (l.d_out, l.d_in), True))
                 out.append((f"l{li}.w_down", (l.d_in, l.d_out), True))
+            elif l.kind == RMSNORM:
+                assert l.d_in == w and l.d_out == w
+                out.append((f"l{li}.norm_weight", (w,), False))
             else:
                 assert l.d_in == w
                 out.append((f"l{li}.weight", (l.d_out, l.d_in), True))
@@ -137,11 +141,15 @@ def init_params(wl: Workload, seed: int = 0) -> List[np.ndarray]:
 
     Matrices: Kaiming-uniform U(-sqrt(6/fan_in), +sqrt(6/fan_in)); the LM head
     uses N(0, 0.02) when ``head_init == "normal002"``.  Biases start at zero.
+    RMSNorm weights are 1 + N(0, 0.1^2) (not all ones, so that the weight's
+    own gradient path carries signal in the checks).
     """
     out = []
     for k, (name, shape, is_mat) in enumerate(wl.param_shapes()):
         g = _rng(seed, 1000 + k)
-        if not is_mat:
+        if name.endswith("norm_weight"):
+            x = (1.0 + 0.1 * g.standard_normal(shape)).astype(np.float32)
+        elif not is_mat:
             x = np.zeros(shape, dtype=np.float32)
         elif name == "head.weight" and wl.head_init == "normal002":
             x = (g.standard_normal(shape, dtype=np.float32) * np.float32(0.02))
@@ -178,7 +186,8 @@ def make_batch(wl: Workload, seed: int = 0, step: int = 1) -> Tuple[np.ndarray, 
 
 
 def weight_decay_mask(wl: Workload, omega: float) -> List[float]:
-    """Decoupled weight-decay coefficient per tensor: omega for matrices, 0 for biases."""
+    """Decoupled weight-decay coefficient per tensor: omega for matrices, 0 for
+    biases and normalisation weights."""
     return [omega if is_mat else 0.0 for _, _, is_mat in wl.param_shapes()]
 
 
@@ -215,8 +224,21 @@ TINY_RAGGED_F32 = Workload("tiny_ragged_f32", 37, 29, (Layer(LINEAR_GELU, 29, 45
 LM_HEAD_WIDE = Workload("lm_head_wide", 256, 128, (), 8192, False, "bf16", "zipf",
                         head_init="normal002", ignore_frac=0.05)
 
+# RMSNorm variants: an LM block whose head input is normalised (one SwiGLU
+# sublayer, then the final norm, as in the paper's Qwen3 models), and an fp32
+# MLP with a norm between two linear layers.
+LM_NORM_SMALL = Workload("lm_norm_small", 260, 128, (Layer(SWIGLU, 128, 320), Layer(RMSNORM, 128, 128)),
+                         777, False, "bf16", "zipf", head_init="normal002", ignore_frac=0.05)
+TINY_NORM_F32 = Workload("tiny_norm_f32", 37, 29, (Layer(LINEAR_GELU, 29, 45, True), Layer(RMSNORM, 45, 45),
+                                                    Layer(LINEAR, 45, 33, True)),
+                         7, True, "f32", "uniform", steps=3, ignore_frac=0.1)
+LM_NORM_BF16 = Workload("lm_norm_bf16", 16384, 2048,
+                        (Layer(SWIGLU, 2048, 8192), Layer(SWIGLU, 2048, 8192), Layer(RMSNORM, 2048, 2048)),
+                        32000, False, "bf16", "zipf", head_init="normal002")
+
 WORKLOADS = {w.name: w for w in (TINY_MLP_F32, VISION_HEAD_BF16, LM_HEAD_BF16, LM_MLP_BF16,
-                                  LM_HEAD_SMALL, LM_MLP_SMALL, VISION_SMALL, TINY_RAGGED_F32, LM_HEAD_WIDE)}
+                                  LM_HEAD_SMALL, LM_MLP_SMALL, VISION_SMALL, TINY_RAGGED_F32, LM_HEAD_WIDE,
+                                  LM_NORM_SMALL, TINY_NORM_F32, LM_NORM_BF16)}
 
 
 # --------------------------------------------------------------------------

@@ -36,6 +36,8 @@ def torch_forward(wl: I.Workload, params, X):
         if l.kind == I.SWIGLU:
             wg, wu, wd = next(it), next(it), next(it)
             x = x + F.linear(F.silu(F.linear(x, wg)) * F.linear(x, wu), wd)
+        elif l.kind == I.RMSNORM:
+            x = F.rms_norm(x, (l.d_in,), weight=next(it), eps=1e-6)
         else:
             w = next(it)
             b = next(it) if l.has_bias else None

@@ -43,7 +43,8 @@ def _compare_step(wl, gout, oref, tol, check_g_h):
             assert G.rel_l2(G.np64(u), ref) < tol, f"u[{k}] {G.rel_l2(G.np64(u), ref)}"
 
 
-@pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "lm_head_small", "vision_small",
+@pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "tiny_norm_f32", "lm_head_small",
+                                  "lm_norm_small", "vision_small",
                                   "lm_mlp_small"])
 @pytest.mark.parametrize("mode", [B.BOM_OUT_U, B.BOM_OUT_G_AND_H])
 def test_single_step_parity(name, mode):
@@ -63,7 +64,8 @@ def test_single_step_parity(name, mode):
     _compare_step(wl, gout, oref, G.TOL[wl.dtype], mode == B.BOM_OUT_G_AND_H)
 
 
-@pytest.mark.parametrize("name,steps", [("tiny_mlp_f32", 5), ("vision_small", 3), ("lm_mlp_small", 3)])
+@pytest.mark.parametrize("name,steps", [("tiny_mlp_f32", 5), ("vision_small", 3), ("lm_mlp_small", 3),
+                                        ("tiny_norm_f32", 3), ("lm_norm_small", 3)])
 def test_multi_step_trajectory(name, steps):
     """Several BOM steps, each followed by the update of every tensor (fp32
     master parameters on the device, bf16 copies for the bf16 path).  Each
@@ -151,7 +153,8 @@ def test_deterministic_reruns():
         assert torch.equal(ga, gb)
 
 
-@pytest.mark.parametrize("name", ["lm_head_small", "lm_mlp_small", "tiny_ragged_f32", "lm_head_wide"])
+@pytest.mark.parametrize("name", ["lm_head_small", "lm_mlp_small", "tiny_ragged_f32", "lm_head_wide",
+                                  "tiny_norm_f32", "lm_norm_small"])
 def test_input_cotangent(name):
     """bom_set_input_grad: the cotangent of X (for the head-only block this is
     dH, the input-side half of the head backward)."""

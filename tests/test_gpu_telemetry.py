@@ -37,7 +37,7 @@ def _groups(wl):
 
 
 @pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "vision_small", "lm_head_small",
-                                  "lm_mlp_small"])
+                                  "lm_mlp_small", "lm_norm_small"])
 def test_own_step_control_with_drift_telemetry(name):
     wl = I.WORKLOADS[name]
     tol = G.TOL[wl.dtype]

@@ -59,7 +59,7 @@ def test_param_count_matches_tiny_config():
 
 
 def test_forward_matches_independent_torch():
-    for wl in (I.TINY_MLP_F32, I.TINY_RAGGED_F32, I.VISION_SMALL, I.LM_MLP_SMALL):
+    for wl in (I.TINY_MLP_F32, I.TINY_RAGGED_F32, I.VISION_SMALL, I.LM_MLP_SMALL, I.TINY_NORM_F32, I.LM_NORM_SMALL):
         params, x, y, _, _ = _setup(wl)
         Z, _ = O.forward(X.oracle_layers(wl), wl.head_bias, params, x)
         Zt = X.torch_forward(wl, [torch.tensor(p) for p in params], torch.tensor(x)).numpy()
@@ -119,9 +119,10 @@ def test_u_decomposition_weights_printed_in_paper(tiny_jac):
 
 
 @pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "vision_small", "lm_mlp_small",
-                                  "lm_head_small"])
+                                  "lm_head_small", "tiny_norm_f32", "lm_norm_small"])
 def test_u_matches_autograd_of_mix_objective(name):
-    """One backward of L_mix (Eq. mix-objective) through torch autograd."""
+    """One backward of L_mix (Eq. mix-objective) through torch autograd (the
+    RMSNorm workloads go through torch.nn.functional.rms_norm)."""
     wl = I.WORKLOADS[name]
     params, x, y, q_prev, t = _setup(wl, seed=1)
     out = O.bom_step(X.oracle_layers(wl), wl.head_bias, params, x, y, q_prev, t, lam=0.5, beta1=0.9)
