@@ -4,7 +4,8 @@
 One timed step = one pass of the whole path over one batch: backbone forward
 (two SwiGLU MLP sublayers), logits + cross-entropy statistics, residuals, s_t,
 the q_t EMA, the head and backbone backward with the reprojection folded in,
-and the BOM-AdamW update of every parameter.  The workload is the largest
+and the BOM-AdamW update of every parameter (fused into the epilogues of the
+weight-gradient GEMMs; --separate-update runs it as its own pass).  The workload is the largest
 single-GPU configuration: 16384 tokens, d = 2048, ffn = 8192, vocabulary 32000,
 166,199,296 parameters (fp32 master weights, bf16 compute copies).
 
@@ -14,7 +15,8 @@ its launches inside the timed steps), the end-to-end number through host
 buffers, the clocks sampled during the timed region, and the oracle timed on
 the host cores on a bounded sample (cpu_baseline).  Two sub-measurements of the
 same metric family ride along: the head-only LM output block (8192 x 768 x
-50257) in tokens/s and the update alone over 1e9 elements in GB/s.
+50257) in tokens/s, the update alone over 1e9 elements in GB/s, and the
+BOM-Adam-mini update of the LM block's parameters in GB/s.
 
 --impl reference times the fp64 CPU oracle on the host cores instead (the
 only reference implementation this method has here).
@@ -54,6 +56,8 @@ def _args():
     p.add_argument("--workload", default="lm_mlp_bf16")
     p.add_argument("--no-extra", action="store_true", help="skip the head-only and update sub-measurements")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
+    p.add_argument("--separate-update", action="store_true",
+                   help="run bom_update after bom_step instead of the update fused into the step")
     p.add_argument("--tokens", type=int, default=0,
                    help="smaller batch of the same workload (profiling captures); 0 = the workload's own")
     return p.parse_args()
@@ -234,8 +238,10 @@ def main():
         vals = I.bf16_to_f32(p) if bf16 else p
         master[o:o + sizes[k]] = torch.from_numpy(vals.ravel()).to(dev)
     shadow.copy_(master.to(shadow.dtype))
-    pviews = [shadow[int(offs_al[k]):int(offs_al[k]) + sizes[k]].view(shapes[k]) for k in range(len(shapes))]
-    gviews = [gradf[int(offs_al[k]):int(offs_al[k]) + sizes[k]].view(shapes[k]) for k in range(len(shapes))]
+    def views(buf):
+        return [buf[int(offs_al[k]):int(offs_al[k]) + sizes[k]].view(shapes[k]) for k in range(len(shapes))]
+
+    pviews, gviews, thviews, vviews = views(shadow), views(gradf), views(master), views(vstate)
     x_np, y_np = I.make_batch(wl, seed=rank, step=1)
     x_host = torch.from_numpy(x_np.view(np.int16) if bf16 else x_np).pin_memory()
     y_host = torch.from_numpy(y_np).pin_memory()
@@ -247,9 +253,17 @@ def main():
     gt = B.BOM_BF16 if bf16 else B.BOM_F32
     N = wl.n_rows
 
+    fused = not a.separate_update
+    if fused:   # BOM-AdamW applied inside bom_step, in the epilogues of the weight-gradient GEMMs
+        B.bom_set_fused_update(model.h, thviews, vviews, I.weight_decay_mask(wl, WD), LR, B2, EPS)
+
     def step(t, xx=x_dev, yy=y_dev):
-        model.step(xx, yy, N, pviews, q, t, gviews, None, stream)
-        B.bom_update(master, gradf, gt, None, vstate, shadow if bf16 else None, P, LR, WD, LAM, B2, EPS, t, stream)
+        if fused:
+            model.step(xx, yy, N, pviews, q, t, None, None, stream)
+        else:
+            model.step(xx, yy, N, pviews, q, t, gviews, None, stream)
+            B.bom_update(master, gradf, gt, None, vstate, shadow if bf16 else None, P, LR, WD, LAM, B2, EPS, t,
+                         stream)
 
     t = 0
     loss_first = None
@@ -368,7 +382,8 @@ def main():
                 "config": {"workload": _workload_desc(wl), "global_batch": world * N, "tokens_per_gpu": N,
                            "parallelism": f"replicas x{world} (no data-path collective)",
                            "l2": "flushed between timed steps (256 MiB write outside the step events)",
-                           "lr": LR, "weight_decay": WD, "lambda": LAM, "beta1": B1, "beta2": B2},
+                           "lr": LR, "weight_decay": WD, "lambda": LAM, "beta1": B1, "beta2": B2,
+                           "update": "fused into the weight-gradient GEMM epilogues" if fused else "separate pass"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
                 "clocks": clk, "loss_first_step": loss_first, "loss": st["loss"], "kernels": kernels,
                 "sub": extra}

@@ -147,6 +147,26 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                     void* const* params, float* q, int64_t t,
                     void* const* grads, void* const* h_out, void* stream);
 
+/* Fused BOM-AdamW update (Section 3.4; Algorithm 1, last two steps) inside
+ * bom_step.  Registers, per parameter tensor, its fp32 master weights theta[k]
+ * and fp32 second moment v[k] (shapes as the parameters, 16-byte aligned) and
+ * its weight decay wd[k] (host array, copied).  Every following bom_step then
+ * applies
+ *   v <- beta2 v + (1-beta2) u^2,
+ *   theta <- (1 - lr wd) theta - lr u / (sqrt(v / (1-beta2^t)) + eps)
+ * to each tensor as soon as its u is complete.  For weight matrices this
+ * happens in the epilogue of the GEMM that forms u, which then writes the
+ * updated weights in the compute dtype into params[k] instead of writing u.
+ * params must therefore be writable, and grads may be NULL (nothing is
+ * written there).  Within the step every weight is last read before its
+ * update.  The numerator is the fp32 u of the accumulator, not a
+ * compute-dtype copy of it.  Requires BOM_OUT_U mode and no own-step output
+ * (bom_step returns BOM_EINVAL otherwise).  No update happens in a step whose
+ * device status latches an error.  lr usually changes per step: call this
+ * again before each step (host-side only).  theta = NULL disables it. */
+bom_status bom_set_fused_update(bom_handle* h, float* const* theta, float* const* v, const float* wd, float lr,
+                                float beta2, float eps);
+
 /* Registers a device buffer dx [max_rows, d_in] (compute dtype) that every
  * following bom_step fills with the cotangent of the input X (the u, or in
  * BOM_OUT_G_AND_H mode the g, cotangent): for a head-only configuration

@@ -30,7 +30,7 @@ EXPORTED = ("bom_param_count", "bom_param_shape", "bom_init", "bom_workspace_byt
             "bom_set_input_grad", "bom_step_outputs", "bom_get_stats", "bom_update", "bom_gemm_bf16", "bom_trace", "bom_trace_read",
             "bom_launch_count", "bom_colsum_noalloc", "bom_set_own_step_output", "bom_own_step_moment",
             "bom_stats_transfer_bytes", "bom_update_blockshared", "bom_sqnorm", "bom_update_clipped",
-            "bom_destroy", "bom_status_string")
+            "bom_set_fused_update", "bom_destroy", "bom_status_string")
 
 
 class bom_trace_entry(C.Structure):
@@ -111,6 +111,8 @@ def lib() -> C.CDLL:
     L.bom_sqnorm.restype = i32
     L.bom_update_clipped.argtypes = [vp, vp, i32, vp, vp, vp, i64, f32, f32, f32, f32, f32, i64, vp, f32, vp]
     L.bom_update_clipped.restype = i32
+    L.bom_set_fused_update.argtypes = [vp, C.POINTER(vp), C.POINTER(vp), C.POINTER(f32), f32, f32, f32]
+    L.bom_set_fused_update.restype = i32
     L.bom_destroy.argtypes = [vp]
     L.bom_destroy.restype = None
     L.bom_status_string.argtypes = [i32]
@@ -198,7 +200,7 @@ def bom_destroy(h) -> None:
 def bom_step(h, x, labels, n_rows: int, params, q, t: int, grads, h_out=None, stream=None) -> None:
     n = len(params)
     P = (C.c_void_p * n)(*[_ptr(p) for p in params])
-    G = (C.c_void_p * n)(*[_ptr(g) for g in grads])
+    G = (C.c_void_p * n)(*[_ptr(g) for g in grads]) if grads is not None else None
     H = (C.c_void_p * n)(*[_ptr(p) for p in h_out]) if h_out is not None else None
     _check(lib().bom_step(h, _ptr(x), _ptr(labels), int(n_rows), P, _ptr(q), int(t), G,
                           H if H is not None else None, _stream(stream)), "bom_step")
@@ -228,6 +230,19 @@ def bom_update(theta, g, g_dtype: int, hvec, v, theta_bf16, n: int, lr: float, w
     _check(lib().bom_update(_ptr(theta), _ptr(g), int(g_dtype), _ptr(hvec), _ptr(v), _ptr(theta_bf16), int(n),
                             float(lr), float(wd), float(lam), float(beta2), float(eps), int(t), _stream(stream)),
            "bom_update")
+
+
+def bom_set_fused_update(h, theta, v, wd, lr: float, beta2: float, eps: float) -> None:
+    """Registers per-tensor fp32 master weights, second moments and weight
+    decays for the update fused into bom_step (``theta=None`` disables it)."""
+    if theta is None:
+        _check(lib().bom_set_fused_update(h, None, None, None, 0.0, 0.0, 0.0), "bom_set_fused_update")
+        return
+    n = len(theta)
+    T = (C.c_void_p * n)(*[_ptr(p) for p in theta])
+    Vv = (C.c_void_p * n)(*[_ptr(p) for p in v])
+    W = (C.c_float * n)(*[float(w) for w in wd])
+    _check(lib().bom_set_fused_update(h, T, Vv, W, float(lr), float(beta2), float(eps)), "bom_set_fused_update")
 
 
 def bom_update_blockshared(theta, g, g_dtype: int, hvec, v_blocks, theta_bf16, n: int, block: int, lr: float,

@@ -72,6 +72,12 @@ struct bom_handle {
     float* rnorm = nullptr;  // ||r_i|| per row (own-step telemetry)
     double* tel_part = nullptr;  // per-block partials of bom_own_step_moment
     std::vector<void*> own_out;  // own-step projection outputs (bom_set_own_step_output)
+    // fused BOM-AdamW update (bom_set_fused_update)
+    bool fused_upd = false;
+    std::vector<float*> upd_theta, upd_v;
+    std::vector<float> upd_wd;
+    float upd_lr = 0.0f, upd_beta2 = 0.0f, upd_eps = 0.0f;
+    float* ubuf = nullptr;   // fp32 u of a vector tensor (bias, norm weight) before its update
     float* part = nullptr;
     void* dx[2] = {nullptr, nullptr};
     void* dG = nullptr;
@@ -196,6 +202,7 @@ size_t carve(bom_handle* h, char* base) {
     h->wsvec = static_cast<float*>(c.take(h->d_model * 4));
     h->rnorm = static_cast<float*>(c.take(n * 4));
     h->tel_part = static_cast<double*>(c.take(4 * kOwnStepMaxBlocks * sizeof(double)));
+    h->ubuf = static_cast<float*>(c.take((V > h->max_width ? V : h->max_width) * 4));
     const int64_t rb = row_blocks(n) > row_blocks(V) ? row_blocks(n) : row_blocks(V);
     h->part = static_cast<float*>(c.take(rb * h->max_width * 4));
     h->dx[0] = c.take(n * h->max_width * e);
@@ -240,6 +247,7 @@ const char* gemm_name(const GemmDesc& g, bool bf16) {
     if (!bf16) return "gemm_simt";
     switch (g.epi_kind) {
         case EPI_LOGITS: return "gemm_tc.logits";
+        case EPI_UPDATE: return "gemm_tc.update.mm";
         case EPI_SWIGLU_FWD: return "gemm_tc.swiglu_fwd";
         case EPI_SWIGLU_BWD: return "gemm_tc.swiglu_bwd";
         default: break;
@@ -251,7 +259,7 @@ const char* gemm_name(const GemmDesc& g, bool bf16) {
 int run_gemm(bom_handle* h, GemmDesc& g, cudaStream_t s) {
     g.epi.sc = h->sc;
     g.epi.in_f32 = h->bf16 ? 0 : 1;
-    if (h->bf16 && g.epi_kind == EPI_LINEAR) {
+    if (h->bf16 && (g.epi_kind == EPI_LINEAR || g.epi_kind == EPI_UPDATE)) {
         g.splitk_ws = h->splitk;
         g.splitk_ws_elems = h->splitk_elems;
     }
@@ -259,8 +267,10 @@ int run_gemm(bom_handle* h, GemmDesc& g, cudaStream_t s) {
     for (int i = 0; i < g.nseg; ++i) k += static_cast<double>(g.K[i]);
     const double n_mma = g.dual_b ? 2.0 * g.N : static_cast<double>(g.N);
     const double flops = 2.0 * static_cast<double>(g.M) * n_mma * k;
-    const double bytes = h->esz * (static_cast<double>(g.M) * k + n_mma * k) +
-                         (g.epi.out_f32 ? 4.0 : h->esz) * static_cast<double>(g.M) * g.N;
+    // output bytes per element: u, or with the fused update theta and v read
+    // and written plus the compute copy
+    const double out_b = g.epi.upd_theta ? 16.0 + h->esz : (g.epi.out_f32 ? 4.0 : h->esz);
+    const double bytes = h->esz * (static_cast<double>(g.M) * k + n_mma * k) + out_b * static_cast<double>(g.M) * g.N;
     return traced(h, s, gemm_name(g, h->bf16), flops, bytes,
                   [&] { return h->bf16 ? launch_gemm_tc(g, s) : launch_gemm_simt(g, s); });
 }
@@ -384,14 +394,18 @@ void bom_destroy(bom_handle* h) {
 
 bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t n, void* const* params, float* q,
                     int64_t t, void* const* grads, void* const* h_out, void* stream) {
-    if (!h || !x || !labels || !params || !q || !grads) return BOM_EINVAL;
+    const bool fused = h != nullptr && h->fused_upd;
+    if (!h || !x || !labels || !params || !q || (!grads && !fused)) return BOM_EINVAL;
     if (n < 1 || n > h->cfg.max_rows || t < 1) return BOM_EINVAL;
     const bool gh = h->cfg.out_mode == BOM_OUT_G_AND_H;
     if (gh != (h_out != nullptr)) return BOM_EINVAL;
+    // the fused update consumes u: one u pass and nothing else that needs it
+    if (fused && (gh || !h->own_out.empty())) return BOM_EINVAL;
     const int np = bom_param_count(&h->cfg);
     for (int i = 0; i < np; ++i) {
-        if (!params[i] || !grads[i] || (gh && !h_out[i])) return BOM_EINVAL;
-        if (!aligned16(params[i]) || !aligned16(grads[i]) || (gh && !aligned16(h_out[i]))) return BOM_ENOTSUP;
+        if (!params[i] || (!fused && !grads[i]) || (gh && !h_out[i])) return BOM_EINVAL;
+        if (!aligned16(params[i]) || (!fused && !aligned16(grads[i])) || (gh && !aligned16(h_out[i])))
+            return BOM_ENOTSUP;
     }
     if (!aligned16(x) || !aligned16(q)) return BOM_ENOTSUP;
 
@@ -508,11 +522,41 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                    launch_colsum(Wh, cf32, dm, V, dm, nullptr, 0, h->s, 1.0f, h->part, h->wsvec, 1, h->sc, s));
 
     // ---------------------------------------------------------------- backward
-    // passes: 0 = u, 1 = g, 2 = h = Jbar^T qhat, 3 = own-step projection Jbar^T s_t
+    // passes: 0 = u, 1 = g, 2 = h = Jbar^T qhat, 3 = own-step projection Jbar^T s_t.
+    // Within the head and every layer the input cotangent is formed before the
+    // weight gradients: a fused update rewrites the compute copy of a weight,
+    // so it runs after the last read of that weight in the step.
     int passes[3], npass = 0;
     passes[npass++] = gh ? 1 : 0;
     if (gh) passes[npass++] = 2;
     if (own) passes[npass++] = 3;
+    const float inv_bc2 = fused ? static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(h->upd_beta2),
+                                                                           static_cast<double>(t))))
+                                : 0.0f;
+    // the GEMM producing u of tensor k updates it in its epilogue
+    auto fuse = [&](GemmDesc& g, int k) {
+        g.epi.upd_theta = h->upd_theta[k];
+        g.epi.upd_v = h->upd_v[k];
+        g.epi.upd_lr = h->upd_lr;
+        g.epi.upd_decay = 1.0f - h->upd_lr * h->upd_wd[k];
+        g.epi.upd_beta2 = h->upd_beta2;
+        g.epi.upd_1mb2 = 1.0f - h->upd_beta2;
+        g.epi.upd_eps = h->upd_eps;
+        g.epi.upd_inv_bc2 = inv_bc2;
+        g.epi.out = params[k];   // the compute copy of the updated weight
+        g.epi.out_f32 = cf32;
+        if (h->bf16) g.epi_kind = EPI_UPDATE;   // tcgen05 path: staged, coalesced update epilogue
+    };
+    // a vector tensor k whose u is in ubuf (fp32): update it and its compute copy
+    auto update_small = [&](int k, int64_t cnt) -> int {
+        int r = launch_update(h->upd_theta[k], h->ubuf, 0, nullptr, h->upd_v[k],
+                              h->bf16 ? static_cast<uint16_t*>(params[k]) : nullptr, cnt, h->upd_lr, h->upd_wd[k],
+                              0.0f, h->upd_beta2, h->upd_eps, inv_bc2, nullptr, 0.0f, h->sc, s);
+        if (r == BOM_OK && !h->bf16 &&
+            cudaMemcpyAsync(params[k], h->upd_theta[k], cnt * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+            r = BOM_ECUDA;
+        return r;
+    };
     for (int pp = 0; pp < npass; ++pp) {
         const int pass = passes[pp];
         void* const* outp = pass == 3 ? h->own_out.data() : (pass == 2 ? h_out : grads);
@@ -522,28 +566,10 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
         const int64_t kfull = pass >= 2 ? 0 : 1;  // the h and own-step passes have no residual term
         const float* tvec = pass == 3 ? h->s : h->qhat;      // broadcast task-space vector
         const float* wtvec = pass == 3 ? h->wsvec : h->wvec; // W^T of it
-        {   // head weight: a R^T H + b qhat (x) c
-            GemmDesc g = gemm1(V, dm, kfull * n, mnmaj(h->Z, h->ldz), mnmaj(xin, dm));
-            g.epi.alpha_const = 1.0f;
-            g.epi.alpha_dev = cr;
-            g.epi.beta_dev = cq;
-            g.epi.r1u = tvec;
-            g.epi.r1v = h->cvec;
-            g.epi.out = outp[head_w];
-            g.epi.ld_out = dm;
-            g.epi.out_f32 = of32;
-            BOM_TRY(run_gemm(h, g, s));
-        }
-        if (head_b >= 0) {
-            const float a = pass == 0 ? 1.0f - cfg.lambda : (pass == 1 || pass == 3 ? 1.0f : 0.0f);
-            const float b = pass == 0 ? cfg.lambda : (pass == 2 ? 1.0f : 0.0f);
-            BOM_TRACED("axpby", 3.0 * V, 12.0 * V, launch_axpby(h->s, h->qhat, a, b, V, outp[head_b], of32, h->sc, s));
-        }
         // the cotangent of X goes out with the u (or g) pass when requested
         const bool want_dx = h->dx_in != nullptr && pass < 2;
-        if (h->lw.empty() && !want_dx) continue;
         int cur = 0;
-        {   // head input: a R W + b 1_{I_t} w^T  (times GELU' of the last layer)
+        if (!h->lw.empty() || want_dx) {   // head input: a R W + b 1_{I_t} w^T  (times GELU' of the last layer)
             GemmDesc g = gemm1(n, dm, kfull * V, kmaj(h->Z, h->ldz), mnmaj(Wh, dm));
             g.epi.alpha_dev = cr;
             g.epi.beta_dev = cq;
@@ -560,24 +586,40 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
             g.epi.out_f32 = cf32;
             BOM_TRY(run_gemm(h, g, s));
         }
+        {   // head weight: a R^T H + b qhat (x) c
+            GemmDesc g = gemm1(V, dm, kfull * n, mnmaj(h->Z, h->ldz), mnmaj(xin, dm));
+            g.epi.alpha_const = 1.0f;
+            g.epi.alpha_dev = cr;
+            g.epi.beta_dev = cq;
+            g.epi.r1u = tvec;
+            g.epi.r1v = h->cvec;
+            g.epi.out = fused ? nullptr : outp[head_w];
+            g.epi.ld_out = dm;
+            g.epi.out_f32 = of32;
+            if (fused) fuse(g, head_w);
+            BOM_TRY(run_gemm(h, g, s));
+        }
+        if (head_b >= 0) {
+            const float a = pass == 0 ? 1.0f - cfg.lambda : (pass == 1 || pass == 3 ? 1.0f : 0.0f);
+            const float b = pass == 0 ? cfg.lambda : (pass == 2 ? 1.0f : 0.0f);
+            BOM_TRACED("axpby", 3.0 * V, 12.0 * V,
+                       launch_axpby(h->s, h->qhat, a, b, V, fused ? h->ubuf : outp[head_b], fused ? 1 : of32, h->sc,
+                                    s));
+            if (fused) BOM_TRY(update_small(head_b, V));
+        }
         for (int l = static_cast<int>(h->lw.size()) - 1; l >= 0; --l) {
             const LayerWs& L = h->lw[l];
             const void* xl = l == 0 ? x : h->lw[l - 1].out;
             const void* dcur = h->dx[cur];
             const int p0 = pidx[l];
             const LayerWs* prev = l > 0 ? &h->lw[l - 1] : nullptr;
+            const bool dx_next = prev != nullptr || want_dx;
+            void* const dxo = prev ? h->dx[cur ^ 1] : h->dx_in;
             if (L.kind == BOM_LAYER_SWIGLU) {
                 const int64_t d = L.d_in, f = L.d_out;
                 const void* Wg = params[p0];
                 const void* Wu = params[p0 + 1];
                 const void* Wd = params[p0 + 2];
-                {   // dW_d = dy^T A
-                    GemmDesc g = gemm1(d, f, n, mnmaj(dcur, d), mnmaj(L.A, f));
-                    g.epi.out = outp[p0 + 2];
-                    g.epi.ld_out = f;
-                    g.epi.out_f32 = of32;
-                    BOM_TRY(run_gemm(h, g, s));
-                }
                 {   // dA = dy W_d, then dG = dA u SiLU'(g), dU = dA SiLU(g)
                     GemmDesc g = gemm1(n, f, d, kmaj(dcur, d), mnmaj(Wd, f));
                     g.epi_kind = EPI_SWIGLU_BWD;
@@ -591,19 +633,7 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                     g.epi.ld_out2 = f;
                     BOM_TRY(run_gemm(h, g, s));
                 }
-                {   // dW_g = dG^T x, dW_u = dU^T x
-                    GemmDesc g = gemm1(f, d, n, mnmaj(h->dG, f), mnmaj(xl, d));
-                    g.epi.out = outp[p0];
-                    g.epi.ld_out = d;
-                    g.epi.out_f32 = of32;
-                    BOM_TRY(run_gemm(h, g, s));
-                    GemmDesc g2 = gemm1(f, d, n, mnmaj(h->dU, f), mnmaj(xl, d));
-                    g2.epi.out = outp[p0 + 1];
-                    g2.epi.ld_out = d;
-                    g2.epi.out_f32 = of32;
-                    BOM_TRY(run_gemm(h, g2, s));
-                }
-                if (prev || want_dx) {   // dx = dy + dG W_g + dU W_u
+                if (dx_next) {   // dx = dy + dG W_g + dU W_u
                     GemmDesc g = gemm1(n, d, f, kmaj(h->dG, f), mnmaj(Wg, d));
                     g.nseg = 2;
                     g.A[1] = kmaj(h->dU, f);
@@ -616,53 +646,76 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                         g.epi.aux = prev->pre;
                         g.epi.ld_aux = prev->d_out;
                     }
-                    g.epi.out = prev ? h->dx[cur ^ 1] : h->dx_in;
+                    g.epi.out = dxo;
                     g.epi.ld_out = d;
                     g.epi.out_f32 = cf32;
                     BOM_TRY(run_gemm(h, g, s));
-                    cur ^= 1;
+                }
+                {   // dW_d = dy^T A
+                    GemmDesc g = gemm1(d, f, n, mnmaj(dcur, d), mnmaj(L.A, f));
+                    g.epi.out = fused ? nullptr : outp[p0 + 2];
+                    g.epi.ld_out = f;
+                    g.epi.out_f32 = of32;
+                    if (fused) fuse(g, p0 + 2);
+                    BOM_TRY(run_gemm(h, g, s));
+                }
+                {   // dW_g = dG^T x, dW_u = dU^T x
+                    GemmDesc g = gemm1(f, d, n, mnmaj(h->dG, f), mnmaj(xl, d));
+                    g.epi.out = fused ? nullptr : outp[p0];
+                    g.epi.ld_out = d;
+                    g.epi.out_f32 = of32;
+                    if (fused) fuse(g, p0);
+                    BOM_TRY(run_gemm(h, g, s));
+                    GemmDesc g2 = gemm1(f, d, n, mnmaj(h->dU, f), mnmaj(xl, d));
+                    g2.epi.out = fused ? nullptr : outp[p0 + 1];
+                    g2.epi.ld_out = d;
+                    g2.epi.out_f32 = of32;
+                    if (fused) fuse(g2, p0 + 1);
+                    BOM_TRY(run_gemm(h, g2, s));
                 }
             } else if (L.kind == BOM_LAYER_RMSNORM) {
                 const int64_t d = L.d_in;
                 const void* gamma = params[p0];
                 // dgamma_j = sum_i rstd_i dy_ij x_ij
                 BOM_TRACED("colsum", 3.0 * n * d, 2.0 * h->esz * n * d,
-                           launch_colsum2(dcur, xl, cf32, d, n, d, nullptr, 0, L.rstd, 1.0f, h->part, outp[p0], of32,
-                                          h->sc, s));
-                if (prev || want_dx) {
+                           launch_colsum2(dcur, xl, cf32, d, n, d, nullptr, 0, L.rstd, 1.0f, h->part,
+                                          fused ? h->ubuf : outp[p0], fused ? 1 : of32, h->sc, s));
+                if (dx_next) {
                     const void* pre = (prev && prev->kind == BOM_LAYER_LINEAR_GELU) ? prev->pre : nullptr;
-                    void* dxo = prev ? h->dx[cur ^ 1] : h->dx_in;
                     BOM_TRACED("rmsnorm_bwd", 8.0 * n * d, 3.0 * h->esz * n * d + 4.0 * n,
                                launch_rmsnorm_bwd(dcur, xl, gamma, L.rstd, pre, dxo, n, d, cf32, h->sc, s));
-                    cur ^= 1;
                 }
+                if (fused) BOM_TRY(update_small(p0, d));   // after the last read of gamma
             } else {
                 const void* W = params[p0];
-                {   // dW = dPre^T x
-                    GemmDesc g = gemm1(L.d_out, L.d_in, n, mnmaj(dcur, L.d_out), mnmaj(xl, L.d_in));
-                    g.epi.out = outp[p0];
-                    g.epi.ld_out = L.d_in;
-                    g.epi.out_f32 = of32;
-                    BOM_TRY(run_gemm(h, g, s));
-                }
-                if (L.bias)
-                    BOM_TRACED("colsum", 2.0 * n * L.d_out, h->esz * n * L.d_out,
-                               launch_colsum(dcur, cf32, L.d_out, n, L.d_out, nullptr, 0, nullptr, 1.0f, h->part,
-                                             outp[p0 + 1], of32, h->sc, s));
-                if (prev || want_dx) {   // dx = dPre W (times GELU' of the previous layer)
+                if (dx_next) {   // dx = dPre W (times GELU' of the previous layer)
                     GemmDesc g = gemm1(n, L.d_in, L.d_out, kmaj(dcur, L.d_out), mnmaj(W, L.d_in));
                     if (prev && prev->kind == BOM_LAYER_LINEAR_GELU) {
                         g.epi.act = ACT_DGELU;
                         g.epi.aux = prev->pre;
                         g.epi.ld_aux = prev->d_out;
                     }
-                    g.epi.out = prev ? h->dx[cur ^ 1] : h->dx_in;
+                    g.epi.out = dxo;
                     g.epi.ld_out = L.d_in;
                     g.epi.out_f32 = cf32;
                     BOM_TRY(run_gemm(h, g, s));
-                    cur ^= 1;
+                }
+                {   // dW = dPre^T x
+                    GemmDesc g = gemm1(L.d_out, L.d_in, n, mnmaj(dcur, L.d_out), mnmaj(xl, L.d_in));
+                    g.epi.out = fused ? nullptr : outp[p0];
+                    g.epi.ld_out = L.d_in;
+                    g.epi.out_f32 = of32;
+                    if (fused) fuse(g, p0);
+                    BOM_TRY(run_gemm(h, g, s));
+                }
+                if (L.bias) {
+                    BOM_TRACED("colsum", 2.0 * n * L.d_out, h->esz * n * L.d_out,
+                               launch_colsum(dcur, cf32, L.d_out, n, L.d_out, nullptr, 0, nullptr, 1.0f, h->part,
+                                             fused ? h->ubuf : outp[p0 + 1], fused ? 1 : of32, h->sc, s));
+                    if (fused) BOM_TRY(update_small(p0 + 1, L.d_out));
                 }
             }
+            if (dx_next) cur ^= 1;
         }
     }
 #undef BOM_TRY
@@ -689,6 +742,29 @@ bom_status bom_set_own_step_output(bom_handle* h, void* const* o) {
         if (!aligned16(p)) return BOM_ENOTSUP;
     }
     h->own_out = v;
+    return BOM_OK;
+}
+
+bom_status bom_set_fused_update(bom_handle* h, float* const* theta, float* const* v, const float* wd, float lr,
+                                float beta2, float eps) {
+    if (!h) return BOM_EINVAL;
+    if (!theta) {
+        h->fused_upd = false;
+        return BOM_OK;
+    }
+    if (!v || !wd || !(beta2 >= 0.0f && beta2 < 1.0f) || !(eps >= 0.0f)) return BOM_EINVAL;
+    const int np = bom_param_count(&h->cfg);
+    for (int i = 0; i < np; ++i) {
+        if (!theta[i] || !v[i]) return BOM_EINVAL;
+        if (!aligned16(theta[i]) || !aligned16(v[i])) return BOM_ENOTSUP;
+    }
+    h->upd_theta.assign(theta, theta + np);
+    h->upd_v.assign(v, v + np);
+    h->upd_wd.assign(wd, wd + np);
+    h->upd_lr = lr;
+    h->upd_beta2 = beta2;
+    h->upd_eps = eps;
+    h->fused_upd = true;
     return BOM_OK;
 }
 
@@ -740,7 +816,7 @@ bom_status bom_update(float* theta, const void* g, int32_t g_dtype, const float*
         return BOM_ENOTSUP;
     const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
     return static_cast<bom_status>(launch_update(theta, g, g_dtype == BOM_BF16, hvec, v, theta_bf16, n, lr, wd,
-                                                 lambda, beta2, eps, inv_bc2, nullptr, 0.0f,
+                                                 lambda, beta2, eps, inv_bc2, nullptr, 0.0f, nullptr,
                                                  static_cast<cudaStream_t>(stream)));
 }
 
@@ -767,7 +843,7 @@ bom_status bom_update_clipped(float* theta, const void* g, int32_t g_dtype, cons
         return BOM_ENOTSUP;
     const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
     return static_cast<bom_status>(launch_update(theta, g, g_dtype == BOM_BF16, hvec, v, theta_bf16, n, lr, wd,
-                                                 lambda, beta2, eps, inv_bc2, sq, max_norm,
+                                                 lambda, beta2, eps, inv_bc2, sq, max_norm, nullptr,
                                                  static_cast<cudaStream_t>(stream)));
 }
 

@@ -30,7 +30,7 @@ __device__ __forceinline__ void latch_status(DevScalars* sc, int code) {
     atomicCAS(&sc->status, 0, code);
 }
 
-enum EpiKind : int { EPI_LINEAR = 0, EPI_LOGITS = 1, EPI_SWIGLU_FWD = 2, EPI_SWIGLU_BWD = 3 };
+enum EpiKind : int { EPI_LINEAR = 0, EPI_LOGITS = 1, EPI_SWIGLU_FWD = 2, EPI_SWIGLU_BWD = 3, EPI_UPDATE = 4 };
 enum ActKind : int { ACT_NONE = 0, ACT_GELU = 1, ACT_DGELU = 2 };
 
 // What a GEMM does with its fp32 accumulator acc[m][n] (m: output row, n: column):
@@ -41,6 +41,8 @@ enum ActKind : int { ACT_NONE = 0, ACT_GELU = 1, ACT_DGELU = 2 };
 //                  the pair (max_n z, sum_n exp(z - max)) goes to stats.
 //   EPI_SWIGLU_FWD the accumulator tile holds [g | u] halves: out2 <- g, out3 <- u, out <- SiLU(g)*u.
 //   EPI_SWIGLU_BWD acc = dA: out <- dA*u*SiLU'(g) (= dG), out2 <- dA*SiLU(g) (= dU), g = aux, u = aux2.
+//   EPI_UPDATE     u = alpha*acc + beta*r1u[m]*r1v[n] is the numerator of a weight: the fused
+//                  BOM-AdamW update of upd_theta / upd_v, out <- the updated weight (compute dtype).
 struct EpiParams {
     float alpha_const;
     const float* alpha_dev;      // optional device factor of alpha
@@ -71,7 +73,26 @@ struct EpiParams {
     float* stats;                // EPI_LOGITS: [M, ld_stats] float2 pairs
     int64_t ld_stats;            // pairs per row (number of column tiles)
     const DevScalars* sc;        // kernels return early when sc->status != 0
+    // Fused BOM-AdamW update (EPI_UPDATE; EPI_LINEAR on the SIMT and split-K
+    // paths): when upd_theta is set, the epilogue value is u of the output
+    // element; the epilogue advances v and theta ([M, ld_out] fp32, the
+    // layout of out) and stores the updated theta into out in out's dtype
+    // (the compute copy) instead of u.
+    float* upd_theta;
+    float* upd_v;
+    float upd_lr, upd_decay, upd_beta2, upd_1mb2, upd_eps, upd_inv_bc2;
 };
+
+// One element of the fused update (Section 3.4): returns the new theta.
+__device__ __forceinline__ float fused_update1(const EpiParams& e, int64_t idx, float u) {
+    float vv = e.upd_v[idx];
+    float th = e.upd_theta[idx];
+    vv = fmaf(e.upd_beta2, vv, e.upd_1mb2 * u * u);
+    th = e.upd_decay * th - e.upd_lr * (u / (sqrtf(vv * e.upd_inv_bc2) + e.upd_eps));
+    e.upd_v[idx] = vv;
+    e.upd_theta[idx] = th;
+    return th;
+}
 
 // ------------------------------------------------------------ activations
 __device__ __forceinline__ float gelu_f(float x) {
@@ -234,48 +255,6 @@ __device__ __forceinline__ EpiRow epi_row(const EpiParams& e, int m, int M) {
     if (e.mask_labels && r.valid) mask = (e.mask_labels[m] != e.ignore_index) ? 1.0f : 0.0f;
     r.beta_bw = e.bw ? b * mask : 0.0f;
     return r;
-}
-
-// Applies EPI_LINEAR to 32 accumulator values of row m, columns [n, n+32).
-__device__ __forceinline__ void epi_linear32(const EpiParams& e, const EpiRow& r, int m, int n, int N,
-                                             float (&v)[32]) {
-    float t[32];
-#pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] *= r.alpha;
-    if (e.bias) {
-        load_row32(e.bias, 0, n, N, e.in_f32, t);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] += t[i];
-    }
-    if (e.r1u) {
-        load_vec32(e.r1v, n, N, t);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] += r.beta_r1 * t[i];
-    }
-    if (e.bw) {
-        load_vec32(e.bw, n, N, t);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] += r.beta_bw * t[i];
-    }
-    if (e.resid) {
-        load_row32(e.resid, static_cast<int64_t>(m) * e.ld_resid, n, N, e.in_f32, t);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] += t[i];
-    }
-    if (e.act == ACT_GELU) {
-        store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, N, e.out2_f32, v);
-        if (!e.out2_f32) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = round_bf16(v[i]);
-        }
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = gelu_f(v[i]);
-    } else if (e.act == ACT_DGELU) {
-        load_row32(e.aux, static_cast<int64_t>(m) * e.ld_aux, n, N, e.in_f32, t);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(t[i]);
-    }
-    store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, N, e.out_f32, v);
 }
 
 // Scalar form of EPI_LINEAR (SIMT GEMM).

@@ -71,6 +71,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const Params p) {
                 v = acc[i][j] + (e.bias ? ld_elem(e.bias, n, e.in_f32) : 0.0f);
             } else {
                 v = epi_linear1(e, r, m, n, acc[i][j]);
+                if (e.upd_theta) v = fused_update1(e, static_cast<int64_t>(m) * e.ld_out + n, v);
             }
             st_elem(e.out, static_cast<int64_t>(m) * e.ld_out + n, e.out_f32, v);
         }

@@ -159,6 +159,50 @@ __device__ __forceinline__ void stg_scatter(void* base, int64_t ld, int row0, in
     stg_scatter_bf16(base, ld, row0, M, n, N, stg, b);
 }
 
+// Fused update through shared memory: lane l holds u of row l of a 32 x 32
+// block; the block goes to a per-warp buffer (33-float pitch: both the
+// row-per-lane writes and the column-per-lane reads hit 32 distinct banks, and
+// the eight buffers leave room for six pipeline stages), then the warp walks
+// the 32 rows with lane l on column l, so every access to theta, v and the
+// compute copy is one coalesced 128-byte (64-byte for bf16) line per row.
+// Eight rows are loaded before any is written.
+constexpr int kUpdPitch = 33;
+constexpr int kUpdStgBytes = 32 * kUpdPitch * 4;
+__device__ __forceinline__ void staged_update32(const EpiParams& e, float* buf, int row0, int M, int n, int N,
+                                               const float (&u)[32]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int k = 0; k < 32; ++k) buf[lane * kUpdPitch + k] = u[k];
+    __syncwarp();
+    const int c = n + lane;
+    if (c < N) {
+#pragma unroll 1
+        for (int r0 = 0; r0 < 32; r0 += 8) {
+            float th[8], vv[8];
+#pragma unroll
+            for (int r = 0; r < 8; ++r) {
+                const int m = row0 + r0 + r;
+                const int64_t idx = static_cast<int64_t>(m < M ? m : 0) * e.ld_out + c;
+                th[r] = m < M ? e.upd_theta[idx] : 0.0f;
+                vv[r] = m < M ? e.upd_v[idx] : 0.0f;
+            }
+#pragma unroll
+            for (int r = 0; r < 8; ++r) {
+                const int m = row0 + r0 + r;
+                if (m >= M) continue;
+                const int64_t idx = static_cast<int64_t>(m) * e.ld_out + c;
+                const float uu = buf[(r0 + r) * kUpdPitch + lane];
+                const float v2 = fmaf(e.upd_beta2, vv[r], e.upd_1mb2 * uu * uu);
+                const float t2 = e.upd_decay * th[r] - e.upd_lr * (uu / (sqrtf(v2 * e.upd_inv_bc2) + e.upd_eps));
+                e.upd_v[idx] = v2;
+                e.upd_theta[idx] = t2;
+                st_elem(e.out, idx, e.out_f32, t2);
+            }
+        }
+    }
+    __syncwarp();
+}
+
 __device__ __forceinline__ float fast_exp(float x) { return exp2f(x * 1.4426950408889634f); }
 __device__ __forceinline__ float fast_sigmoid(float x) { return __frcp_rn(1.0f + fast_exp(-x)); }
 
@@ -187,7 +231,7 @@ struct Cfg {
     static constexpr int B_ROWS = CG == 2 ? 128 : 256;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
-    static constexpr int STG_BYTES = 8 * NBUF * kStgBytes;
+    static constexpr int STG_BYTES = EPI == EPI_UPDATE ? 8 * kUpdStgBytes : 8 * NBUF * kStgBytes;
     // as many stages as fit in the 227 KB a CTA may use beside the staging
     // blocks, the 1 KB alignment slack and the barrier block, at most six (a
     // seventh 32 KB stage measured slower on the linear epilogues)
@@ -425,7 +469,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t ra = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid);
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
-            uint8_t* stg = stg_all + (warp - 2) * C::NBUF * kStgBytes;
+            uint8_t* stg = stg_all + (warp - 2) * (EPI == EPI_UPDATE ? kUpdStgBytes : C::NBUF * kStgBytes);
             if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
             if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
             if (kb_total > 0) {
@@ -485,6 +529,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         }
                         store_row32(out_base, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
                     }
+                }
+            } else if constexpr (EPI == EPI_UPDATE) {
+                const EpiRow r = epi_row(e, m, p.M);
+                float t[32];
+#pragma unroll 1
+                for (int j = 0; j < CPW; ++j) {
+                    const int c = c0 + j;
+                    const int n = n0 + c * 32;
+                    if (n >= p.N) break;
+                    if (kb_total > 0) {
+                        tmem_load32(tbase + c * 32, v);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+                    }
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] *= r.alpha;
+                    if (e.r1u) {
+                        load_vec32(e.r1v, n, p.N, t);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] += r.beta_r1 * t[i];
+                    }
+                    staged_update32(e, reinterpret_cast<float*>(stg), row0, p.M, n, p.N, v);
                 }
             } else if constexpr (EPI == EPI_LOGITS || EPI == EPI_LOGITS_STG) {
                 // per (row, column half) softmax statistics: stats pair nt*2 + h.
@@ -738,7 +805,10 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restr
         for (int s = 0; s < S; ++s) acc += ws[s * total + i];
         const int m = static_cast<int>(i / N), n = static_cast<int>(i - static_cast<int64_t>(m) * N);
         const EpiRow r = epi_row(e, m, M);
-        st_elem(e.out, static_cast<int64_t>(m) * e.ld_out + n, e.out_f32, epi_linear1(e, r, m, n, acc));
+        const int64_t idx = static_cast<int64_t>(m) * e.ld_out + n;
+        float v = epi_linear1(e, r, m, n, acc);
+        if (e.upd_theta) v = fused_update1(e, idx, v);
+        st_elem(e.out, idx, e.out_f32, v);
     }
 }
 
@@ -788,6 +858,9 @@ static int dispatch(const Params& p, int epi_kind, bool a_mn, bool b_mn, bool du
         case EPI_SWIGLU_BWD:
             if (a_mn || !b_mn) return BOM_ENOTSUP;
             return launch_inst<CG, false, true, EPI_SWIGLU_BWD>(p, stream);
+        case EPI_UPDATE:   // weight gradients: dy^T x, both operands MN-major
+            if (!a_mn || !b_mn) return BOM_ENOTSUP;
+            return launch_inst<CG, true, true, EPI_UPDATE>(p, stream);
         default:
             return BOM_EINVAL;
     }
@@ -844,7 +917,7 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     const int tiles = p.tiles_m * p.tiles_n;
     const int units = cg == 2 ? device_sm_count() / 2 : device_sm_count();
     int S = 1;
-    if (g.epi_kind == EPI_LINEAR && g.splitk_ws != nullptr)
+    if ((g.epi_kind == EPI_LINEAR || g.epi_kind == EPI_UPDATE) && g.splitk_ws != nullptr)
         S = choose_split(tiles, units, kb_total, static_cast<int64_t>(g.M) * g.N, g.splitk_ws_elems);
     p.ksplit = S;
     p.kb_split = S > 1 ? (kb_total + S - 1) / S : kb_total;
@@ -861,8 +934,11 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
         p.epi = raw;
         p.split_bytes = static_cast<int64_t>(g.M) * g.N * 4;
     }
-    const int rc = cg == 2 ? dispatch<2>(p, g.epi_kind, a_mn, b_mn, g.dual_b, stream)
-                           : dispatch<1>(p, g.epi_kind, a_mn, b_mn, g.dual_b, stream);
+    // split-K partial tiles are raw (linear epilogue); the update, if any,
+    // runs in the reduction
+    const int kind = S > 1 ? EPI_LINEAR : g.epi_kind;
+    const int rc = cg == 2 ? dispatch<2>(p, kind, a_mn, b_mn, g.dual_b, stream)
+                           : dispatch<1>(p, kind, a_mn, b_mn, g.dual_b, stream);
     if (rc != BOM_OK || S == 1) return rc;
     const int64_t total = static_cast<int64_t>(g.M) * g.N;
     int64_t blocks = (total + 255) / 256;

@@ -92,9 +92,10 @@ int launch_update_blockshared(float* theta, const void* g, int g_bf16, const flo
 
 // BOM-AdamW update (see bom_update in bom.h).  With clip_sq, u is first scaled
 // by min(1, max_norm / (sqrt(*clip_sq) + 1e-6)) (bom_update_clipped).
+// When sc is given the kernel does nothing once the step's status word is set.
 int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,
                   float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, const double* clip_sq,
-                  float max_norm, cudaStream_t s);
+                  float max_norm, const DevScalars* sc, cudaStream_t s);
 
 // *sq += sum u^2 over n elements (u = g, or (1-lambda) g + lambda h), in a fixed
 // order; `part` holds kOwnStepMaxBlocks doubles.

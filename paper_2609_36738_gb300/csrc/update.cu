@@ -40,7 +40,9 @@ template <bool G_BF16, bool HAS_H, bool SHADOW, bool CLIP>
 __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ theta, const void* __restrict__ g,
                                                      const float* __restrict__ h, float* __restrict__ v,
                                                      uint16_t* __restrict__ shadow, int64_t n, UpdCoef c,
-                                                     const double* __restrict__ clip_sq, float max_norm) {
+                                                     const double* __restrict__ clip_sq, float max_norm,
+                                                     const DevScalars* sc) {
+    if (sc != nullptr && sc->status != 0) return;   // inside a step that latched an error
     const float cs = CLIP ? clip_scale(clip_sq, max_norm) : 1.0f;
     const int64_t n4 = n >> 2;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -207,21 +209,22 @@ void dispatch_blockshared(float* theta, const void* g, const float* h, float* vb
 
 template <bool G_BF16, bool HAS_H>
 void dispatch_shadow(float* theta, const void* g, const float* h, float* v, uint16_t* shadow, int64_t n,
-                     const UpdCoef& c, int grid, const double* clip_sq, float max_norm, cudaStream_t s) {
+                     const UpdCoef& c, int grid, const double* clip_sq, float max_norm, const DevScalars* sc,
+                     cudaStream_t s) {
     if (clip_sq) {
         if (shadow)
             update_kernel<G_BF16, HAS_H, true, true><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, clip_sq,
-                                                                          max_norm);
+                                                                          max_norm, sc);
         else
             update_kernel<G_BF16, HAS_H, false, true><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, clip_sq,
-                                                                           max_norm);
+                                                                           max_norm, sc);
     } else {
         if (shadow)
             update_kernel<G_BF16, HAS_H, true, false><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, nullptr,
-                                                                           0.0f);
+                                                                           0.0f, sc);
         else
             update_kernel<G_BF16, HAS_H, false, false><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, nullptr,
-                                                                            0.0f);
+                                                                            0.0f, sc);
     }
     count_launch();
 }
@@ -269,7 +272,7 @@ int device_sm_count();
 
 int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,
                   float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, const double* clip_sq,
-                  float max_norm, cudaStream_t s) {
+                  float max_norm, const DevScalars* sc, cudaStream_t s) {
     if (n <= 0) return BOM_OK;
     UpdCoef c;
     c.lr = lr;
@@ -285,11 +288,11 @@ int launch_update(float* theta, const void* g, int g_bf16, const float* h, float
     if (grid > need) grid = need;
     if (grid < 1) grid = 1;
     if (g_bf16) {
-        if (h) dispatch_shadow<true, true>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, s);
-        else dispatch_shadow<true, false>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, s);
+        if (h) dispatch_shadow<true, true>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, sc, s);
+        else dispatch_shadow<true, false>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, sc, s);
     } else {
-        if (h) dispatch_shadow<false, true>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, s);
-        else dispatch_shadow<false, false>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, s);
+        if (h) dispatch_shadow<false, true>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, sc, s);
+        else dispatch_shadow<false, false>(theta, g, h, v, shadow, n, c, (int)grid, clip_sq, max_norm, sc, s);
     }
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }

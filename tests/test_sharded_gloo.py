@@ -1,11 +1,20 @@
-"""Data-parallel partition of the BOM step on CPU ranks (world size 2, gloo).
+"""Partitions of the BOM step on CPU ranks (world size 2, gloo).
 
-Rows (tokens) split across ranks.  Each rank forms the residuals of its shard,
-then one all-reduce of the column sums of R and of the integer N_t partial
-gives every rank the same s_t, after which q_t updates redundantly.  With the
-global qhat and N_t, each rank back-propagates its own rows; a second
-all-reduce of the per-tensor partial gradients equals the full-batch u.  The
-oracle's full-batch step is the reference (bit-exact counts, fp64 sums)."""
+Data parallel: rows (tokens) split across ranks.  Each rank forms the
+residuals of its shard, then one all-reduce of the column sums of R and of the
+integer N_t partial gives every rank the same s_t, after which q_t updates
+redundantly.  With the global qhat and N_t, each rank back-propagates its own
+rows; a second all-reduce of the per-tensor partial gradients equals the
+full-batch u.
+
+Vocabulary parallel (the head's output columns split across ranks): each rank
+computes its logit columns, the per-row (max, sum exp) pairs are combined
+across ranks into the row log-sum-exp, and s_t, q_t and qhat_t then live
+sharded with no exchange.  The head weight gradient is local to the shard;
+the head-input cotangent is the all-reduced sum of the shards' R W and
+broadcast-row terms.
+
+The oracle's full-batch step is the reference (bit-exact counts, fp64 sums)."""
 import os
 import socket
 
@@ -83,3 +92,68 @@ def test_two_rank_data_parallel_step_equals_full_batch(tmp_path):
         assert X.rel_l2(o[1 + 2 * V:], u_ref) < 1e-12
     # every rank holds the same state after the exchange
     assert np.array_equal(outs[0], outs[1])
+
+
+WL_HEAD = I.LM_HEAD_SMALL
+
+
+def _vocab_rank_main(rank, world, port, out_dir):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        wl = WL_HEAD
+        W = X.params_f64(wl, I.init_params(wl, 6))[0]
+        xb, y = I.make_batch(wl, 6, 1)
+        H = X.x_f64(wl, xb)
+        cols = np.array_split(np.arange(wl.vocab), world)[rank]
+        q_prev = np.random.default_rng(8).standard_normal(wl.vocab) * 0.01
+        Zl = H @ W[cols].T                                   # this rank's logit columns
+        valid = y != I.IGNORE_INDEX
+        n_t = int(valid.sum())                               # labels are replicated: no exchange
+        # row log-sum-exp from the shards' (max, sum exp) pairs
+        m_loc = torch.tensor(Zl.max(axis=1))
+        m_all = m_loc.clone()
+        dist.all_reduce(m_all, op=dist.ReduceOp.MAX)
+        se = torch.tensor(np.exp(Zl - m_all.numpy()[:, None]).sum(axis=1))
+        dist.all_reduce(se)
+        lse = m_all.numpy() + np.log(se.numpy())
+        P = np.exp(Zl - lse[:, None])
+        own = (y[:, None] == cols[None, :]) & valid[:, None]
+        R = np.where(valid[:, None], P - own, 0.0)
+        s = R.sum(axis=0) / n_t                              # sharded s_t: no exchange
+        q, qhat = O.ema_update(q_prev[cols], s, T, B1)
+        dZ = ((1 - LAM) * R + LAM * valid[:, None] * qhat[None, :]) / n_t
+        gW = dZ.T @ H                                         # local rows of the head gradient
+        dH = torch.tensor(dZ @ W[cols])
+        dist.all_reduce(dH)                                   # head-input cotangent
+        np.save(os.path.join(out_dir, f"vrank{rank}.npy"),
+                np.concatenate([[n_t], cols, s, q, gW.ravel(), dH.numpy().ravel()]))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_rank_vocabulary_parallel_head_equals_full_batch(tmp_path):
+    world = 2
+    mp.spawn(_vocab_rank_main, args=(world, _free_port(), str(tmp_path)), nprocs=world, join=True)
+    wl = WL_HEAD
+    params = X.params_f64(wl, I.init_params(wl, 6))
+    xb, y = I.make_batch(wl, 6, 1)
+    q_prev = np.random.default_rng(8).standard_normal(wl.vocab) * 0.01
+    ref = O.bom_step(X.oracle_layers(wl), wl.head_bias, params, X.x_f64(wl, xb), y, q_prev, T, lam=LAM, beta1=B1)
+    d = wl.d_in
+    dHs = []
+    for r in range(world):
+        o = np.load(tmp_path / f"vrank{r}.npy")
+        assert int(o[0]) == ref["n_t"]
+        cols = np.array_split(np.arange(wl.vocab), world)[r]
+        k = 1 + cols.size
+        assert np.array_equal(o[1:k].astype(np.int64), cols)
+        s, q = o[k:k + cols.size], o[k + cols.size:k + 2 * cols.size]
+        assert X.rel_l2(s, ref["s"][cols]) < 1e-13
+        assert X.rel_l2(q, ref["q"][cols]) < 1e-13
+        g0 = k + 2 * cols.size
+        gW = o[g0:g0 + cols.size * d].reshape(cols.size, d)
+        assert X.rel_l2(gW, ref["u"][0][cols]) < 1e-12
+        dHs.append(o[g0 + cols.size * d:])
+    assert X.rel_l2(dHs[0], ref["dX_u"].ravel()) < 1e-12
+    assert np.array_equal(dHs[0], dHs[1])
