@@ -41,6 +41,7 @@ constexpr int GROUP_M = 8;
 struct Params {
     CUtensorMap mapA[2];
     CUtensorMap mapB[2];
+    CUtensorMap mapE[2];   // SwiGLU backward: saved G and U, 32 x 32 boxes, 64-byte swizzle
     int M, N;
     int kb[2];
     int nseg;
@@ -204,7 +205,6 @@ __device__ __forceinline__ void staged_update32(const EpiParams& e, float* buf, 
 }
 
 __device__ __forceinline__ float fast_exp(float x) { return exp2f(x * 1.4426950408889634f); }
-__device__ __forceinline__ float fast_sigmoid(float x) { return __frcp_rn(1.0f + fast_exp(-x)); }
 
 __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
     uint32_t r[32];
@@ -221,6 +221,15 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
 // 128 rows of A and its half (128 rows) of B, so a stage is 32 KB.  Epilogues
 // that move several bf16 streams (logits, SwiGLU) take NBUF staging blocks per
 // epilogue warp and give up pipeline stages for them.
+// SwiGLU backward: the epilogue's per-row operands (the saved G and U) arrive
+// by TMA.  Each epilogue warp owns two slots of a 32-row x 32-column block of
+// G and of U (2 KB each, 64-byte swizzle: chunk k of row r at
+// r * 64 + 16 * (k ^ ((r >> 1) & 3)), so the row-per-lane reads are
+// conflict-free); lane 0 loads block j + 2 into the slot block j has just
+// freed.
+constexpr int kEpiLdBlock = 32 * 64;
+constexpr int kEpiLdWarpBytes = 2 * 2 * kEpiLdBlock;
+
 // Logits epilogue with its output staged through shared memory (chosen when
 // the contraction is short and the epilogue, not the mainloop, sets the pace).
 constexpr int EPI_LOGITS_STG = 16;
@@ -231,13 +240,16 @@ struct Cfg {
     static constexpr int B_ROWS = CG == 2 ? 128 : 256;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
-    static constexpr int STG_BYTES = EPI == EPI_UPDATE ? 8 * kUpdStgBytes : 8 * NBUF * kStgBytes;
+    static constexpr int STG_BYTES = EPI == EPI_UPDATE ? 8 * kUpdStgBytes
+                                     : EPI == EPI_SWIGLU_BWD ? 8 * kEpiLdWarpBytes
+                                                             : 8 * NBUF * kStgBytes;
+    static constexpr int BAR_BYTES = 512;
     // as many stages as fit in the 227 KB a CTA may use beside the staging
     // blocks, the 1 KB alignment slack and the barrier block, at most six (a
     // seventh 32 KB stage measured slower on the linear epilogues)
-    static constexpr int STAGES_FIT = (227 * 1024 - STG_BYTES - 1024 - 256) / (A_BYTES + B_BYTES);
+    static constexpr int STAGES_FIT = (227 * 1024 - STG_BYTES - 1024 - BAR_BYTES) / (A_BYTES + B_BYTES);
     static constexpr int STAGES = STAGES_FIT < 6 ? STAGES_FIT : 6;
-    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 1024 + 256;
+    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 1024 + BAR_BYTES;
     static_assert(STAGES >= 2, "pipeline needs two stages");
     static constexpr int TILE_M = BM * CG;
 };
@@ -257,7 +269,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
     uint64_t* tfull = bars + 2 * STAGES;
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* ebar = drain + 1;   // SwiGLU backward: 2 slots x 8 epilogue warps
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ebar + 16);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* skip_flag = reinterpret_cast<int*>(tmem_slot + 2);
 
@@ -279,6 +292,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             mbar_init(&tempty[a], CG == 2 ? 2 : 256);
         }
         mbar_init(drain, 1);
+        for (int b = 0; b < 16; ++b) mbar_init(&ebar[b], 1);
         *abort_flag = 0;
         *skip_flag = (p.epi.sc != nullptr && p.epi.sc->status != 0) ? 1 : 0;
         fence_barrier_init();
@@ -446,6 +460,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         const EpiParams& e = p.epi;
         constexpr int CPW = BN / 64;  // 32-column chunks per warp
         int it = 0;
+        // SwiGLU backward operand slots of this warp and their barrier phases
+        uint8_t* const eslot = stg_all + (warp - 2) * kEpiLdWarpBytes;
+        uint64_t* const ebw = ebar + 2 * (warp - 2);
+        uint32_t eph = 0, epend = 0;   // phase bit and in-flight flag per slot
+        auto eissue = [&](int slot, int col, int rowg) {   // lane 0 only
+            fence_proxy_async_shared();   // this warp's reads of the slot precede the refill
+            mbar_arrive_expect_tx(&ebw[slot], 2 * kEpiLdBlock);
+            tma_load_2d(eslot + slot * 2 * kEpiLdBlock, &p.mapE[0], &ebw[slot], col, rowg);
+            tma_load_2d(eslot + slot * 2 * kEpiLdBlock + kEpiLdBlock, &p.mapE[1], &ebw[slot], col, rowg);
+            epend |= 1u << slot;
+        };
         for (int w = unit; w < num_work; w += nunits, ++it) {
             const int tile = w / p.ksplit;
             // split-K: each K range stores its raw fp32 tile into its own slice
@@ -470,8 +495,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
             uint8_t* stg = stg_all + (warp - 2) * (EPI == EPI_UPDATE ? kUpdStgBytes : C::NBUF * kStgBytes);
-            if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
-            if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
+            if (EPI == EPI_SWIGLU_BWD) {
+                // the first two blocks of this warp's part of the tile
+                if (lane == 0)
+                    for (int j = 0; j < 2 && j < CPW; ++j)
+                        if (n0 + 32 * (c0 + j) < p.N) eissue(j, n0 + 32 * (c0 + j), row0);
+            } else {
+                if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
+                if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
+            }
             if (kb_total > 0) {
                 if (!mbar_wait_bounded(&tfull[acc], (it >> 1) & 1, abort_flag)) break;
                 tc_fence_after();
@@ -643,38 +675,74 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     stg_scatter(e.out2, e.ld_out2, row0, p.M, n, p.N, stg + kStgBytes, v);
                     stg_scatter(e.out3, e.ld_out3, row0, p.M, n, p.N, stg + 2 * kStgBytes, u);
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const float g = round_bf16(v[i]);
-                        v[i] = g * fast_sigmoid(g) * round_bf16(u[i]);
+                    for (int i = 0; i < 32; i += 2) {   // SiLU(g) * u on the bf16-rounded G and U
+                        const float2 g = make_float2(round_bf16(v[i]), round_bf16(v[i + 1]));
+                        const float2 uu = make_float2(round_bf16(u[i]), round_bf16(u[i + 1]));
+                        const float2 a = mul2(mul2(g, sigmoid2(g)), uu);
+                        v[i] = a.x;
+                        v[i + 1] = a.y;
                     }
                     stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg, v);
                 }
             } else if constexpr (EPI == EPI_SWIGLU_BWD) {
                 float g[32], u[32];
+                bool ok = true;
 #pragma unroll 1
                 for (int j = 0; j < CPW; ++j) {
                     const int c = c0 + j;
                     const int n = n0 + c * 32;
                     if (n >= p.N) break;
+                    const int slot = j & 1;
+                    if (!mbar_wait_bounded(&ebw[slot], (eph >> slot) & 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    eph ^= 1u << slot;
+                    epend &= ~(1u << slot);
+                    {   // row `lane` of the G and U blocks (64-byte swizzle)
+                        const uint8_t* bg = eslot + slot * 2 * kEpiLdBlock + lane * 64;
+                        const int sw = (lane >> 1) & 3;
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const uint4 wg = *reinterpret_cast<const uint4*>(bg + 16 * (k ^ sw));
+                            const uint4 wu = *reinterpret_cast<const uint4*>(bg + kEpiLdBlock + 16 * (k ^ sw));
+                            const uint32_t a4[4] = {wg.x, wg.y, wg.z, wg.w};
+                            const uint32_t b4[4] = {wu.x, wu.y, wu.z, wu.w};
+#pragma unroll
+                            for (int q2 = 0; q2 < 4; ++q2) {
+                                g[8 * k + 2 * q2] = bf16_lo(a4[q2]);
+                                g[8 * k + 2 * q2 + 1] = bf16_hi(a4[q2]);
+                                u[8 * k + 2 * q2] = bf16_lo(b4[q2]);
+                                u[8 * k + 2 * q2 + 1] = bf16_hi(b4[q2]);
+                            }
+                        }
+                    }
+                    fence_proxy_async_shared();   // every lane's reads of the slot before its refill
+                    __syncwarp();
+                    if (lane == 0 && j + 2 < CPW && n + 64 < p.N) eissue(slot, n + 64, row0);
                     tmem_load32(tbase + c * 32, v);
                     if (valid) {
-                        unpack32_dyn(xa, 0, g);
-                        unpack32_dyn(xb, 0, u);
-                        if (j + 1 < CPW) {
-                            load_chunk_bf16(pa, ra, n + 32, p.N, xa, 0);
-                            load_chunk_bf16(pb, rb, n + 32, p.N, xb, 0);
-                        }
                         float du[32];
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const float sg = fast_sigmoid(g[i]);
-                            du[i] = v[i] * g[i] * sg;
-                            v[i] = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
+                        for (int i = 0; i < 32; i += 2) {
+                            // dU = dA SiLU(g), dG = dA u SiLU'(g), SiLU'(g) = s (1 + g (1 - s))
+                            const float2 gg = make_float2(g[i], g[i + 1]);
+                            const float2 sg = sigmoid2(gg);
+                            const float2 vs = mul2(make_float2(v[i], v[i + 1]), sg);
+                            const float2 d_u = mul2(vs, gg);
+                            const float2 k = fma2(gg, add2(make_float2(1.0f, 1.0f), make_float2(-sg.x, -sg.y)),
+                                                  make_float2(1.0f, 1.0f));
+                            const float2 d_g = mul2(mul2(vs, make_float2(u[i], u[i + 1])), k);
+                            du[i] = d_u.x;
+                            du[i + 1] = d_u.y;
+                            v[i] = d_g.x;
+                            v[i + 1] = d_g.y;
                         }
                         store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
                         store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, p.N, e.out2_f32, du);
                     }
                 }
+                if (!ok) break;
             }
             tc_fence_before();
             if constexpr (CG == 2) {
@@ -685,6 +753,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 mbar_arrive(&tempty[acc]);
             }
         }
+        // SwiGLU backward operand loads still in flight (an aborted tile) land
+        // before the CTA may exit
+        if (EPI == EPI_SWIGLU_BWD && lane == 0)
+            for (int sl = 0; sl < 2; ++sl)
+                if (epend & (1u << sl)) mbar_wait_bounded(&ebw[sl], (eph >> sl) & 1u, nullptr);
     }
 
     __syncthreads();
@@ -719,7 +792,8 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // 2-D bf16 tensor map: `inner` contiguous elements per row, `outer` rows of
 // pitch `ld` elements; box of box_inner x box_outer with 128-byte swizzle.
 static bool make_map(CUtensorMap* map, const void* ptr, int64_t inner, int64_t outer, int64_t ld,
-                     uint32_t box_inner, uint32_t box_outer) {
+                     uint32_t box_inner, uint32_t box_outer,
+                     CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
     auto fn = encode_fn();
     if (!fn) return false;
     if ((reinterpret_cast<uintptr_t>(ptr) & 15u) != 0) return false;
@@ -729,7 +803,7 @@ static bool make_map(CUtensorMap* map, const void* ptr, int64_t inner, int64_t o
     cuuint32_t box[2] = {box_inner, box_outer};
     cuuint32_t estr[2] = {1, 1};
     CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
@@ -905,6 +979,10 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
             return BOM_ENOTSUP;
         }
     }
+    if (g.epi_kind == EPI_SWIGLU_BWD &&
+        (!make_map(&p.mapE[0], g.epi.aux, g.N, g.M, g.epi.ld_aux, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B) ||
+         !make_map(&p.mapE[1], g.epi.aux2, g.N, g.M, g.epi.ld_aux2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)))
+        return BOM_ENOTSUP;
     p.M = static_cast<int>(g.M);
     p.N = static_cast<int>(g.N);
     p.nseg = g.nseg;
