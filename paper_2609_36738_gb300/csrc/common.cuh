@@ -158,6 +158,12 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
         : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
     return d;
 }
+// Hardware square root (PTX sqrt.approx.ftz.f32).
+__device__ __forceinline__ float sqrt_fast(float x) {
+    float y;
+    asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
 // Hardware reciprocal (PTX rcp.approx.ftz.f32, about 1 ulp).
 __device__ __forceinline__ float rcp_fast(float x) {
     float y;
