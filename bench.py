@@ -327,6 +327,9 @@ def main():
                 "frac_of_burst_peak": achieved / peaks["bf16_tflops"],
                 "flops_per_launch": fl / cnt, "launches": cnt, "avg_launch_ms": ms / cnt,
                 "share_of_device_time": ms / total_dev}
+        if name == "gemm_tc.update.mm":
+            roof["note"] = ("weight-gradient GEMMs whose epilogue also applies the BOM-AdamW update of each weight "
+                            "(18 B/element of theta, v and the bf16 copy); the time includes that update")
     else:
         achieved = by / (ms / 1e3) / 1e9
         roof = {"bound": "hbm", "kernel": name, "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
