@@ -166,9 +166,8 @@ __device__ __forceinline__ void stg_scatter(void* base, int64_t ld, int row0, in
 // the eight buffers leave room for six pipeline stages), then the warp walks
 // the 32 rows with lane l on column l, so every access to theta, v and the
 // compute copy is one coalesced 128-byte (64-byte for bf16) line per row.
-// Sixteen rows are loaded before any is written; theta and v were prefetched
-// into L2 while the warp waited for the tile's accumulator, and the step uses
-// the hardware square root and reciprocal.
+// Sixteen rows are loaded before any is written, and the step uses the
+// hardware square root and reciprocal.
 constexpr int kUpdPitch = 33;
 constexpr int kUpdStgBytes = 32 * kUpdPitch * 4;
 __device__ __forceinline__ void staged_update32(const EpiParams& e, float* buf, int row0, int M, int n, int N,
@@ -498,20 +497,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
             uint8_t* stg = stg_all + (warp - 2) * (EPI == EPI_UPDATE ? kUpdStgBytes : C::NBUF * kStgBytes);
-            if (EPI == EPI_UPDATE && valid) {
-                // theta and v of this row's part of the tile, into L2 while the
-                // mainloop runs
-                const int col = n0 + 32 * c0;
-                if (col < p.N) {
-                    const int cols = min(p.N - col, 32 * CPW);
-                    const uint32_t bytes = static_cast<uint32_t>(cols * 4) & ~15u;
-                    const int64_t off = static_cast<int64_t>(m) * e.ld_out + col;
-                    if (bytes) {
-                        prefetch_l2_bulk(e.upd_theta + off, bytes);
-                        prefetch_l2_bulk(e.upd_v + off, bytes);
-                    }
-                }
-            }
             if (EPI == EPI_SWIGLU_BWD) {
                 // the first two blocks of this warp's part of the tile
                 if (lane == 0)
