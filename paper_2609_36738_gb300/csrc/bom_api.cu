@@ -275,6 +275,30 @@ int run_gemm(bom_handle* h, GemmDesc& g, cudaStream_t s) {
                   [&] { return h->bf16 ? launch_gemm_tc(g, s) : launch_gemm_simt(g, s); });
 }
 
+// Several GEMMs that share layout, epilogue kind and K as one launch (the
+// tcgen05 path groups them into one work list; the SIMT path runs them in turn).
+int run_gemm_group(bom_handle* h, GemmDesc* gs, int n, cudaStream_t s) {
+    double flops = 0, bytes = 0;
+    for (int i = 0; i < n; ++i) {
+        GemmDesc& g = gs[i];
+        g.epi.sc = h->sc;
+        g.epi.in_f32 = h->bf16 ? 0 : 1;
+        const double k = static_cast<double>(g.K[0]);
+        flops += 2.0 * static_cast<double>(g.M) * g.N * k;
+        const double out_b = g.epi.upd_theta ? 16.0 + h->esz : (g.epi.out_f32 ? 4.0 : h->esz);
+        bytes += h->esz * (static_cast<double>(g.M) * k + static_cast<double>(g.N) * k) +
+                 out_b * static_cast<double>(g.M) * g.N;
+    }
+    return traced(h, s, gemm_name(gs[0], h->bf16), flops, bytes, [&] {
+        if (h->bf16) return launch_gemm_tc_group(gs, n, s);
+        for (int i = 0; i < n; ++i) {
+            const int rc = launch_gemm_simt(gs[i], s);
+            if (rc != BOM_OK) return rc;
+        }
+        return static_cast<int>(BOM_OK);
+    });
+}
+
 #define BOM_TRACED(name, flops, bytes, stmt) \
     traced(h, s, name, (flops), (bytes), [&] { stmt; return static_cast<int>(BOM_OK); })
 
@@ -586,6 +610,11 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
             g.epi.out_f32 = cf32;
             BOM_TRY(run_gemm(h, g, s));
         }
+        // The head weight gradient contracts over the same n rows as the
+        // first sublayer's weight gradients: with a SwiGLU first layer it
+        // waits and runs in one launch with them (every operand stays live).
+        GemmDesc head_dw;
+        const bool defer_head = h->bf16 && kfull == 1 && !h->lw.empty() && h->lw[0].kind == BOM_LAYER_SWIGLU;
         {   // head weight: a R^T H + b qhat (x) c
             GemmDesc g = gemm1(V, dm, kfull * n, mnmaj(h->Z, h->ldz), mnmaj(xin, dm));
             g.epi.alpha_const = 1.0f;
@@ -597,7 +626,10 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
             g.epi.ld_out = dm;
             g.epi.out_f32 = of32;
             if (fused) fuse(g, head_w);
-            BOM_TRY(run_gemm(h, g, s));
+            if (defer_head)
+                head_dw = g;
+            else
+                BOM_TRY(run_gemm(h, g, s));
         }
         if (head_b >= 0) {
             const float a = pass == 0 ? 1.0f - cfg.lambda : (pass == 1 || pass == 3 ? 1.0f : 0.0f);
@@ -651,27 +683,21 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                     g.epi.out_f32 = cf32;
                     BOM_TRY(run_gemm(h, g, s));
                 }
-                {   // dW_d = dy^T A
-                    GemmDesc g = gemm1(d, f, n, mnmaj(dcur, d), mnmaj(L.A, f));
-                    g.epi.out = fused ? nullptr : outp[p0 + 2];
-                    g.epi.ld_out = f;
-                    g.epi.out_f32 = of32;
-                    if (fused) fuse(g, p0 + 2);
-                    BOM_TRY(run_gemm(h, g, s));
-                }
-                {   // dW_g = dG^T x, dW_u = dU^T x
-                    GemmDesc g = gemm1(f, d, n, mnmaj(h->dG, f), mnmaj(xl, d));
-                    g.epi.out = fused ? nullptr : outp[p0];
-                    g.epi.ld_out = d;
-                    g.epi.out_f32 = of32;
-                    if (fused) fuse(g, p0);
-                    BOM_TRY(run_gemm(h, g, s));
-                    GemmDesc g2 = gemm1(f, d, n, mnmaj(h->dU, f), mnmaj(xl, d));
-                    g2.epi.out = fused ? nullptr : outp[p0 + 1];
-                    g2.epi.ld_out = d;
-                    g2.epi.out_f32 = of32;
-                    if (fused) fuse(g2, p0 + 1);
-                    BOM_TRY(run_gemm(h, g2, s));
+                {   // dW_g = dG^T x, dW_u = dU^T x, dW_d = dy^T A: one launch over their tiles
+                    GemmDesc gw[4];
+                    gw[0] = gemm1(f, d, n, mnmaj(h->dG, f), mnmaj(xl, d));
+                    gw[1] = gemm1(f, d, n, mnmaj(h->dU, f), mnmaj(xl, d));
+                    gw[2] = gemm1(d, f, n, mnmaj(dcur, d), mnmaj(L.A, f));
+                    const int pk[3] = {p0, p0 + 1, p0 + 2};
+                    for (int i = 0; i < 3; ++i) {
+                        gw[i].epi.out = fused ? nullptr : outp[pk[i]];
+                        gw[i].epi.ld_out = i < 2 ? d : f;
+                        gw[i].epi.out_f32 = of32;
+                        if (fused) fuse(gw[i], pk[i]);
+                    }
+                    int ng = 3;
+                    if (defer_head && l == 0) gw[ng++] = head_dw;   // the head's, deferred
+                    BOM_TRY(run_gemm_group(h, gw, ng, s));
                 }
             } else if (L.kind == BOM_LAYER_RMSNORM) {
                 const int64_t d = L.d_in;

@@ -40,6 +40,9 @@ struct GemmDesc {
 // Returns BOM_OK or an error status (BOM_ENOTSUP for unsupported layouts,
 // BOM_ECUDA for launch failures).
 int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream);
+// One persistent launch over n <= 4 GEMMs with the same layout, epilogue
+// kind and K and M > 128 (each GEMM launched alone otherwise).
+int launch_gemm_tc_group(const GemmDesc* g, int n, cudaStream_t stream);
 int launch_gemm_simt(const GemmDesc& g, cudaStream_t stream);
 
 // Number of column tiles of EPI_LOGITS statistics produced per row.

@@ -38,6 +38,13 @@ constexpr int NUM_THREADS = 320;  // producer warp, UMMA warp, 8 epilogue warps
 constexpr int TMEM_COLS = 512;
 constexpr int GROUP_M = 8;
 
+constexpr int kMaxGroup = 4;
+struct Prob {
+    CUtensorMap mapA, mapB;
+    int M, N, tiles_m, tiles_n;
+    EpiParams epi;
+};
+
 struct Params {
     CUtensorMap mapA[2];
     CUtensorMap mapB[2];
@@ -52,7 +59,46 @@ struct Params {
     int kb_split;          // k-blocks per K range
     int64_t split_bytes;   // byte distance between the fp32 partial slices of e.out
     EpiParams epi;
+    // Grouped launch: problems 1.. of the group (problem 0 is the fields
+    // above).  All problems share the layout, the epilogue kind and K; their
+    // tiles are numbered one problem after the other.
+    int nprob;
+    int tile_base[kMaxGroup + 1];
+    Prob grp[kMaxGroup - 1];
 };
+
+// Problem of `tile` (a tile index over the whole group) and its tile within it.
+struct ProbView {
+    const CUtensorMap* mapA;
+    const CUtensorMap* mapB;
+    const EpiParams* epi;
+    int M, N, tiles_m, tiles_n, local;
+};
+__device__ __forceinline__ ProbView prob_of(const Params& p, int tile) {
+    int q = 0;
+    while (q + 1 < p.nprob && tile >= p.tile_base[q + 1]) ++q;
+    ProbView v;
+    if (q == 0) {
+        v.mapA = &p.mapA[0];
+        v.mapB = &p.mapB[0];
+        v.epi = &p.epi;
+        v.M = p.M;
+        v.N = p.N;
+        v.tiles_m = p.tiles_m;
+        v.tiles_n = p.tiles_n;
+    } else {
+        const Prob& g = p.grp[q - 1];
+        v.mapA = &g.mapA;
+        v.mapB = &g.mapB;
+        v.epi = &g.epi;
+        v.M = g.M;
+        v.N = g.N;
+        v.tiles_m = g.tiles_m;
+        v.tiles_n = g.tiles_n;
+    }
+    v.local = tile - p.tile_base[q];
+    return v;
+}
 
 __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int& mt, int& nt) {
     const int per_group = GROUP_M * tiles_n;
@@ -319,7 +365,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
     const uint32_t tmem_base = *tmem_slot;
     const bool skip = *skip_flag != 0;
 
-    const int num_tiles = p.tiles_m * p.tiles_n;
+    const int num_tiles = p.tile_base[p.nprob];
     const int num_work = num_tiles * p.ksplit;   // (tile, K-split) work units
     const int kb_total = p.kb[0] + (p.nseg > 1 ? p.kb[1] : 0);
 
@@ -333,8 +379,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             for (int w = unit; ok && w < num_work; w += nunits) {
                 const int tile = w / p.ksplit;
                 const int sp = w - tile * p.ksplit;
+                const ProbView pv = prob_of(p, tile);
                 int mt, nt;
-                tile_coords(tile, p.tiles_m, p.tiles_n, mt, nt);
+                tile_coords(pv.local, pv.tiles_m, pv.tiles_n, mt, nt);
                 const int m_own = mt * C::TILE_M + static_cast<int>(rank) * BM;
                 const int n0 = nt * p.bn_out;
                 const int n_own = n0 + (CG == 2 && !p.dual_b ? static_cast<int>(rank) * C::B_ROWS : 0);
@@ -358,11 +405,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                             else
                                 tma_load_2d(dst, map, &full[stage], x, y);
                         };
+                        // grouped problems have one K segment: their maps come from pv
+                        const CUtensorMap* mA = seg == 0 ? pv.mapA : &p.mapA[1];
+                        const CUtensorMap* mB = seg == 0 ? pv.mapB : &p.mapB[1];
                         if (!A_MN) {
-                            load(a, &p.mapA[seg], k0, m_own);
+                            load(a, mA, k0, m_own);
                         } else {
-                            load(a, &p.mapA[seg], m_own, k0);
-                            load(a + 8192, &p.mapA[seg], m_own + 64, k0);
+                            load(a, mA, m_own, k0);
+                            load(a + 8192, mA, m_own + 64, k0);
                         }
                         if (p.dual_b) {
                             if constexpr (CG == 2) {
@@ -372,10 +422,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                                 load(b + 16384, &p.mapB[1], k0, n0);
                             }
                         } else if (!B_MN) {
-                            load(b, &p.mapB[seg], k0, n_own);
+                            load(b, mB, k0, n_own);
                         } else {
 #pragma unroll
-                            for (int j = 0; j < C::B_ROWS / 64; ++j) load(b + j * 8192, &p.mapB[seg], n_own + 64 * j, k0);
+                            for (int j = 0; j < C::B_ROWS / 64; ++j) load(b + j * 8192, mB, n_own + 64 * j, k0);
                         }
                         issued_mask |= 1u << stage;
                         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -459,7 +509,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         const int q = warp & 3;
         const int h = (warp - 2) >> 2;
         const int row = q * 32 + lane;
-        const EpiParams& e = p.epi;
         constexpr int CPW = BN / 64;  // 32-column chunks per warp
         int it = 0;
         // SwiGLU backward operand slots of this warp and their barrier phases
@@ -475,15 +524,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         };
         for (int w = unit; w < num_work; w += nunits, ++it) {
             const int tile = w / p.ksplit;
+            const ProbView pv = prob_of(p, tile);
+            const EpiParams& e = *pv.epi;
+            const int PM = pv.M, PN = pv.N;
             // split-K: each K range stores its raw fp32 tile into its own slice
             void* const out_base = static_cast<char*>(e.out) + static_cast<int64_t>(w - tile * p.ksplit) * p.split_bytes;
             int mt, nt;
-            tile_coords(tile, p.tiles_m, p.tiles_n, mt, nt);
+            tile_coords(pv.local, pv.tiles_m, pv.tiles_n, mt, nt);
             const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
             const int n0 = nt * p.bn_out;
             const int acc = it & 1;
             const int m = m0 + row;
-            const bool valid = m < p.M;
+            const bool valid = m < PM;
             const int c0 = h * CPW;
             // Per-row epilogue operands do not depend on the accumulator: the
             // warp's first chunk is loaded before the mainloop wait, and each
@@ -501,10 +553,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 // the first two blocks of this warp's part of the tile
                 if (lane == 0)
                     for (int j = 0; j < 2 && j < CPW; ++j)
-                        if (n0 + 32 * (c0 + j) < p.N) eissue(j, n0 + 32 * (c0 + j), row0);
+                        if (n0 + 32 * (c0 + j) < PN) eissue(j, n0 + 32 * (c0 + j), row0);
             } else {
-                if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, p.N, xa, 0);
-                if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, p.N, xb, 0);
+                if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, PN, xa, 0);
+                if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, PN, xb, 0);
             }
             if (kb_total > 0) {
                 if (!mbar_wait_bounded(&tfull[acc], (it >> 1) & 1, abort_flag)) break;
@@ -514,13 +566,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             float v[32];
 
             if constexpr (EPI == EPI_LINEAR) {
-                const EpiRow r = epi_row(e, m, p.M);
+                const EpiRow r = epi_row(e, m, PM);
                 float t[32];
 #pragma unroll 1
                 for (int j = 0; j < CPW; ++j) {
                     const int c = c0 + j;
                     const int n = n0 + c * 32;
-                    if (n >= p.N) break;
+                    if (n >= PN) break;
                     if (kb_total > 0) {
                         tmem_load32(tbase + c * 32, v);
                     } else {
@@ -531,47 +583,47 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] *= r.alpha;
                         if (e.bias) {
-                            load_row32(e.bias, 0, n, p.N, 0, t);
+                            load_row32(e.bias, 0, n, PN, 0, t);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] += t[i];
                         }
                         if (e.r1u) {
-                            load_vec32(e.r1v, n, p.N, t);
+                            load_vec32(e.r1v, n, PN, t);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] += r.beta_r1 * t[i];
                         }
                         if (e.bw) {
-                            load_vec32(e.bw, n, p.N, t);
+                            load_vec32(e.bw, n, PN, t);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] += r.beta_bw * t[i];
                         }
                         if (has_a) {
                             unpack32_dyn(xa, 0, t);
-                            if (j + 1 < CPW) load_chunk_bf16(pa, ra, n + 32, p.N, xa, 0);
+                            if (j + 1 < CPW) load_chunk_bf16(pa, ra, n + 32, PN, xa, 0);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] += t[i];
                         }
                         if (e.act == ACT_GELU) {
-                            store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, p.N, e.out2_f32, v);
+                            store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, PN, e.out2_f32, v);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] = gelu_f(e.out2_f32 ? v[i] : round_bf16(v[i]));
                         } else if (has_b) {
                             unpack32_dyn(xb, 0, t);
-                            if (j + 1 < CPW) load_chunk_bf16(pb, rb, n + 32, p.N, xb, 0);
+                            if (j + 1 < CPW) load_chunk_bf16(pb, rb, n + 32, PN, xb, 0);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) v[i] *= gelu_grad_f(t[i]);
                         }
-                        store_row32(out_base, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
+                        store_row32(out_base, static_cast<int64_t>(m) * e.ld_out, n, PN, e.out_f32, v);
                     }
                 }
             } else if constexpr (EPI == EPI_UPDATE) {
-                const EpiRow r = epi_row(e, m, p.M);
+                const EpiRow r = epi_row(e, m, PM);
                 float t[32];
 #pragma unroll 1
                 for (int j = 0; j < CPW; ++j) {
                     const int c = c0 + j;
                     const int n = n0 + c * 32;
-                    if (n >= p.N) break;
+                    if (n >= PN) break;
                     if (kb_total > 0) {
                         tmem_load32(tbase + c * 32, v);
                     } else {
@@ -581,11 +633,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] *= r.alpha;
                     if (e.r1u) {
-                        load_vec32(e.r1v, n, p.N, t);
+                        load_vec32(e.r1v, n, PN, t);
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] += r.beta_r1 * t[i];
                     }
-                    staged_update32(e, reinterpret_cast<float*>(stg), row0, p.M, n, p.N, v);
+                    staged_update32(e, reinterpret_cast<float*>(stg), row0, PM, n, PN, v);
                 }
             } else if constexpr (EPI == EPI_LOGITS || EPI == EPI_LOGITS_STG) {
                 // per (row, column half) softmax statistics: stats pair nt*2 + h.
@@ -597,20 +649,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 for (int j = 0; j < CPW; ++j) {
                     const int c = c0 + j;
                     const int n = n0 + c * 32;
-                    if (n >= p.N) break;
+                    if (n >= PN) break;
                     tmem_load32(tbase + c * 32, v);
                     if (e.bias) {
-                        load_row32(e.bias, 0, n, p.N, 0, t);
+                        load_row32(e.bias, 0, n, PN, 0, t);
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] += t[i];
                     }
-                    if (n + 32 <= p.N) {
+                    if (n + 32 <= PN) {
                         // full chunk: packed rounding, packed max, paired exponentials
                         uint32_t b[16];
 #pragma unroll
                         for (int i = 0; i < 16; ++i) b[i] = cvt_bf16x2(v[2 * i], v[2 * i + 1]);
                         if constexpr (EPI == EPI_LOGITS_STG)
-                            stg_scatter_bf16(e.out, e.ld_out, row0, p.M, n, p.N, stg, b);
+                            stg_scatter_bf16(e.out, e.ld_out, row0, PM, n, PN, stg, b);
                         else if (valid) {
                             uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(e.out) +
                                                                   static_cast<int64_t>(m) * e.ld_out + n);
@@ -645,18 +697,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = round_bf16(v[i]);
                     if constexpr (EPI == EPI_LOGITS_STG)
-                        stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg, v);
+                        stg_scatter(e.out, e.ld_out, row0, PM, n, PN, stg, v);
                     else if (valid)
-                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, 0, v);
+                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, PN, 0, v);
                     float cm = -INFINITY;
 #pragma unroll
                     for (int i = 0; i < 32; ++i)
-                        if (n + i < p.N) cm = fmaxf(cm, v[i]);
+                        if (n + i < PN) cm = fmaxf(cm, v[i]);
                     const float nm = fmaxf(mx, cm);
                     float s = (mx == -INFINITY) ? 0.0f : sm * fast_exp(mx - nm);
 #pragma unroll
                     for (int i = 0; i < 32; ++i)
-                        if (n + i < p.N) s += fast_exp(v[i] - nm);
+                        if (n + i < PN) s += fast_exp(v[i] - nm);
                     mx = nm;
                     sm = s;
                 }
@@ -671,11 +723,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 for (int j = 0; j < 2; ++j) {
                     const int c = 2 * h + j;
                     const int n = n0 + c * 32;
-                    if (n >= p.N) break;
+                    if (n >= PN) break;
                     tmem_load32(tbase + c * 32, v);
                     tmem_load32(tbase + 128 + c * 32, u);
-                    stg_scatter(e.out2, e.ld_out2, row0, p.M, n, p.N, stg + kStgBytes, v);
-                    stg_scatter(e.out3, e.ld_out3, row0, p.M, n, p.N, stg + 2 * kStgBytes, u);
+                    stg_scatter(e.out2, e.ld_out2, row0, PM, n, PN, stg + kStgBytes, v);
+                    stg_scatter(e.out3, e.ld_out3, row0, PM, n, PN, stg + 2 * kStgBytes, u);
 #pragma unroll
                     for (int i = 0; i < 32; i += 2) {   // SiLU(g) * u on the bf16-rounded G and U
                         const float2 g = make_float2(round_bf16(v[i]), round_bf16(v[i + 1]));
@@ -684,7 +736,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         v[i] = a.x;
                         v[i + 1] = a.y;
                     }
-                    stg_scatter(e.out, e.ld_out, row0, p.M, n, p.N, stg, v);
+                    stg_scatter(e.out, e.ld_out, row0, PM, n, PN, stg, v);
                 }
             } else if constexpr (EPI == EPI_SWIGLU_BWD) {
                 float g[32], u[32];
@@ -693,7 +745,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 for (int j = 0; j < CPW; ++j) {
                     const int c = c0 + j;
                     const int n = n0 + c * 32;
-                    if (n >= p.N) break;
+                    if (n >= PN) break;
                     const int slot = j & 1;
                     if (!mbar_wait_bounded(&ebw[slot], (eph >> slot) & 1u, abort_flag)) {
                         ok = false;
@@ -721,7 +773,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     }
                     fence_proxy_async_shared();   // every lane's reads of the slot before its refill
                     __syncwarp();
-                    if (lane == 0 && j + 2 < CPW && n + 64 < p.N) eissue(slot, n + 64, row0);
+                    if (lane == 0 && j + 2 < CPW && n + 64 < PN) eissue(slot, n + 64, row0);
                     tmem_load32(tbase + c * 32, v);
                     if (valid) {
                         float du[32];
@@ -740,8 +792,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                             v[i] = d_g.x;
                             v[i + 1] = d_g.y;
                         }
-                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, p.N, e.out_f32, v);
-                        store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, p.N, e.out2_f32, du);
+                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, PN, e.out_f32, v);
+                        store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, PN, e.out2_f32, du);
                     }
                 }
                 if (!ok) break;
@@ -846,7 +898,7 @@ static int launch_inst(const Params& p, cudaStream_t stream) {
             max_units = device_sm_count();
         }
     }
-    const int work = p.tiles_m * p.tiles_n * p.ksplit;
+    const int work = p.tile_base[p.nprob] * p.ksplit;
     const int units = work < max_units ? work : max_units;
     if constexpr (CG == 2) {
         cudaLaunchConfig_t cfg = {};
@@ -995,6 +1047,9 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     p.epi = g.epi;
     const int kb_total = p.kb[0] + (p.nseg > 1 ? p.kb[1] : 0);
     const int tiles = p.tiles_m * p.tiles_n;
+    p.nprob = 1;
+    p.tile_base[0] = 0;
+    p.tile_base[1] = tiles;
     const int units = cg == 2 ? device_sm_count() / 2 : device_sm_count();
     int S = 1;
     if ((g.epi_kind == EPI_LINEAR || g.epi_kind == EPI_UPDATE) && g.splitk_ws != nullptr)
@@ -1026,6 +1081,70 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     splitk_reduce_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(g.splitk_ws, p.ksplit, p.M, p.N, g.epi);
     count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+}  // namespace bom
+
+namespace bom {
+
+// One persistent launch over up to kMaxGroup GEMMs that share the operand
+// layout, the epilogue kind and K (the weight gradients of a SwiGLU sublayer,
+// with the head's): their tiles form one work list, so the last wave is
+// shared instead of each GEMM ending on its own partial wave.  Falls back to
+// separate launches when the GEMMs do not fit one launch.
+int launch_gemm_tc_group(const GemmDesc* gs, int n, cudaStream_t stream) {
+    using namespace tc;
+    bool ok = n >= 1 && n <= kMaxGroup;
+    for (int i = 0; ok && i < n; ++i) {
+        const GemmDesc& g = gs[i];
+        ok = g.nseg == 1 && !g.dual_b && !g.epi.in_f32 && g.M > BM && g.N > 0 && g.K[0] == gs[0].K[0] &&
+             g.epi_kind == gs[0].epi_kind && g.A[0].mn_major == gs[0].A[0].mn_major &&
+             g.B[0].mn_major == gs[0].B[0].mn_major && g.M <= INT32_MAX / 2 && g.N <= INT32_MAX / 2;
+    }
+    if (!ok) {
+        for (int i = 0; i < n; ++i) {
+            const int rc = launch_gemm_tc(gs[i], stream);
+            if (rc != BOM_OK) return rc;
+        }
+        return BOM_OK;
+    }
+    Params p;
+    memset(&p, 0, sizeof(p));
+    const GemmDesc& g0 = gs[0];
+    p.kb[0] = static_cast<int>((g0.K[0] + BK - 1) / BK);
+    p.nseg = 1;
+    p.bn_out = BN;
+    p.ksplit = 1;
+    p.kb_split = p.kb[0];
+    p.nprob = n;
+    int tiles = 0;
+    for (int i = 0; i < n; ++i) {
+        const GemmDesc& g = gs[i];
+        CUtensorMap* ma = i == 0 ? &p.mapA[0] : &p.grp[i - 1].mapA;
+        CUtensorMap* mb = i == 0 ? &p.mapB[0] : &p.grp[i - 1].mapB;
+        if (g.K[0] > 0 && (!map_operand(ma, g.A[0], g.M, g.K[0], BM) || !map_operand(mb, g.B[0], g.N, g.K[0], 128)))
+            return BOM_ENOTSUP;
+        const int tm = static_cast<int>((g.M + 2 * BM - 1) / (2 * BM));
+        const int tn = static_cast<int>((g.N + BN - 1) / BN);
+        if (i == 0) {
+            p.M = static_cast<int>(g.M);
+            p.N = static_cast<int>(g.N);
+            p.tiles_m = tm;
+            p.tiles_n = tn;
+            p.epi = g.epi;
+        } else {
+            Prob& q = p.grp[i - 1];
+            q.M = static_cast<int>(g.M);
+            q.N = static_cast<int>(g.N);
+            q.tiles_m = tm;
+            q.tiles_n = tn;
+            q.epi = g.epi;
+        }
+        p.tile_base[i] = tiles;
+        tiles += tm * tn;
+    }
+    p.tile_base[n] = tiles;
+    return dispatch<2>(p, g0.epi_kind, g0.A[0].mn_major, g0.B[0].mn_major, false, stream);
 }
 
 }  // namespace bom

@@ -224,6 +224,12 @@ TINY_RAGGED_F32 = Workload("tiny_ragged_f32", 37, 29, (Layer(LINEAR_GELU, 29, 45
 LM_HEAD_WIDE = Workload("lm_head_wide", 256, 128, (), 8192, False, "bf16", "zipf",
                         head_init="normal002", ignore_frac=0.05)
 
+# SwiGLU widths above one 128-row tile everywhere (d 256, ffn 576), so the
+# three weight-gradient GEMMs of a sublayer run as one grouped launch, with
+# ragged tiles in the ffn direction.
+LM_MLP_MID = Workload("lm_mlp_mid", 300, 256, (Layer(SWIGLU, 256, 576), Layer(SWIGLU, 256, 576)),
+                      1000, False, "bf16", "zipf", head_init="normal002", ignore_frac=0.05)
+
 # RMSNorm variants: an LM block whose head input is normalised (one SwiGLU
 # sublayer, then the final norm, as in the paper's Qwen3 models), and an fp32
 # MLP with a norm between two linear layers.
@@ -238,7 +244,7 @@ LM_NORM_BF16 = Workload("lm_norm_bf16", 16384, 2048,
 
 WORKLOADS = {w.name: w for w in (TINY_MLP_F32, VISION_HEAD_BF16, LM_HEAD_BF16, LM_MLP_BF16,
                                   LM_HEAD_SMALL, LM_MLP_SMALL, VISION_SMALL, TINY_RAGGED_F32, LM_HEAD_WIDE,
-                                  LM_NORM_SMALL, TINY_NORM_F32, LM_NORM_BF16)}
+                                  LM_NORM_SMALL, TINY_NORM_F32, LM_NORM_BF16, LM_MLP_MID)}
 
 
 # --------------------------------------------------------------------------

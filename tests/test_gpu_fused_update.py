@@ -42,7 +42,8 @@ class Fused:
 
 
 @pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "tiny_norm_f32", "vision_small",
-                                  "lm_head_small", "lm_mlp_small", "lm_norm_small", "lm_head_wide"])
+                                  "lm_head_small", "lm_mlp_small", "lm_norm_small", "lm_head_wide",
+                                  "lm_mlp_mid"])
 def test_fused_update_matches_oracle_on_the_same_inputs(name):
     wl = I.WORKLOADS[name]
     tol = G.TOL[wl.dtype]
