@@ -370,6 +370,9 @@ def main():
         extra["lm_head_bf16"] = _head_only(B, torch, dev, stream, a, peaks)
         extra["update_1e9"] = _update_only(B, torch, dev, stream, a, peaks)
         extra["update_adam_mini_lm_block"] = _adam_mini_only(B, torch, dev, stream, a, peaks)
+        extra["update_clipped_lm_block"] = _clipped_update(B, torch, dev, stream, a, peaks)
+        extra["telemetry_step_lm_block"] = _telemetry_step(B, torch, dev, stream, a, peaks)
+        extra["rmsnorm_lm_block"] = _rmsnorm_step(B, torch, dev, stream, a, peaks)
 
     cpu = None
     if rank == 0 and world == 1 and not a.no_cpu:
@@ -483,6 +486,153 @@ def _update_only(B, torch, dev, stream, a, peaks):
     return {"workload": "update sweep, 1e9 elements: read theta f32, g bf16, h f32, v f32; write theta, v "
                         "(22 B/element)", "value": gbs, "unit": "GB/s", "ms": med,
             "frac_of_hbm": gbs / peaks["hbm_gbs"], "peak_source": "measured copy bandwidth"}
+
+
+def _lm_state(B, torch, dev, wl, seed=0):
+    """Device parameters (bf16), fp32 masters, a batch and q for workload wl."""
+    params_np = I.init_params(wl, seed)
+    params = [torch.from_numpy(p.view(np.int16)).to(dev).view(torch.bfloat16) for p in params_np]
+    theta = [torch.from_numpy(I.bf16_to_f32(p)).to(dev) for p in params_np]
+    x_np, y_np = I.make_batch(wl, seed, 1)
+    x = torch.from_numpy(x_np.view(np.int16)).to(dev).view(torch.bfloat16)
+    y = torch.from_numpy(y_np).to(dev)
+    q = torch.zeros(wl.vocab, dtype=torch.float32, device=dev)
+    return params, theta, x, y, q
+
+
+def _timed(torch, stream, fn, n_iter, flush):
+    """Median CUDA-event time (ms) of fn() over n_iter runs, L2 flushed before each."""
+    ms = []
+    for i in range(n_iter):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn(i)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    return statistics.median(ms)
+
+
+def _clipped_update(B, torch, dev, stream, a, peaks):
+    """Global-norm clipping of u over the LM block's 166,199,296 parameters:
+    the fixed-order sum of u^2 (bf16 u) and the clipped BOM-AdamW update."""
+    wl = I.LM_MLP_BF16
+    P = wl.n_params()
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1)
+    theta = torch.randn(P, generator=gen, device=dev) * 1e-2
+    u = (torch.randn(P, generator=gen, device=dev) * 1e-3).to(torch.bfloat16)
+    v = torch.zeros(P, dtype=torch.float32, device=dev)
+    shadow = torch.empty(P, dtype=torch.bfloat16, device=dev)
+    sq = torch.zeros(1, dtype=torch.float64, device=dev)
+    m = B.BomModel(B.config_for(I.TINY_MLP_F32))   # a handle for the partials buffer
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)
+
+    def run(i):
+        sq.zero_()
+        B.bom_sqnorm(m.h, u, B.BOM_BF16, None, LAM, P, sq, stream)
+        B.bom_update_clipped(theta, u, B.BOM_BF16, None, v, shadow, P, LR, WD, LAM, B2, EPS, 4 + i, sq, 1.0, stream)
+
+    for i in range(3):
+        run(i)
+    ms = _timed(torch, stream, run, max(5, a.steps // 2), flush)
+    m.close()
+    gbs = 22.0 * P / (ms / 1e3) / 1e9
+    del theta, u, v, shadow
+    torch.cuda.empty_cache()
+    return {"workload": "global-norm clipping (max norm 1.0) of bf16 u over 166,199,296 parameters: sum of u^2 "
+                        "(2 B/element) + clipped update (read theta, u, v; write theta, v, bf16 copy: 20 B/element)",
+            "value": gbs, "unit": "GB/s", "ms": ms, "frac_of_hbm": gbs / peaks["hbm_gbs"],
+            "peak_source": "measured copy bandwidth"}
+
+
+def _telemetry_step(B, torch, dev, stream, a, peaks):
+    """Own-step control with drift telemetry on the LM block (16384 tokens):
+    one bom_step in G_AND_H mode with an own-step output (backward passes for
+    g, h = Jbar^T qhat and o = Jbar^T s_t, residual norms), then the own-step
+    moment with the drift sums of head and encoder over all parameters."""
+    wl = I.LM_MLP_BF16
+    params, theta, x, y, q = _lm_state(B, torch, dev, wl)
+    f32 = torch.float32
+    grads = [torch.empty_like(p) for p in params]
+    hs = [torch.empty(p.shape, dtype=f32, device=dev) for p in params]
+    os_ = [torch.empty(p.shape, dtype=f32, device=dev) for p in params]
+    Ms = [torch.zeros(p.shape, dtype=f32, device=dev) for p in params]
+    mh = [torch.empty(p.shape, dtype=f32, device=dev) for p in params]
+    sums = torch.zeros((2, 4), dtype=torch.float64, device=dev)
+    m = B.BomModel(B.config_for(wl, LAM, B1, B.BOM_OUT_G_AND_H))
+    B.bom_set_own_step_output(m.h, os_)
+    head = len(params) - 1
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)
+    per = {}
+
+    def moments(t):
+        sums.zero_()
+        for k in range(len(params)):
+            B.bom_own_step_moment(m.h, Ms[k], os_[k], hs[k], mh[k], Ms[k].numel(), B1, t,
+                                  sums[0] if k == head else sums[1], stream)
+
+    def run(i):
+        t = 1 + i
+        m.step(x, y, wl.n_rows, params, q, t, grads, hs, stream)
+        moments(t)
+
+    for i in range(2):
+        run(i)
+    B.bom_trace(m.h, True)
+    ms = _timed(torch, stream, lambda i: run(3 + i), max(3, a.steps // 4), flush)
+    for name, fl, by, kms in B.bom_trace_read(m.h, stream):
+        per[name] = per.get(name, 0.0) + kms
+    mom_ms = _timed(torch, stream, lambda i: moments(20 + i), 3, flush)
+    st = m.stats(stream)
+    s_ = sums.cpu().numpy()
+    P = wl.n_params()
+    m.close()
+    del grads, hs, os_, Ms, mh, params, theta
+    torch.cuda.empty_cache()
+    return {"workload": "LM block + 2 SwiGLU MLPs, 16384 tokens: own-step control step with drift telemetry "
+                        "(forward, task space, three backward passes g / h / own-step, residual norms, "
+                        "M_t and the drift sums over 166,199,296 parameters)",
+            "value": wl.n_rows / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "cancel_ratio": st["cancel"],
+            "drift_cos_head": float(s_[0, 0] / np.sqrt(s_[0, 1] * s_[0, 2])),
+            "drift_cos_encoder": float(s_[1, 0] / np.sqrt(s_[1, 1] * s_[1, 2])),
+            "moment_pass_ms": mom_ms, "moment_pass_gbs": 20.0 * P / (mom_ms / 1e3) / 1e9,
+            "kernels_ms_last_step": {k: round(v, 4) for k, v in sorted(per.items(), key=lambda kv: -kv[1])}}
+
+
+def _rmsnorm_step(B, torch, dev, stream, a, peaks):
+    """The LM block with a final RMSNorm before the head (16384 tokens, the
+    update fused), against the same step without the norm."""
+    wl = I.LM_NORM_BF16
+    params, theta, x, y, q = _lm_state(B, torch, dev, wl)
+    v = [torch.zeros_like(t) for t in theta]
+    m = B.BomModel(B.config_for(wl, LAM, B1))
+    B.bom_set_fused_update(m.h, theta, v, I.weight_decay_mask(wl, WD), LR, B2, EPS)
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)
+
+    def run(i):
+        m.step(x, y, wl.n_rows, params, q, 1 + i, None, None, stream)
+
+    for i in range(3):
+        run(i)
+    B.bom_trace(m.h, True)
+    ms = _timed(torch, stream, lambda i: run(4 + i), max(3, a.steps // 4), flush)
+    per = {}
+    for name, fl, by, kms in B.bom_trace_read(m.h, stream):
+        if name.startswith("rmsnorm") or name == "colsum":
+            d = per.setdefault(name, [0.0, 0.0])
+            d[0] += by
+            d[1] += kms
+    m.stats(stream)
+    m.close()
+    del params, theta, v
+    torch.cuda.empty_cache()
+    return {"workload": "LM block + 2 SwiGLU MLPs + final RMSNorm (gamma, weight decay 0), 16384 tokens, "
+                        "BOM step with the fused update",
+            "value": wl.n_rows / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "norm_kernels": {k: {"ms": round(v[1], 4), "gbs": v[0] / (v[1] / 1e3) / 1e9} for k, v in per.items()}}
 
 
 def _adam_mini_only(B, torch, dev, stream, a, peaks):

@@ -194,7 +194,8 @@ bom_status bom_set_own_step_output(bom_handle* h, void* const* o);
  * in fp64 and a fixed summation order, from which cos(Mhat_t, h_t) and
  * ||Mhat_t - h_t|| / ||Mhat_t|| follow; calling it per tensor range with one
  * sums buffer per group (e.g. head, encoder) gives the paper's split.
- * M, o, hvec, mhat: device fp32 [n]; sums: device fp64 [4] or NULL.
+ * M, o, hvec, mhat: device fp32 [n], 16-byte aligned (else BOM_ENOTSUP);
+ * sums: device fp64 [4] or NULL.
  * Uses a per-handle partials buffer: calls on one handle must be ordered on
  * one stream.  Asynchronous; t >= 1 and 0 <= beta1 < 1 or BOM_EINVAL. */
 bom_status bom_own_step_moment(bom_handle* h, float* M, const float* o, const float* hvec, float* mhat,

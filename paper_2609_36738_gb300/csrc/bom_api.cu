@@ -799,6 +799,7 @@ bom_status bom_own_step_moment(bom_handle* h, float* M, const float* o, const fl
     if (!h || n < 0 || t < 1 || !(beta1 >= 0.0f && beta1 < 1.0f)) return BOM_EINVAL;
     if (n == 0) return BOM_OK;
     if (!M || !o || !mhat || (sums && !hvec)) return BOM_EINVAL;
+    if (!aligned16(M) || !aligned16(o) || !aligned16(mhat) || (hvec && !aligned16(hvec))) return BOM_ENOTSUP;
     const float inv_bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta1), static_cast<double>(t))));
     const int nb = own_step_blocks(n, device_sm_count());
     launch_own_step_moment(M, o, hvec, mhat, n, beta1, inv_bc1, h->tel_part, nb, sums,

@@ -340,20 +340,36 @@ __global__ void __launch_bounds__(256) own_step_moment_kernel(float* __restrict_
                                                               int64_t n, float beta1, float inv_bc1,
                                                               double* __restrict__ part) {
     float s_dot = 0.0f, s_mm = 0.0f, s_hh = 0.0f, s_dd = 0.0f;
+    auto one = [&](float& m, float oo, float h, float& mh) {
+        m = fmaf(beta1, m, (1.0f - beta1) * oo);
+        mh = m * inv_bc1;
+        const float d = mh - h;
+        s_dot = fmaf(mh, h, s_dot);
+        s_mm = fmaf(mh, mh, s_mm);
+        s_hh = fmaf(h, h, s_hh);
+        s_dd = fmaf(d, d, s_dd);
+    };
+    // 16-byte words (all pointers are 16-byte aligned), then the tail
+    const int64_t n4 = n >> 2;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += stride) {
-        const float m = fmaf(beta1, M[i], (1.0f - beta1) * o[i]);
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
+        float4 m = reinterpret_cast<const float4*>(M)[i];
+        const float4 oo = __ldcs(reinterpret_cast<const float4*>(o) + i);
+        const float4 h = hv ? __ldcs(reinterpret_cast<const float4*>(hv) + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 mh;
+        one(m.x, oo.x, h.x, mh.x);
+        one(m.y, oo.y, h.y, mh.y);
+        one(m.z, oo.z, h.z, mh.z);
+        one(m.w, oo.w, h.w, mh.w);
+        reinterpret_cast<float4*>(M)[i] = m;
+        __stcs(reinterpret_cast<float4*>(mhat) + i, mh);
+    }
+    if (blockIdx.x == 0 && threadIdx.x < (n & 3)) {
+        const int64_t i = (n4 << 2) + threadIdx.x;
+        float m = M[i], mh;
+        one(m, o[i], hv ? hv[i] : 0.0f, mh);
         M[i] = m;
-        const float mh = m * inv_bc1;
         mhat[i] = mh;
-        if (hv) {
-            const float h = hv[i];
-            const float d = mh - h;
-            s_dot = fmaf(mh, h, s_dot);
-            s_mm = fmaf(mh, mh, s_mm);
-            s_hh = fmaf(h, h, s_hh);
-            s_dd = fmaf(d, d, s_dd);
-        }
     }
     if (!part) return;
     __shared__ double red[4][8];

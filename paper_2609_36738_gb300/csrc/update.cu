@@ -196,14 +196,87 @@ __global__ void __launch_bounds__(256) update_blockshared_kernel(float* __restri
     }
 }
 
+// Blocks of at most 8192 elements (d % 4 == 0): each thread keeps its words
+// of u and theta in registers from one read, so the block costs one memory
+// round trip before the reduction and none after it.
+constexpr int kRegWords = 8;   // float4 words per thread: 256 x 8 x 4 = 8192 elements
+template <bool G_BF16, bool HAS_H, bool SHADOW>
+__global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __restrict__ theta,
+                                                                     const void* __restrict__ g,
+                                                                     const float* __restrict__ h,
+                                                                     float* __restrict__ vb,
+                                                                     uint16_t* __restrict__ shadow, int64_t n,
+                                                                     int64_t block, UpdCoef c) {
+    __shared__ float red[8];
+    __shared__ float s_den;
+    const int64_t nb = (n + block - 1) / block;
+    for (int64_t b = blockIdx.x; b < nb; b += gridDim.x) {
+        const int64_t e0 = b * block;
+        const int64_t e1 = e0 + block < n ? e0 + block : n;
+        float u[kRegWords][4];
+        float4 th[kRegWords];
+        float acc = 0.0f;
+#pragma unroll
+        for (int k = 0; k < kRegWords; ++k) {
+            const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
+            if (i < e1) {
+                load_u<G_BF16, HAS_H, 4>(g, h, i, c.lam, u[k]);
+                th[k] = __ldcs(reinterpret_cast<const float4*>(theta + i));
+#pragma unroll
+                for (int q = 0; q < 4; ++q) acc = fmaf(u[k][q], u[k][q], acc);
+            }
+        }
+        acc = warp_sum_f(acc);
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float tot = 0.0f;
+#pragma unroll
+            for (int w = 0; w < 8; ++w) tot += red[w];
+            const float vv = fmaf(c.beta2, vb[b], c.one_m_beta2 * (tot / static_cast<float>(e1 - e0)));
+            vb[b] = vv;
+            s_den = sqrtf(vv * c.inv_bc2) + c.eps;
+        }
+        __syncthreads();
+        const float den = s_den;
+#pragma unroll
+        for (int k = 0; k < kRegWords; ++k) {
+            const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
+            if (i < e1) {
+                float4 t = th[k];
+                t.x = c.decay * t.x - c.lr * (u[k][0] / den);
+                t.y = c.decay * t.y - c.lr * (u[k][1] / den);
+                t.z = c.decay * t.z - c.lr * (u[k][2] / den);
+                t.w = c.decay * t.w - c.lr * (u[k][3] / den);
+                __stcs(reinterpret_cast<float4*>(theta + i), t);
+                if constexpr (SHADOW) {
+                    uint2 sh;
+                    sh.x = pack_bf16x2(t.x, t.y);
+                    sh.y = pack_bf16x2(t.z, t.w);
+                    __stcs(reinterpret_cast<uint2*>(shadow + i), sh);
+                }
+            }
+        }
+        __syncthreads();   // red and s_den are reused by the next block
+    }
+}
+
 template <bool G_BF16, bool HAS_H, int VEC>
 void dispatch_blockshared(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
                           int64_t block, const UpdCoef& c, int grid, cudaStream_t s) {
-    if (shadow)
+    if (VEC == 4 && block <= 256 * 4 * kRegWords) {
+        if (shadow)
+            update_blockshared_reg_kernel<G_BF16, HAS_H, true><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n, block,
+                                                                                   c);
+        else
+            update_blockshared_reg_kernel<G_BF16, HAS_H, false><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n,
+                                                                                    block, c);
+    } else if (shadow) {
         update_blockshared_kernel<G_BF16, HAS_H, true, VEC><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n, block, c);
-    else
+    } else {
         update_blockshared_kernel<G_BF16, HAS_H, false, VEC><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n, block,
                                                                                   c);
+    }
     count_launch();
 }
 

@@ -32,8 +32,10 @@ def _close(th_gpu, theta0, ref_th, rel=1e-5):
 # (n, block): per-output-neuron rows of the vision head and LM shapes, a ragged
 # last block, blocks that are not a multiple of 4, one whole-tensor block and
 # blocks of one element (elementwise BOM-AdamW).
+# The register-resident kernel takes blocks of up to 8192 elements (d % 4 = 0);
+# (3 x 16384, 16384) takes the two-sweep kernel, the odd sizes the scalar one.
 CASES = [(3072 * 768, 768), (64 * 2048, 2048), (8 * 8192, 8192), (1000, 300), (29 * 7, 29), (50_001, 50_001),
-         (4099, 1), (3, 5)]
+         (4099, 1), (3, 5), (3 * 16384, 16384)]
 
 
 @pytest.mark.parametrize("n,block", CASES)
