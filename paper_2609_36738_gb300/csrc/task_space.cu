@@ -349,13 +349,11 @@ __global__ void __launch_bounds__(256) own_step_moment_kernel(float* __restrict_
         s_hh = fmaf(h, h, s_hh);
         s_dd = fmaf(d, d, s_dd);
     };
-    // 16-byte words (all pointers are 16-byte aligned), then the tail
+    // 16-byte words (all pointers are 16-byte aligned), two per thread in
+    // flight (the words i and i + stride, in that order), then the tail
     const int64_t n4 = n >> 2;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
-        float4 m = reinterpret_cast<const float4*>(M)[i];
-        const float4 oo = __ldcs(reinterpret_cast<const float4*>(o) + i);
-        const float4 h = hv ? __ldcs(reinterpret_cast<const float4*>(hv) + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+    auto word = [&](int64_t i, float4 m, const float4& oo, const float4& h) {
         float4 mh;
         one(m.x, oo.x, h.x, mh.x);
         one(m.y, oo.y, h.y, mh.y);
@@ -363,7 +361,23 @@ __global__ void __launch_bounds__(256) own_step_moment_kernel(float* __restrict_
         one(m.w, oo.w, h.w, mh.w);
         reinterpret_cast<float4*>(M)[i] = m;
         __stcs(reinterpret_cast<float4*>(mhat) + i, mh);
+    };
+    const float4 zero4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    for (; i + stride < n4; i += 2 * stride) {
+        const int64_t j = i + stride;
+        const float4 ma = reinterpret_cast<const float4*>(M)[i];
+        const float4 mb = reinterpret_cast<const float4*>(M)[j];
+        const float4 oa = __ldcs(reinterpret_cast<const float4*>(o) + i);
+        const float4 ob = __ldcs(reinterpret_cast<const float4*>(o) + j);
+        const float4 ha = hv ? __ldcs(reinterpret_cast<const float4*>(hv) + i) : zero4;
+        const float4 hb = hv ? __ldcs(reinterpret_cast<const float4*>(hv) + j) : zero4;
+        word(i, ma, oa, ha);
+        word(j, mb, ob, hb);
     }
+    if (i < n4)
+        word(i, reinterpret_cast<const float4*>(M)[i], __ldcs(reinterpret_cast<const float4*>(o) + i),
+             hv ? __ldcs(reinterpret_cast<const float4*>(hv) + i) : zero4);
     if (blockIdx.x == 0 && threadIdx.x < (n & 3)) {
         const int64_t i = (n4 << 2) + threadIdx.x;
         float m = M[i], mh;

@@ -16,8 +16,12 @@
 // a fixed order, thread 0 advances v_b, a second sweep applies the update; the
 // second sweep's reads of g and h hit L2.
 #include "kernels.h"
+#include <type_traits>
 
 namespace bom {
+
+int device_sm_count();
+
 namespace {
 
 struct UpdCoef {
@@ -196,34 +200,71 @@ __global__ void __launch_bounds__(256) update_blockshared_kernel(float* __restri
     }
 }
 
-// Blocks of at most 8192 elements (d % 4 == 0): each thread keeps its words
-// of u and theta in registers from one read, so the block costs one memory
-// round trip before the reduction and none after it.
-constexpr int kRegWords = 8;   // float4 words per thread: 256 x 8 x 4 = 8192 elements
-template <bool G_BF16, bool HAS_H, bool SHADOW>
+// Blocks of at most 8192 elements (d % 4 == 0): each thread keeps its WPT
+// words of g (packed as loaded), h and theta in registers from one read, so
+// a block costs one memory round trip before the reduction and none after it;
+// v of the block is fetched with the data.  WPT is the smallest of 1, 2, 4, 8
+// with 1024 WPT >= block, which keeps the registers (and so the number of
+// resident CTAs, whose loads hide the latency) matched to the block.
+constexpr int kRegMaxBlock = 8192;
+template <bool G_BF16>
+struct GWord {
+    using T = typename std::conditional<G_BF16, uint2, float4>::type;
+};
+template <bool G_BF16, bool HAS_H>
+__device__ __forceinline__ void word_u(const typename GWord<G_BF16>::T& gw, const float4& hw, float lam,
+                                       float (&u)[4]) {
+    if constexpr (G_BF16) {
+        u[0] = __uint_as_float(gw.x << 16);
+        u[1] = __uint_as_float(gw.x & 0xFFFF0000u);
+        u[2] = __uint_as_float(gw.y << 16);
+        u[3] = __uint_as_float(gw.y & 0xFFFF0000u);
+    } else {
+        u[0] = gw.x; u[1] = gw.y; u[2] = gw.z; u[3] = gw.w;
+    }
+    if constexpr (HAS_H) {
+        const float hv[4] = {hw.x, hw.y, hw.z, hw.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) u[k] = (1.0f - lam) * u[k] + lam * hv[k];
+    }
+}
+
+template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT>
 __global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __restrict__ theta,
                                                                      const void* __restrict__ g,
                                                                      const float* __restrict__ h,
                                                                      float* __restrict__ vb,
                                                                      uint16_t* __restrict__ shadow, int64_t n,
                                                                      int64_t block, UpdCoef c) {
+    using GW = typename GWord<G_BF16>::T;
     __shared__ float red[8];
     __shared__ float s_den;
     const int64_t nb = (n + block - 1) / block;
     for (int64_t b = blockIdx.x; b < nb; b += gridDim.x) {
         const int64_t e0 = b * block;
         const int64_t e1 = e0 + block < n ? e0 + block : n;
-        float u[kRegWords][4];
-        float4 th[kRegWords];
-        float acc = 0.0f;
+        const float vprev = threadIdx.x == 0 ? vb[b] : 0.0f;
+        GW gw[WPT];
+        float4 hw[WPT];
+        float4 th[WPT];
 #pragma unroll
-        for (int k = 0; k < kRegWords; ++k) {
+        for (int k = 0; k < WPT; ++k) {
             const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
             if (i < e1) {
-                load_u<G_BF16, HAS_H, 4>(g, h, i, c.lam, u[k]);
+                gw[k] = *reinterpret_cast<const GW*>(static_cast<const char*>(g) + i * (G_BF16 ? 2 : 4));
+                if constexpr (HAS_H) hw[k] = *reinterpret_cast<const float4*>(h + i);
                 th[k] = __ldcs(reinterpret_cast<const float4*>(theta + i));
+            }
+        }
+        float acc = 0.0f;
 #pragma unroll
-                for (int q = 0; q < 4; ++q) acc = fmaf(u[k][q], u[k][q], acc);
+        for (int k = 0; k < WPT; ++k) {
+            const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
+            if (i < e1) {
+                float u[4];
+                word_u<G_BF16, HAS_H>(gw[k], hw[k], c.lam, u);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) acc = fmaf(u[q], u[q], acc);
             }
         }
         acc = warp_sum_f(acc);
@@ -233,21 +274,23 @@ __global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __re
             float tot = 0.0f;
 #pragma unroll
             for (int w = 0; w < 8; ++w) tot += red[w];
-            const float vv = fmaf(c.beta2, vb[b], c.one_m_beta2 * (tot / static_cast<float>(e1 - e0)));
+            const float vv = fmaf(c.beta2, vprev, c.one_m_beta2 * (tot / static_cast<float>(e1 - e0)));
             vb[b] = vv;
             s_den = sqrtf(vv * c.inv_bc2) + c.eps;
         }
         __syncthreads();
         const float den = s_den;
 #pragma unroll
-        for (int k = 0; k < kRegWords; ++k) {
+        for (int k = 0; k < WPT; ++k) {
             const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
             if (i < e1) {
+                float u[4];
+                word_u<G_BF16, HAS_H>(gw[k], hw[k], c.lam, u);
                 float4 t = th[k];
-                t.x = c.decay * t.x - c.lr * (u[k][0] / den);
-                t.y = c.decay * t.y - c.lr * (u[k][1] / den);
-                t.z = c.decay * t.z - c.lr * (u[k][2] / den);
-                t.w = c.decay * t.w - c.lr * (u[k][3] / den);
+                t.x = c.decay * t.x - c.lr * (u[0] / den);
+                t.y = c.decay * t.y - c.lr * (u[1] / den);
+                t.z = c.decay * t.z - c.lr * (u[2] / den);
+                t.w = c.decay * t.w - c.lr * (u[3] / den);
                 __stcs(reinterpret_cast<float4*>(theta + i), t);
                 if constexpr (SHADOW) {
                     uint2 sh;
@@ -261,16 +304,38 @@ __global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __re
     }
 }
 
+// Resident CTAs per SM times the SM count, at most the number of blocks.
+template <typename K>
+int resident_grid(K kernel, int64_t nb) {
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, 256, 0) != cudaSuccess || per_sm < 1)
+        per_sm = 1;
+    const int64_t grid = static_cast<int64_t>(device_sm_count()) * per_sm;
+    return static_cast<int>(grid < nb ? grid : nb);
+}
+
+template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT>
+void launch_reg(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n, int64_t block,
+                const UpdCoef& c, cudaStream_t s) {
+    auto k = update_blockshared_reg_kernel<G_BF16, HAS_H, SHADOW, WPT>;
+    k<<<resident_grid(k, (n + block - 1) / block), 256, 0, s>>>(theta, g, h, vb, shadow, n, block, c);
+}
+
+template <bool G_BF16, bool HAS_H, bool SHADOW>
+void launch_reg_wpt(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
+                    int64_t block, const UpdCoef& c, cudaStream_t s) {
+    if (block <= 1024) launch_reg<G_BF16, HAS_H, SHADOW, 1>(theta, g, h, vb, shadow, n, block, c, s);
+    else if (block <= 2048) launch_reg<G_BF16, HAS_H, SHADOW, 2>(theta, g, h, vb, shadow, n, block, c, s);
+    else if (block <= 4096) launch_reg<G_BF16, HAS_H, SHADOW, 4>(theta, g, h, vb, shadow, n, block, c, s);
+    else launch_reg<G_BF16, HAS_H, SHADOW, 8>(theta, g, h, vb, shadow, n, block, c, s);
+}
+
 template <bool G_BF16, bool HAS_H, int VEC>
 void dispatch_blockshared(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
                           int64_t block, const UpdCoef& c, int grid, cudaStream_t s) {
-    if (VEC == 4 && block <= 256 * 4 * kRegWords) {
-        if (shadow)
-            update_blockshared_reg_kernel<G_BF16, HAS_H, true><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n, block,
-                                                                                   c);
-        else
-            update_blockshared_reg_kernel<G_BF16, HAS_H, false><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n,
-                                                                                    block, c);
+    if (VEC == 4 && block <= kRegMaxBlock) {
+        if (shadow) launch_reg_wpt<G_BF16, HAS_H, true>(theta, g, h, vb, shadow, n, block, c, s);
+        else launch_reg_wpt<G_BF16, HAS_H, false>(theta, g, h, vb, shadow, n, block, c, s);
     } else if (shadow) {
         update_blockshared_kernel<G_BF16, HAS_H, true, VEC><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n, block, c);
     } else {
@@ -340,8 +405,6 @@ __global__ void sqnorm_finish_kernel(const double* __restrict__ part, int nblock
 }
 
 }  // namespace
-
-int device_sm_count();
 
 int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,
                   float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, const double* clip_sq,
