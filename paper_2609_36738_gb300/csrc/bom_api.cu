@@ -82,6 +82,8 @@ struct bom_handle {
     void* dx[2] = {nullptr, nullptr};
     void* dG = nullptr;
     void* dU = nullptr;
+    void* dG2 = nullptr;     // the second sublayer's dG, dU while its weight gradients wait
+    void* dU2 = nullptr;
     void* dx_in = nullptr;   // caller buffer for the cotangent of X (bom_set_input_grad)
     float* splitk = nullptr; // fp32 partial tiles of split-K GEMMs
     int64_t splitk_elems = 0;
@@ -210,6 +212,12 @@ size_t carve(bom_handle* h, char* base) {
     if (h->max_ffn > 0) {
         h->dG = c.take(n * h->max_ffn * e);
         h->dU = c.take(n * h->max_ffn * e);
+    }
+    // Two SwiGLU sublayers first: the second one's weight gradients wait for
+    // the first one's launch, so its dG and dU need buffers of their own.
+    if (h->bf16 && h->lw.size() >= 2 && h->lw[0].kind == BOM_LAYER_SWIGLU && h->lw[1].kind == BOM_LAYER_SWIGLU) {
+        h->dG2 = c.take(n * h->lw[1].d_out * e);
+        h->dU2 = c.take(n * h->lw[1].d_out * e);
     }
     if (h->bf16) {
         const int64_t rows = n > V ? n : V;
@@ -611,9 +619,13 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
             BOM_TRY(run_gemm(h, g, s));
         }
         // The head weight gradient contracts over the same n rows as the
-        // first sublayer's weight gradients: with a SwiGLU first layer it
-        // waits and runs in one launch with them (every operand stays live).
+        // sublayers' weight gradients: with a SwiGLU first layer it waits and
+        // runs in one launch with that layer's (every operand stays live), and
+        // so do a SwiGLU second layer's.  One work list over all of them
+        // leaves one partial wave instead of one per launch.
         GemmDesc head_dw;
+        GemmDesc pend[3];
+        int npend = 0;
         const bool defer_head = h->bf16 && kfull == 1 && !h->lw.empty() && h->lw[0].kind == BOM_LAYER_SWIGLU;
         {   // head weight: a R^T H + b qhat (x) c
             GemmDesc g = gemm1(V, dm, kfull * n, mnmaj(h->Z, h->ldz), mnmaj(xin, dm));
@@ -652,6 +664,12 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                 const void* Wg = params[p0];
                 const void* Wu = params[p0 + 1];
                 const void* Wd = params[p0 + 2];
+                // the second sublayer's weight gradients wait for the first's launch:
+                // its dy (dx[cur]) is not written again, the first layer's input
+                // gradient goes to the caller's buffer
+                const bool defer_w = defer_head && l == 1 && h->dG2 != nullptr;
+                void* const dGl = defer_w ? h->dG2 : h->dG;
+                void* const dUl = defer_w ? h->dU2 : h->dU;
                 {   // dA = dy W_d, then dG = dA u SiLU'(g), dU = dA SiLU(g)
                     GemmDesc g = gemm1(n, f, d, kmaj(dcur, d), mnmaj(Wd, f));
                     g.epi_kind = EPI_SWIGLU_BWD;
@@ -659,16 +677,16 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                     g.epi.ld_aux = f;
                     g.epi.aux2 = L.U;
                     g.epi.ld_aux2 = f;
-                    g.epi.out = h->dG;
+                    g.epi.out = dGl;
                     g.epi.ld_out = f;
-                    g.epi.out2 = h->dU;
+                    g.epi.out2 = dUl;
                     g.epi.ld_out2 = f;
                     BOM_TRY(run_gemm(h, g, s));
                 }
                 if (dx_next) {   // dx = dy + dG W_g + dU W_u
-                    GemmDesc g = gemm1(n, d, f, kmaj(h->dG, f), mnmaj(Wg, d));
+                    GemmDesc g = gemm1(n, d, f, kmaj(dGl, f), mnmaj(Wg, d));
                     g.nseg = 2;
-                    g.A[1] = kmaj(h->dU, f);
+                    g.A[1] = kmaj(dUl, f);
                     g.B[1] = mnmaj(Wu, d);
                     g.K[1] = f;
                     g.epi.resid = dcur;
@@ -684,9 +702,9 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                     BOM_TRY(run_gemm(h, g, s));
                 }
                 {   // dW_g = dG^T x, dW_u = dU^T x, dW_d = dy^T A: one launch over their tiles
-                    GemmDesc gw[4];
-                    gw[0] = gemm1(f, d, n, mnmaj(h->dG, f), mnmaj(xl, d));
-                    gw[1] = gemm1(f, d, n, mnmaj(h->dU, f), mnmaj(xl, d));
+                    GemmDesc gw[7];
+                    gw[0] = gemm1(f, d, n, mnmaj(dGl, f), mnmaj(xl, d));
+                    gw[1] = gemm1(f, d, n, mnmaj(dUl, f), mnmaj(xl, d));
                     gw[2] = gemm1(d, f, n, mnmaj(dcur, d), mnmaj(L.A, f));
                     const int pk[3] = {p0, p0 + 1, p0 + 2};
                     for (int i = 0; i < 3; ++i) {
@@ -695,9 +713,16 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                         gw[i].epi.out_f32 = of32;
                         if (fused) fuse(gw[i], pk[i]);
                     }
-                    int ng = 3;
-                    if (defer_head && l == 0) gw[ng++] = head_dw;   // the head's, deferred
-                    BOM_TRY(run_gemm_group(h, gw, ng, s));
+                    if (defer_w) {
+                        for (int i = 0; i < 3; ++i) pend[npend++] = gw[i];
+                    } else {
+                        int ng = 3;
+                        if (defer_head && l == 0) {   // the second sublayer's and the head's, deferred
+                            for (int i = 0; i < npend; ++i) gw[ng++] = pend[i];
+                            gw[ng++] = head_dw;
+                        }
+                        BOM_TRY(run_gemm_group(h, gw, ng, s));
+                    }
                 }
             } else if (L.kind == BOM_LAYER_RMSNORM) {
                 const int64_t d = L.d_in;

@@ -38,7 +38,7 @@ constexpr int NUM_THREADS = 320;  // producer warp, UMMA warp, 8 epilogue warps
 constexpr int TMEM_COLS = 512;
 constexpr int GROUP_M = 8;
 
-constexpr int kMaxGroup = 4;
+constexpr int kMaxGroup = 8;
 struct Prob {
     CUtensorMap mapA, mapB;
     int M, N, tiles_m, tiles_n;
@@ -66,6 +66,8 @@ struct Params {
     int tile_base[kMaxGroup + 1];
     Prob grp[kMaxGroup - 1];
 };
+
+static_assert(sizeof(Params) <= 32764, "kernel parameters exceed the launch limit");
 
 // Problem of `tile` (a tile index over the whole group) and its tile within it.
 struct ProbView {
