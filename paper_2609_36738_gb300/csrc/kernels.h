@@ -15,7 +15,7 @@ constexpr int kRowBlock = 128;
 inline int64_t row_blocks(int64_t n) { return (n + kRowBlock - 1) / kRowBlock; }
 
 // Row-block height of the residual pass (its column partial sums feed s_t).
-constexpr int kResidRows = 32;
+constexpr int kResidRows = 64;
 inline int64_t resid_blocks(int64_t n) { return (n + kResidRows - 1) / kResidRows; }
 
 // Counts N_t, checks every label, latches BOM_ELABEL / BOM_EEMPTY and writes

@@ -143,12 +143,31 @@ __global__ void row_lse_kernel(const void* __restrict__ Z, int z_f32, int64_t ld
     const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int l = threadIdx.x & 31;
     if (row >= n) return;
+    const int32_t y = labels[row];
     const float2* st = stats + row * ntiles;
+    // the first 256 (max, sum) pairs of the row stay in registers: one read
+    // with eight loads in flight per lane (a row of the 32000-column head has
+    // 250); pairs beyond are read again for the sum
+    constexpr int kRegPairs = 8;
+    float2 v[kRegPairs];
+#pragma unroll
+    for (int k = 0; k < kRegPairs; ++k) {
+        const int64_t t = l + 32 * k;
+        v[k] = t < ntiles ? st[t] : make_float2(-INFINITY, 0.0f);
+    }
+    float zy = 0.0f;
+    const bool has_y = y != ignore && y >= 0 && y < V;
+    if (l == 0 && has_y) zy = ld_elem(Z, row * ldz + y, z_f32);
     float m = -INFINITY;
-    for (int64_t t = l; t < ntiles; t += 32) m = fmaxf(m, st[t].x);
+#pragma unroll
+    for (int k = 0; k < kRegPairs; ++k) m = fmaxf(m, v[k].x);
+    for (int64_t t = l + 32 * kRegPairs; t < ntiles; t += 32) m = fmaxf(m, st[t].x);
     m = warp_max(m);
     float s = 0.0f;
-    for (int64_t t = l; t < ntiles; t += 32) {
+#pragma unroll
+    for (int k = 0; k < kRegPairs; ++k)
+        if (v[k].x != -INFINITY) s += v[k].y * expf(v[k].x - m);
+    for (int64_t t = l + 32 * kRegPairs; t < ntiles; t += 32) {
         const float2 p = st[t];
         if (p.x != -INFINITY) s += p.y * expf(p.x - m);
     }
@@ -156,10 +175,7 @@ __global__ void row_lse_kernel(const void* __restrict__ Z, int z_f32, int64_t ld
     if (l == 0) {
         const float L = m + logf(s);
         lse[row] = L;
-        const int32_t y = labels[row];
-        float c = 0.0f;
-        if (y != ignore && y >= 0 && y < V) c = L - ld_elem(Z, row * ldz + y, z_f32);
-        ce[row] = c;
+        ce[row] = has_y ? L - zy : 0.0f;
     }
 }
 
