@@ -677,7 +677,7 @@ def _adam_mini_only(B, torch, dev, stream, a, peaks):
     torch.cuda.empty_cache()
     return {"workload": "BOM-Adam-mini update of the LM block (7 tensors, 166,199,296 parameters), one second "
                         "moment per output neuron: read theta f32, u bf16; write theta f32, bf16 copy "
-                        "(12 B/element; the second read of u inside a block comes from L2)",
+                        "(12 B/element; each block read once into registers when it has at most 8192 elements)",
             "value": gbs, "unit": "GB/s", "ms": med, "frac_of_hbm": gbs / peaks["hbm_gbs"],
             "second_moment_entries": nblocks, "params": P,
             "state_reduction_vs_elementwise": 1.0 - nblocks / P, "peak_source": "measured copy bandwidth"}

@@ -415,12 +415,15 @@ __global__ void __launch_bounds__(256) own_step_moment_kernel(float* __restrict_
     }
 }
 
-// sums[k] += sum_b part[4b + k], in block order.
+// sums[k] += sum_b part[4b + k]: warp k, lane l adds blocks l, l + 32, ... in
+// order, then a fixed shuffle tree (the order depends only on nblocks).
 __global__ void drift_finish_kernel(const double* __restrict__ part, int nblocks, double* __restrict__ sums) {
-    if (threadIdx.x >= 4) return;
+    const int k = threadIdx.x >> 5, l = threadIdx.x & 31;
     double acc = 0.0;
-    for (int b = 0; b < nblocks; ++b) acc += part[4 * b + threadIdx.x];
-    sums[threadIdx.x] += acc;
+    for (int b = l; b < nblocks; b += 32) acc += part[4 * static_cast<int64_t>(b) + k];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (l == 0) sums[k] += acc;
 }
 
 // part[b, j] = sum_{i in row block b} w_i X[i, j] (times Y[i, j] when Y is
@@ -591,7 +594,7 @@ void launch_own_step_moment(float* M, const float* o, const float* hv, float* mh
     own_step_moment_kernel<<<nblocks, 256, 0, s>>>(M, o, hv, mhat, n, beta1, inv_bc1, sums ? part : nullptr);
     count_launch();
     if (sums) {
-        drift_finish_kernel<<<1, 32, 0, s>>>(part, nblocks, sums);
+        drift_finish_kernel<<<1, 128, 0, s>>>(part, nblocks, sums);
         count_launch();
     }
 }

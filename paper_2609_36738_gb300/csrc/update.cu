@@ -229,6 +229,92 @@ __device__ __forceinline__ void word_u(const typename GWord<G_BF16>::T& gw, cons
     }
 }
 
+// One block's words of g, h and theta (and v_b in thread 0) in registers.
+template <bool G_BF16, int WPT>
+struct RowRegs {
+    typename GWord<G_BF16>::T gw[WPT];
+    float4 hw[WPT];
+    float4 th[WPT];
+    float vprev;
+};
+
+template <bool G_BF16, bool HAS_H, int WPT>
+__device__ __forceinline__ void row_load(RowRegs<G_BF16, WPT>& r, const void* g, const float* h, const float* theta,
+                                         const float* vb, int64_t b, int64_t block, int64_t n) {
+    using GW = typename GWord<G_BF16>::T;
+    const int64_t e0 = b * block;
+    const int64_t e1 = e0 + block < n ? e0 + block : n;
+    r.vprev = threadIdx.x == 0 ? vb[b] : 0.0f;
+#pragma unroll
+    for (int k = 0; k < WPT; ++k) {
+        const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
+        if (i < e1) {
+            r.gw[k] = *reinterpret_cast<const GW*>(static_cast<const char*>(g) + i * (G_BF16 ? 2 : 4));
+            if constexpr (HAS_H) r.hw[k] = *reinterpret_cast<const float4*>(h + i);
+            r.th[k] = __ldcs(reinterpret_cast<const float4*>(theta + i));
+        }
+    }
+}
+
+// Reduction, v_b and the update of block b from its registers.
+template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT>
+__device__ __forceinline__ void row_update(const RowRegs<G_BF16, WPT>& r, float* theta, float* vb, uint16_t* shadow,
+                                           int64_t b, int64_t block, int64_t n, const UpdCoef& c, float* red,
+                                           float* s_den) {
+    const int64_t e0 = b * block;
+    const int64_t e1 = e0 + block < n ? e0 + block : n;
+    float acc = 0.0f;
+#pragma unroll
+    for (int k = 0; k < WPT; ++k) {
+        const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
+        if (i < e1) {
+            float u[4];
+            word_u<G_BF16, HAS_H>(r.gw[k], r.hw[k], c.lam, u);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) acc = fmaf(u[q], u[q], acc);
+        }
+    }
+    acc = warp_sum_f(acc);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float tot = 0.0f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) tot += red[w];
+        const float vv = fmaf(c.beta2, r.vprev, c.one_m_beta2 * (tot / static_cast<float>(e1 - e0)));
+        vb[b] = vv;
+        *s_den = sqrtf(vv * c.inv_bc2) + c.eps;
+    }
+    __syncthreads();
+    const float den = *s_den;
+#pragma unroll
+    for (int k = 0; k < WPT; ++k) {
+        const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
+        if (i < e1) {
+            float u[4];
+            word_u<G_BF16, HAS_H>(r.gw[k], r.hw[k], c.lam, u);
+            float4 t = r.th[k];
+            t.x = c.decay * t.x - c.lr * (u[0] / den);
+            t.y = c.decay * t.y - c.lr * (u[1] / den);
+            t.z = c.decay * t.z - c.lr * (u[2] / den);
+            t.w = c.decay * t.w - c.lr * (u[3] / den);
+            __stcs(reinterpret_cast<float4*>(theta + i), t);
+            if constexpr (SHADOW) {
+                uint2 sh;
+                sh.x = pack_bf16x2(t.x, t.y);
+                sh.y = pack_bf16x2(t.z, t.w);
+                __stcs(reinterpret_cast<uint2*>(shadow + i), sh);
+            }
+        }
+    }
+    __syncthreads();   // red and s_den are reused by the next block
+}
+
+// The CTA walks its blocks b, b + grid, ...  Up to 4 words per thread it
+// keeps two register sets: the loads of the next block are issued before the
+// current one is reduced and written, so the CTA keeps a block's reads in
+// flight through its barriers.  At 8 words two sets would cost more resident
+// CTAs than they gain, so those blocks go one at a time.
 template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT>
 __global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __restrict__ theta,
                                                                      const void* __restrict__ g,
@@ -236,71 +322,31 @@ __global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __re
                                                                      float* __restrict__ vb,
                                                                      uint16_t* __restrict__ shadow, int64_t n,
                                                                      int64_t block, UpdCoef c) {
-    using GW = typename GWord<G_BF16>::T;
     __shared__ float red[8];
     __shared__ float s_den;
     const int64_t nb = (n + block - 1) / block;
-    for (int64_t b = blockIdx.x; b < nb; b += gridDim.x) {
-        const int64_t e0 = b * block;
-        const int64_t e1 = e0 + block < n ? e0 + block : n;
-        const float vprev = threadIdx.x == 0 ? vb[b] : 0.0f;
-        GW gw[WPT];
-        float4 hw[WPT];
-        float4 th[WPT];
-#pragma unroll
-        for (int k = 0; k < WPT; ++k) {
-            const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
-            if (i < e1) {
-                gw[k] = *reinterpret_cast<const GW*>(static_cast<const char*>(g) + i * (G_BF16 ? 2 : 4));
-                if constexpr (HAS_H) hw[k] = *reinterpret_cast<const float4*>(h + i);
-                th[k] = __ldcs(reinterpret_cast<const float4*>(theta + i));
-            }
+    const int64_t G = gridDim.x;
+    int64_t b = blockIdx.x;
+    if (b >= nb) return;
+    if constexpr (WPT > 4) {
+        RowRegs<G_BF16, WPT> r;
+        for (; b < nb; b += G) {
+            row_load<G_BF16, HAS_H, WPT>(r, g, h, theta, vb, b, block, n);
+            row_update<G_BF16, HAS_H, SHADOW, WPT>(r, theta, vb, shadow, b, block, n, c, red, &s_den);
         }
-        float acc = 0.0f;
-#pragma unroll
-        for (int k = 0; k < WPT; ++k) {
-            const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
-            if (i < e1) {
-                float u[4];
-                word_u<G_BF16, HAS_H>(gw[k], hw[k], c.lam, u);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) acc = fmaf(u[q], u[q], acc);
-            }
-        }
-        acc = warp_sum_f(acc);
-        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            float tot = 0.0f;
-#pragma unroll
-            for (int w = 0; w < 8; ++w) tot += red[w];
-            const float vv = fmaf(c.beta2, vprev, c.one_m_beta2 * (tot / static_cast<float>(e1 - e0)));
-            vb[b] = vv;
-            s_den = sqrtf(vv * c.inv_bc2) + c.eps;
-        }
-        __syncthreads();
-        const float den = s_den;
-#pragma unroll
-        for (int k = 0; k < WPT; ++k) {
-            const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
-            if (i < e1) {
-                float u[4];
-                word_u<G_BF16, HAS_H>(gw[k], hw[k], c.lam, u);
-                float4 t = th[k];
-                t.x = c.decay * t.x - c.lr * (u[0] / den);
-                t.y = c.decay * t.y - c.lr * (u[1] / den);
-                t.z = c.decay * t.z - c.lr * (u[2] / den);
-                t.w = c.decay * t.w - c.lr * (u[3] / den);
-                __stcs(reinterpret_cast<float4*>(theta + i), t);
-                if constexpr (SHADOW) {
-                    uint2 sh;
-                    sh.x = pack_bf16x2(t.x, t.y);
-                    sh.y = pack_bf16x2(t.z, t.w);
-                    __stcs(reinterpret_cast<uint2*>(shadow + i), sh);
-                }
-            }
-        }
-        __syncthreads();   // red and s_den are reused by the next block
+        return;
+    }
+    RowRegs<G_BF16, WPT> ra, rb;
+    row_load<G_BF16, HAS_H, WPT>(ra, g, h, theta, vb, b, block, n);
+    for (;;) {
+        if (b + G < nb) row_load<G_BF16, HAS_H, WPT>(rb, g, h, theta, vb, b + G, block, n);
+        row_update<G_BF16, HAS_H, SHADOW, WPT>(ra, theta, vb, shadow, b, block, n, c, red, &s_den);
+        b += G;
+        if (b >= nb) break;
+        if (b + G < nb) row_load<G_BF16, HAS_H, WPT>(ra, g, h, theta, vb, b + G, block, n);
+        row_update<G_BF16, HAS_H, SHADOW, WPT>(rb, theta, vb, shadow, b, block, n, c, red, &s_den);
+        b += G;
+        if (b >= nb) break;
     }
 }
 
@@ -397,11 +443,15 @@ __global__ void __launch_bounds__(256) sqnorm_part_kernel(const void* __restrict
     }
 }
 
+// *sq += sum_b part[b]: lane l adds blocks l, l + 32, ... in order, then a
+// fixed shuffle tree (the order depends only on nblocks: deterministic).
 __global__ void sqnorm_finish_kernel(const double* __restrict__ part, int nblocks, double* __restrict__ sq) {
-    if (threadIdx.x != 0) return;
+    const int l = threadIdx.x & 31;
     double t = 0.0;
-    for (int b = 0; b < nblocks; ++b) t += part[b];
-    *sq += t;
+    for (int b = l; b < nblocks; b += 32) t += part[b];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (threadIdx.x == 0) *sq += t;
 }
 
 }  // namespace
