@@ -50,7 +50,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 def _args():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--steps", type=int, default=50)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="lm_mlp_bf16")
@@ -80,13 +80,16 @@ def _workload_desc(wl):
 
 # --------------------------------------------------------------------- clocks
 class ClockSampler:
-    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.hw_slowdown",
+    """nvidia-smi samples every 50 ms; only the samples taken between mark_start()
+    and mark_end() (the timed steps) enter the summary."""
+    FIELDS = ["timestamp", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.hw_slowdown",
               "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
               "clocks_event_reasons.sw_power_cap"]
 
     def __init__(self, gpu_id):
         self.gpu_id = gpu_id
         self.proc = None
+        self.t0 = self.t1 = None
         self.path = os.path.join("/tmp", f"bom_clocks_{os.getpid()}.csv")
 
     def start(self):
@@ -94,9 +97,15 @@ class ClockSampler:
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--query-gpu={','.join(self.FIELDS)}", "--format=csv,noheader,nounits",
-                 "-i", str(self.gpu_id), "-lms", "200"], stdout=self.fh, stderr=subprocess.DEVNULL)
+                 "-i", str(self.gpu_id), "-lms", "50"], stdout=self.fh, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
+
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
 
     def stop(self):
         if self.proc is None:
@@ -107,23 +116,33 @@ class ClockSampler:
         except Exception:
             self.proc.kill()
         self.fh.close()
-        sm, mx, reasons = [], [], set()
+        import datetime
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        rows = []
         for line in open(self.path):
             parts = [x.strip() for x in line.split(",")]
-            if len(parts) < 7:
+            if len(parts) < 8:
                 continue
             try:
-                sm.append(float(parts[0]))
-                mx.append(float(parts[1]))
+                ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                rows.append((ts, float(parts[1]), float(parts[2]), float(parts[3]), parts[4:8]))
             except ValueError:
                 continue
-            for nm, v in zip(names, parts[3:7]):
+        os.remove(self.path)
+        inside = [r for r in rows if self.t0 is not None and self.t1 is not None and self.t0 <= r[0] <= self.t1]
+        use = inside if inside else rows
+        reasons = set()
+        for r in use:
+            for nm, v in zip(names, r[4]):
                 if v.lower().startswith("active"):
                     reasons.add(nm)
-        os.remove(self.path)
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": sorted(reasons), "samples": len(sm)}
+        sm = [r[1] for r in use]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(r[2] for r in use) if use else None,
+                "sm_mhz_min": min(sm) if sm else None,
+                "power_w_median": statistics.median([r[3] for r in use]) if use else None,
+                "reasons": sorted(reasons), "samples": len(sm),
+                "window": "timed steps only" if inside else "whole sampler run (no sample inside the timed steps)"}
 
 
 # --------------------------------------------------------------------- CPU oracle legs
@@ -170,7 +189,8 @@ def run_reference(a):
         return
     wl = I.WORKLOADS[a.workload]
     cores = os.cpu_count()
-    _, desc, n = oracle_sample(wl, budget_s=8.0)
+    # rows per step sized so that warm-up and timed steps together take about 1-2 minutes
+    _, desc, n = oracle_sample(wl, budget_s=min(8.0, 200.0 / max(1, a.steps + a.warmup)))
     for _ in range(a.warmup):
         oracle_sample(wl, n_rows=n)
     vals = []
@@ -290,6 +310,7 @@ def main():
     torch.cuda.synchronize()
     clocks.start()
     time.sleep(0.3)
+    clocks.mark_start()
     for i in range(a.steps):
         flush.zero_()
         t += 1
@@ -303,6 +324,7 @@ def main():
             d[2] += ms
             d[3] += 1
     torch.cuda.synchronize()
+    clocks.mark_end()
     clk = clocks.stop()
     launches = B.bom_launch_count() - launches0
     B.bom_trace(model.h, False)

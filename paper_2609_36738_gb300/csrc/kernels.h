@@ -7,10 +7,14 @@
 
 namespace bom {
 
-// Row-block height of the residual pass and of the column reductions.  The
-// column partial sums of one block are summed in a fixed order afterwards, so
-// every reduction of the step is deterministic (no float atomics).
+// Row-block height that sizes the partial-sum buffers of the column
+// reductions (they use row ranges of at least this many rows).  The column
+// partial sums of one block are summed in a fixed order afterwards, so every
+// reduction of the step is deterministic (no float atomics).
 constexpr int kRowBlock = 128;
+
+// Streaming multiprocessors of the current device (cached on first use).
+int device_sm_count();
 
 inline int64_t row_blocks(int64_t n) { return (n + kRowBlock - 1) / kRowBlock; }
 

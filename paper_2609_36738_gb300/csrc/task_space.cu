@@ -426,73 +426,94 @@ __global__ void drift_finish_kernel(const double* __restrict__ part, int nblocks
     if (l == 0) sums[k] += acc;
 }
 
-// part[b, j] = sum_{i in row block b} w_i X[i, j] (times Y[i, j] when Y is
-// given, same layout as X).  A block covers 32 x VEC columns of one row
-// block: every warp reads 16-byte words of the same columns, the 8 warps take
-// interleaved rows, and the 8 warp sums are added in a fixed order in shared
-// memory (deterministic).
+// part[b, j] = sum_{i in row range b} w_i X[i, j] (times Y[i, j] when Y is
+// given, same layout as X); row range b is [b * rows_per, (b + 1) * rows_per).
+// A block covers 32 x VEC columns of one row range: every warp reads 16-byte
+// words of the same columns, the 8 warps take interleaved rows, and the 8 warp
+// sums are added in a fixed order in shared memory (deterministic).  The host
+// sizes the ranges so that the whole grid is one resident wave and each block
+// streams many rows (colsum_rows_per).
+template <typename T>
+__device__ __forceinline__ float word_elem(const uint4& w, int k) {
+    const uint32_t v = (k >> (sizeof(T) == 2 ? 1 : 0)) == 0   ? w.x
+                       : (k >> (sizeof(T) == 2 ? 1 : 0)) == 1 ? w.y
+                       : (k >> (sizeof(T) == 2 ? 1 : 0)) == 2 ? w.z
+                                                              : w.w;
+    if constexpr (sizeof(T) == 2)
+        return __uint_as_float((k & 1) ? (v & 0xFFFF0000u) : (v << 16));
+    else
+        return __uint_as_float(v);
+}
+
 template <typename T, bool HAS_Y>
-__global__ void __launch_bounds__(256, 2) colsum_part_kernel(const T* __restrict__ X, const T* __restrict__ Y,
-                                                             int64_t ldx, int64_t n,
+__global__ void __launch_bounds__(256, 3) colsum_part_kernel(const T* __restrict__ X, const T* __restrict__ Y,
+                                                             int64_t ldx, int64_t n, int64_t rows_per,
                                                              int64_t d, const int32_t* __restrict__ labels,
                                                              int32_t ignore, const float* __restrict__ wvec,
                                                              float* __restrict__ part, const DevScalars* sc) {
     constexpr int VEC = 16 / sizeof(T);
+    // rows in flight per warp step: 8 words per thread (4 of X and 4 of Y)
+    constexpr int U = HAS_Y ? 4 : 8;
     __shared__ float red[8][32 * VEC];
     if (sc->status != 0) return;
     const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
     const int64_t c0 = static_cast<int64_t>(blockIdx.x) * (32 * VEC) + l * VEC;
-    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kRowBlock;
-    const int64_t r1 = min(r0 + kRowBlock, n);
+    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * rows_per;
+    const int64_t r1 = min(r0 + rows_per, n);
     float acc[VEC];
 #pragma unroll
     for (int k = 0; k < VEC; ++k) acc[k] = 0.0f;
-    const bool vec = (c0 + VEC <= d) && ((ldx % VEC) == 0);
-    constexpr int UNROLL = 8;
-    auto load_word = [&](const T* src) {
-        if (vec) return *reinterpret_cast<const uint4*>(src);
-        uint32_t q[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-        for (int k = 0; k < VEC; ++k) {
-            if (c0 + k >= d) continue;
-            if constexpr (sizeof(T) == 2)
-                q[k >> 1] |= static_cast<uint32_t>(reinterpret_cast<const uint16_t*>(src)[k]) << (16 * (k & 1));
-            else
-                q[k] = reinterpret_cast<const uint32_t*>(src)[k];
-        }
-        return make_uint4(q[0], q[1], q[2], q[3]);
+    auto weight = [&](int64_t r) {
+        if (labels) return labels[r] != ignore ? 1.0f : 0.0f;
+        return wvec ? wvec[r] : 1.0f;
     };
-    auto elem = [](const uint4& w, int k) {
-        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-        if constexpr (sizeof(T) == 2)
-            return __uint_as_float((k & 1) ? (ws[k >> 1] & 0xFFFF0000u) : (ws[k >> 1] << 16));
-        else
-            return __uint_as_float(ws[k]);
-    };
-    for (int64_t rb = r0 + w; rb < r1; rb += 8 * UNROLL) {
-        uint4 raw[UNROLL], raw2[HAS_Y ? UNROLL : 1];
-        float wt[UNROLL];
+    if (c0 + VEC <= d && (ldx % VEC) == 0) {
+        const T* px = X + c0;
+        const T* py = HAS_Y ? Y + c0 : nullptr;
+        int64_t r = r0 + w;
+        for (; r + 8 * (U - 1) < r1; r += 8 * U) {
+            uint4 a[U], b[HAS_Y ? U : 1];
+            float wt[U];
 #pragma unroll
-        for (int u = 0; u < UNROLL; ++u) {
-            const int64_t r = rb + 8 * u;
-            wt[u] = 0.0f;
-            raw[u] = make_uint4(0u, 0u, 0u, 0u);
-            if constexpr (HAS_Y) raw2[u] = make_uint4(0u, 0u, 0u, 0u);
-            if (r >= r1 || c0 >= d) continue;
-            float wr = 1.0f;
-            if (labels) wr = (labels[r] != ignore) ? 1.0f : 0.0f;
-            if (wvec) wr = wvec[r];
-            wt[u] = wr;
-            raw[u] = load_word(X + r * ldx + c0);
-            if constexpr (HAS_Y) raw2[u] = load_word(Y + r * ldx + c0);
+            for (int u = 0; u < U; ++u) {
+                const int64_t off = (r + 8 * u) * ldx;
+                a[u] = __ldcs(reinterpret_cast<const uint4*>(px + off));
+                if constexpr (HAS_Y) b[u] = __ldcs(reinterpret_cast<const uint4*>(py + off));
+                wt[u] = weight(r + 8 * u);
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) {
+                    float x = word_elem<T>(a[u], k);
+                    if constexpr (HAS_Y) x *= word_elem<T>(b[u], k);
+                    acc[k] = fmaf(wt[u], x, acc[k]);
+                }
+            }
         }
-#pragma unroll
-        for (int u = 0; u < UNROLL; ++u) {
+        for (; r < r1; r += 8) {
+            const int64_t off = r * ldx;
+            const uint4 a = __ldcs(reinterpret_cast<const uint4*>(px + off));
+            uint4 b = a;
+            if constexpr (HAS_Y) b = __ldcs(reinterpret_cast<const uint4*>(py + off));
+            const float wr = weight(r);
 #pragma unroll
             for (int k = 0; k < VEC; ++k) {
-                float x = elem(raw[u], k);
-                if constexpr (HAS_Y) x *= elem(raw2[u], k);
-                acc[k] = fmaf(wt[u], x, acc[k]);
+                float x = word_elem<T>(a, k);
+                if constexpr (HAS_Y) x *= word_elem<T>(b, k);
+                acc[k] = fmaf(wr, x, acc[k]);
+            }
+        }
+    } else if (c0 < d) {
+        // ragged last column group or a pitch that breaks 16-byte alignment
+        for (int64_t r = r0 + w; r < r1; r += 8) {
+            const float wr = weight(r);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) {
+                if (c0 + k >= d) break;
+                float x = static_cast<float>(X[r * ldx + c0 + k]);
+                if constexpr (HAS_Y) x *= static_cast<float>(Y[r * ldx + c0 + k]);
+                acc[k] = fmaf(wr, x, acc[k]);
             }
         }
     }
@@ -599,6 +620,18 @@ void launch_own_step_moment(float* M, const float* o, const float* hv, float* mh
     }
 }
 
+// Rows per block of the column reduction: the fewest row ranges that still
+// give every SM three blocks (one resident wave), and never more ranges than
+// row_blocks(n), which is what callers size the partial buffer for.  Whole
+// multiples of 64 rows keep the 8 warps' 8-row unrolled steps full.
+static int64_t colsum_rows_per(int64_t n, int64_t col_groups, int sms) {
+    const int64_t want = std::max<int64_t>(1, (3 * static_cast<int64_t>(sms > 0 ? sms : 1)) / std::max<int64_t>(col_groups, 1));
+    const int64_t ranges = std::min<int64_t>(row_blocks(n), want);
+    int64_t per = (n + ranges - 1) / ranges;
+    per = (per + 63) / 64 * 64;
+    return std::max<int64_t>(per, kRowBlock);
+}
+
 void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, const int32_t* labels,
                    int32_t ignore, const float* wvec, float scale, float* part, void* out, int out_f32,
                    const DevScalars* sc, cudaStream_t s) {
@@ -608,23 +641,28 @@ void launch_colsum(const void* X, int x_f32, int64_t ldx, int64_t n, int64_t d, 
 void launch_colsum2(const void* X, const void* Y, int x_f32, int64_t ldx, int64_t n, int64_t d,
                     const int32_t* labels, int32_t ignore, const float* wvec, float scale, float* part, void* out,
                     int out_f32, const DevScalars* sc, cudaStream_t s) {
-    const int64_t nb = row_blocks(n);
+    const int64_t cols_per_block = x_f32 ? 128 : 256;
+    const int64_t rows_per = colsum_rows_per(n, cdiv(d, cols_per_block), device_sm_count());
+    const int64_t nb = (n + rows_per - 1) / rows_per;
+    dim3 grid(cdiv(d, cols_per_block), static_cast<unsigned>(nb));
     if (x_f32) {
-        dim3 grid(cdiv(d, 128), static_cast<unsigned>(nb));
         auto x = static_cast<const float*>(X);
         auto y = static_cast<const float*>(Y);
-        if (Y) colsum_part_kernel<float, true><<<grid, 256, 0, s>>>(x, y, ldx, n, d, labels, ignore, wvec, part, sc);
-        else colsum_part_kernel<float, false><<<grid, 256, 0, s>>>(x, y, ldx, n, d, labels, ignore, wvec, part, sc);
+        if (Y)
+            colsum_part_kernel<float, true><<<grid, 256, 0, s>>>(x, y, ldx, n, rows_per, d, labels, ignore, wvec,
+                                                                 part, sc);
+        else
+            colsum_part_kernel<float, false><<<grid, 256, 0, s>>>(x, y, ldx, n, rows_per, d, labels, ignore, wvec,
+                                                                  part, sc);
     } else {
-        dim3 grid(cdiv(d, 256), static_cast<unsigned>(nb));
         auto x = static_cast<const __nv_bfloat16*>(X);
         auto y = static_cast<const __nv_bfloat16*>(Y);
         if (Y)
-            colsum_part_kernel<__nv_bfloat16, true><<<grid, 256, 0, s>>>(x, y, ldx, n, d, labels, ignore, wvec,
-                                                                         part, sc);
+            colsum_part_kernel<__nv_bfloat16, true><<<grid, 256, 0, s>>>(x, y, ldx, n, rows_per, d, labels, ignore,
+                                                                         wvec, part, sc);
         else
-            colsum_part_kernel<__nv_bfloat16, false><<<grid, 256, 0, s>>>(x, y, ldx, n, d, labels, ignore, wvec,
-                                                                          part, sc);
+            colsum_part_kernel<__nv_bfloat16, false><<<grid, 256, 0, s>>>(x, y, ldx, n, rows_per, d, labels, ignore,
+                                                                          wvec, part, sc);
     }
     count_launch();
     colsum_finish_kernel<<<cdiv(d, 32), 256, 0, s>>>(part, nb, d, scale, out, out_f32, sc); count_launch();
