@@ -75,6 +75,10 @@ def _workload_desc(wl):
     if wl.name == "lm_mlp_bf16":
         return ("LM output block + 2 SwiGLU MLP sublayers: 16384 tokens, d=2048, ffn=8192, vocab 32000, "
                 "full BOM backward and BOM-AdamW update over 166,199,296 params")
+    if wl.name == "tiny_mlp_f32":
+        return "tiny MLP classifier, fp32: 64 -> 128 (GELU) -> 10 classes, batch 32"
+    if wl.name == "vision_head_bf16":
+        return "vision-style classifier head, bf16: 768 -> 3072 -> 768 (GELU) -> 1000 classes, batch 256"
     return wl.name
 
 
@@ -395,6 +399,7 @@ def main():
         extra["update_clipped_lm_block"] = _clipped_update(B, torch, dev, stream, a, peaks)
         extra["telemetry_step_lm_block"] = _telemetry_step(B, torch, dev, stream, a, peaks)
         extra["rmsnorm_lm_block"] = _rmsnorm_step(B, torch, dev, stream, a, peaks)
+        extra["small_steps_graph"] = _small_steps(B, torch, dev, stream, a)
 
     cpu = None
     if rank == 0 and world == 1 and not a.no_cpu:
@@ -508,6 +513,65 @@ def _update_only(B, torch, dev, stream, a, peaks):
     return {"workload": "update sweep, 1e9 elements: read theta f32, g bf16, h f32, v f32; write theta, v "
                         "(22 B/element)", "value": gbs, "unit": "GB/s", "ms": med,
             "frac_of_hbm": gbs / peaks["hbm_gbs"], "peak_source": "measured copy bandwidth"}
+
+
+def _small_steps(B, torch, dev, stream, a):
+    """The two small configurations (tiny fp32 MLP classifier, batch 32; vision
+    head, 3-layer bf16 MLP at batch 256, 1000 classes), BOM step with the fused
+    update: launched kernel by kernel, and as one captured step (CUDA graph)
+    that reads t and lr from the device.  Steps run back to back (a few MB,
+    L2-resident), so the time includes what launching costs."""
+    out = {}
+    for wl in (I.TINY_MLP_F32, I.VISION_HEAD_BF16):
+        bf16 = wl.dtype == "bf16"
+        res = {}
+        for mode in ("launches", "graph"):
+            params_np = I.init_params(wl, 0)
+            if bf16:
+                params = [torch.from_numpy(p.view(np.int16)).to(dev).view(torch.bfloat16) for p in params_np]
+                theta = [torch.from_numpy(I.bf16_to_f32(p)).to(dev) for p in params_np]
+            else:
+                params = [torch.from_numpy(p.copy()).to(dev) for p in params_np]
+                theta = [torch.from_numpy(p.copy()).to(dev) for p in params_np]
+            v = [torch.zeros(p.shape, dtype=torch.float32, device=dev) for p in params_np]
+            x_np, y_np = I.make_batch(wl, 0, 1)
+            x = (torch.from_numpy(x_np.view(np.int16)).to(dev).view(torch.bfloat16) if bf16
+                 else torch.from_numpy(x_np).to(dev))
+            y = torch.from_numpy(y_np).to(dev)
+            q = torch.zeros(wl.vocab, dtype=torch.float32, device=dev)
+            m = B.BomModel(B.config_for(wl, LAM, B1))
+            B.bom_set_fused_update(m.h, theta, v, I.weight_decay_mask(wl, WD), LR, B2, EPS)
+            g = None
+            if mode == "graph":
+                t_dev = torch.ones(1, dtype=torch.int64, device=dev)
+                B.bom_set_step_scalars(m.h, t_dev, None)
+                g = B.bom_graph_capture(m.h, x, y, wl.n_rows, params, q, None, None)
+                run = lambda t: B.bom_graph_launch(g, stream)
+            else:
+                run = lambda t: m.step(x, y, wl.n_rows, params, q, t, None, None, stream)
+            for t in range(1, a.warmup + 1):
+                run(t)
+            m.stats(stream)
+            K = 200
+            n0 = B.bom_launch_count()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for t in range(a.warmup + 1, a.warmup + 1 + K):
+                run(t)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1) / K
+            kpl = (B.bom_launch_count() - n0) / K
+            m.stats(stream)
+            res[mode] = {"value": wl.n_rows / (ms / 1e3), "unit": "tokens/s", "us_per_step": 1e3 * ms,
+                         "kernels_per_step": kpl}
+            if g is not None:
+                B.bom_graph_destroy(g)
+            m.close()
+        res["workload"] = _workload_desc(wl)
+        res["graph_speedup"] = res["launches"]["us_per_step"] / res["graph"]["us_per_step"]
+        out[wl.name] = res
+    return out
 
 
 def _lm_state(B, torch, dev, wl, seed=0):

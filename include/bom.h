@@ -136,7 +136,8 @@ int64_t bom_workspace_bytes(const bom_config* cfg);
  *   params  bom_param_count device pointers (compute dtype), read only.
  *   q       [d_out] fp32, in/out: q_{t-1} on entry, q_t on exit (unchanged if
  *           the device latches an error).
- *   t       1-based step index (t >= 1) used by the bias correction.
+ *   t       1-based step index (t >= 1) used by the bias correction; ignored
+ *           when a device step counter is registered (bom_set_step_scalars).
  *   grads   bom_param_count output pointers (compute dtype): u, or g in
  *           BOM_OUT_G_AND_H mode.
  *   h_out   BOM_OUT_G_AND_H only: bom_param_count fp32 outputs receiving h;
@@ -166,6 +167,47 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
  * again before each step (host-side only).  theta = NULL disables it. */
 bom_status bom_set_fused_update(bom_handle* h, float* const* theta, float* const* v, const float* wd, float lr,
                                 float beta2, float eps);
+
+/* Step scalars on the device, so that one captured step can be replayed for
+ * every later step (Algorithm 1 with its bias corrections 1/(1-beta1^t) of q
+ * (Section 3.2) and 1/(1-beta2^t) of v (Section 3.4)).
+ *   t_dev   int64 device counter (8-byte aligned) holding the index t >= 1 of
+ *           the next step.  Every following bom_step reads t there instead of
+ *           its t argument (which is then ignored), and increments *t_dev at
+ *           its end when it latched no device error, so a failed step leaves
+ *           t, like q, unchanged.  A counter below 1 latches BOM_EINVAL.
+ *   lr_dev  fp32 device learning rate (4-byte aligned) that the fused update
+ *           reads instead of the lr given to bom_set_fused_update, or NULL.
+ * The bias corrections computed from *t_dev equal the ones the host forms
+ * from the same t (bit for bit), so replayed and directly launched steps give
+ * identical results.  Other entry points (bom_update, ...) still take t and
+ * lr from the host.  t_dev = NULL and lr_dev = NULL return to host scalars.
+ * Returns BOM_ENOTSUP for a misaligned pointer. */
+bom_status bom_set_step_scalars(bom_handle* h, int64_t* t_dev, const float* lr_dev);
+
+typedef struct bom_graph bom_graph;
+
+/* Captures one bom_step with these arguments (as bom_step, without t) into an
+ * executable CUDA graph, for the small, launch-bound configurations where
+ * per-kernel launch cost is a large share of the step.  The graph refers to
+ * the given buffers and to the handle's workspace: they must stay allocated,
+ * and their contents are read and written at each launch, not at capture.
+ * Requires device step scalars (bom_set_step_scalars; BOM_EINVAL otherwise),
+ * so each launch runs the step *t_dev and advances the counter.  The settings
+ * registered on the handle at capture time (fused update, input gradient,
+ * own-step output) are part of the graph; tracing must be off.  The capture
+ * runs on a private stream and executes nothing; the handle's first use of a
+ * GEMM shape may happen inside it.  Steps of one handle, launched directly or
+ * as graphs, must be ordered on one stream. */
+bom_status bom_graph_capture(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                             void* const* params, float* q, void* const* grads, void* const* h_out,
+                             bom_graph** out);
+
+/* Launches a captured step on `stream` (asynchronous). */
+bom_status bom_graph_launch(bom_graph* g, void* stream);
+
+/* Frees a captured step (NULL is a no-op). */
+void bom_graph_destroy(bom_graph* g);
 
 /* Registers a device buffer dx [max_rows, d_in] (compute dtype) that every
  * following bom_step fills with the cotangent of the input X (the u, or in
@@ -288,7 +330,9 @@ bom_status bom_trace(bom_handle* h, int32_t enable);
  * (or -1 on error). */
 int32_t bom_trace_read(bom_handle* h, bom_trace_entry* out, int32_t max, void* stream);
 
-/* Number of kernels this library has launched in the process so far. */
+/* Number of kernels this library has launched in the process so far (a
+ * captured step counts its kernels each time it is launched, not when it is
+ * captured). */
 int64_t bom_launch_count(void);
 
 /* Allocation-free weighted column sum (the paper has no counterpart; this is

@@ -30,7 +30,8 @@ EXPORTED = ("bom_param_count", "bom_param_shape", "bom_init", "bom_workspace_byt
             "bom_set_input_grad", "bom_step_outputs", "bom_get_stats", "bom_update", "bom_gemm_bf16", "bom_trace", "bom_trace_read",
             "bom_launch_count", "bom_colsum_noalloc", "bom_set_own_step_output", "bom_own_step_moment",
             "bom_stats_transfer_bytes", "bom_update_blockshared", "bom_sqnorm", "bom_update_clipped",
-            "bom_set_fused_update", "bom_destroy", "bom_status_string")
+            "bom_set_fused_update", "bom_set_step_scalars", "bom_graph_capture", "bom_graph_launch",
+            "bom_graph_destroy", "bom_destroy", "bom_status_string")
 
 
 class bom_trace_entry(C.Structure):
@@ -113,6 +114,15 @@ def lib() -> C.CDLL:
     L.bom_update_clipped.restype = i32
     L.bom_set_fused_update.argtypes = [vp, C.POINTER(vp), C.POINTER(vp), C.POINTER(f32), f32, f32, f32]
     L.bom_set_fused_update.restype = i32
+    L.bom_set_step_scalars.argtypes = [vp, vp, vp]
+    L.bom_set_step_scalars.restype = i32
+    L.bom_graph_capture.argtypes = [vp, vp, vp, i64, C.POINTER(vp), vp, C.POINTER(vp), C.POINTER(vp),
+                                    C.POINTER(vp)]
+    L.bom_graph_capture.restype = i32
+    L.bom_graph_launch.argtypes = [vp, vp]
+    L.bom_graph_launch.restype = i32
+    L.bom_graph_destroy.argtypes = [vp]
+    L.bom_graph_destroy.restype = None
     L.bom_destroy.argtypes = [vp]
     L.bom_destroy.restype = None
     L.bom_status_string.argtypes = [i32]
@@ -204,6 +214,32 @@ def bom_step(h, x, labels, n_rows: int, params, q, t: int, grads, h_out=None, st
     H = (C.c_void_p * n)(*[_ptr(p) for p in h_out]) if h_out is not None else None
     _check(lib().bom_step(h, _ptr(x), _ptr(labels), int(n_rows), P, _ptr(q), int(t), G,
                           H if H is not None else None, _stream(stream)), "bom_step")
+
+
+def bom_set_step_scalars(h, t_dev, lr_dev=None) -> None:
+    """Registers the device step counter (int64) and, optionally, the device
+    learning rate (fp32) that bom_step reads instead of its host values."""
+    _check(lib().bom_set_step_scalars(h, _ptr(t_dev), _ptr(lr_dev)), "bom_set_step_scalars")
+
+
+def bom_graph_capture(h, x, labels, n_rows: int, params, q, grads, h_out=None) -> C.c_void_p:
+    n = len(params)
+    P = (C.c_void_p * n)(*[_ptr(p) for p in params])
+    G = (C.c_void_p * n)(*[_ptr(g) for g in grads]) if grads is not None else None
+    H = (C.c_void_p * n)(*[_ptr(p) for p in h_out]) if h_out is not None else None
+    g = C.c_void_p()
+    _check(lib().bom_graph_capture(h, _ptr(x), _ptr(labels), int(n_rows), P, _ptr(q), G, H, C.byref(g)),
+           "bom_graph_capture")
+    return g
+
+
+def bom_graph_launch(g, stream=None) -> None:
+    _check(lib().bom_graph_launch(g, _stream(stream)), "bom_graph_launch")
+
+
+def bom_graph_destroy(g) -> None:
+    if g:
+        lib().bom_graph_destroy(g)
 
 
 def bom_set_input_grad(h, dx) -> None:

@@ -77,6 +77,9 @@ struct bom_handle {
     std::vector<float*> upd_theta, upd_v;
     std::vector<float> upd_wd;
     float upd_lr = 0.0f, upd_beta2 = 0.0f, upd_eps = 0.0f;
+    // device step scalars (bom_set_step_scalars): t and lr read by the step's kernels
+    int64_t* t_dev = nullptr;
+    const float* lr_dev = nullptr;
     float* ubuf = nullptr;   // fp32 u of a vector tensor (bias, norm weight) before its update
     float* part = nullptr;
     void* dx[2] = {nullptr, nullptr};
@@ -428,7 +431,7 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                     int64_t t, void* const* grads, void* const* h_out, void* stream) {
     const bool fused = h != nullptr && h->fused_upd;
     if (!h || !x || !labels || !params || !q || (!grads && !fused)) return BOM_EINVAL;
-    if (n < 1 || n > h->cfg.max_rows || t < 1) return BOM_EINVAL;
+    if (n < 1 || n > h->cfg.max_rows || (t < 1 && h->t_dev == nullptr)) return BOM_EINVAL;
     const bool gh = h->cfg.out_mode == BOM_OUT_G_AND_H;
     if (gh != (h_out != nullptr)) return BOM_EINVAL;
     // the fused update consumes u: one u pass and nothing else that needs it
@@ -455,7 +458,17 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
     } while (0)
 
     if (cudaMemsetAsync(&h->sc->status, 0, sizeof(int32_t), s) != cudaSuccess) return BOM_ECUDA;
-    BOM_TRACED("labels_scan", 0, 4.0 * n, launch_labels_scan(labels, n, V, cfg.ignore_index, cfg.lambda, h->sc, s));
+    // step scalars: from the host t and lr, or from the device step counter
+    StepScalarsIn st{};
+    st.lr = fused ? h->upd_lr : 0.0f;
+    st.inv_bc1 = h->t_dev ? 0.0f : inv_bias_correction(cfg.beta1, t);
+    st.inv_bc2 = (fused && !h->t_dev) ? inv_bias_correction(h->upd_beta2, t) : 0.0f;
+    st.t_dev = h->t_dev;
+    st.lr_dev = h->lr_dev;
+    st.beta1 = cfg.beta1;
+    st.beta2 = fused ? h->upd_beta2 : 0.0f;
+    BOM_TRACED("labels_scan", 0, 4.0 * n,
+               launch_labels_scan(labels, n, V, cfg.ignore_index, cfg.lambda, st, h->sc, s));
 
     // ---------------------------------------------------------------- forward
     const void* xin = x;
@@ -535,9 +548,8 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
     // residual pass: reads and rewrites Z once, writes the column partial sums
     BOM_TRACED("residual", 0, 2.0 * h->esz * n * h->ldz + 4.0 * resid_blocks(n) * V + 8.0 * n,
                launch_residual(h->Z, cf32, h->ldz, n, V, h->lse, labels, cfg.ignore_index, h->colpart, h->sc, s));
-    const float inv_bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(cfg.beta1), static_cast<double>(t))));
     BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 20.0 * V,
-               launch_finish_sq(h->colpart, resid_blocks(n), V, cfg.beta1, inv_bc1, q, h->s, h->qhat, h->sc, s));
+               launch_finish_sq(h->colpart, resid_blocks(n), V, cfg.beta1, q, h->s, h->qhat, h->sc, s));
     const bool own = !h->own_out.empty();
     if (own)   // per-row residual norms for the cancellation ratio
         BOM_TRACED("row_norm", 2.0 * n * V, h->esz * n * h->ldz + 4.0 * n,
@@ -562,19 +574,15 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
     passes[npass++] = gh ? 1 : 0;
     if (gh) passes[npass++] = 2;
     if (own) passes[npass++] = 3;
-    const float inv_bc2 = fused ? static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(h->upd_beta2),
-                                                                           static_cast<double>(t))))
-                                : 0.0f;
+    // the fused update takes lr and 1/(1 - beta2^t) from the step scalars
     // the GEMM producing u of tensor k updates it in its epilogue
     auto fuse = [&](GemmDesc& g, int k) {
         g.epi.upd_theta = h->upd_theta[k];
         g.epi.upd_v = h->upd_v[k];
-        g.epi.upd_lr = h->upd_lr;
-        g.epi.upd_decay = 1.0f - h->upd_lr * h->upd_wd[k];
+        g.epi.upd_wd = h->upd_wd[k];
         g.epi.upd_beta2 = h->upd_beta2;
         g.epi.upd_1mb2 = 1.0f - h->upd_beta2;
         g.epi.upd_eps = h->upd_eps;
-        g.epi.upd_inv_bc2 = inv_bc2;
         g.epi.out = params[k];   // the compute copy of the updated weight
         g.epi.out_f32 = cf32;
         if (h->bf16) g.epi_kind = EPI_UPDATE;   // tcgen05 path: staged, coalesced update epilogue
@@ -583,7 +591,7 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
     auto update_small = [&](int k, int64_t cnt) -> int {
         int r = launch_update(h->upd_theta[k], h->ubuf, 0, nullptr, h->upd_v[k],
                               h->bf16 ? static_cast<uint16_t*>(params[k]) : nullptr, cnt, h->upd_lr, h->upd_wd[k],
-                              0.0f, h->upd_beta2, h->upd_eps, inv_bc2, nullptr, 0.0f, h->sc, s);
+                              0.0f, h->upd_beta2, h->upd_eps, 0.0f, nullptr, 0.0f, h->sc, s, true);
         if (r == BOM_OK && !h->bf16 &&
             cudaMemcpyAsync(params[k], h->upd_theta[k], cnt * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
             r = BOM_ECUDA;
@@ -769,6 +777,7 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
             if (dx_next) cur ^= 1;
         }
     }
+    if (h->t_dev) launch_advance_step(h->t_dev, h->sc, s);
 #undef BOM_TRY
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }
@@ -819,20 +828,99 @@ bom_status bom_set_fused_update(bom_handle* h, float* const* theta, float* const
     return BOM_OK;
 }
 
+bom_status bom_set_step_scalars(bom_handle* h, int64_t* t_dev, const float* lr_dev) {
+    if (!h) return BOM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(t_dev) & 7u) != 0 || (reinterpret_cast<uintptr_t>(lr_dev) & 3u) != 0)
+        return BOM_ENOTSUP;
+    h->t_dev = t_dev;
+    h->lr_dev = lr_dev;
+    return BOM_OK;
+}
+
+}  // extern "C"
+
+struct bom_graph {
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    long long kernels = 0;   // kernel nodes: bom_launch_count advances by this much per launch
+};
+
+extern "C" {
+
+bom_status bom_graph_capture(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                             void* const* params, float* q, void* const* grads, void* const* h_out,
+                             bom_graph** out) {
+    if (!h || !out) return BOM_EINVAL;
+    *out = nullptr;
+    if (!h->t_dev || h->tracing) return BOM_EINVAL;
+    cudaStream_t cs = nullptr;
+    if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) return BOM_ECUDA;
+    // relaxed mode: the first launch of a GEMM shape sets kernel attributes
+    // (not stream work) while the capture is open
+    if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeRelaxed) != cudaSuccess) {
+        cudaStreamDestroy(cs);
+        return BOM_ECUDA;
+    }
+    const long long n0 = bom::g_launches.load();
+    const bom_status rc = bom_step(h, x, labels, n_rows, params, q, 0, grads, h_out, cs);
+    // the captured launches ran nothing: they are counted when the graph runs
+    const long long nk = bom::g_launches.load() - n0;
+    bom::g_launches.fetch_sub(nk);
+    cudaGraph_t g = nullptr;
+    const cudaError_t ec = cudaStreamEndCapture(cs, &g);
+    cudaStreamDestroy(cs);
+    if (rc != BOM_OK || ec != cudaSuccess || g == nullptr) {
+        if (g) cudaGraphDestroy(g);
+        cudaGetLastError();
+        return rc != BOM_OK ? rc : BOM_ECUDA;
+    }
+    cudaGraphExec_t ge = nullptr;
+    if (cudaGraphInstantiate(&ge, g, 0) != cudaSuccess) {
+        cudaGraphDestroy(g);
+        cudaGetLastError();
+        return BOM_ECUDA;
+    }
+    bom_graph* G = new (std::nothrow) bom_graph;
+    if (!G) {
+        cudaGraphExecDestroy(ge);
+        cudaGraphDestroy(g);
+        return BOM_ENOMEM;
+    }
+    G->graph = g;
+    G->exec = ge;
+    G->kernels = nk;
+    *out = G;
+    return BOM_OK;
+}
+
+bom_status bom_graph_launch(bom_graph* g, void* stream) {
+    if (!g || !g->exec) return BOM_EINVAL;
+    if (cudaGraphLaunch(g->exec, static_cast<cudaStream_t>(stream)) != cudaSuccess) return BOM_ECUDA;
+    bom::g_launches.fetch_add(g->kernels);
+    return BOM_OK;
+}
+
+void bom_graph_destroy(bom_graph* g) {
+    if (!g) return;
+    if (g->exec) cudaGraphExecDestroy(g->exec);
+    if (g->graph) cudaGraphDestroy(g->graph);
+    delete g;
+}
+
 bom_status bom_own_step_moment(bom_handle* h, float* M, const float* o, const float* hvec, float* mhat, int64_t n,
                                float beta1, int64_t t, double* sums, void* stream) {
     if (!h || n < 0 || t < 1 || !(beta1 >= 0.0f && beta1 < 1.0f)) return BOM_EINVAL;
     if (n == 0) return BOM_OK;
     if (!M || !o || !mhat || (sums && !hvec)) return BOM_EINVAL;
     if (!aligned16(M) || !aligned16(o) || !aligned16(mhat) || (hvec && !aligned16(hvec))) return BOM_ENOTSUP;
-    const float inv_bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta1), static_cast<double>(t))));
+    const float inv_bc1 = inv_bias_correction(beta1, t);
     const int nb = own_step_blocks(n, device_sm_count());
     launch_own_step_moment(M, o, hvec, mhat, n, beta1, inv_bc1, h->tel_part, nb, sums,
                            static_cast<cudaStream_t>(stream));
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }
 
-int64_t bom_stats_transfer_bytes(void) { return static_cast<int64_t>(sizeof(DevScalars)); }
+int64_t bom_stats_transfer_bytes(void) { return static_cast<int64_t>(kStatsBytes); }
 
 bom_status bom_step_outputs(bom_handle* h, const float** qhat, const float** s, const float** lse) {
     if (!h) return BOM_EINVAL;
@@ -846,7 +934,7 @@ bom_status bom_get_stats(bom_handle* h, bom_stats* out, void* stream) {
     if (!h || !out) return BOM_EINVAL;
     if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return BOM_ECUDA;
     DevScalars sc;
-    if (cudaMemcpy(&sc, h->sc, sizeof(sc), cudaMemcpyDeviceToHost) != cudaSuccess) return BOM_ECUDA;
+    if (cudaMemcpy(&sc, h->sc, kStatsBytes, cudaMemcpyDeviceToHost) != cudaSuccess) return BOM_ECUDA;
     out->loss = sc.loss;
     out->n_t = sc.n_t;
     out->status = sc.status;
@@ -866,7 +954,7 @@ bom_status bom_update(float* theta, const void* g, int32_t g_dtype, const float*
     if (!aligned16(theta) || !aligned16(g) || !aligned16(v) || (hvec && !aligned16(hvec)) ||
         (theta_bf16 && !aligned16(theta_bf16)))
         return BOM_ENOTSUP;
-    const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
+    const float inv_bc2 = inv_bias_correction(beta2, t);
     return static_cast<bom_status>(launch_update(theta, g, g_dtype == BOM_BF16, hvec, v, theta_bf16, n, lr, wd,
                                                  lambda, beta2, eps, inv_bc2, nullptr, 0.0f, nullptr,
                                                  static_cast<cudaStream_t>(stream)));
@@ -893,7 +981,7 @@ bom_status bom_update_clipped(float* theta, const void* g, int32_t g_dtype, cons
     if (!aligned16(theta) || !aligned16(g) || !aligned16(v) || (hvec && !aligned16(hvec)) ||
         (theta_bf16 && !aligned16(theta_bf16)))
         return BOM_ENOTSUP;
-    const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
+    const float inv_bc2 = inv_bias_correction(beta2, t);
     return static_cast<bom_status>(launch_update(theta, g, g_dtype == BOM_BF16, hvec, v, theta_bf16, n, lr, wd,
                                                  lambda, beta2, eps, inv_bc2, sq, max_norm, nullptr,
                                                  static_cast<cudaStream_t>(stream)));
@@ -909,7 +997,7 @@ bom_status bom_update_blockshared(float* theta, const void* g, int32_t g_dtype, 
     if (!(beta2 >= 0.0f && beta2 < 1.0f) || !(eps >= 0.0f)) return BOM_EINVAL;
     if (!aligned16(theta) || !aligned16(g) || (hvec && !aligned16(hvec)) || (theta_bf16 && !aligned16(theta_bf16)))
         return BOM_ENOTSUP;
-    const float inv_bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(beta2), static_cast<double>(t))));
+    const float inv_bc2 = inv_bias_correction(beta2, t);
     return static_cast<bom_status>(launch_update_blockshared(theta, g, g_dtype == BOM_BF16, hvec, v_blocks, theta_bf16,
                                                              n, block, lr, wd, lambda, beta2, eps, inv_bc2,
                                                              static_cast<cudaStream_t>(stream)));

@@ -2,6 +2,7 @@
 // block of a step, the GEMM epilogue parameter block, element load/store
 // helpers and the activation functions of the backbone.
 #pragma once
+#include <cstddef>
 #include <cstdint>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -24,7 +25,47 @@ struct DevScalars {
     float loss;            // mean CE over I_t
     float s_norm;          // ||s_t||
     float r_norm_mean;     // N_t^-1 sum_{i in I_t} ||r_i|| (own-step telemetry steps only, else 0)
+    // Step scalars, written by the label scan (the first kernel of a step) from
+    // host values or from the handle's device step counter, and read by the
+    // kernels that need them, so a captured step replays with the current t.
+    float lr;              // learning rate of the fused update
+    float inv_bc1;         // 1 / (1 - beta1^t)
+    float inv_bc2;         // 1 / (1 - beta2^t)
 };
+// Bytes of DevScalars that bom_get_stats copies to the host (the step scalars stay).
+constexpr size_t kStatsBytes = offsetof(DevScalars, lr);
+
+// 1 / (1 - beta^t) for t >= 1, with beta^t by binary powering in double.  The
+// host and the device evaluate the same correctly rounded operations in the
+// same order (no contraction), so a step that takes t from the device counter
+// gets the same float as one given t by the host.
+__host__ __device__ inline float inv_bias_correction(float beta, int64_t t) {
+    double p = 1.0, b = static_cast<double>(beta);
+#ifdef __CUDA_ARCH__
+    for (int64_t k = t; k > 0; k >>= 1) {
+        if (k & 1) p = __dmul_rn(p, b);
+        b = __dmul_rn(b, b);
+    }
+    return __double2float_rn(__ddiv_rn(1.0, __dsub_rn(1.0, p)));
+#else
+    for (int64_t k = t; k > 0; k >>= 1) {
+        if (k & 1) p = p * b;
+        b = b * b;
+    }
+    volatile double pv = p;   // keeps 1 - p a separate rounding
+    return static_cast<float>(1.0 / (1.0 - pv));
+#endif
+}
+
+// Weight-decay factor 1 - lr * wd, formed the same way by every update kernel.
+__device__ __forceinline__ float decay_factor(float lr, float wd) { return __fmaf_rn(-lr, wd, 1.0f); }
+
+// theta' = decay * theta - lr * q, written out so that every update kernel
+// rounds the same way whatever the compiler would contract: the decayed weight
+// stays exact inside one fma, only the step lr * q is rounded first.
+__device__ __forceinline__ float apply_step(float decay, float th, float lr, float q) {
+    return __fmaf_rn(decay, th, -__fmul_rn(lr, q));
+}
 
 __device__ __forceinline__ void latch_status(DevScalars* sc, int code) {
     atomicCAS(&sc->status, 0, code);
@@ -78,17 +119,19 @@ struct EpiParams {
     // element; the epilogue advances v and theta ([M, ld_out] fp32, the
     // layout of out) and stores the updated theta into out in out's dtype
     // (the compute copy) instead of u.
+    // The learning rate and 1/(1 - beta2^t) come from the step scalars in sc.
     float* upd_theta;
     float* upd_v;
-    float upd_lr, upd_decay, upd_beta2, upd_1mb2, upd_eps, upd_inv_bc2;
+    float upd_wd, upd_beta2, upd_1mb2, upd_eps;
 };
 
 // One element of the fused update (Section 3.4): returns the new theta.
 __device__ __forceinline__ float fused_update1(const EpiParams& e, int64_t idx, float u) {
+    const float lr = e.sc->lr, inv_bc2 = e.sc->inv_bc2;
     float vv = e.upd_v[idx];
     float th = e.upd_theta[idx];
     vv = fmaf(e.upd_beta2, vv, e.upd_1mb2 * u * u);
-    th = e.upd_decay * th - e.upd_lr * (u / (sqrtf(vv * e.upd_inv_bc2) + e.upd_eps));
+    th = apply_step(decay_factor(lr, e.upd_wd), th, lr, u / (sqrtf(vv * inv_bc2) + e.upd_eps));
     e.upd_v[idx] = vv;
     e.upd_theta[idx] = th;
     return th;

@@ -219,7 +219,7 @@ __device__ __forceinline__ void stg_scatter(void* base, int64_t ld, int row0, in
 constexpr int kUpdPitch = 33;
 constexpr int kUpdStgBytes = 32 * kUpdPitch * 4;
 __device__ __forceinline__ void staged_update32(const EpiParams& e, float* buf, int row0, int M, int n, int N,
-                                               const float (&u)[32]) {
+                                               const float (&u)[32], float lr, float decay, float inv_bc2) {
     const int lane = threadIdx.x & 31;
 #pragma unroll
     for (int k = 0; k < 32; ++k) buf[lane * kUpdPitch + k] = u[k];
@@ -243,8 +243,7 @@ __device__ __forceinline__ void staged_update32(const EpiParams& e, float* buf, 
                 const int64_t idx = static_cast<int64_t>(m) * e.ld_out + c;
                 const float uu = buf[(r0 + r) * kUpdPitch + lane];
                 const float v2 = fmaf(e.upd_beta2, vv[r], e.upd_1mb2 * uu * uu);
-                const float t2 =
-                    e.upd_decay * th[r] - e.upd_lr * uu * rcp_fast(sqrt_fast(v2 * e.upd_inv_bc2) + e.upd_eps);
+                const float t2 = apply_step(decay, th[r], lr, uu * rcp_fast(sqrt_fast(v2 * inv_bc2) + e.upd_eps));
                 e.upd_v[idx] = v2;
                 e.upd_theta[idx] = t2;
                 st_elem(e.out, idx, e.out_f32, t2);
@@ -620,6 +619,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 }
             } else if constexpr (EPI == EPI_UPDATE) {
                 const EpiRow r = epi_row(e, m, PM);
+                const float lr = e.sc->lr, inv_bc2 = e.sc->inv_bc2;
+                const float decay = decay_factor(lr, e.upd_wd);
                 float t[32];
 #pragma unroll 1
                 for (int j = 0; j < CPW; ++j) {
@@ -639,7 +640,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] += r.beta_r1 * t[i];
                     }
-                    staged_update32(e, reinterpret_cast<float*>(stg), row0, PM, n, PN, v);
+                    staged_update32(e, reinterpret_cast<float*>(stg), row0, PM, n, PN, v, lr, decay, inv_bc2);
                 }
             } else if constexpr (EPI == EPI_LOGITS || EPI == EPI_LOGITS_STG) {
                 // per (row, column half) softmax statistics: stats pair nt*2 + h.

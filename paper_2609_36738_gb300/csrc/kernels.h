@@ -24,8 +24,22 @@ inline int64_t resid_blocks(int64_t n) { return (n + kResidRows - 1) / kResidRow
 
 // Counts N_t, checks every label, latches BOM_ELABEL / BOM_EEMPTY and writes
 // the cotangent coefficients of the four backward passes into sc.
+// Where the step scalars (lr, 1/(1 - beta1^t), 1/(1 - beta2^t)) of a step come
+// from: the host values here, or the device step counter t_dev (and the device
+// learning rate lr_dev) registered with bom_set_step_scalars.  The label scan
+// writes them into sc; a t_dev below 1 latches BOM_EINVAL.
+struct StepScalarsIn {
+    float lr, inv_bc1, inv_bc2;
+    const int64_t* t_dev;
+    const float* lr_dev;
+    float beta1, beta2;
+};
 void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda,
-                        DevScalars* sc, cudaStream_t s);
+                        const StepScalarsIn& st, DevScalars* sc, cudaStream_t s);
+
+// *t_dev += 1 when the step latched no error (the last kernel of a step that
+// reads its t from the device).
+void launch_advance_step(int64_t* t_dev, const DevScalars* sc, cudaStream_t s);
 
 // fp32 path: per-row (max, sum exp) of Z [n, ldz] over V columns (one tile).
 void launch_row_stats_f32(const float* Z, int64_t ldz, int64_t n, int64_t V, float* stats, const DevScalars* sc,
@@ -45,7 +59,7 @@ void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, cons
 
 // s_j = N_t^-1 sum_b colpart[b, j]; q_j <- beta1 q_j + (1-beta1) s_j;
 // qhat_j = q_j * inv_bc1.  q is only written when the status word is clear.
-void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float inv_bc1, float* q,
+void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float* q,
                       float* s_out, float* qhat, DevScalars* sc, cudaStream_t s);
 
 // loss = N_t^-1 sum_i ce_i, ||s|| and, when rnorm is given, r_norm_mean = N_t^-1 sum_i rnorm_i.
@@ -97,9 +111,11 @@ int launch_update_blockshared(float* theta, const void* g, int g_bf16, const flo
 // BOM-AdamW update (see bom_update in bom.h).  With clip_sq, u is first scaled
 // by min(1, max_norm / (sqrt(*clip_sq) + 1e-6)) (bom_update_clipped).
 // When sc is given the kernel does nothing once the step's status word is set.
+// With step_scalars, lr and inv_bc2 are taken from sc's step scalars instead
+// (the vector updates inside bom_step).
 int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,
                   float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, const double* clip_sq,
-                  float max_norm, const DevScalars* sc, cudaStream_t s);
+                  float max_norm, const DevScalars* sc, cudaStream_t s, bool step_scalars = false);
 
 // *sq += sum u^2 over n elements (u = g, or (1-lambda) g + lambda h), in a fixed
 // order; `part` holds kOwnStepMaxBlocks doubles.

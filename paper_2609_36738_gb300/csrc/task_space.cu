@@ -72,8 +72,14 @@ __device__ float block_sum(float v, float* red) {
     return r;  // valid in thread 0
 }
 
+// The step counter advances only after a step that latched no error, so a
+// failed step leaves t, like q, as it was.
+__global__ void advance_step_kernel(int64_t* __restrict__ t, const DevScalars* sc) {
+    if (threadIdx.x == 0 && sc->status == 0) *t += 1;
+}
+
 __global__ void labels_scan_kernel(const int32_t* __restrict__ labels, int64_t n, int64_t V, int32_t ignore,
-                                   float lambda, DevScalars* sc) {
+                                   float lambda, const StepScalarsIn st, DevScalars* sc) {
     __shared__ int s_cnt[32], s_bad[32];
     int cnt = 0, bad = 0;
     for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
@@ -113,6 +119,19 @@ __global__ void labels_scan_kernel(const int32_t* __restrict__ labels, int64_t n
         sc->coef_q[2] = inv;
         sc->coef_r[3] = 0.0f;                   // own-step pass: N_t^-1 s_t
         sc->coef_q[3] = inv;
+        float bc1 = st.inv_bc1, bc2 = st.inv_bc2;
+        if (st.t_dev != nullptr) {
+            const int64_t t = *st.t_dev;
+            if (t < 1) {
+                latch_status(sc, BOM_EINVAL);
+            } else {
+                bc1 = inv_bias_correction(st.beta1, t);
+                bc2 = inv_bias_correction(st.beta2, t);
+            }
+        }
+        sc->lr = st.lr_dev != nullptr ? *st.lr_dev : st.lr;
+        sc->inv_bc1 = bc1;
+        sc->inv_bc2 = bc2;
         sc->loss = 0.0f;
         sc->s_norm = 0.0f;
         sc->r_norm_mean = 0.0f;
@@ -292,7 +311,7 @@ __global__ void __launch_bounds__(256, 3) residual_kernel(T* __restrict__ Z, int
 }
 
 __global__ void __launch_bounds__(256) finish_sq_kernel(const float* __restrict__ colpart, int64_t nblocks, int64_t V,
-                                                        float beta1, float inv_bc1, float* __restrict__ q,
+                                                        float beta1, float* __restrict__ q,
                                                         float* __restrict__ s_out, float* __restrict__ qhat,
                                                         const DevScalars* sc) {
     __shared__ float red[8][33];
@@ -301,6 +320,7 @@ __global__ void __launch_bounds__(256) finish_sq_kernel(const float* __restrict_
     const float acc = fixed_order_column_sum(colpart, nblocks, V, j, red);
     if (threadIdx.x >= 32 || j >= V) return;
     const float s = acc * sc->inv_nt;
+    const float inv_bc1 = sc->inv_bc1;
     const float qn = beta1 * q[j] + (1.0f - beta1) * s;
     q[j] = qn;
     s_out[j] = s;
@@ -552,9 +572,13 @@ inline unsigned cdiv(int64_t a, int64_t b) { return static_cast<unsigned>((a + b
 
 }  // namespace
 
-void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda, DevScalars* sc,
-                        cudaStream_t s) {
-    labels_scan_kernel<<<1, 1024, 0, s>>>(labels, n, V, ignore, lambda, sc); count_launch();
+void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda,
+                        const StepScalarsIn& st, DevScalars* sc, cudaStream_t s) {
+    labels_scan_kernel<<<1, 1024, 0, s>>>(labels, n, V, ignore, lambda, st, sc); count_launch();
+}
+
+void launch_advance_step(int64_t* t_dev, const DevScalars* sc, cudaStream_t s) {
+    advance_step_kernel<<<1, 32, 0, s>>>(t_dev, sc); count_launch();
 }
 
 void launch_row_stats_f32(const float* Z, int64_t ldz, int64_t n, int64_t V, float* stats, const DevScalars* sc,
@@ -582,9 +606,9 @@ void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, cons
     }
 }
 
-void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float inv_bc1, float* q,
+void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float* q,
                       float* s_out, float* qhat, DevScalars* sc, cudaStream_t s) {
-    finish_sq_kernel<<<cdiv(V, 32), 256, 0, s>>>(colpart, nblocks, V, beta1, inv_bc1, q, s_out, qhat, sc); count_launch();
+    finish_sq_kernel<<<cdiv(V, 32), 256, 0, s>>>(colpart, nblocks, V, beta1, q, s_out, qhat, sc); count_launch();
 }
 
 void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, const float* rnorm, DevScalars* sc,

@@ -25,13 +25,25 @@ int device_sm_count();
 namespace {
 
 struct UpdCoef {
-    float lr, decay, lam, beta2, one_m_beta2, eps, inv_bc2;
+    float lr, wd, decay, lam, beta2, one_m_beta2, eps, inv_bc2;
+    int from_step;   // take lr and inv_bc2 from the step scalars (updates inside bom_step)
 };
+
+// The coefficients a kernel uses: lr and 1/(1 - beta2^t) from the step
+// scalars when asked, and the decay factor formed on the device.
+__device__ __forceinline__ UpdCoef resolve_coef(UpdCoef c, const DevScalars* sc) {
+    if (c.from_step && sc != nullptr) {
+        c.lr = sc->lr;
+        c.inv_bc2 = sc->inv_bc2;
+    }
+    c.decay = decay_factor(c.lr, c.wd);
+    return c;
+}
 
 __device__ __forceinline__ float upd1(float& th, float& vv, float u, const UpdCoef& c) {
     vv = fmaf(c.beta2, vv, c.one_m_beta2 * u * u);
     const float den = sqrtf(vv * c.inv_bc2) + c.eps;
-    th = c.decay * th - c.lr * (u / den);
+    th = apply_step(c.decay, th, c.lr, u / den);
     return th;
 }
 
@@ -43,10 +55,11 @@ __device__ __forceinline__ float clip_scale(const double* sq, float max_norm) {
 template <bool G_BF16, bool HAS_H, bool SHADOW, bool CLIP>
 __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ theta, const void* __restrict__ g,
                                                      const float* __restrict__ h, float* __restrict__ v,
-                                                     uint16_t* __restrict__ shadow, int64_t n, UpdCoef c,
+                                                     uint16_t* __restrict__ shadow, int64_t n, UpdCoef c_in,
                                                      const double* __restrict__ clip_sq, float max_norm,
                                                      const DevScalars* sc) {
     if (sc != nullptr && sc->status != 0) return;   // inside a step that latched an error
+    const UpdCoef c = resolve_coef(c_in, sc);
     const float cs = CLIP ? clip_scale(clip_sq, max_norm) : 1.0f;
     const int64_t n4 = n >> 2;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -144,9 +157,10 @@ template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
 __global__ void __launch_bounds__(256) update_blockshared_kernel(float* __restrict__ theta, const void* __restrict__ g,
                                                                  const float* __restrict__ h, float* __restrict__ vb,
                                                                  uint16_t* __restrict__ shadow, int64_t n,
-                                                                 int64_t block, UpdCoef c) {
+                                                                 int64_t block, UpdCoef c_in) {
     __shared__ float red[8];
     __shared__ float s_den;
+    const UpdCoef c = resolve_coef(c_in, nullptr);
     const int64_t nb = (n + block - 1) / block;
     for (int64_t b = blockIdx.x; b < nb; b += gridDim.x) {
         const int64_t e0 = b * block;
@@ -176,10 +190,10 @@ __global__ void __launch_bounds__(256) update_blockshared_kernel(float* __restri
             load_u<G_BF16, HAS_H, VEC>(g, h, i, c.lam, u);
             if constexpr (VEC == 4) {
                 float4 th = __ldcs(reinterpret_cast<const float4*>(theta + i));
-                th.x = c.decay * th.x - c.lr * (u[0] / den);
-                th.y = c.decay * th.y - c.lr * (u[1] / den);
-                th.z = c.decay * th.z - c.lr * (u[2] / den);
-                th.w = c.decay * th.w - c.lr * (u[3] / den);
+                th.x = apply_step(c.decay, th.x, c.lr, u[0] / den);
+                th.y = apply_step(c.decay, th.y, c.lr, u[1] / den);
+                th.z = apply_step(c.decay, th.z, c.lr, u[2] / den);
+                th.w = apply_step(c.decay, th.w, c.lr, u[3] / den);
                 __stcs(reinterpret_cast<float4*>(theta + i), th);
                 if constexpr (SHADOW) {
                     uint2 sh;
@@ -190,7 +204,7 @@ __global__ void __launch_bounds__(256) update_blockshared_kernel(float* __restri
             } else {
 #pragma unroll
                 for (int k = 0; k < VEC; ++k) {
-                    const float th = c.decay * theta[i + k] - c.lr * (u[k] / den);
+                    const float th = apply_step(c.decay, theta[i + k], c.lr, u[k] / den);
                     theta[i + k] = th;
                     if (SHADOW) reinterpret_cast<__nv_bfloat16*>(shadow)[i + k] = __float2bfloat16_rn(th);
                 }
@@ -294,10 +308,10 @@ __device__ __forceinline__ void row_update(const RowRegs<G_BF16, WPT>& r, float*
             float u[4];
             word_u<G_BF16, HAS_H>(r.gw[k], r.hw[k], c.lam, u);
             float4 t = r.th[k];
-            t.x = c.decay * t.x - c.lr * (u[0] / den);
-            t.y = c.decay * t.y - c.lr * (u[1] / den);
-            t.z = c.decay * t.z - c.lr * (u[2] / den);
-            t.w = c.decay * t.w - c.lr * (u[3] / den);
+            t.x = apply_step(c.decay, t.x, c.lr, u[0] / den);
+            t.y = apply_step(c.decay, t.y, c.lr, u[1] / den);
+            t.z = apply_step(c.decay, t.z, c.lr, u[2] / den);
+            t.w = apply_step(c.decay, t.w, c.lr, u[3] / den);
             __stcs(reinterpret_cast<float4*>(theta + i), t);
             if constexpr (SHADOW) {
                 uint2 sh;
@@ -321,9 +335,10 @@ __global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __re
                                                                      const float* __restrict__ h,
                                                                      float* __restrict__ vb,
                                                                      uint16_t* __restrict__ shadow, int64_t n,
-                                                                     int64_t block, UpdCoef c) {
+                                                                     int64_t block, UpdCoef c_in) {
     __shared__ float red[8];
     __shared__ float s_den;
+    const UpdCoef c = resolve_coef(c_in, nullptr);
     const int64_t nb = (n + block - 1) / block;
     const int64_t G = gridDim.x;
     int64_t b = blockIdx.x;
@@ -458,11 +473,13 @@ __global__ void sqnorm_finish_kernel(const double* __restrict__ part, int nblock
 
 int launch_update(float* theta, const void* g, int g_bf16, const float* h, float* v, uint16_t* shadow, int64_t n,
                   float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, const double* clip_sq,
-                  float max_norm, const DevScalars* sc, cudaStream_t s) {
+                  float max_norm, const DevScalars* sc, cudaStream_t s, bool step_scalars) {
     if (n <= 0) return BOM_OK;
     UpdCoef c;
     c.lr = lr;
-    c.decay = 1.0f - lr * wd;
+    c.wd = wd;
+    c.decay = 0.0f;
+    c.from_step = step_scalars ? 1 : 0;
     c.lam = lambda;
     c.beta2 = beta2;
     c.one_m_beta2 = 1.0f - beta2;
@@ -514,7 +531,9 @@ int launch_update_blockshared(float* theta, const void* g, int g_bf16, const flo
     if (n <= 0) return BOM_OK;
     UpdCoef c;
     c.lr = lr;
-    c.decay = 1.0f - lr * wd;
+    c.wd = wd;
+    c.decay = 0.0f;
+    c.from_step = 0;
     c.lam = lambda;
     c.beta2 = beta2;
     c.one_m_beta2 = 1.0f - beta2;
