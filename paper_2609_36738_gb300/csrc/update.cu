@@ -16,6 +16,8 @@
 // a fixed order, thread 0 advances v_b, a second sweep applies the update; the
 // second sweep's reads of g and h hit L2.
 #include "kernels.h"
+#include "tc_ptx.cuh"
+#include <mutex>
 #include <type_traits>
 
 namespace bom {
@@ -149,6 +151,207 @@ __device__ __forceinline__ void load_u(const void* g, const float* h, int64_t i,
                              : static_cast<const float*>(g)[i + k];
             if (HAS_H) x = (1.0f - lam) * x + lam * h[i + k];
             u[k] = x;
+        }
+    }
+}
+
+// Blocks larger than a CTA holds in registers: a cluster of kBlockCluster
+// CTAs takes one block at a time, so a few large blocks (a whole-tensor block
+// of a big weight) still spread over many SMs.  Each CTA sums u^2 over its
+// interleaved share of the block; after a cluster barrier the leading CTA adds
+// the CTA partials from distributed shared memory in rank order (fixed order:
+// deterministic), advances v_b and publishes the denominator, which every CTA
+// reads back after a second barrier; then all update their share (the second
+// read of u mostly hits L2: the cluster's block is its whole working set).
+// Every CTA of a cluster walks the same blocks, so all meet every barrier.
+constexpr int kBlockCluster = 8;
+
+template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
+__global__ void __launch_bounds__(256) update_blockshared_cluster_kernel(float* __restrict__ theta,
+                                                                         const void* __restrict__ g,
+                                                                         const float* __restrict__ h,
+                                                                         float* __restrict__ vb,
+                                                                         uint16_t* __restrict__ shadow, int64_t n,
+                                                                         int64_t block, UpdCoef c_in) {
+    __shared__ float red[8];
+    __shared__ float s_part;   // this CTA's sum of u^2 over its share of the block
+    __shared__ float s_den;    // leading CTA: the block's denominator
+    __shared__ float s_den_local;
+    const UpdCoef c = resolve_coef(c_in, nullptr);
+    const uint32_t rank = cluster_ctarank();
+    const int64_t ncl = gridDim.x / kBlockCluster;
+    const int64_t nb = (n + block - 1) / block;
+    const int64_t stride = static_cast<int64_t>(kBlockCluster) * 256 * VEC;
+    for (int64_t b = blockIdx.x / kBlockCluster; b < nb; b += ncl) {
+        const int64_t e0 = b * block;
+        const int64_t e1 = e0 + block < n ? e0 + block : n;
+        const int64_t i0 = e0 + (static_cast<int64_t>(rank) * 256 + threadIdx.x) * VEC;
+        float acc = 0.0f;
+        int64_t i = i0;
+        for (; i + 3 * stride < e1; i += 4 * stride) {   // four loads in flight per thread
+            float u[4][VEC];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) load_u<G_BF16, HAS_H, VEC>(g, h, i + j * stride, c.lam, u[j]);
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) acc = fmaf(u[j][k], u[j][k], acc);
+        }
+        for (; i < e1; i += stride) {
+            float u[VEC];
+            load_u<G_BF16, HAS_H, VEC>(g, h, i, c.lam, u);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) acc = fmaf(u[k], u[k], acc);
+        }
+        acc = warp_sum_f(acc);
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float tot = 0.0f;
+#pragma unroll
+            for (int w = 0; w < 8; ++w) tot += red[w];
+            s_part = tot;
+        }
+        cluster_sync();   // every CTA's s_part is written
+        if (rank == 0 && threadIdx.x == 0) {
+            float tot = 0.0f;
+            for (uint32_t r = 0; r < kBlockCluster; ++r) tot += ld_shared_cluster_f32(mapa_shared(smem_u32(&s_part), r));
+            const float vv = fmaf(c.beta2, vb[b], c.one_m_beta2 * (tot / static_cast<float>(e1 - e0)));
+            vb[b] = vv;
+            s_den = sqrtf(vv * c.inv_bc2) + c.eps;
+        }
+        cluster_sync();   // s_den is written; every s_part has been read
+        if (threadIdx.x == 0) s_den_local = ld_shared_cluster_f32(mapa_shared(smem_u32(&s_den), 0));
+        __syncthreads();
+        const float den = s_den_local;
+#pragma unroll 2
+        for (int64_t i = i0; i < e1; i += stride) {
+            float u[VEC];
+            load_u<G_BF16, HAS_H, VEC>(g, h, i, c.lam, u);
+            if constexpr (VEC == 4) {
+                float4 th = __ldcs(reinterpret_cast<const float4*>(theta + i));
+                th.x = apply_step(c.decay, th.x, c.lr, u[0] / den);
+                th.y = apply_step(c.decay, th.y, c.lr, u[1] / den);
+                th.z = apply_step(c.decay, th.z, c.lr, u[2] / den);
+                th.w = apply_step(c.decay, th.w, c.lr, u[3] / den);
+                __stcs(reinterpret_cast<float4*>(theta + i), th);
+                if constexpr (SHADOW) {
+                    uint2 sh;
+                    sh.x = pack_bf16x2(th.x, th.y);
+                    sh.y = pack_bf16x2(th.z, th.w);
+                    __stcs(reinterpret_cast<uint2*>(shadow + i), sh);
+                }
+            } else {
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) {
+                    const float th = apply_step(c.decay, theta[i + k], c.lr, u[k] / den);
+                    theta[i + k] = th;
+                    if (SHADOW) reinterpret_cast<__nv_bfloat16*>(shadow)[i + k] = __float2bfloat16_rn(th);
+                }
+            }
+        }
+        // s_den_local and red are rewritten only after the next block's first
+        // cluster barrier, which every thread of this CTA reaches after its reads
+    }
+    cluster_sync();   // no CTA leaves while another may still read its shared memory
+}
+
+// Fewer large blocks than the GPU runs clusters at once (a whole-tensor block
+// of a big weight): the whole grid works on them in three launches.
+//   bs_chunk_sq   part[b * S + j] = sum of u^2 over chunk j of block b (chunks
+//                 of `ch` elements, fixed order within a chunk);
+//   bs_finish     one warp per block adds its S partials (lane-strided, then a
+//                 fixed shuffle tree), advances v_b and writes the denominator;
+//   bs_apply      the elementwise update with its block's denominator.
+template <bool G_BF16, bool HAS_H, int VEC>
+__global__ void __launch_bounds__(256) bs_chunk_sq_kernel(const void* __restrict__ g, const float* __restrict__ h,
+                                                          float lam, int64_t n, int64_t block, int64_t ch, int64_t S,
+                                                          int64_t nchunks, float* __restrict__ part) {
+    __shared__ float red[8];
+    for (int64_t cidx = blockIdx.x; cidx < nchunks; cidx += gridDim.x) {
+        const int64_t b = cidx / S, j = cidx - b * S;
+        const int64_t e0 = b * block + j * ch;
+        int64_t e1 = b * block + block < n ? b * block + block : n;
+        if (e0 + ch < e1) e1 = e0 + ch;
+        const int64_t st = 256 * VEC;
+        float acc = 0.0f;
+        int64_t i = e0 + static_cast<int64_t>(threadIdx.x) * VEC;
+        for (; i + 3 * st < e1; i += 4 * st) {   // four loads in flight per thread
+            float u[4][VEC];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) load_u<G_BF16, HAS_H, VEC>(g, h, i + q * st, lam, u[q]);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) acc = fmaf(u[q][k], u[q][k], acc);
+        }
+        for (; i < e1; i += st) {
+            float u[VEC];
+            load_u<G_BF16, HAS_H, VEC>(g, h, i, lam, u);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) acc = fmaf(u[k], u[k], acc);
+        }
+        acc = warp_sum_f(acc);
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float tot = 0.0f;
+#pragma unroll
+            for (int w = 0; w < 8; ++w) tot += red[w];
+            part[cidx] = tot;
+        }
+        __syncthreads();
+    }
+}
+
+__global__ void __launch_bounds__(256) bs_finish_kernel(const float* __restrict__ part, int64_t S, int64_t nb,
+                                                        int64_t n, int64_t block, float* __restrict__ vb,
+                                                        float* __restrict__ den, UpdCoef c_in) {
+    const UpdCoef c = resolve_coef(c_in, nullptr);
+    const int64_t b = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (b >= nb) return;
+    float t = 0.0f;
+    for (int64_t j = lane; j < S; j += 32) t += part[b * S + j];
+    t = warp_sum_f(t);
+    if (lane == 0) {
+        const int64_t len = b * block + block < n ? block : n - b * block;
+        const float vv = fmaf(c.beta2, vb[b], c.one_m_beta2 * (t / static_cast<float>(len)));
+        vb[b] = vv;
+        den[b] = sqrtf(vv * c.inv_bc2) + c.eps;
+    }
+}
+
+template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
+__global__ void __launch_bounds__(256) bs_apply_kernel(float* __restrict__ theta, const void* __restrict__ g,
+                                                       const float* __restrict__ h, uint16_t* __restrict__ shadow,
+                                                       int64_t n, int64_t block, const float* __restrict__ den,
+                                                       UpdCoef c_in) {
+    const UpdCoef c = resolve_coef(c_in, nullptr);
+    const int64_t nv = n / VEC;   // VEC = 4 only when n and block are multiples of 4
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * 256;
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x; q < nv; q += stride) {
+        const int64_t i = q * VEC;
+        const float d = den[i / block];   // a group of VEC elements never straddles two blocks
+        float u[VEC];
+        load_u<G_BF16, HAS_H, VEC>(g, h, i, c.lam, u);
+        if constexpr (VEC == 4) {
+            float4 th = __ldcs(reinterpret_cast<const float4*>(theta + i));
+            th.x = apply_step(c.decay, th.x, c.lr, u[0] / d);
+            th.y = apply_step(c.decay, th.y, c.lr, u[1] / d);
+            th.z = apply_step(c.decay, th.z, c.lr, u[2] / d);
+            th.w = apply_step(c.decay, th.w, c.lr, u[3] / d);
+            __stcs(reinterpret_cast<float4*>(theta + i), th);
+            if constexpr (SHADOW) {
+                uint2 sh;
+                sh.x = pack_bf16x2(th.x, th.y);
+                sh.y = pack_bf16x2(th.z, th.w);
+                __stcs(reinterpret_cast<uint2*>(shadow + i), sh);
+            }
+        } else {
+            const float th = apply_step(c.decay, theta[i], c.lr, u[0] / d);
+            theta[i] = th;
+            if (SHADOW) reinterpret_cast<__nv_bfloat16*>(shadow)[i] = __float2bfloat16_rn(th);
         }
     }
 }
@@ -391,10 +594,139 @@ void launch_reg_wpt(float* theta, const void* g, const float* h, float* vb, uint
     else launch_reg<G_BF16, HAS_H, SHADOW, 8>(theta, g, h, vb, shadow, n, block, c, s);
 }
 
+template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
+cudaLaunchConfig_t cluster_cfg(cudaLaunchAttribute* at) {
+    cudaLaunchConfig_t cfg = {};
+    at->id = cudaLaunchAttributeClusterDimension;
+    at->val.clusterDim.x = kBlockCluster;
+    at->val.clusterDim.y = 1;
+    at->val.clusterDim.z = 1;
+    cfg.blockDim = dim3(256);
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cfg;
+}
+
+// Clusters of the cluster kernel that run at once (cached per instantiation).
+template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
+int cluster_slots() {
+    static int slots = 0;
+    if (slots == 0) {
+        cudaLaunchAttribute at;
+        cudaLaunchConfig_t cfg = cluster_cfg<G_BF16, HAS_H, SHADOW, VEC>(&at);
+        cfg.gridDim = dim3(static_cast<unsigned>(device_sm_count() / kBlockCluster * kBlockCluster));
+        int m = 0;
+        if (cudaOccupancyMaxActiveClusters(&m, update_blockshared_cluster_kernel<G_BF16, HAS_H, SHADOW, VEC>, &cfg) !=
+                cudaSuccess ||
+            m < 1) {
+            cudaGetLastError();
+            m = device_sm_count() / kBlockCluster;
+        }
+        slots = m > 0 ? m : 1;
+    }
+    return slots;
+}
+
+template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
+int launch_cluster(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
+                   int64_t block, const UpdCoef& c, int64_t nclusters, cudaStream_t s) {
+    cudaLaunchAttribute at;
+    cudaLaunchConfig_t cfg = cluster_cfg<G_BF16, HAS_H, SHADOW, VEC>(&at);
+    cfg.gridDim = dim3(static_cast<unsigned>(nclusters * kBlockCluster));
+    cfg.stream = s;
+    cudaLaunchKernelEx(&cfg, update_blockshared_cluster_kernel<G_BF16, HAS_H, SHADOW, VEC>, theta, g, h, vb, shadow,
+                       n, block, c);
+    count_launch();
+    return BOM_OK;
+}
+
+// A stream-ordered memory pool of the library's own on the current device,
+// kept reserved between calls (release threshold at its maximum), so the few
+// KB of scratch below cost no mapping after the first call and calls on
+// different streams never share a buffer.
+cudaMemPool_t scratch_pool() {
+    static std::mutex mu;
+    static cudaMemPool_t pools[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (pools[dev] == nullptr) {
+        cudaMemPoolProps props = {};
+        props.allocType = cudaMemAllocationTypePinned;
+        props.handleTypes = cudaMemHandleTypeNone;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = dev;
+        cudaMemPool_t pool = nullptr;
+        if (cudaMemPoolCreate(&pool, &props) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        uint64_t keep = ~uint64_t(0);
+        cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
+        pools[dev] = pool;
+    }
+    return pools[dev];
+}
+
+// The grid-wide path; its partials and denominators live in a stream-ordered
+// scratch of (chunks + blocks) floats from scratch_pool, freed on the same
+// stream.
+template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
+int launch_grid_blocks(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
+                       int64_t block, const UpdCoef& c, cudaStream_t s) {
+    const int64_t nb = (n + block - 1) / block;
+    const int64_t G = 4 * static_cast<int64_t>(device_sm_count());
+    int64_t S = (4 * G + nb - 1) / nb;                 // chunks per block: about four per CTA in all
+    int64_t ch = (block + S - 1) / S;
+    ch = (ch + 1023) / 1024 * 1024;                    // whole passes of 256 threads x 4 elements
+    S = (block + ch - 1) / ch;
+    const int64_t nchunks = nb * S;
+    float* scr = nullptr;
+    cudaMemPool_t pool = scratch_pool();
+    if (pool == nullptr || cudaMallocFromPoolAsync(reinterpret_cast<void**>(&scr),
+                                                   static_cast<size_t>(nchunks + nb) * sizeof(float), pool, s) !=
+                               cudaSuccess) {
+        cudaGetLastError();
+        return BOM_ENOMEM;
+    }
+    float* part = scr;
+    float* den = scr + nchunks;
+    const int64_t g1 = nchunks < G ? nchunks : G;
+    bs_chunk_sq_kernel<G_BF16, HAS_H, VEC><<<static_cast<unsigned>(g1), 256, 0, s>>>(g, h, c.lam, n, block, ch, S,
+                                                                                    nchunks, part);
+    count_launch();
+    bs_finish_kernel<<<static_cast<unsigned>((nb + 7) / 8), 256, 0, s>>>(part, S, nb, n, block, vb, den, c);
+    count_launch();
+    const int64_t need = (n / VEC + 255) / 256;
+    int64_t g3 = 8 * static_cast<int64_t>(device_sm_count());
+    if (g3 > need) g3 = need;
+    if (g3 < 1) g3 = 1;
+    bs_apply_kernel<G_BF16, HAS_H, SHADOW, VEC><<<static_cast<unsigned>(g3), 256, 0, s>>>(theta, g, h, shadow, n,
+                                                                                          block, den, c);
+    count_launch();
+    cudaFreeAsync(scr, s);
+    return BOM_OK;
+}
+
+// Blocks above the register-resident size: the cluster kernel when there are
+// enough blocks to occupy every cluster slot, else the grid-wide path.
+template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
+int launch_large_blocks(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
+                        int64_t block, const UpdCoef& c, cudaStream_t s) {
+    const int64_t nb = (n + block - 1) / block;
+    const int64_t slots = cluster_slots<G_BF16, HAS_H, SHADOW, VEC>();
+    if (nb >= slots) return launch_cluster<G_BF16, HAS_H, SHADOW, VEC>(theta, g, h, vb, shadow, n, block, c, slots, s);
+    return launch_grid_blocks<G_BF16, HAS_H, SHADOW, VEC>(theta, g, h, vb, shadow, n, block, c, s);
+}
+
 template <bool G_BF16, bool HAS_H, int VEC>
-void dispatch_blockshared(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
-                          int64_t block, const UpdCoef& c, int grid, cudaStream_t s) {
-    if (VEC == 4 && block <= kRegMaxBlock) {
+int dispatch_blockshared(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
+                         int64_t block, const UpdCoef& c, int grid, cudaStream_t s) {
+    if (block > kRegMaxBlock) {
+        if (shadow) return launch_large_blocks<G_BF16, HAS_H, true, VEC>(theta, g, h, vb, shadow, n, block, c, s);
+        return launch_large_blocks<G_BF16, HAS_H, false, VEC>(theta, g, h, vb, shadow, n, block, c, s);
+    }
+    if (VEC == 4) {
         if (shadow) launch_reg_wpt<G_BF16, HAS_H, true>(theta, g, h, vb, shadow, n, block, c, s);
         else launch_reg_wpt<G_BF16, HAS_H, false>(theta, g, h, vb, shadow, n, block, c, s);
     } else if (shadow) {
@@ -404,6 +736,7 @@ void dispatch_blockshared(float* theta, const void* g, const float* h, float* vb
                                                                                   c);
     }
     count_launch();
+    return BOM_OK;
 }
 
 template <bool G_BF16, bool HAS_H>
@@ -544,23 +877,25 @@ int launch_update_blockshared(float* theta, const void* g, int g_bf16, const flo
     if (grid > nb) grid = nb;
     const bool vec = (block % 4 == 0) && (n % 4 == 0);
     const int gi = static_cast<int>(grid);
+    int rc = BOM_OK;
     if (vec) {
         if (g_bf16) {
-            if (h) dispatch_blockshared<true, true, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
-            else dispatch_blockshared<true, false, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            if (h) rc = dispatch_blockshared<true, true, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            else rc = dispatch_blockshared<true, false, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
         } else {
-            if (h) dispatch_blockshared<false, true, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
-            else dispatch_blockshared<false, false, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            if (h) rc = dispatch_blockshared<false, true, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            else rc = dispatch_blockshared<false, false, 4>(theta, g, h, vb, shadow, n, block, c, gi, s);
         }
     } else {
         if (g_bf16) {
-            if (h) dispatch_blockshared<true, true, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
-            else dispatch_blockshared<true, false, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            if (h) rc = dispatch_blockshared<true, true, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            else rc = dispatch_blockshared<true, false, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
         } else {
-            if (h) dispatch_blockshared<false, true, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
-            else dispatch_blockshared<false, false, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            if (h) rc = dispatch_blockshared<false, true, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
+            else rc = dispatch_blockshared<false, false, 1>(theta, g, h, vb, shadow, n, block, c, gi, s);
         }
     }
+    if (rc != BOM_OK) return rc;
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }
 

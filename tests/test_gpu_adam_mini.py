@@ -30,12 +30,18 @@ def _close(th_gpu, theta0, ref_th, rel=1e-5):
 
 
 # (n, block): per-output-neuron rows of the vision head and LM shapes, a ragged
-# last block, blocks that are not a multiple of 4, one whole-tensor block and
+# last block, blocks that are not a multiple of 4, whole-tensor blocks and
 # blocks of one element (elementwise BOM-AdamW).
-# The register-resident kernel takes blocks of up to 8192 elements (d % 4 = 0);
-# (3 x 16384, 16384) takes the two-sweep kernel, the odd sizes the scalar one.
+# The register-resident kernel takes blocks of up to 8192 elements (d % 4 = 0).
+# Larger blocks take the cluster kernel (eight CTAs per block) when there are
+# at least as many blocks as cluster slots (201 blocks of 10_000; 171 odd-sized
+# ones on its scalar path), else the grid-wide path: the 16-Mi-element
+# whole-tensor block of a 4096 x 4096 weight, one aligned whole-tensor block,
+# a few blocks with a ragged last one, and the odd-sized (50_001, 50_001).
+# Small odd sizes take the scalar kernel.
 CASES = [(3072 * 768, 768), (64 * 2048, 2048), (8 * 8192, 8192), (1000, 300), (29 * 7, 29), (50_001, 50_001),
-         (4099, 1), (3, 5), (3 * 16384, 16384)]
+         (4099, 1), (3, 5), (3 * 16384, 16384), (1 << 20, 1 << 20), (5 * 40_000 + 124, 40_000),
+         (4096 * 4096, 4096 * 4096), (200 * 10_000 + 5_000, 10_000), (170 * 9_001 + 17, 9_001)]
 
 
 @pytest.mark.parametrize("n,block", CASES)
@@ -83,6 +89,24 @@ def test_blockshared_trajectory_and_determinism():
         torch.cuda.synchronize()
         assert G.rel_l2(G.np64(th), ref_th) < 1e-6
         assert G.rel_l2(G.np64(vb), ref_v) < 1e-5
+        outs.append((th.clone(), vb.clone()))
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+
+
+@pytest.mark.parametrize("n,block", [(6 * 65_536 + 36, 65_536), (200 * 10_000 + 5_000, 10_000)])
+def test_blockshared_large_blocks_are_deterministic(n, block):
+    """Blocks spread over many CTAs (the grid-wide path for a few blocks, the
+    cluster kernel for many) add their partial sums in a fixed order: two runs
+    from the same state agree to the bit."""
+    theta, g, h, _ = I.update_sweep_host(n, seed=8)
+    outs = []
+    for _ in range(2):
+        th = G.to_dev(theta)
+        vb = torch.zeros(-(-n // block), dtype=torch.float32, device=G.DEV)
+        for t in range(1, 4):
+            B.bom_update_blockshared(th, G.to_dev(g), B.BOM_BF16, G.to_dev(h), vb, None, n, block, LR, WD, LAM, B2,
+                                     EPS, t)
+        torch.cuda.synchronize()
         outs.append((th.clone(), vb.clone()))
     assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
 
