@@ -280,7 +280,11 @@ bom_status bom_update(float* theta, const void* g, int32_t g_dtype, const float*
  * the last block may be shorter.
  *   v_blocks    [ceil(n / block)] fp32, updated in place (v_0 = 0).
  * Other arguments as bom_update.  block >= 1; sums of u^2 are formed per
- * block in a fixed order (deterministic). */
+ * block in a fixed order (deterministic).  Blocks of more than 8192 elements,
+ * when there are fewer of them than the GPU runs 8-CTA clusters at once, are
+ * spread over the whole grid: that path takes a few KB of stream-ordered
+ * scratch from a memory pool the library keeps per device (BOM_ENOMEM if it
+ * cannot). */
 /* Global-norm clipping of the numerator (pretraining-parameters appendix:
  * language-modeling runs clip at 1.0; convergence appendix: the clipped
  * numerator is what the adaptive update receives).  Two calls:
