@@ -14,6 +14,36 @@ namespace bom {
 // Host-side count of kernel launches made by the library (bom_launch_count).
 void count_launch();
 
+// Programmatic dependent launch.  Every kernel of the library starts with
+// pdl_enter(): it lets the next kernel on the stream be scheduled (its launch
+// and its prologue then overlap this kernel's tail), and waits until the
+// previous kernel has completed and its memory is visible, before touching
+// global memory.  Kernels launched without the attribute pass through both at
+// once, so the order of the stream is kept either way.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_enter() {
+    pdl_trigger();
+    pdl_wait();
+}
+
+// Launches kernel k with the programmatic-stream-serialization attribute.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                            Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k, static_cast<KArgs>(args)...);
+}
+
 // Per-step scalars that live on the device so that no host round trip is
 // needed between the label scan and the kernels that scale by 1/N_t.
 struct DevScalars {

@@ -22,6 +22,7 @@ struct Params {
 };
 
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const Params p) {
+    pdl_enter();
     if (p.epi.sc != nullptr && p.epi.sc->status != 0) return;
     __shared__ float As[TK][TM + 1];
     __shared__ float Bs[TK][TN + 1];
@@ -101,7 +102,7 @@ int launch_gemm_simt(const GemmDesc& g, cudaStream_t stream) {
     p.epi = g.epi;
     dim3 grid(static_cast<unsigned>((g.N + simt::TN - 1) / simt::TN), static_cast<unsigned>((g.M + simt::TM - 1) / simt::TM));
     if (grid.y > 65535) return BOM_ENOTSUP;
-    simt::gemm_simt_kernel<<<grid, 256, 0, stream>>>(p); count_launch();
+    launch_k(simt::gemm_simt_kernel, dim3(grid), dim3(256), 0, stream, p); count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }
 

@@ -305,6 +305,9 @@ struct Cfg {
 
 template <int CG, bool A_MN, bool B_MN, int EPI>
 __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_constant__ Params p) {
+    // the next kernel may be scheduled now; this one's own set-up (barriers,
+    // TMEM, tensor-map prefetch) runs before it waits for the previous kernel
+    pdl_trigger();
     using C = Cfg<CG, EPI>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
@@ -343,7 +346,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         mbar_init(drain, 1);
         for (int b = 0; b < 16; ++b) mbar_init(&ebar[b], 1);
         *abort_flag = 0;
-        *skip_flag = (p.epi.sc != nullptr && p.epi.sc->status != 0) ? 1 : 0;
         fence_barrier_init();
     }
     if (warp == 0 && lane == 0) {
@@ -363,6 +365,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
     __syncthreads();
     if constexpr (CG == 2) cluster_sync();   // barriers of both CTAs initialised before any remote use
     tc_fence_after();
+    pdl_wait();   // the previous kernel's writes (operands, status word) are visible from here on
+    if (threadIdx.x == 0) *skip_flag = (p.epi.sc != nullptr && p.epi.sc->status != 0) ? 1 : 0;
+    __syncthreads();
     const uint32_t tmem_base = *tmem_slot;
     const bool skip = *skip_flag != 0;
 
@@ -909,16 +914,18 @@ static int launch_inst(const Params& p, cudaStream_t stream) {
         cfg.blockDim = dim3(NUM_THREADS);
         cfg.dynamicSmemBytes = C::SMEM;
         cfg.stream = stream;
-        cudaLaunchAttribute at;
-        at.id = cudaLaunchAttributeClusterDimension;
-        at.val.clusterDim.x = 2;
-        at.val.clusterDim.y = 1;
-        at.val.clusterDim.z = 1;
-        cfg.attrs = &at;
-        cfg.numAttrs = 1;
+        cudaLaunchAttribute at[2];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 2;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        at[1].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = at;
+        cfg.numAttrs = 2;
         if (cudaLaunchKernelEx(&cfg, k, p) != cudaSuccess) return BOM_ECUDA;
     } else {
-        k<<<units, NUM_THREADS, C::SMEM, stream>>>(p);
+        launch_k(k, dim3(units), dim3(NUM_THREADS), C::SMEM, stream, p);
     }
     count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
@@ -928,6 +935,7 @@ static int launch_inst(const Params& p, cudaStream_t stream) {
 // the GEMM's linear epilogue.
 __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restrict__ ws, int S, int M, int N,
                                                             const EpiParams e) {
+    pdl_enter();
     if (e.sc != nullptr && e.sc->status != 0) return;
     const int64_t total = static_cast<int64_t>(M) * N;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -1081,7 +1089,7 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     const int64_t total = static_cast<int64_t>(g.M) * g.N;
     int64_t blocks = (total + 255) / 256;
     if (blocks > 8 * device_sm_count()) blocks = 8 * device_sm_count();
-    splitk_reduce_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(g.splitk_ws, p.ksplit, p.M, p.N, g.epi);
+    launch_k(splitk_reduce_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, stream, g.splitk_ws, p.ksplit, p.M, p.N, g.epi);
     count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }

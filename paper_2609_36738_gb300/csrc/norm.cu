@@ -56,6 +56,7 @@ template <typename T, bool VEC8>
 __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const T* __restrict__ x, const T* __restrict__ gamma,
                                                           T* __restrict__ y, float* __restrict__ rstd, int64_t n,
                                                           int64_t d, const DevScalars* sc) {
+    pdl_enter();
     if (sc->status != 0) return;
     const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int l = threadIdx.x & 31;
@@ -102,6 +103,7 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(const T* __restrict__ 
                                                           const T* __restrict__ gamma, const float* __restrict__ rstd,
                                                           const T* __restrict__ pre, T* __restrict__ dx, int64_t n,
                                                           int64_t d, const DevScalars* sc) {
+    pdl_enter();
     if (sc->status != 0) return;
     const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int l = threadIdx.x & 31;
@@ -164,14 +166,14 @@ void launch_rmsnorm_fwd(const void* x, const void* gamma, void* y, float* rstd, 
         auto X = static_cast<const float*>(x);
         auto G = static_cast<const float*>(gamma);
         auto Y = static_cast<float*>(y);
-        if (v8) rmsnorm_fwd_kernel<float, true><<<grid, 256, 0, s>>>(X, G, Y, rstd, n, d, sc);
-        else rmsnorm_fwd_kernel<float, false><<<grid, 256, 0, s>>>(X, G, Y, rstd, n, d, sc);
+        if (v8) launch_k(rmsnorm_fwd_kernel<float, true>, dim3(grid), dim3(256), 0, s, X, G, Y, rstd, n, d, sc);
+        else launch_k(rmsnorm_fwd_kernel<float, false>, dim3(grid), dim3(256), 0, s, X, G, Y, rstd, n, d, sc);
     } else {
         auto X = static_cast<const __nv_bfloat16*>(x);
         auto G = static_cast<const __nv_bfloat16*>(gamma);
         auto Y = static_cast<__nv_bfloat16*>(y);
-        if (v8) rmsnorm_fwd_kernel<__nv_bfloat16, true><<<grid, 256, 0, s>>>(X, G, Y, rstd, n, d, sc);
-        else rmsnorm_fwd_kernel<__nv_bfloat16, false><<<grid, 256, 0, s>>>(X, G, Y, rstd, n, d, sc);
+        if (v8) launch_k(rmsnorm_fwd_kernel<__nv_bfloat16, true>, dim3(grid), dim3(256), 0, s, X, G, Y, rstd, n, d, sc);
+        else launch_k(rmsnorm_fwd_kernel<__nv_bfloat16, false>, dim3(grid), dim3(256), 0, s, X, G, Y, rstd, n, d, sc);
     }
     count_launch();
 }
@@ -186,16 +188,16 @@ void launch_rmsnorm_bwd(const void* dy, const void* x, const void* gamma, const 
         auto g = static_cast<const float*>(gamma);
         auto p = static_cast<const float*>(pre);
         auto o = static_cast<float*>(dx);
-        if (v8) rmsnorm_bwd_kernel<float, true><<<grid, 256, 0, s>>>(a, b, g, rstd, p, o, n, d, sc);
-        else rmsnorm_bwd_kernel<float, false><<<grid, 256, 0, s>>>(a, b, g, rstd, p, o, n, d, sc);
+        if (v8) launch_k(rmsnorm_bwd_kernel<float, true>, dim3(grid), dim3(256), 0, s, a, b, g, rstd, p, o, n, d, sc);
+        else launch_k(rmsnorm_bwd_kernel<float, false>, dim3(grid), dim3(256), 0, s, a, b, g, rstd, p, o, n, d, sc);
     } else {
         auto a = static_cast<const __nv_bfloat16*>(dy);
         auto b = static_cast<const __nv_bfloat16*>(x);
         auto g = static_cast<const __nv_bfloat16*>(gamma);
         auto p = static_cast<const __nv_bfloat16*>(pre);
         auto o = static_cast<__nv_bfloat16*>(dx);
-        if (v8) rmsnorm_bwd_kernel<__nv_bfloat16, true><<<grid, 256, 0, s>>>(a, b, g, rstd, p, o, n, d, sc);
-        else rmsnorm_bwd_kernel<__nv_bfloat16, false><<<grid, 256, 0, s>>>(a, b, g, rstd, p, o, n, d, sc);
+        if (v8) launch_k(rmsnorm_bwd_kernel<__nv_bfloat16, true>, dim3(grid), dim3(256), 0, s, a, b, g, rstd, p, o, n, d, sc);
+        else launch_k(rmsnorm_bwd_kernel<__nv_bfloat16, false>, dim3(grid), dim3(256), 0, s, a, b, g, rstd, p, o, n, d, sc);
     }
     count_launch();
 }

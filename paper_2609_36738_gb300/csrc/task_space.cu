@@ -75,11 +75,13 @@ __device__ float block_sum(float v, float* red) {
 // The step counter advances only after a step that latched no error, so a
 // failed step leaves t, like q, as it was.
 __global__ void advance_step_kernel(int64_t* __restrict__ t, const DevScalars* sc) {
+    pdl_enter();
     if (threadIdx.x == 0 && sc->status == 0) *t += 1;
 }
 
 __global__ void labels_scan_kernel(const int32_t* __restrict__ labels, int64_t n, int64_t V, int32_t ignore,
                                    float lambda, const StepScalarsIn st, DevScalars* sc) {
+    pdl_enter();
     __shared__ int s_cnt[32], s_bad[32];
     int cnt = 0, bad = 0;
     for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
@@ -141,6 +143,7 @@ __global__ void labels_scan_kernel(const int32_t* __restrict__ labels, int64_t n
 // One warp per row.
 __global__ void row_stats_f32_kernel(const float* __restrict__ Z, int64_t ldz, int64_t n, int64_t V,
                                      float2* __restrict__ stats, const DevScalars* sc) {
+    pdl_enter();
     if (sc->status != 0) return;
     const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int l = threadIdx.x & 31;
@@ -158,6 +161,7 @@ __global__ void row_stats_f32_kernel(const float* __restrict__ Z, int64_t ldz, i
 __global__ void row_lse_kernel(const void* __restrict__ Z, int z_f32, int64_t ldz, int64_t n, int64_t V,
                                const float2* __restrict__ stats, int64_t ntiles, const int32_t* __restrict__ labels,
                                int32_t ignore, float* __restrict__ lse, float* __restrict__ ce, const DevScalars* sc) {
+    pdl_enter();
     if (sc->status != 0) return;
     const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int l = threadIdx.x & 31;
@@ -210,6 +214,7 @@ __global__ void __launch_bounds__(256, 3) residual_kernel(T* __restrict__ Z, int
                                                           const float* __restrict__ lse,
                                                           const int32_t* __restrict__ labels, int32_t ignore,
                                                           float* __restrict__ colpart, const DevScalars* sc) {
+    pdl_enter();
     if (sc->status != 0) return;
     const int64_t col0 = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) * VEC;
     const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kResidRows;
@@ -314,6 +319,7 @@ __global__ void __launch_bounds__(256) finish_sq_kernel(const float* __restrict_
                                                         float beta1, float* __restrict__ q,
                                                         float* __restrict__ s_out, float* __restrict__ qhat,
                                                         const DevScalars* sc) {
+    pdl_enter();
     __shared__ float red[8][33];
     if (sc->status != 0) return;
     const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + (threadIdx.x & 31);
@@ -330,6 +336,7 @@ __global__ void __launch_bounds__(256) finish_sq_kernel(const float* __restrict_
 __global__ void __launch_bounds__(1024) scalars_kernel(const float* __restrict__ ce, int64_t n,
                                                        const float* __restrict__ s_vec, int64_t V,
                                                        const float* __restrict__ rnorm, DevScalars* sc) {
+    pdl_enter();
     __shared__ float red[32];
     if (sc->status != 0) return;
     float a = 0.0f;
@@ -355,6 +362,7 @@ __global__ void __launch_bounds__(1024) scalars_kernel(const float* __restrict__
 template <typename T>
 __global__ void __launch_bounds__(256) row_norm_kernel(const T* __restrict__ R, int64_t ldr, int64_t n, int64_t V,
                                                        float* __restrict__ rnorm, const DevScalars* sc) {
+    pdl_enter();
     if (sc->status != 0) return;
     const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int l = threadIdx.x & 31;
@@ -375,6 +383,7 @@ __global__ void __launch_bounds__(256) own_step_moment_kernel(float* __restrict_
                                                               const float* __restrict__ hv, float* __restrict__ mhat,
                                                               int64_t n, float beta1, float inv_bc1,
                                                               double* __restrict__ part) {
+    pdl_enter();
     float s_dot = 0.0f, s_mm = 0.0f, s_hh = 0.0f, s_dd = 0.0f;
     auto one = [&](float& m, float oo, float h, float& mh) {
         m = fmaf(beta1, m, (1.0f - beta1) * oo);
@@ -438,6 +447,7 @@ __global__ void __launch_bounds__(256) own_step_moment_kernel(float* __restrict_
 // sums[k] += sum_b part[4b + k]: warp k, lane l adds blocks l, l + 32, ... in
 // order, then a fixed shuffle tree (the order depends only on nblocks).
 __global__ void drift_finish_kernel(const double* __restrict__ part, int nblocks, double* __restrict__ sums) {
+    pdl_enter();
     const int k = threadIdx.x >> 5, l = threadIdx.x & 31;
     double acc = 0.0;
     for (int b = l; b < nblocks; b += 32) acc += part[4 * static_cast<int64_t>(b) + k];
@@ -471,6 +481,7 @@ __global__ void __launch_bounds__(256, 3) colsum_part_kernel(const T* __restrict
                                                              int64_t d, const int32_t* __restrict__ labels,
                                                              int32_t ignore, const float* __restrict__ wvec,
                                                              float* __restrict__ part, const DevScalars* sc) {
+    pdl_enter();
     constexpr int VEC = 16 / sizeof(T);
     // rows in flight per warp step: 8 words per thread (4 of X and 4 of Y)
     constexpr int U = HAS_Y ? 4 : 8;
@@ -553,6 +564,7 @@ __global__ void __launch_bounds__(256, 3) colsum_part_kernel(const T* __restrict
 __global__ void __launch_bounds__(256) colsum_finish_kernel(const float* __restrict__ part, int64_t nblocks,
                                                             int64_t d, float scale, void* __restrict__ out,
                                                             int out_f32, const DevScalars* sc) {
+    pdl_enter();
     __shared__ float red[8][33];
     if (sc->status != 0) return;
     const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + (threadIdx.x & 31);
@@ -562,6 +574,7 @@ __global__ void __launch_bounds__(256) colsum_finish_kernel(const float* __restr
 
 __global__ void axpby_kernel(const float* __restrict__ s, const float* __restrict__ qh, float a, float b, int64_t V,
                              void* __restrict__ out, int out_f32, const DevScalars* sc) {
+    pdl_enter();
     if (sc->status != 0) return;
     const int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (j >= V) return;
@@ -574,22 +587,22 @@ inline unsigned cdiv(int64_t a, int64_t b) { return static_cast<unsigned>((a + b
 
 void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda,
                         const StepScalarsIn& st, DevScalars* sc, cudaStream_t s) {
-    labels_scan_kernel<<<1, 1024, 0, s>>>(labels, n, V, ignore, lambda, st, sc); count_launch();
+    launch_k(labels_scan_kernel, dim3(1), dim3(1024), 0, s, labels, n, V, ignore, lambda, st, sc); count_launch();
 }
 
 void launch_advance_step(int64_t* t_dev, const DevScalars* sc, cudaStream_t s) {
-    advance_step_kernel<<<1, 32, 0, s>>>(t_dev, sc); count_launch();
+    launch_k(advance_step_kernel, dim3(1), dim3(32), 0, s, t_dev, sc); count_launch();
 }
 
 void launch_row_stats_f32(const float* Z, int64_t ldz, int64_t n, int64_t V, float* stats, const DevScalars* sc,
                           cudaStream_t s) {
-    row_stats_f32_kernel<<<cdiv(n * 32, 256), 256, 0, s>>>(Z, ldz, n, V, reinterpret_cast<float2*>(stats), sc); count_launch();
+    launch_k(row_stats_f32_kernel, dim3(cdiv(n * 32, 256)), dim3(256), 0, s, Z, ldz, n, V, reinterpret_cast<float2*>(stats), sc); count_launch();
 }
 
 void launch_row_lse(const void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* stats, int64_t ntiles,
                     const int32_t* labels, int32_t ignore, float* lse, float* ce, const DevScalars* sc,
                     cudaStream_t s) {
-    row_lse_kernel<<<cdiv(n * 32, 256), 256, 0, s>>>(Z, z_f32, ldz, n, V, reinterpret_cast<const float2*>(stats),
+    launch_k(row_lse_kernel, dim3(cdiv(n * 32, 256)), dim3(256), 0, s, Z, z_f32, ldz, n, V, reinterpret_cast<const float2*>(stats),
                                                       ntiles, labels, ignore, lse, ce, sc); count_launch();
 }
 
@@ -597,32 +610,32 @@ void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, cons
                      int32_t ignore, float* colpart, const DevScalars* sc, cudaStream_t s) {
     if (z_f32) {
         dim3 grid(cdiv(ldz, 256 * 4), static_cast<unsigned>(resid_blocks(n)));
-        residual_kernel<float, 4><<<grid, 256, 0, s>>>(static_cast<float*>(Z), ldz, n, V, lse, labels, ignore,
+        launch_k(residual_kernel<float, 4>, dim3(grid), dim3(256), 0, s, static_cast<float*>(Z), ldz, n, V, lse, labels, ignore,
                                                        colpart, sc); count_launch();
     } else {
         dim3 grid(cdiv(ldz, 256 * 8), static_cast<unsigned>(resid_blocks(n)));
-        residual_kernel<__nv_bfloat16, 8><<<grid, 256, 0, s>>>(static_cast<__nv_bfloat16*>(Z), ldz, n, V, lse,
+        launch_k(residual_kernel<__nv_bfloat16, 8>, dim3(grid), dim3(256), 0, s, static_cast<__nv_bfloat16*>(Z), ldz, n, V, lse,
                                                                labels, ignore, colpart, sc); count_launch();
     }
 }
 
 void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float* q,
                       float* s_out, float* qhat, DevScalars* sc, cudaStream_t s) {
-    finish_sq_kernel<<<cdiv(V, 32), 256, 0, s>>>(colpart, nblocks, V, beta1, q, s_out, qhat, sc); count_launch();
+    launch_k(finish_sq_kernel, dim3(cdiv(V, 32)), dim3(256), 0, s, colpart, nblocks, V, beta1, q, s_out, qhat, sc); count_launch();
 }
 
 void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, const float* rnorm, DevScalars* sc,
                     cudaStream_t s) {
-    scalars_kernel<<<1, 1024, 0, s>>>(ce, n, s_vec, V, rnorm, sc); count_launch();
+    launch_k(scalars_kernel, dim3(1), dim3(1024), 0, s, ce, n, s_vec, V, rnorm, sc); count_launch();
 }
 
 void launch_row_norm(const void* R, int r_f32, int64_t ldr, int64_t n, int64_t V, float* rnorm, const DevScalars* sc,
                      cudaStream_t s) {
     const unsigned grid = static_cast<unsigned>(cdiv(n * 32, 256));
     if (r_f32)
-        row_norm_kernel<float><<<grid, 256, 0, s>>>(static_cast<const float*>(R), ldr, n, V, rnorm, sc);
+        launch_k(row_norm_kernel<float>, dim3(grid), dim3(256), 0, s, static_cast<const float*>(R), ldr, n, V, rnorm, sc);
     else
-        row_norm_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(R), ldr, n, V, rnorm,
+        launch_k(row_norm_kernel<__nv_bfloat16>, dim3(grid), dim3(256), 0, s, static_cast<const __nv_bfloat16*>(R), ldr, n, V, rnorm,
                                                              sc);
     count_launch();
 }
@@ -636,10 +649,10 @@ int own_step_blocks(int64_t n, int sms) {
 
 void launch_own_step_moment(float* M, const float* o, const float* hv, float* mhat, int64_t n, float beta1,
                             float inv_bc1, double* part, int nblocks, double* sums, cudaStream_t s) {
-    own_step_moment_kernel<<<nblocks, 256, 0, s>>>(M, o, hv, mhat, n, beta1, inv_bc1, sums ? part : nullptr);
+    launch_k(own_step_moment_kernel, dim3(nblocks), dim3(256), 0, s, M, o, hv, mhat, n, beta1, inv_bc1, sums ? part : nullptr);
     count_launch();
     if (sums) {
-        drift_finish_kernel<<<1, 128, 0, s>>>(part, nblocks, sums);
+        launch_k(drift_finish_kernel, dim3(1), dim3(128), 0, s, part, nblocks, sums);
         count_launch();
     }
 }
@@ -673,28 +686,28 @@ void launch_colsum2(const void* X, const void* Y, int x_f32, int64_t ldx, int64_
         auto x = static_cast<const float*>(X);
         auto y = static_cast<const float*>(Y);
         if (Y)
-            colsum_part_kernel<float, true><<<grid, 256, 0, s>>>(x, y, ldx, n, rows_per, d, labels, ignore, wvec,
+            launch_k(colsum_part_kernel<float, true>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels, ignore, wvec,
                                                                  part, sc);
         else
-            colsum_part_kernel<float, false><<<grid, 256, 0, s>>>(x, y, ldx, n, rows_per, d, labels, ignore, wvec,
+            launch_k(colsum_part_kernel<float, false>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels, ignore, wvec,
                                                                   part, sc);
     } else {
         auto x = static_cast<const __nv_bfloat16*>(X);
         auto y = static_cast<const __nv_bfloat16*>(Y);
         if (Y)
-            colsum_part_kernel<__nv_bfloat16, true><<<grid, 256, 0, s>>>(x, y, ldx, n, rows_per, d, labels, ignore,
+            launch_k(colsum_part_kernel<__nv_bfloat16, true>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels, ignore,
                                                                          wvec, part, sc);
         else
-            colsum_part_kernel<__nv_bfloat16, false><<<grid, 256, 0, s>>>(x, y, ldx, n, rows_per, d, labels, ignore,
+            launch_k(colsum_part_kernel<__nv_bfloat16, false>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels, ignore,
                                                                           wvec, part, sc);
     }
     count_launch();
-    colsum_finish_kernel<<<cdiv(d, 32), 256, 0, s>>>(part, nb, d, scale, out, out_f32, sc); count_launch();
+    launch_k(colsum_finish_kernel, dim3(cdiv(d, 32)), dim3(256), 0, s, part, nb, d, scale, out, out_f32, sc); count_launch();
 }
 
 void launch_axpby(const float* s_vec, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
                   const DevScalars* sc, cudaStream_t s) {
-    axpby_kernel<<<cdiv(V, 256), 256, 0, s>>>(s_vec, qhat, a, b, V, out, out_f32, sc); count_launch();
+    launch_k(axpby_kernel, dim3(cdiv(V, 256)), dim3(256), 0, s, s_vec, qhat, a, b, V, out, out_f32, sc); count_launch();
 }
 
 }  // namespace bom

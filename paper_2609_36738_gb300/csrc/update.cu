@@ -60,6 +60,7 @@ __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ theta, 
                                                      uint16_t* __restrict__ shadow, int64_t n, UpdCoef c_in,
                                                      const double* __restrict__ clip_sq, float max_norm,
                                                      const DevScalars* sc) {
+    pdl_enter();
     if (sc != nullptr && sc->status != 0) return;   // inside a step that latched an error
     const UpdCoef c = resolve_coef(c_in, sc);
     const float cs = CLIP ? clip_scale(clip_sq, max_norm) : 1.0f;
@@ -173,6 +174,7 @@ __global__ void __launch_bounds__(256) update_blockshared_cluster_kernel(float* 
                                                                          float* __restrict__ vb,
                                                                          uint16_t* __restrict__ shadow, int64_t n,
                                                                          int64_t block, UpdCoef c_in) {
+    pdl_enter();
     __shared__ float red[8];
     __shared__ float s_part;   // this CTA's sum of u^2 over its share of the block
     __shared__ float s_den;    // leading CTA: the block's denominator
@@ -267,6 +269,7 @@ template <bool G_BF16, bool HAS_H, int VEC>
 __global__ void __launch_bounds__(256) bs_chunk_sq_kernel(const void* __restrict__ g, const float* __restrict__ h,
                                                           float lam, int64_t n, int64_t block, int64_t ch, int64_t S,
                                                           int64_t nchunks, float* __restrict__ part) {
+    pdl_enter();
     __shared__ float red[8];
     for (int64_t cidx = blockIdx.x; cidx < nchunks; cidx += gridDim.x) {
         const int64_t b = cidx / S, j = cidx - b * S;
@@ -307,6 +310,7 @@ __global__ void __launch_bounds__(256) bs_chunk_sq_kernel(const void* __restrict
 __global__ void __launch_bounds__(256) bs_finish_kernel(const float* __restrict__ part, int64_t S, int64_t nb,
                                                         int64_t n, int64_t block, float* __restrict__ vb,
                                                         float* __restrict__ den, UpdCoef c_in) {
+    pdl_enter();
     const UpdCoef c = resolve_coef(c_in, nullptr);
     const int64_t b = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
@@ -327,6 +331,7 @@ __global__ void __launch_bounds__(256) bs_apply_kernel(float* __restrict__ theta
                                                        const float* __restrict__ h, uint16_t* __restrict__ shadow,
                                                        int64_t n, int64_t block, const float* __restrict__ den,
                                                        UpdCoef c_in) {
+    pdl_enter();
     const UpdCoef c = resolve_coef(c_in, nullptr);
     const int64_t nv = n / VEC;   // VEC = 4 only when n and block are multiples of 4
     const int64_t stride = static_cast<int64_t>(gridDim.x) * 256;
@@ -361,6 +366,7 @@ __global__ void __launch_bounds__(256) update_blockshared_kernel(float* __restri
                                                                  const float* __restrict__ h, float* __restrict__ vb,
                                                                  uint16_t* __restrict__ shadow, int64_t n,
                                                                  int64_t block, UpdCoef c_in) {
+    pdl_enter();
     __shared__ float red[8];
     __shared__ float s_den;
     const UpdCoef c = resolve_coef(c_in, nullptr);
@@ -539,6 +545,7 @@ __global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __re
                                                                      float* __restrict__ vb,
                                                                      uint16_t* __restrict__ shadow, int64_t n,
                                                                      int64_t block, UpdCoef c_in) {
+    pdl_enter();
     __shared__ float red[8];
     __shared__ float s_den;
     const UpdCoef c = resolve_coef(c_in, nullptr);
@@ -582,7 +589,7 @@ template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT>
 void launch_reg(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n, int64_t block,
                 const UpdCoef& c, cudaStream_t s) {
     auto k = update_blockshared_reg_kernel<G_BF16, HAS_H, SHADOW, WPT>;
-    k<<<resident_grid(k, (n + block - 1) / block), 256, 0, s>>>(theta, g, h, vb, shadow, n, block, c);
+    launch_k(k, dim3(resident_grid(k, (n + block - 1) / block)), dim3(256), 0, s, theta, g, h, vb, shadow, n, block, c);
 }
 
 template <bool G_BF16, bool HAS_H, bool SHADOW>
@@ -594,16 +601,19 @@ void launch_reg_wpt(float* theta, const void* g, const float* h, float* vb, uint
     else launch_reg<G_BF16, HAS_H, SHADOW, 8>(theta, g, h, vb, shadow, n, block, c, s);
 }
 
+// Launch shape of the cluster kernel; at[] must hold two attributes.
 template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
 cudaLaunchConfig_t cluster_cfg(cudaLaunchAttribute* at) {
     cudaLaunchConfig_t cfg = {};
-    at->id = cudaLaunchAttributeClusterDimension;
-    at->val.clusterDim.x = kBlockCluster;
-    at->val.clusterDim.y = 1;
-    at->val.clusterDim.z = 1;
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = kBlockCluster;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.blockDim = dim3(256);
     cfg.attrs = at;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cfg;
 }
 
@@ -612,8 +622,8 @@ template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
 int cluster_slots() {
     static int slots = 0;
     if (slots == 0) {
-        cudaLaunchAttribute at;
-        cudaLaunchConfig_t cfg = cluster_cfg<G_BF16, HAS_H, SHADOW, VEC>(&at);
+        cudaLaunchAttribute at[2];
+        cudaLaunchConfig_t cfg = cluster_cfg<G_BF16, HAS_H, SHADOW, VEC>(at);
         cfg.gridDim = dim3(static_cast<unsigned>(device_sm_count() / kBlockCluster * kBlockCluster));
         int m = 0;
         if (cudaOccupancyMaxActiveClusters(&m, update_blockshared_cluster_kernel<G_BF16, HAS_H, SHADOW, VEC>, &cfg) !=
@@ -630,8 +640,8 @@ int cluster_slots() {
 template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
 int launch_cluster(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
                    int64_t block, const UpdCoef& c, int64_t nclusters, cudaStream_t s) {
-    cudaLaunchAttribute at;
-    cudaLaunchConfig_t cfg = cluster_cfg<G_BF16, HAS_H, SHADOW, VEC>(&at);
+    cudaLaunchAttribute at[2];
+    cudaLaunchConfig_t cfg = cluster_cfg<G_BF16, HAS_H, SHADOW, VEC>(at);
     cfg.gridDim = dim3(static_cast<unsigned>(nclusters * kBlockCluster));
     cfg.stream = s;
     cudaLaunchKernelEx(&cfg, update_blockshared_cluster_kernel<G_BF16, HAS_H, SHADOW, VEC>, theta, g, h, vb, shadow,
@@ -692,16 +702,16 @@ int launch_grid_blocks(float* theta, const void* g, const float* h, float* vb, u
     float* part = scr;
     float* den = scr + nchunks;
     const int64_t g1 = nchunks < G ? nchunks : G;
-    bs_chunk_sq_kernel<G_BF16, HAS_H, VEC><<<static_cast<unsigned>(g1), 256, 0, s>>>(g, h, c.lam, n, block, ch, S,
+    launch_k(bs_chunk_sq_kernel<G_BF16, HAS_H, VEC>, dim3(static_cast<unsigned>(g1)), dim3(256), 0, s, g, h, c.lam, n, block, ch, S,
                                                                                     nchunks, part);
     count_launch();
-    bs_finish_kernel<<<static_cast<unsigned>((nb + 7) / 8), 256, 0, s>>>(part, S, nb, n, block, vb, den, c);
+    launch_k(bs_finish_kernel, dim3(static_cast<unsigned>((nb + 7) / 8)), dim3(256), 0, s, part, S, nb, n, block, vb, den, c);
     count_launch();
     const int64_t need = (n / VEC + 255) / 256;
     int64_t g3 = 8 * static_cast<int64_t>(device_sm_count());
     if (g3 > need) g3 = need;
     if (g3 < 1) g3 = 1;
-    bs_apply_kernel<G_BF16, HAS_H, SHADOW, VEC><<<static_cast<unsigned>(g3), 256, 0, s>>>(theta, g, h, shadow, n,
+    launch_k(bs_apply_kernel<G_BF16, HAS_H, SHADOW, VEC>, dim3(static_cast<unsigned>(g3)), dim3(256), 0, s, theta, g, h, shadow, n,
                                                                                           block, den, c);
     count_launch();
     cudaFreeAsync(scr, s);
@@ -730,9 +740,9 @@ int dispatch_blockshared(float* theta, const void* g, const float* h, float* vb,
         if (shadow) launch_reg_wpt<G_BF16, HAS_H, true>(theta, g, h, vb, shadow, n, block, c, s);
         else launch_reg_wpt<G_BF16, HAS_H, false>(theta, g, h, vb, shadow, n, block, c, s);
     } else if (shadow) {
-        update_blockshared_kernel<G_BF16, HAS_H, true, VEC><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n, block, c);
+        launch_k(update_blockshared_kernel<G_BF16, HAS_H, true, VEC>, dim3(grid), dim3(256), 0, s, theta, g, h, vb, shadow, n, block, c);
     } else {
-        update_blockshared_kernel<G_BF16, HAS_H, false, VEC><<<grid, 256, 0, s>>>(theta, g, h, vb, shadow, n, block,
+        launch_k(update_blockshared_kernel<G_BF16, HAS_H, false, VEC>, dim3(grid), dim3(256), 0, s, theta, g, h, vb, shadow, n, block,
                                                                                   c);
     }
     count_launch();
@@ -745,17 +755,17 @@ void dispatch_shadow(float* theta, const void* g, const float* h, float* v, uint
                      cudaStream_t s) {
     if (clip_sq) {
         if (shadow)
-            update_kernel<G_BF16, HAS_H, true, true><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, clip_sq,
+            launch_k(update_kernel<G_BF16, HAS_H, true, true>, dim3(grid), dim3(256), 0, s, theta, g, h, v, shadow, n, c, clip_sq,
                                                                           max_norm, sc);
         else
-            update_kernel<G_BF16, HAS_H, false, true><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, clip_sq,
+            launch_k(update_kernel<G_BF16, HAS_H, false, true>, dim3(grid), dim3(256), 0, s, theta, g, h, v, shadow, n, c, clip_sq,
                                                                            max_norm, sc);
     } else {
         if (shadow)
-            update_kernel<G_BF16, HAS_H, true, false><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, nullptr,
+            launch_k(update_kernel<G_BF16, HAS_H, true, false>, dim3(grid), dim3(256), 0, s, theta, g, h, v, shadow, n, c, nullptr,
                                                                            0.0f, sc);
         else
-            update_kernel<G_BF16, HAS_H, false, false><<<grid, 256, 0, s>>>(theta, g, h, v, shadow, n, c, nullptr,
+            launch_k(update_kernel<G_BF16, HAS_H, false, false>, dim3(grid), dim3(256), 0, s, theta, g, h, v, shadow, n, c, nullptr,
                                                                             0.0f, sc);
     }
     count_launch();
@@ -766,6 +776,7 @@ void dispatch_shadow(float* theta, const void* g, const float* h, float* v, uint
 template <bool G_BF16, bool HAS_H>
 __global__ void __launch_bounds__(256) sqnorm_part_kernel(const void* __restrict__ g, const float* __restrict__ h,
                                                           float lam, int64_t n, double* __restrict__ part) {
+    pdl_enter();
     float acc = 0.0f;
     const int64_t n4 = n >> 2;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -794,6 +805,7 @@ __global__ void __launch_bounds__(256) sqnorm_part_kernel(const void* __restrict
 // *sq += sum_b part[b]: lane l adds blocks l, l + 32, ... in order, then a
 // fixed shuffle tree (the order depends only on nblocks: deterministic).
 __global__ void sqnorm_finish_kernel(const double* __restrict__ part, int nblocks, double* __restrict__ sq) {
+    pdl_enter();
     const int l = threadIdx.x & 31;
     double t = 0.0;
     for (int b = l; b < nblocks; b += 32) t += part[b];
@@ -846,14 +858,14 @@ int launch_sqnorm(const void* g, int g_bf16, const float* h, float lambda, int64
     if (n <= 0) return BOM_OK;
     const int nb = sqnorm_blocks(n);
     if (g_bf16) {
-        if (h) sqnorm_part_kernel<true, true><<<nb, 256, 0, s>>>(g, h, lambda, n, part);
-        else sqnorm_part_kernel<true, false><<<nb, 256, 0, s>>>(g, h, lambda, n, part);
+        if (h) launch_k(sqnorm_part_kernel<true, true>, dim3(nb), dim3(256), 0, s, g, h, lambda, n, part);
+        else launch_k(sqnorm_part_kernel<true, false>, dim3(nb), dim3(256), 0, s, g, h, lambda, n, part);
     } else {
-        if (h) sqnorm_part_kernel<false, true><<<nb, 256, 0, s>>>(g, h, lambda, n, part);
-        else sqnorm_part_kernel<false, false><<<nb, 256, 0, s>>>(g, h, lambda, n, part);
+        if (h) launch_k(sqnorm_part_kernel<false, true>, dim3(nb), dim3(256), 0, s, g, h, lambda, n, part);
+        else launch_k(sqnorm_part_kernel<false, false>, dim3(nb), dim3(256), 0, s, g, h, lambda, n, part);
     }
     count_launch();
-    sqnorm_finish_kernel<<<1, 32, 0, s>>>(part, nb, sq);
+    launch_k(sqnorm_finish_kernel, dim3(1), dim3(32), 0, s, part, nb, sq);
     count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }
