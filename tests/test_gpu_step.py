@@ -4,6 +4,8 @@ by element, on the same seeded inputs.
 Tolerances (relative L2): 1e-5 for the fp32 path, 2e-2 for bf16 paths; label
 handling (N_t) bit-exact.  Workloads span several GEMM tiles with ragged
 tails, ignored rows, every layer kind, and both output modes."""
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -172,3 +174,38 @@ def test_input_cotangent(name):
     assert G.rel_l2(G.np64(dx), oref["dX_u"]) < tol
     for u, ref in zip(gout["grads"], oref["u"]):
         assert G.rel_l2(G.np64(u), ref) < tol
+
+
+# A Qwen3-sized vocabulary on a small ragged batch: 151,936 columns give 1187
+# column half-tiles per row to merge in the row log-sum-exp and a ragged last
+# tile; the head's input-side GEMM contracts over all of them (split-K).
+LM_HEAD_HUGE_V = dataclasses.replace(I.LM_HEAD_SMALL, name="lm_head_huge_vocab", n_rows=97, vocab=151_936)
+
+
+@pytest.mark.parametrize("mode", [B.BOM_OUT_U, B.BOM_OUT_G_AND_H])
+def test_huge_vocabulary_parity(mode):
+    wl = LM_HEAD_HUGE_V
+    params = I.init_params(wl, seed=2)
+    p64 = X.params_f64(wl, params)
+    x, y = I.make_batch(wl, seed=2, step=1)
+    gpu = G.GpuBom(wl, params, out_mode=mode)
+    gout = gpu.step(x, y, 1)
+    oref = G.oracle_step(wl, p64, x, y, np.zeros(wl.vocab), 1)
+    _compare_step(wl, gout, oref, G.TOL[wl.dtype], mode == B.BOM_OUT_G_AND_H)
+
+
+@pytest.mark.parametrize("name", ["tiny_mlp_f32", "lm_mlp_small"])
+def test_single_supervised_row(name):
+    """N_t = 1: every label but one is the ignore index, so s_t is that row's
+    residual and every mean is over one row."""
+    wl = I.WORKLOADS[name]
+    params = I.init_params(wl, seed=3)
+    p64 = X.params_f64(wl, params)
+    x, y = I.make_batch(wl, seed=3, step=1)
+    y = np.full_like(y, I.IGNORE_INDEX)
+    y[wl.n_rows // 2] = 5
+    gpu = G.GpuBom(wl, params)
+    gout = gpu.step(x, y, 2)
+    oref = G.oracle_step(wl, p64, x, y, np.zeros(wl.vocab), 2)
+    assert gout["stats"]["n_t"] == 1
+    _compare_step(wl, gout, oref, G.TOL[wl.dtype], False)
