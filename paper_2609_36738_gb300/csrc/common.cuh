@@ -304,9 +304,41 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&h);
 }
 
+// 32 bytes to a 32-byte aligned global address in one 256-bit store.
+__device__ __forceinline__ void st_global_v8(void* p, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t a4,
+                                             uint32_t a5, uint32_t a6, uint32_t a7) {
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(a0), "r"(a1), "r"(a2),
+                 "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7)
+                 : "memory");
+}
+
+// One lane writes 32 values of its row.  A full chunk at a 32-byte aligned
+// address leaves in 256-bit stores: each covers a whole 32-byte sector, so a
+// row-per-lane store instruction makes half as many sector writes.
 __device__ __forceinline__ void store_row32(void* base, int64_t row_off, int n, int N, int is_f32,
                                             const float (&v)[32]) {
     if (n + 32 <= N) {
+        char* q = static_cast<char*>(base) + (row_off + n) * (is_f32 ? 4 : 2);
+        if ((reinterpret_cast<uintptr_t>(q) & 31u) == 0) {
+            if (is_f32) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    st_global_v8(q + 32 * i, __float_as_uint(v[8 * i]), __float_as_uint(v[8 * i + 1]),
+                                 __float_as_uint(v[8 * i + 2]), __float_as_uint(v[8 * i + 3]),
+                                 __float_as_uint(v[8 * i + 4]), __float_as_uint(v[8 * i + 5]),
+                                 __float_as_uint(v[8 * i + 6]), __float_as_uint(v[8 * i + 7]));
+            } else {
+#pragma unroll
+                for (int i = 0; i < 2; ++i)
+                    st_global_v8(q + 32 * i, pack_bf16x2(v[16 * i], v[16 * i + 1]),
+                                 pack_bf16x2(v[16 * i + 2], v[16 * i + 3]), pack_bf16x2(v[16 * i + 4], v[16 * i + 5]),
+                                 pack_bf16x2(v[16 * i + 6], v[16 * i + 7]), pack_bf16x2(v[16 * i + 8], v[16 * i + 9]),
+                                 pack_bf16x2(v[16 * i + 10], v[16 * i + 11]),
+                                 pack_bf16x2(v[16 * i + 12], v[16 * i + 13]),
+                                 pack_bf16x2(v[16 * i + 14], v[16 * i + 15]));
+            }
+            return;
+        }
         if (is_f32) {
             float4* p = reinterpret_cast<float4*>(static_cast<float*>(base) + row_off + n);
 #pragma unroll

@@ -118,7 +118,18 @@ template <int NW>
 __device__ __forceinline__ void load_chunk_bf16(const void* base, int64_t row_off, int n, int N, uint4 (&pk)[NW],
                                                 int slot) {
     const uint16_t* p = static_cast<const uint16_t*>(base) + row_off + n;
-    if (n + 32 <= N) {
+    if (n + 32 <= N && (reinterpret_cast<uintptr_t>(p) & 31u) == 0) {
+        // two whole 32-byte sectors in 256-bit loads
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            uint4 a, b;
+            asm("ld.global.nc.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                         : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w), "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w)
+                         : "l"(p + 16 * i));
+            pk[4 * slot + 2 * i] = a;
+            pk[4 * slot + 2 * i + 1] = b;
+        }
+    } else if (n + 32 <= N) {
 #pragma unroll
         for (int i = 0; i < 4; ++i) pk[4 * slot + i] = __ldg(reinterpret_cast<const uint4*>(p) + i);
     } else {
@@ -150,62 +161,6 @@ __device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[NW], int slot, fl
             v[8 * i + 2 * j + 1] = __uint_as_float(ws[j] & 0xFFFF0000u);
         }
     }
-}
-
-// ---------------------------------------------------------------- staged epilogue I/O
-// A warp owns 32 consecutive output rows (one per lane).  Writing "its row"
-// directly makes every warp instruction touch 32 different rows; instead a
-// 32 x 32 bf16 block goes through a per-warp shared-memory buffer: lane l
-// writes row l there, then the warp stores 8 rows per instruction, lane l
-// covering row (l % 8) + 8i and 16-byte segment l / 8, so each row's 64 bytes
-// leave in one coalesced access.  With the 80-byte row pitch (64 data + 16
-// pad) both the row-per-lane writes and the segment reads hit eight distinct
-// 4-bank groups per quarter-warp phase: no bank conflicts.
-constexpr int kStgPitch = 80;
-constexpr int kStgBytes = 32 * kStgPitch;
-
-// Stores the staged block (rows row0.., columns n..n+31) to global memory.
-__device__ __forceinline__ void stg_flush(void* base, int64_t ld, int row0, int M, int n, int N, const uint8_t* stg) {
-    const int lane = threadIdx.x & 31;
-    const int seg = lane >> 3;
-    const int c = n + 8 * seg;
-    __syncwarp();
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int rl = (lane & 7) + 8 * i;
-        const int r = row0 + rl;
-        const uint4 x = *reinterpret_cast<const uint4*>(stg + rl * kStgPitch + seg * 16);
-        uint16_t* p = static_cast<uint16_t*>(base) + static_cast<int64_t>(r) * ld + c;
-        if (r < M) {
-            if (c + 8 <= N) {
-                *reinterpret_cast<uint4*>(p) = x;
-            } else {
-                const uint32_t ws[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-                for (int k = 0; k < 8; ++k)
-                    if (c + k < N) p[k] = static_cast<uint16_t>(ws[k >> 1] >> (16 * (k & 1)));
-            }
-        }
-    }
-    __syncwarp();
-}
-// Lane l contributes row l of a 32 x 32 block as 16 packed bf16 pairs.
-__device__ __forceinline__ void stg_scatter_bf16(void* base, int64_t ld, int row0, int M, int n, int N, uint8_t* stg,
-                                                 const uint32_t (&b)[16]) {
-    const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-        *reinterpret_cast<uint4*>(stg + lane * kStgPitch + k * 16) =
-            make_uint4(b[4 * k], b[4 * k + 1], b[4 * k + 2], b[4 * k + 3]);
-    stg_flush(base, ld, row0, M, n, N, stg);
-}
-// Lane l contributes row l of a 32 x 32 block as fp32 values, stored as bf16.
-__device__ __forceinline__ void stg_scatter(void* base, int64_t ld, int row0, int M, int n, int N, uint8_t* stg,
-                                            const float (&v)[32]) {
-    uint32_t b[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) b[i] = cvt_bf16x2(v[2 * i], v[2 * i + 1]);
-    stg_scatter_bf16(base, ld, row0, M, n, N, stg, b);
 }
 
 // Fused update through shared memory: lane l holds u of row l of a 32 x 32
@@ -267,9 +222,11 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
 // Shared-memory layout of one CTA.  CG = 1: the CTA computes 128 x 256 tiles
 // alone.  CG = 2: a CTA pair (cluster of 2) computes 256 x 256 tiles with
 // tcgen05 cta_group::2 UMMAs issued by the even CTA; each CTA stages its own
-// 128 rows of A and its half (128 rows) of B, so a stage is 32 KB.  Epilogues
-// that move several bf16 streams (logits, SwiGLU) take NBUF staging blocks per
-// epilogue warp and give up pipeline stages for them.
+// 128 rows of A and its half (128 rows) of B, so a stage is 32 KB.  Epilogue
+// stores go straight from each lane's row to global memory in 256-bit stores
+// (whole 32-byte sectors); staging them through shared memory cost pipeline
+// stages and measured slower.  The fused update stages its accumulator chunk
+// (a per-warp block) to walk theta and v by columns.
 // SwiGLU backward: the epilogue's per-row operands (the saved G and U) arrive
 // by TMA.  Each epilogue warp owns two slots of a 32-row x 32-column block of
 // G and of U (2 KB each, 64-byte swizzle: chunk k of row r at
@@ -279,19 +236,12 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
 constexpr int kEpiLdBlock = 32 * 64;
 constexpr int kEpiLdWarpBytes = 2 * 2 * kEpiLdBlock;
 
-// Logits epilogue with its output staged through shared memory (chosen when
-// the contraction is short and the epilogue, not the mainloop, sets the pace).
-constexpr int EPI_LOGITS_STG = 16;
-
 template <int CG, int EPI>
 struct Cfg {
-    static constexpr int NBUF = EPI == EPI_SWIGLU_FWD ? 3 : EPI == EPI_LOGITS_STG ? 1 : 0;
     static constexpr int B_ROWS = CG == 2 ? 128 : 256;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
-    static constexpr int STG_BYTES = EPI == EPI_UPDATE ? 8 * kUpdStgBytes
-                                     : EPI == EPI_SWIGLU_BWD ? 8 * kEpiLdWarpBytes
-                                                             : 8 * NBUF * kStgBytes;
+    static constexpr int STG_BYTES = EPI == EPI_UPDATE ? 8 * kUpdStgBytes : EPI == EPI_SWIGLU_BWD ? 8 * kEpiLdWarpBytes : 0;
     static constexpr int BAR_BYTES = 512;
     // as many stages as fit in the 227 KB a CTA may use beside the staging
     // blocks, the 1 KB alignment slack and the barrier block, at most six (a
@@ -554,7 +504,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t ra = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid);
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
-            uint8_t* stg = stg_all + (warp - 2) * (EPI == EPI_UPDATE ? kUpdStgBytes : C::NBUF * kStgBytes);
+            uint8_t* stg = stg_all + (warp - 2) * (EPI == EPI_UPDATE ? kUpdStgBytes : 0);
             if (EPI == EPI_SWIGLU_BWD) {
                 // the first two blocks of this warp's part of the tile
                 if (lane == 0)
@@ -647,7 +597,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     }
                     staged_update32(e, reinterpret_cast<float*>(stg), row0, PM, n, PN, v, lr, decay, inv_bc2);
                 }
-            } else if constexpr (EPI == EPI_LOGITS || EPI == EPI_LOGITS_STG) {
+            } else if constexpr (EPI == EPI_LOGITS) {
                 // per (row, column half) softmax statistics: stats pair nt*2 + h.
                 // The statistics are taken over the bf16-rounded logits that
                 // are stored, so the residual pass sees a consistent row.
@@ -669,14 +619,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         uint32_t b[16];
 #pragma unroll
                         for (int i = 0; i < 16; ++i) b[i] = cvt_bf16x2(v[2 * i], v[2 * i + 1]);
-                        if constexpr (EPI == EPI_LOGITS_STG)
-                            stg_scatter_bf16(e.out, e.ld_out, row0, PM, n, PN, stg, b);
-                        else if (valid) {
-                            uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(e.out) +
-                                                                  static_cast<int64_t>(m) * e.ld_out + n);
+                        if (valid) {
+                            uint16_t* dst16 = static_cast<uint16_t*>(e.out) + static_cast<int64_t>(m) * e.ld_out + n;
+                            if ((reinterpret_cast<uintptr_t>(dst16) & 31u) == 0) {   // two whole-sector stores
+                                st_global_v8(dst16, b[0], b[1], b[2], b[3], b[4], b[5], b[6], b[7]);
+                                st_global_v8(dst16 + 16, b[8], b[9], b[10], b[11], b[12], b[13], b[14], b[15]);
+                            } else {
+                                uint4* dst = reinterpret_cast<uint4*>(dst16);
 #pragma unroll
-                            for (int i = 0; i < 4; ++i)
-                                dst[i] = make_uint4(b[4 * i], b[4 * i + 1], b[4 * i + 2], b[4 * i + 3]);
+                                for (int i = 0; i < 4; ++i)
+                                    dst[i] = make_uint4(b[4 * i], b[4 * i + 1], b[4 * i + 2], b[4 * i + 3]);
+                            }
                         }
                         uint32_t mb[8];
 #pragma unroll
@@ -704,10 +657,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     // ragged last chunk
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = round_bf16(v[i]);
-                    if constexpr (EPI == EPI_LOGITS_STG)
-                        stg_scatter(e.out, e.ld_out, row0, PM, n, PN, stg, v);
-                    else if (valid)
-                        store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, PN, 0, v);
+                    if (valid) store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, PN, 0, v);
                     float cm = -INFINITY;
 #pragma unroll
                     for (int i = 0; i < 32; ++i)
@@ -734,8 +684,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     if (n >= PN) break;
                     tmem_load32(tbase + c * 32, v);
                     tmem_load32(tbase + 128 + c * 32, u);
-                    stg_scatter(e.out2, e.ld_out2, row0, PM, n, PN, stg + kStgBytes, v);
-                    stg_scatter(e.out3, e.ld_out3, row0, PM, n, PN, stg + 2 * kStgBytes, u);
+                    // each lane writes its own row: whole 32-byte sectors in
+                    // 256-bit stores, no staging (the freed shared memory is a
+                    // sixth pipeline stage)
+                    if (valid) {
+                        store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, PN, 0, v);
+                        store_row32(e.out3, static_cast<int64_t>(m) * e.ld_out3, n, PN, 0, u);
+                    }
 #pragma unroll
                     for (int i = 0; i < 32; i += 2) {   // SiLU(g) * u on the bf16-rounded G and U
                         const float2 g = make_float2(round_bf16(v[i]), round_bf16(v[i + 1]));
@@ -744,7 +699,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         v[i] = a.x;
                         v[i + 1] = a.y;
                     }
-                    stg_scatter(e.out, e.ld_out, row0, PM, n, PN, stg, v);
+                    if (valid) store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, PN, 0, v);
                 }
             } else if constexpr (EPI == EPI_SWIGLU_BWD) {
                 float g[32], u[32];
@@ -988,8 +943,6 @@ static int dispatch(const Params& p, int epi_kind, bool a_mn, bool b_mn, bool du
             return launch_inst<CG, true, false, EPI_LINEAR>(p, stream);
         case EPI_LOGITS:
             if (a_mn || b_mn) return BOM_ENOTSUP;
-            // short contractions: the epilogue dominates, so stage its stores
-            if (p.kb[0] <= 16) return launch_inst<CG, false, false, EPI_LOGITS_STG>(p, stream);
             return launch_inst<CG, false, false, EPI_LOGITS>(p, stream);
         case EPI_SWIGLU_FWD:
             if (a_mn || b_mn || !dual_b) return BOM_ENOTSUP;
