@@ -634,7 +634,15 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
         GemmDesc head_dw;
         GemmDesc pend[3];
         int npend = 0;
-        const bool defer_head = h->bf16 && kfull == 1 && !h->lw.empty() && h->lw[0].kind == BOM_LAYER_SWIGLU;
+        // Up to two Linear layers in front of the head: their cotangents stay in
+        // dx[0] and dx[1] until the pass ends, so their weight gradients and
+        // the head's can run as one grouped launch after the last input
+        // cotangent (every weight is still read before its fused update).
+        bool defer_lin = h->bf16 && kfull == 1 && !h->lw.empty() && h->lw.size() <= 2;
+        for (const LayerWs& L : h->lw)
+            defer_lin = defer_lin && (L.kind == BOM_LAYER_LINEAR || L.kind == BOM_LAYER_LINEAR_GELU);
+        const bool defer_head =
+            (h->bf16 && kfull == 1 && !h->lw.empty() && h->lw[0].kind == BOM_LAYER_SWIGLU) || defer_lin;
         {   // head weight: a R^T H + b qhat (x) c
             GemmDesc g = gemm1(V, dm, kfull * n, mnmaj(h->Z, h->ldz), mnmaj(xin, dm));
             g.epi.alpha_const = 1.0f;
@@ -765,7 +773,18 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
                     g.epi.ld_out = L.d_in;
                     g.epi.out_f32 = of32;
                     if (fused) fuse(g, p0);
-                    BOM_TRY(run_gemm(h, g, s));
+                    if (defer_lin) {
+                        pend[npend++] = g;
+                        if (l == 0) {   // the last layer of the pass: these and the head's, one launch
+                            GemmDesc gw[3];
+                            int ng = 0;
+                            for (int i = 0; i < npend; ++i) gw[ng++] = pend[i];
+                            gw[ng++] = head_dw;
+                            BOM_TRY(run_gemm_group(h, gw, ng, s));
+                        }
+                    } else {
+                        BOM_TRY(run_gemm(h, g, s));
+                    }
                 }
                 if (L.bias) {
                     BOM_TRACED("colsum", 2.0 * n * L.d_out, h->esz * n * L.d_out,
