@@ -6,8 +6,9 @@
 // tile is split between gate and up weights).  Warp roles:
 //   warp 0     one thread issues TMA tile loads (128-byte swizzle) into a
 //              shared-memory ring guarded by mbarriers: 32 KB stages (A rows
-//              and this CTA's half of B), as many as fit beside the epilogue
-//              staging blocks, up to six;
+//              and this CTA's half of B), as many as fit beside the epilogue's
+//              own shared memory (the fused update's blocks, the SwiGLU
+//              backward's G/U slots), up to six;
 //   warp 1     allocates 512 TMEM columns (two 256-column fp32 accumulators)
 //              and, in the even CTA, one thread issues the UMMAs (K = 16),
 //              releasing each smem stage with tcgen05.commit;
