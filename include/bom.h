@@ -54,7 +54,9 @@ typedef enum {
     BOM_ELABEL = 4,    /* device: a label outside [0, d_out) that is not ignore_index */
     BOM_EEMPTY = 5,    /* device: N_t = 0 (Algorithm 1 requires N_t > 0)              */
     BOM_ETIMEOUT = 6,  /* device: a bounded wait inside a kernel ran out              */
-    BOM_ENOTSUP = 7    /* shape or alignment this build does not handle               */
+    BOM_ENOTSUP = 7,   /* shape or alignment this build does not handle               */
+    BOM_ENONFINITE = 8 /* a row's log-sum-exp or its label logit is not finite
+                          (device-detected before any state is written)              */
 } bom_status;
 
 typedef enum { BOM_F32 = 0, BOM_BF16 = 1 } bom_dtype;

@@ -20,7 +20,7 @@ from . import inputs as _inputs
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", "libbom.so")
 
-BOM_OK, BOM_EINVAL, BOM_ENOMEM, BOM_ECUDA, BOM_ELABEL, BOM_EEMPTY, BOM_ETIMEOUT, BOM_ENOTSUP = range(8)
+BOM_OK, BOM_EINVAL, BOM_ENOMEM, BOM_ECUDA, BOM_ELABEL, BOM_EEMPTY, BOM_ETIMEOUT, BOM_ENOTSUP, BOM_ENONFINITE = range(9)
 BOM_F32, BOM_BF16 = 0, 1
 BOM_LAYER_LINEAR, BOM_LAYER_LINEAR_GELU, BOM_LAYER_SWIGLU, BOM_LAYER_RMSNORM = 0, 1, 2, 3
 BOM_OUT_U, BOM_OUT_G_AND_H = 0, 1

@@ -1070,6 +1070,7 @@ const char* bom_status_string(bom_status s) {
         case BOM_EEMPTY: return "BOM_EEMPTY: no supervised outputs (N_t = 0)";
         case BOM_ETIMEOUT: return "BOM_ETIMEOUT: a bounded device wait ran out";
         case BOM_ENOTSUP: return "BOM_ENOTSUP: shape or alignment not supported";
+        case BOM_ENONFINITE: return "BOM_ENONFINITE: non-finite logits (row log-sum-exp or label logit)";
     }
     return "unknown bom_status";
 }

@@ -48,7 +48,7 @@ void launch_row_stats_f32(const float* Z, int64_t ldz, int64_t n, int64_t V, flo
 // Merges per-tile (max, sum exp) pairs into lse[i]; ce[i] = lse_i - z_{i,y_i}
 // for supervised rows, 0 otherwise.
 void launch_row_lse(const void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* stats, int64_t ntiles,
-                    const int32_t* labels, int32_t ignore, float* lse, float* ce, const DevScalars* sc,
+                    const int32_t* labels, int32_t ignore, float* lse, float* ce, DevScalars* sc,
                     cudaStream_t s);
 
 // Z -> R in place: r_ij = exp(z_ij - lse_i) - [j = y_i] on supervised rows, 0 on

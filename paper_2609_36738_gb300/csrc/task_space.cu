@@ -160,7 +160,7 @@ __global__ void row_stats_f32_kernel(const float* __restrict__ Z, int64_t ldz, i
 
 __global__ void row_lse_kernel(const void* __restrict__ Z, int z_f32, int64_t ldz, int64_t n, int64_t V,
                                const float2* __restrict__ stats, int64_t ntiles, const int32_t* __restrict__ labels,
-                               int32_t ignore, float* __restrict__ lse, float* __restrict__ ce, const DevScalars* sc) {
+                               int32_t ignore, float* __restrict__ lse, float* __restrict__ ce, DevScalars* sc) {
     pdl_enter();
     if (sc->status != 0) return;
     const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -199,6 +199,9 @@ __global__ void row_lse_kernel(const void* __restrict__ Z, int z_f32, int64_t ld
         const float L = m + logf(s);
         lse[row] = L;
         ce[row] = has_y ? L - zy : 0.0f;
+        // a non-finite row (ignored or not: its activations still reach the
+        // weight gradients) stops the step before q or any parameter changes
+        if (!isfinite(L) || (has_y && !isfinite(zy))) latch_status(sc, BOM_ENONFINITE);
     }
 }
 
@@ -600,7 +603,7 @@ void launch_row_stats_f32(const float* Z, int64_t ldz, int64_t n, int64_t V, flo
 }
 
 void launch_row_lse(const void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* stats, int64_t ntiles,
-                    const int32_t* labels, int32_t ignore, float* lse, float* ce, const DevScalars* sc,
+                    const int32_t* labels, int32_t ignore, float* lse, float* ce, DevScalars* sc,
                     cudaStream_t s) {
     launch_k(row_lse_kernel, dim3(cdiv(n * 32, 256)), dim3(256), 0, s, Z, z_f32, ldz, n, V, reinterpret_cast<const float2*>(stats),
                                                       ntiles, labels, ignore, lse, ce, sc); count_launch();
