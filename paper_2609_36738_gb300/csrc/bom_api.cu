@@ -21,6 +21,8 @@
 #include <atomic>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "gemm.h"
 #include "kernels.h"
 
@@ -248,11 +250,21 @@ int traced(bom_handle* h, cudaStream_t s, const char* name, double flops, double
     r.name = name;
     r.flops = flops;
     r.bytes = bytes;
+    nvtxRangePushA(name);   // the launch shows up under its kernel class in a profiler timeline
     cudaEventRecord(r.a, s);
     const int rc = launch();
     cudaEventRecord(r.b, s);
+    nvtxRangePop();
     return rc;
 }
+
+// An NVTX range over a whole entry point (closed on every return path).
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange&) = delete;
+    NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 const char* gemm_name(const GemmDesc& g, bool bf16) {
     if (!bf16) return "gemm_simt";
@@ -445,6 +457,7 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
     if (!aligned16(x) || !aligned16(q)) return BOM_ENOTSUP;
 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const NvtxRange nvtx_step("bom_step");
     const bom_config& cfg = h->cfg;
     const int64_t V = cfg.d_out, dm = h->d_model;
     const int cf32 = h->bf16 ? 0 : 1;
