@@ -209,3 +209,42 @@ def test_single_supervised_row(name):
     oref = G.oracle_step(wl, p64, x, y, np.zeros(wl.vocab), 2)
     assert gout["stats"]["n_t"] == 1
     _compare_step(wl, gout, oref, G.TOL[wl.dtype], False)
+
+
+def _guarded(shape, dtype, guard=64, fill=-7.25):
+    """A tensor view of `shape` inside a buffer with `guard` sentinel elements
+    on each side (16-byte aligned for both dtypes)."""
+    n = int(np.prod(shape))
+    buf = torch.full((guard + n + guard,), fill, dtype=dtype, device=G.DEV)
+    return buf, buf[guard:guard + n].view(shape)
+
+
+def _guards_intact(buf, n, guard=64, fill=-7.25):
+    return bool((buf[:guard] == fill).all()) and bool((buf[guard + n:] == fill).all())
+
+
+@pytest.mark.parametrize("name", ["tiny_ragged_f32", "tiny_norm_f32", "vision_small", "lm_head_small",
+                                  "lm_mlp_small", "lm_head_wide", "lm_norm_small"])
+@pytest.mark.parametrize("mode", [B.BOM_OUT_U, B.BOM_OUT_G_AND_H])
+def test_outputs_stay_inside_their_buffers(name, mode):
+    """Canary regions around every output (u or g, h, the input cotangent and
+    q): a step on ragged shapes writes none of them."""
+    wl = I.WORKLOADS[name]
+    params = I.init_params(wl, seed=4)
+    x, y = I.make_batch(wl, seed=4, step=1)
+    gpu = G.GpuBom(wl, params, out_mode=mode)
+    cdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    gb = [_guarded(p.shape, cdt) for p in gpu.params]
+    hb = [_guarded(p.shape, torch.float32) for p in gpu.params] if mode == B.BOM_OUT_G_AND_H else None
+    dxb = _guarded((wl.n_rows, wl.d_in), cdt)
+    qb = _guarded((wl.vocab,), torch.float32)
+    qb[1].zero_()
+    B.bom_set_input_grad(gpu.model.h, dxb[1])
+    xd = G.to_dev(x)
+    yd = torch.from_numpy(np.ascontiguousarray(y, dtype=np.int32)).to(G.DEV)
+    gpu.model.step(xd, yd, wl.n_rows, gpu.params, qb[1], 1, [v for _, v in gb],
+                   [v for _, v in hb] if hb else None)
+    assert gpu.model.stats()["code"] == B.BOM_OK
+    for buf, view in gb + (hb or []) + [dxb, qb]:
+        assert _guards_intact(buf, view.numel())
+        assert torch.isfinite(view.float()).all()
