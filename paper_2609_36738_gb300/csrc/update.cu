@@ -423,12 +423,14 @@ __global__ void __launch_bounds__(256) update_blockshared_kernel(float* __restri
     }
 }
 
-// Blocks of at most 8192 elements (d % 4 == 0): each thread keeps its WPT
-// words of g (packed as loaded), h and theta in registers from one read, so
-// a block costs one memory round trip before the reduction and none after it;
-// v of the block is fetched with the data.  WPT is the smallest of 1, 2, 4, 8
-// with 1024 WPT >= block, which keeps the registers (and so the number of
-// resident CTAs, whose loads hide the latency) matched to the block.
+// Blocks of at most 8192 elements (d % 4 == 0): each of the CTA's NT threads
+// keeps its WPT words of g (packed as loaded), h and theta in registers from
+// one read, so a block costs one memory round trip before the reduction and
+// none after it; v of the block is fetched with the data.  Blocks up to 4096
+// elements use 256 threads and WPT 1, 2 or 4 (the smallest with
+// 1024 WPT >= block, which keeps the registers, and so the resident CTAs
+// whose loads hide the latency, matched to the block); larger ones use 512
+// threads and WPT 4, so every block size keeps two register sets.
 constexpr int kRegMaxBlock = 8192;
 template <bool G_BF16>
 struct GWord {
@@ -461,7 +463,7 @@ struct RowRegs {
     float vprev;
 };
 
-template <bool G_BF16, bool HAS_H, int WPT>
+template <bool G_BF16, bool HAS_H, int WPT, int NT>
 __device__ __forceinline__ void row_load(RowRegs<G_BF16, WPT>& r, const void* g, const float* h, const float* theta,
                                          const float* vb, int64_t b, int64_t block, int64_t n) {
     using GW = typename GWord<G_BF16>::T;
@@ -470,7 +472,7 @@ __device__ __forceinline__ void row_load(RowRegs<G_BF16, WPT>& r, const void* g,
     r.vprev = threadIdx.x == 0 ? vb[b] : 0.0f;
 #pragma unroll
     for (int k = 0; k < WPT; ++k) {
-        const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
+        const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + NT * k);
         if (i < e1) {
             r.gw[k] = *reinterpret_cast<const GW*>(static_cast<const char*>(g) + i * (G_BF16 ? 2 : 4));
             if constexpr (HAS_H) r.hw[k] = *reinterpret_cast<const float4*>(h + i);
@@ -480,7 +482,7 @@ __device__ __forceinline__ void row_load(RowRegs<G_BF16, WPT>& r, const void* g,
 }
 
 // Reduction, v_b and the update of block b from its registers.
-template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT>
+template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT, int NT>
 __device__ __forceinline__ void row_update(const RowRegs<G_BF16, WPT>& r, float* theta, float* vb, uint16_t* shadow,
                                            int64_t b, int64_t block, int64_t n, const UpdCoef& c, float* red,
                                            float* s_den) {
@@ -489,7 +491,7 @@ __device__ __forceinline__ void row_update(const RowRegs<G_BF16, WPT>& r, float*
     float acc = 0.0f;
 #pragma unroll
     for (int k = 0; k < WPT; ++k) {
-        const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
+        const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + NT * k);
         if (i < e1) {
             float u[4];
             word_u<G_BF16, HAS_H>(r.gw[k], r.hw[k], c.lam, u);
@@ -503,7 +505,7 @@ __device__ __forceinline__ void row_update(const RowRegs<G_BF16, WPT>& r, float*
     if (threadIdx.x == 0) {
         float tot = 0.0f;
 #pragma unroll
-        for (int w = 0; w < 8; ++w) tot += red[w];
+        for (int w = 0; w < NT / 32; ++w) tot += red[w];
         const float vv = fmaf(c.beta2, r.vprev, c.one_m_beta2 * (tot / static_cast<float>(e1 - e0)));
         vb[b] = vv;
         *s_den = sqrtf(vv * c.inv_bc2) + c.eps;
@@ -512,7 +514,7 @@ __device__ __forceinline__ void row_update(const RowRegs<G_BF16, WPT>& r, float*
     const float den = *s_den;
 #pragma unroll
     for (int k = 0; k < WPT; ++k) {
-        const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + 256 * k);
+        const int64_t i = e0 + 4 * (static_cast<int64_t>(threadIdx.x) + NT * k);
         if (i < e1) {
             float u[4];
             word_u<G_BF16, HAS_H>(r.gw[k], r.hw[k], c.lam, u);
@@ -533,43 +535,33 @@ __device__ __forceinline__ void row_update(const RowRegs<G_BF16, WPT>& r, float*
     __syncthreads();   // red and s_den are reused by the next block
 }
 
-// The CTA walks its blocks b, b + grid, ...  Up to 4 words per thread it
-// keeps two register sets: the loads of the next block are issued before the
-// current one is reduced and written, so the CTA keeps a block's reads in
-// flight through its barriers.  At 8 words two sets would cost more resident
-// CTAs than they gain, so those blocks go one at a time.
-template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT>
-__global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __restrict__ theta,
-                                                                     const void* __restrict__ g,
-                                                                     const float* __restrict__ h,
-                                                                     float* __restrict__ vb,
-                                                                     uint16_t* __restrict__ shadow, int64_t n,
-                                                                     int64_t block, UpdCoef c_in) {
+// The CTA walks its blocks b, b + grid, ... with two register sets: the
+// loads of the next block are issued before the current one is reduced and
+// written, so the CTA keeps a block's reads in flight through its barriers.
+template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT, int NT>
+__global__ void __launch_bounds__(NT) update_blockshared_reg_kernel(float* __restrict__ theta,
+                                                                    const void* __restrict__ g,
+                                                                    const float* __restrict__ h,
+                                                                    float* __restrict__ vb,
+                                                                    uint16_t* __restrict__ shadow, int64_t n,
+                                                                    int64_t block, UpdCoef c_in) {
     pdl_enter();
-    __shared__ float red[8];
+    __shared__ float red[NT / 32];
     __shared__ float s_den;
     const UpdCoef c = resolve_coef(c_in, nullptr);
     const int64_t nb = (n + block - 1) / block;
     const int64_t G = gridDim.x;
     int64_t b = blockIdx.x;
     if (b >= nb) return;
-    if constexpr (WPT > 4) {
-        RowRegs<G_BF16, WPT> r;
-        for (; b < nb; b += G) {
-            row_load<G_BF16, HAS_H, WPT>(r, g, h, theta, vb, b, block, n);
-            row_update<G_BF16, HAS_H, SHADOW, WPT>(r, theta, vb, shadow, b, block, n, c, red, &s_den);
-        }
-        return;
-    }
     RowRegs<G_BF16, WPT> ra, rb;
-    row_load<G_BF16, HAS_H, WPT>(ra, g, h, theta, vb, b, block, n);
+    row_load<G_BF16, HAS_H, WPT, NT>(ra, g, h, theta, vb, b, block, n);
     for (;;) {
-        if (b + G < nb) row_load<G_BF16, HAS_H, WPT>(rb, g, h, theta, vb, b + G, block, n);
-        row_update<G_BF16, HAS_H, SHADOW, WPT>(ra, theta, vb, shadow, b, block, n, c, red, &s_den);
+        if (b + G < nb) row_load<G_BF16, HAS_H, WPT, NT>(rb, g, h, theta, vb, b + G, block, n);
+        row_update<G_BF16, HAS_H, SHADOW, WPT, NT>(ra, theta, vb, shadow, b, block, n, c, red, &s_den);
         b += G;
         if (b >= nb) break;
-        if (b + G < nb) row_load<G_BF16, HAS_H, WPT>(ra, g, h, theta, vb, b + G, block, n);
-        row_update<G_BF16, HAS_H, SHADOW, WPT>(rb, theta, vb, shadow, b, block, n, c, red, &s_den);
+        if (b + G < nb) row_load<G_BF16, HAS_H, WPT, NT>(ra, g, h, theta, vb, b + G, block, n);
+        row_update<G_BF16, HAS_H, SHADOW, WPT, NT>(rb, theta, vb, shadow, b, block, n, c, red, &s_den);
         b += G;
         if (b >= nb) break;
     }
@@ -577,28 +569,29 @@ __global__ void __launch_bounds__(256) update_blockshared_reg_kernel(float* __re
 
 // Resident CTAs per SM times the SM count, at most the number of blocks.
 template <typename K>
-int resident_grid(K kernel, int64_t nb) {
+int resident_grid(K kernel, int64_t nb, int nt) {
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, 256, 0) != cudaSuccess || per_sm < 1)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, nt, 0) != cudaSuccess || per_sm < 1)
         per_sm = 1;
     const int64_t grid = static_cast<int64_t>(device_sm_count()) * per_sm;
     return static_cast<int>(grid < nb ? grid : nb);
 }
 
-template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT>
+template <bool G_BF16, bool HAS_H, bool SHADOW, int WPT, int NT>
 void launch_reg(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n, int64_t block,
                 const UpdCoef& c, cudaStream_t s) {
-    auto k = update_blockshared_reg_kernel<G_BF16, HAS_H, SHADOW, WPT>;
-    launch_k(k, dim3(resident_grid(k, (n + block - 1) / block)), dim3(256), 0, s, theta, g, h, vb, shadow, n, block, c);
+    auto k = update_blockshared_reg_kernel<G_BF16, HAS_H, SHADOW, WPT, NT>;
+    launch_k(k, dim3(resident_grid(k, (n + block - 1) / block, NT)), dim3(NT), 0, s, theta, g, h, vb, shadow, n,
+             block, c);
 }
 
 template <bool G_BF16, bool HAS_H, bool SHADOW>
 void launch_reg_wpt(float* theta, const void* g, const float* h, float* vb, uint16_t* shadow, int64_t n,
                     int64_t block, const UpdCoef& c, cudaStream_t s) {
-    if (block <= 1024) launch_reg<G_BF16, HAS_H, SHADOW, 1>(theta, g, h, vb, shadow, n, block, c, s);
-    else if (block <= 2048) launch_reg<G_BF16, HAS_H, SHADOW, 2>(theta, g, h, vb, shadow, n, block, c, s);
-    else if (block <= 4096) launch_reg<G_BF16, HAS_H, SHADOW, 4>(theta, g, h, vb, shadow, n, block, c, s);
-    else launch_reg<G_BF16, HAS_H, SHADOW, 8>(theta, g, h, vb, shadow, n, block, c, s);
+    if (block <= 1024) launch_reg<G_BF16, HAS_H, SHADOW, 1, 256>(theta, g, h, vb, shadow, n, block, c, s);
+    else if (block <= 2048) launch_reg<G_BF16, HAS_H, SHADOW, 2, 256>(theta, g, h, vb, shadow, n, block, c, s);
+    else if (block <= 4096) launch_reg<G_BF16, HAS_H, SHADOW, 4, 256>(theta, g, h, vb, shadow, n, block, c, s);
+    else launch_reg<G_BF16, HAS_H, SHADOW, 4, 512>(theta, g, h, vb, shadow, n, block, c, s);
 }
 
 // Launch shape of the cluster kernel; at[] must hold two attributes.
