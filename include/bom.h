@@ -29,10 +29,16 @@
  *   bom_get_stats synchronises.
  * - Host-checkable problems (null pointers, bad sizes, t < 1, unaligned
  *   pointers) return an error immediately and enqueue nothing.  Problems only
- *   the device can see (a bad label, N_t = 0, a bounded wait that ran out) are
- *   latched in a device status word of the handle; every later kernel of the
- *   step skips its work, q is left unmodified, and bom_get_stats returns the
- *   latched code.  The word is cleared at the start of each bom_step.
+ *   the device can see (a bad label, N_t = 0, non-finite logits, a device step
+ *   counter below 1, a bounded wait that ran out) are latched in a device
+ *   status word of the handle; every later kernel of the step skips its work,
+ *   q (and, with the fused update, every parameter and v) is left unmodified,
+ *   and bom_get_stats returns the latched code.  The word is cleared at the
+ *   start of each bom_step.
+ * - Kernels are launched with programmatic dependent launch: a kernel may be
+ *   scheduled while the previous one on the stream finishes, but it waits for
+ *   that one's completion before touching memory, so stream order holds for
+ *   the caller's own work before and after every call.
  * - Alignment: every bf16 tensor used by the tensor-core path needs a 16-byte
  *   aligned base and a row length that is a multiple of 8 elements (TMA rule);
  *   otherwise BOM_ENOTSUP.
@@ -166,7 +172,8 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
  * compute-dtype copy of it.  Requires BOM_OUT_U mode and no own-step output
  * (bom_step returns BOM_EINVAL otherwise).  No update happens in a step whose
  * device status latches an error.  lr usually changes per step: call this
- * again before each step (host-side only).  theta = NULL disables it. */
+ * again before each step (host-side only), or register a device learning rate
+ * with bom_set_step_scalars.  theta = NULL disables it. */
 bom_status bom_set_fused_update(bom_handle* h, float* const* theta, float* const* v, const float* wd, float lr,
                                 float beta2, float eps);
 
