@@ -908,27 +908,32 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restr
 }
 
 // Number of K ranges for a GEMM with `tiles` output tiles on `units` resident
-// tile walkers.  Split only when the waves would leave the GPU under 75% busy
-// (the fp32 partials cost more than milder quantisation does);
-// among 2..8 ranges (>= 16 k-blocks each, partials fitting the scratch) take
-// the best busy fraction less 1 point per range, if it beats no split by more
-// than 8 points.
+// tile walkers.  GEMMs that keep the GPU at least 75% busy are not split (the
+// fp32 partials cost more than milder quantisation does).  Otherwise the
+// split minimises an estimate of the time in k-block steps: waves x (k-blocks
+// per range + 2 for storing a tile), plus for a split the reduction (about 14
+// steps of launch and fixed cost, and the partials' round trip through memory
+// at about 5e-6 steps per fp32 element); among 2..8 ranges of at least 8
+// k-blocks whose partials fit the scratch, the cheapest that saves 10% over
+// no split.
 static int choose_split(int tiles, int units, int kb_total, int64_t mn, int64_t ws_elems) {
-    auto eff = [&](int s) {
-        const double w = static_cast<double>(tiles) * s;
-        const double waves = std::ceil(w / units);
-        return w / (waves * units);
+    auto waves = [&](int s) { return (static_cast<int64_t>(tiles) * s + units - 1) / units; };
+    if (static_cast<double>(tiles) / (static_cast<double>(waves(1)) * units) >= 0.75) return 1;
+    auto cost = [&](int s) {
+        const double per = std::ceil(static_cast<double>(kb_total) / s) + 2.0;
+        double c = static_cast<double>(waves(s)) * per;
+        if (s > 1) c += 14.0 + 5e-6 * static_cast<double>(s) * static_cast<double>(mn);
+        return c;
     };
-    const double e1 = eff(1);
-    if (e1 >= 0.75) return 1;
+    const double c1 = cost(1);
     int best = 1;
-    double best_score = e1 - 0.01;
+    double best_cost = c1;
     for (int s = 2; s <= 8; ++s) {
-        if (kb_total / s < 16 || static_cast<int64_t>(s) * mn > ws_elems) break;
-        const double e = eff(s);
-        if (e >= e1 + 0.08 && e - 0.01 * s > best_score) {
+        if (kb_total / s < 8 || static_cast<int64_t>(s) * mn > ws_elems) break;
+        const double c = cost(s);
+        if (c < 0.9 * c1 && c < best_cost) {
             best = s;
-            best_score = e - 0.01 * s;
+            best_cost = c;
         }
     }
     return best;
