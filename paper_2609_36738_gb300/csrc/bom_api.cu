@@ -14,6 +14,13 @@
 //             then the backbone VJPs, with (a, b) = N_t^-1 (1-lambda, lambda)
 //             for u, N_t^-1 (1, 0) for g and N_t^-1 (0, 1) for h; the
 //             own-step pass (telemetry) broadcasts s_t in place of qhat.
+// With the fused update registered, each weight is updated in the epilogue of
+// the GEMM that forms its u (the weight gradients of a block run as one
+// grouped launch after its last input cotangent), and each vector right
+// after its gradient.  The step's scalars (lr, 1/(1-beta1^t), 1/(1-beta2^t))
+// live in the device scalar block, written by the label scan from the host's
+// values or from a registered device step counter, so a captured step
+// (bom_graph_capture) replays correctly for every later t.
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
