@@ -478,12 +478,15 @@ __device__ __forceinline__ float word_elem(const uint4& w, int k) {
         return __uint_as_float(v);
 }
 
+// With `out` given (a single row range), the block writes the final column
+// sums, scaled and in out's dtype, instead of partials.
 template <typename T, bool HAS_Y>
 __global__ void __launch_bounds__(256, 3) colsum_part_kernel(const T* __restrict__ X, const T* __restrict__ Y,
                                                              int64_t ldx, int64_t n, int64_t rows_per,
                                                              int64_t d, const int32_t* __restrict__ labels,
                                                              int32_t ignore, const float* __restrict__ wvec,
-                                                             float* __restrict__ part, const DevScalars* sc) {
+                                                             float* __restrict__ part, void* __restrict__ out,
+                                                             int out_f32, float scale, const DevScalars* sc) {
     pdl_enter();
     constexpr int VEC = 16 / sizeof(T);
     // rows in flight per warp step: 8 words per thread (4 of X and 4 of Y)
@@ -560,7 +563,10 @@ __global__ void __launch_bounds__(256, 3) colsum_part_kernel(const T* __restrict
         float a = 0.0f;
 #pragma unroll
         for (int k = 0; k < 8; ++k) a += red[k][j];
-        part[static_cast<int64_t>(blockIdx.y) * d + c] = a;
+        if (out != nullptr)
+            st_elem(out, c, out_f32, a * scale);
+        else
+            part[static_cast<int64_t>(blockIdx.y) * d + c] = a;
     }
 }
 
@@ -682,30 +688,36 @@ void launch_colsum2(const void* X, const void* Y, int x_f32, int64_t ldx, int64_
                     const int32_t* labels, int32_t ignore, const float* wvec, float scale, float* part, void* out,
                     int out_f32, const DevScalars* sc, cudaStream_t s) {
     const int64_t cols_per_block = x_f32 ? 128 : 256;
-    const int64_t rows_per = colsum_rows_per(n, cdiv(d, cols_per_block), device_sm_count());
+    // a batch within one row range: its blocks write the result directly and
+    // the finishing launch is skipped
+    const bool single = n <= kRowBlock;
+    const int64_t rows_per = single ? (n > 0 ? n : 1) : colsum_rows_per(n, cdiv(d, cols_per_block), device_sm_count());
     const int64_t nb = (n + rows_per - 1) / rows_per;
-    dim3 grid(cdiv(d, cols_per_block), static_cast<unsigned>(nb));
+    void* const direct = single ? out : nullptr;
+    dim3 grid(cdiv(d, cols_per_block), static_cast<unsigned>(nb > 0 ? nb : 1));
     if (x_f32) {
         auto x = static_cast<const float*>(X);
         auto y = static_cast<const float*>(Y);
         if (Y)
-            launch_k(colsum_part_kernel<float, true>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels, ignore, wvec,
-                                                                 part, sc);
+            launch_k(colsum_part_kernel<float, true>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels,
+                     ignore, wvec, part, direct, out_f32, scale, sc);
         else
-            launch_k(colsum_part_kernel<float, false>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels, ignore, wvec,
-                                                                  part, sc);
+            launch_k(colsum_part_kernel<float, false>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels,
+                     ignore, wvec, part, direct, out_f32, scale, sc);
     } else {
         auto x = static_cast<const __nv_bfloat16*>(X);
         auto y = static_cast<const __nv_bfloat16*>(Y);
         if (Y)
-            launch_k(colsum_part_kernel<__nv_bfloat16, true>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels, ignore,
-                                                                         wvec, part, sc);
+            launch_k(colsum_part_kernel<__nv_bfloat16, true>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d,
+                     labels, ignore, wvec, part, direct, out_f32, scale, sc);
         else
-            launch_k(colsum_part_kernel<__nv_bfloat16, false>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per, d, labels, ignore,
-                                                                          wvec, part, sc);
+            launch_k(colsum_part_kernel<__nv_bfloat16, false>, dim3(grid), dim3(256), 0, s, x, y, ldx, n, rows_per,
+                     d, labels, ignore, wvec, part, direct, out_f32, scale, sc);
     }
     count_launch();
-    launch_k(colsum_finish_kernel, dim3(cdiv(d, 32)), dim3(256), 0, s, part, nb, d, scale, out, out_f32, sc); count_launch();
+    if (single) return;
+    launch_k(colsum_finish_kernel, dim3(cdiv(d, 32)), dim3(256), 0, s, part, nb, d, scale, out, out_f32, sc);
+    count_launch();
 }
 
 void launch_axpby(const float* s_vec, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
