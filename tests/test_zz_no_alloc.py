@@ -66,3 +66,20 @@ def test_noalloc_colsum_rejects_sizes_beyond_its_scratch():
     with pytest.raises(B.BomError) as e:
         B.bom_colsum_noalloc(x, B.BOM_BF16, 4096, 128 * 600, 2048, None, out)
     assert e.value.code == B.BOM_ENOTSUP
+
+
+def test_noalloc_colsum_at_the_scratch_limit():
+    """ceil(n / 128) * n_cols = 2^20 exactly (65,536 rows x 2,048 columns) is
+    accepted and matches the GEMM entry; one row more is refused."""
+    n, d = 128 * 512, 2048
+    x, _, ref = _case(3, n + 1, d, False)
+    out = torch.full((d,), float("nan"), dtype=torch.float32, device=G.DEV)
+    with pytest.raises(B.BomError) as e:
+        B.bom_colsum_noalloc(x, B.BOM_BF16, d, n + 1, d, None, out)
+    assert e.value.code == B.BOM_ENOTSUP
+    # the first n rows: the reference is the full sum minus the last row
+    B.bom_colsum_noalloc(x, B.BOM_BF16, d, n, d, None, out)
+    torch.cuda.synchronize()
+    want = G.np64(ref) - G.np64(x[n].float())
+    assert torch.isfinite(out).all()
+    assert G.rel_l2(G.np64(out), want) < TOL
