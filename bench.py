@@ -334,11 +334,7 @@ def main():
     B.bom_trace(model.h, False)
     st = model.stats(stream)
     step_ms = [e0.elapsed_time(e1) for e0, e1 in ev]
-    tot_ms = sum(step_ms)
-    if dist is not None:
-        tt = torch.tensor([tot_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        tot_ms = float(tt.item())
+    tot_ms = _max_over_ranks(dist, sum(step_ms), dev)
     value = world * N * a.steps / (tot_ms / 1e3)
 
     # ---------------------------------------------------------------- dominant kernel roofline
@@ -378,6 +374,8 @@ def main():
     # ---------------------------------------------------------------- end to end through host buffers
     e2e_steps = max(3, a.steps // 2)
     h2d = x_host.numel() * x_host.element_size() + y_host.numel() * y_host.element_size()
+    if dist is not None:
+        dist.barrier()
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for i in range(e2e_steps):
@@ -386,7 +384,7 @@ def main():
         yy = y_host.to(dev, non_blocking=True)
         step(t, xx.view(torch.bfloat16) if bf16 else xx, yy)
         model.stats(stream)        # device -> host read of the step's loss / status (syncs)
-    e2e_s = time.perf_counter() - t0
+    e2e_s = _max_over_ranks(dist, time.perf_counter() - t0, dev)
     e2e = {"value": world * N * e2e_steps / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
            "d2h_bytes_per_step": B.bom_stats_transfer_bytes()}
 
@@ -424,6 +422,17 @@ def main():
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
+
+
+def _max_over_ranks(dist, x, dev):
+    """The largest of a per-rank time over all ranks (x itself on one rank),
+    so a whole-job rate is set by the slowest replica."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
 
 
 def _ncu_traffic(kernel_name):

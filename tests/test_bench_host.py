@@ -61,3 +61,29 @@ def test_missing_nvidia_smi_is_reported():
     s = bench.ClockSampler("0")
     out = s.stop()
     assert out["sm_mhz"] is None and out["reasons"] == ["nvidia-smi unavailable"]
+
+
+def _max_rank_main(rank, world, port, out_dir):
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    got = bench._max_over_ranks(dist, 1.0 + 2.5 * rank, "cpu")
+    with open(os.path.join(out_dir, f"r{rank}.txt"), "w") as f:
+        f.write(repr(got))
+    dist.destroy_process_group()
+
+
+def test_step_time_is_the_maximum_over_ranks(tmp_path):
+    """The whole-job rate divides by the slowest rank's time: every rank gets
+    the maximum (two gloo ranks on the CPU); one rank keeps its own."""
+    import socket
+
+    import torch.multiprocessing as mp
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    mp.spawn(_max_rank_main, args=(2, port, str(tmp_path)), nprocs=2, join=True)
+    for r in range(2):
+        assert float(open(tmp_path / f"r{r}.txt").read()) == 3.5
+    assert bench._max_over_ranks(None, 1.25, "cpu") == 1.25
