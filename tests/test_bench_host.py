@@ -87,3 +87,23 @@ def test_step_time_is_the_maximum_over_ranks(tmp_path):
     for r in range(2):
         assert float(open(tmp_path / f"r{r}.txt").read()) == 3.5
     assert bench._max_over_ranks(None, 1.25, "cpu") == 1.25
+
+
+def test_traffic_is_reported_only_for_the_captured_source(tmp_path, monkeypatch):
+    """roofline.traffic comes from the committed ncu record while the kernel's
+    source file still has the hash recorded with the capture; a changed source
+    or a kernel without a record gives null."""
+    import hashlib
+    import json
+
+    src = tmp_path / "k.cu"
+    src.write_text("// kernel as captured\n")
+    (tmp_path / "profiles").mkdir()
+    rec = {"k": {"source": "k.cu", "sha256": hashlib.sha256(src.read_bytes()).hexdigest(),
+                 "dram_bytes_per_launch": 123}}
+    (tmp_path / "profiles" / "ncu_traffic.json").write_text(json.dumps(rec))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench._ncu_traffic("k") == 123
+    assert bench._ncu_traffic("other") is None
+    src.write_text("// kernel changed after the capture\n")
+    assert bench._ncu_traffic("k") is None
