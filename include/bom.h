@@ -131,11 +131,15 @@ bom_status bom_param_shape(const bom_config* cfg, int32_t index, int64_t* rows, 
 /* Creates a handle: validates cfg, copies it, and allocates the device
  * workspace (activations, logits/residuals, row statistics, column partial
  * sums, scalars) for max_rows rows on the current device.  The handle owns
- * only that workspace.  Returns BOM_EINVAL on a bad config, BOM_ENOMEM when
- * the workspace does not fit. */
+ * only that workspace.  Returns BOM_EINVAL on a bad config, BOM_ENOTSUP for
+ * max_rows above 4,194,240 (64-row blocks of the per-row passes run along
+ * one grid dimension of at most 65,535 blocks), on the fp32 path for an
+ * output width above the same bound, and for a bf16 width that is not a
+ * multiple of 8; BOM_ENOMEM when the workspace does not fit. */
 bom_status bom_init(bom_handle** out, const bom_config* cfg);
 
-/* Bytes of device workspace bom_init would allocate for cfg. */
+/* Bytes of device workspace bom_init would allocate for cfg (-1 for a cfg
+ * bom_init refuses). */
 int64_t bom_workspace_bytes(const bom_config* cfg);
 
 /* One BOM step (Algorithm 1 up to the update numerator).

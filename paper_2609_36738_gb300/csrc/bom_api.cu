@@ -128,6 +128,10 @@ bom_status check_config(const bom_config* cfg, std::vector<LayerWs>* lw_out, int
     if (!(cfg->lambda >= 0.0f && cfg->lambda <= 1.0f)) return BOM_EINVAL;
     if (!(cfg->beta1 >= 0.0f && cfg->beta1 < 1.0f)) return BOM_EINVAL;
     if (cfg->max_rows > (1ll << 30) || cfg->d_out > (1ll << 30)) return BOM_ENOTSUP;
+    // The residual pass and the fp32 GEMM put 64-row blocks on gridDim.y (at
+    // most 65535 blocks): refused here, before any step could stop half done.
+    constexpr int64_t kMaxGridRows = static_cast<int64_t>(kResidRows) * 65535;
+    if (cfg->max_rows > kMaxGridRows) return BOM_ENOTSUP;
     const bool bf16 = cfg->compute == BOM_BF16;
     std::vector<LayerWs> lw;
     int64_t w = cfg->d_in, mw = cfg->d_in, mf = 0;
@@ -162,6 +166,11 @@ bom_status check_config(const bom_config* cfg, std::vector<LayerWs>* lw_out, int
         if (cfg->d_in % 8) return BOM_ENOTSUP;
         for (auto& x : lw)
             if (x.d_out % 8 || x.d_in % 8) return BOM_ENOTSUP;
+    } else {
+        // fp32 weight gradients run with M = the output width of the head or layer
+        if (cfg->d_out > kMaxGridRows) return BOM_ENOTSUP;
+        for (auto& x : lw)
+            if (x.d_out > kMaxGridRows) return BOM_ENOTSUP;
     }
     *d_model = w;
     *max_width = mw;

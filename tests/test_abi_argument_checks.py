@@ -129,3 +129,20 @@ def test_null_handles_are_rejected(built):
     assert _code(B.bom_sqnorm, None, ALIGNED, B.BOM_BF16, None, 0.5, 16, ALIGNED, stream=0) == B.BOM_EINVAL
     assert _code(B.bom_own_step_moment, None, ALIGNED, ALIGNED, ALIGNED, ALIGNED, 16, 0.9, 1, stream=0) == B.BOM_EINVAL
     assert _code(B.bom_trace, None, True) == B.BOM_EINVAL
+
+
+def test_grid_row_limits_are_refused_at_init(built):
+    """Per-row passes put 64-row blocks on gridDim.y (at most 65,535), so
+    max_rows above 4,194,240 is refused when the handle is made, as is an fp32
+    output width above the same bound (its weight-gradient GEMM has M = that
+    width); the bf16 path takes any vocabulary up to 2^30."""
+    lim = 64 * 65535
+    lin = [(B.BOM_LAYER_LINEAR_GELU, 1, 64, 128)]
+    assert B.bom_workspace_bytes(B.make_config(lim, 64, 10, lin, True, B.BOM_F32)) > 0
+    assert B.bom_workspace_bytes(B.make_config(lim + 1, 64, 10, lin, True, B.BOM_F32)) == -1
+    assert B.bom_workspace_bytes(B.make_config(lim + 1, 64, 10, [], False, B.BOM_BF16)) == -1
+    assert B.bom_workspace_bytes(B.make_config(16, 64, lim, lin, True, B.BOM_F32)) > 0
+    assert B.bom_workspace_bytes(B.make_config(16, 64, lim + 1, lin, True, B.BOM_F32)) == -1
+    wide = [(B.BOM_LAYER_LINEAR_GELU, 1, 64, lim + 1)]
+    assert B.bom_workspace_bytes(B.make_config(16, 64, 10, wide, True, B.BOM_F32)) == -1
+    assert B.bom_workspace_bytes(B.make_config(16, 64, lim + 1, [], False, B.BOM_BF16)) > 0
