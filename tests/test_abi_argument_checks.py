@@ -146,3 +146,16 @@ def test_grid_row_limits_are_refused_at_init(built):
     wide = [(B.BOM_LAYER_LINEAR_GELU, 1, 64, lim + 1)]
     assert B.bom_workspace_bytes(B.make_config(16, 64, 10, wide, True, B.BOM_F32)) == -1
     assert B.bom_workspace_bytes(B.make_config(16, 64, lim + 1, [], False, B.BOM_BF16)) > 0
+
+
+def test_binding_fails_loudly_without_the_library(tmp_path, monkeypatch):
+    """There is no CPU fallback: with libbom.so absent, loading the library and
+    every compute entry point raise instead of computing anything."""
+    monkeypatch.setattr(B, "LIB_PATH", str(tmp_path / "libbom.so"))
+    monkeypatch.setattr(B, "_LIB", None)
+    with pytest.raises(RuntimeError, match="missing"):
+        B.lib()
+    with pytest.raises(RuntimeError, match="missing"):
+        B.bom_update(**_upd())
+    with pytest.raises(RuntimeError, match="missing"):
+        B.bom_workspace_bytes(B.make_config(16, 64, 10, [], False, B.BOM_F32))
