@@ -19,6 +19,7 @@
 //              the mainloop of tile i+1.
 // Every mbarrier wait is bounded; a wait that runs out latches BOM_ETIMEOUT,
 // all roles unwind, in-flight TMA loads and UMMAs are drained, TMEM is freed.
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 #include <mutex>
@@ -835,8 +836,14 @@ template <int CG, bool A_MN, bool B_MN, int EPI>
 static int launch_inst(const Params& p, cudaStream_t stream) {
     using C = Cfg<CG, EPI>;
     auto k = gemm_kernel<CG, A_MN, B_MN, EPI>;
-    // Resident tile walkers: CTAs (CG = 1) or CTA pairs (CG = 2) that fit at once.
-    static int max_units = 0;
+    // Resident tile walkers: CTAs (CG = 1) or CTA pairs (CG = 2) that fit at
+    // once, found (and the kernel's shared-memory attribute set, which is a
+    // per-device setting) on the first launch on each device.
+    constexpr int kMaxDev = 64;
+    static std::atomic<int> units_dev[kMaxDev];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return BOM_ECUDA;
+    int max_units = units_dev[dev].load(std::memory_order_relaxed);
     if (max_units == 0) {
         if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) != cudaSuccess)
             return BOM_ECUDA;
@@ -861,6 +868,7 @@ static int launch_inst(const Params& p, cudaStream_t stream) {
         } else {
             max_units = device_sm_count();
         }
+        units_dev[dev].store(max_units, std::memory_order_relaxed);
     }
     const int work = p.tile_base[p.nprob] * p.ksplit;
     const int units = work < max_units ? work : max_units;
@@ -966,13 +974,24 @@ static int dispatch(const Params& p, int epi_kind, bool a_mn, bool b_mn, bool du
 
 }  // namespace tc
 
+// Cached per device ordinal (atomics: concurrent first calls from several
+// host threads store the same value).
 int device_sm_count() {
-    static int n = 0;
+    constexpr int kMaxDev = 64;
+    static std::atomic<int> cached[kMaxDev];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        dev = 0;
+    }
+    int n = (dev >= 0 && dev < kMaxDev) ? cached[dev].load(std::memory_order_relaxed) : 0;
     if (n == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+            cudaGetLastError();
+            n = 0;
+        }
         if (n <= 0) n = 1;
+        if (dev >= 0 && dev < kMaxDev) cached[dev].store(n, std::memory_order_relaxed);
     }
     return n;
 }

@@ -57,7 +57,12 @@ extern "C" bom_status bom_colsum_noalloc(const void* x, int32_t dtype, int64_t l
     if (!x || !out || n_rows < 1 || n_cols < 1 || ldx < n_cols) return BOM_EINVAL;
     if (dtype != BOM_F32 && dtype != BOM_BF16) return BOM_EINVAL;
     if ((reinterpret_cast<uintptr_t>(x) & 15u) != 0) return BOM_ENOTSUP;
-    if (row_blocks(n_rows) * n_cols > kNoAllocScratchFloats || row_blocks(n_rows) > 65535) return BOM_ENOTSUP;
+    // Each factor is bounded before the product is formed, so no size the
+    // caller passes can overflow the check: the row ranges run along
+    // gridDim.y (at most 65535) and each holds n_cols partial sums.
+    if (n_cols > kNoAllocScratchFloats) return BOM_ENOTSUP;
+    const int64_t ranges = n_rows / kRowBlock + (n_rows % kRowBlock != 0 ? 1 : 0);
+    if (ranges > 65535 || ranges > kNoAllocScratchFloats / n_cols) return BOM_ENOTSUP;
     DeviceScratch* d = nullptr;
     const bom_status st = scratch_for_current_device(&d);
     if (st != BOM_OK) return st;

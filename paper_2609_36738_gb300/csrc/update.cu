@@ -15,6 +15,7 @@
 // One CTA per block (grid-stride over blocks): a first sweep forms sum u^2 in
 // a fixed order, thread 0 advances v_b, a second sweep applies the update; the
 // second sweep's reads of g and h hit L2.
+#include <atomic>
 #include "kernels.h"
 #include "tc_ptx.cuh"
 #include <mutex>
@@ -610,10 +611,18 @@ cudaLaunchConfig_t cluster_cfg(cudaLaunchAttribute* at) {
     return cfg;
 }
 
-// Clusters of the cluster kernel that run at once (cached per instantiation).
+// Clusters of the cluster kernel that run at once (cached per instantiation
+// and device).
 template <bool G_BF16, bool HAS_H, bool SHADOW, int VEC>
 int cluster_slots() {
-    static int slots = 0;
+    constexpr int kMaxDev = 64;
+    static std::atomic<int> slots_dev[kMaxDev];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) {
+        cudaGetLastError();
+        dev = 0;
+    }
+    int slots = slots_dev[dev].load(std::memory_order_relaxed);
     if (slots == 0) {
         cudaLaunchAttribute at[2];
         cudaLaunchConfig_t cfg = cluster_cfg<G_BF16, HAS_H, SHADOW, VEC>(at);
@@ -626,6 +635,7 @@ int cluster_slots() {
             m = device_sm_count() / kBlockCluster;
         }
         slots = m > 0 ? m : 1;
+        slots_dev[dev].store(slots, std::memory_order_relaxed);
     }
     return slots;
 }

@@ -115,6 +115,11 @@ def test_bom_gemm_bf16_checks(built, over, code):
     (dict(x=UNALIGNED), "BOM_ENOTSUP"),
     # ceil(n_rows / 128) * n_cols above the fixed 2^20-float scratch
     (dict(n_rows=129, n_cols=(1 << 19) + 8, ldx=(1 << 19) + 8), "BOM_ENOTSUP"),
+    # more than 65,535 row ranges of 128 rows, with few columns
+    (dict(n_rows=128 * 65535 + 1, n_cols=8, ldx=8), "BOM_ENOTSUP"),
+    # sizes whose product would overflow 64 bits are refused, not wrapped
+    (dict(n_rows=1 << 40, n_cols=(1 << 62) + 1, ldx=(1 << 62) + 1), "BOM_ENOTSUP"),
+    (dict(n_rows=(1 << 62) + 1, n_cols=8, ldx=8), "BOM_ENOTSUP"),
 ])
 def test_bom_colsum_noalloc_checks(built, over, code):
     a = dict(x=ALIGNED, dtype=B.BOM_BF16, ldx=64, n_rows=256, n_cols=64, weights=None, out=ALIGNED, stream=0)

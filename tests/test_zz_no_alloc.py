@@ -1,8 +1,14 @@
-"""bom_colsum_noalloc: the allocation-free column sum, for callers that may not
-allocate device memory (stream capture in global mode, externally managed
-device memory).  Its result must match the library's GEMM entry point
-bom_gemm_bf16 computing the same weighted sum as a 1-row GEMM, on two calls in
-a row that reuse the library's fixed scratch array.
+"""bom_colsum_noalloc: the allocation-free column sum.
+
+Some callers may not allocate device memory at the moment they need this
+reduction: code running while its stream is captured into a CUDA graph in
+global capture mode (where cudaMalloc is an error), and runtimes that hand out
+every device byte from their own pool.  The entry point therefore works out of
+a fixed scratch array inside the library.  Its result is checked here against
+an fp64 numpy sum of the same input values (bf16 or fp32, times fp32 weights),
+on two calls in a row that reuse the shared scratch, on the single-range path
+(at most 128 rows, no finishing launch), at exactly its size limit, and inside
+a global-mode stream capture after a first call outside it.
 
 The file is named to run last, so a failure here cannot hide the results of
 the other GPU tests in a run that stops at the first failure."""
@@ -16,7 +22,9 @@ from tests import _gpu as G
 
 pytestmark = pytest.mark.gpu
 
-TOL = G.TOL["f32"]   # both sides sum exact bf16 x bf16 products in fp32
+# fp32 accumulation over at most 65,536 rows of unit-scale values: relative
+# error far below 1e-5 of the fp64 sum's norm
+TOL = G.TOL["f32"]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -24,39 +32,51 @@ def _built():
     G.ensure_built()
 
 
-def _rup(a, b):
-    return (a + b - 1) // b * b
-
-
-def _case(seed, n, d, weighted):
+def _case(seed, n, d, dtype, weighted):
+    """Device input and weights, with the fp64 reference sum of the exact
+    values the device sees."""
     rng = np.random.default_rng(seed)
-    x_bits = I.bf16_bits(rng.standard_normal((n, d), dtype=np.float32))
-    x = G.to_dev(x_bits)
-    if weighted:
-        # weights exactly representable in bf16, so the GEMM operand is exact too
-        w_bits = I.bf16_bits(rng.standard_normal(n, dtype=np.float32))
+    vals = rng.standard_normal((n, d), dtype=np.float32)
+    if dtype == B.BOM_BF16:
+        bits = I.bf16_bits(vals)
+        x = G.to_dev(bits)
+        x64 = I.bf16_to_f64(bits)
     else:
-        w_bits = I.bf16_bits(np.ones(n, dtype=np.float32))
-    w32 = torch.from_numpy(I.bf16_to_f32(w_bits)).to(G.DEV)
-    # reference through the existing entry point: D[1, d] = w^T X as a GEMM with
-    # A = w (1 x n, K-major) and B = X (d x n, stored MN-major as X itself)
-    lda = _rup(n, 8)
-    a = np.zeros((1, lda), dtype=np.uint16)
-    a[0, :n] = w_bits
-    ref = torch.full((1, _rup(d, 4)), float("nan"), dtype=torch.float32, device=G.DEV)
-    B.bom_gemm_bf16(G.to_dev(a), lda, 0, x, d, 1, ref, ref.shape[1], 1, d, n, 1.0)
-    return x, (w32 if weighted else None), ref[0, :d]
+        x = G.to_dev(vals)
+        x64 = vals.astype(np.float64)
+    w = rng.standard_normal(n).astype(np.float32) if weighted else None
+    ref = (w.astype(np.float64)[:, None] * x64).sum(axis=0) if weighted else x64.sum(axis=0)
+    return x, (torch.from_numpy(w).to(G.DEV) if weighted else None), ref
 
 
-def test_noalloc_colsum_matches_gemm_entry_on_two_calls():
+def _run(x, dtype, n, d, w):
+    out = torch.full((d,), float("nan"), dtype=torch.float32, device=G.DEV)
+    B.bom_colsum_noalloc(x, dtype, d, n, d, w, out)
+    return out
+
+
+@pytest.mark.parametrize("dtype", [B.BOM_BF16, B.BOM_F32])
+def test_noalloc_colsum_matches_fp64_sum_on_two_calls(dtype):
+    # a multi-range call, then a different shape on the same scratch
     cases = [(1, 3001, 520, True), (2, 700, 2048, False)]
+    outs = []
     for seed, n, d, weighted in cases:
-        x, w, ref = _case(seed, n, d, weighted)
-        out = torch.full((d,), float("nan"), dtype=torch.float32, device=G.DEV)
-        B.bom_colsum_noalloc(x, B.BOM_BF16, d, n, d, w, out)
-        torch.cuda.synchronize()
+        x, w, ref = _case(seed, n, d, dtype, weighted)
+        outs.append((_run(x, dtype, n, d, w), ref))
+    torch.cuda.synchronize()
+    for out, ref in outs:
         assert torch.isfinite(out).all()
-        assert G.rel_l2(G.np64(out), G.np64(ref)) < TOL
+        assert G.rel_l2(G.np64(out), ref) < TOL
+
+
+@pytest.mark.parametrize("dtype", [B.BOM_BF16, B.BOM_F32])
+def test_noalloc_colsum_single_range(dtype):
+    """At most 128 rows: one row range, whose blocks write the result directly."""
+    for seed, n, d in ((3, 128, 264), (4, 1, 40), (5, 77, 1024)):
+        x, w, ref = _case(seed, n, d, dtype, True)
+        out = _run(x, dtype, n, d, w)
+        torch.cuda.synchronize()
+        assert G.rel_l2(G.np64(out), ref) < TOL
 
 
 def test_noalloc_colsum_rejects_sizes_beyond_its_scratch():
@@ -70,16 +90,38 @@ def test_noalloc_colsum_rejects_sizes_beyond_its_scratch():
 
 def test_noalloc_colsum_at_the_scratch_limit():
     """ceil(n / 128) * n_cols = 2^20 exactly (65,536 rows x 2,048 columns) is
-    accepted and matches the GEMM entry; one row more is refused."""
+    accepted and matches the fp64 sum; one row more is refused."""
     n, d = 128 * 512, 2048
-    x, _, ref = _case(3, n + 1, d, False)
+    x, _, _ = _case(6, n + 1, d, B.BOM_BF16, False)
     out = torch.full((d,), float("nan"), dtype=torch.float32, device=G.DEV)
     with pytest.raises(B.BomError) as e:
         B.bom_colsum_noalloc(x, B.BOM_BF16, d, n + 1, d, None, out)
     assert e.value.code == B.BOM_ENOTSUP
-    # the first n rows: the reference is the full sum minus the last row
     B.bom_colsum_noalloc(x, B.BOM_BF16, d, n, d, None, out)
     torch.cuda.synchronize()
-    want = G.np64(ref) - G.np64(x[n].float())
+    ref = G.np64(x[:n]).sum(axis=0)
     assert torch.isfinite(out).all()
-    assert G.rel_l2(G.np64(out), want) < TOL
+    assert G.rel_l2(G.np64(out), ref) < TOL
+
+
+def test_noalloc_colsum_inside_a_global_mode_capture():
+    """A first call outside any capture resolves the scratch address on this
+    device; the same call then runs inside a stream capture in global mode
+    (where an allocation would fail the capture) and the replayed graph gives
+    the fp64 sum."""
+    n, d = 2000, 768
+    x, w, ref = _case(7, n, d, B.BOM_BF16, True)
+    out = torch.full((d,), float("nan"), dtype=torch.float32, device=G.DEV)
+    B.bom_colsum_noalloc(x, B.BOM_BF16, d, n, d, w, out)
+    torch.cuda.synchronize()
+    out.fill_(float("nan"))
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="global"):
+        B.bom_colsum_noalloc(x, B.BOM_BF16, d, n, d, w, out)
+    torch.cuda.synchronize()
+    assert torch.isnan(out).all()   # capture executed nothing
+    for _ in range(2):
+        out.fill_(float("nan"))
+        g.replay()
+        torch.cuda.synchronize()
+        assert G.rel_l2(G.np64(out), ref) < TOL
