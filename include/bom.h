@@ -61,8 +61,10 @@ typedef enum {
     BOM_EEMPTY = 5,    /* device: N_t = 0 (Algorithm 1 requires N_t > 0)              */
     BOM_ETIMEOUT = 6,  /* device: a bounded wait inside a kernel ran out              */
     BOM_ENOTSUP = 7,   /* shape or alignment this build does not handle               */
-    BOM_ENONFINITE = 8 /* a row's log-sum-exp or its label logit is not finite
-                          (device-detected before any state is written)              */
+    BOM_ENONFINITE = 8, /* a row's log-sum-exp or its label logit is not finite
+                           (device-detected before any state is written)             */
+    BOM_ESHARD = 9      /* device: another row shard of a sharded step latched an
+                           error (bom_step_shard_end), so this shard stopped too   */
 } bom_status;
 
 typedef enum { BOM_F32 = 0, BOM_BF16 = 1 } bom_dtype;
@@ -159,6 +161,58 @@ int64_t bom_workspace_bytes(const bom_config* cfg);
 bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
                     void* const* params, float* q, int64_t t,
                     void* const* grads, void* const* h_out, void* stream);
+
+/* Row-sharded step: the data-parallel split of bom_step at its one exchange
+ * (Algorithm 1: s_t is the mean of r_i over the supervised set I_t of the
+ * whole batch, and the surrogate's N_t^-1 is the same count; LM construction
+ * appendix: ignored targets leave both means).  A batch split by rows over
+ * several handles (one per rank, or several on one GPU) computes the step of
+ * the whole batch in two calls per shard, with one sum of a small vector
+ * between them:
+ *
+ *   bom_step_shard_begin  forward of this shard's rows, logits, row
+ *                         log-sum-exp and residuals R (kept in the handle's
+ *                         workspace), then this shard's part of the exchange
+ *                         vector xch, fp64 [d_out + 3]:
+ *                           xch[j]         sum_{i in I_t^shard} r_ij, j < d_out
+ *                           xch[d_out]     sum_{i in I_t^shard} CE_i
+ *                           xch[d_out + 1] |I_t^shard| (an integer value)
+ *                           xch[d_out + 2] 1 if this shard latched a device
+ *                                          error, else 0 (then the sums are 0)
+ *                         A shard may hold no supervised row.
+ *   the caller            sums the shards' vectors elementwise (one
+ *                         all-reduce of d_out + 3 doubles across ranks), so
+ *                         that every shard receives the same summed vector;
+ *   bom_step_shard_end    from the summed vector: N_t, s_t, the loss,
+ *                         q_t = beta1 q_{t-1} + (1-beta1) s_t and qhat_t (every
+ *                         shard forms the same q), then the backward of this
+ *                         shard's rows with the cotangent
+ *                         N_t^-1 [(1-lambda) r_i + lambda qhat_t].  grads[] (and
+ *                         h_out[]) receive this shard's share of u (of g and
+ *                         h): the shares of all shards sum to the whole
+ *                         batch's u, which is the caller's gradient all-reduce
+ *                         (the head's rank-1 term uses this shard's
+ *                         colsum_{I_t^shard}(H); the head bias share is
+ *                         (1-lambda) s^shard + lambda (N_t^shard / N_t) qhat).
+ *
+ * Both calls take the arguments of bom_step (x, labels, n_rows, params: the
+ * same buffers and values in both, unchanged in between); begin takes no q,
+ * t or outputs.  One handle per shard; nothing else may run on the handle
+ * between the two calls.  begin clears the handle's status word, end keeps
+ * it: a device error of begin (bad label, non-finite logits) stops this
+ * shard's end, and through xch[d_out + 2] every other shard's end with
+ * BOM_ESHARD; a whole batch without supervised rows latches BOM_EEMPTY in
+ * every shard.  q (and the device step counter) change only in an end whose
+ * status stays clear.  With bom_set_step_scalars, end reads t there and
+ * advances it.  Not with the fused update or an own-step output registered
+ * (BOM_EINVAL): the update follows the caller's gradient sum.
+ *   xch     device fp64 [d_out + 3], 8-byte aligned (BOM_ENOTSUP otherwise);
+ *           begin writes it, end reads it. */
+bom_status bom_step_shard_begin(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                                void* const* params, double* xch, void* stream);
+bom_status bom_step_shard_end(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                              void* const* params, float* q, int64_t t, const double* xch,
+                              void* const* grads, void* const* h_out, void* stream);
 
 /* Fused BOM-AdamW update (Section 3.4; Algorithm 1, last two steps) inside
  * bom_step.  Registers, per parameter tensor, its fp32 master weights theta[k]

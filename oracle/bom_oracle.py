@@ -354,6 +354,86 @@ def head_input_grad_rows(R, W, valid, qhat, n_t, lam, token_rows):
     return mix_cotangent_rows(R, valid, qhat, n_t, lam, token_rows) @ np.asarray(W, dtype=F64)
 
 
+def mix_grad_rows(layers, head_bias, params, saved, R, valid, qhat, n_t, lam, rows):
+    """Sampled output rows of u = (1 - lambda) g + lambda Jbar^T qhat for EVERY
+    parameter tensor (Eq. mix-gradient), for full-size checks of a whole
+    network where `backward` would form every weight gradient in full.
+
+    The reverse pass is the one of `backward`, with the L_mix logit cotangent
+    dZ = N_t^-1 [(1 - lambda) R + lambda 1_{I_t} qhat^T] (Eq. mix-objective,
+    differentiated in the logits), walked from the head down:
+      head input:  dZ W = N_t^-1 [(1 - lambda) R W + lambda 1_{I_t} (W^T qhat)^T]
+                   over every row (dZ itself is never formed);
+      SwiGLU:      dW_d = dy^T A, dA = dy W_d, dG = dA * U * SiLU'(G),
+                   dU = dA * SiLU(G), dW_g = dG^T x, dW_u = dU^T x,
+                   dx = dy + dG W_g + dU W_u;
+      Linear(+GELU): dpre = dx (* GELU'(pre)), dW = dpre^T x, db = sum_i dpre_i,
+                   dx = dpre W;
+      RMSNorm:     dgamma = sum_i dy_i * xhat_i, dx = r (dy gamma - xhat
+                   mean_j(dy_j gamma_j xhat_j)).
+    Every cotangent is carried over all rows; a weight gradient is formed only
+    on its sampled output rows.  rows[k] lists, for tensor k (interface order),
+    the output rows of a matrix (row j of dW is column j of the layer's output
+    cotangent contracted with its input) or the elements of a vector.  The
+    input cotangent of the first layer is not needed and not formed.
+    Returns one array per tensor: [len(rows[k]), cols] or [len(rows[k])]."""
+    per_layer, (hw, hb) = _split_params(layers, head_bias, params)
+    tape, h_last = saved
+    R = np.asarray(R, dtype=F64)
+    qhat = np.asarray(qhat, dtype=F64)
+    vf = np.asarray(valid, dtype=F64)
+    a, b = (1.0 - lam) / n_t, lam / n_t
+    out: List[np.ndarray] = [None] * len(params)
+    k = len(params) - 1
+    if hb is not None:
+        rb = np.asarray(rows[k])
+        # sum_i dZ_ij = a sum_{i in I_t} r_ij + b N_t qhat_j (R is zero off I_t)
+        out[k] = a * R[:, rb].sum(axis=0) + b * n_t * qhat[rb]
+        k -= 1
+    rw = np.asarray(rows[k])
+    out[k] = (a * R[:, rw] + b * vf[:, None] * qhat[None, rw]).T @ h_last
+    k -= 1
+    hw = np.asarray(hw, dtype=F64)
+    dx = a * (R @ hw) + b * vf[:, None] * (hw.T @ qhat)[None, :]
+    for li in range(len(layers) - 1, -1, -1):
+        kind = layers[li][0]
+        rec = tape[li]
+        below = li > 0
+        if kind == "swiglu":
+            wg, wu, wd = per_layer[li]
+            _, x, G, U, A = rec
+            dy = dx
+            out[k] = dy[:, np.asarray(rows[k])].T @ A
+            dA = dy @ wd
+            dG = dA * U * silu_prime(G)
+            dU = dA * silu(G)
+            del dA
+            out[k - 1] = dU[:, np.asarray(rows[k - 1])].T @ x
+            out[k - 2] = dG[:, np.asarray(rows[k - 2])].T @ x
+            k -= 3
+            dx = dy + dG @ wg + dU @ wu if below else None
+        elif kind == "rmsnorm":
+            (gamma,) = per_layer[li]
+            _, x, r, xhat = rec
+            rg = np.asarray(rows[k])
+            out[k] = (dx[:, rg] * xhat[:, rg]).sum(axis=0)
+            k -= 1
+            if below:
+                dxhat = dx * gamma
+                dx = r * (dxhat - xhat * np.mean(dxhat * xhat, axis=1, keepdims=True))
+        else:
+            w, bias = per_layer[li]
+            _, x, pre = rec
+            dpre = dx * gelu_prime(pre) if kind == "linear_gelu" else dx
+            if bias is not None:
+                out[k] = dpre[:, np.asarray(rows[k])].sum(axis=0)
+                k -= 1
+            out[k] = dpre[:, np.asarray(rows[k])].T @ x
+            k -= 1
+            dx = dpre @ w if below else None
+    return out
+
+
 # --------------------------------------------------------------------------
 # Drift telemetry and the own-step control (Section 3.3, Eq. jacobian-drift
 # and Eq. drift-telemetry; stale-control and drift-measurement appendices).

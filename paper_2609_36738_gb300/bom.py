@@ -20,13 +20,15 @@ from . import inputs as _inputs
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", "libbom.so")
 
-BOM_OK, BOM_EINVAL, BOM_ENOMEM, BOM_ECUDA, BOM_ELABEL, BOM_EEMPTY, BOM_ETIMEOUT, BOM_ENOTSUP, BOM_ENONFINITE = range(9)
+(BOM_OK, BOM_EINVAL, BOM_ENOMEM, BOM_ECUDA, BOM_ELABEL, BOM_EEMPTY, BOM_ETIMEOUT, BOM_ENOTSUP, BOM_ENONFINITE,
+ BOM_ESHARD) = range(10)
 BOM_F32, BOM_BF16 = 0, 1
 BOM_LAYER_LINEAR, BOM_LAYER_LINEAR_GELU, BOM_LAYER_SWIGLU, BOM_LAYER_RMSNORM = 0, 1, 2, 3
 BOM_OUT_U, BOM_OUT_G_AND_H = 0, 1
 
 # Every symbol include/bom.h declares.
 EXPORTED = ("bom_param_count", "bom_param_shape", "bom_init", "bom_workspace_bytes", "bom_step",
+            "bom_step_shard_begin", "bom_step_shard_end",
             "bom_set_input_grad", "bom_step_outputs", "bom_get_stats", "bom_update", "bom_gemm_bf16", "bom_trace", "bom_trace_read",
             "bom_launch_count", "bom_colsum_noalloc", "bom_set_own_step_output", "bom_own_step_moment",
             "bom_stats_transfer_bytes", "bom_update_blockshared", "bom_sqnorm", "bom_update_clipped",
@@ -82,6 +84,10 @@ def lib() -> C.CDLL:
     L.bom_workspace_bytes.restype = i64
     L.bom_step.argtypes = [vp, vp, vp, i64, C.POINTER(vp), vp, i64, C.POINTER(vp), C.POINTER(vp), vp]
     L.bom_step.restype = i32
+    L.bom_step_shard_begin.argtypes = [vp, vp, vp, i64, C.POINTER(vp), vp, vp]
+    L.bom_step_shard_begin.restype = i32
+    L.bom_step_shard_end.argtypes = [vp, vp, vp, i64, C.POINTER(vp), vp, i64, vp, C.POINTER(vp), C.POINTER(vp), vp]
+    L.bom_step_shard_end.restype = i32
     L.bom_set_input_grad.argtypes = [vp, vp]
     L.bom_set_input_grad.restype = i32
     L.bom_step_outputs.argtypes = [vp, C.POINTER(vp), C.POINTER(vp), C.POINTER(vp)]
@@ -214,6 +220,22 @@ def bom_step(h, x, labels, n_rows: int, params, q, t: int, grads, h_out=None, st
     H = (C.c_void_p * n)(*[_ptr(p) for p in h_out]) if h_out is not None else None
     _check(lib().bom_step(h, _ptr(x), _ptr(labels), int(n_rows), P, _ptr(q), int(t), G,
                           H if H is not None else None, _stream(stream)), "bom_step")
+
+
+def bom_step_shard_begin(h, x, labels, n_rows: int, params, xch, stream=None) -> None:
+    n = len(params)
+    P = (C.c_void_p * n)(*[_ptr(p) for p in params])
+    _check(lib().bom_step_shard_begin(h, _ptr(x), _ptr(labels), int(n_rows), P, _ptr(xch), _stream(stream)),
+           "bom_step_shard_begin")
+
+
+def bom_step_shard_end(h, x, labels, n_rows: int, params, q, t: int, xch, grads, h_out=None, stream=None) -> None:
+    n = len(params)
+    P = (C.c_void_p * n)(*[_ptr(p) for p in params])
+    G = (C.c_void_p * n)(*[_ptr(g) for g in grads]) if grads is not None else None
+    H = (C.c_void_p * n)(*[_ptr(p) for p in h_out]) if h_out is not None else None
+    _check(lib().bom_step_shard_end(h, _ptr(x), _ptr(labels), int(n_rows), P, _ptr(q), int(t), _ptr(xch), G, H,
+                                    _stream(stream)), "bom_step_shard_end")
 
 
 def bom_set_step_scalars(h, t_dev, lr_dev=None) -> None:

@@ -100,6 +100,8 @@ struct bom_handle {
     float* splitk = nullptr; // fp32 partial tiles of split-K GEMMs
     int64_t splitk_elems = 0;
     int64_t last_n = 0;
+    int64_t shard_n = 0;     // rows of the first half of a sharded step (0: none pending)
+    float* sshard = nullptr; // this shard's s^shard = N_t^-1 sum_{i in I_t^shard} r_i (sharded steps)
     // tracing: one event pair per launch of the current step
     struct TraceRec {
         const char* name = nullptr;
@@ -220,6 +222,7 @@ size_t carve(bom_handle* h, char* base) {
     h->colpart = static_cast<float*>(c.take(resid_blocks(n) * V * 4));
     h->s = static_cast<float*>(c.take(V * 4));
     h->qhat = static_cast<float*>(c.take(V * 4));
+    h->sshard = static_cast<float*>(c.take(V * 4));
     h->cvec = static_cast<float*>(c.take(h->d_model * 4));
     h->wvec = static_cast<float*>(c.take(h->d_model * 4));
     h->wsvec = static_cast<float*>(c.take(h->d_model * 4));
@@ -455,30 +458,65 @@ void bom_destroy(bom_handle* h) {
     delete h;
 }
 
-bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t n, void* const* params, float* q,
-                    int64_t t, void* const* grads, void* const* h_out, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// The three uses of one step body: a whole step, and the two halves of a
+// row-sharded step around the caller's sum of the exchange vector.
+enum StepPart { kStepFull = 0, kShardBegin = 1, kShardEnd = 2 };
+
+bom_status check_step_args(bom_handle* h, const void* x, const int32_t* labels, int64_t n, void* const* params,
+                           const float* q, int64_t t, void* const* grads, void* const* h_out, int part) {
     const bool fused = h != nullptr && h->fused_upd;
-    if (!h || !x || !labels || !params || !q || (!grads && !fused)) return BOM_EINVAL;
-    if (n < 1 || n > h->cfg.max_rows || (t < 1 && h->t_dev == nullptr)) return BOM_EINVAL;
+    if (!h || !x || !labels || !params) return BOM_EINVAL;
+    if (n < 1 || n > h->cfg.max_rows) return BOM_EINVAL;
+    // a sharded step's update follows the caller's gradient sum, and the
+    // own-step telemetry needs every row's residual norm
+    if (part != kStepFull && (fused || !h->own_out.empty())) return BOM_EINVAL;
+    const int np = bom_param_count(&h->cfg);
+    if (part == kShardBegin) {
+        for (int i = 0; i < np; ++i) {
+            if (!params[i]) return BOM_EINVAL;
+            if (!aligned16(params[i])) return BOM_ENOTSUP;
+        }
+        return aligned16(x) ? BOM_OK : BOM_ENOTSUP;
+    }
+    if (!q || (!grads && !fused)) return BOM_EINVAL;
+    if (t < 1 && h->t_dev == nullptr) return BOM_EINVAL;
     const bool gh = h->cfg.out_mode == BOM_OUT_G_AND_H;
     if (gh != (h_out != nullptr)) return BOM_EINVAL;
     // the fused update consumes u: one u pass and nothing else that needs it
     if (fused && (gh || !h->own_out.empty())) return BOM_EINVAL;
-    const int np = bom_param_count(&h->cfg);
     for (int i = 0; i < np; ++i) {
         if (!params[i] || (!fused && !grads[i]) || (gh && !h_out[i])) return BOM_EINVAL;
         if (!aligned16(params[i]) || (!fused && !aligned16(grads[i])) || (gh && !aligned16(h_out[i])))
             return BOM_ENOTSUP;
     }
     if (!aligned16(x) || !aligned16(q)) return BOM_ENOTSUP;
+    return BOM_OK;
+}
 
+// One step (part = kStepFull), or one half of a row-sharded step: kShardBegin
+// runs the forward and the residual pass and writes this shard's exchange
+// vector to xch_out; kShardEnd reads the summed vector xch_in and runs the
+// rest (s_t, q_t, qhat_t, the backward of this shard's rows).  Arguments are
+// checked by the caller.
+bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_t n, void* const* params, float* q,
+                     int64_t t, void* const* grads, void* const* h_out, void* stream, int part, double* xch_out,
+                     const double* xch_in) {
+    const bool fused = h->fused_upd;
+    const bool gh = h->cfg.out_mode == BOM_OUT_G_AND_H;
+    const bool shard = part != kStepFull;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const NvtxRange nvtx_step("bom_step");
     const bom_config& cfg = h->cfg;
     const int64_t V = cfg.d_out, dm = h->d_model;
     const int cf32 = h->bf16 ? 0 : 1;
     h->last_n = n;
-    h->trace_n = 0;
+    // a traced sharded step records both halves
+    if (part != kShardEnd) h->trace_n = 0;
+    // the second half of a sharded step needs the first half's rows in the workspace
+    h->shard_n = part == kShardBegin ? n : 0;
     int rc = BOM_OK;
 #define BOM_TRY(expr)                                     \
     do {                                                  \
@@ -486,26 +524,37 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
         if (rc != BOM_OK) return static_cast<bom_status>(rc); \
     } while (0)
 
-    if (cudaMemsetAsync(&h->sc->status, 0, sizeof(int32_t), s) != cudaSuccess) return BOM_ECUDA;
     // step scalars: from the host t and lr, or from the device step counter
+    // (a shard's first half has no t: its scalars are set by the second)
     StepScalarsIn st{};
     st.lr = fused ? h->upd_lr : 0.0f;
-    st.inv_bc1 = h->t_dev ? 0.0f : inv_bias_correction(cfg.beta1, t);
+    st.inv_bc1 = (h->t_dev || part == kShardBegin) ? 0.0f : inv_bias_correction(cfg.beta1, t);
     st.inv_bc2 = (fused && !h->t_dev) ? inv_bias_correction(h->upd_beta2, t) : 0.0f;
-    st.t_dev = h->t_dev;
+    st.t_dev = part == kShardBegin ? nullptr : h->t_dev;
     st.lr_dev = h->lr_dev;
     st.beta1 = cfg.beta1;
     st.beta2 = fused ? h->upd_beta2 : 0.0f;
-    BOM_TRACED("labels_scan", 0, 4.0 * n,
-               launch_labels_scan(labels, n, V, cfg.ignore_index, cfg.lambda, st, h->sc, s));
+    if (part != kShardEnd) {   // the second half keeps the status word of the first
+        if (cudaMemsetAsync(&h->sc->status, 0, sizeof(int32_t), s) != cudaSuccess) return BOM_ECUDA;
+        BOM_TRACED("labels_scan", 0, 4.0 * n,
+                   launch_labels_scan(labels, n, V, cfg.ignore_index, cfg.lambda, st, h->sc, s, shard));
+    }
 
     // ---------------------------------------------------------------- forward
+    // (the second half of a sharded step finds the activations, R and the
+    // residual pass's column partials of its rows in the workspace)
+    const bool run_fwd = part != kShardEnd;
     const void* xin = x;
     int pi = 0;
     std::vector<int> pidx(h->lw.size());
     for (size_t l = 0; l < h->lw.size(); ++l) {
         LayerWs& L = h->lw[l];
         pidx[l] = pi;
+        if (!run_fwd) {
+            pi += L.kind == BOM_LAYER_SWIGLU ? 3 : (L.kind == BOM_LAYER_RMSNORM ? 1 : (L.bias ? 2 : 1));
+            xin = L.out;
+            continue;
+        }
         if (L.kind == BOM_LAYER_SWIGLU) {
             const void* Wg = params[pi];
             const void* Wu = params[pi + 1];
@@ -555,7 +604,7 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
     const void* Wh = params[pi++];
     const int head_b = cfg.head_bias ? pi++ : -1;
     const void* bh = head_b >= 0 ? params[head_b] : nullptr;
-    {
+    if (run_fwd) {
         GemmDesc g = gemm1(n, V, dm, kmaj(xin, dm), kmaj(Wh, dm));
         g.epi_kind = EPI_LOGITS;
         g.epi.bias = bh;
@@ -566,24 +615,41 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
         g.epi.ld_stats = h->ntiles;
         BOM_TRY(run_gemm(h, g, s));
     }
-    if (!h->bf16)
+    if (run_fwd && !h->bf16)
         BOM_TRACED("row_stats_f32", 0, 4.0 * n * V,
                    launch_row_stats_f32(static_cast<const float*>(h->Z), h->ldz, n, V, h->stats, h->sc, s));
 
     // ---------------------------------------------------------------- task space
-    BOM_TRACED("row_lse", 0, 8.0 * n * h->ntiles + 12.0 * n,
-               launch_row_lse(h->Z, cf32, h->ldz, n, V, h->stats, h->ntiles, labels, cfg.ignore_index, h->lse,
-                              h->ce, h->sc, s));
-    // residual pass: reads and rewrites Z once, writes the column partial sums
-    BOM_TRACED("residual", 0, 2.0 * h->esz * n * h->ldz + 4.0 * resid_blocks(n) * V + 8.0 * n,
-               launch_residual(h->Z, cf32, h->ldz, n, V, h->lse, labels, cfg.ignore_index, h->colpart, h->sc, s));
-    BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 20.0 * V,
-               launch_finish_sq(h->colpart, resid_blocks(n), V, cfg.beta1, q, h->s, h->qhat, h->sc, s));
+    if (run_fwd) {
+        BOM_TRACED("row_lse", 0, 8.0 * n * h->ntiles + 12.0 * n,
+                   launch_row_lse(h->Z, cf32, h->ldz, n, V, h->stats, h->ntiles, labels, cfg.ignore_index, h->lse,
+                                  h->ce, h->sc, s));
+        // residual pass: reads and rewrites Z once, writes the column partial sums
+        BOM_TRACED("residual", 0, 2.0 * h->esz * n * h->ldz + 4.0 * resid_blocks(n) * V + 8.0 * n,
+                   launch_residual(h->Z, cf32, h->ldz, n, V, h->lse, labels, cfg.ignore_index, h->colpart, h->sc,
+                                   s));
+    }
+    if (part == kShardBegin) {   // this shard's sums, for the caller's exchange
+        BOM_TRACED("shard_sums", 0, 4.0 * resid_blocks(n) * V + 4.0 * n + 8.0 * (V + 3),
+                   launch_shard_sums(h->colpart, resid_blocks(n), h->ce, n, V, xch_out, h->sc, s));
+        return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+    }
+    if (part == kShardEnd) {
+        BOM_TRACED("shard_scalars", 0, 8.0 * 3, launch_shard_scalars_in(xch_in, V, cfg.lambda, st, h->sc, s));
+        BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 8.0 * V + 24.0 * V,
+                   launch_shard_finish_sq(xch_in, h->colpart, resid_blocks(n), V, cfg.beta1, q, h->s, h->qhat,
+                                          h->sshard, h->sc, s));
+    } else {
+        BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 20.0 * V,
+                   launch_finish_sq(h->colpart, resid_blocks(n), V, cfg.beta1, q, h->s, h->qhat, h->sc, s));
+    }
     const bool own = !h->own_out.empty();
     if (own)   // per-row residual norms for the cancellation ratio
         BOM_TRACED("row_norm", 2.0 * n * V, h->esz * n * h->ldz + 4.0 * n,
                    launch_row_norm(h->Z, cf32, h->ldz, n, V, h->rnorm, h->sc, s));
-    BOM_TRACED("scalars", 0, 4.0 * (n + V), launch_scalars(h->ce, n, h->s, V, own ? h->rnorm : nullptr, h->sc, s));
+    // (a sharded step's loss comes from the shards' summed CE)
+    BOM_TRACED("scalars", 0, 4.0 * (n + V),
+               launch_scalars(shard ? nullptr : h->ce, n, h->s, V, own ? h->rnorm : nullptr, h->sc, s));
     // c = colsum_{I_t}(H) and w = W^T qhat (the rank-1 / broadcast factors of the reprojection)
     BOM_TRACED("colsum", 2.0 * n * dm, h->esz * n * dm,
                launch_colsum(xin, cf32, dm, n, dm, labels, cfg.ignore_index, nullptr, 1.0f, h->part, h->cvec, 1,
@@ -691,9 +757,13 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
         if (head_b >= 0) {
             const float a = pass == 0 ? 1.0f - cfg.lambda : (pass == 1 || pass == 3 ? 1.0f : 0.0f);
             const float b = pass == 0 ? cfg.lambda : (pass == 2 ? 1.0f : 0.0f);
-            BOM_TRACED("axpby", 3.0 * V, 12.0 * V,
-                       launch_axpby(h->s, h->qhat, a, b, V, fused ? h->ubuf : outp[head_b], fused ? 1 : of32, h->sc,
-                                    s));
+            if (shard)   // this shard's share: a s^shard + b (N_t^shard / N_t) qhat
+                BOM_TRACED("axpby", 3.0 * V, 12.0 * V,
+                           launch_shard_bias(h->sshard, h->qhat, a, b, V, outp[head_b], of32, h->sc, s));
+            else
+                BOM_TRACED("axpby", 3.0 * V, 12.0 * V,
+                           launch_axpby(h->s, h->qhat, a, b, V, fused ? h->ubuf : outp[head_b], fused ? 1 : of32,
+                                        h->sc, s));
             if (fused) BOM_TRY(update_small(head_b, V));
         }
         for (int l = static_cast<int>(h->lw.size()) - 1; l >= 0; --l) {
@@ -828,6 +898,39 @@ bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t
     if (h->t_dev) launch_advance_step(h->t_dev, h->sc, s);
 #undef BOM_TRY
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+bom_status bom_step(bom_handle* h, const void* x, const int32_t* labels, int64_t n, void* const* params, float* q,
+                    int64_t t, void* const* grads, void* const* h_out, void* stream) {
+    const bom_status rc = check_step_args(h, x, labels, n, params, q, t, grads, h_out, kStepFull);
+    if (rc != BOM_OK) return rc;
+    const NvtxRange nvtx_step("bom_step");
+    return step_impl(h, x, labels, n, params, q, t, grads, h_out, stream, kStepFull, nullptr, nullptr);
+}
+
+bom_status bom_step_shard_begin(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                                void* const* params, double* xch, void* stream) {
+    const bom_status rc = check_step_args(h, x, labels, n_rows, params, nullptr, 1, nullptr, nullptr, kShardBegin);
+    if (rc != BOM_OK) return rc;
+    if (!xch) return BOM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(xch) & 7u) != 0) return BOM_ENOTSUP;
+    const NvtxRange nvtx_step("bom_step_shard_begin");
+    return step_impl(h, x, labels, n_rows, params, nullptr, 1, nullptr, nullptr, stream, kShardBegin, xch, nullptr);
+}
+
+bom_status bom_step_shard_end(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                              void* const* params, float* q, int64_t t, const double* xch, void* const* grads,
+                              void* const* h_out, void* stream) {
+    const bom_status rc = check_step_args(h, x, labels, n_rows, params, q, t, grads, h_out, kShardEnd);
+    if (rc != BOM_OK) return rc;
+    if (!xch || n_rows != h->shard_n) return BOM_EINVAL;   // no matching first half
+    if ((reinterpret_cast<uintptr_t>(xch) & 7u) != 0) return BOM_ENOTSUP;
+    const NvtxRange nvtx_step("bom_step_shard_end");
+    return step_impl(h, x, labels, n_rows, params, q, t, grads, h_out, stream, kShardEnd, nullptr, xch);
 }
 
 bom_status bom_set_input_grad(bom_handle* h, void* dx) {
@@ -1100,6 +1203,7 @@ const char* bom_status_string(bom_status s) {
         case BOM_ETIMEOUT: return "BOM_ETIMEOUT: a bounded device wait ran out";
         case BOM_ENOTSUP: return "BOM_ENOTSUP: shape or alignment not supported";
         case BOM_ENONFINITE: return "BOM_ENONFINITE: non-finite logits (row log-sum-exp or label logit)";
+        case BOM_ESHARD: return "BOM_ESHARD: another row shard of the sharded step latched an error";
     }
     return "unknown bom_status";
 }

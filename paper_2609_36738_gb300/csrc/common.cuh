@@ -61,6 +61,10 @@ struct DevScalars {
     float lr;              // learning rate of the fused update
     float inv_bc1;         // 1 / (1 - beta1^t)
     float inv_bc2;         // 1 / (1 - beta2^t)
+    // Row-sharded steps (bom_step_shard_begin / _end): this shard's share of
+    // the supervised rows, N_t^shard / N_t, which scales its share of the
+    // broadcast qhat term of the head bias gradient.
+    float shard_frac;
 };
 // Bytes of DevScalars that bom_get_stats copies to the host (the step scalars stay).
 constexpr size_t kStatsBytes = offsetof(DevScalars, lr);

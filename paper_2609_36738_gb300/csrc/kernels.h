@@ -34,8 +34,9 @@ struct StepScalarsIn {
     const float* lr_dev;
     float beta1, beta2;
 };
+// allow_empty (the first half of a row-sharded step): N_t = 0 is not an error.
 void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda,
-                        const StepScalarsIn& st, DevScalars* sc, cudaStream_t s);
+                        const StepScalarsIn& st, DevScalars* sc, cudaStream_t s, bool allow_empty = false);
 
 // *t_dev += 1 when the step latched no error (the last kernel of a step that
 // reads its t from the device).
@@ -62,7 +63,25 @@ void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, cons
 void launch_finish_sq(const float* colpart, int64_t nblocks, int64_t V, float beta1, float* q,
                       float* s_out, float* qhat, DevScalars* sc, cudaStream_t s);
 
-// loss = N_t^-1 sum_i ce_i, ||s|| and, when rnorm is given, r_norm_mean = N_t^-1 sum_i rnorm_i.
+// Row-sharded step (see bom_step_shard_begin / _end in bom.h).
+// xch[0, V) = fixed-order column sums of colpart, xch[V] = sum_i ce_i,
+// xch[V+1] = this shard's N_t, xch[V+2] = 1 if the status word is set.
+void launch_shard_sums(const float* colpart, int64_t nblocks, const float* ce, int64_t n, int64_t V, double* xch,
+                       const DevScalars* sc, cudaStream_t s);
+// From the summed xch: N_t, 1/N_t, cotangent coefficients, loss, step scalars,
+// shard_frac; latches BOM_ESHARD / BOM_EEMPTY.
+void launch_shard_scalars_in(const double* xch, int64_t V, float lambda, const StepScalarsIn& st, DevScalars* sc,
+                             cudaStream_t s);
+// s = xch / N_t, q EMA, qhat, and s_shard = (this shard's column sums) / N_t.
+void launch_shard_finish_sq(const double* xch, const float* colpart, int64_t nblocks, int64_t V, float beta1,
+                            float* q, float* s_out, float* qhat, float* s_shard, const DevScalars* sc,
+                            cudaStream_t s);
+// out[j] = a s_shard[j] + b shard_frac qhat[j] (this shard's head bias share).
+void launch_shard_bias(const float* s_shard, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
+                       const DevScalars* sc, cudaStream_t s);
+
+// loss = N_t^-1 sum_i ce_i (kept as it is when ce is NULL), ||s|| and, when
+// rnorm is given, r_norm_mean = N_t^-1 sum_i rnorm_i.
 void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, const float* rnorm, DevScalars* sc,
                     cudaStream_t s);
 

@@ -79,8 +79,10 @@ __global__ void advance_step_kernel(int64_t* __restrict__ t, const DevScalars* s
     if (threadIdx.x == 0 && sc->status == 0) *t += 1;
 }
 
+// allow_empty: a row shard of a sharded step may hold no supervised row; only
+// the whole batch's N_t must be positive (checked when the shards' sums meet).
 __global__ void labels_scan_kernel(const int32_t* __restrict__ labels, int64_t n, int64_t V, int32_t ignore,
-                                   float lambda, const StepScalarsIn st, DevScalars* sc) {
+                                   float lambda, const StepScalarsIn st, int allow_empty, DevScalars* sc) {
     pdl_enter();
     __shared__ int s_cnt[32], s_bad[32];
     int cnt = 0, bad = 0;
@@ -109,7 +111,7 @@ __global__ void labels_scan_kernel(const int32_t* __restrict__ labels, int64_t n
         sc->n_t = c;
         if (b > 0)
             latch_status(sc, BOM_ELABEL);
-        else if (c == 0)
+        else if (c == 0 && !allow_empty)
             latch_status(sc, BOM_EEMPTY);
         const float inv = c > 0 ? 1.0f / static_cast<float>(c) : 0.0f;
         sc->inv_nt = inv;
@@ -343,8 +345,10 @@ __global__ void __launch_bounds__(1024) scalars_kernel(const float* __restrict__
     __shared__ float red[32];
     if (sc->status != 0) return;
     float a = 0.0f;
-    for (int64_t i = threadIdx.x; i < n; i += 1024) a += ce[i];
-    a = block_sum<1024>(a, red);
+    if (ce) {
+        for (int64_t i = threadIdx.x; i < n; i += 1024) a += ce[i];
+        a = block_sum<1024>(a, red);
+    }
     float b = 0.0f;
     for (int64_t j = threadIdx.x; j < V; j += 1024) b += s_vec[j] * s_vec[j];
     b = block_sum<1024>(b, red);
@@ -354,7 +358,7 @@ __global__ void __launch_bounds__(1024) scalars_kernel(const float* __restrict__
         c = block_sum<1024>(c, red);
     }
     if (threadIdx.x == 0) {
-        sc->loss = a * sc->inv_nt;
+        if (ce) sc->loss = a * sc->inv_nt;   // else set from the shards' summed CE
         sc->s_norm = sqrtf(b);
         sc->r_norm_mean = c * sc->inv_nt;
     }
@@ -590,13 +594,133 @@ __global__ void axpby_kernel(const float* __restrict__ s, const float* __restric
     st_elem(out, j, out_f32, a * s[j] + b * qh[j]);
 }
 
+// ---------------------------------------------------------------------------
+// Row-sharded step (Algorithm 1's batch mean over I_t split by rows).  A shard
+// writes the sums that couple its rows to the others: the column sums of its
+// residuals, its CE sum, its |I_t^shard| and an error flag, in fp64 so that
+// any number of shards adds them exactly enough (the counts exactly).
+// xch[j] for j < V: sum_{i in I_t^shard} r_ij (the fixed-order fp32 column sum
+// of the residual pass's partials); nothing is read when the shard latched an
+// error (zeros are written).
+__global__ void __launch_bounds__(256) shard_colsum_kernel(const float* __restrict__ colpart, int64_t nblocks,
+                                                           int64_t V, double* __restrict__ xch,
+                                                           const DevScalars* sc) {
+    pdl_enter();
+    __shared__ float red[8][33];
+    const bool ok = sc->status == 0;
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + (threadIdx.x & 31);
+    const float acc = fixed_order_column_sum(colpart, ok ? nblocks : 0, V, j, red);
+    if (threadIdx.x < 32 && j < V) xch[j] = ok ? static_cast<double>(acc) : 0.0;
+}
+
+// xch[V] = sum_{i in I_t^shard} CE_i (fixed order), xch[V+1] = |I_t^shard|,
+// xch[V+2] = 1 when this shard latched an error, else 0.
+__global__ void __launch_bounds__(1024) shard_scalars_out_kernel(const float* __restrict__ ce, int64_t n,
+                                                                 int64_t V, double* __restrict__ xch,
+                                                                 const DevScalars* sc) {
+    pdl_enter();
+    __shared__ float red[32];
+    const bool ok = sc->status == 0;
+    float a = 0.0f;
+    if (ok)
+        for (int64_t i = threadIdx.x; i < n; i += 1024) a += ce[i];
+    a = block_sum<1024>(a, red);
+    if (threadIdx.x == 0) {
+        xch[V] = ok ? static_cast<double>(a) : 0.0;
+        xch[V + 1] = ok ? static_cast<double>(sc->n_t) : 0.0;
+        xch[V + 2] = ok ? 0.0 : 1.0;
+    }
+}
+
+// The second half of a sharded step begins here, from the summed vector:
+// N_t of the whole batch, the cotangent coefficients, the loss, the step
+// scalars and this shard's share N_t^shard / N_t.  Any shard's error stops
+// every shard (BOM_ESHARD where this one had none), and so does N_t = 0.
+__global__ void shard_scalars_in_kernel(const double* __restrict__ xch, int64_t V, float lambda,
+                                        const StepScalarsIn st, DevScalars* sc) {
+    pdl_enter();
+    if (threadIdx.x != 0) return;
+    const int32_t n_loc = sc->n_t;
+    const double nt_d = xch[V + 1];
+    const int64_t nt = nt_d >= 0.0 && nt_d < 4.0e18 ? static_cast<int64_t>(nt_d) : -1;
+    if (xch[V + 2] != 0.0)
+        latch_status(sc, BOM_ESHARD);
+    else if (nt == 0)
+        latch_status(sc, BOM_EEMPTY);
+    else if (nt < 0 || nt > INT32_MAX || static_cast<double>(nt) != nt_d)
+        latch_status(sc, BOM_EINVAL);   // not a sum of row counts
+    const bool ok = sc->status == 0;
+    sc->n_t = ok ? static_cast<int32_t>(nt) : 0;
+    const float inv = ok ? 1.0f / static_cast<float>(nt) : 0.0f;
+    sc->inv_nt = inv;
+    sc->shard_frac = ok ? static_cast<float>(static_cast<double>(n_loc) / nt_d) : 0.0f;
+    sc->coef_r[0] = (1.0f - lambda) * inv;
+    sc->coef_q[0] = lambda * inv;
+    sc->coef_r[1] = inv;
+    sc->coef_q[1] = 0.0f;
+    sc->coef_r[2] = 0.0f;
+    sc->coef_q[2] = inv;
+    sc->coef_r[3] = 0.0f;
+    sc->coef_q[3] = inv;
+    float bc1 = st.inv_bc1, bc2 = st.inv_bc2;
+    if (st.t_dev != nullptr) {
+        const int64_t t = *st.t_dev;
+        if (t < 1) {
+            latch_status(sc, BOM_EINVAL);
+        } else {
+            bc1 = inv_bias_correction(st.beta1, t);
+            bc2 = inv_bias_correction(st.beta2, t);
+        }
+    }
+    sc->lr = st.lr_dev != nullptr ? *st.lr_dev : st.lr;
+    sc->inv_bc1 = bc1;
+    sc->inv_bc2 = bc2;
+    sc->loss = ok ? static_cast<float>(xch[V] / nt_d) : 0.0f;
+    sc->s_norm = 0.0f;
+    sc->r_norm_mean = 0.0f;
+}
+
+// s_j = N_t^-1 xch[j], q_j <- beta1 q_j + (1-beta1) s_j, qhat_j = q_j / (1-beta1^t)
+// from the summed vector (every shard forms the same q), and this shard's
+// share s^shard_j = N_t^-1 sum_{i in I_t^shard} r_ij from its own partials.
+__global__ void __launch_bounds__(256) shard_finish_sq_kernel(const double* __restrict__ xch,
+                                                              const float* __restrict__ colpart, int64_t nblocks,
+                                                              int64_t V, float beta1, float* __restrict__ q,
+                                                              float* __restrict__ s_out, float* __restrict__ qhat,
+                                                              float* __restrict__ s_shard, const DevScalars* sc) {
+    pdl_enter();
+    __shared__ float red[8][33];
+    if (sc->status != 0) return;
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + (threadIdx.x & 31);
+    const float loc = fixed_order_column_sum(colpart, nblocks, V, j, red);
+    if (threadIdx.x >= 32 || j >= V) return;
+    const float inv = sc->inv_nt;
+    const float s = static_cast<float>(xch[j]) * inv;
+    const float qn = beta1 * q[j] + (1.0f - beta1) * s;
+    q[j] = qn;
+    s_out[j] = s;
+    qhat[j] = qn * sc->inv_bc1;
+    s_shard[j] = loc * inv;
+}
+
+// This shard's share of the head bias numerator: a s^shard + b (N_t^shard / N_t) qhat.
+__global__ void shard_bias_kernel(const float* __restrict__ s_shard, const float* __restrict__ qh, float a, float b,
+                                  int64_t V, void* __restrict__ out, int out_f32, const DevScalars* sc) {
+    pdl_enter();
+    if (sc->status != 0) return;
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (j >= V) return;
+    st_elem(out, j, out_f32, a * s_shard[j] + b * sc->shard_frac * qh[j]);
+}
+
 inline unsigned cdiv(int64_t a, int64_t b) { return static_cast<unsigned>((a + b - 1) / b); }
 
 }  // namespace
 
 void launch_labels_scan(const int32_t* labels, int64_t n, int64_t V, int32_t ignore, float lambda,
-                        const StepScalarsIn& st, DevScalars* sc, cudaStream_t s) {
-    launch_k(labels_scan_kernel, dim3(1), dim3(1024), 0, s, labels, n, V, ignore, lambda, st, sc); count_launch();
+                        const StepScalarsIn& st, DevScalars* sc, cudaStream_t s, bool allow_empty) {
+    launch_k(labels_scan_kernel, dim3(1), dim3(1024), 0, s, labels, n, V, ignore, lambda, st, allow_empty ? 1 : 0, sc);
+    count_launch();
 }
 
 void launch_advance_step(int64_t* t_dev, const DevScalars* sc, cudaStream_t s) {
@@ -723,6 +847,34 @@ void launch_colsum2(const void* X, const void* Y, int x_f32, int64_t ldx, int64_
 void launch_axpby(const float* s_vec, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
                   const DevScalars* sc, cudaStream_t s) {
     launch_k(axpby_kernel, dim3(cdiv(V, 256)), dim3(256), 0, s, s_vec, qhat, a, b, V, out, out_f32, sc); count_launch();
+}
+
+void launch_shard_sums(const float* colpart, int64_t nblocks, const float* ce, int64_t n, int64_t V, double* xch,
+                       const DevScalars* sc, cudaStream_t s) {
+    launch_k(shard_colsum_kernel, dim3(cdiv(V, 32)), dim3(256), 0, s, colpart, nblocks, V, xch, sc);
+    count_launch();
+    launch_k(shard_scalars_out_kernel, dim3(1), dim3(1024), 0, s, ce, n, V, xch, sc);
+    count_launch();
+}
+
+void launch_shard_scalars_in(const double* xch, int64_t V, float lambda, const StepScalarsIn& st, DevScalars* sc,
+                             cudaStream_t s) {
+    launch_k(shard_scalars_in_kernel, dim3(1), dim3(32), 0, s, xch, V, lambda, st, sc);
+    count_launch();
+}
+
+void launch_shard_finish_sq(const double* xch, const float* colpart, int64_t nblocks, int64_t V, float beta1,
+                            float* q, float* s_out, float* qhat, float* s_shard, const DevScalars* sc,
+                            cudaStream_t s) {
+    launch_k(shard_finish_sq_kernel, dim3(cdiv(V, 32)), dim3(256), 0, s, xch, colpart, nblocks, V, beta1, q, s_out,
+             qhat, s_shard, sc);
+    count_launch();
+}
+
+void launch_shard_bias(const float* s_shard, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
+                       const DevScalars* sc, cudaStream_t s) {
+    launch_k(shard_bias_kernel, dim3(cdiv(V, 256)), dim3(256), 0, s, s_shard, qhat, a, b, V, out, out_f32, sc);
+    count_launch();
 }
 
 }  // namespace bom

@@ -49,7 +49,8 @@ class GpuBom:
         self.wl = wl
         self.out_mode = out_mode
         self.model = B.BomModel(B.config_for(wl, lam, beta1, out_mode, max_rows))
-        self.params = [to_dev(p) for p in params_np]
+        # numpy parameters are uploaded; device tensors are copied
+        self.params = [p.clone() if isinstance(p, torch.Tensor) else to_dev(p) for p in params_np]
         self.q = torch.zeros(wl.vocab, dtype=torch.float32, device=DEV)
 
     def step(self, x_np, y_np, t, check=True):

@@ -35,9 +35,9 @@ def test_library_exports_every_declared_symbol(built):
 
 
 def test_status_strings(built):
-    for code in range(B.BOM_ENONFINITE + 1):
+    for code in range(B.BOM_ESHARD + 1):
         assert B.status_string(code).startswith("BOM_")
-    assert B.status_string(B.BOM_ENONFINITE + 1) == "unknown bom_status"
+    assert B.status_string(B.BOM_ESHARD + 1) == "unknown bom_status"
 
 
 def test_param_layout_matches_workload_description(built):

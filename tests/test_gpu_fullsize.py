@@ -2,11 +2,12 @@
 
 The fp64 oracle runs the full forward and the task-space pass (s_t, q_t,
 qhat_t, CE, row log-sum-exp) on every row.  Where its full reverse pass would
-take too long in fp64, it computes sampled rows of the head weight gradient
-and of the head-input cotangent, and the tests check properties that hold at
-any size: the vocabulary-column sums of u_W vanish (rows of R and qhat sum to
-zero), and one backward of the mixed cotangent equals the mix of the two
-separate passes, u = (1 - lambda) g + lambda h (Eq. mix-gradient)."""
+take too long in fp64, it restates that pass for sampled output rows of every
+weight gradient (every cotangent is still formed over all rows), and the
+tests also check properties that hold at any size: the vocabulary-column sums
+of u_W vanish (rows of R and qhat sum to zero), and one backward of the mixed
+cotangent equals the mix of the two separate passes, u = (1 - lambda) g +
+lambda h (Eq. mix-gradient)."""
 import numpy as np
 import pytest
 import torch
@@ -53,6 +54,11 @@ def _check_task_space(gout, ref):
     assert abs(gout["s"].sum()) <= 1e-5 * np.abs(gout["s"]).sum() + 1e-7
 
 
+def _outputs(model, wl):
+    qp, sp, lp = model.outputs()
+    return {"qhat": G.host_f32(qp, wl.vocab), "s": G.host_f32(sp, wl.vocab), "lse": G.host_f32(lp, wl.n_rows)}
+
+
 def _sample(n, k, seed, extra=()):
     rng = np.random.default_rng(seed)
     return np.unique(np.concatenate([rng.integers(0, n, k), np.array(extra, dtype=np.int64)]))
@@ -87,39 +93,100 @@ def test_lm_output_block_full_size():
     assert np.abs(u_w.sum(axis=0)).max() <= 2e-2 * np.abs(u_w).sum(axis=0).max()
 
 
+def _dev_rows(t, rows):
+    """float64 host copy of rows `rows` (first index) of a device tensor."""
+    return G.np64(t.index_select(0, torch.from_numpy(np.asarray(rows, dtype=np.int64)).to(t.device)))
+
+
+def _weighted_step_err(th_gpu, th_in, th_ref, v_ref, t, b2):
+    """Relative L2 error of the update step theta - theta_in, each element
+    weighed by its own sqrt(vhat) (the oracle's): in that metric the step is
+    lr u / (1 + eps/sqrt(vhat)) plus the decay, so the measure is of the order
+    of the relative error of u itself, whatever the size of an element's
+    own step."""
+    w = np.sqrt(v_ref / (1.0 - b2 ** t))
+    return G.rel_l2((th_gpu - th_in) * w, (th_ref - th_in) * w)
+
+
 def test_lm_block_with_swiglu_mlps_full_size():
-    """16384 tokens, two SwiGLU MLPs (d 2048, ffn 8192), head 32000 x 2048:
-    s_t, q_t, CE, lse on every row (fp64 forward), u_W of the head on sampled
-    rows, and u = (1-lambda) g + lambda h for every tensor."""
+    """16384 tokens, two SwiGLU MLPs (d 2048, ffn 8192), head 32000 x 2048, in
+    the launch configuration bench.py times: the BOM-AdamW update fused into
+    the step (lr 1e-4, weight decay 0.1 on the matrices), one batch repeated.
+    Two fused steps move the state; at t = 3 the fp64 oracle runs on the inputs
+    that step reads (bf16 parameters, q_2, theta and v) and checks
+      - s_t, q_t, qhat_t, CE and lse on every row, N_t exactly;
+      - u of all seven tensors on sampled rows (a second handle writes u from
+        the same inputs; Eq. mix-gradient through the head and both
+        sublayers);
+      - theta and v of the fused step on the same rows (Section 3.4);
+      - u = (1 - lambda) g + lambda h for every tensor (a G_AND_H handle)."""
     wl = I.LM_MLP_BF16
+    lr, wd_mat, b2, eps, t_chk = 1e-4, 0.1, 0.999, 1e-8, 3
+    F = lambda v: float(np.float32(v))
+    wds = I.weight_decay_mask(wl, wd_mat)
     params = I.init_params(wl, 0)
     x, y = I.make_batch(wl, 0, 1)
-    t, q0 = 2, _q0(wl.vocab)
-    gpu = G.GpuBom(wl, params)
-    gpu.q.copy_(torch.from_numpy(q0))
-    gout = gpu.step(x, y, t)
-    grads_u = [G.np64(g) for g in gout["grads"]]
-    del gout["grads"]
+    fz = G.GpuBom(wl, params)
+    theta = [torch.from_numpy(I.bf16_to_f32(p)).to(G.DEV) for p in params]
+    v = [torch.zeros(p.shape, dtype=torch.float32, device=G.DEV) for p in params]
+    B.bom_set_fused_update(fz.model.h, theta, v, wds, lr, b2, eps)
+    xd = G.to_dev(x)
+    yd = torch.from_numpy(np.ascontiguousarray(y, dtype=np.int32)).to(G.DEV)
+    for t in range(1, t_chk):
+        fz.model.step(xd, yd, wl.n_rows, fz.params, fz.q, t, None, None)
+        assert fz.model.stats()["code"] == B.BOM_OK
 
-    gh = G.GpuBom(wl, params, out_mode=B.BOM_OUT_G_AND_H)
-    gh.q.copy_(torch.from_numpy(q0))
-    o2 = gh.step(x, y, t)
-    for k, u in enumerate(grads_u):
-        mix = (1 - LAM) * G.np64(o2["grads"][k]) + LAM * G.np64(o2["h"][k])
-        assert G.rel_l2(u, mix) < TOL, k
-    del o2, gh
+    # the inputs of step t_chk, as the fused step will read them
+    p_in = [p.clone() for p in fz.params]
+    q_in = G.np64(fz.q)
+    rng = np.random.default_rng(3)
+    rows = [np.unique(np.concatenate([rng.integers(0, p.shape[0], 64), [0, p.shape[0] - 1]])) for p in params]
+    th_in = [_dev_rows(a, r) for a, r in zip(theta, rows)]
+    v_in = [_dev_rows(a, r) for a, r in zip(v, rows)]
 
-    p64 = X.params_f64(wl, params)
-    Z, saved = O.forward(X.oracle_layers(wl), False, p64, I.bf16_to_f64(x))
-    ref = _task_space(Z, y, q0, t)
+    # u from the same inputs on a handle that writes it
+    us = G.GpuBom(wl, p_in)
+    us.q.copy_(fz.q)
+    gout = us.step(x, y, t_chk)
+    u_rows = [_dev_rows(g, r) for g, r in zip(gout["grads"], rows)]
+    # g and h on a third handle: one mixed backward equals the mix of the two
+    gh = G.GpuBom(wl, p_in, out_mode=B.BOM_OUT_G_AND_H)
+    gh.q.copy_(fz.q)
+    o2 = gh.step(x, y, t_chk)
+    for k, u in enumerate(gout["grads"]):
+        mix = (1 - LAM) * o2["grads"][k].double() + LAM * o2["h"][k].double()
+        assert G.rel_l2(G.np64(u), G.np64(mix)) < TOL, k
+    del o2, gh, gout, us
+    torch.cuda.empty_cache()
+
+    # the fused step the bench times
+    fz.model.step(xd, yd, wl.n_rows, fz.params, fz.q, t_chk, None, None)
+    assert fz.model.stats()["code"] == B.BOM_OK
+    th_out = [_dev_rows(a, r) for a, r in zip(theta, rows)]
+    v_out = [_dev_rows(a, r) for a, r in zip(v, rows)]
+
+    # the oracle on the same inputs
+    p64 = [G.np64(p) for p in p_in]
+    del p_in
+    layers = X.oracle_layers(wl)
+    Z, saved = O.forward(layers, False, p64, I.bf16_to_f64(x))
+    ref = _task_space(Z, y, q_in.astype(np.float32), t_chk)
     del Z
-    _check_task_space(gout, ref)
-    h_last = saved[1]
-    rv = _sample(wl.vocab, 64, 3, extra=(0, 1, 2, wl.vocab - 1))
-    gw = O.head_weight_grad_rows(ref["R"], h_last, ref["valid"], ref["qhat"], ref["n_t"], LAM, rv)
-    u_head = grads_u[-1]
-    assert G.rel_l2(u_head[rv], gw) < TOL
-    assert np.abs(u_head.sum(axis=0)).max() <= 2e-2 * np.abs(u_head).sum(axis=0).max()
+    _check_task_space({"stats": fz.model.stats(), "q": G.np64(fz.q), **_outputs(fz.model, wl)}, ref)
+    want = O.mix_grad_rows(layers, False, p64, saved, ref["R"], ref["valid"], ref["qhat"], ref["n_t"], LAM, rows)
+    del saved, ref
+    worst = {}
+    for k in range(len(params)):
+        e_u = G.rel_l2(u_rows[k], want[k])
+        th_ref, v_ref = O.bom_update(th_in[k], want[k], v_in[k], F(lr), F(wds[k]), t_chk, F(b2), F(eps))
+        e_th = G.rel_l2(th_out[k], th_ref)
+        e_v = G.rel_l2(v_out[k], v_ref)
+        e_step = _weighted_step_err(th_out[k], th_in[k], th_ref, v_ref, t_chk, b2)
+        worst[k] = (e_u, e_th, e_v, e_step)
+        assert e_u < TOL, (k, e_u)
+        assert e_th < TOL and e_v < TOL and e_step < TOL, (k, e_th, e_v, e_step)
+    print("LM block full size, rel L2 per tensor (u, theta, v, weighted step):",
+          {k: tuple(f"{e:.2e}" for e in w) for k, w in worst.items()})
 
 
 def test_vision_head_twenty_steps_full_size():
