@@ -75,3 +75,22 @@ class GpuBom:
 def oracle_step(wl, params64, x_np, y_np, q_prev, t, lam=0.5, beta1=0.9):
     return O.bom_step(X.oracle_layers(wl), wl.head_bias, params64, X.x_f64(wl, x_np), y_np, q_prev, t,
                       lam=lam, beta1=beta1)
+
+
+def weighted_step_check(th_gpu, th_in, th_ref, v_ref, t, beta2, tol):
+    """Error and bound of an update step theta - theta_in (Section 3.4), each
+    element weighed by its own sqrt(vhat) of the oracle: in that metric the
+    step is about lr u, so its error is of the order of the error of u
+    whatever the size of the element's own step (an element with tiny u still
+    moves by about lr, and at t = 1 by -lr sign(u)).  The bound is tol times
+    the weighted step, plus half an fp32 ulp of each updated element (the GPU
+    stores theta in fp32: a step of lr = 1e-3 on theta near 1 is resolved to
+    about 6e-5 of itself, whatever the accuracy of u).  Returns (err, bound)."""
+    w = np.sqrt(np.asarray(v_ref, dtype=np.float64) / (1.0 - beta2 ** t))
+    d = (np.asarray(th_gpu) - th_in) * w
+    ref = (np.asarray(th_ref) - th_in) * w
+    half_ulp = 0.5 * np.abs(np.spacing(np.asarray(th_ref, dtype=np.float32))).astype(np.float64)
+    err = float(np.linalg.norm(d - ref))
+    bound = tol * float(np.linalg.norm(ref)) + float(np.linalg.norm(half_ulp * w))
+    return err, bound
+
