@@ -38,12 +38,14 @@ constexpr int BN = 256;
 constexpr int BK = 64;  // one 128-byte swizzle atom of bf16 along K
 constexpr int NUM_THREADS = 320;  // producer warp, UMMA warp, 8 epilogue warps
 constexpr int TMEM_COLS = 512;
+// Tile raster: groups of group_m consecutive m-tiles with m fastest inside a
+// group (group_m = 1: n fastest along whole rows of tiles).  See raster_group.
 constexpr int GROUP_M = 8;
 
 constexpr int kMaxGroup = 8;
 struct Prob {
     CUtensorMap mapA, mapB;
-    int M, N, tiles_m, tiles_n;
+    int M, N, tiles_m, tiles_n, group_m;
     EpiParams epi;
 };
 
@@ -55,6 +57,7 @@ struct Params {
     int kb[2];
     int nseg;
     int tiles_m, tiles_n;
+    int group_m;           // raster group of problem 0 (raster_group)
     int dual_b;
     int bn_out;
     int ksplit;            // K ranges per output tile (1: no split)
@@ -76,7 +79,7 @@ struct ProbView {
     const CUtensorMap* mapA;
     const CUtensorMap* mapB;
     const EpiParams* epi;
-    int M, N, tiles_m, tiles_n, local;
+    int M, N, tiles_m, tiles_n, group_m, local;
 };
 __device__ __forceinline__ ProbView prob_of(const Params& p, int tile) {
     int q = 0;
@@ -90,6 +93,7 @@ __device__ __forceinline__ ProbView prob_of(const Params& p, int tile) {
         v.N = p.N;
         v.tiles_m = p.tiles_m;
         v.tiles_n = p.tiles_n;
+        v.group_m = p.group_m;
     } else {
         const Prob& g = p.grp[q - 1];
         v.mapA = &g.mapA;
@@ -99,16 +103,17 @@ __device__ __forceinline__ ProbView prob_of(const Params& p, int tile) {
         v.N = g.N;
         v.tiles_m = g.tiles_m;
         v.tiles_n = g.tiles_n;
+        v.group_m = g.group_m;
     }
     v.local = tile - p.tile_base[q];
     return v;
 }
 
-__device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int& mt, int& nt) {
-    const int per_group = GROUP_M * tiles_n;
+__device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int group_m, int& mt, int& nt) {
+    const int per_group = group_m * tiles_n;
     const int g = tile / per_group;
-    const int first_m = g * GROUP_M;
-    const int gsz = min(tiles_m - first_m, GROUP_M);
+    const int first_m = g * group_m;
+    const int gsz = min(tiles_m - first_m, group_m);
     const int r = tile - g * per_group;
     mt = first_m + r % gsz;
     nt = r / gsz;
@@ -339,7 +344,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 const int sp = w - tile * p.ksplit;
                 const ProbView pv = prob_of(p, tile);
                 int mt, nt;
-                tile_coords(pv.local, pv.tiles_m, pv.tiles_n, mt, nt);
+                tile_coords(pv.local, pv.tiles_m, pv.tiles_n, pv.group_m, mt, nt);
                 const int m_own = mt * C::TILE_M + static_cast<int>(rank) * BM;
                 const int n0 = nt * p.bn_out;
                 const int n_own = n0 + (CG == 2 && !p.dual_b ? static_cast<int>(rank) * C::B_ROWS : 0);
@@ -488,7 +493,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             // split-K: each K range stores its raw fp32 tile into its own slice
             void* const out_base = static_cast<char*>(e.out) + static_cast<int64_t>(w - tile * p.ksplit) * p.split_bytes;
             int mt, nt;
-            tile_coords(pv.local, pv.tiles_m, pv.tiles_n, mt, nt);
+            tile_coords(pv.local, pv.tiles_m, pv.tiles_n, pv.group_m, mt, nt);
             const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
             const int n0 = nt * p.bn_out;
             const int acc = it & 1;
@@ -915,6 +920,16 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restr
     }
 }
 
+// Raster of a GEMM's tiles.  The persistent walkers take tiles in order, so
+// the tiles in flight at once are a window of consecutive tile indices; the
+// operand panels they read are shared in L2 only while all their readers run
+// together.  A GEMM at most 8 tiles wide (the weight gradients, input
+// cotangents and down projection of the step, all with long K: 8 MB panels
+// and more) walks whole rows of tiles, so every A panel's readers are
+// consecutive and run in the same wave; wider GEMMs keep groups of 8 m-tiles,
+// m fastest, so a window of tiles reads about as many A panels as B panels.
+static int raster_group(int tiles_m, int tiles_n) { return tiles_n <= 8 ? 1 : GROUP_M; }
+
 // Number of K ranges for a GEMM with `tiles` output tiles on `units` resident
 // tile walkers.  GEMMs that keep the GPU at least 75% busy are not split (the
 // fp32 partials cost more than milder quantisation does).  Otherwise the
@@ -1033,6 +1048,7 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     p.bn_out = g.dual_b ? 128 : BN;
     p.tiles_m = static_cast<int>((g.M + BM * cg - 1) / (BM * cg));
     p.tiles_n = static_cast<int>((g.N + p.bn_out - 1) / p.bn_out);
+    p.group_m = raster_group(p.tiles_m, p.tiles_n);
     p.epi = g.epi;
     const int kb_total = p.kb[0] + (p.nseg > 1 ? p.kb[1] : 0);
     const int tiles = p.tiles_m * p.tiles_n;
@@ -1120,6 +1136,7 @@ int launch_gemm_tc_group(const GemmDesc* gs, int n, cudaStream_t stream) {
             p.N = static_cast<int>(g.N);
             p.tiles_m = tm;
             p.tiles_n = tn;
+            p.group_m = raster_group(tm, tn);
             p.epi = g.epi;
         } else {
             Prob& q = p.grp[i - 1];
@@ -1127,6 +1144,7 @@ int launch_gemm_tc_group(const GemmDesc* gs, int n, cudaStream_t stream) {
             q.N = static_cast<int>(g.N);
             q.tiles_m = tm;
             q.tiles_n = tn;
+            q.group_m = raster_group(tm, tn);
             q.epi = g.epi;
         }
         p.tile_base[i] = tiles;
