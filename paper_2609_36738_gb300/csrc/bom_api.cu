@@ -534,10 +534,14 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     st.lr_dev = h->lr_dev;
     st.beta1 = cfg.beta1;
     st.beta2 = fused ? h->upd_beta2 : 0.0f;
+    // A small whole step runs its task-space pass, label scan included, as one
+    // cluster launch after the logits (the forward reads no label).
+    const bool small = part == kStepFull && h->own_out.empty() && task_small_usable(n, V, dm, cf32);
     if (part != kShardEnd) {   // the second half keeps the status word of the first
         if (cudaMemsetAsync(&h->sc->status, 0, sizeof(int32_t), s) != cudaSuccess) return BOM_ECUDA;
-        BOM_TRACED("labels_scan", 0, 4.0 * n,
-                   launch_labels_scan(labels, n, V, cfg.ignore_index, cfg.lambda, st, h->sc, s, shard));
+        if (!small)
+            BOM_TRACED("labels_scan", 0, 4.0 * n,
+                       launch_labels_scan(labels, n, V, cfg.ignore_index, cfg.lambda, st, h->sc, s, shard));
     }
 
     // ---------------------------------------------------------------- forward
@@ -615,12 +619,25 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
         g.epi.ld_stats = h->ntiles;
         BOM_TRY(run_gemm(h, g, s));
     }
-    if (run_fwd && !h->bf16)
+    if (run_fwd && !h->bf16 && !small)
         BOM_TRACED("row_stats_f32", 0, 4.0 * n * V,
                    launch_row_stats_f32(static_cast<const float*>(h->Z), h->ldz, n, V, h->stats, h->sc, s));
 
     // ---------------------------------------------------------------- task space
-    if (run_fwd) {
+    const bool own = !h->own_out.empty();
+    // with one u pass the small task pass also writes the head bias numerator
+    const bool small_bias = small && !gh && head_b >= 0;
+    if (small) {
+        void* hb = small_bias ? (fused ? static_cast<void*>(h->ubuf) : grads[head_b]) : nullptr;
+        BOM_TRY(traced(h, s, "task_small", 2.0 * V * dm,
+                       2.0 * h->esz * n * h->ldz + h->esz * (n + V) * dm + 12.0 * V, [&] {
+                           return launch_task_small(h->Z, cf32, h->ldz, labels, n, V, cfg.ignore_index, cfg.lambda,
+                                                    cfg.beta1, xin, Wh, dm, q, h->s, h->qhat, h->lse, h->cvec,
+                                                    h->wvec, hb, fused ? 1 : cf32, 1.0f - cfg.lambda, cfg.lambda, st,
+                                                    h->sc, s);
+                       }));
+    }
+    if (run_fwd && !small) {
         BOM_TRACED("row_lse", 0, 8.0 * n * h->ntiles + 12.0 * n,
                    launch_row_lse(h->Z, cf32, h->ldz, n, V, h->stats, h->ntiles, labels, cfg.ignore_index, h->lse,
                                   h->ce, h->sc, s));
@@ -639,23 +656,24 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
         BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 8.0 * V + 24.0 * V,
                    launch_shard_finish_sq(xch_in, h->colpart, resid_blocks(n), V, cfg.beta1, q, h->s, h->qhat,
                                           h->sshard, h->sc, s));
-    } else {
+    } else if (!small) {
         BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 20.0 * V,
                    launch_finish_sq(h->colpart, resid_blocks(n), V, cfg.beta1, q, h->s, h->qhat, h->sc, s));
     }
-    const bool own = !h->own_out.empty();
     if (own)   // per-row residual norms for the cancellation ratio
         BOM_TRACED("row_norm", 2.0 * n * V, h->esz * n * h->ldz + 4.0 * n,
                    launch_row_norm(h->Z, cf32, h->ldz, n, V, h->rnorm, h->sc, s));
-    // (a sharded step's loss comes from the shards' summed CE)
-    BOM_TRACED("scalars", 0, 4.0 * (n + V),
-               launch_scalars(shard ? nullptr : h->ce, n, h->s, V, own ? h->rnorm : nullptr, h->sc, s));
-    // c = colsum_{I_t}(H) and w = W^T qhat (the rank-1 / broadcast factors of the reprojection)
-    BOM_TRACED("colsum", 2.0 * n * dm, h->esz * n * dm,
-               launch_colsum(xin, cf32, dm, n, dm, labels, cfg.ignore_index, nullptr, 1.0f, h->part, h->cvec, 1,
-                             h->sc, s));
-    BOM_TRACED("colsum", 2.0 * V * dm, h->esz * V * dm,
-               launch_colsum(Wh, cf32, dm, V, dm, nullptr, 0, h->qhat, 1.0f, h->part, h->wvec, 1, h->sc, s));
+    if (!small) {
+        // (a sharded step's loss comes from the shards' summed CE)
+        BOM_TRACED("scalars", 0, 4.0 * (n + V),
+                   launch_scalars(shard ? nullptr : h->ce, n, h->s, V, own ? h->rnorm : nullptr, h->sc, s));
+        // c = colsum_{I_t}(H) and w = W^T qhat (the rank-1 / broadcast factors of the reprojection)
+        BOM_TRACED("colsum", 2.0 * n * dm, h->esz * n * dm,
+                   launch_colsum(xin, cf32, dm, n, dm, labels, cfg.ignore_index, nullptr, 1.0f, h->part, h->cvec,
+                                 1, h->sc, s));
+        BOM_TRACED("colsum", 2.0 * V * dm, h->esz * V * dm,
+                   launch_colsum(Wh, cf32, dm, V, dm, nullptr, 0, h->qhat, 1.0f, h->part, h->wvec, 1, h->sc, s));
+    }
     if (own)
         BOM_TRACED("colsum", 2.0 * V * dm, h->esz * V * dm,
                    launch_colsum(Wh, cf32, dm, V, dm, nullptr, 0, h->s, 1.0f, h->part, h->wsvec, 1, h->sc, s));
@@ -760,6 +778,8 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
             if (shard)   // this shard's share: a s^shard + b (N_t^shard / N_t) qhat
                 BOM_TRACED("axpby", 3.0 * V, 12.0 * V,
                            launch_shard_bias(h->sshard, h->qhat, a, b, V, outp[head_b], of32, h->sc, s));
+            else if (small_bias)
+                ;   // written by the small task pass
             else
                 BOM_TRACED("axpby", 3.0 * V, 12.0 * V,
                            launch_axpby(h->s, h->qhat, a, b, V, fused ? h->ubuf : outp[head_b], fused ? 1 : of32,

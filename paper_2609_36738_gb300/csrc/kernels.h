@@ -80,6 +80,22 @@ void launch_shard_finish_sq(const double* xch, const float* colpart, int64_t nbl
 void launch_shard_bias(const float* s_shard, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
                        const DevScalars* sc, cudaStream_t s);
 
+// Task-space pass of a small step in one cluster launch (task_small.cu):
+// label check and N_t, row log-sum-exp and CE, R over Z, s_t, q_t, qhat_t,
+// the step scalars, c = colsum_{I_t}(H) (H [n, dm]), w = W^T qhat (W [V, dm])
+// and, when hb_out is given, the head bias numerator hb_a s + hb_b qhat.  Used
+// for n <= 4096 rows, V and dm <= 8192 and n V <= 2^19 when a cluster of 8
+// CTAs fits on the device (task_small_usable).
+constexpr int64_t kTaskSmallMaxRows = 4096;
+constexpr int64_t kTaskSmallMaxV = 8192;
+constexpr int64_t kTaskSmallMaxD = 8192;
+constexpr int64_t kTaskSmallMaxElems = int64_t(1) << 19;
+bool task_small_usable(int64_t n, int64_t V, int64_t dm, int z_f32);
+int launch_task_small(const void* Z, int z_f32, int64_t ldz, const int32_t* labels, int64_t n, int64_t V,
+                      int32_t ignore, float lambda, float beta1, const void* H, const void* W, int64_t dm, float* q,
+                      float* s_out, float* qhat, float* lse, float* cvec, float* wvec, void* hb_out, int hb_f32,
+                      float hb_a, float hb_b, const StepScalarsIn& st, DevScalars* sc, cudaStream_t s);
+
 // loss = N_t^-1 sum_i ce_i (kept as it is when ce is NULL), ||s|| and, when
 // rnorm is given, r_norm_mean = N_t^-1 sum_i rnorm_i.
 void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, const float* rnorm, DevScalars* sc,

@@ -1,0 +1,428 @@
+// Task-space pass of a small step in one cluster launch.
+//
+// For small batches and output spaces (the classification settings: batch 32
+// x 10 classes, batch 256 x 1000 classes) the task-space part of Algorithm 1
+// is a handful of tiny reductions, and as separate kernels each costs its
+// launch and pipeline fill rather than its work.  One cluster of 8 CTAs does
+// all of it, with the cross-CTA sums in distributed shared memory (added in
+// rank order, so the result is deterministic):
+//   phase 1 (rows split over the CTAs): label check and N_t, the row
+//           log-sum-exp and CE from the logits, r_i = softmax(z_i) - onehot(y_i)
+//           written over Z (0 on ignored rows), column sums of R and of
+//           1_{I_t} H over the CTA's rows;
+//   phase 2 (vocabulary columns split): s_t = N_t^-1 sum_i r_i,
+//           q_t = beta1 q_{t-1} + (1-beta1) s_t, qhat_t = q_t / (1-beta1^t)
+//           (Section 3.2), the head bias numerator a s + b qhat, the step
+//           scalars (N_t, cotangent coefficients, loss, lr and both bias
+//           corrections) and c = colsum_{I_t}(H);
+//   phase 3 (the CTA's vocabulary rows of W): partial sums of W^T qhat;
+//   phase 4 (d split): w = W^T qhat, ||s_t||.
+// Error precedence follows the multi-kernel path: a bad label or N_t = 0
+// first, then a device step counter below 1, then non-finite logits; q and
+// every output of phase 2 on are written only when no error is latched.
+#include <cooperative_groups.h>
+
+#include <atomic>
+
+#include "kernels.h"
+
+namespace bom {
+
+namespace {
+
+namespace cg = cooperative_groups;
+
+constexpr int kSmallCluster = 8;
+constexpr int kSmallThreads = 1024;
+
+struct TaskSmallArgs {
+    const void* Z;
+    int64_t ldz;
+    const int32_t* labels;
+    int64_t n, V;
+    int32_t ignore;
+    float lambda, beta1;
+    const void* H;      // head input [n, dm] (row pitch dm)
+    const void* W;      // head weight [V, dm]
+    int64_t dm;
+    float* q;
+    float* s_out;
+    float* qhat;
+    float* lse;
+    float* cvec;
+    float* wvec;
+    void* hb_out;       // head bias numerator hb_a s + hb_b qhat, or NULL
+    int hb_f32;
+    float hb_a, hb_b;
+    StepScalarsIn st;
+    DevScalars* sc;
+};
+
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max_f(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+template <typename T>
+__device__ __forceinline__ float ld_t(const void* p, int64_t i) {
+    if constexpr (sizeof(T) == 4)
+        return static_cast<const float*>(p)[i];
+    else
+        return __bfloat162float(static_cast<const __nv_bfloat16*>(p)[i]);
+}
+template <typename T>
+__device__ __forceinline__ void st_t(void* p, int64_t i, float v) {
+    if constexpr (sizeof(T) == 4)
+        static_cast<float*>(p)[i] = v;
+    else
+        static_cast<__nv_bfloat16*>(p)[i] = __float2bfloat16_rn(v);
+}
+
+// Shared memory of one CTA (floats unless noted), sized by the host:
+//   colp[V]   column sums of R over the CTA's rows
+//   cp[dm]    column sums of 1_{I_t} H over the CTA's rows
+//   wp[dm]    partial W^T qhat over the CTA's vocabulary rows
+//   qh[vs]    qhat of the CTA's vocabulary slice
+//   lse_s[rp], lab_s[rp] (int)   the CTA's rows
+//   red: per-warp CE, N_t, bad-label and non-finite counts [4][32], totals
+template <typename T>
+__global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const TaskSmallArgs a) {
+    pdl_enter();
+    cg::cluster_group cl = cg::this_cluster();
+    const int C = static_cast<int>(cl.num_blocks());
+    const int c = static_cast<int>(cl.block_rank());
+    const int64_t V = a.V, dm = a.dm, n = a.n;
+    const int64_t rp = (n + C - 1) / C;             // rows per CTA
+    const int64_t vs = (V + C - 1) / C;             // vocabulary columns per CTA
+    const int64_t ds = (dm + C - 1) / C;            // d columns per CTA
+    extern __shared__ float sm[];
+    float* colp = sm;
+    float* cp = colp + V;
+    float* wp = cp + dm;
+    float* qh = wp + dm;
+    float* lse_s = qh + vs;
+    int* lab_s = reinterpret_cast<int*>(lse_s + rp);
+    float* wce = reinterpret_cast<float*>(lab_s + rp);
+    int* wnt = reinterpret_cast<int*>(wce + 32);
+    int* wbad = wnt + 32;
+    int* wnf = wbad + 32;
+    float* tot_f = reinterpret_cast<float*>(wnf + 32);   // [0] CE sum, [1] sum s^2 of the slice
+    int* tot_i = reinterpret_cast<int*>(tot_f + 2);      // [0] N_t, [1] bad, [2] non-finite
+
+    const int tid = threadIdx.x, w = tid >> 5, l = tid & 31;
+    const bool live = a.sc->status == 0;
+    const int64_t r0 = c * rp < n ? c * rp : n;
+    const int64_t r1 = r0 + rp < n ? r0 + rp : n;
+
+    // ---- phase 1a: one warp per row
+    float ce_w = 0.0f;
+    int nt_w = 0, bad_w = 0, nf_w = 0;
+    if (live) {
+        for (int64_t r = r0 + w; r < r1; r += kSmallThreads / 32) {
+            const int32_t y = a.labels[r];
+            const bool sup = y != a.ignore;
+            const bool ok_y = sup && y >= 0 && y < V;
+            float m = -INFINITY;
+            for (int64_t j = l; j < V; j += 32) m = fmaxf(m, ld_t<T>(a.Z, r * a.ldz + j));
+            m = warp_max_f(m);
+            float s = 0.0f;
+            for (int64_t j = l; j < V; j += 32) s += expf(ld_t<T>(a.Z, r * a.ldz + j) - m);
+            s = warp_sum_f(s);
+            if (l == 0) {
+                const float L = m + logf(s);
+                lse_s[r - r0] = L;
+                lab_s[r - r0] = ok_y ? y : -1;
+                a.lse[r] = L;
+                const float zy = ok_y ? ld_t<T>(a.Z, r * a.ldz + y) : 0.0f;
+                if (sup && !ok_y) ++bad_w;
+                if (ok_y) {
+                    ++nt_w;
+                    ce_w += L - zy;
+                }
+                if (!isfinite(L) || (ok_y && !isfinite(zy))) ++nf_w;
+            }
+        }
+    }
+    if (l == 0) {
+        wce[w] = ce_w;
+        wnt[w] = nt_w;
+        wbad[w] = bad_w;
+        wnf[w] = nf_w;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        float ce = 0.0f;
+        int nt = 0, bad = 0, nf = 0;
+        for (int k = 0; k < kSmallThreads / 32; ++k) {
+            ce += wce[k];
+            nt += wnt[k];
+            bad += wbad[k];
+            nf += wnf[k];
+        }
+        tot_f[0] = ce;
+        tot_i[0] = nt;
+        tot_i[1] = bad;
+        tot_i[2] = nf;
+    }
+    // ---- phase 1b: one thread per column, the CTA's rows in order
+    if (live) {
+        for (int64_t j = tid; j < V; j += kSmallThreads) {
+            float acc = 0.0f;
+            for (int64_t r = r0; r < r1; ++r) {
+                const int y = lab_s[r - r0];
+                float p = 0.0f;
+                if (y >= 0) {
+                    p = expf(ld_t<T>(a.Z, r * a.ldz + j) - lse_s[r - r0]);
+                    if (j == y) p -= 1.0f;
+                }
+                st_t<T>(const_cast<void*>(a.Z), r * a.ldz + j, p);
+                acc += p;
+            }
+            colp[j] = acc;
+        }
+        for (int64_t k = tid; k < dm; k += kSmallThreads) {
+            float acc = 0.0f;
+            for (int64_t r = r0; r < r1; ++r)
+                if (lab_s[r - r0] >= 0) acc += ld_t<T>(a.H, r * dm + k);
+            cp[k] = acc;
+        }
+    }
+    cl.sync();
+
+    // ---- phase 2: totals, status, s / q / qhat of the CTA's vocabulary slice
+    __shared__ int s_code;
+    __shared__ float s_inv_nt, s_bc1, s_bc2;
+    if (tid == 0) {
+        float ce = 0.0f;
+        int nt = 0, bad = 0, nf = 0;
+        for (int cc = 0; cc < C; ++cc) {
+            const float* tf = cl.map_shared_rank(tot_f, cc);
+            const int* ti = cl.map_shared_rank(tot_i, cc);
+            ce += tf[0];
+            nt += ti[0];
+            bad += ti[1];
+            nf += ti[2];
+        }
+        float bc1 = a.st.inv_bc1, bc2 = a.st.inv_bc2;
+        bool t_bad = false;
+        if (a.st.t_dev != nullptr) {
+            const int64_t t = *a.st.t_dev;
+            if (t < 1) {
+                t_bad = true;
+            } else {
+                bc1 = inv_bias_correction(a.st.beta1, t);
+                bc2 = inv_bias_correction(a.st.beta2, t);
+            }
+        }
+        int code = live ? 0 : -1;
+        if (live) {
+            if (bad > 0)
+                code = BOM_ELABEL;
+            else if (nt == 0)
+                code = BOM_EEMPTY;
+            else if (t_bad)
+                code = BOM_EINVAL;
+            else if (nf > 0)
+                code = BOM_ENONFINITE;
+        }
+        const float inv = nt > 0 ? 1.0f / static_cast<float>(nt) : 0.0f;
+        s_code = code;
+        s_inv_nt = inv;
+        s_bc1 = bc1;
+        s_bc2 = bc2;
+        if (c == 0 && live) {
+            DevScalars* sc = a.sc;
+            if (code > 0) latch_status(sc, code);
+            sc->n_t = nt;
+            sc->inv_nt = inv;
+            sc->coef_r[0] = (1.0f - a.lambda) * inv;
+            sc->coef_q[0] = a.lambda * inv;
+            sc->coef_r[1] = inv;
+            sc->coef_q[1] = 0.0f;
+            sc->coef_r[2] = 0.0f;
+            sc->coef_q[2] = inv;
+            sc->coef_r[3] = 0.0f;
+            sc->coef_q[3] = inv;
+            sc->lr = a.st.lr_dev != nullptr ? *a.st.lr_dev : a.st.lr;
+            sc->inv_bc1 = bc1;
+            sc->inv_bc2 = bc2;
+            sc->loss = ce * inv;
+            sc->s_norm = 0.0f;
+            sc->r_norm_mean = 0.0f;
+        }
+    }
+    __syncthreads();
+    const bool ok = s_code == 0;
+    const int64_t j0 = c * vs < V ? c * vs : V;
+    const int64_t j1 = j0 + vs < V ? j0 + vs : V;
+    float ss = 0.0f;
+    if (ok) {
+        const float inv = s_inv_nt, bc1 = s_bc1;
+        for (int64_t j = j0 + tid; j < j1; j += kSmallThreads) {
+            float acc = 0.0f;
+            for (int cc = 0; cc < C; ++cc) acc += cl.map_shared_rank(colp, cc)[j];
+            const float s = acc * inv;
+            const float qn = a.beta1 * a.q[j] + (1.0f - a.beta1) * s;
+            const float qhat = qn * bc1;
+            a.q[j] = qn;
+            a.s_out[j] = s;
+            a.qhat[j] = qhat;
+            qh[j - j0] = qhat;
+            ss += s * s;
+            if (a.hb_out) st_elem(a.hb_out, j, a.hb_f32, a.hb_a * s + a.hb_b * qhat);
+        }
+        const int64_t k0 = c * ds < dm ? c * ds : dm;
+        const int64_t k1 = k0 + ds < dm ? k0 + ds : dm;
+        for (int64_t k = k0 + tid; k < k1; k += kSmallThreads) {
+            float acc = 0.0f;
+            for (int cc = 0; cc < C; ++cc) acc += cl.map_shared_rank(cp, cc)[k];
+            a.cvec[k] = acc;
+        }
+    }
+    ss = warp_sum_f(ss);
+    if (l == 0) wce[w] = ss;
+    __syncthreads();
+    if (tid == 0) {
+        float t = 0.0f;
+        for (int k = 0; k < kSmallThreads / 32; ++k) t += wce[k];
+        tot_f[1] = t;
+    }
+    // ---- phase 3: partial W^T qhat over the CTA's vocabulary rows
+    if (ok) {
+        for (int64_t k = tid; k < dm; k += kSmallThreads) {
+            float acc = 0.0f;
+            for (int64_t j = j0; j < j1; ++j) acc += qh[j - j0] * ld_t<T>(a.W, j * dm + k);
+            wp[k] = acc;
+        }
+    }
+    cl.sync();
+    // ---- phase 4: w = W^T qhat over the d slice, ||s_t||
+    if (ok) {
+        const int64_t k0 = c * ds < dm ? c * ds : dm;
+        const int64_t k1 = k0 + ds < dm ? k0 + ds : dm;
+        for (int64_t k = k0 + tid; k < k1; k += kSmallThreads) {
+            float acc = 0.0f;
+            for (int cc = 0; cc < C; ++cc) acc += cl.map_shared_rank(wp, cc)[k];
+            a.wvec[k] = acc;
+        }
+        if (c == 0 && tid == 0) {
+            float t = 0.0f;
+            for (int cc = 0; cc < C; ++cc) t += cl.map_shared_rank(tot_f, cc)[1];
+            a.sc->s_norm = sqrtf(t);
+        }
+    }
+    cl.sync();   // no CTA leaves while another still reads its shared memory
+}
+
+size_t task_small_smem(int64_t n, int64_t V, int64_t dm) {
+    const int64_t rp = (n + kSmallCluster - 1) / kSmallCluster;
+    const int64_t vs = (V + kSmallCluster - 1) / kSmallCluster;
+    return static_cast<size_t>(4 * (V + 2 * dm + vs + 2 * rp + 4 * 32 + 2 + 3) + 64);
+}
+
+template <typename T>
+cudaLaunchConfig_t small_cfg(cudaLaunchAttribute (&at)[2], size_t smem, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kSmallCluster);
+    cfg.blockDim = dim3(kSmallThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = kSmallCluster;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    return cfg;
+}
+
+// Per device: the kernel's shared-memory limit is raised once, and the path
+// is used only if a cluster of the largest size fits on the device.
+template <typename T>
+bool small_ready() {
+    constexpr int kMaxDev = 64;
+    static std::atomic<int> state[kMaxDev];   // 0 unknown, 1 usable, 2 not
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) {
+        cudaGetLastError();
+        return false;
+    }
+    int st = state[dev].load(std::memory_order_relaxed);
+    if (st == 0) {
+        const size_t smem = task_small_smem(kTaskSmallMaxRows, kTaskSmallMaxV, kTaskSmallMaxD);
+        bool ok = cudaFuncSetAttribute(task_small_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem)) == cudaSuccess;
+        if (ok) {
+            cudaLaunchAttribute at[2];
+            cudaLaunchConfig_t cfg = small_cfg<T>(at, smem, nullptr);
+            int nc = 0;
+            ok = cudaOccupancyMaxActiveClusters(&nc, task_small_kernel<T>, &cfg) == cudaSuccess && nc >= 1;
+        }
+        cudaGetLastError();
+        st = ok ? 1 : 2;
+        state[dev].store(st, std::memory_order_relaxed);
+    }
+    return st == 1;
+}
+
+}  // namespace
+
+bool task_small_usable(int64_t n, int64_t V, int64_t dm, int z_f32) {
+    if (n < 1 || n > kTaskSmallMaxRows || V > kTaskSmallMaxV || dm > kTaskSmallMaxD || n * V > kTaskSmallMaxElems)
+        return false;
+    return z_f32 ? small_ready<float>() : small_ready<__nv_bfloat16>();
+}
+
+int launch_task_small(const void* Z, int z_f32, int64_t ldz, const int32_t* labels, int64_t n, int64_t V,
+                      int32_t ignore, float lambda, float beta1, const void* H, const void* W, int64_t dm, float* q,
+                      float* s_out, float* qhat, float* lse, float* cvec, float* wvec, void* hb_out, int hb_f32,
+                      float hb_a, float hb_b, const StepScalarsIn& st, DevScalars* sc, cudaStream_t s) {
+    if (!task_small_usable(n, V, dm, z_f32)) return BOM_ENOTSUP;
+    TaskSmallArgs a;
+    a.Z = Z;
+    a.ldz = ldz;
+    a.labels = labels;
+    a.n = n;
+    a.V = V;
+    a.ignore = ignore;
+    a.lambda = lambda;
+    a.beta1 = beta1;
+    a.H = H;
+    a.W = W;
+    a.dm = dm;
+    a.q = q;
+    a.s_out = s_out;
+    a.qhat = qhat;
+    a.lse = lse;
+    a.cvec = cvec;
+    a.wvec = wvec;
+    a.hb_out = hb_out;
+    a.hb_f32 = hb_f32;
+    a.hb_a = hb_a;
+    a.hb_b = hb_b;
+    a.st = st;
+    a.sc = sc;
+    const size_t smem = task_small_smem(n, V, dm);
+    cudaLaunchAttribute at[2];
+    cudaError_t e;
+    if (z_f32) {
+        cudaLaunchConfig_t cfg = small_cfg<float>(at, smem, s);
+        e = cudaLaunchKernelEx(&cfg, task_small_kernel<float>, a);
+    } else {
+        cudaLaunchConfig_t cfg = small_cfg<__nv_bfloat16>(at, smem, s);
+        e = cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16>, a);
+    }
+    if (e != cudaSuccess) return BOM_ECUDA;
+    count_launch();
+    return BOM_OK;
+}
+
+}  // namespace bom
