@@ -1,13 +1,15 @@
 // SIMT fp32 GEMM (no TF32) for the fp32 configuration, where the parity bar is
 // a relative L2 error of 1e-5 that TF32 tensor cores cannot meet.  64 x 64
-// output tile per 256-thread block, 4 x 4 outputs per thread, K in steps of 16
-// through shared memory; operands in either K-major or MN-major layout.
+// output tile per 256-thread block, 4 x 4 outputs per thread, K in steps of 64
+// through shared memory (the fp32 shapes are small: their K of 10 to a few
+// hundred takes one to a few steps, each thread's 32 loads of a step in
+// flight at once); operands in either K-major or MN-major layout.
 #include "gemm.h"
 
 namespace bom {
 namespace simt {
 
-constexpr int TM = 64, TN = 64, TK = 16;
+constexpr int TM = 64, TN = 64, TK = 64;
 
 struct Params {
     const float* A[2];
@@ -33,17 +35,29 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const Params p) {
         const float* A = p.A[s];
         const float* B = p.B[s];
         for (int64_t k0 = 0; k0 < p.K[s]; k0 += TK) {
-            for (int i = threadIdx.x; i < TK * TM; i += 256) {
+            // every load of the step issued before any is stored
+            constexpr int PER = TK * TM / 256;
+            float av[PER], bv[PER];
+#pragma unroll
+            for (int u = 0; u < PER; ++u) {
+                const int i = threadIdx.x + 256 * u;
                 const int kk = i / TM, mm = i % TM;
                 const int m = m0 + mm;
                 const int64_t k = k0 + kk;
-                As[kk][mm] = (m < p.M && k < p.K[s]) ? A[m * p.a_sm[s] + k * p.a_sk[s]] : 0.0f;
+                av[u] = (m < p.M && k < p.K[s]) ? A[m * p.a_sm[s] + k * p.a_sk[s]] : 0.0f;
                 const int n = n0 + mm;
-                Bs[kk][mm] = (n < p.N && k < p.K[s]) ? B[n * p.b_sn[s] + k * p.b_sk[s]] : 0.0f;
+                bv[u] = (n < p.N && k < p.K[s]) ? B[n * p.b_sn[s] + k * p.b_sk[s]] : 0.0f;
+            }
+#pragma unroll
+            for (int u = 0; u < PER; ++u) {
+                const int i = threadIdx.x + 256 * u;
+                As[i / TM][i % TM] = av[u];
+                Bs[i / TM][i % TM] = bv[u];
             }
             __syncthreads();
-#pragma unroll
-            for (int kk = 0; kk < TK; ++kk) {
+            const int kn = static_cast<int>(p.K[s] - k0 < TK ? p.K[s] - k0 : TK);
+#pragma unroll 16
+            for (int kk = 0; kk < kn; ++kk) {
                 float a[4], b[4];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) a[i] = As[kk][ty + 16 * i];

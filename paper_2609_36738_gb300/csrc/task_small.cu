@@ -34,6 +34,9 @@ namespace cg = cooperative_groups;
 
 constexpr int kSmallCluster = 8;
 constexpr int kSmallThreads = 1024;
+// Row-group partials of the chunked column sums: RG * dm <= 1024 * 8 floats
+// (RG = 1024 / (dm / elements per 16-byte word), or 1).
+constexpr int kSmallPart = 8192;
 
 struct TaskSmallArgs {
     const void* Z;
@@ -83,19 +86,81 @@ __device__ __forceinline__ void st_t(void* p, int64_t i, float v) {
     else
         static_cast<__nv_bfloat16*>(p)[i] = __float2bfloat16_rn(v);
 }
+// Element e of a 16-byte word holding 16 / sizeof(T) values.
+template <typename T>
+__device__ __forceinline__ float word_at(const uint4& w, int e) {
+    const uint32_t x = (e * static_cast<int>(sizeof(T)) / 4) == 0   ? w.x
+                       : (e * static_cast<int>(sizeof(T)) / 4) == 1 ? w.y
+                       : (e * static_cast<int>(sizeof(T)) / 4) == 2 ? w.z
+                                                                     : w.w;
+    if constexpr (sizeof(T) == 4)
+        return __uint_as_float(x);
+    else
+        return __uint_as_float((e & 1) ? (x & 0xFFFF0000u) : (x << 16));
+}
+
+// part[g * dm + k] = sum over rows j = j0 + g, j0 + g + RG, ... < j1 of
+// wt(j) * X[j, k], for g < RG row groups: thread (kc, g) reads its rows' word
+// kc of 16 bytes, four rows in flight.  RG * KC <= 1024 (RG = 1024 / KC).
+// `vec` selects 16-byte words (rows 16-byte aligned, dm a multiple of the
+// word) or single elements.
+template <typename T, class Wt>
+__device__ __forceinline__ void colsum_tile(const void* X, int64_t dm, int64_t j0, int64_t j1, bool vec, Wt wt,
+                                            float* part, int RG) {
+    const int EPC = vec ? 16 / static_cast<int>(sizeof(T)) : 1;
+    const int64_t KC = (dm + EPC - 1) / EPC;
+    for (int64_t idx = threadIdx.x; idx < KC * RG; idx += kSmallThreads) {
+        const int64_t kc = idx % KC;
+        const int g = static_cast<int>(idx / KC);
+        float acc[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
+        int64_t j = j0 + g;
+        if (vec) {
+            const T* base = static_cast<const T*>(X) + kc * EPC;
+            for (; j + 3 * RG < j1; j += 4 * RG) {
+                uint4 w[4];
+                float f[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    w[u] = __ldg(reinterpret_cast<const uint4*>(base + (j + u * RG) * dm));
+                    f[u] = wt(j + u * RG);
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        if (e < EPC) acc[e] = fmaf(f[u], word_at<T>(w[u], e), acc[e]);
+            }
+            for (; j < j1; j += RG) {
+                const uint4 w = __ldg(reinterpret_cast<const uint4*>(base + j * dm));
+                const float f = wt(j);
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    if (e < EPC) acc[e] = fmaf(f, word_at<T>(w, e), acc[e]);
+            }
+        } else {
+            for (; j < j1; j += RG) acc[0] = fmaf(wt(j), ld_t<T>(X, j * dm + kc), acc[0]);
+        }
+        for (int e = 0; e < EPC; ++e)
+            if (kc * EPC + e < dm) part[g * dm + kc * EPC + e] = acc[e];
+    }
+}
 
 // Shared memory of one CTA (floats unless noted), sized by the host:
-//   colp[V]   column sums of R over the CTA's rows
-//   cp[dm]    column sums of 1_{I_t} H over the CTA's rows
-//   wp[dm]    partial W^T qhat over the CTA's vocabulary rows
-//   qh[vs]    qhat of the CTA's vocabulary slice
+//   colp[V]     column sums of R over the CTA's rows
+//   cp[dm]      column sums of 1_{I_t} H over the CTA's rows
+//   wp[dm]      partial W^T qhat over the CTA's vocabulary rows
+//   part[8192]  row-group partials of the two chunked column sums
+//   qh[vs]      qhat of the CTA's vocabulary slice
 //   lse_s[rp], lab_s[rp] (int)   the CTA's rows
-//   red: per-warp CE, N_t, bad-label and non-finite counts [4][32], totals
+//   per-warp CE, N_t, bad-label and non-finite counts [4][32], totals
 template <typename T>
 __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const TaskSmallArgs a) {
     pdl_enter();
     cg::cluster_group cl = cg::this_cluster();
-    const int C = static_cast<int>(cl.num_blocks());
+    constexpr int C = kSmallCluster;
+    constexpr int EPC = 16 / static_cast<int>(sizeof(T));
     const int c = static_cast<int>(cl.block_rank());
     const int64_t V = a.V, dm = a.dm, n = a.n;
     const int64_t rp = (n + C - 1) / C;             // rows per CTA
@@ -105,7 +170,8 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
     float* colp = sm;
     float* cp = colp + V;
     float* wp = cp + dm;
-    float* qh = wp + dm;
+    float* part = wp + dm;
+    float* qh = part + kSmallPart;
     float* lse_s = qh + vs;
     int* lab_s = reinterpret_cast<int*>(lse_s + rp);
     float* wce = reinterpret_cast<float*>(lab_s + rp);
@@ -119,20 +185,49 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
     const bool live = a.sc->status == 0;
     const int64_t r0 = c * rp < n ? c * rp : n;
     const int64_t r1 = r0 + rp < n ? r0 + rp : n;
+    // rows of H and W start on 16 bytes when dm fills whole words
+    const bool hw_vec = (dm % EPC) == 0;
+    const int64_t KC = hw_vec ? dm / EPC : dm;
+    const int RG = static_cast<int>(kSmallThreads / KC > 0 ? kSmallThreads / KC : 1);
 
-    // ---- phase 1a: one warp per row
+    // ---- phase 1a: one warp per row, the row read as 16-byte words (Z rows
+    // are padded to whole 128-byte lines), four words in flight per lane
     float ce_w = 0.0f;
     int nt_w = 0, bad_w = 0, nf_w = 0;
     if (live) {
+        const int64_t nw = (V + EPC - 1) / EPC;
         for (int64_t r = r0 + w; r < r1; r += kSmallThreads / 32) {
             const int32_t y = a.labels[r];
             const bool sup = y != a.ignore;
             const bool ok_y = sup && y >= 0 && y < V;
+            const T* zr = static_cast<const T*>(a.Z) + r * a.ldz;
             float m = -INFINITY;
-            for (int64_t j = l; j < V; j += 32) m = fmaxf(m, ld_t<T>(a.Z, r * a.ldz + j));
+            for (int64_t b = l; b < nw; b += 128) {
+                uint4 wd[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (b + 32 * u < nw) wd[u] = *reinterpret_cast<const uint4*>(zr + (b + 32 * u) * EPC);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (b + 32 * u < nw)
+#pragma unroll
+                        for (int e = 0; e < EPC; ++e)
+                            if ((b + 32 * u) * EPC + e < V) m = fmaxf(m, word_at<T>(wd[u], e));
+            }
             m = warp_max_f(m);
             float s = 0.0f;
-            for (int64_t j = l; j < V; j += 32) s += expf(ld_t<T>(a.Z, r * a.ldz + j) - m);
+            for (int64_t b = l; b < nw; b += 128) {
+                uint4 wd[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (b + 32 * u < nw) wd[u] = *reinterpret_cast<const uint4*>(zr + (b + 32 * u) * EPC);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (b + 32 * u < nw)
+#pragma unroll
+                        for (int e = 0; e < EPC; ++e)
+                            if ((b + 32 * u) * EPC + e < V) s += expf(word_at<T>(wd[u], e) - m);
+            }
             s = warp_sum_f(s);
             if (l == 0) {
                 const float L = m + logf(s);
@@ -170,26 +265,37 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
         tot_i[1] = bad;
         tot_i[2] = nf;
     }
-    // ---- phase 1b: one thread per column, the CTA's rows in order
+    // ---- phase 1b: one thread per column, the CTA's rows in order, eight in flight
     if (live) {
         for (int64_t j = tid; j < V; j += kSmallThreads) {
             float acc = 0.0f;
-            for (int64_t r = r0; r < r1; ++r) {
-                const int y = lab_s[r - r0];
-                float p = 0.0f;
-                if (y >= 0) {
-                    p = expf(ld_t<T>(a.Z, r * a.ldz + j) - lse_s[r - r0]);
-                    if (j == y) p -= 1.0f;
+            for (int64_t rb = r0; rb < r1; rb += 8) {
+                float z[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) z[u] = rb + u < r1 ? ld_t<T>(a.Z, (rb + u) * a.ldz + j) : 0.0f;
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int64_t r = rb + u;
+                    if (r >= r1) break;
+                    const int y = lab_s[r - r0];
+                    float p = 0.0f;
+                    if (y >= 0) {
+                        p = expf(z[u] - lse_s[r - r0]);
+                        if (j == y) p -= 1.0f;
+                    }
+                    st_t<T>(const_cast<void*>(a.Z), r * a.ldz + j, p);
+                    acc += p;
                 }
-                st_t<T>(const_cast<void*>(a.Z), r * a.ldz + j, p);
-                acc += p;
             }
             colp[j] = acc;
         }
+        // c over the CTA's rows: 1_{I_t} H, in row groups, then the groups in order
+        colsum_tile<T>(a.H, dm, r0, r1, hw_vec, [&](int64_t r) { return lab_s[r - r0] >= 0 ? 1.0f : 0.0f; },
+                       part, RG);
+        __syncthreads();
         for (int64_t k = tid; k < dm; k += kSmallThreads) {
             float acc = 0.0f;
-            for (int64_t r = r0; r < r1; ++r)
-                if (lab_s[r - r0] >= 0) acc += ld_t<T>(a.H, r * dm + k);
+            for (int g = 0; g < RG; ++g) acc += part[g * dm + k];
             cp[k] = acc;
         }
     }
@@ -201,6 +307,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
     if (tid == 0) {
         float ce = 0.0f;
         int nt = 0, bad = 0, nf = 0;
+#pragma unroll
         for (int cc = 0; cc < C; ++cc) {
             const float* tf = cl.map_shared_rank(tot_f, cc);
             const int* ti = cl.map_shared_rank(tot_i, cc);
@@ -261,12 +368,18 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
     const bool ok = s_code == 0;
     const int64_t j0 = c * vs < V ? c * vs : V;
     const int64_t j1 = j0 + vs < V ? j0 + vs : V;
+    const int64_t k0 = c * ds < dm ? c * ds : dm;
+    const int64_t k1 = k0 + ds < dm ? k0 + ds : dm;
     float ss = 0.0f;
     if (ok) {
         const float inv = s_inv_nt, bc1 = s_bc1;
         for (int64_t j = j0 + tid; j < j1; j += kSmallThreads) {
+            float pv[C];
+#pragma unroll
+            for (int cc = 0; cc < C; ++cc) pv[cc] = cl.map_shared_rank(colp, cc)[j];
             float acc = 0.0f;
-            for (int cc = 0; cc < C; ++cc) acc += cl.map_shared_rank(colp, cc)[j];
+#pragma unroll
+            for (int cc = 0; cc < C; ++cc) acc += pv[cc];
             const float s = acc * inv;
             const float qn = a.beta1 * a.q[j] + (1.0f - a.beta1) * s;
             const float qhat = qn * bc1;
@@ -277,11 +390,13 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
             ss += s * s;
             if (a.hb_out) st_elem(a.hb_out, j, a.hb_f32, a.hb_a * s + a.hb_b * qhat);
         }
-        const int64_t k0 = c * ds < dm ? c * ds : dm;
-        const int64_t k1 = k0 + ds < dm ? k0 + ds : dm;
         for (int64_t k = k0 + tid; k < k1; k += kSmallThreads) {
+            float pv[C];
+#pragma unroll
+            for (int cc = 0; cc < C; ++cc) pv[cc] = cl.map_shared_rank(cp, cc)[k];
             float acc = 0.0f;
-            for (int cc = 0; cc < C; ++cc) acc += cl.map_shared_rank(cp, cc)[k];
+#pragma unroll
+            for (int cc = 0; cc < C; ++cc) acc += pv[cc];
             a.cvec[k] = acc;
         }
     }
@@ -293,26 +408,32 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
         for (int k = 0; k < kSmallThreads / 32; ++k) t += wce[k];
         tot_f[1] = t;
     }
-    // ---- phase 3: partial W^T qhat over the CTA's vocabulary rows
+    // ---- phase 3: partial W^T qhat over the CTA's vocabulary rows (row
+    // groups of 16-byte words, then the groups in order)
     if (ok) {
+        colsum_tile<T>(a.W, dm, j0, j1, hw_vec, [&](int64_t j) { return qh[j - j0]; }, part, RG);
+        __syncthreads();
         for (int64_t k = tid; k < dm; k += kSmallThreads) {
             float acc = 0.0f;
-            for (int64_t j = j0; j < j1; ++j) acc += qh[j - j0] * ld_t<T>(a.W, j * dm + k);
+            for (int g = 0; g < RG; ++g) acc += part[g * dm + k];
             wp[k] = acc;
         }
     }
     cl.sync();
     // ---- phase 4: w = W^T qhat over the d slice, ||s_t||
     if (ok) {
-        const int64_t k0 = c * ds < dm ? c * ds : dm;
-        const int64_t k1 = k0 + ds < dm ? k0 + ds : dm;
         for (int64_t k = k0 + tid; k < k1; k += kSmallThreads) {
+            float pv[C];
+#pragma unroll
+            for (int cc = 0; cc < C; ++cc) pv[cc] = cl.map_shared_rank(wp, cc)[k];
             float acc = 0.0f;
-            for (int cc = 0; cc < C; ++cc) acc += cl.map_shared_rank(wp, cc)[k];
+#pragma unroll
+            for (int cc = 0; cc < C; ++cc) acc += pv[cc];
             a.wvec[k] = acc;
         }
         if (c == 0 && tid == 0) {
             float t = 0.0f;
+#pragma unroll
             for (int cc = 0; cc < C; ++cc) t += cl.map_shared_rank(tot_f, cc)[1];
             a.sc->s_norm = sqrtf(t);
         }
@@ -323,7 +444,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
 size_t task_small_smem(int64_t n, int64_t V, int64_t dm) {
     const int64_t rp = (n + kSmallCluster - 1) / kSmallCluster;
     const int64_t vs = (V + kSmallCluster - 1) / kSmallCluster;
-    return static_cast<size_t>(4 * (V + 2 * dm + vs + 2 * rp + 4 * 32 + 2 + 3) + 64);
+    return static_cast<size_t>(4 * (V + 2 * dm + kSmallPart + vs + 2 * rp + 4 * 32 + 2 + 3) + 64);
 }
 
 template <typename T>
