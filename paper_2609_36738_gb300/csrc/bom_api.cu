@@ -44,8 +44,9 @@ struct LayerWs {
     int64_t width_out = 0;   // width of the layer output
     void* pre = nullptr;     // LINEAR_GELU pre-activation [n, d_out]
     void* out = nullptr;     // layer output [n, width_out]
-    void* G = nullptr;       // SWIGLU gate pre-activation [n, ffn]
-    void* U = nullptr;       // SWIGLU up projection [n, ffn]
+    void* G = nullptr;       // SWIGLU gate and up pre-activations, interleaved per 32
+                             // columns: [G 32 | U 32] blocks, row pitch gu_ld
+    int64_t gu_ld = 0;       // 2 * ffn rounded up to 64
     void* A = nullptr;       // SWIGLU SiLU(G) * U [n, ffn]
     float* rstd = nullptr;   // RMSNORM 1 / sqrt(mean x^2 + eps) per row [n]
 };
@@ -200,8 +201,10 @@ size_t carve(bom_handle* h, char* base) {
     h->sc = static_cast<DevScalars*>(c.take(sizeof(DevScalars)));
     for (auto& L : h->lw) {
         if (L.kind == BOM_LAYER_SWIGLU) {
-            L.G = c.take(n * L.d_out * e);
-            L.U = c.take(n * L.d_out * e);
+            // G and U of each 32 columns share one 128-byte line of a row: the
+            // forward writes whole lines, the backward epilogue reads one box
+            L.gu_ld = 2 * round_up(L.d_out, 32);
+            L.G = c.take(n * L.gu_ld * e);
             L.A = c.take(n * L.d_out * e);
         } else if (L.kind == BOM_LAYER_LINEAR_GELU) {
             L.pre = c.take(n * L.d_out * e);
@@ -572,9 +575,7 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
             g.epi.out = L.A;
             g.epi.ld_out = f;
             g.epi.out2 = L.G;
-            g.epi.ld_out2 = f;
-            g.epi.out3 = L.U;
-            g.epi.ld_out3 = f;
+            g.epi.ld_out2 = L.gu_ld;
             BOM_TRY(run_gemm(h, g, s));
             GemmDesc g2 = gemm1(n, d, f, kmaj(L.A, f), kmaj(Wd, f));
             g2.epi.resid = xin;
@@ -809,9 +810,7 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                     GemmDesc g = gemm1(n, f, d, kmaj(dcur, d), mnmaj(Wd, f));
                     g.epi_kind = EPI_SWIGLU_BWD;
                     g.epi.aux = L.G;
-                    g.epi.ld_aux = f;
-                    g.epi.aux2 = L.U;
-                    g.epi.ld_aux2 = f;
+                    g.epi.ld_aux = L.gu_ld;
                     g.epi.out = dGl;
                     g.epi.ld_out = f;
                     g.epi.out2 = dUl;

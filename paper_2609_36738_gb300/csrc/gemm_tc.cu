@@ -52,7 +52,7 @@ struct Prob {
 struct Params {
     CUtensorMap mapA[2];
     CUtensorMap mapB[2];
-    CUtensorMap mapE[2];   // SwiGLU backward: saved G and U, 32 x 32 boxes, 64-byte swizzle
+    CUtensorMap mapE[2];   // SwiGLU backward: saved G|U blocks, 32 rows x 64 columns, 128-byte swizzle
     int M, N;
     int kb[2];
     int nseg;
@@ -480,9 +480,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         uint32_t eph = 0, epend = 0;   // phase bit and in-flight flag per slot
         auto eissue = [&](int slot, int col, int rowg) {   // lane 0 only
             fence_proxy_async_shared();   // this warp's reads of the slot precede the refill
+            // the 32-column block of G and U is one 128-byte line per row
             mbar_arrive_expect_tx(&ebw[slot], 2 * kEpiLdBlock);
-            tma_load_2d(eslot + slot * 2 * kEpiLdBlock, &p.mapE[0], &ebw[slot], col, rowg);
-            tma_load_2d(eslot + slot * 2 * kEpiLdBlock + kEpiLdBlock, &p.mapE[1], &ebw[slot], col, rowg);
+            tma_load_2d(eslot + slot * 2 * kEpiLdBlock, &p.mapE[0], &ebw[slot], 2 * col, rowg);
             epend |= 1u << slot;
         };
         for (int w = unit; w < num_work; w += nunits, ++it) {
@@ -695,8 +695,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     // 256-bit stores, no staging (the freed shared memory is a
                     // sixth pipeline stage)
                     if (valid) {
-                        store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, PN, 0, v);
-                        store_row32(e.out3, static_cast<int64_t>(m) * e.ld_out3, n, PN, 0, u);
+                        // G and U of the 32 columns side by side in one 128-byte
+                        // line of the interleaved buffer (row pitch ld_out2)
+                        const int64_t ro = static_cast<int64_t>(m) * e.ld_out2 + 2 * n;
+                        const int cnt = PN - n < 32 ? PN - n : 32;
+                        store_row32(e.out2, ro, 0, cnt, 0, v);
+                        store_row32(e.out2, ro + 32, 0, cnt, 0, u);
                     }
 #pragma unroll
                     for (int i = 0; i < 32; i += 2) {   // SiLU(g) * u on the bf16-rounded G and U
@@ -723,13 +727,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     }
                     eph ^= 1u << slot;
                     epend &= ~(1u << slot);
-                    {   // row `lane` of the G and U blocks (64-byte swizzle)
-                        const uint8_t* bg = eslot + slot * 2 * kEpiLdBlock + lane * 64;
-                        const int sw = (lane >> 1) & 3;
+                    {   // row `lane` of the G|U block (128-byte swizzle: logical
+                        // 16-byte chunk k at chunk k ^ (lane & 7); G in 0-3, U in 4-7)
+                        const uint8_t* bg = eslot + slot * 2 * kEpiLdBlock + lane * 128;
+                        const int sw = lane & 7;
 #pragma unroll
                         for (int k = 0; k < 4; ++k) {
                             const uint4 wg = *reinterpret_cast<const uint4*>(bg + 16 * (k ^ sw));
-                            const uint4 wu = *reinterpret_cast<const uint4*>(bg + kEpiLdBlock + 16 * (k ^ sw));
+                            const uint4 wu = *reinterpret_cast<const uint4*>(bg + 16 * ((k + 4) ^ sw));
                             const uint32_t a4[4] = {wg.x, wg.y, wg.z, wg.w};
                             const uint32_t b4[4] = {wu.x, wu.y, wu.z, wu.w};
 #pragma unroll
@@ -1038,8 +1043,7 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
         }
     }
     if (g.epi_kind == EPI_SWIGLU_BWD &&
-        (!make_map(&p.mapE[0], g.epi.aux, g.N, g.M, g.epi.ld_aux, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B) ||
-         !make_map(&p.mapE[1], g.epi.aux2, g.N, g.M, g.epi.ld_aux2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)))
+        !make_map(&p.mapE[0], g.epi.aux, g.epi.ld_aux, g.M, g.epi.ld_aux, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
         return BOM_ENOTSUP;
     p.M = static_cast<int>(g.M);
     p.N = static_cast<int>(g.N);
