@@ -53,6 +53,11 @@ struct LayerWs {
 
 int64_t round_up(int64_t a, int64_t b) { return (a + b - 1) / b * b; }
 
+// Rows up to which a step with the update registered writes u and updates
+// every tensor in one streaming launch instead of in the weight-gradient
+// GEMMs' epilogues (see bom_handle::uscr).
+constexpr int64_t kUpdSepRows = 1024;
+
 }  // namespace
 
 struct bom_handle {
@@ -91,6 +96,12 @@ struct bom_handle {
     int64_t* t_dev = nullptr;
     const float* lr_dev = nullptr;
     float* ubuf = nullptr;   // fp32 u of a vector tensor (bias, norm weight) before its update
+    // Small batches (max_rows <= kUpdSepRows): fp32 u of every tensor, so
+    // that a step with the update registered writes u from the weight-gradient
+    // GEMMs and updates all tensors in one streaming launch (with a K of a few
+    // hundred rows the update epilogue of those GEMMs is latency-bound).
+    float* uscr = nullptr;
+    std::vector<int64_t> uoff, unum;   // per tensor: offset in uscr (16-byte aligned), elements
     float* part = nullptr;
     void* dx[2] = {nullptr, nullptr};
     void* dG = nullptr;
@@ -232,6 +243,21 @@ size_t carve(bom_handle* h, char* base) {
     h->rnorm = static_cast<float*>(c.take(n * 4));
     h->tel_part = static_cast<double*>(c.take(4 * kOwnStepMaxBlocks * sizeof(double)));
     h->ubuf = static_cast<float*>(c.take((V > h->max_width ? V : h->max_width) * 4));
+    if (n <= kUpdSepRows) {
+        const int np = bom_param_count(&h->cfg);
+        h->uoff.assign(np, 0);
+        h->unum.assign(np, 0);
+        int64_t tot = 0;
+        for (int k = 0; k < np; ++k) {
+            int64_t r = 0, cc = 0;
+            bom_param_shape(&h->cfg, k, &r, &cc);
+            h->unum[k] = r * (cc > 0 ? cc : 1);
+            h->uoff[k] = tot;
+            tot += round_up(h->unum[k], 4);
+        }
+        h->uscr = np <= kMultiUpdMax ? static_cast<float*>(c.take(tot * 4)) : nullptr;
+        if (np > kMultiUpdMax) h->uoff.clear();
+    }
     const int64_t rb = row_blocks(n) > row_blocks(V) ? row_blocks(n) : row_blocks(V);
     h->part = static_cast<float*>(c.take(rb * h->max_width * 4));
     h->dx[0] = c.take(n * h->max_width * e);
@@ -511,6 +537,18 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     const bool fused = h->fused_upd;
     const bool gh = h->cfg.out_mode == BOM_OUT_G_AND_H;
     const bool shard = part != kStepFull;
+    // a small batch with the update registered: u of every tensor to the
+    // scratch, then one update launch for all of them at the end of the step
+    const bool upd_sep = fused && h->uscr != nullptr && n <= kUpdSepRows;
+    // where the fp32 u of vector tensor k goes when the update is registered
+    auto uvec = [&](int k) -> float* { return upd_sep ? h->uscr + h->uoff[k] : h->ubuf; };
+    // With at most two backbone layers their output cotangents stay in the two
+    // ping-pong buffers until the step ends, so for a batch of at most 128 rows
+    // a Linear layer's bias gradient (their column sum) is formed by the final
+    // update itself, in the order of the column reduction over one range.
+    const bool fold_bias = upd_sep && h->lw.size() <= 2 && n <= kRowBlock;
+    std::vector<const void*> usrc;
+    if (fold_bias) usrc.assign(bom_param_count(&h->cfg), nullptr);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const bom_config& cfg = h->cfg;
     const int64_t V = cfg.d_out, dm = h->d_model;
@@ -629,7 +667,7 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     // with one u pass the small task pass also writes the head bias numerator
     const bool small_bias = small && !gh && head_b >= 0;
     if (small) {
-        void* hb = small_bias ? (fused ? static_cast<void*>(h->ubuf) : grads[head_b]) : nullptr;
+        void* hb = small_bias ? (fused ? static_cast<void*>(uvec(head_b)) : grads[head_b]) : nullptr;
         BOM_TRY(traced(h, s, "task_small", 2.0 * V * dm,
                        2.0 * h->esz * n * h->ldz + h->esz * (n + V) * dm + 12.0 * V, [&] {
                            return launch_task_small(h->Z, cf32, h->ldz, labels, n, V, cfg.ignore_index, cfg.lambda,
@@ -691,6 +729,11 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     // the fused update takes lr and 1/(1 - beta2^t) from the step scalars
     // the GEMM producing u of tensor k updates it in its epilogue
     auto fuse = [&](GemmDesc& g, int k) {
+        if (upd_sep) {   // u to the scratch; the update runs after the pass
+            g.epi.out = h->uscr + h->uoff[k];
+            g.epi.out_f32 = 1;
+            return;
+        }
         g.epi.upd_theta = h->upd_theta[k];
         g.epi.upd_v = h->upd_v[k];
         g.epi.upd_wd = h->upd_wd[k];
@@ -783,9 +826,9 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                 ;   // written by the small task pass
             else
                 BOM_TRACED("axpby", 3.0 * V, 12.0 * V,
-                           launch_axpby(h->s, h->qhat, a, b, V, fused ? h->ubuf : outp[head_b], fused ? 1 : of32,
+                           launch_axpby(h->s, h->qhat, a, b, V, fused ? uvec(head_b) : outp[head_b], fused ? 1 : of32,
                                         h->sc, s));
-            if (fused) BOM_TRY(update_small(head_b, V));
+            if (fused && !upd_sep) BOM_TRY(update_small(head_b, V));
         }
         for (int l = static_cast<int>(h->lw.size()) - 1; l >= 0; --l) {
             const LayerWs& L = h->lw[l];
@@ -864,13 +907,13 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                 // dgamma_j = sum_i rstd_i dy_ij x_ij
                 BOM_TRACED("colsum", 3.0 * n * d, 2.0 * h->esz * n * d,
                            launch_colsum2(dcur, xl, cf32, d, n, d, nullptr, 0, L.rstd, 1.0f, h->part,
-                                          fused ? h->ubuf : outp[p0], fused ? 1 : of32, h->sc, s));
+                                          fused ? uvec(p0) : outp[p0], fused ? 1 : of32, h->sc, s));
                 if (dx_next) {
                     const void* pre = (prev && prev->kind == BOM_LAYER_LINEAR_GELU) ? prev->pre : nullptr;
                     BOM_TRACED("rmsnorm_bwd", 8.0 * n * d, 3.0 * h->esz * n * d + 4.0 * n,
                                launch_rmsnorm_bwd(dcur, xl, gamma, L.rstd, pre, dxo, n, d, cf32, h->sc, s));
                 }
-                if (fused) BOM_TRY(update_small(p0, d));   // after the last read of gamma
+                if (fused && !upd_sep) BOM_TRY(update_small(p0, d));   // after the last read of gamma
             } else {
                 const void* W = params[p0];
                 if (dx_next) {   // dx = dPre W (times GELU' of the previous layer)
@@ -904,15 +947,37 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                         BOM_TRY(run_gemm(h, g, s));
                     }
                 }
-                if (L.bias) {
+                if (L.bias && fold_bias) {
+                    usrc[p0 + 1] = dcur;   // its column sum over the n rows is u of the bias
+                } else if (L.bias) {
                     BOM_TRACED("colsum", 2.0 * n * L.d_out, h->esz * n * L.d_out,
                                launch_colsum(dcur, cf32, L.d_out, n, L.d_out, nullptr, 0, nullptr, 1.0f, h->part,
-                                             fused ? h->ubuf : outp[p0 + 1], fused ? 1 : of32, h->sc, s));
-                    if (fused) BOM_TRY(update_small(p0 + 1, L.d_out));
+                                             fused ? uvec(p0 + 1) : outp[p0 + 1], fused ? 1 : of32, h->sc, s));
+                    if (fused && !upd_sep) BOM_TRY(update_small(p0 + 1, L.d_out));
                 }
             }
             if (dx_next) cur ^= 1;
         }
+    }
+    if (upd_sep) {   // every tensor's BOM-AdamW update, after its last read in the step
+        const int np = bom_param_count(&cfg);
+        std::vector<float*> th(np), vv(np);
+        std::vector<const float*> uu(np);
+        std::vector<void*> cp(np);
+        std::vector<int64_t> rows(np, n);
+        for (int k = 0; k < np; ++k) {
+            th[k] = h->upd_theta[k];
+            vv[k] = h->upd_v[k];
+            uu[k] = h->uscr + h->uoff[k];
+            cp[k] = params[k];
+        }
+        int64_t tot = 0;
+        for (int k = 0; k < np; ++k) tot += h->unum[k];
+        BOM_TRY(traced(h, s, "update", 0, 22.0 * tot, [&] {
+            return launch_update_multi(np, th.data(), vv.data(), uu.data(), cp.data(), cf32, h->unum.data(),
+                                       h->upd_wd.data(), fold_bias ? usrc.data() : nullptr, rows.data(),
+                                       h->upd_beta2, h->upd_eps, h->sc, s);
+        }));
     }
     if (h->t_dev) launch_advance_step(h->t_dev, h->sc, s);
 #undef BOM_TRY

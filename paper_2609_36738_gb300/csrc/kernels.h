@@ -152,6 +152,16 @@ int launch_update(float* theta, const void* g, int g_bf16, const float* h, float
                   float lr, float wd, float lambda, float beta2, float eps, float inv_bc2, const double* clip_sq,
                   float max_norm, const DevScalars* sc, cudaStream_t s, bool step_scalars = false);
 
+// BOM-AdamW update of up to kMultiUpdMax tensors in one launch: fp32 theta,
+// v and u (16-byte aligned) and the compute copy of each (bf16, or fp32 when
+// copy_f32); lr and 1/(1 - beta2^t) from the step scalars in sc; nothing when
+// sc's status is set.  A tensor k with src[k] given is a bias whose u is the
+// column sum of src[k] [rows[k], n[k]] (compute dtype, rows in order).
+constexpr int kMultiUpdMax = 24;
+int launch_update_multi(int ntensor, float* const* theta, float* const* v, const float* const* u, void* const* copy,
+                        int copy_f32, const int64_t* n, const float* wd, const void* const* src, const int64_t* rows,
+                        float beta2, float eps, const DevScalars* sc, cudaStream_t s);
+
 // *sq += sum u^2 over n elements (u = g, or (1-lambda) g + lambda h), in a fixed
 // order; `part` holds kOwnStepMaxBlocks doubles.
 int launch_sqnorm(const void* g, int g_bf16, const float* h, float lambda, int64_t n, double* part, double* sq,

@@ -848,6 +848,140 @@ int launch_update(float* theta, const void* g, int g_bf16, const float* h, float
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }
 
+namespace {
+
+// BOM-AdamW update of several tensors in one launch (the update after a small
+// step's weight gradients; see launch_update_multi).  Each tensor's elements
+// are walked as 16-byte words (fp32 theta, v and u; bf16 compute copy), the
+// tensors one after another in a single grid-stride range.
+struct MultiUpdTable {
+    int ntensor;
+    int copy_f32;                      // compute copies in fp32 (else bf16)
+    int64_t word0[kMultiUpdMax + 1];   // first word of each tensor in the joint range
+    float* theta[kMultiUpdMax];
+    float* v[kMultiUpdMax];
+    const float* u[kMultiUpdMax];
+    void* copy[kMultiUpdMax];
+    int64_t n[kMultiUpdMax];
+    float wd[kMultiUpdMax];
+    // a bias whose u is the column sum of a cotangent: u_j = sum_i src[i, j]
+    // over `rows` rows in order (src [rows, n], compute dtype), else null
+    const void* src[kMultiUpdMax];
+    int64_t rows[kMultiUpdMax];
+};
+
+__global__ void __launch_bounds__(256) update_multi_kernel(const __grid_constant__ MultiUpdTable tb, UpdCoef c_in,
+                                                           const DevScalars* sc) {
+    pdl_enter();
+    if (sc != nullptr && sc->status != 0) return;
+    const int64_t words = tb.word0[tb.ntensor];
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    int k = 0;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < words; i += stride) {
+        while (i >= tb.word0[k + 1]) ++k;   // words only increase along a thread's walk
+        UpdCoef c = c_in;
+        c.wd = tb.wd[k];
+        c = resolve_coef(c, sc);
+        const int64_t w = i - tb.word0[k];
+        const int64_t e0 = 4 * w;
+        const int64_t len = tb.n[k];
+        if (tb.src[k] != nullptr) {   // a bias: u from the column sums of its cotangent
+            const bool f32 = tb.copy_f32 != 0;
+            for (int64_t e = e0; e < e0 + 4 && e < len; ++e) {
+                // rows r = 8q + w in eight interleaved sums, then w = 0..7 in
+                // order: the order of the step's column reduction over one
+                // range of at most 128 rows, so both give the same bits there
+                float a8[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) a8[q] = 0.0f;
+                const int64_t rows = tb.rows[k];
+                int64_t r = 0;
+                for (; r + 8 <= rows; r += 8) {
+                    float x[8];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) x[q] = ld_elem(tb.src[k], (r + q) * len + e, f32 ? 1 : 0);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) a8[q] += x[q];
+                }
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    if (r + q < rows) a8[q] += ld_elem(tb.src[k], (r + q) * len + e, f32 ? 1 : 0);
+                float u = 0.0f;
+#pragma unroll
+                for (int q = 0; q < 8; ++q) u += a8[q];
+                float th = tb.theta[k][e], vv = tb.v[k][e];
+                upd1(th, vv, u, c);
+                tb.theta[k][e] = th;
+                tb.v[k][e] = vv;
+                st_elem(tb.copy[k], e, f32 ? 1 : 0, th);
+            }
+        } else if (e0 + 4 <= len) {
+            float4 th = __ldcs(reinterpret_cast<const float4*>(tb.theta[k]) + w);
+            float4 vv = __ldcs(reinterpret_cast<const float4*>(tb.v[k]) + w);
+            const float4 u = __ldcs(reinterpret_cast<const float4*>(tb.u[k]) + w);
+            upd1(th.x, vv.x, u.x, c);
+            upd1(th.y, vv.y, u.y, c);
+            upd1(th.z, vv.z, u.z, c);
+            upd1(th.w, vv.w, u.w, c);
+            __stcs(reinterpret_cast<float4*>(tb.theta[k]) + w, th);
+            __stcs(reinterpret_cast<float4*>(tb.v[k]) + w, vv);
+            if (tb.copy_f32) {
+                __stcs(reinterpret_cast<float4*>(tb.copy[k]) + w, th);
+            } else {
+                uint2 sh;
+                sh.x = pack_bf16x2(th.x, th.y);
+                sh.y = pack_bf16x2(th.z, th.w);
+                __stcs(reinterpret_cast<uint2*>(tb.copy[k]) + w, sh);
+            }
+        } else {
+            for (int64_t e = e0; e < len; ++e) {
+                float th = tb.theta[k][e], vv = tb.v[k][e];
+                upd1(th, vv, tb.u[k][e], c);
+                tb.theta[k][e] = th;
+                tb.v[k][e] = vv;
+                st_elem(tb.copy[k], e, tb.copy_f32, th);
+            }
+        }
+    }
+}
+
+}  // namespace
+
+int launch_update_multi(int ntensor, float* const* theta, float* const* v, const float* const* u, void* const* copy,
+                        int copy_f32, const int64_t* n, const float* wd, const void* const* src, const int64_t* rows,
+                        float beta2, float eps, const DevScalars* sc, cudaStream_t s) {
+    if (ntensor < 1 || ntensor > kMultiUpdMax) return BOM_EINVAL;
+    MultiUpdTable tb = {};
+    tb.ntensor = ntensor;
+    tb.copy_f32 = copy_f32;
+    int64_t words = 0;
+    for (int k = 0; k < ntensor; ++k) {
+        tb.word0[k] = words;
+        tb.theta[k] = theta[k];
+        tb.v[k] = v[k];
+        tb.u[k] = u[k];
+        tb.copy[k] = copy[k];
+        tb.n[k] = n[k];
+        tb.wd[k] = wd[k];
+        tb.src[k] = src ? src[k] : nullptr;
+        tb.rows[k] = rows ? rows[k] : 0;
+        words += (n[k] + 3) / 4;
+    }
+    tb.word0[ntensor] = words;
+    UpdCoef c = {};
+    c.from_step = 1;   // lr and 1/(1 - beta2^t) from the step scalars
+    c.beta2 = beta2;
+    c.one_m_beta2 = 1.0f - beta2;
+    c.eps = eps;
+    int64_t grid = static_cast<int64_t>(device_sm_count()) * 8;
+    const int64_t need = (words + 255) / 256;
+    if (grid > need) grid = need;
+    if (grid < 1) grid = 1;
+    launch_k(update_multi_kernel, dim3(static_cast<unsigned>(grid)), dim3(256), 0, s, tb, c, sc);
+    count_launch();
+    return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+}
+
 int sqnorm_blocks(int64_t n) {
     int64_t b = static_cast<int64_t>(device_sm_count()) * 4;
     const int64_t need = ((n >> 2) + 255) / 256;

@@ -230,6 +230,12 @@ LM_HEAD_WIDE = Workload("lm_head_wide", 256, 128, (), 8192, False, "bf16", "zipf
 LM_MLP_MID = Workload("lm_mlp_mid", 300, 256, (Layer(SWIGLU, 256, 576), Layer(SWIGLU, 256, 576)),
                       1000, False, "bf16", "zipf", head_init="normal002", ignore_frac=0.05)
 
+# More than 1024 rows with small widths: with the update registered, a step
+# of this size applies it in the weight-gradient GEMMs' epilogues (smaller
+# batches write u and update every tensor in one launch afterwards).
+LM_MLP_K1100 = Workload("lm_mlp_k1100", 1100, 128, (Layer(SWIGLU, 128, 320), Layer(SWIGLU, 128, 320)),
+                        777, False, "bf16", "zipf", head_init="normal002", ignore_frac=0.05)
+
 # RMSNorm variants: an LM block whose head input is normalised (one SwiGLU
 # sublayer, then the final norm, as in the paper's Qwen3 models), and an fp32
 # MLP with a norm between two linear layers.
@@ -244,7 +250,7 @@ LM_NORM_BF16 = Workload("lm_norm_bf16", 16384, 2048,
 
 WORKLOADS = {w.name: w for w in (TINY_MLP_F32, VISION_HEAD_BF16, LM_HEAD_BF16, LM_MLP_BF16,
                                   LM_HEAD_SMALL, LM_MLP_SMALL, VISION_SMALL, TINY_RAGGED_F32, LM_HEAD_WIDE,
-                                  LM_NORM_SMALL, TINY_NORM_F32, LM_NORM_BF16, LM_MLP_MID)}
+                                  LM_NORM_SMALL, TINY_NORM_F32, LM_NORM_BF16, LM_MLP_MID, LM_MLP_K1100)}
 
 
 # --------------------------------------------------------------------------
