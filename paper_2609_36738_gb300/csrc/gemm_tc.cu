@@ -37,7 +37,12 @@ constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = 64;  // one 128-byte swizzle atom of bf16 along K
 constexpr int NUM_THREADS = 320;  // producer warp, UMMA warp, 8 epilogue warps
-constexpr int TMEM_COLS = 512;
+// Narrow single-CTA tiles (128 x 64) for linear-epilogue GEMMs whose 256 x 256
+// tiles would keep at most a quarter of the SMs busy: the epilogue of such a
+// GEMM (bias, GELU or its derivative, residual, one row per thread) takes
+// longer than its mainloop, and 128 x 64 tiles spread it over four times as
+// many SMs.
+constexpr int kBnSmall = 64;
 // Tile raster: groups of group_m consecutive m-tiles with m fastest inside a
 // group (group_m = 1: n fastest along whole rows of tiles).  See raster_group.
 constexpr int GROUP_M = 8;
@@ -243,9 +248,12 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
 constexpr int kEpiLdBlock = 32 * 64;
 constexpr int kEpiLdWarpBytes = 2 * 2 * kEpiLdBlock;
 
-template <int CG, int EPI>
+template <int CG, int EPI, int BNT>
 struct Cfg {
-    static constexpr int B_ROWS = CG == 2 ? 128 : 256;
+    static_assert(BNT == BN || (CG == 1 && BNT == kBnSmall), "narrow tiles are single-CTA only");
+    static constexpr int B_ROWS = CG == 2 ? BN / 2 : BNT;
+    // two accumulators of BNT fp32 columns (an allocation is a power of two >= 32)
+    static constexpr int TMEM_COLS = 2 * BNT;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
     static constexpr int STG_BYTES = EPI == EPI_UPDATE ? 8 * kUpdStgBytes : EPI == EPI_SWIGLU_BWD ? 8 * kEpiLdWarpBytes : 0;
@@ -260,12 +268,12 @@ struct Cfg {
     static constexpr int TILE_M = BM * CG;
 };
 
-template <int CG, bool A_MN, bool B_MN, int EPI>
+template <int CG, bool A_MN, bool B_MN, int EPI, int BNT>
 __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_constant__ Params p) {
     // the next kernel may be scheduled now; this one's own set-up (barriers,
     // TMEM, tensor-map prefetch) runs before it waits for the previous kernel
     pdl_trigger();
-    using C = Cfg<CG, EPI>;
+    using C = Cfg<CG, EPI, BNT>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -311,10 +319,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
     }
     if (warp == 1) {
         if constexpr (CG == 2) {
-            tmem_alloc_pair(tmem_slot, TMEM_COLS);
+            tmem_alloc_pair(tmem_slot, C::TMEM_COLS);
             tmem_relinquish_pair();
         } else {
-            tmem_alloc(tmem_slot, TMEM_COLS);
+            tmem_alloc(tmem_slot, C::TMEM_COLS);
             tmem_relinquish();
         }
     }
@@ -408,7 +416,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
     } else if (!skip && warp == 1) {
         // ------------------------------------------------------------ UMMA issuer (even CTA)
         if (lane == 0 && kb_total > 0 && leader) {
-            constexpr uint32_t idesc = idesc_bf16_f32(C::TILE_M, BN, A_MN, B_MN);
+            constexpr uint32_t idesc = idesc_bf16_f32(C::TILE_M, BNT, A_MN, B_MN);
             constexpr uint32_t b_lbo = 8192;   // MN-major: next 64-column chunk
             int stage = 0;
             uint32_t phase = 0;
@@ -421,7 +429,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 const int nk = min(p.kb_split, kb_total - sp * p.kb_split);
                 if (!mbar_wait_bounded(&tempty[acc], aph ^ 1u, abort_flag)) break;
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BNT);
                 for (int kb = 0; kb < nk; ++kb) {
                     if (!mbar_wait_bounded(&full[stage], phase, abort_flag)) {
                         ok = false;
@@ -472,7 +480,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         const int q = warp & 3;
         const int h = (warp - 2) >> 2;
         const int row = q * 32 + lane;
-        constexpr int CPW = BN / 64;  // 32-column chunks per warp
+        constexpr int CPW = BNT / 64;  // 32-column chunks per warp
         int it = 0;
         // SwiGLU backward operand slots of this warp and their barrier phases
         uint8_t* const eslot = stg_all + (warp - 2) * kEpiLdWarpBytes;
@@ -525,7 +533,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 if (!mbar_wait_bounded(&tfull[acc], (it >> 1) & 1, abort_flag)) break;
                 tc_fence_after();
             }
-            const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+            const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BNT);
             float v[32];
 
             if constexpr (EPI == EPI_LINEAR) {
@@ -795,9 +803,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         __syncwarp();
         tc_fence_after();
         if constexpr (CG == 2)
-            tmem_dealloc_pair(tmem_base, TMEM_COLS);
+            tmem_dealloc_pair(tmem_base, C::TMEM_COLS);
         else
-            tmem_dealloc(tmem_base, TMEM_COLS);
+            tmem_dealloc(tmem_base, C::TMEM_COLS);
     }
     if (threadIdx.x == 0 && *abort_flag && p.epi.sc != nullptr)
         latch_status(const_cast<DevScalars*>(p.epi.sc), BOM_ETIMEOUT);
@@ -842,10 +850,10 @@ static bool map_operand(CUtensorMap* map, const Operand& o, int64_t rows, int64_
     return make_map(map, o.ptr, K, rows, o.ld, 64, rows_box);
 }
 
-template <int CG, bool A_MN, bool B_MN, int EPI>
+template <int CG, bool A_MN, bool B_MN, int EPI, int BNT = BN>
 static int launch_inst(const Params& p, cudaStream_t stream) {
-    using C = Cfg<CG, EPI>;
-    auto k = gemm_kernel<CG, A_MN, B_MN, EPI>;
+    using C = Cfg<CG, EPI, BNT>;
+    auto k = gemm_kernel<CG, A_MN, B_MN, EPI, BNT>;
     // Resident tile walkers: CTAs (CG = 1) or CTA pairs (CG = 2) that fit at
     // once, found (and the kernel's shared-memory attribute set, which is a
     // per-device setting) on the first launch on each device.
@@ -967,6 +975,13 @@ static int choose_split(int tiles, int units, int kb_total, int64_t mn, int64_t 
     return best;
 }
 
+// Linear epilogue on narrow single-CTA tiles; A K-major (the forward layers
+// and the input cotangents of the small configurations).
+static int dispatch_narrow(const Params& p, bool b_mn, cudaStream_t stream) {
+    return b_mn ? launch_inst<1, false, true, EPI_LINEAR, kBnSmall>(p, stream)
+                : launch_inst<1, false, false, EPI_LINEAR, kBnSmall>(p, stream);
+}
+
 template <int CG>
 static int dispatch(const Params& p, int epi_kind, bool a_mn, bool b_mn, bool dual_b, cudaStream_t stream) {
     switch (epi_kind) {
@@ -1023,12 +1038,17 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     if (g.M <= 0 || g.N <= 0) return BOM_OK;
     if (g.M > INT32_MAX / 2 || g.N > INT32_MAX / 2) return BOM_ENOTSUP;
     if (g.epi.in_f32) return BOM_ENOTSUP;   // epilogue operands are bf16 on this engine
-    // CTA pairs (256-row tiles) whenever there is more than one 128-row tile.
-    const int cg = g.M > BM ? 2 : 1;
+    const bool a_mn = g.A[0].mn_major, b_mn = g.B[0].mn_major;
+    // CTA pairs (256-row tiles) whenever there is more than one 128-row tile,
+    // unless the 256-column tiles would leave three quarters of the SMs idle:
+    // then single CTAs with 128 x 64 tiles (linear epilogue, A K-major).
+    const int64_t wide_ctas = ((g.M + BM - 1) / BM) * ((g.N + BN - 1) / BN);
+    const bool narrow = g.epi_kind == EPI_LINEAR && !g.dual_b && !a_mn && 4 * wide_ctas <= device_sm_count();
+    const int cg = (g.M > BM && !narrow) ? 2 : 1;
     Params p;
     memset(&p, 0, sizeof(p));
-    const bool a_mn = g.A[0].mn_major, b_mn = g.B[0].mn_major;
-    const uint32_t b_rows = (cg == 2 || g.dual_b) ? 128 : 256;   // B rows one CTA loads per stage
+    // B rows one CTA loads per stage
+    const uint32_t b_rows = narrow ? kBnSmall : (cg == 2 || g.dual_b) ? 128 : 256;
     for (int s = 0; s < g.nseg; ++s) {
         if (g.A[s].mn_major != a_mn || g.B[s].mn_major != b_mn) return BOM_ENOTSUP;
         p.kb[s] = static_cast<int>((g.K[s] + BK - 1) / BK);
@@ -1049,7 +1069,7 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     p.N = static_cast<int>(g.N);
     p.nseg = g.nseg;
     p.dual_b = g.dual_b ? 1 : 0;
-    p.bn_out = g.dual_b ? 128 : BN;
+    p.bn_out = narrow ? kBnSmall : g.dual_b ? 128 : BN;
     p.tiles_m = static_cast<int>((g.M + BM * cg - 1) / (BM * cg));
     p.tiles_n = static_cast<int>((g.N + p.bn_out - 1) / p.bn_out);
     p.group_m = raster_group(p.tiles_m, p.tiles_n);
@@ -1081,8 +1101,9 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     // split-K partial tiles are raw (linear epilogue); the update, if any,
     // runs in the reduction
     const int kind = S > 1 ? EPI_LINEAR : g.epi_kind;
-    const int rc = cg == 2 ? dispatch<2>(p, kind, a_mn, b_mn, g.dual_b, stream)
-                           : dispatch<1>(p, kind, a_mn, b_mn, g.dual_b, stream);
+    const int rc = narrow    ? dispatch_narrow(p, b_mn, stream)
+                   : cg == 2 ? dispatch<2>(p, kind, a_mn, b_mn, g.dual_b, stream)
+                             : dispatch<1>(p, kind, a_mn, b_mn, g.dual_b, stream);
     if (rc != BOM_OK || S == 1) return rc;
     const int64_t total = static_cast<int64_t>(g.M) * g.N;
     int64_t blocks = (total + 255) / 256;
