@@ -49,6 +49,10 @@ struct LayerWs {
     int64_t gu_ld = 0;       // 2 * ffn rounded up to 64
     void* A = nullptr;       // SWIGLU SiLU(G) * U [n, ffn]
     float* rstd = nullptr;   // RMSNORM 1 / sqrt(mean x^2 + eps) per row [n]
+    // a biased Linear layer of a small batch (bf16): fp32 column sums of its
+    // output cotangent per 32-row block [ceil(n / 32), d_out], written by the
+    // epilogue of the GEMM that produces the cotangent
+    float* cspart = nullptr;
 };
 
 int64_t round_up(int64_t a, int64_t b) { return (a + b - 1) / b * b; }
@@ -222,6 +226,8 @@ size_t carve(bom_handle* h, char* base) {
         } else if (L.kind == BOM_LAYER_RMSNORM) {
             L.rstd = static_cast<float*>(c.take(n * 4));
         }
+        if (h->bf16 && L.bias && n <= kUpdSepRows && (L.kind == BOM_LAYER_LINEAR || L.kind == BOM_LAYER_LINEAR_GELU))
+            L.cspart = static_cast<float*>(c.take((n + 31) / 32 * L.d_out * 4));
         L.out = c.take(n * L.width_out * e);
     }
     // logits rows start on 128-byte boundaries: each 64-byte row segment an
@@ -547,8 +553,20 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     // a Linear layer's bias gradient (their column sum) is formed by the final
     // update itself, in the order of the column reduction over one range.
     const bool fold_bias = upd_sep && h->lw.size() <= 2 && n <= kRowBlock;
+    // Otherwise (bf16) the GEMM that writes a biased Linear layer's output
+    // cotangent also writes its column sums per 32-row block, and the final
+    // update adds those up: no column-reduction launches.
+    const bool cs_fused = upd_sep && h->bf16 && !fold_bias;
     std::vector<const void*> usrc;
-    if (fold_bias) usrc.assign(bom_param_count(&h->cfg), nullptr);
+    std::vector<int64_t> urows;
+    std::vector<int> usf32;
+    if (fold_bias || cs_fused) {
+        const int npar = bom_param_count(&h->cfg);
+        usrc.assign(npar, nullptr);
+        urows.assign(npar, n);
+        usf32.assign(npar, h->bf16 ? 0 : 1);
+    }
+    std::vector<char> cs_ready(h->lw.size(), 0);   // per layer: its cotangent's column sums are being written
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const bom_config& cfg = h->cfg;
     const int64_t V = cfg.d_out, dm = h->d_model;
@@ -781,6 +799,11 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
             g.epi.out = h->lw.empty() ? h->dx_in : h->dx[cur];
             g.epi.ld_out = dm;
             g.epi.out_f32 = cf32;
+            if (cs_fused && !h->lw.empty() && h->lw.back().cspart != nullptr) {
+                g.epi.colsum = h->lw.back().cspart;
+                g.epi.ld_colsum = h->lw.back().d_out;
+                cs_ready.back() = 1;
+            }
             BOM_TRY(run_gemm(h, g, s));
         }
         // The head weight gradient contracts over the same n rows as the
@@ -876,6 +899,11 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                     g.epi.out = dxo;
                     g.epi.ld_out = d;
                     g.epi.out_f32 = cf32;
+                    if (cs_fused && prev && prev->cspart != nullptr) {
+                        g.epi.colsum = prev->cspart;
+                        g.epi.ld_colsum = prev->d_out;
+                        cs_ready[l - 1] = 1;
+                    }
                     BOM_TRY(run_gemm(h, g, s));
                 }
                 {   // dW_g = dG^T x, dW_u = dU^T x, dW_d = dy^T A: one launch over their tiles
@@ -926,6 +954,11 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                     g.epi.out = dxo;
                     g.epi.ld_out = L.d_in;
                     g.epi.out_f32 = cf32;
+                    if (cs_fused && prev && prev->cspart != nullptr) {
+                        g.epi.colsum = prev->cspart;
+                        g.epi.ld_colsum = prev->d_out;
+                        cs_ready[l - 1] = 1;
+                    }
                     BOM_TRY(run_gemm(h, g, s));
                 }
                 {   // dW = dPre^T x
@@ -949,6 +982,10 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                 }
                 if (L.bias && fold_bias) {
                     usrc[p0 + 1] = dcur;   // its column sum over the n rows is u of the bias
+                } else if (L.bias && cs_ready[l]) {
+                    usrc[p0 + 1] = L.cspart;   // u of the bias: the sum of the block column sums
+                    urows[p0 + 1] = (n + 31) / 32;
+                    usf32[p0 + 1] = 1;
                 } else if (L.bias) {
                     BOM_TRACED("colsum", 2.0 * n * L.d_out, h->esz * n * L.d_out,
                                launch_colsum(dcur, cf32, L.d_out, n, L.d_out, nullptr, 0, nullptr, 1.0f, h->part,
@@ -964,7 +1001,6 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
         std::vector<float*> th(np), vv(np);
         std::vector<const float*> uu(np);
         std::vector<void*> cp(np);
-        std::vector<int64_t> rows(np, n);
         for (int k = 0; k < np; ++k) {
             th[k] = h->upd_theta[k];
             vv[k] = h->upd_v[k];
@@ -975,7 +1011,8 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
         for (int k = 0; k < np; ++k) tot += h->unum[k];
         BOM_TRY(traced(h, s, "update", 0, 22.0 * tot, [&] {
             return launch_update_multi(np, th.data(), vv.data(), uu.data(), cp.data(), cf32, h->unum.data(),
-                                       h->upd_wd.data(), fold_bias ? usrc.data() : nullptr, rows.data(),
+                                       h->upd_wd.data(), usrc.empty() ? nullptr : usrc.data(),
+                                       urows.empty() ? nullptr : urows.data(), usf32.empty() ? nullptr : usf32.data(),
                                        h->upd_beta2, h->upd_eps, h->sc, s);
         }));
     }

@@ -157,6 +157,12 @@ struct EpiParams {
     float* upd_theta;
     float* upd_v;
     float upd_wd, upd_beta2, upd_1mb2, upd_eps;
+    // Column sums of the stored output (EPI_LINEAR on the tcgen05 engine, no
+    // split-K): colsum[b * ld_colsum + n] = sum of out[m, n] over the 32 rows
+    // m of block b (rows past M count 0), as stored (bf16-rounded when out is
+    // bf16).  Null: none.
+    float* colsum;
+    int64_t ld_colsum;
 };
 
 // One element of the fused update (Section 3.4): returns the new theta.
@@ -199,6 +205,23 @@ __device__ __forceinline__ void st_elem(void* base, int64_t idx, int is_f32, flo
         static_cast<__nv_bfloat16*>(base)[idx] = __float2bfloat16_rn(v);
 }
 __device__ __forceinline__ float round_bf16(float v) { return __bfloat162float(__float2bfloat16_rn(v)); }
+
+// Column sums of a warp's 32 x 32 block (x: this lane's row): a butterfly
+// that halves the columns each lane holds at every level, so lane i returns
+// the sum of column i over the 32 lanes (a fixed order, 31 shuffles).
+__device__ __forceinline__ float warp_colsum32(float (&x)[32], int lane) {
+#pragma unroll
+    for (int s = 16; s >= 1; s >>= 1) {
+        const bool up = (lane & s) != 0;
+#pragma unroll
+        for (int i = 0; i < s; ++i) {
+            const float send = up ? x[i] : x[i + s];
+            const float keep = up ? x[i + s] : x[i];
+            x[i] = keep + __shfl_xor_sync(0xffffffffu, send, s);
+        }
+    }
+    return x[0];
+}
 
 // ---------------------------------------------------------------- packed arithmetic
 // Instruction-lean forms for the epilogues and streaming passes that are

@@ -586,6 +586,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         }
                         store_row32(out_base, static_cast<int64_t>(m) * e.ld_out, n, PN, e.out_f32, v);
                     }
+                    if (e.colsum != nullptr) {
+                        // the 32 rows of this warp, column by column: lane i
+                        // ends with the sum of column n + i
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) t[i] = valid ? (e.out_f32 ? v[i] : round_bf16(v[i])) : 0.0f;
+                        const float cs = warp_colsum32(t, lane);
+                        if (row0 < PM && n + lane < PN)
+                            e.colsum[static_cast<int64_t>(row0 >> 5) * e.ld_colsum + n + lane] = cs;
+                    }
                 }
             } else if constexpr (EPI == EPI_UPDATE) {
                 const EpiRow r = epi_row(e, m, PM);
@@ -975,9 +984,11 @@ static int choose_split(int tiles, int units, int kb_total, int64_t mn, int64_t 
     return best;
 }
 
-// Linear epilogue on narrow single-CTA tiles; A K-major (the forward layers
-// and the input cotangents of the small configurations).
-static int dispatch_narrow(const Params& p, bool b_mn, cudaStream_t stream) {
+// Linear epilogue on narrow single-CTA tiles: A K-major (the forward layers
+// and the input cotangents of the small configurations), or both operands
+// MN-major (their weight gradients, K = the batch rows).
+static int dispatch_narrow(const Params& p, bool a_mn, bool b_mn, cudaStream_t stream) {
+    if (a_mn) return b_mn ? launch_inst<1, true, true, EPI_LINEAR, kBnSmall>(p, stream) : BOM_ENOTSUP;
     return b_mn ? launch_inst<1, false, true, EPI_LINEAR, kBnSmall>(p, stream)
                 : launch_inst<1, false, false, EPI_LINEAR, kBnSmall>(p, stream);
 }
@@ -1081,7 +1092,8 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     p.tile_base[1] = tiles;
     const int units = cg == 2 ? device_sm_count() / 2 : device_sm_count();
     int S = 1;
-    if ((g.epi_kind == EPI_LINEAR || g.epi_kind == EPI_UPDATE) && g.splitk_ws != nullptr)
+    // (column sums are formed in the tile epilogue: no split)
+    if ((g.epi_kind == EPI_LINEAR || g.epi_kind == EPI_UPDATE) && g.splitk_ws != nullptr && g.epi.colsum == nullptr)
         S = choose_split(tiles, units, kb_total, static_cast<int64_t>(g.M) * g.N, g.splitk_ws_elems);
     p.ksplit = S;
     p.kb_split = S > 1 ? (kb_total + S - 1) / S : kb_total;
@@ -1101,7 +1113,7 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
     // split-K partial tiles are raw (linear epilogue); the update, if any,
     // runs in the reduction
     const int kind = S > 1 ? EPI_LINEAR : g.epi_kind;
-    const int rc = narrow    ? dispatch_narrow(p, b_mn, stream)
+    const int rc = narrow    ? dispatch_narrow(p, a_mn, b_mn, stream)
                    : cg == 2 ? dispatch<2>(p, kind, a_mn, b_mn, g.dual_b, stream)
                              : dispatch<1>(p, kind, a_mn, b_mn, g.dual_b, stream);
     if (rc != BOM_OK || S == 1) return rc;
@@ -1142,8 +1154,14 @@ int launch_gemm_tc_group(const GemmDesc* gs, int n, cudaStream_t stream) {
     memset(&p, 0, sizeof(p));
     const GemmDesc& g0 = gs[0];
     p.kb[0] = static_cast<int>((g0.K[0] + BK - 1) / BK);
+    // Weight gradients over a short K (at most 16 k-blocks: small batches)
+    // with a linear epilogue (u to memory) spend most of a 256 x 256 tile in
+    // its epilogue, and their few hundred tiles end on a partial wave of
+    // CTA pairs: single CTAs with 128 x 64 tiles instead.
+    const bool narrow = g0.epi_kind == EPI_LINEAR && p.kb[0] <= 16 && g0.A[0].mn_major && g0.B[0].mn_major;
+    const int tile_m = narrow ? BM : 2 * BM, tile_n = narrow ? kBnSmall : BN;
     p.nseg = 1;
-    p.bn_out = BN;
+    p.bn_out = tile_n;
     p.ksplit = 1;
     p.kb_split = p.kb[0];
     p.nprob = n;
@@ -1152,10 +1170,11 @@ int launch_gemm_tc_group(const GemmDesc* gs, int n, cudaStream_t stream) {
         const GemmDesc& g = gs[i];
         CUtensorMap* ma = i == 0 ? &p.mapA[0] : &p.grp[i - 1].mapA;
         CUtensorMap* mb = i == 0 ? &p.mapB[0] : &p.grp[i - 1].mapB;
-        if (g.K[0] > 0 && (!map_operand(ma, g.A[0], g.M, g.K[0], BM) || !map_operand(mb, g.B[0], g.N, g.K[0], 128)))
+        if (g.K[0] > 0 && (!map_operand(ma, g.A[0], g.M, g.K[0], BM) ||
+                           !map_operand(mb, g.B[0], g.N, g.K[0], narrow ? kBnSmall : 128)))
             return BOM_ENOTSUP;
-        const int tm = static_cast<int>((g.M + 2 * BM - 1) / (2 * BM));
-        const int tn = static_cast<int>((g.N + BN - 1) / BN);
+        const int tm = static_cast<int>((g.M + tile_m - 1) / tile_m);
+        const int tn = static_cast<int>((g.N + tile_n - 1) / tile_n);
         if (i == 0) {
             p.M = static_cast<int>(g.M);
             p.N = static_cast<int>(g.N);
@@ -1176,6 +1195,7 @@ int launch_gemm_tc_group(const GemmDesc* gs, int n, cudaStream_t stream) {
         tiles += tm * tn;
     }
     p.tile_base[n] = tiles;
+    if (narrow) return dispatch_narrow(p, true, true, stream);
     return dispatch<2>(p, g0.epi_kind, g0.A[0].mn_major, g0.B[0].mn_major, false, stream);
 }
 

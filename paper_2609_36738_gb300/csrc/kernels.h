@@ -156,11 +156,12 @@ int launch_update(float* theta, const void* g, int g_bf16, const float* h, float
 // v and u (16-byte aligned) and the compute copy of each (bf16, or fp32 when
 // copy_f32); lr and 1/(1 - beta2^t) from the step scalars in sc; nothing when
 // sc's status is set.  A tensor k with src[k] given is a bias whose u is the
-// column sum of src[k] [rows[k], n[k]] (compute dtype, rows in order).
+// column sum of src[k] [rows[k], n[k]] (rows in order; fp32 when src_f32[k]
+// is 1, else the compute dtype; src_f32 null: the compute dtype).
 constexpr int kMultiUpdMax = 24;
 int launch_update_multi(int ntensor, float* const* theta, float* const* v, const float* const* u, void* const* copy,
                         int copy_f32, const int64_t* n, const float* wd, const void* const* src, const int64_t* rows,
-                        float beta2, float eps, const DevScalars* sc, cudaStream_t s);
+                        const int* src_f32, float beta2, float eps, const DevScalars* sc, cudaStream_t s);
 
 // *sq += sum u^2 over n elements (u = g, or (1-lambda) g + lambda h), in a fixed
 // order; `part` holds kOwnStepMaxBlocks doubles.

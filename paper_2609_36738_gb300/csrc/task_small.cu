@@ -117,27 +117,25 @@ __device__ __forceinline__ void colsum_tile(const void* X, int64_t dm, int64_t j
         for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
         int64_t j = j0 + g;
         if (vec) {
+            // batches of four rows, the last one predicated (a missing row
+            // reads nothing and has weight 0): every batch has its four loads
+            // in flight, and the rows are still added in increasing order
             const T* base = static_cast<const T*>(X) + kc * EPC;
-            for (; j + 3 * RG < j1; j += 4 * RG) {
+            for (; j < j1; j += 4 * RG) {
                 uint4 w[4];
                 float f[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    w[u] = __ldg(reinterpret_cast<const uint4*>(base + (j + u * RG) * dm));
-                    f[u] = wt(j + u * RG);
+                    const int64_t jj = j + u * RG;
+                    w[u] = jj < j1 ? __ldg(reinterpret_cast<const uint4*>(base + jj * dm)) : make_uint4(0u, 0u, 0u, 0u);
+                    f[u] = jj < j1 ? wt(jj) : 0.0f;
                 }
 #pragma unroll
                 for (int u = 0; u < 4; ++u)
+                    if (j + u * RG < j1)
 #pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        if (e < EPC) acc[e] = fmaf(f[u], word_at<T>(w[u], e), acc[e]);
-            }
-            for (; j < j1; j += RG) {
-                const uint4 w = __ldg(reinterpret_cast<const uint4*>(base + j * dm));
-                const float f = wt(j);
-#pragma unroll
-                for (int e = 0; e < 8; ++e)
-                    if (e < EPC) acc[e] = fmaf(f, word_at<T>(w, e), acc[e]);
+                        for (int e = 0; e < 8; ++e)
+                            if (e < EPC) acc[e] = fmaf(f[u], word_at<T>(w[u], e), acc[e]);
             }
         } else {
             for (; j < j1; j += RG) acc[0] = fmaf(wt(j), ld_t<T>(X, j * dm + kc), acc[0]);
@@ -182,6 +180,17 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
     int* tot_i = reinterpret_cast<int*>(tot_f + 2);      // [0] N_t, [1] bad, [2] non-finite
 
     const int tid = threadIdx.x, w = tid >> 5, l = tid & 31;
+    // the device step counter and learning rate are loaded now and kept
+    // after phase 1a, so that their latency is off the single-thread chain of
+    // phase 2
+    __shared__ int64_t s_t;
+    __shared__ float s_lr;
+    int64_t t_ld = 1;
+    float lr_ld = a.st.lr;
+    if (tid == 0) {
+        if (a.st.t_dev != nullptr) t_ld = __ldcg(a.st.t_dev);
+        if (a.st.lr_dev != nullptr) lr_ld = __ldcg(a.st.lr_dev);
+    }
     const bool live = a.sc->status == 0;
     const int64_t r0 = c * rp < n ? c * rp : n;
     const int64_t r1 = r0 + rp < n ? r0 + rp : n;
@@ -194,7 +203,8 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
     // are padded to whole 128-byte lines), four words in flight per lane
     float ce_w = 0.0f;
     int nt_w = 0, bad_w = 0, nf_w = 0;
-    if (live) {
+    {   // read whatever the status word says (it only gates the writes), so
+        // that its latency overlaps the row reads
         const int64_t nw = (V + EPC - 1) / EPC;
         for (int64_t r = r0 + w; r < r1; r += kSmallThreads / 32) {
             const int32_t y = a.labels[r];
@@ -202,6 +212,71 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
             const bool ok_y = sup && y >= 0 && y < V;
             const T* zr = static_cast<const T*>(a.Z) + r * a.ldz;
             float m = -INFINITY;
+            if (nw <= 128) {
+                // the whole row in registers (four words per lane): one read
+                // for the maximum, the sum and z_y
+                uint4 wd[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    wd[u] = l + 32 * u < nw ? *reinterpret_cast<const uint4*>(zr + (l + 32 * u) * EPC)
+                                            : make_uint4(0u, 0u, 0u, 0u);
+                if constexpr (sizeof(T) == 2) {
+                    // packed maximum on the raw bf16 pairs (columns past V
+                    // masked to -inf), so the unpacked values live only in
+                    // the sum below
+                    uint32_t mm = 0xFF80FF80u;
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int64_t c0 = (l + 32 * u) * EPC;
+                        const uint32_t x4[4] = {wd[u].x, wd[u].y, wd[u].z, wd[u].w};
+#pragma unroll
+                        for (int q2 = 0; q2 < 4; ++q2) {
+                            const int64_t cc = c0 + 2 * q2;
+                            const uint32_t lo = cc < V ? (x4[q2] & 0xFFFFu) : 0xFF80u;
+                            const uint32_t hi = cc + 1 < V ? (x4[q2] & 0xFFFF0000u) : 0xFF800000u;
+                            mm = max_bf16x2(mm, lo | hi);
+                        }
+                    }
+                    m = fmaxf(bf16_lo(mm), bf16_hi(mm));
+                } else {
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+#pragma unroll
+                        for (int e = 0; e < EPC; ++e)
+                            if ((l + 32 * u) * EPC + e < V) m = fmaxf(m, word_at<T>(wd[u], e));
+                }
+                m = warp_max_f(m);
+                float s = 0.0f;
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+#pragma unroll
+                    for (int e = 0; e < EPC; ++e)
+                        if ((l + 32 * u) * EPC + e < V) s += expf(word_at<T>(wd[u], e) - m);
+                s = warp_sum_f(s);
+                // z_y from the lane holding word y / EPC (ok_y is the same on every lane)
+                float zy = 0.0f;
+                if (ok_y) {
+                    const int kw = y / EPC, ey = y - kw * EPC, su = kw >> 5;
+                    float cand = 0.0f;
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+                        if (u == su) cand = word_at<T>(wd[u], ey);
+                    zy = __shfl_sync(0xffffffffu, cand, kw & 31);
+                }
+                if (l == 0) {
+                    const float L = m + logf(s);
+                    lse_s[r - r0] = L;
+                    lab_s[r - r0] = ok_y ? y : -1;
+                    if (live) a.lse[r] = L;
+                    if (sup && !ok_y) ++bad_w;
+                    if (ok_y) {
+                        ++nt_w;
+                        ce_w += L - zy;
+                    }
+                    if (!isfinite(L) || (ok_y && !isfinite(zy))) ++nf_w;
+                }
+                continue;
+            }
             for (int64_t b = l; b < nw; b += 128) {
                 uint4 wd[4];
 #pragma unroll
@@ -233,7 +308,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
                 const float L = m + logf(s);
                 lse_s[r - r0] = L;
                 lab_s[r - r0] = ok_y ? y : -1;
-                a.lse[r] = L;
+                if (live) a.lse[r] = L;
                 const float zy = ok_y ? ld_t<T>(a.Z, r * a.ldz + y) : 0.0f;
                 if (sup && !ok_y) ++bad_w;
                 if (ok_y) {
@@ -249,6 +324,10 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
         wnt[w] = nt_w;
         wbad[w] = bad_w;
         wnf[w] = nf_w;
+    }
+    if (tid == 0) {
+        s_t = t_ld;
+        s_lr = lr_ld;
     }
     __syncthreads();
     if (tid == 0) {
@@ -301,9 +380,14 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
     }
     cl.sync();
 
-    // ---- phase 2: totals, status, s / q / qhat of the CTA's vocabulary slice
-    __shared__ int s_code;
-    __shared__ float s_inv_nt, s_bc1, s_bc2;
+    // ---- phase 2: totals, status, s / q / qhat of the CTA's vocabulary slice.
+    // The two bias corrections (fp64 products) are formed by two other
+    // threads at the same time as the totals.
+    __shared__ int s_code, s_nt;
+    __shared__ float s_inv_nt, s_bc1, s_bc2, s_tot_ce;
+    const bool t_bad = a.st.t_dev != nullptr && s_t < 1;
+    if (tid == 32) s_bc1 = (a.st.t_dev != nullptr && !t_bad) ? inv_bias_correction(a.st.beta1, s_t) : a.st.inv_bc1;
+    if (tid == 64) s_bc2 = (a.st.t_dev != nullptr && !t_bad) ? inv_bias_correction(a.st.beta2, s_t) : a.st.inv_bc2;
     if (tid == 0) {
         float ce = 0.0f;
         int nt = 0, bad = 0, nf = 0;
@@ -315,17 +399,6 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
             nt += ti[0];
             bad += ti[1];
             nf += ti[2];
-        }
-        float bc1 = a.st.inv_bc1, bc2 = a.st.inv_bc2;
-        bool t_bad = false;
-        if (a.st.t_dev != nullptr) {
-            const int64_t t = *a.st.t_dev;
-            if (t < 1) {
-                t_bad = true;
-            } else {
-                bc1 = inv_bias_correction(a.st.beta1, t);
-                bc2 = inv_bias_correction(a.st.beta2, t);
-            }
         }
         int code = live ? 0 : -1;
         if (live) {
@@ -340,10 +413,15 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
         }
         const float inv = nt > 0 ? 1.0f / static_cast<float>(nt) : 0.0f;
         s_code = code;
+        s_nt = nt;
         s_inv_nt = inv;
-        s_bc1 = bc1;
-        s_bc2 = bc2;
-        if (c == 0 && live) {
+        s_tot_ce = ce;
+    }
+    __syncthreads();
+    if (tid == 0 && c == 0 && live) {
+        const int code = s_code, nt = s_nt;
+        const float inv = s_inv_nt, ce = s_tot_ce;
+        {
             DevScalars* sc = a.sc;
             if (code > 0) latch_status(sc, code);
             sc->n_t = nt;
@@ -356,9 +434,9 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
             sc->coef_q[2] = inv;
             sc->coef_r[3] = 0.0f;
             sc->coef_q[3] = inv;
-            sc->lr = a.st.lr_dev != nullptr ? *a.st.lr_dev : a.st.lr;
-            sc->inv_bc1 = bc1;
-            sc->inv_bc2 = bc2;
+            sc->lr = s_lr;
+            sc->inv_bc1 = s_bc1;
+            sc->inv_bc2 = s_bc2;
             sc->loss = ce * inv;
             sc->s_norm = 0.0f;
             sc->r_norm_mean = 0.0f;

@@ -865,9 +865,11 @@ struct MultiUpdTable {
     int64_t n[kMultiUpdMax];
     float wd[kMultiUpdMax];
     // a bias whose u is the column sum of a cotangent: u_j = sum_i src[i, j]
-    // over `rows` rows in order (src [rows, n], compute dtype), else null
+    // over `rows` rows in order (src [rows, n]: the cotangent in the compute
+    // dtype, or fp32 column sums of its 32-row blocks), else null
     const void* src[kMultiUpdMax];
     int64_t rows[kMultiUpdMax];
+    int src_f32[kMultiUpdMax];
 };
 
 __global__ void __launch_bounds__(256) update_multi_kernel(const __grid_constant__ MultiUpdTable tb, UpdCoef c_in,
@@ -885,8 +887,57 @@ __global__ void __launch_bounds__(256) update_multi_kernel(const __grid_constant
         const int64_t w = i - tb.word0[k];
         const int64_t e0 = 4 * w;
         const int64_t len = tb.n[k];
-        if (tb.src[k] != nullptr) {   // a bias: u from the column sums of its cotangent
-            const bool f32 = tb.copy_f32 != 0;
+        if (tb.src[k] != nullptr && tb.src_f32[k] && e0 + 4 <= len && (len & 3) == 0) {
+            // a bias whose u sums fp32 rows (16-byte aligned): the word's four
+            // columns at once, every row load and theta, v in flight together;
+            // per column the same order of additions as the loop below
+            const float4* sp = static_cast<const float4*>(tb.src[k]) + w;
+            const int64_t rstride = len / 4;
+            float4 th = __ldcs(reinterpret_cast<const float4*>(tb.theta[k]) + w);
+            float4 vv = __ldcs(reinterpret_cast<const float4*>(tb.v[k]) + w);
+            float4 a8[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) a8[q] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            const int64_t rows = tb.rows[k];
+            int64_t r = 0;
+            for (; r + 8 <= rows; r += 8) {
+                float4 x[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) x[q] = sp[(r + q) * rstride];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    a8[q].x += x[q].x;
+                    a8[q].y += x[q].y;
+                    a8[q].z += x[q].z;
+                    a8[q].w += x[q].w;
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (r + q < rows) {
+                    const float4 x = sp[(r + q) * rstride];
+                    a8[q].x += x.x;
+                    a8[q].y += x.y;
+                    a8[q].z += x.z;
+                    a8[q].w += x.w;
+                }
+            float4 u = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                u.x += a8[q].x;
+                u.y += a8[q].y;
+                u.z += a8[q].z;
+                u.w += a8[q].w;
+            }
+            upd1(th.x, vv.x, u.x, c);
+            upd1(th.y, vv.y, u.y, c);
+            upd1(th.z, vv.z, u.z, c);
+            upd1(th.w, vv.w, u.w, c);
+            reinterpret_cast<float4*>(tb.theta[k])[w] = th;
+            reinterpret_cast<float4*>(tb.v[k])[w] = vv;
+            for (int j = 0; j < 4; ++j) st_elem(tb.copy[k], e0 + j, tb.copy_f32, j == 0 ? th.x : j == 1 ? th.y : j == 2 ? th.z : th.w);
+        } else if (tb.src[k] != nullptr) {   // a bias: u from the column sums of its cotangent
+            const int f32 = tb.src_f32[k];
             for (int64_t e = e0; e < e0 + 4 && e < len; ++e) {
                 // rows r = 8q + w in eight interleaved sums, then w = 0..7 in
                 // order: the order of the step's column reduction over one
@@ -899,13 +950,13 @@ __global__ void __launch_bounds__(256) update_multi_kernel(const __grid_constant
                 for (; r + 8 <= rows; r += 8) {
                     float x[8];
 #pragma unroll
-                    for (int q = 0; q < 8; ++q) x[q] = ld_elem(tb.src[k], (r + q) * len + e, f32 ? 1 : 0);
+                    for (int q = 0; q < 8; ++q) x[q] = ld_elem(tb.src[k], (r + q) * len + e, f32);
 #pragma unroll
                     for (int q = 0; q < 8; ++q) a8[q] += x[q];
                 }
 #pragma unroll
                 for (int q = 0; q < 8; ++q)
-                    if (r + q < rows) a8[q] += ld_elem(tb.src[k], (r + q) * len + e, f32 ? 1 : 0);
+                    if (r + q < rows) a8[q] += ld_elem(tb.src[k], (r + q) * len + e, f32);
                 float u = 0.0f;
 #pragma unroll
                 for (int q = 0; q < 8; ++q) u += a8[q];
@@ -913,7 +964,7 @@ __global__ void __launch_bounds__(256) update_multi_kernel(const __grid_constant
                 upd1(th, vv, u, c);
                 tb.theta[k][e] = th;
                 tb.v[k][e] = vv;
-                st_elem(tb.copy[k], e, f32 ? 1 : 0, th);
+                st_elem(tb.copy[k], e, tb.copy_f32, th);
             }
         } else if (e0 + 4 <= len) {
             float4 th = __ldcs(reinterpret_cast<const float4*>(tb.theta[k]) + w);
@@ -949,7 +1000,7 @@ __global__ void __launch_bounds__(256) update_multi_kernel(const __grid_constant
 
 int launch_update_multi(int ntensor, float* const* theta, float* const* v, const float* const* u, void* const* copy,
                         int copy_f32, const int64_t* n, const float* wd, const void* const* src, const int64_t* rows,
-                        float beta2, float eps, const DevScalars* sc, cudaStream_t s) {
+                        const int* src_f32, float beta2, float eps, const DevScalars* sc, cudaStream_t s) {
     if (ntensor < 1 || ntensor > kMultiUpdMax) return BOM_EINVAL;
     MultiUpdTable tb = {};
     tb.ntensor = ntensor;
@@ -965,6 +1016,7 @@ int launch_update_multi(int ntensor, float* const* theta, float* const* v, const
         tb.wd[k] = wd[k];
         tb.src[k] = src ? src[k] : nullptr;
         tb.rows[k] = rows ? rows[k] : 0;
+        tb.src_f32[k] = src_f32 ? src_f32[k] : copy_f32;
         words += (n[k] + 3) / 4;
     }
     tb.word0[ntensor] = words;

@@ -44,9 +44,11 @@ class Fused:
 # Up to 1024 rows the bf16 step writes u and updates every tensor in one
 # launch after the pass; lm_mlp_k1100 (1100 rows) takes the update in the
 # weight-gradient GEMMs' epilogues, as the full-size LM block does.
+# vision_mid and vision_head_bf16 (300 and 256 rows) take the bias gradients
+# from the column sums of 32-row blocks formed in the cotangent GEMMs.
 @pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "tiny_norm_f32", "vision_small",
-                                  "lm_head_small", "lm_mlp_small", "lm_norm_small", "lm_head_wide",
-                                  "lm_mlp_mid", "lm_mlp_k1100"])
+                                  "vision_mid", "vision_head_bf16", "lm_head_small", "lm_mlp_small",
+                                  "lm_norm_small", "lm_head_wide", "lm_mlp_mid", "lm_mlp_k1100"])
 def test_fused_update_matches_oracle_on_the_same_inputs(name):
     wl = I.WORKLOADS[name]
     tol = G.TOL[wl.dtype]
