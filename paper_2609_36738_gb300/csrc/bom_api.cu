@@ -667,13 +667,18 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     const void* bh = head_b >= 0 ? params[head_b] : nullptr;
     if (run_fwd) {
         GemmDesc g = gemm1(n, V, dm, kmaj(xin, dm), kmaj(Wh, dm));
-        g.epi_kind = EPI_LOGITS;
+        // the small task pass forms the row statistics from Z itself: on the
+        // tensor-core engine its logits are a plain linear GEMM (narrow tiles
+        // when there are few), without the per-tile softmax statistics
+        g.epi_kind = small && h->bf16 ? EPI_LINEAR : EPI_LOGITS;
         g.epi.bias = bh;
         g.epi.out = h->Z;
         g.epi.ld_out = h->ldz;
         g.epi.out_f32 = cf32;
-        g.epi.stats = h->stats;
-        g.epi.ld_stats = h->ntiles;
+        if (g.epi_kind == EPI_LOGITS) {
+            g.epi.stats = h->stats;
+            g.epi.ld_stats = h->ntiles;
+        }
         BOM_TRY(run_gemm(h, g, s));
     }
     if (run_fwd && !h->bf16 && !small)

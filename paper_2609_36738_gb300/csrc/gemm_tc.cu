@@ -529,6 +529,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, PN, xa, 0);
                 if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, PN, xb, 0);
             }
+            // linear epilogue: the row's factors, and on narrow tiles (one
+            // chunk per warp) the chunk's bias and broadcast row, are read
+            // before the accumulator is waited for
+            EpiRow r_lin{};
+            float vb[32], vw[32];
+            if constexpr (EPI == EPI_LINEAR) {
+                r_lin = epi_row(e, m, PM);
+                if constexpr (CPW == 1) {
+                    const int nf = n0 + 32 * c0;
+                    if (valid && nf < PN) {
+                        if (e.bias) load_row32(e.bias, 0, nf, PN, 0, vb);
+                        if (e.bw) load_vec32(e.bw, nf, PN, vw);
+                    }
+                }
+            }
             if (kb_total > 0) {
                 if (!mbar_wait_bounded(&tfull[acc], (it >> 1) & 1, abort_flag)) break;
                 tc_fence_after();
@@ -537,7 +552,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             float v[32];
 
             if constexpr (EPI == EPI_LINEAR) {
-                const EpiRow r = epi_row(e, m, PM);
+                const EpiRow r = r_lin;
                 float t[32];
 #pragma unroll 1
                 for (int j = 0; j < CPW; ++j) {
@@ -554,9 +569,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] *= r.alpha;
                         if (e.bias) {
-                            load_row32(e.bias, 0, n, PN, 0, t);
+                            if (CPW > 1) load_row32(e.bias, 0, n, PN, 0, vb);
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) v[i] += t[i];
+                            for (int i = 0; i < 32; ++i) v[i] += vb[i];
                         }
                         if (e.r1u) {
                             load_vec32(e.r1v, n, PN, t);
@@ -564,9 +579,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                             for (int i = 0; i < 32; ++i) v[i] += r.beta_r1 * t[i];
                         }
                         if (e.bw) {
-                            load_vec32(e.bw, n, PN, t);
+                            if (CPW > 1) load_vec32(e.bw, n, PN, vw);
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) v[i] += r.beta_bw * t[i];
+                            for (int i = 0; i < 32; ++i) v[i] += r.beta_bw * vw[i];
                         }
                         if (has_a) {
                             unpack32_dyn(xa, 0, t);
@@ -590,8 +605,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         // the 32 rows of this warp, column by column: lane i
                         // ends with the sum of column n + i
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) t[i] = valid ? (e.out_f32 ? v[i] : round_bf16(v[i])) : 0.0f;
-                        const float cs = warp_colsum32(t, lane);
+                        for (int i = 0; i < 32; ++i) v[i] = valid ? (e.out_f32 ? v[i] : round_bf16(v[i])) : 0.0f;
+                        const float cs = warp_colsum32(v, lane);
                         if (row0 < PM && n + lane < PN)
                             e.colsum[static_cast<int64_t>(row0 >> 5) * e.ld_colsum + n + lane] = cs;
                     }

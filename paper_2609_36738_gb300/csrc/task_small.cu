@@ -3,8 +3,8 @@
 // For small batches and output spaces (the classification settings: batch 32
 // x 10 classes, batch 256 x 1000 classes) the task-space part of Algorithm 1
 // is a handful of tiny reductions, and as separate kernels each costs its
-// launch and pipeline fill rather than its work.  One cluster of 8 CTAs does
-// all of it, with the cross-CTA sums in distributed shared memory (added in
+// launch and pipeline fill rather than its work.  One cluster of 16 CTAs (8
+// where the device allows no larger cluster) does all of it, with the cross-CTA sums in distributed shared memory (added in
 // rank order, so the result is deterministic):
 //   phase 1 (rows split over the CTAs): label check and N_t, the row
 //           log-sum-exp and CE from the logits, r_i = softmax(z_i) - onehot(y_i)
@@ -32,7 +32,11 @@ namespace {
 
 namespace cg = cooperative_groups;
 
-constexpr int kSmallCluster = 8;
+// Cluster sizes: 16 CTAs where the device allows a cluster of that size
+// (non-portable), else the portable 8; the per-CTA rows, vocabulary and d
+// slices, and with them the serial rounds of loads of each phase, halve with 16.
+constexpr int kSmallClusterMax = 16;
+constexpr int kSmallClusterMin = 8;
 constexpr int kSmallThreads = 1024;
 // Row-group partials of the chunked column sums: RG * dm <= 1024 * 8 floats
 // (RG = 1024 / (dm / elements per 16-byte word), or 1).
@@ -153,11 +157,10 @@ __device__ __forceinline__ void colsum_tile(const void* X, int64_t dm, int64_t j
 //   qh[vs]      qhat of the CTA's vocabulary slice
 //   lse_s[rp], lab_s[rp] (int)   the CTA's rows
 //   per-warp CE, N_t, bad-label and non-finite counts [4][32], totals
-template <typename T>
+template <typename T, int C>
 __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const TaskSmallArgs a) {
     pdl_enter();
     cg::cluster_group cl = cg::this_cluster();
-    constexpr int C = kSmallCluster;
     constexpr int EPC = 16 / static_cast<int>(sizeof(T));
     const int c = static_cast<int>(cl.block_rank());
     const int64_t V = a.V, dm = a.dm, n = a.n;
@@ -519,21 +522,20 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
     cl.sync();   // no CTA leaves while another still reads its shared memory
 }
 
-size_t task_small_smem(int64_t n, int64_t V, int64_t dm) {
-    const int64_t rp = (n + kSmallCluster - 1) / kSmallCluster;
-    const int64_t vs = (V + kSmallCluster - 1) / kSmallCluster;
+size_t task_small_smem(int64_t n, int64_t V, int64_t dm, int C) {
+    const int64_t rp = (n + C - 1) / C;
+    const int64_t vs = (V + C - 1) / C;
     return static_cast<size_t>(4 * (V + 2 * dm + kSmallPart + vs + 2 * rp + 4 * 32 + 2 + 3) + 64);
 }
 
-template <typename T>
-cudaLaunchConfig_t small_cfg(cudaLaunchAttribute (&at)[2], size_t smem, cudaStream_t s) {
+cudaLaunchConfig_t small_cfg(cudaLaunchAttribute (&at)[2], int C, size_t smem, cudaStream_t s) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(kSmallCluster);
+    cfg.gridDim = dim3(C);
     cfg.blockDim = dim3(kSmallThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = kSmallCluster;
+    at[0].val.clusterDim.x = C;
     at[0].val.clusterDim.y = 1;
     at[0].val.clusterDim.z = 1;
     at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -543,33 +545,46 @@ cudaLaunchConfig_t small_cfg(cudaLaunchAttribute (&at)[2], size_t smem, cudaStre
     return cfg;
 }
 
-// Per device: the kernel's shared-memory limit is raised once, and the path
-// is used only if a cluster of the largest size fits on the device.
+// Whether a cluster of C CTAs of the kernel at its largest shared-memory
+// size fits on the current device (the attributes are per-device settings).
+template <typename T, int C>
+bool cluster_fits() {
+    const size_t smem = task_small_smem(kTaskSmallMaxRows, kTaskSmallMaxV, kTaskSmallMaxD, C);
+    bool ok = cudaFuncSetAttribute(task_small_kernel<T, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   static_cast<int>(smem)) == cudaSuccess;
+    if (ok && C > 8)
+        ok = cudaFuncSetAttribute(task_small_kernel<T, C>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) ==
+             cudaSuccess;
+    if (ok) {
+        cudaLaunchAttribute at[2];
+        cudaLaunchConfig_t cfg = small_cfg(at, C, smem, nullptr);
+        int nc = 0;
+        ok = cudaOccupancyMaxActiveClusters(&nc, task_small_kernel<T, C>, &cfg) == cudaSuccess && nc >= 1;
+    }
+    cudaGetLastError();
+    return ok;
+}
+
+// Per device, found once: the largest cluster size the path can run with
+// (0: the path is not usable).
 template <typename T>
-bool small_ready() {
+int small_cluster() {
     constexpr int kMaxDev = 64;
-    static std::atomic<int> state[kMaxDev];   // 0 unknown, 1 usable, 2 not
+    static std::atomic<int> state[kMaxDev];   // 0 unknown, -1 not usable, else the cluster size
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) {
         cudaGetLastError();
-        return false;
+        return 0;
     }
     int st = state[dev].load(std::memory_order_relaxed);
     if (st == 0) {
-        const size_t smem = task_small_smem(kTaskSmallMaxRows, kTaskSmallMaxV, kTaskSmallMaxD);
-        bool ok = cudaFuncSetAttribute(task_small_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem)) == cudaSuccess;
-        if (ok) {
-            cudaLaunchAttribute at[2];
-            cudaLaunchConfig_t cfg = small_cfg<T>(at, smem, nullptr);
-            int nc = 0;
-            ok = cudaOccupancyMaxActiveClusters(&nc, task_small_kernel<T>, &cfg) == cudaSuccess && nc >= 1;
-        }
-        cudaGetLastError();
-        st = ok ? 1 : 2;
+        // both sizes are set up: a launch may take the smaller one
+        const bool fits_min = cluster_fits<T, kSmallClusterMin>();
+        const bool fits_max = fits_min && cluster_fits<T, kSmallClusterMax>();
+        st = fits_max ? kSmallClusterMax : fits_min ? kSmallClusterMin : -1;
         state[dev].store(st, std::memory_order_relaxed);
     }
-    return st == 1;
+    return st > 0 ? st : 0;
 }
 
 }  // namespace
@@ -577,7 +592,7 @@ bool small_ready() {
 bool task_small_usable(int64_t n, int64_t V, int64_t dm, int z_f32) {
     if (n < 1 || n > kTaskSmallMaxRows || V > kTaskSmallMaxV || dm > kTaskSmallMaxD || n * V > kTaskSmallMaxElems)
         return false;
-    return z_f32 ? small_ready<float>() : small_ready<__nv_bfloat16>();
+    return (z_f32 ? small_cluster<float>() : small_cluster<__nv_bfloat16>()) > 0;
 }
 
 int launch_task_small(const void* Z, int z_f32, int64_t ldz, const int32_t* labels, int64_t n, int64_t V,
@@ -609,16 +624,20 @@ int launch_task_small(const void* Z, int z_f32, int64_t ldz, const int32_t* labe
     a.hb_b = hb_b;
     a.st = st;
     a.sc = sc;
-    const size_t smem = task_small_smem(n, V, dm);
+    // the larger cluster only where its CTAs get work: tiny passes (a few
+    // dozen rows and classes) keep 8, whose cluster barriers cost less
+    const int cmax = z_f32 ? small_cluster<float>() : small_cluster<__nv_bfloat16>();
+    const int C = (n > 64 || V * dm > 65536) ? cmax : kSmallClusterMin;
+    const size_t smem = task_small_smem(n, V, dm, C);
     cudaLaunchAttribute at[2];
+    const cudaLaunchConfig_t cfg = small_cfg(at, C, smem, s);
     cudaError_t e;
-    if (z_f32) {
-        cudaLaunchConfig_t cfg = small_cfg<float>(at, smem, s);
-        e = cudaLaunchKernelEx(&cfg, task_small_kernel<float>, a);
-    } else {
-        cudaLaunchConfig_t cfg = small_cfg<__nv_bfloat16>(at, smem, s);
-        e = cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16>, a);
-    }
+    if (z_f32)
+        e = C == kSmallClusterMax ? cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMax>, a)
+                                  : cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMin>, a);
+    else
+        e = C == kSmallClusterMax ? cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMax>, a)
+                                  : cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMin>, a);
     if (e != cudaSuccess) return BOM_ECUDA;
     count_launch();
     return BOM_OK;
