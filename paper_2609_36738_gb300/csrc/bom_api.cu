@@ -368,6 +368,7 @@ int run_gemm_group(bom_handle* h, GemmDesc* gs, int n, cudaStream_t s) {
     }
     return traced(h, s, gemm_name(gs[0], h->bf16), flops, bytes, [&] {
         if (h->bf16) return launch_gemm_tc_group(gs, n, s);
+        if (n <= 4) return launch_gemm_simt_group(gs, n, s);
         for (int i = 0; i < n; ++i) {
             const int rc = launch_gemm_simt(gs[i], s);
             if (rc != BOM_OK) return rc;
@@ -823,7 +824,7 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
         // dx[0] and dx[1] until the pass ends, so their weight gradients and
         // the head's can run as one grouped launch after the last input
         // cotangent (every weight is still read before its fused update).
-        bool defer_lin = h->bf16 && kfull == 1 && !h->lw.empty() && h->lw.size() <= 2;
+        bool defer_lin = kfull == 1 && !h->lw.empty() && h->lw.size() <= 2;
         for (const LayerWs& L : h->lw)
             defer_lin = defer_lin && (L.kind == BOM_LAYER_LINEAR || L.kind == BOM_LAYER_LINEAR_GELU);
         const bool defer_head =

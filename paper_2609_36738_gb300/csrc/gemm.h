@@ -44,6 +44,8 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream);
 // kind and K and M > 128 (each GEMM launched alone otherwise).
 int launch_gemm_tc_group(const GemmDesc* g, int n, cudaStream_t stream);
 int launch_gemm_simt(const GemmDesc& g, cudaStream_t stream);
+// One launch over n <= 4 GEMMs on the SIMT engine.
+int launch_gemm_simt_group(const GemmDesc* g, int n, cudaStream_t stream);
 
 // Number of column tiles of EPI_LOGITS statistics produced per row.
 int64_t tc_logit_tiles(int64_t N);

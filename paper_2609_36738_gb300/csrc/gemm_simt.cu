@@ -23,9 +23,18 @@ struct Params {
     EpiParams epi;
 };
 
-__global__ void __launch_bounds__(256) gemm_simt_kernel(const Params p) {
+// Up to kMaxGroup GEMMs in one launch: blockIdx.z picks the GEMM, whose
+// tiles are the first of the grid's x and y.
+constexpr int kMaxGroup = 4;
+struct Group {
+    Params p[kMaxGroup];
+};
+
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const __grid_constant__ Group grp) {
     pdl_enter();
+    const Params& p = grp.p[blockIdx.z];
     if (p.epi.sc != nullptr && p.epi.sc->status != 0) return;
+    if (static_cast<int>(blockIdx.x) * TN >= p.N || static_cast<int>(blockIdx.y) * TM >= p.M) return;
     __shared__ float As[TK][TM + 1];
     __shared__ float Bs[TK][TN + 1];
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -95,11 +104,12 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const Params p) {
 
 }  // namespace simt
 
-int launch_gemm_simt(const GemmDesc& g, cudaStream_t stream) {
-    if (g.M <= 0 || g.N <= 0) return BOM_OK;
+namespace {
+
+int simt_params(const GemmDesc& g, simt::Params& p) {
     if (g.dual_b || (g.epi_kind != EPI_LINEAR && g.epi_kind != EPI_LOGITS)) return BOM_ENOTSUP;
     if (g.M > INT32_MAX / 2 || g.N > INT32_MAX / 2) return BOM_ENOTSUP;
-    simt::Params p{};
+    p = simt::Params{};
     p.nseg = g.nseg;
     for (int s = 0; s < g.nseg; ++s) {
         p.A[s] = static_cast<const float*>(g.A[s].ptr);
@@ -114,10 +124,35 @@ int launch_gemm_simt(const GemmDesc& g, cudaStream_t stream) {
     p.N = static_cast<int>(g.N);
     p.epi_kind = g.epi_kind;
     p.epi = g.epi;
-    dim3 grid(static_cast<unsigned>((g.N + simt::TN - 1) / simt::TN), static_cast<unsigned>((g.M + simt::TM - 1) / simt::TM));
-    if (grid.y > 65535) return BOM_ENOTSUP;
-    launch_k(simt::gemm_simt_kernel, dim3(grid), dim3(256), 0, stream, p); count_launch();
+    if ((g.M + simt::TM - 1) / simt::TM > 65535) return BOM_ENOTSUP;
+    return BOM_OK;
+}
+
+}  // namespace
+
+// One launch over n <= 4 GEMMs (the grid covers the largest; each GEMM's
+// blocks beyond its own tiles return at once).
+int launch_gemm_simt_group(const GemmDesc* gs, int n, cudaStream_t stream) {
+    if (n < 1 || n > simt::kMaxGroup) return BOM_EINVAL;
+    simt::Group grp{};
+    int64_t gx = 0, gy = 0;
+    int live = 0;
+    for (int i = 0; i < n; ++i) {
+        if (gs[i].M <= 0 || gs[i].N <= 0) continue;
+        const int rc = simt_params(gs[i], grp.p[live]);
+        if (rc != BOM_OK) return rc;
+        const int64_t x = (gs[i].N + simt::TN - 1) / simt::TN, y = (gs[i].M + simt::TM - 1) / simt::TM;
+        gx = x > gx ? x : gx;
+        gy = y > gy ? y : gy;
+        ++live;
+    }
+    if (live == 0) return BOM_OK;
+    launch_k(simt::gemm_simt_kernel, dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy), live), dim3(256), 0,
+             stream, grp);
+    count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }
+
+int launch_gemm_simt(const GemmDesc& g, cudaStream_t stream) { return launch_gemm_simt_group(&g, 1, stream); }
 
 }  // namespace bom

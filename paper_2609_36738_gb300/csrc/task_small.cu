@@ -4,7 +4,8 @@
 // x 10 classes, batch 256 x 1000 classes) the task-space part of Algorithm 1
 // is a handful of tiny reductions, and as separate kernels each costs its
 // launch and pipeline fill rather than its work.  One cluster of 16 CTAs (8
-// where the device allows no larger cluster) does all of it, with the cross-CTA sums in distributed shared memory (added in
+// where the device allows no larger cluster or the pass is a few dozen rows,
+// a single CTA for the tiniest) does all of it, with the cross-CTA sums in distributed shared memory (added in
 // rank order, so the result is deterministic):
 //   phase 1 (rows split over the CTAs): label check and N_t, the row
 //           log-sum-exp and CE from the logits, r_i = softmax(z_i) - onehot(y_i)
@@ -37,6 +38,10 @@ namespace cg = cooperative_groups;
 // slices, and with them the serial rounds of loads of each phase, halve with 16.
 constexpr int kSmallClusterMax = 16;
 constexpr int kSmallClusterMin = 8;
+// A pass of a few hundred logits and a few thousand head weights runs in one
+// CTA (a cluster of one): its phases are a few loads deep, and the cluster
+// barriers and distributed-memory sums would cost more than they split.
+constexpr int kSmallClusterOne = 1;
 constexpr int kSmallThreads = 1024;
 // Row-group partials of the chunked column sums: RG * dm <= 1024 * 8 floats
 // (RG = 1024 / (dm / elements per 16-byte word), or 1).
@@ -578,8 +583,8 @@ int small_cluster() {
     }
     int st = state[dev].load(std::memory_order_relaxed);
     if (st == 0) {
-        // both sizes are set up: a launch may take the smaller one
-        const bool fits_min = cluster_fits<T, kSmallClusterMin>();
+        // every size is set up: a launch may take a smaller one
+        const bool fits_min = cluster_fits<T, kSmallClusterMin>() && cluster_fits<T, kSmallClusterOne>();
         const bool fits_max = fits_min && cluster_fits<T, kSmallClusterMax>();
         st = fits_max ? kSmallClusterMax : fits_min ? kSmallClusterMin : -1;
         state[dev].store(st, std::memory_order_relaxed);
@@ -624,20 +629,23 @@ int launch_task_small(const void* Z, int z_f32, int64_t ldz, const int32_t* labe
     a.hb_b = hb_b;
     a.st = st;
     a.sc = sc;
-    // the larger cluster only where its CTAs get work: tiny passes (a few
-    // dozen rows and classes) keep 8, whose cluster barriers cost less
+    // the larger cluster only where its CTAs get work: passes of a few dozen
+    // rows keep 8, whose cluster barriers cost less, and tiny ones run in one CTA
     const int cmax = z_f32 ? small_cluster<float>() : small_cluster<__nv_bfloat16>();
-    const int C = (n > 64 || V * dm > 65536) ? cmax : kSmallClusterMin;
+    const bool tiny = n * V <= 4096 && V * dm <= 32768 && n * dm <= 32768;
+    const int C = tiny ? kSmallClusterOne : (n > 64 || V * dm > 65536) ? cmax : kSmallClusterMin;
     const size_t smem = task_small_smem(n, V, dm, C);
     cudaLaunchAttribute at[2];
     const cudaLaunchConfig_t cfg = small_cfg(at, C, smem, s);
     cudaError_t e;
     if (z_f32)
-        e = C == kSmallClusterMax ? cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMax>, a)
-                                  : cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMin>, a);
+        e = C == kSmallClusterMax   ? cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMax>, a)
+            : C == kSmallClusterMin ? cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMin>, a)
+                                    : cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterOne>, a);
     else
-        e = C == kSmallClusterMax ? cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMax>, a)
-                                  : cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMin>, a);
+        e = C == kSmallClusterMax   ? cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMax>, a)
+            : C == kSmallClusterMin ? cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMin>, a)
+                                    : cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterOne>, a);
     if (e != cudaSuccess) return BOM_ECUDA;
     count_launch();
     return BOM_OK;
