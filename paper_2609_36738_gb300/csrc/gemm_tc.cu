@@ -239,14 +239,19 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
 // (whole 32-byte sectors); staging them through shared memory cost pipeline
 // stages and measured slower.  The fused update stages its accumulator chunk
 // (a per-warp block) to walk theta and v by columns.
-// SwiGLU backward: the epilogue's per-row operands (the saved G and U) arrive
-// by TMA.  Each epilogue warp owns two slots of a 32-row x 32-column block of
-// G and of U (2 KB each, 64-byte swizzle: chunk k of row r at
-// r * 64 + 16 * (k ^ ((r >> 1) & 3)), so the row-per-lane reads are
-// conflict-free); lane 0 loads block j + 2 into the slot block j has just
-// freed.
+// SwiGLU backward: the epilogue's per-row operands (the saved G and U,
+// interleaved per 32 columns in one 128-byte line of a row) arrive by TMA.
+// Each epilogue warp owns kEpiSlots slots of a 32-row block of [G 32 | U 32]
+// (4 KB, 128-byte swizzle: 16-byte chunk k of row r at r * 128 + 16 * (k ^ (r & 7)),
+// so the row-per-lane reads are conflict-free); lane 0 loads block
+// j + kEpiSlots into the slot block j has just freed.
 constexpr int kEpiLdBlock = 32 * 64;
-constexpr int kEpiLdWarpBytes = 2 * 2 * kEpiLdBlock;
+// One slot per warp (the next block loads while the current one is
+// processed): the 32 KB this frees is a sixth pipeline stage, which the
+// mainloop needs more than the epilogue needs a second block in flight
+// (same-box A/B: 0.78 -> 0.74-0.75 ms per step for the two launches).
+constexpr int kEpiSlots = 1;   // G|U blocks in flight per epilogue warp
+constexpr int kEpiLdWarpBytes = kEpiSlots * 2 * kEpiLdBlock;
 
 template <int CG, int EPI, int BNT>
 struct Cfg {
@@ -521,9 +526,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
             uint8_t* stg = stg_all + (warp - 2) * (EPI == EPI_UPDATE ? kUpdStgBytes : 0);
             if (EPI == EPI_SWIGLU_BWD) {
-                // the first two blocks of this warp's part of the tile
+                // the first blocks of this warp's part of the tile
                 if (lane == 0)
-                    for (int j = 0; j < 2 && j < CPW; ++j)
+                    for (int j = 0; j < kEpiSlots && j < CPW; ++j)
                         if (n0 + 32 * (c0 + j) < PN) eissue(j, n0 + 32 * (c0 + j), row0);
             } else {
                 if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, PN, xa, 0);
@@ -752,7 +757,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     const int c = c0 + j;
                     const int n = n0 + c * 32;
                     if (n >= PN) break;
-                    const int slot = j & 1;
+                    const int slot = j % kEpiSlots;
                     if (!mbar_wait_bounded(&ebw[slot], (eph >> slot) & 1u, abort_flag)) {
                         ok = false;
                         break;
@@ -780,7 +785,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                     }
                     fence_proxy_async_shared();   // every lane's reads of the slot before its refill
                     __syncwarp();
-                    if (lane == 0 && j + 2 < CPW && n + 64 < PN) eissue(slot, n + 64, row0);
+                    if (lane == 0 && j + kEpiSlots < CPW && n + 32 * kEpiSlots < PN)
+                        eissue(slot, n + 32 * kEpiSlots, row0);
                     tmem_load32(tbase + c * 32, v);
                     if (valid) {
                         float du[32];
@@ -817,7 +823,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         // SwiGLU backward operand loads still in flight (an aborted tile) land
         // before the CTA may exit
         if (EPI == EPI_SWIGLU_BWD && lane == 0)
-            for (int sl = 0; sl < 2; ++sl)
+            for (int sl = 0; sl < kEpiSlots; ++sl)
                 if (epend & (1u << sl)) mbar_wait_bounded(&ebw[sl], (eph >> sl) & 1u, nullptr);
     }
 
