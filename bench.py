@@ -388,18 +388,52 @@ def main():
                    "gbs": v[1] / (v[2] / 1e3) / 1e9} for k, v in sorted(per_kernel.items(), key=lambda kv: -kv[1][2])}
 
     # ---------------------------------------------------------------- end to end through host buffers
+    # Every step copies its inputs from pinned host memory and reads its
+    # statistics (loss, N_t, status) back into pinned host memory.  The copy
+    # of step i+1's inputs runs on a second stream into the other of two
+    # device buffers while step i computes (a step waits for its own copy, a
+    # copy for the step that last used its buffer), and step i's statistics
+    # are read and checked on the host while step i+1 runs; the last step's
+    # before the clock stops.
     e2e_steps = max(3, a.steps // 2)
     h2d = x_host.numel() * x_host.element_size() + y_host.numel() * y_host.element_size()
+    copy_stream = torch.cuda.Stream(device=dev)
+    xb = [torch.empty_like(x_host, device=dev) for _ in range(2)]
+    yb = [torch.empty_like(y_host, device=dev) for _ in range(2)]
+    copied = [torch.cuda.Event() for _ in range(2)]
+    freed = [torch.cuda.Event() for _ in range(2)]
+    for e in freed:
+        e.record(stream)
+    sbuf = [torch.empty(B.bom_stats_transfer_bytes(), dtype=torch.uint8).pin_memory() for _ in range(2)]
+    sdone = [torch.cuda.Event() for _ in range(2)]
+
+    def issue_copy(j):
+        with torch.cuda.stream(copy_stream):
+            copy_stream.wait_event(freed[j % 2])
+            xb[j % 2].copy_(x_host, non_blocking=True)
+            yb[j % 2].copy_(y_host, non_blocking=True)
+            copied[j % 2].record(copy_stream)
+
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize()
     t0 = time.perf_counter()
+    issue_copy(0)
     for i in range(e2e_steps):
         t += 1
-        xx = x_host.to(dev, non_blocking=True)
-        yy = y_host.to(dev, non_blocking=True)
-        step(t, xx.view(torch.bfloat16) if bf16 else xx, yy)
-        model.stats(stream)        # device -> host read of the step's loss / status (syncs)
+        if i + 1 < e2e_steps:
+            issue_copy(i + 1)
+        stream.wait_event(copied[i % 2])
+        xx = xb[i % 2]
+        step(t, xx.view(torch.bfloat16) if bf16 else xx, yb[i % 2])
+        freed[i % 2].record(stream)
+        B.bom_get_stats_async(model.h, sbuf[i % 2], stream)   # device -> host read of the step's statistics
+        sdone[i % 2].record(stream)
+        if i > 0:
+            sdone[(i - 1) % 2].synchronize()
+            B.bom_stats_decode(sbuf[(i - 1) % 2])   # raises if that step latched an error
+    sdone[(e2e_steps - 1) % 2].synchronize()
+    B.bom_stats_decode(sbuf[(e2e_steps - 1) % 2])
     e2e_s = _max_over_ranks(dist, time.perf_counter() - t0, dev)
     e2e = {"value": world * N * e2e_steps / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
            "d2h_bytes_per_step": B.bom_stats_transfer_bytes()}

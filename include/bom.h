@@ -322,6 +322,19 @@ bom_status bom_step_outputs(bom_handle* h, const float** qhat, const float** s, 
  * the latched device status (BOM_OK when the step succeeded). */
 bom_status bom_get_stats(bom_handle* h, bom_stats* out, void* stream);
 
+/* The same statistics without a synchronisation: enqueues on `stream`, after
+ * the work already there, a copy of bom_stats_transfer_bytes() bytes of the
+ * device statistics block into host memory `dst` (caller-owned; page-locked
+ * for the copy to be asynchronous), and returns.  Once the stream has passed
+ * that point (an event recorded after the call, say), bom_stats_decode(dst,
+ * out) fills `out` and returns the latched status, as bom_get_stats does.
+ * A later step on the handle overwrites the device block, not `dst`: a
+ * caller that keeps one step in flight reads step t's statistics while step
+ * t + 1 runs (the loss read-back of a training loop).  BOM_EINVAL for NULL
+ * h or dst, BOM_ECUDA when the copy cannot be enqueued. */
+bom_status bom_get_stats_async(bom_handle* h, void* dst, void* stream);
+bom_status bom_stats_decode(const void* src, bom_stats* out);
+
 /* BOM-AdamW update over a flat range of n elements (Section 3.4).
  *   theta       [n] fp32 master parameters, updated in place.
  *   g           [n] in g_dtype (BOM_F32 or BOM_BF16): u itself when hvec is

@@ -29,7 +29,8 @@ BOM_OUT_U, BOM_OUT_G_AND_H = 0, 1
 # Every symbol include/bom.h declares.
 EXPORTED = ("bom_param_count", "bom_param_shape", "bom_init", "bom_workspace_bytes", "bom_step",
             "bom_step_shard_begin", "bom_step_shard_end",
-            "bom_set_input_grad", "bom_step_outputs", "bom_get_stats", "bom_update", "bom_gemm_bf16", "bom_trace", "bom_trace_read",
+            "bom_set_input_grad", "bom_step_outputs", "bom_get_stats", "bom_get_stats_async", "bom_stats_decode",
+            "bom_update", "bom_gemm_bf16", "bom_trace", "bom_trace_read",
             "bom_launch_count", "bom_colsum_noalloc", "bom_set_own_step_output", "bom_own_step_moment",
             "bom_stats_transfer_bytes", "bom_update_blockshared", "bom_sqnorm", "bom_update_clipped",
             "bom_set_fused_update", "bom_set_step_scalars", "bom_graph_capture", "bom_graph_launch",
@@ -94,6 +95,10 @@ def lib() -> C.CDLL:
     L.bom_step_outputs.restype = i32
     L.bom_get_stats.argtypes = [vp, C.POINTER(bom_stats), vp]
     L.bom_get_stats.restype = i32
+    L.bom_get_stats_async.argtypes = [vp, vp, vp]
+    L.bom_get_stats_async.restype = i32
+    L.bom_stats_decode.argtypes = [vp, C.POINTER(bom_stats)]
+    L.bom_stats_decode.restype = i32
     L.bom_update.argtypes = [vp, vp, i32, vp, vp, vp, i64, f32, f32, f32, f32, f32, i64, vp]
     L.bom_update.restype = i32
     L.bom_gemm_bf16.argtypes = [vp, i64, i32, vp, i64, i32, vp, i64, i64, i64, i64, f32, vp]
@@ -279,6 +284,22 @@ def bom_get_stats(h, stream=None, check: bool = True) -> dict:
     code = lib().bom_get_stats(h, C.byref(st), _stream(stream))
     if check:
         _check(code, "bom_get_stats")
+    return dict(loss=st.loss, n_t=st.n_t, status=st.status, s_norm=st.s_norm, r_norm_mean=st.r_norm_mean,
+                cancel=st.cancel, code=code)
+
+
+def bom_get_stats_async(h, dst, stream=None) -> None:
+    """Enqueue the copy of the last step's statistics block into host memory
+    ``dst`` (a pinned uint8 tensor of bom_stats_transfer_bytes() bytes)."""
+    _check(lib().bom_get_stats_async(h, _ptr(dst), _stream(stream)), "bom_get_stats_async")
+
+
+def bom_stats_decode(src, check: bool = True) -> dict:
+    """The statistics held in ``src`` (filled by bom_get_stats_async)."""
+    st = bom_stats()
+    code = lib().bom_stats_decode(_ptr(src), C.byref(st))
+    if check:
+        _check(code, "bom_stats_decode")
     return dict(loss=st.loss, n_t=st.n_t, status=st.status, s_norm=st.s_norm, r_norm_mean=st.r_norm_mean,
                 cancel=st.cancel, code=code)
 

@@ -1208,6 +1208,27 @@ bom_status bom_step_outputs(bom_handle* h, const float** qhat, const float** s, 
     return BOM_OK;
 }
 
+bom_status bom_stats_decode(const void* src, bom_stats* out) {
+    if (!src || !out) return BOM_EINVAL;
+    DevScalars sc;
+    memcpy(&sc, src, kStatsBytes);
+    out->loss = sc.loss;
+    out->n_t = sc.n_t;
+    out->status = sc.status;
+    out->s_norm = sc.s_norm;
+    out->r_norm_mean = sc.r_norm_mean;
+    out->cancel = sc.r_norm_mean > 0.0f ? sc.s_norm / sc.r_norm_mean : 0.0f;
+    return static_cast<bom_status>(sc.status);
+}
+
+bom_status bom_get_stats_async(bom_handle* h, void* dst, void* stream) {
+    if (!h || !dst) return BOM_EINVAL;
+    return cudaMemcpyAsync(dst, h->sc, kStatsBytes, cudaMemcpyDeviceToHost, static_cast<cudaStream_t>(stream)) ==
+                   cudaSuccess
+               ? BOM_OK
+               : BOM_ECUDA;
+}
+
 bom_status bom_get_stats(bom_handle* h, bom_stats* out, void* stream) {
     if (!h || !out) return BOM_EINVAL;
     if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return BOM_ECUDA;
