@@ -1019,10 +1019,11 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
             return launch_update_multi(np, th.data(), vv.data(), uu.data(), cp.data(), cf32, h->unum.data(),
                                        h->upd_wd.data(), usrc.empty() ? nullptr : usrc.data(),
                                        urows.empty() ? nullptr : urows.data(), usf32.empty() ? nullptr : usf32.data(),
-                                       h->upd_beta2, h->upd_eps, h->sc, s);
+                                       h->upd_beta2, h->upd_eps, h->sc, h->t_dev, s);
         }));
     }
-    if (h->t_dev) launch_advance_step(h->t_dev, h->sc, s);
+    // the update of a small step advances the device step counter itself
+    if (h->t_dev && !upd_sep) launch_advance_step(h->t_dev, h->sc, s);
 #undef BOM_TRY
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }

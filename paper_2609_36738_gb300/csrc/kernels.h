@@ -157,11 +157,13 @@ int launch_update(float* theta, const void* g, int g_bf16, const float* h, float
 // copy_f32); lr and 1/(1 - beta2^t) from the step scalars in sc; nothing when
 // sc's status is set.  A tensor k with src[k] given is a bias whose u is the
 // column sum of src[k] [rows[k], n[k]] (rows in order; fp32 when src_f32[k]
-// is 1, else the compute dtype; src_f32 null: the compute dtype).
+// is 1, else the compute dtype; src_f32 null: the compute dtype).  t_adv
+// (or null): a device step counter advanced by one when sc's status is clear.
 constexpr int kMultiUpdMax = 24;
 int launch_update_multi(int ntensor, float* const* theta, float* const* v, const float* const* u, void* const* copy,
                         int copy_f32, const int64_t* n, const float* wd, const void* const* src, const int64_t* rows,
-                        const int* src_f32, float beta2, float eps, const DevScalars* sc, cudaStream_t s);
+                        const int* src_f32, float beta2, float eps, const DevScalars* sc, int64_t* t_adv,
+                        cudaStream_t s);
 
 // *sq += sum u^2 over n elements (u = g, or (1-lambda) g + lambda h), in a fixed
 // order; `part` holds kOwnStepMaxBlocks doubles.

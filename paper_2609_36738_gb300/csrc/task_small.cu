@@ -4,8 +4,8 @@
 // x 10 classes, batch 256 x 1000 classes) the task-space part of Algorithm 1
 // is a handful of tiny reductions, and as separate kernels each costs its
 // launch and pipeline fill rather than its work.  One cluster of 16 CTAs (8
-// where the device allows no larger cluster or the pass is a few dozen rows,
-// a single CTA for the tiniest) does all of it, with the cross-CTA sums in distributed shared memory (added in
+// where the device allows no larger cluster or the pass is a few dozen rows)
+// does all of it, with the cross-CTA sums in distributed shared memory (added in
 // rank order, so the result is deterministic):
 //   phase 1 (rows split over the CTAs): label check and N_t, the row
 //           log-sum-exp and CE from the logits, r_i = softmax(z_i) - onehot(y_i)
@@ -38,10 +38,11 @@ namespace cg = cooperative_groups;
 // slices, and with them the serial rounds of loads of each phase, halve with 16.
 constexpr int kSmallClusterMax = 16;
 constexpr int kSmallClusterMin = 8;
-// A pass of a few hundred logits and a few thousand head weights runs in one
-// CTA (a cluster of one): its phases are a few loads deep, and the cluster
-// barriers and distributed-memory sums would cost more than they split.
-constexpr int kSmallClusterOne = 1;
+// A pass whose logits, head inputs and head weights fit in one CTA's shared
+// memory together (the tiny classifier: 32 x 10 logits, 32 x 128 inputs) runs
+// from there (task_tiny_kernel): one round of loads, then every phase at
+// shared-memory latency.
+constexpr int64_t kTinyStageFloats = 16384;
 constexpr int kSmallThreads = 1024;
 // Row-group partials of the chunked column sums: RG * dm <= 1024 * 8 floats
 // (RG = 1024 / (dm / elements per 16-byte word), or 1).
@@ -527,6 +528,226 @@ __global__ void __launch_bounds__(kSmallThreads, 1) task_small_kernel(const Task
     cl.sync();   // no CTA leaves while another still reads its shared memory
 }
 
+// The same pass for tiny sizes, in one CTA from shared memory: Z, H and W
+// are read once into shared memory (fp32), then the phases of the cluster
+// kernel run on those copies with the same outputs and the same error
+// precedence; R still goes to Z in global memory for the backward GEMMs.
+// Shared memory (floats): zs[n V], hs[n dm], ws[V dm], lse_s[n], lab_s[n]
+// (int), colp[V], qh[V], cs[dm].
+template <typename T>
+__global__ void __launch_bounds__(kSmallThreads, 1) task_tiny_kernel(const TaskSmallArgs a) {
+    pdl_enter();
+    const int64_t V = a.V, dm = a.dm, n = a.n;
+    extern __shared__ float sm[];
+    float* zs = sm;
+    float* hs = zs + n * V;
+    float* ws = hs + n * dm;
+    float* lse_s = ws + V * dm;
+    int* lab_s = reinterpret_cast<int*>(lse_s + n);
+    float* colp = reinterpret_cast<float*>(lab_s + n);
+    float* qh = colp + V;
+    float* cs = qh + V;
+    __shared__ float wf[32];
+    __shared__ int wi[3][32];
+    __shared__ int s_code, s_nt;
+    __shared__ float s_inv_nt, s_bc1, s_bc2, s_ce, s_ss;
+    __shared__ int64_t s_t;
+    const int tid = threadIdx.x, w = tid >> 5, l = tid & 31;
+
+    // the device step counter and learning rate (thread 0 reads them; the
+    // counter goes to shared memory for the two bias-correction threads)
+    int64_t t_ld = 1;
+    float lr_ld = a.st.lr;
+    if (tid == 0) {
+        if (a.st.t_dev != nullptr) t_ld = __ldcg(a.st.t_dev);
+        if (a.st.lr_dev != nullptr) lr_ld = __ldcg(a.st.lr_dev);
+        s_t = t_ld;
+    }
+    const bool live = a.sc->status == 0;
+    // stage Z, H and W: one index space, eight loads in flight per thread
+    {
+        const int64_t e0 = n * V, e1 = e0 + n * dm, e2 = e1 + V * dm;
+        for (int64_t base = 0; base < e2; base += 8 * kSmallThreads) {
+            float v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int64_t i = base + u * kSmallThreads + tid;
+                if (i < e0)
+                    v[u] = ld_t<T>(a.Z, (i / V) * a.ldz + i % V);
+                else if (i < e1)
+                    v[u] = ld_t<T>(a.H, i - e0);
+                else if (i < e2)
+                    v[u] = ld_t<T>(a.W, i - e1);
+                else
+                    v[u] = 0.0f;
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int64_t i = base + u * kSmallThreads + tid;
+                if (i < e2) sm[i] = v[u];
+            }
+        }
+    }
+    __syncthreads();
+
+    // rows: one warp per row, log-sum-exp, CE, label check
+    float ce_w = 0.0f;
+    int nt_w = 0, bad_w = 0, nf_w = 0;
+    for (int64_t r = w; r < n; r += kSmallThreads / 32) {
+        const int32_t y = a.labels[r];
+        const bool sup = y != a.ignore;
+        const bool ok_y = sup && y >= 0 && y < V;
+        const float* zr = zs + r * V;
+        float m = -INFINITY;
+        for (int64_t j = l; j < V; j += 32) m = fmaxf(m, zr[j]);
+        m = warp_max_f(m);
+        float sum = 0.0f;
+        for (int64_t j = l; j < V; j += 32) sum += expf(zr[j] - m);
+        sum = warp_sum_f(sum);
+        if (l == 0) {
+            const float L = m + logf(sum);
+            const float zy = ok_y ? zr[y] : 0.0f;
+            lse_s[r] = L;
+            lab_s[r] = ok_y ? y : -1;
+            if (live) a.lse[r] = L;
+            if (sup && !ok_y) ++bad_w;
+            if (ok_y) {
+                ++nt_w;
+                ce_w += L - zy;
+            }
+            if (!isfinite(L) || (ok_y && !isfinite(zy))) ++nf_w;
+        }
+    }
+    if (l == 0) {
+        wf[w] = ce_w;
+        wi[0][w] = nt_w;
+        wi[1][w] = bad_w;
+        wi[2][w] = nf_w;
+    }
+    __syncthreads();
+    // R over Z (0 on rows outside I_t), kept in zs for the column sums
+    for (int64_t i = tid; i < n * V; i += kSmallThreads) {
+        const int64_t r = i / V, j = i % V;
+        const int y = lab_s[r];
+        float pr = 0.0f;
+        if (y >= 0) {
+            pr = expf(zs[i] - lse_s[r]);
+            if (j == y) pr -= 1.0f;
+        }
+        zs[i] = pr;
+        if (live) st_t<T>(const_cast<void*>(a.Z), r * a.ldz + j, pr);
+    }
+    if (tid == 0) {
+        float ce = 0.0f;
+        int nt = 0, bad = 0, nf = 0;
+        for (int k = 0; k < kSmallThreads / 32; ++k) {
+            ce += wf[k];
+            nt += wi[0][k];
+            bad += wi[1][k];
+            nf += wi[2][k];
+        }
+        const bool t_bad = a.st.t_dev != nullptr && t_ld < 1;
+        int code = live ? 0 : -1;
+        if (live) {
+            if (bad > 0)
+                code = BOM_ELABEL;
+            else if (nt == 0)
+                code = BOM_EEMPTY;
+            else if (t_bad)
+                code = BOM_EINVAL;
+            else if (nf > 0)
+                code = BOM_ENONFINITE;
+        }
+        s_code = code;
+        s_nt = nt;
+        s_inv_nt = nt > 0 ? 1.0f / static_cast<float>(nt) : 0.0f;
+        s_ce = ce;
+    }
+    // the two fp64 bias corrections beside it
+    if (tid == 32)
+        s_bc1 = (a.st.t_dev != nullptr && s_t >= 1) ? inv_bias_correction(a.st.beta1, s_t) : a.st.inv_bc1;
+    if (tid == 64)
+        s_bc2 = (a.st.t_dev != nullptr && s_t >= 1) ? inv_bias_correction(a.st.beta2, s_t) : a.st.inv_bc2;
+    __syncthreads();
+    // column sums of R and of 1_{I_t} H, rows in order
+    for (int64_t j = tid; j < V; j += kSmallThreads) {
+        float acc = 0.0f;
+        for (int64_t r = 0; r < n; ++r) acc += zs[r * V + j];
+        colp[j] = acc;
+    }
+    for (int64_t k = tid; k < dm; k += kSmallThreads) {
+        float acc = 0.0f;
+        for (int64_t r = 0; r < n; ++r)
+            if (lab_s[r] >= 0) acc += hs[r * dm + k];
+        cs[k] = acc;
+    }
+    if (tid == 0 && live) {
+        DevScalars* sc = a.sc;
+        const int code = s_code;
+        const float inv = s_inv_nt;
+        if (code > 0) latch_status(sc, code);
+        sc->n_t = s_nt;
+        sc->inv_nt = inv;
+        sc->coef_r[0] = (1.0f - a.lambda) * inv;
+        sc->coef_q[0] = a.lambda * inv;
+        sc->coef_r[1] = inv;
+        sc->coef_q[1] = 0.0f;
+        sc->coef_r[2] = 0.0f;
+        sc->coef_q[2] = inv;
+        sc->coef_r[3] = 0.0f;
+        sc->coef_q[3] = inv;
+        sc->lr = lr_ld;
+        sc->inv_bc1 = s_bc1;
+        sc->inv_bc2 = s_bc2;
+        sc->loss = s_ce * inv;
+        sc->s_norm = 0.0f;
+        sc->r_norm_mean = 0.0f;
+    }
+    __syncthreads();
+    const bool ok = s_code == 0;
+    // s_t, q_t, qhat_t (Section 3.2), the head bias numerator, c
+    float ss = 0.0f;
+    if (ok) {
+        const float inv = s_inv_nt, bc1 = s_bc1;
+        for (int64_t j = tid; j < V; j += kSmallThreads) {
+            const float sv = colp[j] * inv;
+            const float qn = a.beta1 * a.q[j] + (1.0f - a.beta1) * sv;
+            const float qhat = qn * bc1;
+            a.q[j] = qn;
+            a.s_out[j] = sv;
+            a.qhat[j] = qhat;
+            qh[j] = qhat;
+            ss += sv * sv;
+            if (a.hb_out) st_elem(a.hb_out, j, a.hb_f32, a.hb_a * sv + a.hb_b * qhat);
+        }
+        for (int64_t k = tid; k < dm; k += kSmallThreads) a.cvec[k] = cs[k];
+    }
+    ss = warp_sum_f(ss);
+    if (l == 0) wf[w] = ss;
+    __syncthreads();
+    if (tid == 0) {
+        float t = 0.0f;
+        for (int k = 0; k < kSmallThreads / 32; ++k) t += wf[k];
+        s_ss = t;
+    }
+    // w = W^T qhat, vocabulary rows in order
+    if (ok)
+        for (int64_t k = tid; k < dm; k += kSmallThreads) {
+            float acc = 0.0f;
+            for (int64_t j = 0; j < V; ++j) acc = fmaf(qh[j], ws[j * dm + k], acc);
+            a.wvec[k] = acc;
+        }
+    if (ok && tid == 0) a.sc->s_norm = sqrtf(s_ss);
+}
+
+size_t task_tiny_smem(int64_t n, int64_t V, int64_t dm) {
+    return static_cast<size_t>(4 * (n * V + n * dm + V * dm + 2 * n + 2 * V + dm) + 64);
+}
+
+bool tiny_fits(int64_t n, int64_t V, int64_t dm) {
+    return n * V + n * dm + V * dm <= kTinyStageFloats && n <= 1024 && V <= 1024 && dm <= 1024;
+}
+
 size_t task_small_smem(int64_t n, int64_t V, int64_t dm, int C) {
     const int64_t rp = (n + C - 1) / C;
     const int64_t vs = (V + C - 1) / C;
@@ -584,7 +805,12 @@ int small_cluster() {
     int st = state[dev].load(std::memory_order_relaxed);
     if (st == 0) {
         // every size is set up: a launch may take a smaller one
-        const bool fits_min = cluster_fits<T, kSmallClusterMin>() && cluster_fits<T, kSmallClusterOne>();
+        // the tiny pass: at most kTinyStageFloats staged and n, V, d <= 1024
+        const size_t tiny_smem = 4 * (kTinyStageFloats + 5 * 1024) + 64;
+        const bool tiny_ok = cudaFuncSetAttribute(task_tiny_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                  static_cast<int>(tiny_smem)) == cudaSuccess;
+        cudaGetLastError();
+        const bool fits_min = cluster_fits<T, kSmallClusterMin>() && tiny_ok;
         const bool fits_max = fits_min && cluster_fits<T, kSmallClusterMax>();
         st = fits_max ? kSmallClusterMax : fits_min ? kSmallClusterMin : -1;
         state[dev].store(st, std::memory_order_relaxed);
@@ -629,23 +855,28 @@ int launch_task_small(const void* Z, int z_f32, int64_t ldz, const int32_t* labe
     a.hb_b = hb_b;
     a.st = st;
     a.sc = sc;
+    if (tiny_fits(n, V, dm)) {   // one CTA from shared memory
+        const size_t smem = task_tiny_smem(n, V, dm);
+        const cudaError_t e = z_f32 ? launch_k(task_tiny_kernel<float>, dim3(1), dim3(kSmallThreads), smem, s, a)
+                                    : launch_k(task_tiny_kernel<__nv_bfloat16>, dim3(1), dim3(kSmallThreads), smem, s, a);
+        if (e != cudaSuccess) return BOM_ECUDA;
+        count_launch();
+        return BOM_OK;
+    }
     // the larger cluster only where its CTAs get work: passes of a few dozen
-    // rows keep 8, whose cluster barriers cost less, and tiny ones run in one CTA
+    // rows keep 8, whose cluster barriers cost less
     const int cmax = z_f32 ? small_cluster<float>() : small_cluster<__nv_bfloat16>();
-    const bool tiny = n * V <= 4096 && V * dm <= 32768 && n * dm <= 32768;
-    const int C = tiny ? kSmallClusterOne : (n > 64 || V * dm > 65536) ? cmax : kSmallClusterMin;
+    const int C = (n > 64 || V * dm > 65536) ? cmax : kSmallClusterMin;
     const size_t smem = task_small_smem(n, V, dm, C);
     cudaLaunchAttribute at[2];
     const cudaLaunchConfig_t cfg = small_cfg(at, C, smem, s);
     cudaError_t e;
     if (z_f32)
-        e = C == kSmallClusterMax   ? cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMax>, a)
-            : C == kSmallClusterMin ? cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMin>, a)
-                                    : cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterOne>, a);
+        e = C == kSmallClusterMax ? cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMax>, a)
+                                  : cudaLaunchKernelEx(&cfg, task_small_kernel<float, kSmallClusterMin>, a);
     else
-        e = C == kSmallClusterMax   ? cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMax>, a)
-            : C == kSmallClusterMin ? cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMin>, a)
-                                    : cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterOne>, a);
+        e = C == kSmallClusterMax ? cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMax>, a)
+                                  : cudaLaunchKernelEx(&cfg, task_small_kernel<__nv_bfloat16, kSmallClusterMin>, a);
     if (e != cudaSuccess) return BOM_ECUDA;
     count_launch();
     return BOM_OK;

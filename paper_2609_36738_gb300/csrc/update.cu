@@ -873,9 +873,12 @@ struct MultiUpdTable {
 };
 
 __global__ void __launch_bounds__(256) update_multi_kernel(const __grid_constant__ MultiUpdTable tb, UpdCoef c_in,
-                                                           const DevScalars* sc) {
+                                                           const DevScalars* sc, int64_t* t_adv) {
     pdl_enter();
     if (sc != nullptr && sc->status != 0) return;
+    // the step succeeded: advance the device step counter (nothing in this
+    // launch reads it; the next step's kernels start after this one ends)
+    if (t_adv != nullptr && blockIdx.x == 0 && threadIdx.x == 0) *t_adv += 1;
     const int64_t words = tb.word0[tb.ntensor];
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     int k = 0;
@@ -1000,7 +1003,8 @@ __global__ void __launch_bounds__(256) update_multi_kernel(const __grid_constant
 
 int launch_update_multi(int ntensor, float* const* theta, float* const* v, const float* const* u, void* const* copy,
                         int copy_f32, const int64_t* n, const float* wd, const void* const* src, const int64_t* rows,
-                        const int* src_f32, float beta2, float eps, const DevScalars* sc, cudaStream_t s) {
+                        const int* src_f32, float beta2, float eps, const DevScalars* sc, int64_t* t_adv,
+                        cudaStream_t s) {
     if (ntensor < 1 || ntensor > kMultiUpdMax) return BOM_EINVAL;
     MultiUpdTable tb = {};
     tb.ntensor = ntensor;
@@ -1029,7 +1033,7 @@ int launch_update_multi(int ntensor, float* const* theta, float* const* v, const
     const int64_t need = (words + 255) / 256;
     if (grid > need) grid = need;
     if (grid < 1) grid = 1;
-    launch_k(update_multi_kernel, dim3(static_cast<unsigned>(grid)), dim3(256), 0, s, tb, c, sc);
+    launch_k(update_multi_kernel, dim3(static_cast<unsigned>(grid)), dim3(256), 0, s, tb, c, sc, t_adv);
     count_launch();
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }

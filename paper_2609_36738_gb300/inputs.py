@@ -221,6 +221,10 @@ VISION_SMALL = Workload("vision_small", 70, 96,
 VISION_MID = Workload("vision_mid", 300, 96,
                       (Layer(LINEAR_GELU, 96, 200, True), Layer(LINEAR_GELU, 200, 88, True)),
                       130, True, "bf16", "uniform", steps=3)
+# A tiny bf16 classifier (48 rows, 26 classes): its task-space pass runs in
+# one CTA from shared memory, as the fp32 tiny ones do.
+TINY_BF16 = Workload("tiny_bf16", 48, 64, (Layer(LINEAR_GELU, 64, 96, True),), 26, True, "bf16", "uniform",
+                     steps=3, ignore_frac=0.1)
 TINY_RAGGED_F32 = Workload("tiny_ragged_f32", 37, 29, (Layer(LINEAR_GELU, 29, 45, True),
                                                        Layer(LINEAR, 45, 33, True)),
                            7, True, "f32", "uniform", steps=3, ignore_frac=0.1)
@@ -257,7 +261,7 @@ LM_NORM_BF16 = Workload("lm_norm_bf16", 16384, 2048,
 WORKLOADS = {w.name: w for w in (TINY_MLP_F32, VISION_HEAD_BF16, LM_HEAD_BF16, LM_MLP_BF16,
                                   LM_HEAD_SMALL, LM_MLP_SMALL, VISION_SMALL, TINY_RAGGED_F32, LM_HEAD_WIDE,
                                   LM_NORM_SMALL, TINY_NORM_F32, LM_NORM_BF16, LM_MLP_MID, LM_MLP_K1100,
-                                  VISION_MID)}
+                                  VISION_MID, TINY_BF16)}
 
 
 # --------------------------------------------------------------------------

@@ -45,7 +45,7 @@ def _compare_step(wl, gout, oref, tol, check_g_h):
             assert G.rel_l2(G.np64(u), ref) < tol, f"u[{k}] {G.rel_l2(G.np64(u), ref)}"
 
 
-@pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "tiny_norm_f32", "lm_head_small",
+@pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "tiny_norm_f32", "tiny_bf16", "lm_head_small",
                                   "lm_norm_small", "vision_small",
                                   "lm_mlp_small", "lm_mlp_mid"])
 @pytest.mark.parametrize("mode", [B.BOM_OUT_U, B.BOM_OUT_G_AND_H])
@@ -223,7 +223,7 @@ def _guards_intact(buf, n, guard=64, fill=-7.25):
     return bool((buf[:guard] == fill).all()) and bool((buf[guard + n:] == fill).all())
 
 
-@pytest.mark.parametrize("name", ["tiny_ragged_f32", "tiny_norm_f32", "vision_small", "lm_head_small",
+@pytest.mark.parametrize("name", ["tiny_ragged_f32", "tiny_norm_f32", "tiny_bf16", "vision_small", "lm_head_small",
                                   "lm_mlp_small", "lm_head_wide", "lm_norm_small"])
 @pytest.mark.parametrize("mode", [B.BOM_OUT_U, B.BOM_OUT_G_AND_H])
 def test_outputs_stay_inside_their_buffers(name, mode):
