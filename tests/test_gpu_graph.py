@@ -114,8 +114,9 @@ def test_graph_replay_equals_direct_steps(name):
         B.bom_graph_destroy(g)
 
 
-def test_device_counter_errors_leave_state_and_counter_unchanged():
-    wl = I.LM_MLP_SMALL
+@pytest.mark.parametrize("name", ["lm_mlp_small", "tiny_mlp_f32", "vision_small"])
+def test_device_counter_errors_leave_state_and_counter_unchanged(name):
+    wl = I.WORKLOADS[name]
     r = Run(wl, 13, True)
     x, y = I.make_batch(wl, 13, 1)
     r.load(x, y)

@@ -110,8 +110,11 @@ def test_multi_step_trajectory(name, steps):
             assert G.rel_l2(G.np64(master[k]), p64[k]) < tol
 
 
-def test_device_errors_leave_q_unchanged():
-    wl = I.LM_HEAD_SMALL
+# lm_head_small: the cluster task pass; tiny_mlp_f32, tiny_bf16: the one-CTA
+# shared-memory pass
+@pytest.mark.parametrize("name", ["lm_head_small", "tiny_mlp_f32", "tiny_bf16"])
+def test_device_errors_leave_q_unchanged(name):
+    wl = I.WORKLOADS[name]
     params = I.init_params(wl, seed=0)
     x, y = I.make_batch(wl, seed=0, step=1)
     gpu = G.GpuBom(wl, params)
