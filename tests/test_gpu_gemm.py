@@ -1,6 +1,7 @@
 """The tcgen05 GEMM engine (bom_gemm_bf16) against an fp64 matmul of the same
-bf16 operands, for every operand layout, on shapes spanning several 128 x 256
-tiles with ragged tails, K tails and the empty-K case."""
+bf16 operands, for every operand layout, on shapes spanning several tiles
+(narrow 128 x 64 and CTA-pair 256 x 256) with ragged tails, K tails and the
+empty-K case."""
 import numpy as np
 import pytest
 import torch
@@ -38,7 +39,12 @@ def _operand(rng, rows, K, mn_major):
 
 
 @pytest.mark.parametrize("a_mn,b_mn", [(0, 0), (0, 1), (1, 0), (1, 1)])
-@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (300, 520, 200), (1, 7, 8), (257, 1000, 136), (640, 768, 1024)])
+# The first five shapes have few enough 256 x 256 tiles to run on 128 x 64
+# single-CTA tiles when A is K-major; the last two have enough to keep the
+# CTA-pair tiles, with ragged M, N and K (130 rows: a pair whose odd CTA has
+# two valid rows).
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (300, 520, 200), (1, 7, 8), (257, 1000, 136), (640, 768, 1024),
+                                   (1000, 2500, 300), (130, 9000, 96)])
 def test_gemm_layouts(a_mn, b_mn, M, N, K):
     rng = np.random.default_rng(M * 7 + N * 13 + K)
     A, lda, Av = _operand(rng, M, K, a_mn)
