@@ -225,6 +225,13 @@ VISION_MID = Workload("vision_mid", 300, 96,
 # one CTA from shared memory, as the fp32 tiny ones do.
 TINY_BF16 = Workload("tiny_bf16", 48, 64, (Layer(LINEAR_GELU, 64, 96, True),), 26, True, "bf16", "uniform",
                      steps=3, ignore_frac=0.1)
+# A batch of 1200 rows with a 1536-wide GELU layer: its first forward layer
+# and the second layer's input cotangent have enough tiles for CTA-pair
+# 256 x 256 tiles (bias + GELU, and GELU' epilogues on that path), ragged in
+# rows; above 1024 rows the update stays in the weight-gradient epilogues.
+VISION_WIDE = Workload("vision_wide", 1200, 256,
+                       (Layer(LINEAR_GELU, 256, 1536, True), Layer(LINEAR_GELU, 1536, 256, True)),
+                       500, True, "bf16", "uniform", steps=2, ignore_frac=0.05)
 TINY_RAGGED_F32 = Workload("tiny_ragged_f32", 37, 29, (Layer(LINEAR_GELU, 29, 45, True),
                                                        Layer(LINEAR, 45, 33, True)),
                            7, True, "f32", "uniform", steps=3, ignore_frac=0.1)
@@ -261,7 +268,7 @@ LM_NORM_BF16 = Workload("lm_norm_bf16", 16384, 2048,
 WORKLOADS = {w.name: w for w in (TINY_MLP_F32, VISION_HEAD_BF16, LM_HEAD_BF16, LM_MLP_BF16,
                                   LM_HEAD_SMALL, LM_MLP_SMALL, VISION_SMALL, TINY_RAGGED_F32, LM_HEAD_WIDE,
                                   LM_NORM_SMALL, TINY_NORM_F32, LM_NORM_BF16, LM_MLP_MID, LM_MLP_K1100,
-                                  VISION_MID, TINY_BF16)}
+                                  VISION_MID, TINY_BF16, VISION_WIDE)}
 
 
 # --------------------------------------------------------------------------

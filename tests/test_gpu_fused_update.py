@@ -47,7 +47,7 @@ class Fused:
 # vision_mid and vision_head_bf16 (300 and 256 rows) take the bias gradients
 # from the column sums of 32-row blocks formed in the cotangent GEMMs.
 @pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "tiny_norm_f32", "tiny_bf16", "vision_small",
-                                  "vision_mid", "vision_head_bf16", "lm_head_small", "lm_mlp_small",
+                                  "vision_mid", "vision_head_bf16", "vision_wide", "lm_head_small", "lm_mlp_small",
                                   "lm_norm_small", "lm_head_wide", "lm_mlp_mid", "lm_mlp_k1100"])
 def test_fused_update_matches_oracle_on_the_same_inputs(name):
     wl = I.WORKLOADS[name]

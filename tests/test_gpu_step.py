@@ -46,7 +46,7 @@ def _compare_step(wl, gout, oref, tol, check_g_h):
 
 
 @pytest.mark.parametrize("name", ["tiny_mlp_f32", "tiny_ragged_f32", "tiny_norm_f32", "tiny_bf16", "lm_head_small",
-                                  "lm_norm_small", "vision_small",
+                                  "lm_norm_small", "vision_small", "vision_wide",
                                   "lm_mlp_small", "lm_mlp_mid"])
 @pytest.mark.parametrize("mode", [B.BOM_OUT_U, B.BOM_OUT_G_AND_H])
 def test_single_step_parity(name, mode):
