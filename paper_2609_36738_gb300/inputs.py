@@ -225,11 +225,12 @@ VISION_MID = Workload("vision_mid", 300, 96,
 # one CTA from shared memory, as the fp32 tiny ones do.
 TINY_BF16 = Workload("tiny_bf16", 48, 64, (Layer(LINEAR_GELU, 64, 96, True),), 26, True, "bf16", "uniform",
                      steps=3, ignore_frac=0.1)
-# A batch of 1200 rows with a 1536-wide GELU layer: its first forward layer
+# A batch of 1000 rows with a 1536-wide GELU layer: its first forward layer
 # and the second layer's input cotangent have enough tiles for CTA-pair
 # 256 x 256 tiles (bias + GELU, and GELU' epilogues on that path), ragged in
-# rows; above 1024 rows the update stays in the weight-gradient epilogues.
-VISION_WIDE = Workload("vision_wide", 1200, 256,
+# rows; with the update registered, that cotangent GEMM also forms the first
+# layer's bias column sums per 32-row block on the pair tiles.
+VISION_WIDE = Workload("vision_wide", 1000, 256,
                        (Layer(LINEAR_GELU, 256, 1536, True), Layer(LINEAR_GELU, 1536, 256, True)),
                        500, True, "bf16", "uniform", steps=2, ignore_frac=0.05)
 TINY_RAGGED_F32 = Workload("tiny_ragged_f32", 37, 29, (Layer(LINEAR_GELU, 29, 45, True),
