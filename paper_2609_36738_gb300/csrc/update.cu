@@ -890,8 +890,9 @@ __global__ void __launch_bounds__(256) update_multi_kernel(const __grid_constant
         const int64_t w = i - tb.word0[k];
         const int64_t e0 = 4 * w;
         const int64_t len = tb.n[k];
-        if (tb.src[k] != nullptr && tb.src_f32[k] && e0 + 4 <= len && (len & 3) == 0) {
-            // a bias whose u sums fp32 rows (16-byte aligned): the word's four
+        if (tb.src[k] != nullptr && tb.src_f32[k] && e0 + 4 <= len && (len & 3) == 0 &&
+            (reinterpret_cast<uintptr_t>(tb.src[k]) & 15u) == 0) {
+            // a bias whose u sums fp32 rows (16-byte aligned rows): the word's four
             // columns at once, every row load and theta, v in flight together;
             // per column the same order of additions as the loop below
             const float4* sp = static_cast<const float4*>(tb.src[k]) + w;
