@@ -63,8 +63,9 @@ typedef enum {
     BOM_ENOTSUP = 7,   /* shape or alignment this build does not handle               */
     BOM_ENONFINITE = 8, /* a row's log-sum-exp or its label logit is not finite
                            (device-detected before any state is written)             */
-    BOM_ESHARD = 9      /* device: another row shard of a sharded step latched an
-                           error (bom_step_shard_end), so this shard stopped too   */
+    BOM_ESHARD = 9      /* device: another shard of a sharded step latched an error
+                           (bom_step_shard_end, bom_step_vshard_mid), so this
+                           shard stopped too                                        */
 } bom_status;
 
 typedef enum { BOM_F32 = 0, BOM_BF16 = 1 } bom_dtype;
@@ -213,6 +214,75 @@ bom_status bom_step_shard_begin(bom_handle* h, const void* x, const int32_t* lab
 bom_status bom_step_shard_end(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
                               void* const* params, float* q, int64_t t, const double* xch,
                               void* const* grads, void* const* h_out, void* stream);
+
+/* Vocabulary-sharded step: the head's output columns (the vocabulary or the
+ * classes) split over several handles, every shard with the whole batch and
+ * the same backbone.  A row's residual r_ij = exp(z_ij - lse_i) - [j = y_i]
+ * (Algorithm 1; Section 3.2) needs the other shards' columns only through the
+ * row log-sum-exp lse_i, and s_t, q_t and qhat_t are per column, so they shard
+ * with no exchange; the head's input cotangent is a sum over the shards'
+ * columns (a R W + b 1_{I_t} (W^T qhat)^T, Eq. mix-gradient).  A step is three
+ * calls per shard and two exchanges:
+ *
+ *   bom_step_vshard_begin  label check and N_t over the whole vocabulary,
+ *                          forward, this shard's logits, and its part of each
+ *                          row's log-sum-exp:
+ *                            lse_part[i] = log sum_{j in shard} exp(z_ij)
+ *                          (NaN on every row when this shard latched an
+ *                          error);
+ *   the caller             gathers every shard's lse_part into
+ *                          lse_parts[n_shards, n_rows], in one shard order
+ *                          that is the same for every shard (an all-gather);
+ *   bom_step_vshard_mid    the row log-sum-exp from the parts (combined in
+ *                          that order, so every shard holds the same float),
+ *                          R over this shard's columns, s_t, q_t, qhat_t of
+ *                          its columns, the head's weight and bias rows of u
+ *                          (complete: no other shard adds to them), and this
+ *                          shard's part of the head's input cotangent, fp32,
+ *                          in dh_part[n_rows, d] (times GELU' of the last
+ *                          layer when it is a LINEAR_GELU);
+ *   the caller             sums the shards' dh_part elementwise into dh_sum
+ *                          (an all-reduce);
+ *   bom_step_vshard_end    the backbone's backward from dh_sum: u of every
+ *                          backbone tensor, the same on every shard (no
+ *                          gradient exchange), and the cotangent of X when an
+ *                          input-gradient buffer is registered.
+ *
+ * The handle's cfg.d_out is this shard's width V_s; its head W [V_s, d] (and
+ * bias [V_s]) are rows v_first .. v_first + V_s - 1 of the whole head, and q
+ * holds the same V_s entries of the task-space EMA.  Labels are ids of the
+ * whole vocabulary [0, v_total) or ignore_index; a supervised row whose label
+ * lies outside this shard has no one-hot term here, and counts in N_t like
+ * any other.  The three calls take the same x, labels, n_rows and params,
+ * unchanged in between, in this order on one stream, and nothing else may run
+ * on the handle between them; begin takes no q, t or outputs, end no q or t.
+ * grads[] has bom_param_count entries in both mid and end: mid writes the
+ * head's, end the backbone's.  bom_get_stats after mid: n_t of the batch, loss
+ * = this shard's part of the mean CE (the rows whose label it holds; the
+ * shards' parts add up to the loss), s_norm = the norm of this shard's part
+ * of s_t.  An error of one shard's begin (a non-finite logit) stops every
+ * other shard's mid with BOM_ESHARD through the NaN parts; a bad label or an
+ * empty I_t stops every shard (each checks the whole batch).  q changes only
+ * in a mid whose status stays clear; with bom_set_step_scalars, mid reads t
+ * there and end advances it.  BOM_OUT_U only, and not with the fused update
+ * or an own-step output registered (BOM_EINVAL).
+ *   v_total    vocabulary size, 1 <= v_total <= INT32_MAX
+ *   v_first    this shard's first id, 0 <= v_first <= v_total - cfg.d_out
+ *   lse_part   device fp32 [n_rows], 4-byte aligned (BOM_ENOTSUP otherwise)
+ *   lse_parts  device fp32 [n_shards, n_rows], 1 <= n_shards <= 4096
+ *   dh_part, dh_sum  device fp32 [n_rows, d] (d: the head's input width),
+ *              16-byte aligned; needed when the handle has backbone layers or
+ *              an input-gradient buffer (NULL allowed otherwise).
+ * A mid or end without the matching earlier part (other n_rows, another call
+ * in between, an earlier part that failed) returns BOM_EINVAL. */
+bom_status bom_step_vshard_begin(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                                 void* const* params, int64_t v_total, int64_t v_first, float* lse_part,
+                                 void* stream);
+bom_status bom_step_vshard_mid(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                               void* const* params, float* q, int64_t t, const float* lse_parts, int32_t n_shards,
+                               void* const* grads, float* dh_part, void* stream);
+bom_status bom_step_vshard_end(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                               void* const* params, const float* dh_sum, void* const* grads, void* stream);
 
 /* Fused BOM-AdamW update (Section 3.4; Algorithm 1, last two steps) inside
  * bom_step.  Registers, per parameter tensor, its fp32 master weights theta[k]

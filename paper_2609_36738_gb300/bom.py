@@ -29,6 +29,7 @@ BOM_OUT_U, BOM_OUT_G_AND_H = 0, 1
 # Every symbol include/bom.h declares.
 EXPORTED = ("bom_param_count", "bom_param_shape", "bom_init", "bom_workspace_bytes", "bom_step",
             "bom_step_shard_begin", "bom_step_shard_end",
+            "bom_step_vshard_begin", "bom_step_vshard_mid", "bom_step_vshard_end",
             "bom_set_input_grad", "bom_step_outputs", "bom_get_stats", "bom_get_stats_async", "bom_stats_decode",
             "bom_update", "bom_gemm_bf16", "bom_trace", "bom_trace_read",
             "bom_launch_count", "bom_colsum_noalloc", "bom_set_own_step_output", "bom_own_step_moment",
@@ -89,6 +90,12 @@ def lib() -> C.CDLL:
     L.bom_step_shard_begin.restype = i32
     L.bom_step_shard_end.argtypes = [vp, vp, vp, i64, C.POINTER(vp), vp, i64, vp, C.POINTER(vp), C.POINTER(vp), vp]
     L.bom_step_shard_end.restype = i32
+    L.bom_step_vshard_begin.argtypes = [vp, vp, vp, i64, C.POINTER(vp), i64, i64, vp, vp]
+    L.bom_step_vshard_begin.restype = i32
+    L.bom_step_vshard_mid.argtypes = [vp, vp, vp, i64, C.POINTER(vp), vp, i64, vp, i32, C.POINTER(vp), vp, vp]
+    L.bom_step_vshard_mid.restype = i32
+    L.bom_step_vshard_end.argtypes = [vp, vp, vp, i64, C.POINTER(vp), vp, C.POINTER(vp), vp]
+    L.bom_step_vshard_end.restype = i32
     L.bom_set_input_grad.argtypes = [vp, vp]
     L.bom_set_input_grad.restype = i32
     L.bom_step_outputs.argtypes = [vp, C.POINTER(vp), C.POINTER(vp), C.POINTER(vp)]
@@ -241,6 +248,31 @@ def bom_step_shard_end(h, x, labels, n_rows: int, params, q, t: int, xch, grads,
     H = (C.c_void_p * n)(*[_ptr(p) for p in h_out]) if h_out is not None else None
     _check(lib().bom_step_shard_end(h, _ptr(x), _ptr(labels), int(n_rows), P, _ptr(q), int(t), _ptr(xch), G, H,
                                     _stream(stream)), "bom_step_shard_end")
+
+
+def bom_step_vshard_begin(h, x, labels, n_rows: int, params, v_total: int, v_first: int, lse_part,
+                          stream=None) -> None:
+    n = len(params)
+    P = (C.c_void_p * n)(*[_ptr(p) for p in params])
+    _check(lib().bom_step_vshard_begin(h, _ptr(x), _ptr(labels), int(n_rows), P, int(v_total), int(v_first),
+                                       _ptr(lse_part), _stream(stream)), "bom_step_vshard_begin")
+
+
+def bom_step_vshard_mid(h, x, labels, n_rows: int, params, q, t: int, lse_parts, n_shards: int, grads,
+                        dh_part=None, stream=None) -> None:
+    n = len(params)
+    P = (C.c_void_p * n)(*[_ptr(p) for p in params])
+    G = (C.c_void_p * n)(*[_ptr(g) for g in grads]) if grads is not None else None
+    _check(lib().bom_step_vshard_mid(h, _ptr(x), _ptr(labels), int(n_rows), P, _ptr(q), int(t), _ptr(lse_parts),
+                                     int(n_shards), G, _ptr(dh_part), _stream(stream)), "bom_step_vshard_mid")
+
+
+def bom_step_vshard_end(h, x, labels, n_rows: int, params, dh_sum, grads, stream=None) -> None:
+    n = len(params)
+    P = (C.c_void_p * n)(*[_ptr(p) for p in params])
+    G = (C.c_void_p * n)(*[_ptr(g) for g in grads]) if grads is not None else None
+    _check(lib().bom_step_vshard_end(h, _ptr(x), _ptr(labels), int(n_rows), P, _ptr(dh_sum), G, _stream(stream)),
+           "bom_step_vshard_end")
 
 
 def bom_set_step_scalars(h, t_dev, lr_dev=None) -> None:

@@ -118,6 +118,11 @@ struct bom_handle {
     int64_t last_n = 0;
     int64_t shard_n = 0;     // rows of the first half of a sharded step (0: none pending)
     float* sshard = nullptr; // this shard's s^shard = N_t^-1 sum_{i in I_t^shard} r_i (sharded steps)
+    // vocabulary-sharded step: the whole vocabulary, this shard's first id, the
+    // rows of the step in progress and how far it got (0 none, 1 after begin,
+    // 2 after mid)
+    int64_t vs_total = 0, vs_first = 0, vs_n = 0;
+    int vs_stage = 0;
     // tracing: one event pair per launch of the current step
     struct TraceRec {
         const char* name = nullptr;
@@ -498,9 +503,22 @@ void bom_destroy(bom_handle* h) {
 
 namespace {
 
-// The three uses of one step body: a whole step, and the two halves of a
-// row-sharded step around the caller's sum of the exchange vector.
-enum StepPart { kStepFull = 0, kShardBegin = 1, kShardEnd = 2 };
+// The uses of one step body: a whole step, the two halves of a row-sharded
+// step around the caller's sum of the exchange vector, and the three parts of
+// a vocabulary-sharded step around the caller's two exchanges (the row
+// log-sum-exp parts, then the head's input cotangent).
+enum StepPart { kStepFull = 0, kShardBegin = 1, kShardEnd = 2, kVBegin = 3, kVMid = 4, kVEnd = 5 };
+// Most shards whose row log-sum-exp parts one middle part combines.
+constexpr int32_t kMaxVocabShards = 4096;
+
+// Caller buffers of a vocabulary-sharded step (see bom_step_vshard_*).
+struct VShardIo {
+    float* lse_part = nullptr;        // begin: this shard's part of each row's log-sum-exp [n]
+    const float* lse_parts = nullptr; // mid: every shard's part [nsh, n], in shard order
+    int32_t nsh = 0;
+    float* dh_part = nullptr;         // mid: this shard's part of the head's input cotangent [n, d]
+    const float* dh_sum = nullptr;    // end: the shards' parts summed [n, d]
+};
 
 bom_status check_step_args(bom_handle* h, const void* x, const int32_t* labels, int64_t n, void* const* params,
                            const float* q, int64_t t, void* const* grads, void* const* h_out, int part) {
@@ -510,11 +528,14 @@ bom_status check_step_args(bom_handle* h, const void* x, const int32_t* labels, 
     // a sharded step's update follows the caller's gradient sum, and the
     // own-step telemetry needs every row's residual norm
     if (part != kStepFull && (fused || !h->own_out.empty())) return BOM_EINVAL;
+    // a vocabulary-sharded step has one cotangent pass (one exchange of it)
+    if (part >= kVBegin && h->cfg.out_mode != BOM_OUT_U) return BOM_EINVAL;
     const int np = bom_param_count(&h->cfg);
-    if (part == kShardBegin) {
+    if (part == kShardBegin || part == kVBegin || part == kVEnd) {
+        if (part == kVEnd && !grads) return BOM_EINVAL;
         for (int i = 0; i < np; ++i) {
-            if (!params[i]) return BOM_EINVAL;
-            if (!aligned16(params[i])) return BOM_ENOTSUP;
+            if (!params[i] || (part == kVEnd && !grads[i])) return BOM_EINVAL;
+            if (!aligned16(params[i]) || (part == kVEnd && !aligned16(grads[i]))) return BOM_ENOTSUP;
         }
         return aligned16(x) ? BOM_OK : BOM_ENOTSUP;
     }
@@ -540,10 +561,13 @@ bom_status check_step_args(bom_handle* h, const void* x, const int32_t* labels, 
 // checked by the caller.
 bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_t n, void* const* params, float* q,
                      int64_t t, void* const* grads, void* const* h_out, void* stream, int part, double* xch_out,
-                     const double* xch_in) {
+                     const double* xch_in, const VShardIo* vio = nullptr) {
     const bool fused = h->fused_upd;
     const bool gh = h->cfg.out_mode == BOM_OUT_G_AND_H;
-    const bool shard = part != kStepFull;
+    const bool shard = part == kShardBegin || part == kShardEnd;   // row-sharded
+    const bool vshard = part >= kVBegin;                             // vocabulary-sharded
+    // the parts that begin a step (clear the status word, restart the trace)
+    const bool first_part = part == kStepFull || part == kShardBegin || part == kVBegin;
     // a small batch with the update registered: u of every tensor to the
     // scratch, then one update launch for all of them at the end of the step
     const bool upd_sep = fused && h->uscr != nullptr && n <= kUpdSepRows;
@@ -573,10 +597,11 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     const int64_t V = cfg.d_out, dm = h->d_model;
     const int cf32 = h->bf16 ? 0 : 1;
     h->last_n = n;
-    // a traced sharded step records both halves
-    if (part != kShardEnd) h->trace_n = 0;
+    // a traced sharded step records all its parts
+    if (first_part) h->trace_n = 0;
     // the second half of a sharded step needs the first half's rows in the workspace
     h->shard_n = part == kShardBegin ? n : 0;
+    if (!vshard) h->vs_stage = 0;
     int rc = BOM_OK;
 #define BOM_TRY(expr)                                     \
     do {                                                  \
@@ -588,26 +613,29 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     // (a shard's first half has no t: its scalars are set by the second)
     StepScalarsIn st{};
     st.lr = fused ? h->upd_lr : 0.0f;
-    st.inv_bc1 = (h->t_dev || part == kShardBegin) ? 0.0f : inv_bias_correction(cfg.beta1, t);
+    const bool no_t = part == kShardBegin || part == kVBegin;   // first halves take no t
+    st.inv_bc1 = (h->t_dev || no_t) ? 0.0f : inv_bias_correction(cfg.beta1, t);
     st.inv_bc2 = (fused && !h->t_dev) ? inv_bias_correction(h->upd_beta2, t) : 0.0f;
-    st.t_dev = part == kShardBegin ? nullptr : h->t_dev;
+    st.t_dev = no_t ? nullptr : h->t_dev;
     st.lr_dev = h->lr_dev;
     st.beta1 = cfg.beta1;
     st.beta2 = fused ? h->upd_beta2 : 0.0f;
     // A small whole step runs its task-space pass, label scan included, as one
     // cluster launch after the logits (the forward reads no label).
     const bool small = part == kStepFull && h->own_out.empty() && task_small_usable(n, V, dm, cf32);
-    if (part != kShardEnd) {   // the second half keeps the status word of the first
+    if (first_part) {   // later parts keep the status word of the first
         if (cudaMemsetAsync(&h->sc->status, 0, sizeof(int32_t), s) != cudaSuccess) return BOM_ECUDA;
+        // a vocabulary shard checks labels against the whole vocabulary
         if (!small)
             BOM_TRACED("labels_scan", 0, 4.0 * n,
-                       launch_labels_scan(labels, n, V, cfg.ignore_index, cfg.lambda, st, h->sc, s, shard));
+                       launch_labels_scan(labels, n, vshard ? h->vs_total : V, cfg.ignore_index, cfg.lambda, st,
+                                          h->sc, s, shard));
     }
 
     // ---------------------------------------------------------------- forward
     // (the second half of a sharded step finds the activations, R and the
     // residual pass's column partials of its rows in the workspace)
-    const bool run_fwd = part != kShardEnd;
+    const bool run_fwd = first_part;
     const void* xin = x;
     int pi = 0;
     std::vector<int> pidx(h->lw.size());
@@ -700,6 +728,21 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                                                     h->sc, s);
                        }));
     }
+    if (part == kVBegin) {   // this shard's part of each row's log-sum-exp, for the caller's exchange
+        BOM_TRACED("lse_part", 0, 8.0 * n * h->ntiles + 4.0 * n,
+                   launch_vshard_lse_part(h->stats, h->ntiles, n, vio->lse_part, h->sc, s));
+        return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+    }
+    if (part == kVMid) {
+        // the row log-sum-exp from every shard's part, then R over this shard's
+        // columns (the label of column j is vs_first + j)
+        BOM_TRACED("row_lse", 0, 4.0 * vio->nsh * n + 12.0 * n,
+                   launch_vshard_lse(vio->lse_parts, vio->nsh, n, h->Z, cf32, h->ldz, h->vs_first, V, labels,
+                                     cfg.ignore_index, h->lse, h->ce, st, h->sc, s));
+        BOM_TRACED("residual", 0, 2.0 * h->esz * n * h->ldz + 4.0 * resid_blocks(n) * V + 8.0 * n,
+                   launch_residual(h->Z, cf32, h->ldz, n, V, h->lse, labels, cfg.ignore_index, h->colpart, h->sc, s,
+                                   h->vs_first));
+    }
     if (run_fwd && !small) {
         BOM_TRACED("row_lse", 0, 8.0 * n * h->ntiles + 12.0 * n,
                    launch_row_lse(h->Z, cf32, h->ldz, n, V, h->stats, h->ntiles, labels, cfg.ignore_index, h->lse,
@@ -719,15 +762,16 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
         BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 8.0 * V + 24.0 * V,
                    launch_shard_finish_sq(xch_in, h->colpart, resid_blocks(n), V, cfg.beta1, q, h->s, h->qhat,
                                           h->sshard, h->sc, s));
-    } else if (!small) {
+    } else if (!small && part != kVEnd) {
         BOM_TRACED("finish_sq", 0, 4.0 * resid_blocks(n) * V + 20.0 * V,
                    launch_finish_sq(h->colpart, resid_blocks(n), V, cfg.beta1, q, h->s, h->qhat, h->sc, s));
     }
     if (own)   // per-row residual norms for the cancellation ratio
         BOM_TRACED("row_norm", 2.0 * n * V, h->esz * n * h->ldz + 4.0 * n,
                    launch_row_norm(h->Z, cf32, h->ldz, n, V, h->rnorm, h->sc, s));
-    if (!small) {
-        // (a sharded step's loss comes from the shards' summed CE)
+    if (!small && part != kVEnd) {
+        // (a row-sharded step's loss comes from the shards' summed CE; a
+        // vocabulary shard's is its part of the batch's)
         BOM_TRACED("scalars", 0, 4.0 * (n + V),
                    launch_scalars(shard ? nullptr : h->ce, n, h->s, V, own ? h->rnorm : nullptr, h->sc, s));
         // c = colsum_{I_t}(H) and w = W^T qhat (the rank-1 / broadcast factors of the reprojection)
@@ -790,7 +834,12 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
         // the cotangent of X goes out with the u (or g) pass when requested
         const bool want_dx = h->dx_in != nullptr && pass < 2;
         int cur = 0;
-        if (!h->lw.empty() || want_dx) {   // head input: a R W + b 1_{I_t} w^T  (times GELU' of the last layer)
+        void* const dh_dst = h->lw.empty() ? h->dx_in : h->dx[cur];
+        if ((!h->lw.empty() || want_dx) && part == kVEnd) {
+            // the head's input cotangent: the vocabulary shards' parts summed by
+            // the caller, in the compute dtype
+            BOM_TRACED("cast", 0, (4.0 + h->esz) * n * dm, launch_cast_f32(vio->dh_sum, dh_dst, n * dm, cf32, h->sc, s));
+        } else if (!h->lw.empty() || want_dx) {   // head input: a R W + b 1_{I_t} w^T  (times GELU' of the last layer)
             GemmDesc g = gemm1(n, dm, kfull * V, kmaj(h->Z, h->ldz), mnmaj(Wh, dm));
             g.epi.alpha_dev = cr;
             g.epi.beta_dev = cq;
@@ -802,9 +851,11 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                 g.epi.aux = h->lw.back().pre;
                 g.epi.ld_aux = h->lw.back().d_out;
             }
-            g.epi.out = h->lw.empty() ? h->dx_in : h->dx[cur];
+            // a vocabulary shard's part goes to the caller in fp32, for the sum
+            // over shards (the GELU' factor distributes over it)
+            g.epi.out = part == kVMid ? static_cast<void*>(vio->dh_part) : dh_dst;
             g.epi.ld_out = dm;
-            g.epi.out_f32 = cf32;
+            g.epi.out_f32 = part == kVMid ? 1 : cf32;
             if (cs_fused && !h->lw.empty() && h->lw.back().cspart != nullptr) {
                 g.epi.colsum = h->lw.back().cspart;
                 g.epi.ld_colsum = h->lw.back().d_out;
@@ -824,12 +875,14 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
         // dx[0] and dx[1] until the pass ends, so their weight gradients and
         // the head's can run as one grouped launch after the last input
         // cotangent (every weight is still read before its fused update).
-        bool defer_lin = kfull == 1 && !h->lw.empty() && h->lw.size() <= 2;
+        // (a vocabulary shard's head weight gradient runs in its middle part,
+        // the backbone's in its last)
+        bool defer_lin = !vshard && kfull == 1 && !h->lw.empty() && h->lw.size() <= 2;
         for (const LayerWs& L : h->lw)
             defer_lin = defer_lin && (L.kind == BOM_LAYER_LINEAR || L.kind == BOM_LAYER_LINEAR_GELU);
         const bool defer_head =
-            (h->bf16 && kfull == 1 && !h->lw.empty() && h->lw[0].kind == BOM_LAYER_SWIGLU) || defer_lin;
-        {   // head weight: a R^T H + b qhat (x) c
+            (!vshard && h->bf16 && kfull == 1 && !h->lw.empty() && h->lw[0].kind == BOM_LAYER_SWIGLU) || defer_lin;
+        if (part != kVEnd) {   // head weight: a R^T H + b qhat (x) c
             GemmDesc g = gemm1(V, dm, kfull * n, mnmaj(h->Z, h->ldz), mnmaj(xin, dm));
             g.epi.alpha_const = 1.0f;
             g.epi.alpha_dev = cr;
@@ -845,7 +898,7 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
             else
                 BOM_TRY(run_gemm(h, g, s));
         }
-        if (head_b >= 0) {
+        if (head_b >= 0 && part != kVEnd) {
             const float a = pass == 0 ? 1.0f - cfg.lambda : (pass == 1 || pass == 3 ? 1.0f : 0.0f);
             const float b = pass == 0 ? cfg.lambda : (pass == 2 ? 1.0f : 0.0f);
             if (shard)   // this shard's share: a s^shard + b (N_t^shard / N_t) qhat
@@ -859,6 +912,9 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                                         h->sc, s));
             if (fused && !upd_sep) BOM_TRY(update_small(head_b, V));
         }
+        // a vocabulary shard's middle part ends with its head: the backbone
+        // waits for the caller's sum of the input cotangent's parts
+        if (part == kVMid) return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
         for (int l = static_cast<int>(h->lw.size()) - 1; l >= 0; --l) {
             const LayerWs& L = h->lw[l];
             const void* xl = l == 0 ? x : h->lw[l - 1].out;
@@ -1059,6 +1115,65 @@ bom_status bom_step_shard_end(bom_handle* h, const void* x, const int32_t* label
     if ((reinterpret_cast<uintptr_t>(xch) & 7u) != 0) return BOM_ENOTSUP;
     const NvtxRange nvtx_step("bom_step_shard_end");
     return step_impl(h, x, labels, n_rows, params, q, t, grads, h_out, stream, kShardEnd, nullptr, xch);
+}
+
+bom_status bom_step_vshard_begin(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                                 void* const* params, int64_t v_total, int64_t v_first, float* lse_part,
+                                 void* stream) {
+    bom_status rc = check_step_args(h, x, labels, n_rows, params, nullptr, 1, nullptr, nullptr, kVBegin);
+    if (rc != BOM_OK) return rc;
+    if (!lse_part || v_total < 1 || v_total > INT32_MAX || v_first < 0 || v_first > v_total - h->cfg.d_out)
+        return BOM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(lse_part) & 3u) != 0) return BOM_ENOTSUP;
+    const NvtxRange nvtx_step("bom_step_vshard_begin");
+    h->vs_stage = 0;
+    h->vs_total = v_total;
+    h->vs_first = v_first;
+    VShardIo io;
+    io.lse_part = lse_part;
+    rc = step_impl(h, x, labels, n_rows, params, nullptr, 1, nullptr, nullptr, stream, kVBegin, nullptr, nullptr, &io);
+    if (rc == BOM_OK) {
+        h->vs_n = n_rows;
+        h->vs_stage = 1;
+    }
+    return rc;
+}
+
+bom_status bom_step_vshard_mid(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                               void* const* params, float* q, int64_t t, const float* lse_parts, int32_t n_shards,
+                               void* const* grads, float* dh_part, void* stream) {
+    bom_status rc = check_step_args(h, x, labels, n_rows, params, q, t, grads, nullptr, kVMid);
+    if (rc != BOM_OK) return rc;
+    if (h->vs_stage != 1 || n_rows != h->vs_n) return BOM_EINVAL;   // no matching first part
+    if (!lse_parts || n_shards < 1 || n_shards > kMaxVocabShards) return BOM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(lse_parts) & 3u) != 0) return BOM_ENOTSUP;
+    const bool need_dh = !h->lw.empty() || h->dx_in != nullptr;
+    if (need_dh && !dh_part) return BOM_EINVAL;
+    if (need_dh && !aligned16(dh_part)) return BOM_ENOTSUP;
+    const NvtxRange nvtx_step("bom_step_vshard_mid");
+    VShardIo io;
+    io.lse_parts = lse_parts;
+    io.nsh = n_shards;
+    io.dh_part = dh_part;
+    h->vs_stage = 0;
+    rc = step_impl(h, x, labels, n_rows, params, q, t, grads, nullptr, stream, kVMid, nullptr, nullptr, &io);
+    if (rc == BOM_OK) h->vs_stage = 2;
+    return rc;
+}
+
+bom_status bom_step_vshard_end(bom_handle* h, const void* x, const int32_t* labels, int64_t n_rows,
+                               void* const* params, const float* dh_sum, void* const* grads, void* stream) {
+    bom_status rc = check_step_args(h, x, labels, n_rows, params, nullptr, 1, grads, nullptr, kVEnd);
+    if (rc != BOM_OK) return rc;
+    if (h->vs_stage != 2 || n_rows != h->vs_n) return BOM_EINVAL;   // no matching middle part
+    const bool need_dh = !h->lw.empty() || h->dx_in != nullptr;
+    if (need_dh && !dh_sum) return BOM_EINVAL;
+    if (need_dh && !aligned16(dh_sum)) return BOM_ENOTSUP;
+    const NvtxRange nvtx_step("bom_step_vshard_end");
+    VShardIo io;
+    io.dh_sum = dh_sum;
+    h->vs_stage = 0;
+    return step_impl(h, x, labels, n_rows, params, nullptr, 1, grads, nullptr, stream, kVEnd, nullptr, nullptr, &io);
 }
 
 bom_status bom_set_input_grad(bom_handle* h, void* dx) {

@@ -55,8 +55,9 @@ void launch_row_lse(const void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V,
 // Z -> R in place: r_ij = exp(z_ij - lse_i) - [j = y_i] on supervised rows, 0 on
 // the others and in the padding columns [V, ldz); colpart[b, j] receives the
 // fp32 column sums of r over row block b.
+// yoff: the label of column j is yoff + j (a vocabulary shard's first id; 0 otherwise).
 void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* lse, const int32_t* labels,
-                     int32_t ignore, float* colpart, const DevScalars* sc, cudaStream_t s);
+                     int32_t ignore, float* colpart, const DevScalars* sc, cudaStream_t s, int64_t yoff = 0);
 
 // s_j = N_t^-1 sum_b colpart[b, j]; q_j <- beta1 q_j + (1-beta1) s_j;
 // qhat_j = q_j * inv_bc1.  q is only written when the status word is clear.
@@ -79,6 +80,19 @@ void launch_shard_finish_sq(const double* xch, const float* colpart, int64_t nbl
 // out[j] = a s_shard[j] + b shard_frac qhat[j] (this shard's head bias share).
 void launch_shard_bias(const float* s_shard, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
                        const DevScalars* sc, cudaStream_t s);
+
+// Vocabulary-sharded step (see bom_step_vshard_begin / _mid / _end in bom.h).
+// lse_part[i] = log sum over this shard's columns of exp(z_ij), from the
+// per-tile statistics (NaN on every row when the status word is set).
+void launch_vshard_lse_part(const float* stats, int64_t ntiles, int64_t n, float* lse_part, DevScalars* sc,
+                            cudaStream_t s);
+// lse[i] from the shards' parts [nsh, n] in shard order, ce[i] on the rows whose
+// label lies in [v0, v0 + Vloc), the step scalars; BOM_ESHARD on a NaN part.
+void launch_vshard_lse(const float* parts, int32_t nsh, int64_t n, const void* Z, int z_f32, int64_t ldz, int64_t v0,
+                       int64_t Vloc, const int32_t* labels, int32_t ignore, float* lse, float* ce,
+                       const StepScalarsIn& st, DevScalars* sc, cudaStream_t s);
+// dst[0, n) = src (bf16 round to nearest, or fp32); 16-byte aligned buffers.
+void launch_cast_f32(const float* src, void* dst, int64_t n, int dst_f32, const DevScalars* sc, cudaStream_t s);
 
 // Task-space pass of a small step in one cluster launch (task_small.cu):
 // label check and N_t, row log-sum-exp and CE, R over Z, s_t, q_t, qhat_t,

@@ -218,7 +218,8 @@ template <typename T, int VEC>
 __global__ void __launch_bounds__(256, 3) residual_kernel(T* __restrict__ Z, int64_t ldz, int64_t n, int64_t V,
                                                           const float* __restrict__ lse,
                                                           const int32_t* __restrict__ labels, int32_t ignore,
-                                                          float* __restrict__ colpart, const DevScalars* sc) {
+                                                          int64_t yoff, float* __restrict__ colpart,
+                                                          const DevScalars* sc) {
     pdl_enter();
     if (sc->status != 0) return;
     const int64_t col0 = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) * VEC;
@@ -264,7 +265,7 @@ __global__ void __launch_bounds__(256, 3) residual_kernel(T* __restrict__ Z, int
                         if (col0 + 2 * j + 1 >= V) pr[j].y = 0.0f;
                     }
                 }
-                const int64_t yy = static_cast<int64_t>(y) - col0;
+                const int64_t yy = static_cast<int64_t>(y) - yoff - col0;
                 if (yy >= 0 && yy < VEC) {   // this word holds the label column
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
@@ -307,7 +308,7 @@ __global__ void __launch_bounds__(256, 3) residual_kernel(T* __restrict__ Z, int
                     const int64_t c = col0 + k;
                     float p = 0.0f;
                     if (valid && c < V) p = expf(__uint_as_float(ws[k]) - L);
-                    if (valid && c == y) p -= 1.0f;
+                    if (valid && c + yoff == y) p -= 1.0f;
                     rv[k] = p;
                     csum[k] += p;
                 }
@@ -713,6 +714,117 @@ __global__ void shard_bias_kernel(const float* __restrict__ s_shard, const float
     st_elem(out, j, out_f32, a * s_shard[j] + b * sc->shard_frac * qh[j]);
 }
 
+// ---------------------------------------------------------------------------
+// Vocabulary-sharded step: the head's output columns split over shards.  The
+// residual r_ij = exp(z_ij - lse_i) - [j = y_i] (Algorithm 1) couples a row's
+// columns only through its log-sum-exp, so each shard sends one number per
+// row, and s_t, q_t and qhat_t of its columns need no exchange at all.
+//
+// This shard's part of each row's log-sum-exp, log sum_{j in shard} exp(z_ij),
+// from the per-tile (max, sum exp) pairs of the logits epilogue (one warp per
+// row, the pairs in tile order).  A shard that latched an error writes NaN on
+// every row, and a row whose part is not finite latches BOM_ENONFINITE and
+// writes NaN: the shards that combine the parts stop on it.
+__global__ void __launch_bounds__(256) vshard_lse_part_kernel(const float2* __restrict__ stats, int64_t ntiles,
+                                                              int64_t n, float* __restrict__ lse_part,
+                                                              DevScalars* sc) {
+    pdl_enter();
+    const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int l = threadIdx.x & 31;
+    if (row >= n) return;
+    if (sc->status != 0) {
+        if (l == 0) lse_part[row] = __int_as_float(0x7fc00000);
+        return;
+    }
+    const float2* st = stats + row * ntiles;
+    float m = -INFINITY;
+    for (int64_t t = l; t < ntiles; t += 32) m = fmaxf(m, st[t].x);
+    m = warp_max(m);
+    float s = 0.0f;
+    for (int64_t t = l; t < ntiles; t += 32) {
+        const float2 p = st[t];
+        if (p.x != -INFINITY) s += p.y * expf(p.x - m);
+    }
+    s = warp_sum(s);
+    if (l == 0) {
+        const float L = m + logf(s);
+        if (!isfinite(L)) latch_status(sc, BOM_ENONFINITE);
+        lse_part[row] = isfinite(L) ? L : __int_as_float(0x7fc00000);
+    }
+}
+
+// Row log-sum-exp from every shard's part, combined in shard order (every
+// shard computes the same float): lse_i = M + log sum_r exp(part[r, i] - M),
+// M = max_r part[r, i].  ce_i = lse_i - z_{i,y_i} on the supervised rows whose
+// label column this shard holds (y_i - v0 in [0, Vloc)), 0 on the others, so
+// the shards' CE sums add up to the batch's.  A NaN part (a shard that
+// stopped) latches BOM_ESHARD.  Thread 0 also writes the step scalars (host t,
+// or the device step counter), which the first half had no t for.
+__global__ void __launch_bounds__(256) vshard_lse_kernel(const float* __restrict__ parts, int32_t nsh, int64_t n,
+                                                         const void* __restrict__ Z, int z_f32, int64_t ldz,
+                                                         int64_t v0, int64_t Vloc,
+                                                         const int32_t* __restrict__ labels, int32_t ignore,
+                                                         float* __restrict__ lse, float* __restrict__ ce,
+                                                         const StepScalarsIn st, DevScalars* sc) {
+    pdl_enter();
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        float bc1 = st.inv_bc1;
+        if (st.t_dev != nullptr) {
+            const int64_t t = *st.t_dev;
+            if (t < 1)
+                latch_status(sc, BOM_EINVAL);
+            else
+                bc1 = inv_bias_correction(st.beta1, t);
+        }
+        sc->inv_bc1 = bc1;
+    }
+    if (sc->status != 0) return;
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    float M = -INFINITY;
+    bool stopped = false;
+    for (int r = 0; r < nsh; ++r) {
+        const float p = parts[static_cast<int64_t>(r) * n + i];
+        stopped = stopped || isnan(p);
+        M = fmaxf(M, p);
+    }
+    if (stopped) {
+        latch_status(sc, BOM_ESHARD);
+        return;
+    }
+    float S = 0.0f;
+    for (int r = 0; r < nsh; ++r) S += expf(parts[static_cast<int64_t>(r) * n + i] - M);
+    const float L = M + logf(S);
+    const int32_t y = labels[i];
+    const int64_t yl = static_cast<int64_t>(y) - v0;
+    const bool owned = y != ignore && yl >= 0 && yl < Vloc;
+    const float zy = owned ? ld_elem(Z, i * ldz + yl, z_f32) : 0.0f;
+    lse[i] = L;
+    ce[i] = owned ? L - zy : 0.0f;
+    if (!isfinite(L) || (owned && !isfinite(zy))) latch_status(sc, BOM_ENONFINITE);
+}
+
+// dst = src over n elements (fp32 to bf16 by round to nearest even, or an
+// fp32 copy): the summed input cotangent of the head, in the compute dtype the
+// backbone's backward reads.  Four elements per thread from 16-byte aligned
+// buffers, the last n mod 4 one by one.
+__global__ void __launch_bounds__(256) cast_f32_kernel(const float* __restrict__ src, void* __restrict__ dst,
+                                                       int64_t n, int dst_f32, const DevScalars* sc) {
+    pdl_enter();
+    if (sc->status != 0) return;
+    const int64_t n4 = n / 4;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    const int64_t k0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    for (int64_t k = k0; k < n4; k += stride) {
+        const float4 v = reinterpret_cast<const float4*>(src)[k];
+        if (dst_f32)
+            reinterpret_cast<float4*>(dst)[k] = v;
+        else
+            reinterpret_cast<uint2*>(dst)[k] = make_uint2(cvt_bf16x2(v.x, v.y), cvt_bf16x2(v.z, v.w));
+    }
+    for (int64_t k = 4 * n4 + k0; k < n; k += stride) st_elem(dst, k, dst_f32, src[k]);
+}
+
 inline unsigned cdiv(int64_t a, int64_t b) { return static_cast<unsigned>((a + b - 1) / b); }
 
 }  // namespace
@@ -740,15 +852,15 @@ void launch_row_lse(const void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V,
 }
 
 void launch_residual(void* Z, int z_f32, int64_t ldz, int64_t n, int64_t V, const float* lse, const int32_t* labels,
-                     int32_t ignore, float* colpart, const DevScalars* sc, cudaStream_t s) {
+                     int32_t ignore, float* colpart, const DevScalars* sc, cudaStream_t s, int64_t yoff) {
     if (z_f32) {
         dim3 grid(cdiv(ldz, 256 * 4), static_cast<unsigned>(resid_blocks(n)));
         launch_k(residual_kernel<float, 4>, dim3(grid), dim3(256), 0, s, static_cast<float*>(Z), ldz, n, V, lse, labels, ignore,
-                                                       colpart, sc); count_launch();
+                                                       yoff, colpart, sc); count_launch();
     } else {
         dim3 grid(cdiv(ldz, 256 * 8), static_cast<unsigned>(resid_blocks(n)));
         launch_k(residual_kernel<__nv_bfloat16, 8>, dim3(grid), dim3(256), 0, s, static_cast<__nv_bfloat16*>(Z), ldz, n, V, lse,
-                                                               labels, ignore, colpart, sc); count_launch();
+                                                               labels, ignore, yoff, colpart, sc); count_launch();
     }
 }
 
@@ -874,6 +986,29 @@ void launch_shard_finish_sq(const double* xch, const float* colpart, int64_t nbl
 void launch_shard_bias(const float* s_shard, const float* qhat, float a, float b, int64_t V, void* out, int out_f32,
                        const DevScalars* sc, cudaStream_t s) {
     launch_k(shard_bias_kernel, dim3(cdiv(V, 256)), dim3(256), 0, s, s_shard, qhat, a, b, V, out, out_f32, sc);
+    count_launch();
+}
+
+void launch_vshard_lse_part(const float* stats, int64_t ntiles, int64_t n, float* lse_part, DevScalars* sc,
+                            cudaStream_t s) {
+    launch_k(vshard_lse_part_kernel, dim3(cdiv(n * 32, 256)), dim3(256), 0, s, reinterpret_cast<const float2*>(stats),
+             ntiles, n, lse_part, sc);
+    count_launch();
+}
+
+void launch_vshard_lse(const float* parts, int32_t nsh, int64_t n, const void* Z, int z_f32, int64_t ldz, int64_t v0,
+                       int64_t Vloc, const int32_t* labels, int32_t ignore, float* lse, float* ce,
+                       const StepScalarsIn& st, DevScalars* sc, cudaStream_t s) {
+    launch_k(vshard_lse_kernel, dim3(cdiv(n, 256)), dim3(256), 0, s, parts, nsh, n, Z, z_f32, ldz, v0, Vloc, labels,
+             ignore, lse, ce, st, sc);
+    count_launch();
+}
+
+void launch_cast_f32(const float* src, void* dst, int64_t n, int dst_f32, const DevScalars* sc, cudaStream_t s) {
+    const int64_t n4 = n / 4;
+    int64_t blocks = cdiv(n4 > 0 ? n4 : 1, 256);
+    if (blocks > 8 * device_sm_count()) blocks = 8 * device_sm_count();
+    launch_k(cast_f32_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, s, src, dst, n, dst_f32, sc);
     count_launch();
 }
 

@@ -164,3 +164,14 @@ def test_binding_fails_loudly_without_the_library(tmp_path, monkeypatch):
         B.bom_update(**_upd())
     with pytest.raises(RuntimeError, match="missing"):
         B.bom_workspace_bytes(B.make_config(16, 64, 10, [], False, B.BOM_F32))
+
+
+def test_sharded_step_calls_refuse_a_null_handle(built):
+    """The row- and vocabulary-sharded parts check the handle before anything
+    else (no device is touched)."""
+    P = [ALIGNED]
+    assert _code(B.bom_step_shard_begin, None, ALIGNED, ALIGNED, 4, P, ALIGNED, stream=0) == B.BOM_EINVAL
+    assert _code(B.bom_step_vshard_begin, None, ALIGNED, ALIGNED, 4, P, 10, 0, ALIGNED, stream=0) == B.BOM_EINVAL
+    assert _code(B.bom_step_vshard_mid, None, ALIGNED, ALIGNED, 4, P, ALIGNED, 1, ALIGNED, 2, [ALIGNED], ALIGNED,
+                 stream=0) == B.BOM_EINVAL
+    assert _code(B.bom_step_vshard_end, None, ALIGNED, ALIGNED, 4, P, ALIGNED, [ALIGNED], stream=0) == B.BOM_EINVAL
