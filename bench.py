@@ -58,6 +58,10 @@ def _args():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="lm_mlp_bf16")
     p.add_argument("--no-extra", action="store_true", help="skip the head-only and update sub-measurements")
+    p.add_argument("--parallel", default=None, choices=["replicas", "dp"],
+                   help="replicas: independent steps per rank (the default on one GPU); dp: the data-parallel "
+                        "step, rows split across ranks, one all-reduce of the V + 3 exchange sums and one of "
+                        "the gradient shares, then the update (the default under torchrun)")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
     p.add_argument("--separate-update", action="store_true",
                    help="run bom_update after bom_step instead of the update fused into the step")
@@ -248,7 +252,9 @@ def main():
     if a.tokens:
         import dataclasses
         wl = dataclasses.replace(wl, n_rows=a.tokens)
-    params_np = I.init_params(wl, seed=rank)
+    dp = (a.parallel or ("dp" if world > 1 else "replicas")) == "dp"
+    # data-parallel ranks hold one model; replicas are independent models
+    params_np = I.init_params(wl, seed=0 if dp else rank)
     shapes = [s for _, s, _ in wl.param_shapes()]
     sizes = [int(np.prod(s)) for s in shapes]
     offs = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int64)
@@ -280,13 +286,23 @@ def main():
     gt = B.BOM_BF16 if bf16 else B.BOM_F32
     N = wl.n_rows
 
-    fused = not a.separate_update
+    # the data-parallel step updates after the gradient sum: a separate update pass
+    fused = not a.separate_update and not dp
     if fused:   # BOM-AdamW applied inside bom_step, in the epilogues of the weight-gradient GEMMs
         B.bom_set_fused_update(model.h, thviews, vviews, I.weight_decay_mask(wl, WD), LR, B2, EPS)
+    xch = torch.zeros(wl.vocab + 3, dtype=torch.float64, device=dev)
+
+    def allreduce(tensor):   # on the step's stream (torch's current stream)
+        if dist is not None:
+            dist.all_reduce(tensor)
 
     def step(t, xx=x_dev, yy=y_dev):
         if fused:
             model.step(xx, yy, N, pviews, q, t, None, None, stream)
+        elif dp:
+            dp_step(B, model.h, xx, yy, N, pviews, q, t, xch, gviews, gradf, allreduce, stream)
+            B.bom_update(master, gradf, gt, None, vstate, shadow if bf16 else None, P, LR, WD, LAM, B2, EPS, t,
+                         stream)
         else:
             model.step(xx, yy, N, pviews, q, t, gviews, None, stream)
             B.bom_update(master, gradf, gt, None, vstate, shadow if bf16 else None, P, LR, WD, LAM, B2, EPS, t,
@@ -476,10 +492,14 @@ def main():
                 "data": "synthetic: seeded N(0,1) inputs, Kaiming-uniform MLP weights, N(0,0.02) head, "
                         "Zipf(1.1) labels",
                 "config": {"workload": _workload_desc(wl), "global_batch": world * N, "tokens_per_gpu": N,
-                           "parallelism": f"replicas x{world} (no data-path collective)",
+                           "parallelism": (f"dp{world}: rows split across ranks, all-reduce of the V + 3 exchange "
+                                           "sums and of the bf16 gradient shares, separate update; measured on "
+                                           "one GPU only" if dp else f"replicas x{world} (no data-path collective)"),
                            "l2": "flushed between timed steps (256 MiB write outside the step events)",
                            "lr": LR, "weight_decay": WD, "lambda": LAM, "beta1": B1, "beta2": B2,
-                           "update": "fused into the weight-gradient GEMM epilogues" if fused else "separate pass"},
+                           "update": "fused into the weight-gradient GEMM epilogues" if fused else "separate pass",
+                           "step": ("bom_step_shard_begin, all-reduce, bom_step_shard_end, all-reduce, bom_update"
+                                    if dp else "bom_step" + ("" if fused else ", bom_update"))},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
                 "clocks": clk, "loss_first_step": loss_first, "loss": st["loss"], "kernels": kernels,
                 "sub": extra}
@@ -487,6 +507,23 @@ def main():
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
+
+
+def dp_step(lib, h, x, y, n_rows, params, q, t, xch, grads, grad_flat, allreduce, stream=None):
+    """One data-parallel BOM step of this rank's rows.  Algorithm 1's s_t and
+    the surrogate's 1/N_t are means over the supervised rows of the whole
+    batch, so the step splits at one exchange: this rank's part up to the
+    column sums of its residuals (bom_step_shard_begin writes them, its CE sum,
+    its N_t and an error flag into xch, V + 3 doubles), the sum of every rank's
+    xch, the rest of the step with the whole batch's N_t, s_t and qhat_t
+    (bom_step_shard_end writes this rank's share of u into grads, views of
+    grad_flat), then the sum of the ranks' shares.  `allreduce(t)` sums a
+    tensor over the ranks in place (nothing on one rank); `lib` is the
+    binding module."""
+    lib.bom_step_shard_begin(h, x, y, n_rows, params, xch, stream)
+    allreduce(xch)
+    lib.bom_step_shard_end(h, x, y, n_rows, params, q, t, xch, grads, None, stream)
+    allreduce(grad_flat)
 
 
 def _max_over_ranks(dist, x, dev):

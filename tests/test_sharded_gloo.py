@@ -157,3 +157,99 @@ def test_two_rank_vocabulary_parallel_head_equals_full_batch(tmp_path):
         dHs.append(o[g0 + cols.size * d:])
     assert X.rel_l2(dHs[0], ref["dX_u"].ravel()) < 1e-12
     assert np.array_equal(dHs[0], dHs[1])
+
+
+class _OracleShardCalls:
+    """Stands in for the library's two row-shard calls on CPU ranks: the same
+    exchange-vector layout (column sums of R, CE sum, N_t, error flag) and the
+    same gradient shares, computed by the oracle, so that bench.dp_step's
+    order of calls and collectives runs on gloo ranks without a GPU."""
+
+    def __init__(self, wl, params64, lam, beta1):
+        self.wl, self.p, self.lam, self.beta1 = wl, params64, lam, beta1
+        self.layers = X.oracle_layers(wl)
+        self.calls = []
+
+    def bom_step_shard_begin(self, h, x, y, n, params, xch, stream=None):
+        self.calls.append("begin")
+        V = self.wl.vocab
+        Z, saved = O.forward(self.layers, self.wl.head_bias, self.p, x)
+        valid = y != I.IGNORE_INDEX
+        R = O.residuals(Z, y, valid)
+        lse = O.log_sum_exp_rows(Z)
+        ce = float(np.sum((lse - Z[np.arange(len(y)), np.where(valid, y, 0)])[valid]))
+        xch[:V] = torch.from_numpy(R.sum(axis=0))
+        xch[V] = ce
+        xch[V + 1] = float(valid.sum())
+        xch[V + 2] = 0.0
+        self.state = (saved, R, valid)
+
+    def bom_step_shard_end(self, h, x, y, n, params, q, t, xch, grads, h_out, stream=None):
+        self.calls.append("end")
+        V = self.wl.vocab
+        saved, R, valid = self.state
+        n_t = float(xch[V + 1])
+        s = xch[:V].numpy() / n_t
+        q_new, qhat = O.ema_update(q.numpy().copy(), s, t, self.beta1)
+        q.copy_(torch.from_numpy(q_new))
+        dZ = ((1 - self.lam) * R + self.lam * valid[:, None] * qhat[None, :]) / n_t
+        gr, _, _ = O.backward(self.layers, self.wl.head_bias, self.p, saved, dZ)
+        for g, v in zip(grads, gr):
+            g.copy_(torch.from_numpy(np.asarray(v).reshape(g.shape)))
+
+
+def _bench_dp_rank_main(rank, world, port, out_dir):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        import bench
+        params = X.params_f64(WL, I.init_params(WL, 4))
+        xb, y = I.make_batch(WL, 4, 1)
+        x = X.x_f64(WL, xb)
+        rows = np.array_split(np.arange(WL.n_rows), world)[rank]
+        q_prev = np.random.default_rng(5).standard_normal(WL.vocab) * 0.01
+        q_prev -= q_prev.mean()
+        lib = _OracleShardCalls(WL, params, LAM, B1)
+        sizes = [p.size for p in params]
+        flat = torch.zeros(sum(sizes), dtype=torch.float64)
+        views = [v.view(p.shape) for v, p in zip(torch.split(flat, sizes), params)]
+        xch = torch.full((WL.vocab + 3,), float("nan"), dtype=torch.float64)
+        q = torch.from_numpy(q_prev.copy())
+        order = []
+
+        def allreduce(tensor):
+            order.append("allreduce")
+            dist.all_reduce(tensor)
+
+        bench.dp_step(lib, None, x[rows], y[rows], rows.size, params, q, T, xch, views, flat, allreduce)
+        calls = [c for c in lib.calls]
+        np.save(os.path.join(out_dir, f"dp{rank}.npy"), np.concatenate([[xch[WL.vocab + 1].item()], q.numpy(),
+                                                                         flat.numpy()]))
+        with open(os.path.join(out_dir, f"dp{rank}.txt"), "w") as f:
+            f.write(" ".join(calls) + " | " + " ".join(order))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_bench_data_parallel_step_on_two_gloo_ranks(tmp_path):
+    """bench.dp_step, the data-parallel step of bench.py --gpus N: begin, the
+    sum of the exchange vectors, end, the sum of the gradient shares.  On two
+    gloo ranks with the oracle standing in for the library's shard calls,
+    every rank ends with the whole batch's N_t, q and u."""
+    world = 2
+    mp.spawn(_bench_dp_rank_main, args=(world, _free_port(), str(tmp_path)), nprocs=world, join=True)
+    layers = X.oracle_layers(WL)
+    params = X.params_f64(WL, I.init_params(WL, 4))
+    xb, y = I.make_batch(WL, 4, 1)
+    q_prev = np.random.default_rng(5).standard_normal(WL.vocab) * 0.01
+    q_prev -= q_prev.mean()
+    ref = O.bom_step(layers, WL.head_bias, params, X.x_f64(WL, xb), y, q_prev, T, lam=LAM, beta1=B1)
+    u_ref = np.concatenate([u.ravel() for u in ref["u"]])
+    V = WL.vocab
+    outs = [np.load(tmp_path / f"dp{r}.npy") for r in range(world)]
+    for r, o in enumerate(outs):
+        assert int(o[0]) == ref["n_t"]
+        assert X.rel_l2(o[1:1 + V], ref["q"]) < 1e-14
+        assert X.rel_l2(o[1 + V:], u_ref) < 1e-12
+        assert (tmp_path / f"dp{r}.txt").read_text() == "begin end | allreduce allreduce"
+    assert np.array_equal(outs[0], outs[1])
