@@ -7,8 +7,8 @@
 //   warp 0     one thread issues TMA tile loads (128-byte swizzle) into a
 //              shared-memory ring guarded by mbarriers: 32 KB stages (A rows
 //              and this CTA's half of B), as many as fit beside the epilogue's
-//              own shared memory (the fused update's blocks, the SwiGLU
-//              backward's G/U slots), up to six;
+//              own shared memory (the SwiGLU backward's G/U slots), up to
+//              six;
 //   warp 1     allocates 512 TMEM columns (two 256-column fp32 accumulators)
 //              and, in the even CTA, one thread issues the UMMAs (K = 16),
 //              releasing each smem stage with tcgen05.commit;
@@ -175,49 +175,81 @@ __device__ __forceinline__ void unpack32_dyn(const uint4 (&pk)[NW], int slot, fl
     }
 }
 
-// Fused update through shared memory: lane l holds u of row l of a 32 x 32
-// block; the block goes to a per-warp buffer (33-float pitch: both the
-// row-per-lane writes and the column-per-lane reads hit 32 distinct banks, and
-// the eight buffers leave room for six pipeline stages), then the warp walks
-// the 32 rows with lane l on column l, so every access to theta, v and the
-// compute copy is one coalesced 128-byte (64-byte for bf16) line per row.
-// Sixteen rows are loaded before any is written, and the step uses the
+// 32 bytes from a 32-byte aligned global address in one 256-bit load (plain,
+// coherent: the fused update rewrites what it reads).
+__device__ __forceinline__ void ld_global_v8(const void* p, float (&v)[8]) {
+    uint32_t r[8];
+    asm volatile("ld.global.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "l"(p)
+                 : "memory");
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// BOM-AdamW update of one element (Section 3.4): v' = b2 v + (1-b2) u^2,
+// theta' = (1 - lr wd) theta - lr u / (sqrt(v' / (1-b2^t)) + eps), with the
 // hardware square root and reciprocal.
-constexpr int kUpdPitch = 33;
-constexpr int kUpdStgBytes = 32 * kUpdPitch * 4;
-__device__ __forceinline__ void staged_update32(const EpiParams& e, float* buf, int row0, int M, int n, int N,
-                                               const float (&u)[32], float lr, float decay, float inv_bc2) {
-    const int lane = threadIdx.x & 31;
+__device__ __forceinline__ void update1(const EpiParams& e, float u, float& th, float& v, float lr, float decay,
+                                        float inv_bc2) {
+    v = fmaf(e.upd_beta2, v, e.upd_1mb2 * u * u);
+    th = apply_step(decay, th, lr, u * rcp_fast(sqrt_fast(v * inv_bc2) + e.upd_eps));
+}
+
+// Fused update, one row per lane: lane l holds u of its own row m, columns
+// [n, n + 32), and reads and rewrites that row's theta and v and writes its
+// compute copy.  Where the row segment is whole and 32-byte aligned every
+// access is a 256-bit load or store of a whole sector (16 columns of theta and
+// v in flight at a time), as in the other epilogues.  Against a transpose of
+// each 32 x 32 block through shared memory (to walk theta and v in 128-byte
+// lines by rows) it issues about a ninth as many memory instructions for the
+// same sectors, and the grouped weight-gradient launch of the LM block took
+// 3.24 instead of 3.33 ms (same-box A/B).
+__device__ __forceinline__ void row_update32(const EpiParams& e, int m, int M, int n, int N, const float (&u)[32],
+                                             float lr, float decay, float inv_bc2) {
+    if (m >= M) return;
+    const int64_t off = static_cast<int64_t>(m) * e.ld_out + n;
+    float* const th = e.upd_theta + off;
+    float* const vv = e.upd_v + off;
+    float t2[32];
+    if (n + 32 <= N && ((reinterpret_cast<uintptr_t>(th) | reinterpret_cast<uintptr_t>(vv)) & 31u) == 0) {
 #pragma unroll
-    for (int k = 0; k < 32; ++k) buf[lane * kUpdPitch + k] = u[k];
-    __syncwarp();
-    const int c = n + lane;
-    if (c < N) {
-#pragma unroll 1
-        for (int r0 = 0; r0 < 32; r0 += 16) {
-            float th[16], vv[16];
+        for (int h = 0; h < 2; ++h) {
+            float a[2][8], b[2][8];
 #pragma unroll
-            for (int r = 0; r < 16; ++r) {
-                const int m = row0 + r0 + r;
-                const int64_t idx = static_cast<int64_t>(m < M ? m : 0) * e.ld_out + c;
-                th[r] = m < M ? e.upd_theta[idx] : 0.0f;
-                vv[r] = m < M ? e.upd_v[idx] : 0.0f;
+            for (int k = 0; k < 2; ++k) {
+                ld_global_v8(th + 16 * h + 8 * k, a[k]);
+                ld_global_v8(vv + 16 * h + 8 * k, b[k]);
             }
 #pragma unroll
-            for (int r = 0; r < 16; ++r) {
-                const int m = row0 + r0 + r;
-                if (m >= M) continue;
-                const int64_t idx = static_cast<int64_t>(m) * e.ld_out + c;
-                const float uu = buf[(r0 + r) * kUpdPitch + lane];
-                const float v2 = fmaf(e.upd_beta2, vv[r], e.upd_1mb2 * uu * uu);
-                const float t2 = apply_step(decay, th[r], lr, uu * rcp_fast(sqrt_fast(v2 * inv_bc2) + e.upd_eps));
-                e.upd_v[idx] = v2;
-                e.upd_theta[idx] = t2;
-                st_elem(e.out, idx, e.out_f32, t2);
+            for (int k = 0; k < 2; ++k) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    update1(e, u[16 * h + 8 * k + i], a[k][i], b[k][i], lr, decay, inv_bc2);
+                    t2[16 * h + 8 * k + i] = a[k][i];
+                }
+                st_global_v8(th + 16 * h + 8 * k, __float_as_uint(a[k][0]), __float_as_uint(a[k][1]),
+                             __float_as_uint(a[k][2]), __float_as_uint(a[k][3]), __float_as_uint(a[k][4]),
+                             __float_as_uint(a[k][5]), __float_as_uint(a[k][6]), __float_as_uint(a[k][7]));
+                st_global_v8(vv + 16 * h + 8 * k, __float_as_uint(b[k][0]), __float_as_uint(b[k][1]),
+                             __float_as_uint(b[k][2]), __float_as_uint(b[k][3]), __float_as_uint(b[k][4]),
+                             __float_as_uint(b[k][5]), __float_as_uint(b[k][6]), __float_as_uint(b[k][7]));
+            }
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+            t2[i] = 0.0f;
+            if (n + i < N) {
+                float a = th[i], b = vv[i];
+                update1(e, u[i], a, b, lr, decay, inv_bc2);
+                th[i] = a;
+                vv[i] = b;
+                t2[i] = a;
             }
         }
     }
-    __syncwarp();
+    store_row32(e.out, static_cast<int64_t>(m) * e.ld_out, n, N, e.out_f32, t2);
 }
 
 __device__ __forceinline__ float fast_exp(float x) { return exp2f(x * 1.4426950408889634f); }
@@ -237,8 +269,8 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
 // 128 rows of A and its half (128 rows) of B, so a stage is 32 KB.  Epilogue
 // stores go straight from each lane's row to global memory in 256-bit stores
 // (whole 32-byte sectors); staging them through shared memory cost pipeline
-// stages and measured slower.  The fused update stages its accumulator chunk
-// (a per-warp block) to walk theta and v by columns.
+// stages and measured slower.  The fused update reads and rewrites theta and v
+// the same way, one row per lane.
 // SwiGLU backward: the epilogue's per-row operands (the saved G and U,
 // interleaved per 32 columns in one 128-byte line of a row) arrive by TMA.
 // Each epilogue warp owns kEpiSlots slots of a 32-row block of [G 32 | U 32]
@@ -261,11 +293,12 @@ struct Cfg {
     static constexpr int TMEM_COLS = 2 * BNT;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
-    static constexpr int STG_BYTES = EPI == EPI_UPDATE ? 8 * kUpdStgBytes : EPI == EPI_SWIGLU_BWD ? 8 * kEpiLdWarpBytes : 0;
+    static constexpr int STG_BYTES = EPI == EPI_SWIGLU_BWD ? 8 * kEpiLdWarpBytes : 0;
     static constexpr int BAR_BYTES = 512;
     // as many stages as fit in the 227 KB a CTA may use beside the staging
     // blocks, the 1 KB alignment slack and the barrier block, at most six (a
-    // seventh 32 KB stage measured slower on the linear epilogues)
+    // seventh 32 KB stage measured slower on the linear epilogues, and no
+    // faster under the fused update)
     static constexpr int STAGES_FIT = (227 * 1024 - STG_BYTES - 1024 - BAR_BYTES) / (A_BYTES + B_BYTES);
     static constexpr int STAGES = STAGES_FIT < 6 ? STAGES_FIT : 6;
     static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 1024 + BAR_BYTES;
@@ -524,7 +557,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t ra = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux : e.ld_resid);
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
-            uint8_t* stg = stg_all + (warp - 2) * (EPI == EPI_UPDATE ? kUpdStgBytes : 0);
             if (EPI == EPI_SWIGLU_BWD) {
                 // the first blocks of this warp's part of the tile
                 if (lane == 0)
@@ -639,7 +671,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] += r.beta_r1 * t[i];
                     }
-                    staged_update32(e, reinterpret_cast<float*>(stg), row0, PM, n, PN, v, lr, decay, inv_bc2);
+                    row_update32(e, m, PM, n, PN, v, lr, decay, inv_bc2);
                 }
             } else if constexpr (EPI == EPI_LOGITS) {
                 // per (row, column half) softmax statistics: stats pair nt*2 + h.

@@ -253,3 +253,35 @@ def test_host_checks_of_the_vocab_sharded_calls():
     gh = G.GpuBom(wl, I.init_params(wl, 0), out_mode=B.BOM_OUT_G_AND_H)
     assert code(B.bom_step_vshard_begin, gh.model.h, xd, yd, n, gh.params, 2 * V, 0, part) == B.BOM_EINVAL
     torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("name", ["lm_head_wide", "lm_mlp_k1100"])
+def test_one_shard_holding_the_whole_head_equals_bom_step_bit_for_bit(name):
+    """With one shard the combine of the row parts is exact (M + log 1) and
+    the fp32 cotangent part is rounded to the compute dtype once, as the whole
+    step's epilogue rounds it, so the three parts run the whole step's
+    arithmetic in the same order.  (Both workloads take the general task-space
+    path: n V is above the small pass's limit.)"""
+    wl = I.WORKLOADS[name]
+    params = I.init_params(wl, 45)
+    x, y = I.make_batch(wl, 45, 1)
+    q0, t = _q0(wl.vocab, 35), 2
+    head_only = len(wl.layers) == 0
+    shards = _run_vshards(wl, params, x, y, q0, t, [], input_grad=head_only)
+    g = G.GpuBom(wl, params)
+    g.q.copy_(torch.from_numpy(q0))
+    dx = None
+    if head_only:
+        dx = torch.empty((wl.n_rows, wl.d_in), dtype=torch.bfloat16, device=G.DEV)
+        B.bom_set_input_grad(g.model.h, dx)
+    out = g.step(x, y, t)
+    s = shards[0]
+    assert s["stats"]["n_t"] == out["stats"]["n_t"]
+    assert s["stats"]["loss"] == out["stats"]["loss"]
+    assert np.array_equal(s["q"], out["q"])
+    for k in ("qhat", "s", "lse"):
+        assert np.array_equal(s[k], out[k]), k
+    for k, (a, b) in enumerate(zip(s["grads"], out["grads"])):
+        assert torch.equal(a, b), k
+    if head_only:
+        assert torch.equal(s["dx"], dx)
