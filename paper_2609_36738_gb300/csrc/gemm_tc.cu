@@ -200,7 +200,8 @@ __device__ __forceinline__ void update1(const EpiParams& e, float u, float& th, 
 // [n, n + 32), and reads and rewrites that row's theta and v and writes its
 // compute copy.  Where the row segment is whole and 32-byte aligned every
 // access is a 256-bit load or store of a whole sector (16 columns of theta and
-// v in flight at a time), as in the other epilogues.  Against a transpose of
+// v in flight at a time), as in the other epilogues; 16-byte aligned rows take
+// 128-bit accesses, ragged ones single elements.  Against a transpose of
 // each 32 x 32 block through shared memory (to walk theta and v in 128-byte
 // lines by rows) it issues about a ninth as many memory instructions for the
 // same sectors, and the grouped weight-gradient launch of the LM block took
@@ -234,6 +235,29 @@ __device__ __forceinline__ void row_update32(const EpiParams& e, int m, int M, i
                 st_global_v8(vv + 16 * h + 8 * k, __float_as_uint(b[k][0]), __float_as_uint(b[k][1]),
                              __float_as_uint(b[k][2]), __float_as_uint(b[k][3]), __float_as_uint(b[k][4]),
                              __float_as_uint(b[k][5]), __float_as_uint(b[k][6]), __float_as_uint(b[k][7]));
+            }
+        }
+    } else if (n + 32 <= N && ((reinterpret_cast<uintptr_t>(th) | reinterpret_cast<uintptr_t>(vv)) & 15u) == 0) {
+        // rows that are only 16-byte aligned: 128-bit accesses, 8 columns at a time
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            float4 a[2], b[2];
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+                a[j] = reinterpret_cast<const float4*>(th)[2 * k + j];
+                b[j] = reinterpret_cast<const float4*>(vv)[2 * k + j];
+            }
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+                float* pa = &a[j].x;
+                float* pb = &b[j].x;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    update1(e, u[8 * k + 4 * j + i], pa[i], pb[i], lr, decay, inv_bc2);
+                    t2[8 * k + 4 * j + i] = pa[i];
+                }
+                reinterpret_cast<float4*>(th)[2 * k + j] = a[j];
+                reinterpret_cast<float4*>(vv)[2 * k + j] = b[j];
             }
         }
     } else {

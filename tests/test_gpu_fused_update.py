@@ -144,3 +144,33 @@ def test_fused_update_argument_checks():
     B.bom_set_fused_update(f.gpu.model.h, None, None, None, 0.0, 0.0, 0.0)
     with pytest.raises(B.BomError):           # disabled again: grads are required
         f.step(x, y, 1)
+
+
+def test_fused_update_on_rows_only_16_byte_aligned_gives_the_same_bits():
+    """theta and v placed 16 bytes past a 32-byte boundary (the ABI asks for
+    16-byte alignment only): the update epilogue takes its 128-bit form
+    instead of its 256-bit one, with the same arithmetic per element, so
+    theta, v and the compute copies equal those of an aligned run bit for
+    bit.  lm_mlp_k1100 (1100 rows) applies the update in the weight-gradient
+    GEMMs' epilogues."""
+    wl = I.LM_MLP_K1100
+    ref = Fused(wl, seed=6)
+    off = Fused(wl, seed=6)
+
+    def shifted(a):   # same values, data pointer 16 bytes past a 32-byte boundary
+        buf = torch.zeros(a.numel() + 4, dtype=a.dtype, device=a.device)
+        view = buf[4:].view(a.shape)
+        view.copy_(a)
+        assert view.data_ptr() % 32 == 16
+        return view
+
+    off.theta = [shifted(a) for a in off.theta]
+    off.v = [shifted(a) for a in off.v]
+    B.bom_set_fused_update(off.gpu.model.h, off.theta, off.v, off.wd, LR, B2, EPS)
+    for t in range(1, 4):
+        x, y = I.make_batch(wl, seed=6, step=t)
+        ref.step(x, y, t)
+        off.step(x, y, t)
+    torch.cuda.synchronize()
+    for a, b in zip(ref.theta + ref.v + ref.gpu.params, off.theta + off.v + off.gpu.params):
+        assert torch.equal(a, b)
