@@ -796,12 +796,17 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     if (own) passes[npass++] = 3;
     // the fused update takes lr and 1/(1 - beta2^t) from the step scalars
     // the GEMM producing u of tensor k updates it in its epilogue
-    auto fuse = [&](GemmDesc& g, int k) {
-        if (upd_sep) {   // u to the scratch; the update runs after the pass
+    // A small bf16 step updates the weights of a grouped weight-gradient
+    // launch in its epilogue too (narrow 128 x 64 tiles, one row per lane):
+    // only the other tensors' u goes through the scratch to the final update.
+    std::vector<char> upd_in_gemm(upd_sep ? bom_param_count(&cfg) : 0, 0);
+    auto fuse = [&](GemmDesc& g, int k, bool grouped) {
+        if (upd_sep && !(h->bf16 && grouped)) {   // u to the scratch; the update runs after the pass
             g.epi.out = h->uscr + h->uoff[k];
             g.epi.out_f32 = 1;
             return;
         }
+        if (upd_sep) upd_in_gemm[k] = 1;
         g.epi.upd_theta = h->upd_theta[k];
         g.epi.upd_v = h->upd_v[k];
         g.epi.upd_wd = h->upd_wd[k];
@@ -810,7 +815,7 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
         g.epi.upd_eps = h->upd_eps;
         g.epi.out = params[k];   // the compute copy of the updated weight
         g.epi.out_f32 = cf32;
-        if (h->bf16) g.epi_kind = EPI_UPDATE;   // tcgen05 path: staged, coalesced update epilogue
+        if (h->bf16) g.epi_kind = EPI_UPDATE;   // tcgen05 path: the update epilogue, one row per lane
     };
     // a vector tensor k whose u is in ubuf (fp32): update it and its compute copy
     auto update_small = [&](int k, int64_t cnt) -> int {
@@ -892,7 +897,7 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
             g.epi.out = fused ? nullptr : outp[head_w];
             g.epi.ld_out = dm;
             g.epi.out_f32 = of32;
-            if (fused) fuse(g, head_w);
+            if (fused) fuse(g, head_w, defer_head);
             if (defer_head)
                 head_dw = g;
             else
@@ -978,7 +983,7 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                         gw[i].epi.out = fused ? nullptr : outp[pk[i]];
                         gw[i].epi.ld_out = i < 2 ? d : f;
                         gw[i].epi.out_f32 = of32;
-                        if (fused) fuse(gw[i], pk[i]);
+                        if (fused) fuse(gw[i], pk[i], true);
                     }
                     if (defer_w) {
                         for (int i = 0; i < 3; ++i) pend[npend++] = gw[i];
@@ -1028,7 +1033,7 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
                     g.epi.out = fused ? nullptr : outp[p0];
                     g.epi.ld_out = L.d_in;
                     g.epi.out_f32 = of32;
-                    if (fused) fuse(g, p0);
+                    if (fused) fuse(g, p0, defer_lin);
                     if (defer_lin) {
                         pend[npend++] = g;
                         if (l == 0) {   // the last layer of the pass: these and the head's, one launch
@@ -1058,28 +1063,40 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
             if (dx_next) cur ^= 1;
         }
     }
-    if (upd_sep) {   // every tensor's BOM-AdamW update, after its last read in the step
+    bool advanced = false;
+    if (upd_sep) {   // the other tensors' BOM-AdamW update, after their last read in the step
         const int np = bom_param_count(&cfg);
-        std::vector<float*> th(np), vv(np);
-        std::vector<const float*> uu(np);
-        std::vector<void*> cp(np);
-        for (int k = 0; k < np; ++k) {
-            th[k] = h->upd_theta[k];
-            vv[k] = h->upd_v[k];
-            uu[k] = h->uscr + h->uoff[k];
-            cp[k] = params[k];
-        }
+        std::vector<float*> th, vv;
+        std::vector<const float*> uu;
+        std::vector<void*> cp;
+        std::vector<int64_t> nn, rr;
+        std::vector<float> wd;
+        std::vector<const void*> src;
+        std::vector<int> sf;
         int64_t tot = 0;
-        for (int k = 0; k < np; ++k) tot += h->unum[k];
-        BOM_TRY(traced(h, s, "update", 0, 22.0 * tot, [&] {
-            return launch_update_multi(np, th.data(), vv.data(), uu.data(), cp.data(), cf32, h->unum.data(),
-                                       h->upd_wd.data(), usrc.empty() ? nullptr : usrc.data(),
-                                       urows.empty() ? nullptr : urows.data(), usf32.empty() ? nullptr : usf32.data(),
-                                       h->upd_beta2, h->upd_eps, h->sc, h->t_dev, s);
-        }));
+        for (int k = 0; k < np; ++k) {
+            if (upd_in_gemm[k]) continue;
+            th.push_back(h->upd_theta[k]);
+            vv.push_back(h->upd_v[k]);
+            uu.push_back(h->uscr + h->uoff[k]);
+            cp.push_back(params[k]);
+            nn.push_back(h->unum[k]);
+            wd.push_back(h->upd_wd[k]);
+            src.push_back(usrc.empty() ? nullptr : usrc[k]);
+            rr.push_back(urows.empty() ? 0 : urows[k]);
+            sf.push_back(usf32.empty() ? cf32 : usf32[k]);
+            tot += h->unum[k];
+        }
+        if (!th.empty()) {
+            BOM_TRY(traced(h, s, "update", 0, 22.0 * tot, [&] {
+                return launch_update_multi(static_cast<int>(th.size()), th.data(), vv.data(), uu.data(), cp.data(),
+                                           cf32, nn.data(), wd.data(), src.data(), rr.data(), sf.data(),
+                                           h->upd_beta2, h->upd_eps, h->sc, h->t_dev, s);
+            }));
+            advanced = true;   // the update of a small step advances the device step counter itself
+        }
     }
-    // the update of a small step advances the device step counter itself
-    if (h->t_dev && !upd_sep) launch_advance_step(h->t_dev, h->sc, s);
+    if (h->t_dev && !advanced) launch_advance_step(h->t_dev, h->sc, s);
 #undef BOM_TRY
     return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
 }

@@ -1061,10 +1061,14 @@ static int choose_split(int tiles, int units, int kb_total, int64_t mn, int64_t 
     return best;
 }
 
-// Linear epilogue on narrow single-CTA tiles: A K-major (the forward layers
-// and the input cotangents of the small configurations), or both operands
-// MN-major (their weight gradients, K = the batch rows).
-static int dispatch_narrow(const Params& p, bool a_mn, bool b_mn, cudaStream_t stream) {
+// Narrow single-CTA tiles: the linear epilogue with A K-major (the forward
+// layers and the input cotangents of the small configurations), or with both
+// operands MN-major (their weight gradients, K = the batch rows), and the
+// fused update of those weight gradients.
+static int dispatch_narrow(const Params& p, bool a_mn, bool b_mn, cudaStream_t stream, int epi_kind = EPI_LINEAR) {
+    if (epi_kind == EPI_UPDATE)
+        return a_mn && b_mn ? launch_inst<1, true, true, EPI_UPDATE, kBnSmall>(p, stream) : BOM_ENOTSUP;
+    if (epi_kind != EPI_LINEAR) return BOM_ENOTSUP;
     if (a_mn) return b_mn ? launch_inst<1, true, true, EPI_LINEAR, kBnSmall>(p, stream) : BOM_ENOTSUP;
     return b_mn ? launch_inst<1, false, true, EPI_LINEAR, kBnSmall>(p, stream)
                 : launch_inst<1, false, false, EPI_LINEAR, kBnSmall>(p, stream);
@@ -1232,10 +1236,11 @@ int launch_gemm_tc_group(const GemmDesc* gs, int n, cudaStream_t stream) {
     const GemmDesc& g0 = gs[0];
     p.kb[0] = static_cast<int>((g0.K[0] + BK - 1) / BK);
     // Weight gradients over a short K (at most 16 k-blocks: small batches)
-    // with a linear epilogue (u to memory) spend most of a 256 x 256 tile in
-    // its epilogue, and their few hundred tiles end on a partial wave of
-    // CTA pairs: single CTAs with 128 x 64 tiles instead.
-    const bool narrow = g0.epi_kind == EPI_LINEAR && p.kb[0] <= 16 && g0.A[0].mn_major && g0.B[0].mn_major;
+    // with a linear epilogue (u to memory) or the fused update spend most of a
+    // 256 x 256 tile in its epilogue, and their few hundred tiles end on a
+    // partial wave of CTA pairs: single CTAs with 128 x 64 tiles instead.
+    const bool narrow = (g0.epi_kind == EPI_LINEAR || g0.epi_kind == EPI_UPDATE) && p.kb[0] <= 16 &&
+                        g0.A[0].mn_major && g0.B[0].mn_major;
     const int tile_m = narrow ? BM : 2 * BM, tile_n = narrow ? kBnSmall : BN;
     p.nseg = 1;
     p.bn_out = tile_n;
@@ -1272,7 +1277,7 @@ int launch_gemm_tc_group(const GemmDesc* gs, int n, cudaStream_t stream) {
         tiles += tm * tn;
     }
     p.tile_base[n] = tiles;
-    if (narrow) return dispatch_narrow(p, true, true, stream);
+    if (narrow) return dispatch_narrow(p, true, true, stream, g0.epi_kind);
     return dispatch<2>(p, g0.epi_kind, g0.A[0].mn_major, g0.B[0].mn_major, false, stream);
 }
 
