@@ -57,7 +57,6 @@ struct Prob {
 struct Params {
     CUtensorMap mapA[2];
     CUtensorMap mapB[2];
-    CUtensorMap mapE[2];   // SwiGLU backward: saved G|U blocks, 32 rows x 64 columns, 128-byte swizzle
     int M, N;
     int kb[2];
     int nseg;
@@ -296,18 +295,23 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32]) {
 // stages and measured slower.  The fused update reads and rewrites theta and v
 // the same way, one row per lane.
 // SwiGLU backward: the epilogue's per-row operands (the saved G and U,
-// interleaved per 32 columns in one 128-byte line of a row) arrive by TMA.
-// Each epilogue warp owns kEpiSlots slots of a 32-row block of [G 32 | U 32]
-// (4 KB, 128-byte swizzle: 16-byte chunk k of row r at r * 128 + 16 * (k ^ (r & 7)),
-// so the row-per-lane reads are conflict-free); lane 0 loads block
-// j + kEpiSlots into the slot block j has just freed.
-constexpr int kEpiLdBlock = 32 * 64;
-// One slot per warp (the next block loads while the current one is
-// processed): the 32 KB this frees is a sixth pipeline stage, which the
-// mainloop needs more than the epilogue needs a second block in flight
-// (same-box A/B: 0.78 -> 0.74-0.75 ms per step for the two launches).
-constexpr int kEpiSlots = 1;   // G|U blocks in flight per epilogue warp
-constexpr int kEpiLdWarpBytes = kEpiSlots * 2 * kEpiLdBlock;
+// interleaved per 32 columns in one 128-byte line of a row) are read by each
+// lane for its own row in four 256-bit loads, the next chunk's line while the
+// current one is processed.
+
+// One 128-byte line (a [G 32 | U 32] block of the interleaved saved gate and up
+// pre-activations, 32-byte aligned) in four 256-bit loads: G in w[0..3], U in w[4..7].
+__device__ __forceinline__ void load_line128(const void* p, uint4 (&w)[8]) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        uint4 a, b;
+        asm("ld.global.nc.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+            : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w), "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w)
+            : "l"(static_cast<const char*>(p) + 32 * i));
+        w[2 * i] = a;
+        w[2 * i + 1] = b;
+    }
+}
 
 template <int CG, int EPI, int BNT>
 struct Cfg {
@@ -317,7 +321,7 @@ struct Cfg {
     static constexpr int TMEM_COLS = 2 * BNT;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
-    static constexpr int STG_BYTES = EPI == EPI_SWIGLU_BWD ? 8 * kEpiLdWarpBytes : 0;
+    static constexpr int STG_BYTES = 0;
     static constexpr int BAR_BYTES = 512;
     // as many stages as fit in the 227 KB a CTA may use beside the staging
     // blocks, the 1 KB alignment slack and the barrier block, at most six (a
@@ -348,8 +352,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
     uint64_t* tfull = bars + 2 * STAGES;
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
-    uint64_t* ebar = drain + 1;   // SwiGLU backward: 2 slots x 8 epilogue warps
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ebar + 16);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int* skip_flag = reinterpret_cast<int*>(tmem_slot + 2);
 
@@ -371,7 +374,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             mbar_init(&tempty[a], CG == 2 ? 2 : 256);
         }
         mbar_init(drain, 1);
-        for (int b = 0; b < 16; ++b) mbar_init(&ebar[b], 1);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -544,17 +546,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
         const int row = q * 32 + lane;
         constexpr int CPW = BNT / 64;  // 32-column chunks per warp
         int it = 0;
-        // SwiGLU backward operand slots of this warp and their barrier phases
-        uint8_t* const eslot = stg_all + (warp - 2) * kEpiLdWarpBytes;
-        uint64_t* const ebw = ebar + 2 * (warp - 2);
-        uint32_t eph = 0, epend = 0;   // phase bit and in-flight flag per slot
-        auto eissue = [&](int slot, int col, int rowg) {   // lane 0 only
-            fence_proxy_async_shared();   // this warp's reads of the slot precede the refill
-            // the 32-column block of G and U is one 128-byte line per row
-            mbar_arrive_expect_tx(&ebw[slot], 2 * kEpiLdBlock);
-            tma_load_2d(eslot + slot * 2 * kEpiLdBlock, &p.mapE[0], &ebw[slot], 2 * col, rowg);
-            epend |= 1u << slot;
-        };
         for (int w = unit; w < num_work; w += nunits, ++it) {
             const int tile = w / p.ksplit;
             const ProbView pv = prob_of(p, tile);
@@ -574,6 +565,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             // warp's first chunk is loaded before the mainloop wait, and each
             // later chunk while the previous one is being processed.
             uint4 xa[4], xb[4];
+            uint4 gu[8];   // SwiGLU backward: the current chunk's [G 32 | U 32] line
             const bool has_a = valid && ((EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.resid != nullptr));
             const bool has_b = valid && ((EPI == EPI_SWIGLU_BWD) || (EPI == EPI_LINEAR && e.act == ACT_DGELU));
             const void* pa = EPI == EPI_SWIGLU_BWD ? e.aux : e.resid;
@@ -582,10 +574,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
             const int64_t rb = static_cast<int64_t>(m) * (EPI == EPI_SWIGLU_BWD ? e.ld_aux2 : e.ld_aux);
             const int row0 = m0 + q * 32;   // first of the warp's 32 rows
             if (EPI == EPI_SWIGLU_BWD) {
-                // the first blocks of this warp's part of the tile
-                if (lane == 0)
-                    for (int j = 0; j < kEpiSlots && j < CPW; ++j)
-                        if (n0 + 32 * (c0 + j) < PN) eissue(j, n0 + 32 * (c0 + j), row0);
+                // the line of this warp's first chunk
+                if (valid && n0 + 32 * c0 < PN)
+                    load_line128(static_cast<const uint16_t*>(pa) + ra + 2 * (n0 + 32 * c0), gu);
             } else {
                 if (has_a) load_chunk_bf16(pa, ra, n0 + 32 * c0, PN, xa, 0);
                 if (has_b) load_chunk_bf16(pb, rb, n0 + 32 * c0, PN, xb, 0);
@@ -807,42 +798,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 }
             } else if constexpr (EPI == EPI_SWIGLU_BWD) {
                 float g[32], u[32];
-                bool ok = true;
 #pragma unroll 1
                 for (int j = 0; j < CPW; ++j) {
                     const int c = c0 + j;
                     const int n = n0 + c * 32;
                     if (n >= PN) break;
-                    const int slot = j % kEpiSlots;
-                    if (!mbar_wait_bounded(&ebw[slot], (eph >> slot) & 1u, abort_flag)) {
-                        ok = false;
-                        break;
-                    }
-                    eph ^= 1u << slot;
-                    epend &= ~(1u << slot);
-                    {   // row `lane` of the G|U block (128-byte swizzle: logical
-                        // 16-byte chunk k at chunk k ^ (lane & 7); G in 0-3, U in 4-7)
-                        const uint8_t* bg = eslot + slot * 2 * kEpiLdBlock + lane * 128;
-                        const int sw = lane & 7;
+                    // this row's [G 32 | U 32] line (loaded during the previous chunk)
 #pragma unroll
-                        for (int k = 0; k < 4; ++k) {
-                            const uint4 wg = *reinterpret_cast<const uint4*>(bg + 16 * (k ^ sw));
-                            const uint4 wu = *reinterpret_cast<const uint4*>(bg + 16 * ((k + 4) ^ sw));
-                            const uint32_t a4[4] = {wg.x, wg.y, wg.z, wg.w};
-                            const uint32_t b4[4] = {wu.x, wu.y, wu.z, wu.w};
+                    for (int k = 0; k < 4; ++k) {
+                        const uint32_t a4[4] = {gu[k].x, gu[k].y, gu[k].z, gu[k].w};
+                        const uint32_t b4[4] = {gu[k + 4].x, gu[k + 4].y, gu[k + 4].z, gu[k + 4].w};
 #pragma unroll
-                            for (int q2 = 0; q2 < 4; ++q2) {
-                                g[8 * k + 2 * q2] = bf16_lo(a4[q2]);
-                                g[8 * k + 2 * q2 + 1] = bf16_hi(a4[q2]);
-                                u[8 * k + 2 * q2] = bf16_lo(b4[q2]);
-                                u[8 * k + 2 * q2 + 1] = bf16_hi(b4[q2]);
-                            }
+                        for (int q2 = 0; q2 < 4; ++q2) {
+                            g[8 * k + 2 * q2] = bf16_lo(a4[q2]);
+                            g[8 * k + 2 * q2 + 1] = bf16_hi(a4[q2]);
+                            u[8 * k + 2 * q2] = bf16_lo(b4[q2]);
+                            u[8 * k + 2 * q2 + 1] = bf16_hi(b4[q2]);
                         }
                     }
-                    fence_proxy_async_shared();   // every lane's reads of the slot before its refill
-                    __syncwarp();
-                    if (lane == 0 && j + kEpiSlots < CPW && n + 32 * kEpiSlots < PN)
-                        eissue(slot, n + 32 * kEpiSlots, row0);
+                    if (valid && j + 1 < CPW && n + 32 < PN)
+                        load_line128(static_cast<const uint16_t*>(pa) + ra + 2 * (n + 32), gu);
                     tmem_load32(tbase + c * 32, v);
                     if (valid) {
                         float du[32];
@@ -865,7 +840,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                         store_row32(e.out2, static_cast<int64_t>(m) * e.ld_out2, n, PN, e.out2_f32, du);
                     }
                 }
-                if (!ok) break;
             }
             tc_fence_before();
             if constexpr (CG == 2) {
@@ -876,11 +850,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
                 mbar_arrive(&tempty[acc]);
             }
         }
-        // SwiGLU backward operand loads still in flight (an aborted tile) land
-        // before the CTA may exit
-        if (EPI == EPI_SWIGLU_BWD && lane == 0)
-            for (int sl = 0; sl < kEpiSlots; ++sl)
-                if (epend & (1u << sl)) mbar_wait_bounded(&ebw[sl], (eph >> sl) & 1u, nullptr);
     }
 
     __syncthreads();
@@ -1154,9 +1123,6 @@ int launch_gemm_tc(const GemmDesc& g, cudaStream_t stream) {
             return BOM_ENOTSUP;
         }
     }
-    if (g.epi_kind == EPI_SWIGLU_BWD &&
-        !make_map(&p.mapE[0], g.epi.aux, g.epi.ld_aux, g.M, g.epi.ld_aux, 64, 32, CU_TENSOR_MAP_SWIZZLE_128B))
-        return BOM_ENOTSUP;
     p.M = static_cast<int>(g.M);
     p.N = static_cast<int>(g.N);
     p.nseg = g.nseg;
