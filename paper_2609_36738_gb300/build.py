@@ -19,8 +19,8 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libbom.so")
 
-SOURCES = ["bom_api.cu", "gemm_tc.cu", "gemm_simt.cu", "task_space.cu", "task_small.cu", "norm.cu", "update.cu",
-           "noalloc.cu"]
+SOURCES = ["bom_api.cu", "gemm_tc.cu", "gemm_simt.cu", "task_space.cu", "task_small.cu", "tiny_step.cu", "norm.cu",
+           "update.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

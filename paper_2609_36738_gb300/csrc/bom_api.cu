@@ -623,6 +623,65 @@ bom_status step_impl(bom_handle* h, const void* x, const int32_t* labels, int64_
     // A small whole step runs its task-space pass, label scan included, as one
     // cluster launch after the logits (the forward reads no label).
     const bool small = part == kStepFull && h->own_out.empty() && task_small_usable(n, V, dm, cf32);
+    // A small fp32 MLP classifier (the tiny configurations: a few dozen rows,
+    // at most two Linear layers) runs its whole step in one CTA.
+    if (part == kStepFull && !h->bf16 && !gh && h->own_out.empty() && h->dx_in == nullptr &&
+        h->lw.size() <= static_cast<size_t>(kTinyStepMaxLayers)) {
+        bool lin = true;
+        for (const LayerWs& L : h->lw) lin = lin && (L.kind == BOM_LAYER_LINEAR || L.kind == BOM_LAYER_LINEAR_GELU);
+        TinyStepArgs ta{};
+        const int nl = static_cast<int>(h->lw.size());
+        int dim[kTinyStepMaxLayers + 2] = {};
+        bool bias[kTinyStepMaxLayers + 1] = {};
+        dim[0] = static_cast<int>(cfg.d_in);
+        for (int k = 0; k < nl; ++k) {
+            dim[k + 1] = static_cast<int>(h->lw[k].d_out);
+            bias[k] = h->lw[k].bias;
+        }
+        dim[nl + 1] = static_cast<int>(V);
+        bias[nl] = cfg.head_bias != 0;
+        if (lin && cfg.d_in <= kTinyStepMaxWidth && V <= kTinyStepMaxWidth &&
+            tiny_step_layout(static_cast<int>(n), nl, dim, bias, &ta.lay)) {
+            ta.x = static_cast<const float*>(x);
+            ta.labels = labels;
+            ta.n = static_cast<int>(n);
+            ta.nl = nl;
+            for (int k = 0; k <= nl + 1; ++k) ta.dim[k] = dim[k];
+            int pt = 0;
+            for (int k = 0; k <= nl; ++k) {
+                if (k < nl) ta.gelu[k] = h->lw[k].kind == BOM_LAYER_LINEAR_GELU ? 1 : 0;
+                ta.tw[k] = pt;
+                ta.W[k] = static_cast<const float*>(params[pt++]);
+                ta.tb[k] = bias[k] ? pt : -1;
+                ta.b[k] = bias[k] ? static_cast<const float*>(params[pt++]) : nullptr;
+            }
+            for (int t2 = 0; t2 < pt; ++t2) {
+                ta.u[t2] = fused ? nullptr : static_cast<float*>(grads[t2]);
+                ta.theta[t2] = fused ? h->upd_theta[t2] : nullptr;
+                ta.v[t2] = fused ? h->upd_v[t2] : nullptr;
+                ta.wd[t2] = fused ? h->upd_wd[t2] : 0.0f;
+                ta.copy[t2] = static_cast<float*>(params[t2]);
+            }
+            ta.ignore = cfg.ignore_index;
+            ta.lambda = cfg.lambda;
+            ta.beta1 = cfg.beta1;
+            ta.q = q;
+            ta.qhat_out = h->qhat;
+            ta.s_out = h->s;
+            ta.lse_out = h->lse;
+            ta.beta2 = fused ? h->upd_beta2 : 0.0f;
+            ta.eps = fused ? h->upd_eps : 0.0f;
+            ta.st = st;
+            ta.sc = h->sc;
+            ta.t_adv = h->t_dev;
+            if (cudaMemsetAsync(&h->sc->status, 0, sizeof(int32_t), s) != cudaSuccess) return BOM_ECUDA;
+            double fl = 0.0;
+            for (int k = 0; k <= nl; ++k) fl += 6.0 * n * dim[k] * dim[k + 1];
+            BOM_TRY(traced(h, s, "tiny_step", fl, 4.0 * (n * dim[0] + 3.0 * ta.lay.floats),
+                           [&] { return launch_tiny_step(ta, s); }));
+            return cudaPeekAtLastError() == cudaSuccess ? BOM_OK : BOM_ECUDA;
+        }
+    }
     if (first_part) {   // later parts keep the status word of the first
         if (cudaMemsetAsync(&h->sc->status, 0, sizeof(int32_t), s) != cudaSuccess) return BOM_ECUDA;
         // a vocabulary shard checks labels against the whole vocabulary

@@ -110,6 +110,47 @@ int launch_task_small(const void* Z, int z_f32, int64_t ldz, const int32_t* labe
                       float* s_out, float* qhat, float* lse, float* cvec, float* wvec, void* hb_out, int hb_f32,
                       float hb_a, float hb_b, const StepScalarsIn& st, DevScalars* sc, cudaStream_t s);
 
+// Whole step of a small fp32 MLP classifier (at most two Linear / Linear+GELU
+// layers before the head, at most 128 rows, widths at most 1024, everything in
+// 192 KB of shared memory) in one CTA (tiny_step.cu): forward, task space,
+// backward and either the fused update or u.  The layout holds the
+// shared-memory offsets (floats) of the staged operands and intermediates.
+constexpr int kTinyStepMaxLayers = 2;
+constexpr int kTinyStepMaxRows = 128;
+constexpr int kTinyStepMaxWidth = 1024;
+constexpr int64_t kTinyStepMaxFloats = 48 * 1024;
+struct TinyLayout {
+    int x, W[kTinyStepMaxLayers + 1], b[kTinyStepMaxLayers + 1], pre[kTinyStepMaxLayers], act[kTinyStepMaxLayers];
+    int z, g[2], lse, lab, qh, sv, floats;
+};
+struct TinyStepArgs {
+    const float* x;                              // [n, dim[0]]
+    const int32_t* labels;                       // [n]
+    int n, nl;                                   // rows, backbone layers
+    int dim[kTinyStepMaxLayers + 2];             // input width, layer widths, classes
+    int gelu[kTinyStepMaxLayers];                // layer k applies GELU
+    const float* W[kTinyStepMaxLayers + 1];      // layer weights [dim[k+1], dim[k]]; the head last
+    const float* b[kTinyStepMaxLayers + 1];      // biases, or null
+    int tw[kTinyStepMaxLayers + 1];              // tensor index of W[k] (parameter order)
+    int tb[kTinyStepMaxLayers + 1];              // tensor index of b[k], or -1
+    int32_t ignore;
+    float lambda, beta1;
+    float* q;                                    // [V] in/out
+    float *qhat_out, *s_out, *lse_out;           // the handle's outputs
+    float* u[2 * kTinyStepMaxLayers + 2];        // u per tensor (when theta is null)
+    float* theta[2 * kTinyStepMaxLayers + 2];    // fused update: fp32 masters, or null
+    float* v[2 * kTinyStepMaxLayers + 2];
+    float wd[2 * kTinyStepMaxLayers + 2];
+    float* copy[2 * kTinyStepMaxLayers + 2];     // compute copies (the parameters)
+    float beta2, eps;
+    StepScalarsIn st;
+    DevScalars* sc;
+    int64_t* t_adv;                              // device step counter advanced when clear, or null
+    TinyLayout lay;
+};
+bool tiny_step_layout(int n, int nl, const int* dim, const bool* bias, TinyLayout* lay);
+int launch_tiny_step(const TinyStepArgs& a, cudaStream_t s);
+
 // loss = N_t^-1 sum_i ce_i (kept as it is when ce is NULL), ||s|| and, when
 // rnorm is given, r_norm_mean = N_t^-1 sum_i rnorm_i.
 void launch_scalars(const float* ce, int64_t n, const float* s_vec, int64_t V, const float* rnorm, DevScalars* sc,
