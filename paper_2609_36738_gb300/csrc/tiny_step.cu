@@ -31,9 +31,11 @@ namespace {
 constexpr int kTinyThreads = 1024;
 constexpr int kTinyWarps = kTinyThreads / 32;
 
-// Odd row pitch for the shared-memory copies: lanes that walk different rows
-// at the same column hit different banks.
-__host__ __device__ inline int tiny_pitch(int d) { return d | 1; }
+// Row pitch of the shared-memory copies: a multiple of 4 floats (rows load as
+// 16-byte words) that is 4 more than a multiple of 8, so the 16-byte words
+// that eight lanes load from eight consecutive rows at one column fall in
+// different bank quads; the padding columns stay zero.
+__host__ __device__ inline int tiny_pitch(int d) { return ((d + 7) & ~7) + 4; }
 
 __device__ __forceinline__ float tw_sum(float v) {
 #pragma unroll
@@ -67,6 +69,8 @@ __global__ void __launch_bounds__(kTinyThreads, 1) tiny_step_kernel(const TinySt
     if (a.sc->status != 0) return;   // an earlier kernel of the step failed
 
     // ---------------------------------------------------------------- loads
+    for (int i = tid; i < L.floats; i += kTinyThreads) sm[i] = 0.0f;   // zero padding
+    __syncthreads();
     tiny_stage(sm + L.x, a.x, n, a.dim[0], tiny_pitch(a.dim[0]));
     for (int k = 0; k <= nl; ++k) {
         tiny_stage(sm + L.W[k], a.W[k], a.dim[k + 1], a.dim[k], tiny_pitch(a.dim[k]));
@@ -96,13 +100,34 @@ __global__ void __launch_bounds__(kTinyThreads, 1) tiny_step_kernel(const TinySt
         float* pre = k < nl ? sm + L.pre[k] : sm + L.z;
         float* out = k < nl ? sm + L.act[k] : nullptr;
         const bool gelu = k < nl && a.gelu[k];
-        for (int i0 = tid; i0 < n * dout; i0 += kTinyThreads) {
-            const int i = i0 / dout, j = i0 - i * dout;
-            float acc = 0.0f;
-            for (int c = 0; c < din; ++c) acc = fmaf(xin[i * pin + c], W[j * pin + c], acc);
-            if (b) acc += b[j];
-            pre[i * pout + j] = acc;
-            if (out) out[i * pout + j] = gelu ? gelu_f(acc) : acc;
+        // four rows per thread: each 16-byte word of W serves four rows
+        const int nb = (n + 3) >> 2, c4 = (din + 3) >> 2;
+        for (int i0 = tid; i0 < nb * dout; i0 += kTinyThreads) {
+            const int ib = i0 / dout, j = i0 - ib * dout;
+            const int nr = min(4, n - 4 * ib);
+            const float4* wr = reinterpret_cast<const float4*>(W + j * pin);
+            float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            for (int c = 0; c < c4; ++c) {
+                const float4 wv = wr[c];
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    if (r >= nr) break;
+                    const float4 xv = reinterpret_cast<const float4*>(xin + (4 * ib + r) * pin)[c];
+                    acc[r] = fmaf(xv.x, wv.x, acc[r]);
+                    acc[r] = fmaf(xv.y, wv.y, acc[r]);
+                    acc[r] = fmaf(xv.z, wv.z, acc[r]);
+                    acc[r] = fmaf(xv.w, wv.w, acc[r]);
+                }
+            }
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                if (r >= nr) break;
+                const int i = 4 * ib + r;
+                float v = acc[r];
+                if (b) v += b[j];
+                pre[i * pout + j] = v;
+                if (out) out[i * pout + j] = gelu ? gelu_f(v) : v;
+            }
         }
         __syncthreads();
     }
@@ -265,12 +290,23 @@ __global__ void __launch_bounds__(kTinyThreads, 1) tiny_step_kernel(const TinySt
         const float* xin = act(k);
         const float* W = sm + L.W[k];
         const int tw = a.tw[k], tb = a.tb[k];
-        // weight: u_W[j, c] = sum_i dcur[i, j] xin[i, c]
-        for (int i0 = tid; i0 < dout * din; i0 += kTinyThreads) {
-            const int j = i0 / din, c = i0 - j * din;
-            float acc = 0.0f;
-            for (int r = 0; r < n; ++r) acc = fmaf(dcur[r * pcur + j], xin[r * pin + c], acc);
-            emit(tw, i0, acc);
+        // weight: u_W[j, c] = sum_i dcur[i, j] xin[i, c], four output rows j per
+        // thread (one 16-byte word of dcur per row i serves all four)
+        const int jb4 = (dout + 3) >> 2;
+        for (int i0 = tid; i0 < jb4 * din; i0 += kTinyThreads) {
+            const int jb = i0 / din, c = i0 - jb * din;
+            float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            for (int r = 0; r < n; ++r) {
+                const float4 dv = reinterpret_cast<const float4*>(dcur + r * pcur)[jb];
+                const float xv = xin[r * pin + c];
+                acc[0] = fmaf(dv.x, xv, acc[0]);
+                acc[1] = fmaf(dv.y, xv, acc[1]);
+                acc[2] = fmaf(dv.z, xv, acc[2]);
+                acc[3] = fmaf(dv.w, xv, acc[3]);
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                if (4 * jb + q < dout) emit(tw, static_cast<int64_t>(4 * jb + q) * din + c, acc[q]);
         }
         // bias: the head's is (1-lambda) s + lambda qhat, a layer's the column sum of its cotangent
         if (tb >= 0)
