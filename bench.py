@@ -645,7 +645,8 @@ def _small_steps(B, torch, dev, stream, a):
     head, 3-layer bf16 MLP at batch 256, 1000 classes), BOM step with the fused
     update: launched kernel by kernel, and as one captured step (CUDA graph)
     that reads t and lr from the device.  Steps run back to back (a few MB,
-    L2-resident), so the time includes what launching costs."""
+    L2-resident), so the time includes what launching costs; each timing
+    starts a second after the previous GPU work."""
     out = {}
     for wl in (I.TINY_MLP_F32, I.VISION_HEAD_BF16):
         bf16 = wl.dtype == "bf16"
@@ -674,14 +675,22 @@ def _small_steps(B, torch, dev, stream, a):
                 run = lambda t: B.bom_graph_launch(g, stream)
             else:
                 run = lambda t: m.step(x, y, wl.n_rows, params, q, t, None, None, stream)
-            for t in range(1, a.warmup + 1):
+            # a second without GPU work first: the power cap is a running
+            # average, so this light workload then runs at the SM clock it
+            # holds on its own, not at the one the preceding (power-capped)
+            # measurements left
+            torch.cuda.synchronize()
+            time.sleep(1.0)
+            t = 0
+            for _ in range(a.warmup):
+                t += 1
                 run(t)
             m.stats(stream)
             K = 200
             n0 = B.bom_launch_count()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            for t in range(a.warmup + 1, a.warmup + 1 + K):
+            for t in range(t + 1, t + 1 + K):
                 run(t)
             e1.record(stream)
             torch.cuda.synchronize()
