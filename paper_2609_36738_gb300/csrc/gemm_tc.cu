@@ -5,10 +5,9 @@
 // single CTAs compute 128 x 256 tiles (128 x 128 output columns when the B
 // tile is split between gate and up weights).  Warp roles:
 //   warp 0     one thread issues TMA tile loads (128-byte swizzle) into a
-//              shared-memory ring guarded by mbarriers: 32 KB stages (A rows
-//              and this CTA's half of B), as many as fit beside the epilogue's
-//              own shared memory (the SwiGLU backward's G/U slots), up to
-//              six;
+//              shared-memory ring guarded by mbarriers: as many stages (A
+//              rows and this CTA's part of B: 32 KB for a CTA pair) as fit,
+//              at most six;
 //   warp 1     allocates 512 TMEM columns (two 256-column fp32 accumulators)
 //              and, in the even CTA, one thread issues the UMMAs (K = 16),
 //              releasing each smem stage with tcgen05.commit;
@@ -321,15 +320,14 @@ struct Cfg {
     static constexpr int TMEM_COLS = 2 * BNT;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
-    static constexpr int STG_BYTES = 0;
     static constexpr int BAR_BYTES = 512;
-    // as many stages as fit in the 227 KB a CTA may use beside the staging
-    // blocks, the 1 KB alignment slack and the barrier block, at most six (a
-    // seventh 32 KB stage measured slower on the linear epilogues, and no
-    // faster under the fused update)
-    static constexpr int STAGES_FIT = (227 * 1024 - STG_BYTES - 1024 - BAR_BYTES) / (A_BYTES + B_BYTES);
+    // as many stages as fit in the 227 KB a CTA may use beside the 1 KB
+    // alignment slack and the barrier block, at most six (a seventh 32 KB
+    // stage measured slower on the linear and SwiGLU backward epilogues, and
+    // no faster under the fused update)
+    static constexpr int STAGES_FIT = (227 * 1024 - 1024 - BAR_BYTES) / (A_BYTES + B_BYTES);
     static constexpr int STAGES = STAGES_FIT < 6 ? STAGES_FIT : 6;
-    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 1024 + BAR_BYTES;
+    static constexpr int SMEM = STAGES * (A_BYTES + B_BYTES) + 1024 + BAR_BYTES;
     static_assert(STAGES >= 2, "pipeline needs two stages");
     static constexpr int TILE_M = BM * CG;
 };
@@ -345,8 +343,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) gemm_kernel(const __grid_const
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sA = smem;
     uint8_t* sB = smem + STAGES * C::A_BYTES;
-    uint8_t* stg_all = sB + STAGES * C::B_BYTES;   // epilogue staging blocks
-    uint64_t* bars = reinterpret_cast<uint64_t*>(stg_all + C::STG_BYTES);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + STAGES * C::B_BYTES);
     uint64_t* full = bars;
     uint64_t* empty = bars + STAGES;
     uint64_t* tfull = bars + 2 * STAGES;
