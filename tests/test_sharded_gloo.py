@@ -253,3 +253,47 @@ def test_bench_data_parallel_step_on_two_gloo_ranks(tmp_path):
         assert X.rel_l2(o[1 + V:], u_ref) < 1e-12
         assert (tmp_path / f"dp{r}.txt").read_text() == "begin end | allreduce allreduce"
     assert np.array_equal(outs[0], outs[1])
+
+
+def _vocab_lse_parts_rank_main(rank, world, port, out_dir):
+    """The exchange bom_step_vshard_begin / _mid use: each rank's part of a
+    row's log-sum-exp over its own columns, all-gathered in rank order, then
+    combined on every rank as M + log sum_r exp(part_r - M)."""
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        wl = WL_HEAD
+        W = X.params_f64(wl, I.init_params(wl, 7))[0]
+        xb, y = I.make_batch(wl, 7, 1)
+        H = X.x_f64(wl, xb)
+        cols = np.array_split(np.arange(wl.vocab), world)[rank]
+        Zl = H @ W[cols].T
+        part = torch.tensor(O.log_sum_exp_rows(Zl))          # this rank's part of every row
+        parts = [torch.zeros_like(part) for _ in range(world)]
+        dist.all_gather(parts, part)
+        P = torch.stack(parts).numpy()                         # [world, n], rank order
+        M = P.max(axis=0)
+        lse = M + np.log(np.exp(P - M[None, :]).sum(axis=0))
+        valid = y != I.IGNORE_INDEX
+        own = valid & (y >= cols[0]) & (y <= cols[-1])
+        ce_part = float(np.sum((lse - Zl[np.arange(len(y)), np.where(own, y - cols[0], 0)])[own]))
+        np.save(os.path.join(out_dir, f"lrank{rank}.npy"), np.concatenate([lse, [ce_part]]))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_vocabulary_lse_parts_combine_to_the_whole_row_and_the_ce_parts_to_the_loss(tmp_path):
+    world = 3
+    mp.spawn(_vocab_lse_parts_rank_main, args=(world, _free_port(), str(tmp_path)), nprocs=world, join=True)
+    wl = WL_HEAD
+    params = X.params_f64(wl, I.init_params(wl, 7))
+    xb, y = I.make_batch(wl, 7, 1)
+    Z, _ = O.forward(X.oracle_layers(wl), wl.head_bias, params, X.x_f64(wl, xb))
+    valid, n_t = O.supervised_set(y, wl.vocab)
+    ce, lse = O.cross_entropy(Z, y, valid, n_t)
+    outs = [np.load(tmp_path / f"lrank{r}.npy") for r in range(world)]
+    for o in outs:
+        assert X.rel_l2(o[:-1], lse) < 1e-14
+        assert np.array_equal(o[:-1], outs[0][:-1])            # every rank combines the same floats
+    # each supervised row's CE lies in exactly one rank's part; the parts add up to the loss
+    assert abs(sum(o[-1] for o in outs) / n_t - ce) < 1e-12 * abs(ce)
