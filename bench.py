@@ -58,10 +58,12 @@ def _args():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="lm_mlp_bf16")
     p.add_argument("--no-extra", action="store_true", help="skip the head-only and update sub-measurements")
-    p.add_argument("--parallel", default=None, choices=["replicas", "dp"],
+    p.add_argument("--parallel", default=None, choices=["replicas", "dp", "vocab"],
                    help="replicas: independent steps per rank (the default on one GPU); dp: the data-parallel "
                         "step, rows split across ranks, one all-reduce of the V + 3 exchange sums and one of "
-                        "the gradient shares, then the update (the default under torchrun)")
+                        "the gradient shares, then the update (the default under torchrun); vocab: the head's "
+                        "columns split across ranks, every rank with the whole batch, an all-gather of the row "
+                        "log-sum-exp parts and an all-reduce of the head's input cotangent, then the update")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
     p.add_argument("--separate-update", action="store_true",
                    help="run bom_update after bom_step instead of the update fused into the step")
@@ -252,10 +254,21 @@ def main():
     if a.tokens:
         import dataclasses
         wl = dataclasses.replace(wl, n_rows=a.tokens)
-    dp = (a.parallel or ("dp" if world > 1 else "replicas")) == "dp"
-    # data-parallel ranks hold one model; replicas are independent models
-    params_np = I.init_params(wl, seed=0 if dp else rank)
-    shapes = [s for _, s, _ in wl.param_shapes()]
+    mode = a.parallel or ("dp" if world > 1 else "replicas")
+    dp, vocab_par = mode == "dp", mode == "vocab"
+    # data- and vocabulary-parallel ranks hold one model; replicas are independent models
+    params_np = I.init_params(wl, seed=rank if mode == "replicas" else 0)
+    V_total, v_first, wl_model = wl.vocab, 0, wl
+    if vocab_par:   # this rank's rows of the head (and of its bias)
+        import dataclasses
+        cols = np.array_split(np.arange(V_total), world)[rank]
+        v_first = int(cols[0])
+        hw = len(params_np) - (2 if wl.head_bias else 1)
+        params_np = list(params_np)
+        for k in range(hw, len(params_np)):
+            params_np[k] = np.ascontiguousarray(params_np[k][v_first:v_first + cols.size])
+        wl_model = dataclasses.replace(wl, vocab=int(cols.size))
+    shapes = [s for _, s, _ in wl_model.param_shapes()]
     sizes = [int(np.prod(s)) for s in shapes]
     offs = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int64)
     # pad every tensor to 8 elements so each view is 16-byte aligned
@@ -275,19 +288,19 @@ def main():
         return [buf[int(offs_al[k]):int(offs_al[k]) + sizes[k]].view(shapes[k]) for k in range(len(shapes))]
 
     pviews, gviews, thviews, vviews = views(shadow), views(gradf), views(master), views(vstate)
-    x_np, y_np = I.make_batch(wl, seed=rank, step=1)
+    x_np, y_np = I.make_batch(wl, seed=0 if vocab_par else rank, step=1)   # vocabulary ranks share the batch
     x_host = torch.from_numpy(x_np.view(np.int16) if bf16 else x_np).pin_memory()
     y_host = torch.from_numpy(y_np).pin_memory()
     x_dev = (x_host.to(dev).view(torch.bfloat16) if bf16 else x_host.to(dev))
     y_dev = y_host.to(dev)
-    q = torch.zeros(wl.vocab, dtype=torch.float32, device=dev)
-    model = B.BomModel(B.config_for(wl, LAM, B1))
+    q = torch.zeros(wl_model.vocab, dtype=torch.float32, device=dev)
+    model = B.BomModel(B.config_for(wl_model, LAM, B1))
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)   # 256 MiB > L2
     gt = B.BOM_BF16 if bf16 else B.BOM_F32
     N = wl.n_rows
 
-    # the data-parallel step updates after the gradient sum: a separate update pass
-    fused = not a.separate_update and not dp
+    # the sharded steps update after their exchanges: a separate update pass
+    fused = not a.separate_update and not dp and not vocab_par
     if fused:   # BOM-AdamW applied inside bom_step, in the epilogues of the weight-gradient GEMMs
         B.bom_set_fused_update(model.h, thviews, vviews, I.weight_decay_mask(wl, WD), LR, B2, EPS)
     xch = torch.zeros(wl.vocab + 3, dtype=torch.float64, device=dev)
@@ -296,11 +309,27 @@ def main():
         if dist is not None:
             dist.all_reduce(tensor)
 
+    if vocab_par:
+        lse_part = torch.empty(N, dtype=torch.float32, device=dev)
+        lse_parts = torch.empty((world, N), dtype=torch.float32, device=dev)
+        dh = torch.empty((N, wl.d_model), dtype=torch.float32, device=dev)
+
+    def allgather(out, part):
+        if dist is not None:
+            dist.all_gather(list(out.unbind(0)), part)
+        else:
+            out[0].copy_(part)
+
     def step(t, xx=x_dev, yy=y_dev):
         if fused:
             model.step(xx, yy, N, pviews, q, t, None, None, stream)
         elif dp:
             dp_step(B, model.h, xx, yy, N, pviews, q, t, xch, gviews, gradf, allreduce, stream)
+            B.bom_update(master, gradf, gt, None, vstate, shadow if bf16 else None, P, LR, WD, LAM, B2, EPS, t,
+                         stream)
+        elif vocab_par:
+            vocab_step(B, model.h, xx, yy, N, pviews, V_total, v_first, q, t, lse_part, lse_parts, dh, gviews,
+                       allgather, allreduce, stream)
             B.bom_update(master, gradf, gt, None, vstate, shadow if bf16 else None, P, LR, WD, LAM, B2, EPS, t,
                          stream)
         else:
@@ -348,7 +377,10 @@ def main():
     st = model.stats(stream)
     step_ms = [e0.elapsed_time(e1) for e0, e1 in ev]
     tot_ms = _max_over_ranks(dist, sum(step_ms), dev)
-    value = world * N * a.steps / (tot_ms / 1e3)
+    # tokens the whole job processes per step: every rank's rows, except under
+    # vocabulary parallelism, where all ranks work on the same rows
+    job_rows = N if vocab_par else world * N
+    value = job_rows * a.steps / (tot_ms / 1e3)
 
     # the per-kernel split: separate steps with an event pair around every
     # launch (the device time of each kernel class and its algorithmic work)
@@ -451,7 +483,7 @@ def main():
     sdone[(e2e_steps - 1) % 2].synchronize()
     B.bom_stats_decode(sbuf[(e2e_steps - 1) % 2])
     e2e_s = _max_over_ranks(dist, time.perf_counter() - t0, dev)
-    e2e = {"value": world * N * e2e_steps / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+    e2e = {"value": job_rows * e2e_steps / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
            "d2h_bytes_per_step": B.bom_stats_transfer_bytes()}
 
     # ---------------------------------------------------------------- sub-measurements
@@ -487,19 +519,26 @@ def main():
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": a.steps,
-                "warmup": a.warmup, "ms_per_step": tot_ms / a.steps, "higher_is_better": True, "scaling": "weak",
+                "warmup": a.warmup, "ms_per_step": tot_ms / a.steps, "higher_is_better": True,
+                "scaling": "strong" if vocab_par else "weak",
                 "vs_baseline": None, "dtype": "bf16" if bf16 else "f32",
                 "data": "synthetic: seeded N(0,1) inputs, Kaiming-uniform MLP weights, N(0,0.02) head, "
                         "Zipf(1.1) labels",
-                "config": {"workload": _workload_desc(wl), "global_batch": world * N, "tokens_per_gpu": N,
+                "config": {"workload": _workload_desc(wl), "global_batch": job_rows, "tokens_per_gpu": N,
                            "parallelism": (f"dp{world}: rows split across ranks, all-reduce of the V + 3 exchange "
                                            "sums and of the bf16 gradient shares, separate update; measured on "
-                                           "one GPU only" if dp else f"replicas x{world} (no data-path collective)"),
+                                           "one GPU only" if dp else
+                                           f"vocab{world}: head columns split across ranks, every rank with the "
+                                           "whole batch, all-gather of the row log-sum-exp parts and all-reduce "
+                                           "of the head's input cotangent, separate update; not measured on "
+                                           "hardware" if vocab_par else f"replicas x{world} (no data-path collective)"),
                            "l2": "flushed between timed steps (256 MiB write outside the step events)",
                            "lr": LR, "weight_decay": WD, "lambda": LAM, "beta1": B1, "beta2": B2,
                            "update": "fused into the weight-gradient GEMM epilogues" if fused else "separate pass",
                            "step": ("bom_step_shard_begin, all-reduce, bom_step_shard_end, all-reduce, bom_update"
-                                    if dp else "bom_step" + ("" if fused else ", bom_update"))},
+                                    if dp else "bom_step_vshard_begin, all-gather, bom_step_vshard_mid, all-reduce, "
+                                    "bom_step_vshard_end, bom_update" if vocab_par else
+                                    "bom_step" + ("" if fused else ", bom_update"))},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
                 "clocks": clk, "loss_first_step": loss_first, "loss": st["loss"], "kernels": kernels,
                 "sub": extra}
@@ -524,6 +563,27 @@ def dp_step(lib, h, x, y, n_rows, params, q, t, xch, grads, grad_flat, allreduce
     allreduce(xch)
     lib.bom_step_shard_end(h, x, y, n_rows, params, q, t, xch, grads, None, stream)
     allreduce(grad_flat)
+
+
+def vocab_step(lib, h, x, y, n_rows, params, v_total, v_first, q, t, lse_part, lse_parts, dh, grads, allgather,
+               allreduce, stream=None):
+    """One vocabulary-parallel BOM step: this rank holds rows v_first.. of the
+    head (and the same rows of q), the whole backbone and the whole batch.  A
+    row's residual needs the other ranks' columns only through its
+    log-sum-exp (Algorithm 1), and the head's input cotangent is a sum over
+    columns (Eq. mix-gradient): this rank's part of each row's log-sum-exp
+    (bom_step_vshard_begin), the parts of every rank gathered in rank order
+    into lse_parts, the residuals, s_t, q_t and the head rows of u of this
+    rank's columns with its part of the cotangent (bom_step_vshard_mid), the
+    sum of the parts, and the backbone's backward from it
+    (bom_step_vshard_end), whose u is the same on every rank.
+    `allgather(out, part)` fills out[r] with rank r's part, `allreduce(t)`
+    sums a tensor over the ranks in place; `lib` is the binding module."""
+    lib.bom_step_vshard_begin(h, x, y, n_rows, params, v_total, v_first, lse_part, stream)
+    allgather(lse_parts, lse_part)
+    lib.bom_step_vshard_mid(h, x, y, n_rows, params, q, t, lse_parts, lse_parts.shape[0], grads, dh, stream)
+    allreduce(dh)
+    lib.bom_step_vshard_end(h, x, y, n_rows, params, dh, grads, stream)
 
 
 def _max_over_ranks(dist, x, dev):

@@ -297,3 +297,118 @@ def test_vocabulary_lse_parts_combine_to_the_whole_row_and_the_ce_parts_to_the_l
         assert np.array_equal(o[:-1], outs[0][:-1])            # every rank combines the same floats
     # each supervised row's CE lies in exactly one rank's part; the parts add up to the loss
     assert abs(sum(o[-1] for o in outs) / n_t - ce) < 1e-12 * abs(ce)
+
+
+class _OracleVocabCalls:
+    """Stands in for the library's three vocabulary-shard calls on CPU ranks,
+    computed by the oracle: this rank's log-sum-exp part, then (from every
+    rank's parts) its residuals, s_t, q_t, head rows of u and its part of the
+    head's input cotangent, then the backbone's backward from the summed
+    cotangent (the oracle's reverse pass with an identity head, so that the
+    cotangent of the head input is the given sum)."""
+
+    def __init__(self, wl, params64, cols, lam, beta1):
+        self.wl, self.p, self.cols, self.lam, self.beta1 = wl, params64, cols, lam, beta1
+        self.layers = X.oracle_layers(wl)
+        self.hw = len(params64) - (2 if wl.head_bias else 1)
+        self.calls = []
+
+    def bom_step_vshard_begin(self, h, x, y, n, params, v_total, v_first, lse_part, stream=None):
+        self.calls.append("begin")
+        assert v_first == self.cols[0] and v_total == self.wl.vocab
+        Z, saved = O.forward(self.layers, self.wl.head_bias, self.p, x)
+        self.Zr, self.saved = Z[:, self.cols], saved
+        lse_part.copy_(torch.from_numpy(O.log_sum_exp_rows(self.Zr)))
+
+    def bom_step_vshard_mid(self, h, x, y, n, params, q, t, lse_parts, n_shards, grads, dh, stream=None):
+        self.calls.append("mid")
+        P = lse_parts.numpy()
+        assert P.shape[0] == n_shards
+        M = P.max(axis=0)
+        lse = M + np.log(np.exp(P - M[None, :]).sum(axis=0))
+        valid = y != I.IGNORE_INDEX
+        n_t = int(valid.sum())
+        onehot = (y[:, None] == self.cols[None, :]) & valid[:, None]
+        R = np.where(valid[:, None], np.exp(self.Zr - lse[:, None]) - onehot, 0.0)
+        s = R.sum(axis=0) / n_t
+        q_new, qhat = O.ema_update(q.numpy().copy(), s, t, self.beta1)
+        q.copy_(torch.from_numpy(q_new))
+        dZ = ((1 - self.lam) * R + self.lam * valid[:, None] * qhat[None, :]) / n_t
+        grads[self.hw].copy_(torch.from_numpy(dZ.T @ self.saved[1]))
+        dh.copy_(torch.from_numpy(dZ @ self.p[self.hw][self.cols]))
+
+    def bom_step_vshard_end(self, h, x, y, n, params, dh_sum, grads, stream=None):
+        self.calls.append("end")
+        d = self.saved[1].shape[1]
+        gr, _, _ = O.backward(self.layers, False, list(self.p[:self.hw]) + [np.eye(d)], self.saved, dh_sum.numpy())
+        for k in range(self.hw):
+            grads[k].copy_(torch.from_numpy(gr[k]))
+
+
+def _bench_vocab_rank_main(rank, world, port, out_dir):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        import bench
+        wl = WL
+        params = X.params_f64(wl, I.init_params(wl, 8))
+        xb, y = I.make_batch(wl, 8, 1)          # every rank holds the whole batch
+        x = X.x_f64(wl, xb)
+        cols = np.array_split(np.arange(wl.vocab), world)[rank]
+        q_prev = np.random.default_rng(9).standard_normal(wl.vocab) * 0.01
+        lib = _OracleVocabCalls(wl, params, cols, LAM, B1)
+        n, d = wl.n_rows, wl.d_model
+        grads = [torch.zeros(p.shape, dtype=torch.float64) for p in params]
+        grads[lib.hw] = torch.zeros((cols.size, d), dtype=torch.float64)
+        q = torch.from_numpy(q_prev[cols].copy())
+        lse_part = torch.zeros(n, dtype=torch.float64)
+        lse_parts = torch.zeros((world, n), dtype=torch.float64)
+        dh = torch.zeros((n, d), dtype=torch.float64)
+        order = []
+
+        def allgather(out, part):
+            order.append("allgather")
+            dist.all_gather(list(out.unbind(0)), part)
+
+        def allreduce(tensor):
+            order.append("allreduce")
+            dist.all_reduce(tensor)
+
+        bench.vocab_step(lib, None, x, y, n, params, wl.vocab, int(cols[0]), q, T, lse_part, lse_parts, dh, grads,
+                         allgather, allreduce)
+        np.save(os.path.join(out_dir, f"vb{rank}.npy"),
+                np.concatenate([q.numpy()] + [g.numpy().ravel() for g in grads]))
+        with open(os.path.join(out_dir, f"vb{rank}.txt"), "w") as f:
+            f.write(" ".join(lib.calls) + " | " + " ".join(order))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_bench_vocabulary_parallel_step_on_two_gloo_ranks(tmp_path):
+    """bench.vocab_step, the vocabulary-parallel step of bench.py --parallel
+    vocab: begin, the all-gather of the row log-sum-exp parts, mid, the
+    all-reduce of the head's input cotangent, end.  On two gloo ranks with the
+    oracle standing in for the library's three calls, every rank ends with its
+    entries of q and rows of the head's u, and the whole batch's u of every
+    backbone tensor."""
+    world = 2
+    mp.spawn(_bench_vocab_rank_main, args=(world, _free_port(), str(tmp_path)), nprocs=world, join=True)
+    wl = WL
+    layers = X.oracle_layers(wl)
+    params = X.params_f64(wl, I.init_params(wl, 8))
+    xb, y = I.make_batch(wl, 8, 1)
+    q_prev = np.random.default_rng(9).standard_normal(wl.vocab) * 0.01
+    ref = O.bom_step(layers, wl.head_bias, params, X.x_f64(wl, xb), y, q_prev, T, lam=LAM, beta1=B1)
+    hw = len(params) - (2 if wl.head_bias else 1)
+    backbone = np.concatenate([ref["u"][k].ravel() for k in range(hw)])
+    outs = []
+    for r in range(world):
+        cols = np.array_split(np.arange(wl.vocab), world)[r]
+        o = np.load(tmp_path / f"vb{r}.npy")
+        assert X.rel_l2(o[:cols.size], ref["q"][cols]) < 1e-13
+        nb = backbone.size
+        assert X.rel_l2(o[cols.size:cols.size + nb], backbone) < 1e-12
+        assert X.rel_l2(o[cols.size + nb:], ref["u"][hw][cols].ravel()) < 1e-12
+        assert (tmp_path / f"vb{r}.txt").read_text() == "begin mid end | allgather allreduce"
+        outs.append(o[cols.size:cols.size + nb])
+    assert np.array_equal(outs[0], outs[1])   # the backbone's u is the same on every rank
